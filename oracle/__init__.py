@@ -1,0 +1,241 @@
+"""ctypes wrapper of the CPU oracle (``gcpsl_oracle.c``).
+
+TEST INFRASTRUCTURE ONLY: imported by the tests, the smoke check and the CPU
+baseline leg of the benchmark, never by the product package.  The oracle is a
+plain fp64 restatement of one GCPSL local round and of fusion; see the C
+file's header for what it computes and which passages it follows.
+"""
+from __future__ import annotations
+
+import ctypes as ct
+import os
+import subprocess
+from pathlib import Path
+
+import numpy as np
+
+HERE = Path(__file__).resolve().parent
+LIBDIR = HERE / "lib"
+LIB = LIBDIR / "libgcpsl_oracle.so"
+SRC = HERE / "gcpsl_oracle.c"
+
+
+def build(force: bool = False) -> Path:
+    """Compile the oracle with gcc (OpenMP when available)."""
+    if LIB.exists() and not force and LIB.stat().st_mtime >= SRC.stat().st_mtime:
+        return LIB
+    LIBDIR.mkdir(exist_ok=True)
+    tmp = LIBDIR / f".tmp_{os.getpid()}.so"
+    base = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", str(SRC), "-o", str(tmp), "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True, capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    os.replace(tmp, LIB)
+    return LIB
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = ct.CDLL(str(build()))
+        _declare(_lib)
+    return _lib
+
+
+def _p(t):
+    return ct.POINTER(t)
+
+
+def _declare(L):
+    u32p, i32p, f64p, f32p = _p(ct.c_uint32), _p(ct.c_int32), _p(ct.c_double), _p(ct.c_float)
+    L.orc_philox4x32_10.argtypes = [u32p, u32p, u32p]
+    L.orc_epoch_perm.argtypes = [i32p, ct.c_int64, ct.c_uint32, ct.c_uint32, ct.c_uint64, i32p]
+    L.orc_sample_round.argtypes = [i32p, ct.c_int64, ct.c_int, i32p, ct.c_int, i32p, i32p]
+    L.orc_sample_round.restype = ct.c_int
+    L.orc_num_params.argtypes = [ct.c_int, ct.c_int]
+    L.orc_num_params.restype = ct.c_int64
+    L.orc_forward_backward.argtypes = [ct.c_int, ct.c_int, ct.c_double, f64p, ct.c_int, f64p, i32p,
+                                       f64p, f64p, f64p, f64p, f64p]
+    L.orc_fuse_arrays.argtypes = [ct.c_int, ct.c_int64, f64p, f64p, f64p]
+    L.orc_init.argtypes = [ct.c_int, ct.c_int, ct.c_double, ct.c_double, ct.c_double, ct.c_int,
+                           ct.c_double, ct.c_int, ct.c_int, i32p, ct.c_int, ct.c_int, ct.c_uint64,
+                           ct.c_int, f32p, i32p, i32p, ct.c_int64, f32p, _p(ct.c_void_p)]
+    L.orc_destroy.argtypes = [ct.c_void_p]
+    L.orc_step.argtypes = [ct.c_void_p]
+    L.orc_fuse.argtypes = [ct.c_void_p]
+    L.orc_get_params.argtypes = [ct.c_void_p, ct.c_int, ct.c_int, f64p]
+    L.orc_set_params.argtypes = [ct.c_void_p, ct.c_int, f64p]
+    L.orc_get_sample.argtypes = [ct.c_void_p, i32p, i32p]
+    L.orc_get_stats.argtypes = [ct.c_void_p, f64p, i32p]
+    L.orc_get_cut.argtypes = [ct.c_void_p, ct.c_int, f64p]
+    L.orc_get_cut.restype = ct.c_int64
+    L.orc_get_q.argtypes = [ct.c_void_p, f64p]
+    L.orc_rounds.argtypes = [ct.c_void_p]
+    L.orc_rounds.restype = ct.c_int64
+    L.orc_set_threads.argtypes = [ct.c_int]
+    L.orc_get_threads.restype = ct.c_int
+
+
+def _ptr(a, t):
+    return a.ctypes.data_as(ct.POINTER(t))
+
+
+def philox4x32_10(ctr, key):
+    c = np.ascontiguousarray(ctr, dtype=np.uint32)
+    k = np.ascontiguousarray(key, dtype=np.uint32)
+    o = np.zeros(4, dtype=np.uint32)
+    lib().orc_philox4x32_10(_ptr(c, ct.c_uint32), _ptr(k, ct.c_uint32), _ptr(o, ct.c_uint32))
+    return o
+
+
+def epoch_perm(ids, cluster: int, epoch: int, seed: int):
+    ids = np.ascontiguousarray(ids, dtype=np.int32)
+    out = np.empty_like(ids)
+    lib().orc_epoch_perm(_ptr(ids, ct.c_int32), ids.size, cluster, epoch, seed, _ptr(out, ct.c_int32))
+    return out
+
+
+def sample_round(perm, s: int, B: int, owner, K: int):
+    perm = np.ascontiguousarray(perm, dtype=np.int32)
+    owner = np.ascontiguousarray(owner, dtype=np.int32)
+    idx = np.empty(B, dtype=np.int32)
+    counts = np.empty(K, dtype=np.int32)
+    act = lib().orc_sample_round(_ptr(perm, ct.c_int32), s, B, _ptr(owner, ct.c_int32), K,
+                                 _ptr(idx, ct.c_int32), _ptr(counts, ct.c_int32))
+    return idx, counts, act
+
+
+def num_params(arch: int, segment: int) -> int:
+    return int(lib().orc_num_params(arch, segment))
+
+
+def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smoothing: float = 0.0,
+                     want_grad: bool = True):
+    """(loss, grad[P] or None, cut_act, cut_grad, logits) for one replica."""
+    params = np.ascontiguousarray(params, dtype=np.float64)
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    labels = np.ascontiguousarray(labels, dtype=np.int32)
+    B = labels.size
+    P = num_params(arch, 0) + num_params(arch, 1)
+    loss = np.zeros(1)
+    grad = np.zeros(P) if want_grad else None
+    ncut = _cut_elems(arch, B)
+    ca, cg = np.zeros(ncut), np.zeros(ncut)
+    logits = np.zeros(B * 10)
+    rc = lib().orc_forward_backward(arch, int(bf16), label_smoothing, _ptr(params, ct.c_double), B,
+                                    _ptr(x, ct.c_double), _ptr(labels, ct.c_int32),
+                                    _ptr(loss, ct.c_double),
+                                    _ptr(grad, ct.c_double) if want_grad else None,
+                                    _ptr(ca, ct.c_double), _ptr(cg, ct.c_double),
+                                    _ptr(logits, ct.c_double))
+    if rc:
+        raise RuntimeError(f"oracle forward_backward failed: {rc}")
+    return float(loss[0]), grad, ca, cg, logits.reshape(B, 10)
+
+
+def _cut_elems(arch: int, B: int) -> int:
+    return B * {0: 16 * 16 * 16, 1: 64 * 16 * 16}[arch]
+
+
+def cut_shape(arch: int):
+    return {0: (16, 16, 16), 1: (64, 16, 16)}[arch]
+
+
+def fuse_arrays(q, theta):
+    q = np.ascontiguousarray(q, dtype=np.float64)
+    theta = np.ascontiguousarray(theta, dtype=np.float64)
+    C, P = theta.shape
+    out = np.zeros(P)
+    lib().orc_fuse_arrays(C, P, _ptr(q, ct.c_double), _ptr(theta, ct.c_double), _ptr(out, ct.c_double))
+    return out
+
+
+def set_threads(n: int):
+    lib().orc_set_threads(n)
+
+
+def get_threads() -> int:
+    return int(lib().orc_get_threads())
+
+
+class Oracle:
+    """C cluster workloads stepped in lockstep by the CPU oracle."""
+
+    def __init__(self, arch, K, C, assignment, B, F, seed, images, labels, owner, init_params,
+                 lr=0.05, momentum=0.0, weight_decay=0.0, nesterov=False, label_smoothing=0.0,
+                 bf16=False, cluster_base=0):
+        self.arch, self.K, self.C, self.B = arch, K, C, B
+        # the context reads the images in place: keep them alive here
+        self._images = np.ascontiguousarray(images, dtype=np.float32)
+        self._labels = np.ascontiguousarray(labels, dtype=np.int32)
+        self._owner = np.ascontiguousarray(owner, dtype=np.int32)
+        self._assign = np.ascontiguousarray(assignment, dtype=np.int32)
+        p = np.ascontiguousarray(init_params, dtype=np.float32)
+        h = ct.c_void_p()
+        rc = lib().orc_init(arch, int(bf16), lr, momentum, weight_decay, int(nesterov),
+                            label_smoothing, K, C, _ptr(self._assign, ct.c_int32), B, F, seed,
+                            cluster_base, _ptr(self._images, ct.c_float),
+                            _ptr(self._labels, ct.c_int32), _ptr(self._owner, ct.c_int32),
+                            self._images.shape[0], _ptr(p, ct.c_float), ct.byref(h))
+        if rc:
+            raise ValueError(f"oracle init failed: {rc}")
+        self._h = h
+        self.P_client = num_params(arch, 0)
+        self.P_server = num_params(arch, 1)
+
+    def __del__(self):
+        if getattr(self, "_h", None):
+            lib().orc_destroy(self._h)
+            self._h = None
+
+    def step(self):
+        rc = lib().orc_step(self._h)
+        if rc:
+            raise RuntimeError(f"oracle step failed: {rc}")
+
+    def fuse(self):
+        lib().orc_fuse(self._h)
+
+    def params(self, cluster: int, segment: int):
+        n = self.P_client if segment == 0 else self.P_server
+        out = np.zeros(n)
+        lib().orc_get_params(self._h, cluster, segment, _ptr(out, ct.c_double))
+        return out
+
+    def all_params(self, cluster: int):
+        return np.concatenate([self.params(cluster, 0), self.params(cluster, 1)])
+
+    def set_params(self, cluster: int, blob):
+        blob = np.ascontiguousarray(blob, dtype=np.float64)
+        lib().orc_set_params(self._h, cluster, _ptr(blob, ct.c_double))
+
+    def sample(self):
+        idx = np.zeros((self.C, self.B), dtype=np.int32)
+        counts = np.zeros((self.C, self.K), dtype=np.int32)
+        lib().orc_get_sample(self._h, _ptr(idx, ct.c_int32), _ptr(counts, ct.c_int32))
+        return idx, counts
+
+    def stats(self):
+        loss = np.zeros(self.C)
+        act = np.zeros(self.C, dtype=np.int32)
+        lib().orc_get_stats(self._h, _ptr(loss, ct.c_double), _ptr(act, ct.c_int32))
+        return loss, act
+
+    def cut(self, which: int):
+        n = lib().orc_get_cut(self._h, which, None)
+        out = np.zeros(n)
+        lib().orc_get_cut(self._h, which, _ptr(out, ct.c_double))
+        return out.reshape((self.C, self.B) + cut_shape(self.arch))
+
+    def q(self):
+        out = np.zeros(self.C)
+        lib().orc_get_q(self._h, _ptr(out, ct.c_double))
+        return out
+
+    @property
+    def rounds(self) -> int:
+        return int(lib().orc_rounds(self._h))

@@ -1,0 +1,142 @@
+"""Seeded synthetic inputs for the GCPSL training step.
+
+This module only draws random inputs: images, labels, the per-client data
+split and the initial split-model parameters.  It holds none of the method's
+arithmetic (no sampling, no forward/backward, no update, no fusion), so that
+both the CUDA library and the CPU oracle can take their inputs from it.
+
+Stand-in for CIFAR-10 (Section V-A uses CIFAR-10/100, which are not available
+here): 32x32x3 images with N(0,1) pixels and 10 classes.  The client split is a
+per-class Dirichlet draw (the paper's Section V-A uses an extended-Dirichlet
+protocol with two classes per client; the plain per-class Dirichlet(alpha) is
+the recipe these workloads use instead).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+IMG_C, IMG_H, IMG_W = 3, 32, 32
+IMG_ELEMS = IMG_C * IMG_H * IMG_W
+
+# Seeds of the five input streams (data, split, clustering, init, sampler).
+SEED_DATA, SEED_SPLIT, SEED_CLUSTER, SEED_INIT, SEED_SAMPLER = 0, 1, 2, 3, 4
+
+
+@dataclass
+class Dataset:
+    images: np.ndarray   # float32 [n, 3, 32, 32], NCHW
+    labels: np.ndarray   # int32 [n]
+    owner: np.ndarray    # int32 [n], client id of each example
+    num_classes: int
+    num_clients: int
+
+
+def make_images(n: int, seed: int = SEED_DATA) -> np.ndarray:
+    """n images of N(0,1) float32 pixels, NCHW."""
+    rng = np.random.default_rng(seed)
+    return rng.standard_normal((n, IMG_C, IMG_H, IMG_W), dtype=np.float32)
+
+
+def make_labels(n: int, num_classes: int, balanced: bool, seed: int = SEED_DATA) -> np.ndarray:
+    """Labels: exactly n/num_classes per class in shuffled order when
+    `balanced`, otherwise i.i.d. uniform."""
+    rng = np.random.default_rng(seed + 1_000_003)
+    if balanced:
+        if n % num_classes:
+            raise ValueError("balanced labels need n divisible by num_classes")
+        lab = np.repeat(np.arange(num_classes, dtype=np.int32), n // num_classes)
+        rng.shuffle(lab)
+        return lab
+    return rng.integers(0, num_classes, size=n, dtype=np.int32)
+
+
+def dirichlet_split(labels: np.ndarray, num_clients: int, alpha: float,
+                    seed: int = SEED_SPLIT) -> np.ndarray:
+    """Owner of every example under a per-class Dirichlet(alpha) split.
+
+    For each class in increasing order: draw p ~ Dir(alpha * 1_K); give client
+    k floor(p_k * n_class) examples; hand the remaining examples one each to the
+    clients with the largest fractional parts (ties to the lower client id);
+    shuffle the class's examples and deal them out in client order.  Clients
+    may end up with no examples.
+    """
+    rng = np.random.default_rng(seed)
+    owner = np.full(labels.shape[0], -1, dtype=np.int32)
+    num_classes = int(labels.max()) + 1 if labels.size else 0
+    for c in range(num_classes):
+        ex = np.flatnonzero(labels == c)
+        n_c = ex.size
+        p = rng.dirichlet(np.full(num_clients, alpha))
+        raw = p * n_c
+        cnt = np.floor(raw).astype(np.int64)
+        rem = n_c - int(cnt.sum())
+        frac = raw - cnt
+        # largest fractional part first, ties to the lower client id
+        order = np.lexsort((np.arange(num_clients), -frac))
+        cnt[order[:rem]] += 1
+        rng.shuffle(ex)
+        owner[ex] = np.repeat(np.arange(num_clients, dtype=np.int32), cnt)
+    assert (owner >= 0).all()
+    return owner
+
+
+def make_dataset(n: int, num_classes: int, num_clients: int, alpha: float,
+                 balanced: bool, seed_data: int = SEED_DATA,
+                 seed_split: int = SEED_SPLIT) -> Dataset:
+    images = make_images(n, seed_data)
+    labels = make_labels(n, num_classes, balanced, seed_data)
+    owner = dirichlet_split(labels, num_clients, alpha, seed_split)
+    return Dataset(images, labels, owner, num_classes, num_clients)
+
+
+# ---------------------------------------------------------------------------
+# Split-model parameter shapes, in PyTorch state_dict order (conv weights
+# OIHW), client segment first.  Conv layers are 3x3, stride 1, padding 1,
+# with bias; every conv is followed by ReLU; `pool` adds a 2x2/2 max-pool.
+# ---------------------------------------------------------------------------
+ARCH_TINY_CNN, ARCH_SPLIT_CNN, ARCH_RESNET18 = 0, 1, 2
+
+ARCHS = {
+    # (cin, cout, H, W, pool) per conv layer; fc (in, out)
+    ARCH_TINY_CNN: dict(client=[(3, 16, 32, 32, 1)],
+                        server=[(16, 32, 16, 16, 1)], fc=(2048, 10)),
+    ARCH_SPLIT_CNN: dict(client=[(3, 32, 32, 32, 0), (32, 64, 32, 32, 1)],
+                         server=[(64, 128, 16, 16, 1), (128, 128, 8, 8, 1)],
+                         fc=(2048, 10)),
+}
+
+
+def param_shapes(arch: int, segment: str):
+    """[(name, shape)] for one segment ('client' or 'server')."""
+    spec = ARCHS[arch]
+    out = []
+    for i, (cin, cout, _h, _w, _p) in enumerate(spec[segment]):
+        out.append((f"{segment}.conv{i}.weight", (cout, cin, 3, 3)))
+        out.append((f"{segment}.conv{i}.bias", (cout,)))
+    if segment == "server":
+        fin, fout = spec["fc"]
+        out.append(("server.fc.weight", (fout, fin)))
+        out.append(("server.fc.bias", (fout,)))
+    return out
+
+
+def num_params(arch: int, segment: str) -> int:
+    return int(sum(np.prod(s) for _n, s in param_shapes(arch, segment)))
+
+
+def init_params(arch: int, seed: int = SEED_INIT) -> np.ndarray:
+    """One float32 blob, client segment then server segment, drawn like
+    PyTorch's default layer init: U(-1/sqrt(fan_in), 1/sqrt(fan_in)) for
+    weights and biases of every conv and linear layer."""
+    rng = np.random.default_rng(seed)
+    parts = []
+    for seg in ("client", "server"):
+        shapes = param_shapes(arch, seg)
+        for (name, shape) in shapes:
+            if name.endswith(".weight"):
+                fan_in = int(np.prod(shape[1:]))
+            bound = 1.0 / np.sqrt(fan_in)
+            parts.append(rng.uniform(-bound, bound, size=shape).astype(np.float32).ravel())
+    return np.concatenate(parts)

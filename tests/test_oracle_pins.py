@@ -1,0 +1,336 @@
+"""Pins of the CPU oracle against facts fixed outside it.
+
+Each test ties one part of the oracle to something other than itself:
+published known-answer vectors (Philox), the invariants of Eq. 1-3, brute
+force, closed forms, finite differences, and PyTorch's own fp64 conv /
+max-pool / cross-entropy / SGD routines (which the oracle does not call).
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as Fn
+
+import oracle
+from paper_2609_29395_gb300 import synth, clustering
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# --------------------------------------------------------------------------
+# Philox4x32-10
+# --------------------------------------------------------------------------
+def _kat_rows():
+    rows = []
+    for line in open(os.path.join(GOLD, "philox4x32_10_kat.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        v = [int(t, 16) for t in line.split()]
+        rows.append((v[:4], v[4:6], v[6:10]))
+    return rows
+
+
+@pytest.mark.parametrize("ctr,key,expect", _kat_rows())
+def test_philox_known_answers(ctr, key, expect):
+    assert list(oracle.philox4x32_10(ctr, key)) == expect
+
+
+# --------------------------------------------------------------------------
+# Sampler (Eq. 1, epoch rule of Section III-A, Eq. 3)
+# --------------------------------------------------------------------------
+def _keys(ids, cluster, epoch, seed):
+    key = [seed & 0xFFFFFFFF, seed >> 32]
+    k64 = []
+    for j in ids:
+        o = oracle.philox4x32_10([int(j), epoch, cluster, 0], key)
+        k64.append((int(o[0]) << 32) | int(o[1]))
+    return k64
+
+
+def test_epoch_perm_is_the_key_order():
+    rng = np.random.default_rng(11)
+    ids = np.sort(rng.choice(5000, size=300, replace=False)).astype(np.int32)
+    seed = 0x1234_5678_9ABC_DEF0
+    perm = oracle.epoch_perm(ids, 3, 7, seed)
+    k = _keys(ids, 3, 7, seed)
+    expect = [j for _, j in sorted(zip(k, ids.tolist()))]
+    assert perm.tolist() == expect
+    # a different epoch or cluster gives a different order
+    assert oracle.epoch_perm(ids, 3, 8, seed).tolist() != expect
+    assert oracle.epoch_perm(ids, 4, 7, seed).tolist() != expect
+
+
+def test_epoch_perm_uniform_chi2():
+    """Position of each id over many epochs is uniform (chi-square)."""
+    from scipy.stats import chisquare
+    ids = np.arange(6, dtype=np.int32) * 5 + 1
+    E = 3000
+    pos = np.zeros((6, 6))
+    for e in range(E):
+        p = oracle.epoch_perm(ids, 0, e, 4)
+        for i, j in enumerate(p):
+            pos[(j - 1) // 5, i] += 1
+    stat, pval = chisquare(pos.ravel(), np.full(36, E / 6))
+    assert pval > 1e-4, (stat, pval)
+
+
+def _small_world(seed=5, n=600, K=24, C=3):
+    rng = np.random.default_rng(seed)
+    owner = rng.integers(0, K, size=n).astype(np.int32)
+    assign = clustering.random_clustering(K, C, seed)
+    return owner, assign
+
+
+def test_sample_round_invariants():
+    owner, assign = _small_world()
+    K, C, B = 24, 3, 16
+    for n in range(C):
+        ids = np.flatnonzero(assign[owner] == n).astype(np.int32)
+        holdings = np.bincount(owner[ids], minlength=K)
+        members = np.flatnonzero(assign == n)
+        r = ids.size // B
+        perm = oracle.epoch_perm(ids, n, 0, 4)
+        assert sorted(perm.tolist()) == ids.tolist()
+        seen = []
+        cum = np.zeros(K, dtype=np.int64)
+        for s in range(r):
+            idx, counts, act = oracle.sample_round(perm, s, B, owner, K)
+            assert counts.sum() == B                                   # Eq. 1
+            assert (counts <= holdings).all()
+            assert (counts[np.setdiff1d(np.arange(K), members)] == 0).all()
+            assert act == (counts > 0).sum() <= min(B, members.size)   # |A| <= B
+            rho = 1 - act / members.size
+            assert rho >= max(0.0, 1 - B / members.size) - 1e-12       # Eq. 3
+            key = list(zip(owner[idx].tolist(), idx.tolist()))
+            assert key == sorted(key)
+            assert (np.bincount(owner[idx], minlength=K) == counts).all()
+            cum += counts
+            seen += idx.tolist()
+        assert (cum <= holdings).all()
+        assert len(seen) == len(set(seen)) == r * B                     # once per epoch
+
+
+def test_gpsl_bound_worked_values():
+    for line in open(os.path.join(GOLD, "gpsl_bounds.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        K, B, bound = line.split()
+        assert max(0.0, 1 - int(B) / int(K)) == pytest.approx(float(bound))
+
+
+# --------------------------------------------------------------------------
+# Forward / backward
+# --------------------------------------------------------------------------
+def _torch_model(arch, blob):
+    """fp64 PyTorch forward of the split model from a canonical blob."""
+    spec = synth.ARCHS[arch]
+    convs = spec["client"] + spec["server"]
+    t = torch.from_numpy(np.asarray(blob, dtype=np.float64)).clone().requires_grad_(True)
+    off = 0
+    ws = []
+    for (cin, cout, _h, _w, pool) in convs:
+        nw = cout * cin * 9
+        ws.append((t[off:off + nw].view(cout, cin, 3, 3), t[off + nw:off + nw + cout], pool))
+        off += nw + cout
+    fin, fout = spec["fc"]
+    fw = t[off:off + fin * fout].view(fout, fin)
+    fb = t[off + fin * fout:off + fin * fout + fout]
+    ncl = len(spec["client"])
+
+    def fwd(x):
+        z = None
+        for i, (w, b, pool) in enumerate(ws):
+            x = Fn.relu(Fn.conv2d(x, w, b, padding=1))
+            if pool:
+                x = Fn.max_pool2d(x, 2)
+            if i == ncl - 1:
+                z = x
+                z.retain_grad()
+        return Fn.linear(x.flatten(1), fw, fb), z
+    return t, fwd
+
+
+@pytest.mark.parametrize("arch,B", [(synth.ARCH_TINY_CNN, 4), (synth.ARCH_SPLIT_CNN, 2)])
+def test_forward_backward_matches_torch_fp64(arch, B):
+    rng = np.random.default_rng(3)
+    blob = synth.init_params(arch, seed=9).astype(np.float64)
+    x = rng.standard_normal((B, 3, 32, 32))
+    y = rng.integers(0, 10, size=B).astype(np.int32)
+    loss, grad, ca, cg, logits = oracle.forward_backward(arch, blob, x, y)
+    t, fwd = _torch_model(arch, blob)
+    out, z = fwd(torch.from_numpy(x))
+    tl = Fn.cross_entropy(out, torch.from_numpy(y.astype(np.int64)))
+    tl.backward()
+    assert loss == pytest.approx(tl.item(), rel=1e-12, abs=1e-12)
+    np.testing.assert_allclose(logits, out.detach().numpy(), rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(grad, t.grad.numpy(), rtol=1e-9, atol=1e-13)
+    np.testing.assert_allclose(ca, z.detach().numpy().ravel(), rtol=1e-11, atol=1e-13)
+    np.testing.assert_allclose(cg, z.grad.numpy().ravel(), rtol=1e-9, atol=1e-14)
+
+
+def test_label_smoothing_matches_torch():
+    arch, B = synth.ARCH_TINY_CNN, 3
+    rng = np.random.default_rng(4)
+    blob = synth.init_params(arch, seed=2).astype(np.float64)
+    x = rng.standard_normal((B, 3, 32, 32))
+    y = rng.integers(0, 10, size=B).astype(np.int32)
+    loss, grad, *_ = oracle.forward_backward(arch, blob, x, y, label_smoothing=0.1)
+    t, fwd = _torch_model(arch, blob)
+    out, _ = fwd(torch.from_numpy(x))
+    tl = Fn.cross_entropy(out, torch.from_numpy(y.astype(np.int64)), label_smoothing=0.1)
+    tl.backward()
+    assert loss == pytest.approx(tl.item(), rel=1e-12)
+    np.testing.assert_allclose(grad, t.grad.numpy(), rtol=1e-9, atol=1e-13)
+
+
+def test_finite_differences():
+    """Central differences of the oracle's own loss agree with its gradient."""
+    arch, B = synth.ARCH_TINY_CNN, 2
+    rng = np.random.default_rng(8)
+    blob = synth.init_params(arch, seed=5).astype(np.float64)
+    x = rng.standard_normal((B, 3, 32, 32))
+    y = np.array([3, 7], dtype=np.int32)
+    _, grad, *_ = oracle.forward_backward(arch, blob, x, y)
+    # a few coordinates from every tensor (conv0 w/b, conv1 w/b, fc w/b)
+    bounds = np.cumsum([0, 432, 16, 4608, 32, 20480, 10])
+    picks = [int(rng.integers(bounds[i], bounds[i + 1])) for i in range(6) for _ in range(4)]
+    h = 1e-6
+    for p in picks:
+        bp, bm = blob.copy(), blob.copy()
+        bp[p] += h
+        bm[p] -= h
+        lp = oracle.forward_backward(arch, bp, x, y, want_grad=False)[0]
+        lm = oracle.forward_backward(arch, bm, x, y, want_grad=False)[0]
+        fd = (lp - lm) / (2 * h)
+        assert fd == pytest.approx(grad[p], rel=1e-5, abs=1e-9), p
+
+
+def test_zero_weights_give_ln10():
+    for arch in (synth.ARCH_TINY_CNN, synth.ARCH_SPLIT_CNN):
+        P = oracle.num_params(arch, 0) + oracle.num_params(arch, 1)
+        x = np.random.default_rng(0).standard_normal((2, 3, 32, 32))
+        loss, *_ = oracle.forward_backward(arch, np.zeros(P), x, np.array([1, 9], np.int32),
+                                           want_grad=False)
+        assert loss == pytest.approx(math.log(10.0), rel=1e-15)
+
+
+def test_bf16_mode_rounds_only():
+    """bf16 operand mode stays close to fp64 (a rounding mode, not a new op)."""
+    arch, B = synth.ARCH_TINY_CNN, 4
+    rng = np.random.default_rng(1)
+    blob = synth.init_params(arch, seed=1).astype(np.float64)
+    x = rng.standard_normal((B, 3, 32, 32))
+    y = rng.integers(0, 10, size=B).astype(np.int32)
+    l64, g64, *_ = oracle.forward_backward(arch, blob, x, y)
+    l16, g16, *_ = oracle.forward_backward(arch, blob, x, y, bf16=True)
+    assert abs(l64 - l16) < 2e-2
+    assert np.linalg.norm(g16 - g64) / np.linalg.norm(g64) < 5e-2
+    assert l64 != l16
+
+
+# --------------------------------------------------------------------------
+# Fusion (Eq. 5)
+# --------------------------------------------------------------------------
+def test_fusion_identity():
+    rng = np.random.default_rng(2)
+    th = rng.standard_normal(1000).astype(np.float32).astype(np.float64)
+    q = np.array([0.1, 0.2, 0.3, 0.4])
+    out = oracle.fuse_arrays(q, np.stack([th] * 4))
+    np.testing.assert_allclose(out, th, rtol=1e-15)
+    assert (out.astype(np.float32) == th.astype(np.float32)).all()
+
+
+def test_fusion_closed_form():
+    C, P = 5, 64
+    q = np.arange(1, C + 1, dtype=np.float64)
+    q /= q.sum()
+    theta = np.stack([np.full(P, float(n)) for n in range(C)])
+    out = oracle.fuse_arrays(q, theta)
+    np.testing.assert_allclose(out, np.full(P, sum(q[n] * n for n in range(C))), rtol=1e-15)
+
+
+# --------------------------------------------------------------------------
+# Whole rounds: C = 1 is GPSL; concurrent == sequential; fusion in the loop
+# --------------------------------------------------------------------------
+def _tiny_world(n=256, K=8, seed=0):
+    ds = synth.make_dataset(n, 10, K, 0.5, balanced=False, seed_data=seed, seed_split=seed + 1)
+    return ds
+
+
+def test_single_cluster_is_gpsl_against_torch_sgd():
+    """C=1 with every client in it is plain GPSL: replay its batches through
+    PyTorch fp64 autograd and torch.optim.SGD(momentum=0.9)."""
+    arch, B, K = synth.ARCH_TINY_CNN, 8, 8
+    ds = _tiny_world(K=K)
+    blob = synth.init_params(arch, seed=3)
+    orc = oracle.Oracle(arch, K, 1, np.zeros(K, np.int32), B, 0, 4, ds.images, ds.labels,
+                        ds.owner, blob, lr=0.05, momentum=0.9)
+    t, fwd = _torch_model(arch, blob.astype(np.float64))
+    opt = torch.optim.SGD([t], lr=0.05, momentum=0.9)
+    for _ in range(4):
+        orc.step()
+        idx, counts = orc.sample()
+        assert counts.sum() == B
+        opt.zero_grad()
+        out, _ = fwd(torch.from_numpy(ds.images[idx[0]].astype(np.float64)))
+        Fn.cross_entropy(out, torch.from_numpy(ds.labels[idx[0]].astype(np.int64))).backward()
+        opt.step()
+        np.testing.assert_allclose(orc.all_params(0), t.detach().numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_concurrent_equals_sequential_then_fusion():
+    """C clusters in one context == each cluster alone (cluster_base = n),
+    and the context's fusion == Eq. 5 over the separate replicas."""
+    arch, B, K, C = synth.ARCH_TINY_CNN, 8, 8, 2
+    ds = _tiny_world(K=K, seed=2)
+    assign = clustering.random_clustering(K, C, 2)
+    blob = synth.init_params(arch, seed=3)
+    common = dict(lr=0.05, momentum=0.9)
+    grouped = oracle.Oracle(arch, K, C, assign, B, 0, 4, ds.images, ds.labels, ds.owner, blob,
+                            **common)
+    alone = [oracle.Oracle(arch, K, 1, np.where(assign == n, 0, -1).astype(np.int32), B, 0, 4,
+                           ds.images, ds.labels, ds.owner, blob, cluster_base=n, **common)
+             for n in range(C)]
+    for _ in range(3):
+        grouped.step()
+        for a in alone:
+            a.step()
+    gi, gc = grouped.sample()
+    for n in range(C):
+        ai, ac = alone[n].sample()
+        assert (ai[0] == gi[n]).all() and (ac[0] == gc[n]).all()
+        assert (alone[n].all_params(0) == grouped.all_params(n)).all()
+    q = grouped.q()
+    sizes = np.bincount(assign[ds.owner], minlength=C)
+    np.testing.assert_allclose(q, sizes / sizes.sum(), rtol=0, atol=0)
+    fused = oracle.fuse_arrays(q, np.stack([a.all_params(0) for a in alone]))
+    grouped.fuse()
+    for n in range(C):
+        assert (grouped.all_params(n) == fused).all()
+
+
+def test_fusion_every_F_rounds_in_the_loop():
+    arch, B, K, C, F = synth.ARCH_TINY_CNN, 8, 8, 2, 2
+    ds = _tiny_world(K=K, seed=3)
+    assign = clustering.random_clustering(K, C, 1)
+    blob = synth.init_params(arch, seed=3)
+    orc = oracle.Oracle(arch, K, C, assign, B, F, 4, ds.images, ds.labels, ds.owner, blob,
+                        lr=0.05)
+    orc.step()
+    assert not (orc.all_params(0) == orc.all_params(1)).all()
+    orc.step()                                   # round 2: fused, replicas equal
+    assert (orc.all_params(0) == orc.all_params(1)).all()
+
+
+def test_init_rejects_bad_inputs():
+    arch, K = synth.ARCH_TINY_CNN, 8
+    ds = _tiny_world(K=K)
+    blob = synth.init_params(arch)
+    with pytest.raises(ValueError):   # cluster smaller than B
+        oracle.Oracle(arch, K, 1, np.zeros(K, np.int32), 10_000, 0, 4, ds.images, ds.labels,
+                      ds.owner, blob)
+    with pytest.raises(ValueError):   # assignment out of range
+        oracle.Oracle(arch, K, 2, np.full(K, 2, np.int32), 8, 0, 4, ds.images, ds.labels,
+                      ds.owner, blob)
