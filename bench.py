@@ -1,0 +1,417 @@
+#!/usr/bin/env python3
+"""Benchmark of one GCPSL local round of all C cluster workloads on GB300.
+
+A step is one call of gcpsl_step: GPSL sampling of B examples in every
+cluster, client forward to the cut, server forward, softmax cross-entropy,
+backward to the cut gradient and through the client segment, per-replica SGD,
+and fusion every F rounds (amortised: it runs inside the timed steps whose
+round number is a multiple of F).
+
+Default workload: 50,000 synthetic 32x32x3 images (N(0,1) pixels, 10
+balanced classes), K=256 clients with a Dirichlet(0.3) split, C=4 random
+clusters, B=64, F=50, SplitCNN, SGD lr 0.05 momentum 0.9, bf16 operands.
+
+Prints ONE JSON line (rank 0).  `value` is examples/s summed over the C
+clusters (and over ranks for --gpus N: each rank runs an independent copy of
+the workload on its own GPU; nothing is exchanged between ranks).  Between
+timed steps a 256 MiB buffer is written to flush the 129 MB L2; each step is
+timed with CUDA events on the library's stream.
+
+--impl reference times the CPU oracle (plain fp64 C, all host cores) on a
+bounded sample of the same workload: each step is one forward/backward of a
+few examples of cluster 0 plus that replica's SGD update.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "examples/sec summed over C clusters on 1 GB300; % tensor-pipe peak; fusion GB/s"
+UNIT = "examples/s"
+FLUSH_BYTES = 256 << 20
+
+# DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by
+# kernel kind; valid only while the kernel source hashes to the recorded value.
+NCU_TRAFFIC = {}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="splitcnn_c4")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true", help="skip e2e/serialized/fusion legs")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"],
+                    src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work per kernel kind and round (FLOPs for contractions, bytes
+# for the elementwise/bandwidth kernels)
+# ---------------------------------------------------------------------------
+def work_per_round(w, esz):
+    from paper_2609_29395_gb300 import synth
+    spec = synth.ARCHS[w.arch]
+    convs = spec["client"] + spec["server"]
+    C, B = w.num_clusters, w.B
+    P = synth.num_params(w.arch, "client") + synth.num_params(w.arch, "server")
+    fwd = dgrad = wgrad = 0
+    for i, (cin, cout, h, ww, _p) in enumerate(convs):
+        f = 2.0 * C * B * h * ww * cout * 9 * cin
+        fwd += f
+        wgrad += f
+        if i > 0:
+            dgrad += f
+    fin, fout = spec["fc"]
+    fc = 2.0 * C * B * fin * fout
+    return {
+        "conv_fwd": ("tensor", fwd), "conv_dgrad": ("tensor", dgrad),
+        "conv_wgrad": ("tensor", wgrad), "fc_fwd": ("tensor", fc),
+        "fc_bwd": ("tensor", 2 * fc),
+        "sgd": ("hbm", C * P * (4 * 5 + (2 if esz == 2 else 0))),
+        "fuse": ("hbm", C * P * (4 + 4 + (2 if esz == 2 else 0))),
+    }
+
+
+def kernel_source_hash(kind):
+    src = {"conv_fwd": "conv_simt.cu", "conv_dgrad": "conv_simt.cu", "conv_wgrad": "conv_simt.cu",
+           "sgd": "optim.cu", "fuse": "optim.cu"}.get(kind)
+    if not src:
+        return None
+    p = os.path.join(ROOT, "paper_2609_29395_gb300", "csrc", src)
+    return hashlib.sha256(open(p, "rb").read()).hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+
+    def __init__(self, gpu_index):
+        self.proc = None
+        self.gpu = gpu_index
+
+    def __enter__(self):
+        q = ("clocks.sm,clocks.max.sm,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            try:
+                sm.append(float(f[0]))
+                mx = float(f[1])
+            except (ValueError, IndexError):
+                continue
+            for nm, v in zip(names, f[3:7]):
+                if v.lower() in ("active", "1", "yes"):
+                    reasons.add(nm)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+def cpu_baseline(w, ds, assign, params, budget_s=15.0):
+    """The oracle as it stands, on this host's cores: repeated forward/
+    backward of a small batch of cluster-0 examples (bf16-operand mode when
+    the workload is bf16).  Returns (examples/s, threads, description)."""
+    import oracle
+    ids = np.flatnonzero(assign[ds.owner] == 0)[:8]
+    x = ds.images[ids].astype(np.float64)
+    y = ds.labels[ids]
+    done, t0 = 0, time.perf_counter()
+    while True:
+        oracle.forward_backward(w.arch, params.astype(np.float64), x, y, bf16=w.bf16)
+        done += len(ids)
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return done / dt, oracle.get_threads(), (
+        f"{done} examples of cluster 0 in batches of {len(ids)} (forward+backward, fp64, "
+        f"{'bf16-operand' if w.bf16 else 'fp32'} rounding), {dt:.1f} s")
+
+
+def run_reference(args, w):
+    """Reference arm: the CPU oracle as it stands, timed on the host cores."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2609_29395_gb300 import configs
+    ds, assign, params = configs.build_inputs(w)
+    ids = np.flatnonzero(assign[ds.owner] == 0)[:4]
+    x = ds.images[ids].astype(np.float64)
+    y = ds.labels[ids]
+    blob = params.astype(np.float64)
+
+    def one():
+        oracle.forward_backward(w.arch, blob, x, y, bf16=w.bf16)
+    for _ in range(args.warmup):
+        one()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one()
+    dt = time.perf_counter() - t0
+    v = args.steps * len(ids) / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "C": w.num_clusters, "K": w.num_clients,
+                   "n": w.n, "sample": f"{len(ids)} examples of cluster 0 per step"},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.get_threads(),
+                         "kind": "oracle",
+                         "sample": f"forward+backward of {len(ids)} cluster-0 examples per step"},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    args = parse()
+    from paper_2609_29395_gb300 import configs
+    w = configs.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, w)
+
+    rank, world, local = dist_env()
+    import torch
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import __graft_entry__
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
+        __graft_entry__.build()
+    import paper_2609_29395_gb300 as pkg
+
+    ds, assign, params = configs.build_inputs(w)
+    ctx = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
+                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=w.bf16)
+    # a dedicated stream: the library, the events and the L2 flush all use it
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    ctx.set_stream(stream.cuda_stream)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+
+    for _ in range(args.warmup):
+        ctx.step()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    ctx.set_timing(True)
+    ctx.reset_kernel_times()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        wall0 = time.perf_counter()
+        for i in range(K):
+            flush.fill_(float(i))
+            ev[i][0].record(stream)
+            ctx.step()
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+    if world > 1:
+        dist.barrier()
+    ctx.set_timing(False)
+    step_ms = sum(a.elapsed_time(b) for a, b in ev)
+    ktimes = ctx.kernel_times()
+    if world > 1:
+        t = torch.tensor([step_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        step_ms = float(t.item())
+    examples = w.num_clusters * w.B * K * world
+    value = examples / (step_ms / 1e3)
+    launches = sum(n for n, _ in ktimes.values())
+
+    # dominant kernel and its roofline
+    peaks = load_peaks()
+    work = work_per_round(w, 2 if w.bf16 else 4)
+    top = max(ktimes.items(), key=lambda kv: kv[1][1])
+    kind, (n_launch, k_ms) = top
+    bound, per_round = work.get(kind, ("hbm", None))
+    roof = {"kernel": kind, "launches": n_launch, "avg_launch_ms": k_ms / max(n_launch, 1)}
+    if per_round is not None:
+        rounds = K
+        if kind == "fuse":
+            rounds = max(n_launch, 1)
+        total_work = per_round * rounds
+        secs = k_ms / 1e3
+        if bound == "tensor":
+            ach = total_work / secs / 1e12
+            peak = peaks["bf16_sus"] if w.bf16 else None
+            roof.update(bound="tensor", achieved=ach, unit="TFLOP/s")
+            if peak is None:  # fp32 path runs on CUDA cores: no tensor peak applies
+                peak = peaks["bf16_sus"]
+            roof.update(peak=peak, frac=ach / peak, peak_src=f"bf16 sustained, {peaks['src']}")
+        else:
+            ach = total_work / secs / 1e9
+            roof.update(bound="hbm", achieved=ach, unit="GB/s", peak=peaks["hbm"],
+                        frac=ach / peaks["hbm"], peak_src=f"HBM copy, {peaks['src']}")
+    rec = NCU_TRAFFIC.get(kind)
+    roof["traffic"] = rec["bytes"] if rec and rec["src_hash"] == kernel_source_hash(kind) else None
+
+    breakdown = {k: {"launches": n, "ms_per_round": ms / K} for k, (n, ms) in
+                 sorted(ktimes.items(), key=lambda kv: -kv[1][1])}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": step_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.bf16 else "f32",
+        "data": "synthetic",
+        "config": {"workload": f"{w.name}: n={w.n} K={w.num_clients} C={w.num_clusters} "
+                               f"B={w.B} F={w.F} SplitCNN" if w.arch == 1 else w.name,
+                   "global_batch": w.num_clusters * w.B * world, "parallelism": f"replicas{world}",
+                   "l2": "flushed between timed steps (256 MiB write)"},
+        "roofline": roof, "gpu_launches": launches, "wall_s": wall,
+        "kernels": breakdown,
+    }
+    clocks = clk.summary()
+    line["clocks"] = clocks
+
+    if rank == 0 and not args.no_extras:
+        line["e2e"] = e2e_leg(pkg, w, ds, assign, params, torch, flush, max(10, K // 3))
+        line["serialized"] = serialized_leg(pkg, w, ds, assign, params, torch, flush,
+                                            max(5, K // 6), value)
+        line["fusion"] = fusion_leg(ctx, w, torch, flush, peaks)
+    if rank == 0 and not args.no_cpu_baseline:
+        v, cores, desc = cpu_baseline(w, ds, assign, params)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": desc}
+    ctx.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def e2e_leg(pkg, w, ds, assign, params, torch, flush, K):
+    """The same metric through the public API with the images in pinned host
+    memory (data_on_host): every round reads its C*B sampled fp32 images from
+    host memory over NVLink-C2C and returns the per-cluster loss and |A| to
+    the host (gcpsl_step with stats, which synchronises)."""
+    ctx = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
+                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=w.bf16,
+                      data_on_host=True)
+    for _ in range(3):
+        ctx.step(stats=True)
+    tot = 0.0
+    for i in range(K):
+        flush.fill_(float(i))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        ctx.step(stats=True)
+        tot += time.perf_counter() - t0
+    ctx.close()
+    return {"value": w.num_clusters * w.B * K / tot, "unit": UNIT,
+            "h2d_bytes_per_step": w.num_clusters * w.B * 3072 * 4,
+            "d2h_bytes_per_step": w.num_clusters * 8,
+            "how": "gcpsl_step(stats) wall time; images gathered from pinned host memory"}
+
+
+def serialized_leg(pkg, w, ds, assign, params, torch, flush, K, grouped_value):
+    """The paper's sequential control on one GPU: the C workloads as C
+    one-cluster contexts stepped one after another (same kernels)."""
+    ctxs = [pkg.Context(w.arch, w.num_clients, 1, np.where(assign == n, 0, -1).astype(np.int32),
+                        w.B, 0, 4, ds.images, ds.labels, ds.owner, params, lr=w.lr,
+                        momentum=w.momentum, bf16=w.bf16, cluster_id_base=n)
+            for n in range(w.num_clusters)]
+    stream = torch.cuda.current_stream()
+    for c in ctxs:
+        c.set_stream(stream.cuda_stream)
+        c.step()
+    tot = 0.0
+    for i in range(K):
+        flush.fill_(float(i))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for c in ctxs:
+            c.step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        tot += a.elapsed_time(b)
+    for c in ctxs:
+        c.close()
+    v = w.num_clusters * w.B * K / (tot / 1e3)
+    return {"value": v, "unit": UNIT, "grouped_over_serialized": grouped_value / v}
+
+
+def fusion_leg(ctx, w, torch, flush, peaks):
+    """Explicit fusion calls, L2 flushed before each: achieved GB/s of
+    reading C*P fp32 and writing C*P fp32 (+ the bf16 shadow)."""
+    stream = torch.cuda.current_stream()
+    P = ctx.P_client + ctx.P_server
+    nbytes = w.num_clusters * P * (4 + 4 + (2 if w.bf16 else 0))
+    tot, K = 0.0, 20
+    for i in range(K):
+        flush.fill_(float(i))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        ctx.fuse()
+        b.record(stream)
+        torch.cuda.synchronize()
+        tot += a.elapsed_time(b)
+    gbs = nbytes * K / (tot / 1e3) / 1e9
+    return {"bytes_per_call": nbytes, "ms_per_call": tot / K, "achieved_gbs": gbs,
+            "frac_of_hbm": gbs / peaks["hbm"]}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

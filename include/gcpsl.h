@@ -1,0 +1,203 @@
+/*
+ * gcpsl.h -- C ABI of the GB300 GCPSL training-step library (libgcpsl.so).
+ *
+ * GCPSL ("Concurrent Split Learning Through Stable Client Clustering",
+ * Kohankhaki, Rentschler, Schmeink) assigns K clients to N fixed clusters,
+ * runs one GPSL workload with a fixed batch B per cluster, and fuses the
+ * split-model replicas every F local rounds (Algorithm 2).  This library
+ * keeps the C cluster replicas (the paper's N) resident on one GPU and runs
+ * one local round of all of them per call, as grouped CUDA kernels with the
+ * replica index in the grid.
+ *
+ * Conventions shared by every entry point
+ *  - Every call returns a gcpsl_status and never aborts the process.
+ *  - Host pointers passed in are owned by the caller.  gcpsl_init copies
+ *    what it needs (except the images with data_on_host = 1, see below), so
+ *    the caller may free its arrays after init returns.
+ *  - The context owns all device memory it allocates; gcpsl_destroy frees it.
+ *  - gcpsl_step and gcpsl_fuse are asynchronous on the context's stream;
+ *    every getter synchronises that stream first.
+ *  - After a CUDA error or a device-side timeout the context is "sticky":
+ *    later calls return GCPSL_E_STATE.  gcpsl_last_error describes the cause.
+ *  - One host thread at a time per context.
+ */
+#ifndef GCPSL_H
+#define GCPSL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  GCPSL_OK = 0,
+  GCPSL_E_INVAL = 1,        /* bad argument (value, size, NULL) */
+  GCPSL_E_NOMEM = 2,        /* host or device allocation failed */
+  GCPSL_E_CUDA = 3,         /* a CUDA runtime call failed */
+  GCPSL_E_STATE = 4,        /* call on a context in the error state */
+  GCPSL_E_TIMEOUT = 5,      /* a device-side wait gave up */
+  GCPSL_E_UNSUPPORTED = 6   /* architecture / dtype combination not built */
+} gcpsl_status;
+
+/* Split-model architectures.  Conv layers are 3x3, stride 1, padding 1, with
+ * bias, each followed by ReLU; "pool" is a 2x2 stride-2 max-pool.
+ *  TINY_CNN : client conv 3->16 pool | server conv 16->32 pool, FC 2048->10
+ *  SPLIT_CNN: client conv 3->32, conv 32->64 pool (cut 64x16x16) |
+ *             server conv 64->128 pool, conv 128->128 pool, FC 2048->10   */
+enum { GCPSL_TINY_CNN = 0, GCPSL_SPLIT_CNN = 1, GCPSL_RESNET18 = 2 };
+enum { GCPSL_F32 = 0, GCPSL_BF16 = 1 };
+enum { GCPSL_CLIENT = 0, GCPSL_SERVER = 1 };
+enum { GCPSL_CUT_ACT = 0, GCPSL_CUT_GRAD = 1 };
+
+/* Model and optimiser description.
+ *  operand_dtype: GCPSL_F32 computes in fp32 throughout; GCPSL_BF16 stores
+ *    weights (as a shadow of the fp32 master), activations and gradients of
+ *    activations in bf16 and accumulates in fp32.
+ *  SGD follows PyTorch: g += weight_decay*theta; v = momentum*v + g (v starts
+ *    at 0, so the first round takes v = g); theta -= lr*(nesterov ? g +
+ *    momentum*v : v); with momentum 0, theta -= lr*g.
+ *  label_smoothing e: cross-entropy target (1-e)*onehot + e/classes.
+ *  cluster_id_base: cluster n draws its sampler keys with cluster id
+ *    cluster_id_base + n (lets C one-cluster contexts reproduce one
+ *    C-cluster context exactly).
+ *  data_on_host: 0 = images copied to device memory at init; 1 = images stay
+ *    in pinned, device-mapped host memory owned by the context and each round
+ *    gathers its B sampled images per cluster from there.               */
+typedef struct {
+  int arch;
+  int operand_dtype;
+  float lr, momentum, weight_decay;
+  int nesterov;
+  float label_smoothing;
+  int cluster_id_base;
+  int data_on_host;
+} gcpsl_model_desc;
+
+/* Training data of all K clients (Section III-A: client k owns D_k).
+ *  images: n x 3 x 32 x 32 fp32, NCHW;  labels: n values in [0, classes);
+ *  owner: client id of each example, in [0, K).                          */
+typedef struct {
+  const float* images;
+  const int32_t* labels;
+  const int32_t* owner;
+  int64_t n;
+  int num_classes;        /* must be 10 for the built architectures */
+} gcpsl_dataset;
+
+/* Per-round statistics, written by gcpsl_step when non-NULL (forces a sync).
+ *  loss[n]: mean softmax cross-entropy of cluster n's batch;
+ *  active[n]: |A_{n,t}|, clients that supplied >= 1 example (Eq. 3).     */
+typedef struct {
+  float* loss;            /* caller-owned, C entries */
+  int32_t* active;        /* caller-owned, C entries */
+} gcpsl_step_stats;
+
+typedef struct gcpsl_ctx gcpsl_ctx;
+
+/* gcpsl_init -- set up C cluster workloads (Algorithm 2, "initialize all
+ * split-model replicas equally").
+ *  desc: model/optimiser; K clients; C clusters;
+ *  assignment[K]: cluster of each client (Algorithm 1's fixed map), in
+ *    [0, C), or -1 for a client this context does not serve;
+ *  B: per-cluster batch (Eq. 1, sum_k b_{k,t} = B); F: fuse after every F-th
+ *    round (0 = never; gcpsl_fuse can still be called);
+ *  seed: sampler seed (Philox4x32-10 key);
+ *  data: the dataset (see gcpsl_dataset);
+ *  init_params: NULL or the initial parameters of one replica as fp32, client
+ *    segment then server segment, each in PyTorch state_dict order (conv
+ *    weights OIHW, linear weight [out][in]); NULL draws them from a fixed
+ *    Philox stream as U(-1/sqrt(fan_in), 1/sqrt(fan_in));
+ *  out: receives the context.
+ * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < 0, assignment
+ * outside [-1, C), owner outside [0, K), labels outside [0, classes), a
+ * cluster with fewer than B examples.  Fusion weights are
+ * q_n = n_c / sum_m n_m over this context's clusters (Eq. 5).            */
+gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_t* assignment,
+                        int B, int F, uint64_t seed, const gcpsl_dataset* data,
+                        const float* init_params, gcpsl_ctx** out);
+
+/* gcpsl_step -- one local round of every cluster (Algorithm 2's inner loop
+ * body): GPSL sampling of B examples (Eq. 1; epoch = one pass over a random
+ * permutation of the cluster's examples, the n_c mod B remainder left out),
+ * client-segment forward to the cut, server forward, softmax cross-entropy
+ * (mean over the batch), backward to the cut gradient and through the client
+ * segment, and an SGD update of every replica; then, when the number of
+ * rounds taken is a multiple of F, fusion (Eq. 5).  stats may be NULL.   */
+gcpsl_status gcpsl_step(gcpsl_ctx* ctx, gcpsl_step_stats* stats);
+
+/* gcpsl_fuse -- Eq. 5: theta_bar = sum_n q_n theta_n for all parameters,
+ * written back to every replica (Section IV-C broadcast).  Momentum buffers
+ * stay per replica.                                                      */
+gcpsl_status gcpsl_fuse(gcpsl_ctx* ctx);
+
+/* gcpsl_get_params -- copy replica `cluster`'s parameters of `segment`
+ * (GCPSL_CLIENT / GCPSL_SERVER) as fp32 in the init_params order into dst.
+ * dst == NULL (or len too small) only reports the needed count in *needed
+ * (and returns GCPSL_E_INVAL if dst is non-NULL but too small).          */
+gcpsl_status gcpsl_get_params(gcpsl_ctx* ctx, int cluster, int segment, float* dst, size_t len,
+                              size_t* needed);
+
+/* gcpsl_set_params -- overwrite replica `cluster`'s parameters (both
+ * segments, init_params order and length).  Momentum is left unchanged.  */
+gcpsl_status gcpsl_set_params(gcpsl_ctx* ctx, int cluster, const float* src, size_t len);
+
+/* gcpsl_get_momentum / gcpsl_set_momentum -- replica `cluster`'s SGD
+ * momentum buffer (Section IV-C: optimiser state stays per replica), both
+ * segments in the init_params order; len must equal the parameter count.
+ * With set_params this checkpoints and restores a replica exactly.       */
+gcpsl_status gcpsl_get_momentum(gcpsl_ctx* ctx, int cluster, float* dst, size_t len);
+gcpsl_status gcpsl_set_momentum(gcpsl_ctx* ctx, int cluster, const float* src, size_t len);
+
+/* gcpsl_get_pool_codes -- the last round's max-pool decisions of conv layer
+ * `layer` (0-based over client then server layers; it must be pooled), one
+ * byte per pooled output, laid out [C][B][channels][h/2][w/2]: bits 0-1 are
+ * the window position of the first maximum in row-major order, bit 2 is set
+ * when that maximum is positive (the output then carries a gradient).     */
+gcpsl_status gcpsl_get_pool_codes(gcpsl_ctx* ctx, int layer, uint8_t* dst, size_t len);
+
+/* gcpsl_get_cut -- the last round's cut activation z (GCPSL_CUT_ACT) or cut
+ * gradient dL/dz (GCPSL_CUT_GRAD) of every cluster as fp32, laid out
+ * [C][B][channels][h][w].  len is in floats; dst NULL reports nothing but
+ * returns GCPSL_E_INVAL (use gcpsl_cut_elems).                           */
+gcpsl_status gcpsl_get_cut(gcpsl_ctx* ctx, int which, float* dst, size_t len);
+size_t gcpsl_cut_elems(const gcpsl_ctx* ctx);
+
+/* gcpsl_get_sample -- the last round's batches: idx[C][B] global example
+ * ids ordered by (owner, id) within each cluster, and counts[C][K] with
+ * counts[n][k] = b_{k,t} of Eq. 1 (0 for clients outside cluster n).
+ * Either pointer may be NULL.                                            */
+gcpsl_status gcpsl_get_sample(gcpsl_ctx* ctx, int32_t* idx, int32_t* counts);
+
+/* gcpsl_num_params -- parameters per replica of a segment (-1: bad arch). */
+int64_t gcpsl_num_params(int arch, int segment);
+
+/* gcpsl_rounds -- local rounds taken so far.                             */
+int64_t gcpsl_rounds(const gcpsl_ctx* ctx);
+
+/* gcpsl_set_stream -- run on the caller's cudaStream_t (passed as void*);
+ * NULL returns to the context's own stream.  Synchronises the old stream. */
+gcpsl_status gcpsl_set_stream(gcpsl_ctx* ctx, void* cuda_stream);
+
+/* Kernel timing: when enabled, every kernel the context launches is
+ * bracketed by CUDA events on its stream.  gcpsl_kernel_times fills, for up
+ * to `cap` kernel kinds, the name (static string), the number of launches
+ * and the summed device milliseconds since the last reset, and returns the
+ * number of kinds (synchronises).                                        */
+gcpsl_status gcpsl_set_timing(gcpsl_ctx* ctx, int enable);
+int gcpsl_kernel_times(gcpsl_ctx* ctx, const char** names, int64_t* launches, double* ms,
+                       int cap);
+void gcpsl_reset_kernel_times(gcpsl_ctx* ctx);
+
+/* gcpsl_last_error -- static description of the context's last failure
+ * (or of the last failed gcpsl_init when ctx is NULL).                   */
+const char* gcpsl_last_error(const gcpsl_ctx* ctx);
+
+/* gcpsl_destroy -- free the context (NULL is a no-op).                   */
+void gcpsl_destroy(gcpsl_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GCPSL_H */

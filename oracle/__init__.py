@@ -76,6 +76,14 @@ def _declare(L):
     L.orc_get_q.argtypes = [ct.c_void_p, f64p]
     L.orc_rounds.argtypes = [ct.c_void_p]
     L.orc_rounds.restype = ct.c_int64
+    L.orc_get_momentum.argtypes = [ct.c_void_p, ct.c_int, f64p]
+    L.orc_set_momentum.argtypes = [ct.c_void_p, ct.c_int, f64p]
+    L.orc_set_tie_tol.argtypes = [ct.c_void_p, ct.c_double]
+    L.orc_set_tie_tol.restype = None
+    L.orc_get_pool_cand.argtypes = [ct.c_void_p, ct.c_int, _p(ct.c_uint8)]
+    L.orc_get_pool_cand.restype = ct.c_int64
+    L.orc_get_ties.argtypes = [ct.c_void_p, i32p]
+    L.orc_get_ties.restype = None
     L.orc_set_threads.argtypes = [ct.c_int]
     L.orc_get_threads.restype = ct.c_int
 
@@ -212,6 +220,35 @@ class Oracle:
     def set_params(self, cluster: int, blob):
         blob = np.ascontiguousarray(blob, dtype=np.float64)
         lib().orc_set_params(self._h, cluster, _ptr(blob, ct.c_double))
+
+    def momentum(self, cluster: int):
+        out = np.zeros(self.P_client + self.P_server)
+        lib().orc_get_momentum(self._h, cluster, _ptr(out, ct.c_double))
+        return out
+
+    def set_momentum(self, cluster: int, v):
+        v = np.ascontiguousarray(v, dtype=np.float64)
+        lib().orc_set_momentum(self._h, cluster, _ptr(v, ct.c_double))
+
+    def set_tie_tol(self, tol: float):
+        lib().orc_set_tie_tol(self._h, tol)
+
+    def pool_cand(self, layer: int):
+        """Per pooled window of the last round, [C][B][cout][Ho][Wo] bytes:
+        bits 0-3 valid argmax positions, bit 4 max > 0, bit 5 sign ambiguous
+        (None for a layer without pooling)."""
+        n = lib().orc_get_pool_cand(self._h, layer, None)
+        if n == 0:
+            return None
+        out = np.zeros(n, dtype=np.uint8)
+        lib().orc_get_pool_cand(self._h, layer, _ptr(out, ct.c_uint8))
+        return out.reshape(self.C, self.B, -1)
+
+    def ties(self):
+        """[C][B] number of ambiguous pooled windows per example, last round."""
+        out = np.zeros((self.C, self.B), dtype=np.int32)
+        lib().orc_get_ties(self._h, _ptr(out, ct.c_int32))
+        return out
 
     def sample(self):
         idx = np.zeros((self.C, self.B), dtype=np.int32)

@@ -274,26 +274,44 @@ static void conv3x3_dgrad(int B, int cin, int cout, int H, int W, const double* 
 }
 
 /* out = maxpool2x2(relu(y)) or relu(y); arg = first maximum of the window in
- * row-major order (0..3). */
+ * row-major order (0..3).
+ * cand (pooled layers) describes how sharp each window's decision is, for
+ * comparisons against an implementation that accumulates in another order:
+ * bits 0-3 = the positions q with relu(y_q) >= best - tol*rms(y), rms over
+ * the whole layer (the valid maxima), bit 4 = best > 0, bit 5 = the window's
+ * largest y lies within tol*rms(y) of zero (the ReLU decision itself is
+ * ambiguous).  With tol = 0 only exact ties are candidates. */
 static void relu_pool_fwd(int B, int C, int H, int W, int pool, const double* y, double* out,
-                          int8_t* arg) {
+                          int8_t* arg, uint8_t* cand, double tol) {
   if (!pool) {
     for (int64_t i = 0; i < (int64_t)B * C * H * W; ++i) out[i] = y[i] > 0.0 ? y[i] : 0.0;
     return;
   }
+  double rms = 0.0;
+  for (int64_t i = 0; i < (int64_t)B * C * H * W; ++i) rms += y[i] * y[i];
+  rms = sqrt(rms / ((double)B * C * H * W));
   int Ho = H / 2, Wo = W / 2;
   for (int64_t bc = 0; bc < (int64_t)B * C; ++bc)
     for (int ph = 0; ph < Ho; ++ph)
       for (int pw = 0; pw < Wo; ++pw) {
         const double* yp = y + bc * H * W;
-        double best = 0.0; int bi = 0;
+        double v[4], best = 0.0, ymax = 0.0; int bi = 0;
         for (int q = 0; q < 4; ++q) {
-          double v = yp[(2 * ph + q / 2) * W + 2 * pw + q % 2];
-          v = v > 0.0 ? v : 0.0;
-          if (q == 0 || v > best) { best = v; bi = q; }
+          v[q] = yp[(2 * ph + q / 2) * W + 2 * pw + q % 2];
+          if (q == 0 || v[q] > ymax) ymax = v[q];
+          v[q] = v[q] > 0.0 ? v[q] : 0.0;
+          if (q == 0 || v[q] > best) { best = v[q]; bi = q; }
         }
-        out[(bc * Ho + ph) * Wo + pw] = best;
-        arg[(bc * Ho + ph) * Wo + pw] = (int8_t)bi;
+        int64_t o = (bc * Ho + ph) * Wo + pw;
+        out[o] = best;
+        arg[o] = (int8_t)bi;
+        if (cand) {
+          uint8_t m = 0;
+          for (int q = 0; q < 4; ++q) if (v[q] >= best - tol * rms) m |= (uint8_t)(1u << q);
+          if (best > 0.0) m |= 16u;
+          if (fabs(ymax) <= tol * rms) m |= 32u;
+          cand[o] = m;
+        }
       }
 }
 
@@ -327,6 +345,7 @@ typedef struct {
   double* act[5];     /* act[0] = input, act[i+1] = output of conv i */
   double* pre[4];     /* pre-activation of conv i */
   int8_t* arg[4];
+  uint8_t* cand[4];   /* decision sharpness of each pooled window (see relu_pool_fwd) */
   double* dact[5];
   double* dpre;
   double* h;          /* flattened features [B, fc_in] */
@@ -341,7 +360,7 @@ static int64_t conv_out_elems(const conv_l* c, int B) {
 
 static void work_free(work_t* w) {
   for (int i = 0; i < 5; ++i) { free(w->act[i]); free(w->dact[i]); }
-  for (int i = 0; i < 4; ++i) { free(w->pre[i]); free(w->arg[i]); }
+  for (int i = 0; i < 4; ++i) { free(w->pre[i]); free(w->arg[i]); free(w->cand[i]); }
   free(w->dpre); free(w->h); free(w->logits); free(w->dlogits); free(w->wr);
   memset(w, 0, sizeof(*w));
 }
@@ -357,6 +376,7 @@ static int work_alloc(work_t* w, const arch_t* a, const offs_t* o, int B) {
     if (np > maxpre) maxpre = np;
     w->pre[i] = (double*)calloc((size_t)np, sizeof(double));
     w->arg[i] = (int8_t*)calloc((size_t)np, 1);
+    w->cand[i] = (uint8_t*)calloc((size_t)np, 1);
     w->act[i + 1] = (double*)calloc((size_t)conv_out_elems(&a->conv[i], B), sizeof(double));
     w->dact[i + 1] = (double*)calloc((size_t)conv_out_elems(&a->conv[i], B), sizeof(double));
   }
@@ -373,7 +393,7 @@ static int work_alloc(work_t* w, const arch_t* a, const offs_t* o, int B) {
 
 static int fwd_bwd(const arch_t* a, const offs_t* o, int bf16, double label_smoothing,
                    const double* params, int B, const int32_t* labels, work_t* w,
-                   double* loss_out, double* grad) {
+                   double* loss_out, double* grad, double tie_tol) {
   int L = a->ncl + a->nsv;
   /* operand copy: bf16(theta) for weights in bf16 mode; biases stay exact */
   memcpy(w->wr, params, sizeof(double) * (size_t)o->p_total);
@@ -386,7 +406,8 @@ static int fwd_bwd(const arch_t* a, const offs_t* o, int bf16, double label_smoo
   for (int i = 0; i < L; ++i) {
     const conv_l* c = &a->conv[i];
     conv3x3_fwd(B, c->cin, c->cout, c->h, c->w, w->act[i], w->wr + o->w[i], w->wr + o->b[i], w->pre[i]);
-    relu_pool_fwd(B, c->cout, c->h, c->w, c->pool, w->pre[i], w->act[i + 1], w->arg[i]);
+    relu_pool_fwd(B, c->cout, c->h, c->w, c->pool, w->pre[i], w->act[i + 1], w->arg[i],
+                  w->cand[i], tie_tol);
     round_buf(w->act[i + 1], conv_out_elems(c, B), bf16);
   }
   /* flatten (C, H, W) order == NCHW memory order of act[L] */
@@ -465,7 +486,7 @@ int orc_forward_backward(int arch, int bf16, double label_smoothing, const doubl
   if (work_alloc(&w, &a, &o, B)) return ORC_ENOMEM;
   memcpy(w.act[0], x, sizeof(double) * (size_t)B * 3072);
   double* g = grad ? grad : NULL;
-  int rc = fwd_bwd(&a, &o, bf16, label_smoothing, params, B, labels, &w, loss, g);
+  int rc = fwd_bwd(&a, &o, bf16, label_smoothing, params, B, labels, &w, loss, g, 0.0);
   int64_t ncut = conv_out_elems(&a.conv[a.ncl - 1], B);
   if (cut_act) memcpy(cut_act, w.act[a.ncl], sizeof(double) * (size_t)ncut);
   if (cut_grad && g) memcpy(cut_grad, w.dact[a.ncl], sizeof(double) * (size_t)ncut);
@@ -507,6 +528,9 @@ typedef struct {
   int64_t ncut;
   work_t w;
   double* xbuf; int32_t* ybuf;
+  double tie_tol;                             /* see relu_pool_fwd */
+  uint8_t* cand[4];                           /* [C][B][cout][Ho][Wo] of the last round */
+  int32_t* ties;                              /* [C][B] ambiguous windows per example */
 } orc_ctx;
 
 void orc_destroy(orc_ctx* c);
@@ -570,6 +594,11 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   c->cut_act = (double*)calloc((size_t)(C * c->ncut), sizeof(double));
   c->cut_grad = (double*)calloc((size_t)(C * c->ncut), sizeof(double));
   c->ybuf = (int32_t*)calloc((size_t)B, sizeof(int32_t));
+  c->tie_tol = 1e-3;
+  for (int i = 0; i < a.ncl + a.nsv; ++i)
+    if (a.conv[i].pool)
+      c->cand[i] = (uint8_t*)calloc((size_t)C * conv_out_elems(&a.conv[i], B), 1);
+  c->ties = (int32_t*)calloc((size_t)C * B, sizeof(int32_t));
   if (!c->theta || !c->mom || !c->grad || !c->cut_act || !c->cut_grad ||
       work_alloc(&c->w, &a, &c->o, B)) { orc_destroy(c); return ORC_ENOMEM; }
   *out = c;
@@ -582,7 +611,8 @@ void orc_destroy(orc_ctx* c) {
   free(c->ids); free(c->perm); free(c->nc); free(c->cur_epoch); free(c->q);
   free(c->labels); free(c->owner); free(c->theta); free(c->mom); free(c->grad);
   free(c->idx); free(c->counts); free(c->loss); free(c->active);
-  free(c->cut_act); free(c->cut_grad); free(c->ybuf);
+  free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties);
+  for (int i = 0; i < 4; ++i) free(c->cand[i]);
   work_free(&c->w);
   free(c);
 }
@@ -634,8 +664,19 @@ int orc_step(orc_ctx* c) {
     }
     int64_t P = c->o.p_total;
     int rc = fwd_bwd(&c->a, &c->o, c->bf16, c->ls, c->theta + k * P, B, c->ybuf, &c->w,
-                     &c->loss[k], c->grad + k * P);
+                     &c->loss[k], c->grad + k * P, c->tie_tol);
     if (rc) return rc;
+    for (int b = 0; b < B; ++b) c->ties[(int64_t)k * B + b] = 0;
+    for (int i = 0; i < c->a.ncl + c->a.nsv; ++i) {
+      if (!c->cand[i]) continue;
+      int64_t per = conv_out_elems(&c->a.conv[i], B);
+      memcpy(c->cand[i] + k * per, c->w.cand[i], (size_t)per);
+      for (int64_t e = 0; e < per; ++e) {
+        uint8_t m = c->w.cand[i][e];
+        int multi = (m & 15u) != 1u && (m & 15u) != 2u && (m & 15u) != 4u && (m & 15u) != 8u;
+        if (((m & 16u) && multi) || (m & 32u)) c->ties[(int64_t)k * B + e / (per / B)]++;
+      }
+    }
     memcpy(c->cut_act + k * c->ncut, c->w.act[c->a.ncl], sizeof(double) * (size_t)c->ncut);
     memcpy(c->cut_grad + k * c->ncut, c->w.dact[c->a.ncl], sizeof(double) * (size_t)c->ncut);
   }
@@ -676,6 +717,35 @@ void orc_get_stats(const orc_ctx* c, double* loss, int32_t* active) {
 int64_t orc_get_cut(const orc_ctx* c, int which, double* dst) {
   if (dst) memcpy(dst, which ? c->cut_grad : c->cut_act, sizeof(double) * (size_t)(c->C * c->ncut));
   return c->C * c->ncut;
+}
+
+/* momentum buffer of one replica, canonical order, both segments */
+int orc_get_momentum(const orc_ctx* c, int cluster, double* dst) {
+  if (cluster < 0 || cluster >= c->C) return ORC_EINVAL;
+  memcpy(dst, c->mom + (int64_t)cluster * c->o.p_total, sizeof(double) * (size_t)c->o.p_total);
+  return ORC_OK;
+}
+
+int orc_set_momentum(orc_ctx* c, int cluster, const double* src) {
+  if (cluster < 0 || cluster >= c->C) return ORC_EINVAL;
+  memcpy(c->mom + (int64_t)cluster * c->o.p_total, src, sizeof(double) * (size_t)c->o.p_total);
+  return ORC_OK;
+}
+
+void orc_set_tie_tol(orc_ctx* c, double tol) { c->tie_tol = tol; }
+
+/* decision sharpness of pooled layer `layer` in the last round,
+ * [C][B][cout][Ho][Wo]; returns the element count (0: layer not pooled) */
+int64_t orc_get_pool_cand(const orc_ctx* c, int layer, uint8_t* dst) {
+  if (layer < 0 || layer >= c->a.ncl + c->a.nsv || !c->cand[layer]) return 0;
+  int64_t n = c->C * conv_out_elems(&c->a.conv[layer], c->B);
+  if (dst) memcpy(dst, c->cand[layer], (size_t)n);
+  return n;
+}
+
+/* ambiguous windows per example in the last round, [C][B] */
+void orc_get_ties(const orc_ctx* c, int32_t* dst) {
+  memcpy(dst, c->ties, sizeof(int32_t) * (size_t)c->C * c->B);
 }
 
 void orc_get_q(const orc_ctx* c, double* q) { memcpy(q, c->q, sizeof(double) * (size_t)c->C); }

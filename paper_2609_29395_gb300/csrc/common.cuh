@@ -1,0 +1,114 @@
+// Internal declarations of libgcpsl.so (not part of the C ABI).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace gcpsl {
+
+typedef __nv_bfloat16 bf16;
+
+// ---------------------------------------------------------------------------
+// Split-model description.  Conv layers: 3x3, stride 1, pad 1, bias, ReLU,
+// optional 2x2/2 max-pool.  Activations are NHWC with the replica index
+// outermost: [C][B][H][W][ch].
+// ---------------------------------------------------------------------------
+struct ConvSpec { int cin, cout, h, w, pool; };
+struct ArchSpec {
+  int ncl, nsv;          // client / server conv layers (ncl + nsv <= 4)
+  ConvSpec conv[4];
+  int fc_in, fc_out;
+  // parameter offsets within one replica, same order as the PyTorch
+  // state_dict: conv{i}.weight, conv{i}.bias, ..., fc.weight, fc.bias
+  int64_t off_w[4], off_b[4], off_fcw, off_fcb, p_client, p_total;
+  int L() const { return ncl + nsv; }
+  int out_h(int i) const { return conv[i].pool ? conv[i].h / 2 : conv[i].h; }
+  int out_w(int i) const { return conv[i].pool ? conv[i].w / 2 : conv[i].w; }
+};
+bool make_arch(int id, ArchSpec* a);
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon et al., SC'11): ten rounds, two 32x32 -> 64-bit
+// products per round, key bumped by the Weyl increments between rounds.
+// ---------------------------------------------------------------------------
+__host__ __device__ inline void philox4x32_10(uint32_t c[4], uint32_t k0, uint32_t k1) {
+  const uint32_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u;
+  const uint32_t W0 = 0x9E3779B9u, W1 = 0xBB67AE85u;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) { k0 += W0; k1 += W1; }
+    uint64_t p0 = (uint64_t)M0 * c[0];
+    uint64_t p1 = (uint64_t)M1 * c[2];
+    uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ k0;
+    uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ k1;
+    c[1] = (uint32_t)p1;
+    c[3] = (uint32_t)p0;
+    c[0] = n0;
+    c[2] = n2;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Element conversions for the two storage types
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+// ---------------------------------------------------------------------------
+// Kernel launchers (each enqueues on `s`; return the launch error)
+// ---------------------------------------------------------------------------
+// sampler.cu
+cudaError_t launch_epoch_keys(cudaStream_t s, const int32_t* ids, const int64_t* off,
+                              const int32_t* rounds, const int64_t* d_t, int cluster_base,
+                              uint64_t seed, uint64_t* keys, int C, int64_t max_nc);
+cudaError_t launch_epoch_rank(cudaStream_t s, const int32_t* ids, const int64_t* off,
+                              const int32_t* rounds, const int64_t* d_t, const uint64_t* keys,
+                              int32_t* perm, int C, int64_t max_nc);
+cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* off,
+                          const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
+                          const int32_t* labels, int K, int B, int C, int32_t* idx,
+                          int32_t* counts, int32_t* active, int32_t* y);
+template <typename T>
+cudaError_t launch_gather(cudaStream_t s, const float* images, const int32_t* idx, int CB, T* x0);
+
+// conv_simt.cu
+template <typename T>
+cudaError_t launch_conv_fwd_simt(cudaStream_t s, const T* x, const T* w, int64_t w_rs,
+                                 const float* bias, int64_t b_rs, T* out, uint8_t* code, int C,
+                                 int B, const ConvSpec& cs);
+template <typename T>
+cudaError_t launch_relu_pool_bwd(cudaStream_t s, const T* dout, const uint8_t* code,
+                                 const T* act, T* g, int C, int B, const ConvSpec& cs);
+template <typename T>
+cudaError_t launch_conv_dgrad_simt(cudaStream_t s, const T* g, const T* w, int64_t w_rs, T* dx,
+                                   int C, int B, const ConvSpec& cs);
+template <typename T>
+cudaError_t launch_conv_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* dw,
+                                   int64_t dw_rs, int C, int B, const ConvSpec& cs);
+template <typename T>
+cudaError_t launch_bias_grad(cudaStream_t s, const T* g, float* db, int64_t db_rs, int C, int B,
+                             const ConvSpec& cs);
+
+// head.cu
+template <typename T>
+cudaError_t launch_fc_fwd(cudaStream_t s, const T* h, const T* w, int64_t w_rs, const float* b,
+                          int64_t b_rs, float* logits, int C, int B, int fin, int fout);
+cudaError_t launch_softmax_ce(cudaStream_t s, const float* logits, const int32_t* y, float* loss,
+                              float* dlogits, int C, int B, int fout, float label_smoothing);
+template <typename T>
+cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const T* h, const T* w,
+                          int64_t w_rs, float* dw, float* db, int64_t g_rs, T* dh, int C, int B,
+                          int fin, int fout);
+
+// optim.cu
+cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,
+                       bf16* shadow, int64_t n, float lr, float momentum, float wd,
+                       int nesterov, int64_t* d_t);
+cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,
+                        int64_t P);
+
+}  // namespace gcpsl

@@ -1,0 +1,749 @@
+// Host side of libgcpsl.so: the C ABI declared in include/gcpsl.h.
+//
+// A context holds C cluster workloads (the paper's N execution slots,
+// Section III-A) resident on one GPU: every replica's fp32 parameters,
+// momentum and gradients as one [C][P] store, the bf16 operand shadow, the
+// activations of the current round as [C][B][H][W][ch] tensors, the sampler
+// state, and the dataset.  gcpsl_step enqueues one local round of every
+// cluster (Algorithm 2's inner loop body) as grouped kernels on one stream.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "gcpsl.h"
+
+using namespace gcpsl;
+
+// ---------------------------------------------------------------------------
+// Architectures
+// ---------------------------------------------------------------------------
+bool gcpsl::make_arch(int id, ArchSpec* a) {
+  std::memset(a, 0, sizeof(*a));
+  if (id == GCPSL_TINY_CNN) {
+    a->ncl = 1; a->nsv = 1;
+    a->conv[0] = {3, 16, 32, 32, 1};
+    a->conv[1] = {16, 32, 16, 16, 1};
+  } else if (id == GCPSL_SPLIT_CNN) {
+    a->ncl = 2; a->nsv = 2;
+    a->conv[0] = {3, 32, 32, 32, 0};
+    a->conv[1] = {32, 64, 32, 32, 1};
+    a->conv[2] = {64, 128, 16, 16, 1};
+    a->conv[3] = {128, 128, 8, 8, 1};
+  } else {
+    return false;
+  }
+  a->fc_in = 2048; a->fc_out = 10;
+  int64_t p = 0;
+  for (int i = 0; i < a->L(); ++i) {
+    if (i == a->ncl) a->p_client = p;
+    a->off_w[i] = p; p += (int64_t)a->conv[i].cout * 9 * a->conv[i].cin;
+    a->off_b[i] = p; p += a->conv[i].cout;
+  }
+  a->off_fcw = p; p += (int64_t)a->fc_out * a->fc_in;
+  a->off_fcb = p; p += a->fc_out;
+  a->p_total = p;
+  return true;
+}
+
+// ---------------------------------------------------------------------------
+// Kernel timing with CUDA events on the context's stream
+// ---------------------------------------------------------------------------
+namespace {
+
+struct KernelTimer {
+  std::vector<const char*> names;
+  std::vector<int64_t> launches;
+  std::vector<double> ms;
+  struct Pending { int kind; cudaEvent_t a, b; };
+  std::vector<Pending> pending;
+  std::vector<cudaEvent_t> pool;
+  int cur_kind = -1;
+  cudaEvent_t cur_a = nullptr;
+
+  int kind(const char* name) {
+    for (size_t i = 0; i < names.size(); ++i)
+      if (names[i] == name || std::strcmp(names[i], name) == 0) return (int)i;
+    names.push_back(name); launches.push_back(0); ms.push_back(0.0);
+    return (int)names.size() - 1;
+  }
+  cudaEvent_t get() {
+    if (!pool.empty()) { cudaEvent_t e = pool.back(); pool.pop_back(); return e; }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+  }
+  void begin(const char* name, cudaStream_t s) {
+    cur_kind = kind(name);
+    cur_a = get();
+    cudaEventRecord(cur_a, s);
+  }
+  void end(cudaStream_t s) {
+    cudaEvent_t b = get();
+    cudaEventRecord(b, s);
+    pending.push_back({cur_kind, cur_a, b});
+  }
+  void collect() {
+    for (auto& p : pending) {
+      float t = 0.f;
+      if (cudaEventSynchronize(p.b) == cudaSuccess && cudaEventElapsedTime(&t, p.a, p.b) == cudaSuccess) {
+        ms[p.kind] += t;
+        launches[p.kind] += 1;
+      }
+      pool.push_back(p.a); pool.push_back(p.b);
+    }
+    pending.clear();
+  }
+  void reset() {
+    collect();
+    std::fill(launches.begin(), launches.end(), 0);
+    std::fill(ms.begin(), ms.end(), 0.0);
+  }
+  void destroy() {
+    collect();
+    for (auto e : pool) cudaEventDestroy(e);
+    pool.clear();
+  }
+};
+
+thread_local std::string g_init_error;
+
+}  // namespace
+
+struct gcpsl_ctx {
+  gcpsl_model_desc desc{};
+  ArchSpec a{};
+  int K = 0, C = 0, B = 0, F = 0;
+  uint64_t seed = 0;
+  bool bf = false;
+  size_t esz = 4;
+  cudaStream_t own_stream = nullptr, stream = nullptr;
+
+  int64_t n = 0;
+  float* d_images = nullptr;       // device copy, or device view of h_images
+  float* h_images = nullptr;       // pinned mapped host copy (data_on_host)
+  int32_t* d_labels = nullptr;
+  int32_t* d_owner = nullptr;
+
+  std::vector<int64_t> h_off;      // [C+1] offsets of the clusters' id lists
+  std::vector<int32_t> h_rounds;   // r_n = n_c / B
+  std::vector<float> h_q;          // fusion weights
+  int64_t max_nc = 0;
+  int64_t* d_off = nullptr;
+  int32_t* d_rounds = nullptr;
+  int32_t* d_ids = nullptr;
+  int32_t* d_perm = nullptr;
+  uint64_t* d_keys = nullptr;
+  float* d_q = nullptr;
+
+  int64_t P = 0;
+  float* d_theta = nullptr;        // [C][P] fp32 master, kernel layout
+  float* d_mom = nullptr;
+  float* d_grad = nullptr;
+  bf16* d_shadow = nullptr;        // [C][P] bf16 operand copy (bf16 mode)
+
+  void* d_x0 = nullptr;
+  void* d_act[5] = {};             // d_act[i+1] = output of conv i
+  void* d_dact[5] = {};
+  uint8_t* d_code[4] = {};
+  void* d_g = nullptr;
+  float* d_logits = nullptr;
+  float* d_dlogits = nullptr;
+  int32_t* d_y = nullptr;
+  int32_t* d_idx = nullptr;
+  int32_t* d_counts = nullptr;
+  int32_t* d_active = nullptr;
+  float* d_loss = nullptr;
+  int64_t* d_t = nullptr;
+  float* h_loss = nullptr;         // pinned staging
+  int32_t* h_active = nullptr;
+
+  int64_t t = 0;
+  gcpsl_status sticky = GCPSL_OK;
+  std::string err;
+  std::vector<void*> allocs;
+  bool timing = false;
+  KernelTimer timer;
+};
+
+namespace {
+
+gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  if (c) {
+    c->err = buf;
+    if (st == GCPSL_E_CUDA || st == GCPSL_E_TIMEOUT) c->sticky = st;
+  } else {
+    g_init_error = buf;
+  }
+  return st;
+}
+
+#define CK(call)                                                                           \
+  do {                                                                                     \
+    cudaError_t _e = (call);                                                               \
+    if (_e != cudaSuccess)                                                                 \
+      return fail(c, _e == cudaErrorMemoryAllocation ? GCPSL_E_NOMEM : GCPSL_E_CUDA,       \
+                  "%s failed: %s (%s:%d)", #call, cudaGetErrorString(_e), __FILE__, __LINE__); \
+  } while (0)
+
+// launch through the timer when enabled
+#define LAUNCH(name, call)                                                                 \
+  do {                                                                                     \
+    if (c->timing) c->timer.begin(name, c->stream);                                        \
+    cudaError_t _e = (call);                                                               \
+    if (c->timing) c->timer.end(c->stream);                                                \
+    if (_e != cudaSuccess)                                                                 \
+      return fail(c, GCPSL_E_CUDA, "kernel %s: %s", name, cudaGetErrorString(_e));        \
+  } while (0)
+
+template <typename P>
+gcpsl_status dalloc(gcpsl_ctx* c, P** p, size_t bytes) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
+  if (e != cudaSuccess)
+    return fail(c, GCPSL_E_NOMEM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
+  c->allocs.push_back(q);
+  *p = (P*)q;
+  return GCPSL_OK;
+}
+#define DALLOC(p, bytes)                                   \
+  do {                                                     \
+    gcpsl_status _s = dalloc(c, &(p), (size_t)(bytes));    \
+    if (_s != GCPSL_OK) return _s;                         \
+  } while (0)
+
+// canonical (PyTorch) <-> kernel layout of one replica's parameters.
+// conv weight: OIHW <-> [co][kh][kw][ci]; linear weight: input index
+// ch*HoWo + h*Wo + w <-> (h*Wo + w)*ch + ch_idx.
+void to_kernel_layout(const ArchSpec& a, const float* can, float* ker) {
+  std::memcpy(ker, can, sizeof(float) * (size_t)a.p_total);
+  for (int i = 0; i < a.L(); ++i) {
+    const ConvSpec& s = a.conv[i];
+    const float* src = can + a.off_w[i];
+    float* dst = ker + a.off_w[i];
+    for (int co = 0; co < s.cout; ++co)
+      for (int ci = 0; ci < s.cin; ++ci)
+        for (int t = 0; t < 9; ++t)
+          dst[((int64_t)co * 9 + t) * s.cin + ci] = src[((int64_t)co * s.cin + ci) * 9 + t];
+  }
+  const int l = a.L() - 1, ch = a.conv[l].cout, hw = a.out_h(l) * a.out_w(l);
+  for (int j = 0; j < a.fc_out; ++j)
+    for (int cc = 0; cc < ch; ++cc)
+      for (int p = 0; p < hw; ++p)
+        ker[a.off_fcw + (int64_t)j * a.fc_in + (int64_t)p * ch + cc] =
+            can[a.off_fcw + (int64_t)j * a.fc_in + (int64_t)cc * hw + p];
+}
+
+void to_canonical_layout(const ArchSpec& a, const float* ker, float* can) {
+  std::memcpy(can, ker, sizeof(float) * (size_t)a.p_total);
+  for (int i = 0; i < a.L(); ++i) {
+    const ConvSpec& s = a.conv[i];
+    const float* src = ker + a.off_w[i];
+    float* dst = can + a.off_w[i];
+    for (int co = 0; co < s.cout; ++co)
+      for (int ci = 0; ci < s.cin; ++ci)
+        for (int t = 0; t < 9; ++t)
+          dst[((int64_t)co * s.cin + ci) * 9 + t] = src[((int64_t)co * 9 + t) * s.cin + ci];
+  }
+  const int l = a.L() - 1, ch = a.conv[l].cout, hw = a.out_h(l) * a.out_w(l);
+  for (int j = 0; j < a.fc_out; ++j)
+    for (int cc = 0; cc < ch; ++cc)
+      for (int p = 0; p < hw; ++p)
+        can[a.off_fcw + (int64_t)j * a.fc_in + (int64_t)cc * hw + p] =
+            ker[a.off_fcw + (int64_t)j * a.fc_in + (int64_t)p * ch + cc];
+}
+
+// U(-1/sqrt(fan_in), 1/sqrt(fan_in)) from Philox(counter = (p, 0, 0, 0x5eed))
+void seeded_init(const ArchSpec& a, uint64_t seed, float* can) {
+  auto fill = [&](int64_t off, int64_t cnt, int64_t fan_in) {
+    const float bound = 1.0f / std::sqrt((float)fan_in);
+    for (int64_t p = off; p < off + cnt; ++p) {
+      uint32_t ctr[4] = {(uint32_t)p, (uint32_t)(p >> 32), 0u, 0x5eedu};
+      philox4x32_10(ctr, (uint32_t)seed, (uint32_t)(seed >> 32));
+      const float u = (float)(ctr[0] >> 8) * (1.0f / 16777216.0f);
+      can[p] = (2.0f * u - 1.0f) * bound;
+    }
+  };
+  for (int i = 0; i < a.L(); ++i) {
+    const int64_t fan = (int64_t)a.conv[i].cin * 9;
+    fill(a.off_w[i], (int64_t)a.conv[i].cout * fan, fan);
+    fill(a.off_b[i], a.conv[i].cout, fan);
+  }
+  fill(a.off_fcw, (int64_t)a.fc_out * a.fc_in, a.fc_in);
+  fill(a.off_fcb, a.fc_out, a.fc_in);
+}
+
+gcpsl_status check_usable(gcpsl_ctx* c) {
+  if (!c) return GCPSL_E_INVAL;
+  if (c->sticky != GCPSL_OK) return GCPSL_E_STATE;
+  return GCPSL_OK;
+}
+
+int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
+  if (i == 0) return (int64_t)c->C * c->B * 1024 * 3;
+  const int l = i - 1;
+  return (int64_t)c->C * c->B * c->a.out_h(l) * c->a.out_w(l) * c->a.conv[l].cout;
+}
+
+// ---------------------------------------------------------------------------
+// One local round of every cluster
+// ---------------------------------------------------------------------------
+template <typename T>
+gcpsl_status enqueue_round(gcpsl_ctx* c) {
+  cudaStream_t s = c->stream;
+  const ArchSpec& a = c->a;
+  const int C = c->C, B = c->B;
+  const int64_t P = c->P;
+  const T* wts = c->bf ? (const T*)(const void*)c->d_shadow : (const T*)(const void*)c->d_theta;
+  T* act[5];
+  T* dact[5];
+  for (int i = 0; i <= a.L(); ++i) { act[i] = (T*)c->d_act[i]; dact[i] = (T*)c->d_dact[i]; }
+  T* g = (T*)c->d_g;
+
+  // GPSL sampling (Eq. 1) and the gather of the sampled images
+  LAUNCH("epoch_keys", launch_epoch_keys(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
+                                         c->desc.cluster_id_base, c->seed, c->d_keys, C,
+                                         c->max_nc));
+  LAUNCH("epoch_rank", launch_epoch_rank(s, c->d_ids, c->d_off, c->d_rounds, c->d_t, c->d_keys,
+                                         c->d_perm, C, c->max_nc));
+  LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_t, c->d_owner,
+                                 c->d_labels, c->K, B, C, c->d_idx, c->d_counts, c->d_active,
+                                 c->d_y));
+  LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, act[0]));
+
+  // client segment to the cut, then the server segment
+  for (int i = 0; i < a.L(); ++i)
+    LAUNCH("conv_fwd", launch_conv_fwd_simt<T>(s, act[i], wts + a.off_w[i], P,
+                                               c->d_theta + a.off_b[i], P, act[i + 1],
+                                               c->d_code[i], C, B, a.conv[i]));
+  LAUNCH("fc_fwd", launch_fc_fwd<T>(s, act[a.L()], wts + a.off_fcw, P, c->d_theta + a.off_fcb, P,
+                                    c->d_logits, C, B, a.fc_in, a.fc_out));
+  LAUNCH("softmax_ce", launch_softmax_ce(s, c->d_logits, c->d_y, c->d_loss, c->d_dlogits, C, B,
+                                         a.fc_out, c->desc.label_smoothing));
+  LAUNCH("fc_bwd", launch_fc_bwd<T>(s, c->d_dlogits, act[a.L()], wts + a.off_fcw, P,
+                                    c->d_grad + a.off_fcw, c->d_grad + a.off_fcb, P, dact[a.L()],
+                                    C, B, a.fc_in, a.fc_out));
+  // backward to the cut gradient (dact[ncl]) and through the client segment
+  for (int i = a.L() - 1; i >= 0; --i) {
+    LAUNCH("relu_pool_bwd", launch_relu_pool_bwd<T>(s, dact[i + 1], c->d_code[i], act[i + 1], g,
+                                                    C, B, a.conv[i]));
+    LAUNCH("conv_wgrad", launch_conv_wgrad_simt<T>(s, act[i], g, c->d_grad + a.off_w[i], P, C, B,
+                                                   a.conv[i]));
+    LAUNCH("bias_grad", launch_bias_grad<T>(s, g, c->d_grad + a.off_b[i], P, C, B, a.conv[i]));
+    if (i > 0)
+      LAUNCH("conv_dgrad", launch_conv_dgrad_simt<T>(s, g, wts + a.off_w[i], P, dact[i], C, B,
+                                                     a.conv[i]));
+  }
+  LAUNCH("sgd", launch_sgd(s, c->d_theta, c->d_mom, c->d_grad, c->d_shadow, (int64_t)C * P,
+                           c->desc.lr, c->desc.momentum, c->desc.weight_decay,
+                           c->desc.nesterov, c->d_t));
+  return GCPSL_OK;
+}
+
+gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
+  if (c->C == 1) return GCPSL_OK;                 // q_1 = 1: the identity
+  LAUNCH("fuse", launch_fuse(c->stream, c->d_theta, c->d_shadow, c->d_q, c->C, c->P));
+  return GCPSL_OK;
+}
+
+void free_all(gcpsl_ctx* c) {
+  if (c->stream) cudaStreamSynchronize(c->stream);
+  c->timer.destroy();
+  for (void* p : c->allocs) cudaFree(p);
+  c->allocs.clear();
+  if (c->h_images) cudaFreeHost(c->h_images);
+  if (c->h_loss) cudaFreeHost(c->h_loss);
+  if (c->h_active) cudaFreeHost(c->h_active);
+  if (c->own_stream) cudaStreamDestroy(c->own_stream);
+}
+
+gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
+                       const int32_t* assignment, int B, int F, uint64_t seed,
+                       const gcpsl_dataset* data, const float* init_params) {
+  c->desc = *desc;
+  c->K = K; c->C = C; c->B = B; c->F = F; c->seed = seed;
+  c->bf = desc->operand_dtype == GCPSL_BF16;
+  c->esz = c->bf ? 2 : 4;
+  const ArchSpec& a = c->a;
+  c->P = a.p_total;
+  c->n = data->n;
+
+  // clusters: ascending example ids per cluster, r_n, q_n (Eq. 5)
+  std::vector<int64_t> nc(C, 0);
+  for (int64_t i = 0; i < data->n; ++i) {
+    const int k = assignment[data->owner[i]];
+    if (k >= 0) nc[k]++;
+  }
+  int64_t total = 0;
+  for (int k = 0; k < C; ++k) {
+    if (nc[k] < B)
+      return fail(nullptr, GCPSL_E_INVAL, "cluster %d holds %lld examples, fewer than B=%d", k,
+                  (long long)nc[k], B);
+    total += nc[k];
+    c->max_nc = std::max(c->max_nc, nc[k]);
+  }
+  c->h_off.assign(C + 1, 0);
+  for (int k = 0; k < C; ++k) c->h_off[k + 1] = c->h_off[k] + nc[k];
+  std::vector<int32_t> ids(total);
+  std::vector<int64_t> fill(c->h_off.begin(), c->h_off.end() - 1);
+  for (int64_t i = 0; i < data->n; ++i) {
+    const int k = assignment[data->owner[i]];
+    if (k >= 0) ids[fill[k]++] = (int32_t)i;
+  }
+  c->h_rounds.resize(C);
+  c->h_q.resize(C);
+  for (int k = 0; k < C; ++k) {
+    c->h_rounds[k] = (int32_t)(nc[k] / B);
+    c->h_q[k] = (float)((double)nc[k] / (double)total);
+  }
+
+  CK(cudaStreamCreateWithFlags(&c->own_stream, cudaStreamNonBlocking));
+  c->stream = c->own_stream;
+
+  // dataset
+  const size_t img_bytes = sizeof(float) * (size_t)data->n * 3072;
+  if (desc->data_on_host) {
+    CK(cudaHostAlloc((void**)&c->h_images, img_bytes, cudaHostAllocMapped | cudaHostAllocPortable));
+    std::memcpy(c->h_images, data->images, img_bytes);
+    CK(cudaHostGetDevicePointer((void**)&c->d_images, c->h_images, 0));
+  } else {
+    DALLOC(c->d_images, img_bytes);
+    CK(cudaMemcpy(c->d_images, data->images, img_bytes, cudaMemcpyHostToDevice));
+  }
+  DALLOC(c->d_labels, sizeof(int32_t) * data->n);
+  DALLOC(c->d_owner, sizeof(int32_t) * data->n);
+  CK(cudaMemcpy(c->d_labels, data->labels, sizeof(int32_t) * data->n, cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(c->d_owner, data->owner, sizeof(int32_t) * data->n, cudaMemcpyHostToDevice));
+  DALLOC(c->d_off, sizeof(int64_t) * (C + 1));
+  DALLOC(c->d_rounds, sizeof(int32_t) * C);
+  DALLOC(c->d_q, sizeof(float) * C);
+  DALLOC(c->d_ids, sizeof(int32_t) * total);
+  DALLOC(c->d_perm, sizeof(int32_t) * total);
+  DALLOC(c->d_keys, sizeof(uint64_t) * total);
+  CK(cudaMemcpy(c->d_off, c->h_off.data(), sizeof(int64_t) * (C + 1), cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(c->d_rounds, c->h_rounds.data(), sizeof(int32_t) * C, cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(c->d_q, c->h_q.data(), sizeof(float) * C, cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(c->d_ids, ids.data(), sizeof(int32_t) * total, cudaMemcpyHostToDevice));
+
+  // parameters: C identical replicas
+  std::vector<float> can(c->P), ker(c->P);
+  if (init_params) std::memcpy(can.data(), init_params, sizeof(float) * c->P);
+  else seeded_init(a, seed, can.data());
+  to_kernel_layout(a, can.data(), ker.data());
+  const size_t pb = sizeof(float) * (size_t)(C * c->P);
+  DALLOC(c->d_theta, pb);
+  DALLOC(c->d_mom, pb);
+  DALLOC(c->d_grad, pb);
+  CK(cudaMemset(c->d_mom, 0, pb));
+  CK(cudaMemset(c->d_grad, 0, pb));
+  for (int k = 0; k < C; ++k)
+    CK(cudaMemcpy(c->d_theta + (int64_t)k * c->P, ker.data(), sizeof(float) * c->P,
+                  cudaMemcpyHostToDevice));
+  if (c->bf) {
+    DALLOC(c->d_shadow, sizeof(bf16) * (size_t)(C * c->P));
+    std::vector<bf16> sh(c->P);
+    for (int64_t p = 0; p < c->P; ++p) sh[p] = __float2bfloat16_rn(ker[p]);
+    for (int k = 0; k < C; ++k)
+      CK(cudaMemcpy(c->d_shadow + (int64_t)k * c->P, sh.data(), sizeof(bf16) * c->P,
+                    cudaMemcpyHostToDevice));
+  }
+
+  // activations of one round
+  int64_t gmax = 0;
+  for (int i = 0; i <= a.L(); ++i) {
+    DALLOC(c->d_act[i], c->esz * act_elems(c, i));
+    DALLOC(c->d_dact[i], c->esz * act_elems(c, i));
+  }
+  for (int i = 0; i < a.L(); ++i) {
+    if (a.conv[i].pool) DALLOC(c->d_code[i], act_elems(c, i + 1));
+    gmax = std::max(gmax, (int64_t)C * B * a.conv[i].h * a.conv[i].w * a.conv[i].cout);
+  }
+  DALLOC(c->d_g, c->esz * gmax);
+  DALLOC(c->d_logits, sizeof(float) * C * B * a.fc_out);
+  DALLOC(c->d_dlogits, sizeof(float) * C * B * a.fc_out);
+  DALLOC(c->d_y, sizeof(int32_t) * C * B);
+  DALLOC(c->d_idx, sizeof(int32_t) * C * B);
+  DALLOC(c->d_counts, sizeof(int32_t) * (size_t)C * K);
+  DALLOC(c->d_active, sizeof(int32_t) * C);
+  DALLOC(c->d_loss, sizeof(float) * C);
+  DALLOC(c->d_t, sizeof(int64_t));
+  CK(cudaMemset(c->d_t, 0, sizeof(int64_t)));
+  CK(cudaMemset(c->d_idx, 0, sizeof(int32_t) * C * B));
+  CK(cudaMemset(c->d_counts, 0, sizeof(int32_t) * (size_t)C * K));
+  CK(cudaHostAlloc((void**)&c->h_loss, sizeof(float) * C, cudaHostAllocDefault));
+  CK(cudaHostAlloc((void**)&c->h_active, sizeof(int32_t) * C, cudaHostAllocDefault));
+  CK(cudaDeviceSynchronize());
+  return GCPSL_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+extern "C" {
+
+int64_t gcpsl_num_params(int arch, int segment) {
+  ArchSpec a;
+  if (!make_arch(arch, &a)) return -1;
+  if (segment == GCPSL_CLIENT) return a.p_client;
+  if (segment == GCPSL_SERVER) return a.p_total - a.p_client;
+  return -1;
+}
+
+gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_t* assignment,
+                        int B, int F, uint64_t seed, const gcpsl_dataset* data,
+                        const float* init_params, gcpsl_ctx** out) {
+  gcpsl_ctx* c = nullptr;
+  if (!out) return fail(nullptr, GCPSL_E_INVAL, "out is NULL");
+  *out = nullptr;
+  if (!desc || !assignment || !data || !data->images || !data->labels || !data->owner)
+    return fail(nullptr, GCPSL_E_INVAL, "NULL argument");
+  if (K <= 0 || C <= 0 || B <= 0 || B > 1024 || F < 0 || data->n <= 0 || data->n > INT32_MAX)
+    return fail(nullptr, GCPSL_E_INVAL, "bad size (K=%d C=%d B=%d F=%d n=%lld)", K, C, B, F,
+                (long long)data->n);
+  if (data->num_classes != 10)
+    return fail(nullptr, GCPSL_E_INVAL, "num_classes must be 10");
+  if (desc->operand_dtype != GCPSL_F32 && desc->operand_dtype != GCPSL_BF16)
+    return fail(nullptr, GCPSL_E_INVAL, "unknown operand_dtype %d", desc->operand_dtype);
+  if (!(desc->lr >= 0.f) || !(desc->label_smoothing >= 0.f && desc->label_smoothing < 1.f))
+    return fail(nullptr, GCPSL_E_INVAL, "bad lr or label_smoothing");
+  ArchSpec a;
+  if (!make_arch(desc->arch, &a))
+    return fail(nullptr, GCPSL_E_UNSUPPORTED, "architecture %d is not built", desc->arch);
+  for (int k = 0; k < K; ++k)
+    if (assignment[k] < -1 || assignment[k] >= C)
+      return fail(nullptr, GCPSL_E_INVAL, "assignment[%d]=%d outside [-1, %d)", k, assignment[k], C);
+  for (int64_t i = 0; i < data->n; ++i) {
+    if (data->owner[i] < 0 || data->owner[i] >= K)
+      return fail(nullptr, GCPSL_E_INVAL, "owner[%lld]=%d outside [0, %d)", (long long)i,
+                  data->owner[i], K);
+    if (data->labels[i] < 0 || data->labels[i] >= data->num_classes)
+      return fail(nullptr, GCPSL_E_INVAL, "label[%lld]=%d out of range", (long long)i,
+                  data->labels[i]);
+  }
+  c = new (std::nothrow) gcpsl_ctx();
+  if (!c) return fail(nullptr, GCPSL_E_NOMEM, "host allocation failed");
+  c->a = a;
+  gcpsl_status st = init_impl(c, desc, K, C, assignment, B, F, seed, data, init_params);
+  if (st != GCPSL_OK) {
+    if (!c->err.empty()) g_init_error = c->err;
+    free_all(c);
+    delete c;
+    return st;
+  }
+  *out = c;
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_step(gcpsl_ctx* c, gcpsl_step_stats* stats) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  st = c->bf ? enqueue_round<bf16>(c) : enqueue_round<float>(c);
+  if (st != GCPSL_OK) return st;
+  c->t++;
+  if (c->F > 0 && c->t % c->F == 0) {
+    st = enqueue_fuse(c);
+    if (st != GCPSL_OK) return st;
+  }
+  if (stats && (stats->loss || stats->active)) {
+    CK(cudaMemcpyAsync(c->h_loss, c->d_loss, sizeof(float) * c->C, cudaMemcpyDeviceToHost,
+                       c->stream));
+    CK(cudaMemcpyAsync(c->h_active, c->d_active, sizeof(int32_t) * c->C, cudaMemcpyDeviceToHost,
+                       c->stream));
+    CK(cudaStreamSynchronize(c->stream));
+    if (stats->loss) std::memcpy(stats->loss, c->h_loss, sizeof(float) * c->C);
+    if (stats->active) std::memcpy(stats->active, c->h_active, sizeof(int32_t) * c->C);
+  }
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_fuse(gcpsl_ctx* c) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  return enqueue_fuse(c);
+}
+
+gcpsl_status gcpsl_get_params(gcpsl_ctx* c, int cluster, int segment, float* dst, size_t len,
+                              size_t* needed) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (cluster < 0 || cluster >= c->C || (segment != GCPSL_CLIENT && segment != GCPSL_SERVER))
+    return fail(c, GCPSL_E_INVAL, "bad cluster %d or segment %d", cluster, segment);
+  const int64_t lo = segment == GCPSL_CLIENT ? 0 : c->a.p_client;
+  const int64_t hi = segment == GCPSL_CLIENT ? c->a.p_client : c->a.p_total;
+  if (needed) *needed = (size_t)(hi - lo);
+  if (!dst) return GCPSL_OK;
+  if (len < (size_t)(hi - lo)) return fail(c, GCPSL_E_INVAL, "dst too small");
+  std::vector<float> ker(c->P), can(c->P);
+  CK(cudaStreamSynchronize(c->stream));
+  CK(cudaMemcpy(ker.data(), c->d_theta + (int64_t)cluster * c->P, sizeof(float) * c->P,
+                cudaMemcpyDeviceToHost));
+  to_canonical_layout(c->a, ker.data(), can.data());
+  std::memcpy(dst, can.data() + lo, sizeof(float) * (size_t)(hi - lo));
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_set_params(gcpsl_ctx* c, int cluster, const float* src, size_t len) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (cluster < 0 || cluster >= c->C || !src || len != (size_t)c->P)
+    return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
+  std::vector<float> ker(c->P);
+  to_kernel_layout(c->a, src, ker.data());
+  CK(cudaStreamSynchronize(c->stream));
+  CK(cudaMemcpy(c->d_theta + (int64_t)cluster * c->P, ker.data(), sizeof(float) * c->P,
+                cudaMemcpyHostToDevice));
+  if (c->bf) {
+    std::vector<bf16> sh(c->P);
+    for (int64_t p = 0; p < c->P; ++p) sh[p] = __float2bfloat16_rn(ker[p]);
+    CK(cudaMemcpy(c->d_shadow + (int64_t)cluster * c->P, sh.data(), sizeof(bf16) * c->P,
+                  cudaMemcpyHostToDevice));
+  }
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_get_momentum(gcpsl_ctx* c, int cluster, float* dst, size_t len) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (cluster < 0 || cluster >= c->C || !dst || len != (size_t)c->P)
+    return fail(c, GCPSL_E_INVAL, "bad cluster, dst or len");
+  std::vector<float> ker(c->P);
+  CK(cudaStreamSynchronize(c->stream));
+  CK(cudaMemcpy(ker.data(), c->d_mom + (int64_t)cluster * c->P, sizeof(float) * c->P,
+                cudaMemcpyDeviceToHost));
+  to_canonical_layout(c->a, ker.data(), dst);
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_set_momentum(gcpsl_ctx* c, int cluster, const float* src, size_t len) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (cluster < 0 || cluster >= c->C || !src || len != (size_t)c->P)
+    return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
+  std::vector<float> ker(c->P);
+  to_kernel_layout(c->a, src, ker.data());
+  CK(cudaStreamSynchronize(c->stream));
+  CK(cudaMemcpy(c->d_mom + (int64_t)cluster * c->P, ker.data(), sizeof(float) * c->P,
+                cudaMemcpyHostToDevice));
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_get_pool_codes(gcpsl_ctx* c, int layer, uint8_t* dst, size_t len) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (layer < 0 || layer >= c->a.L() || !c->a.conv[layer].pool || !dst)
+    return fail(c, GCPSL_E_INVAL, "layer %d has no pooling or dst is NULL", layer);
+  const int64_t n = act_elems(c, layer + 1);
+  if (len < (size_t)n) return fail(c, GCPSL_E_INVAL, "dst too small");
+  std::vector<uint8_t> raw(n);
+  CK(cudaStreamSynchronize(c->stream));
+  CK(cudaMemcpy(raw.data(), c->d_code[layer], n, cudaMemcpyDeviceToHost));
+  const int ch = c->a.conv[layer].cout, hw = c->a.out_h(layer) * c->a.out_w(layer);
+  for (int64_t cb = 0; cb < (int64_t)c->C * c->B; ++cb)
+    for (int p = 0; p < hw; ++p)
+      for (int k = 0; k < ch; ++k) dst[(cb * ch + k) * hw + p] = raw[(cb * hw + p) * ch + k];
+  return GCPSL_OK;
+}
+
+size_t gcpsl_cut_elems(const gcpsl_ctx* c) {
+  if (!c) return 0;
+  return (size_t)act_elems(c, c->a.ncl);
+}
+
+gcpsl_status gcpsl_get_cut(gcpsl_ctx* c, int which, float* dst, size_t len) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  const int64_t n = act_elems(c, c->a.ncl);
+  if (!dst || len < (size_t)n || (which != GCPSL_CUT_ACT && which != GCPSL_CUT_GRAD))
+    return fail(c, GCPSL_E_INVAL, "bad dst, len or which");
+  const void* src = which == GCPSL_CUT_ACT ? c->d_act[c->a.ncl] : c->d_dact[c->a.ncl];
+  std::vector<unsigned char> raw((size_t)n * c->esz);
+  CK(cudaStreamSynchronize(c->stream));
+  CK(cudaMemcpy(raw.data(), src, raw.size(), cudaMemcpyDeviceToHost));
+  const int l = c->a.ncl - 1;
+  const int ch = c->a.conv[l].cout, hw = c->a.out_h(l) * c->a.out_w(l);
+  for (int64_t cb = 0; cb < (int64_t)c->C * c->B; ++cb)
+    for (int p = 0; p < hw; ++p)
+      for (int k = 0; k < ch; ++k) {
+        const int64_t si = (cb * hw + p) * ch + k;
+        float v;
+        if (c->bf) {
+          uint16_t h;
+          std::memcpy(&h, raw.data() + 2 * si, 2);
+          uint32_t u = (uint32_t)h << 16;
+          std::memcpy(&v, &u, 4);
+        } else {
+          std::memcpy(&v, raw.data() + 4 * si, 4);
+        }
+        dst[(cb * ch + k) * hw + p] = v;
+      }
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_get_sample(gcpsl_ctx* c, int32_t* idx, int32_t* counts) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  CK(cudaStreamSynchronize(c->stream));
+  if (idx) CK(cudaMemcpy(idx, c->d_idx, sizeof(int32_t) * c->C * c->B, cudaMemcpyDeviceToHost));
+  if (counts)
+    CK(cudaMemcpy(counts, c->d_counts, sizeof(int32_t) * (size_t)c->C * c->K,
+                  cudaMemcpyDeviceToHost));
+  return GCPSL_OK;
+}
+
+int64_t gcpsl_rounds(const gcpsl_ctx* c) { return c ? c->t : -1; }
+
+gcpsl_status gcpsl_set_stream(gcpsl_ctx* c, void* stream) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  CK(cudaStreamSynchronize(c->stream));
+  c->stream = stream ? (cudaStream_t)stream : c->own_stream;
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_set_timing(gcpsl_ctx* c, int enable) {
+  if (!c) return GCPSL_E_INVAL;
+  c->timing = enable != 0;
+  return GCPSL_OK;
+}
+
+int gcpsl_kernel_times(gcpsl_ctx* c, const char** names, int64_t* launches, double* ms, int cap) {
+  if (!c) return -1;
+  cudaStreamSynchronize(c->stream);
+  c->timer.collect();
+  const int n = (int)c->timer.names.size();
+  for (int i = 0; i < n && i < cap; ++i) {
+    if (names) names[i] = c->timer.names[i];
+    if (launches) launches[i] = c->timer.launches[i];
+    if (ms) ms[i] = c->timer.ms[i];
+  }
+  return n;
+}
+
+void gcpsl_reset_kernel_times(gcpsl_ctx* c) {
+  if (!c) return;
+  cudaStreamSynchronize(c->stream);
+  c->timer.reset();
+}
+
+const char* gcpsl_last_error(const gcpsl_ctx* c) {
+  return c ? c->err.c_str() : g_init_error.c_str();
+}
+
+void gcpsl_destroy(gcpsl_ctx* c) {
+  if (!c) return;
+  free_all(c);
+  delete c;
+}
+
+}  // extern "C"

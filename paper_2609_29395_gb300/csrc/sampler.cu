@@ -1,0 +1,154 @@
+// GPSL global sampling inside each cluster (Eq. 1; epoch rule of
+// Section III-A) and the gather of the sampled images.
+//
+// Epoch permutation of cluster n: every example id j of the cluster gets the
+// 64-bit key (o0 << 32 | o1) of Philox4x32-10(counter = (j, epoch, n', 0),
+// key = seed), n' = cluster_base + n, and the epoch order is the ids sorted by
+// (key, j).  Round s of the epoch takes positions [sB, sB + B) and orders them
+// by (owner, j).  The sort is a rank count: rank(i) = #{m : (k_m, j_m) <
+// (k_i, j_i)}, which is exact, deterministic and needs no scratch; it runs
+// once per epoch per cluster (every n_c / B rounds).
+//
+// The round counter t lives in device memory so that a captured step can be
+// replayed: cluster n is in epoch t / r_n, round t % r_n.
+#include "common.cuh"
+
+namespace gcpsl {
+
+namespace {
+
+constexpr int kRankThreads = 256;
+
+__global__ void k_epoch_keys(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
+                             const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
+                             int cluster_base, uint32_t s0, uint32_t s1,
+                             uint64_t* __restrict__ keys) {
+  const int c = blockIdx.y;
+  const int64_t t = *d_t;
+  const int64_t r = rounds[c];
+  if (t % r != 0) return;                       // not an epoch boundary
+  const uint32_t epoch = (uint32_t)(t / r);
+  const int64_t base = off[c], n = off[c + 1] - base;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  uint32_t ctr[4] = {(uint32_t)ids[base + i], epoch, (uint32_t)(cluster_base + c), 0u};
+  philox4x32_10(ctr, s0, s1);
+  keys[base + i] = ((uint64_t)ctr[0] << 32) | ctr[1];
+}
+
+__device__ __forceinline__ bool key_less(uint64_t ka, int32_t ja, uint64_t kb, int32_t jb) {
+  return ka < kb || (ka == kb && ja < jb);
+}
+
+__global__ void __launch_bounds__(kRankThreads)
+k_epoch_rank(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
+             const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
+             const uint64_t* __restrict__ keys, int32_t* __restrict__ perm) {
+  __shared__ uint64_t sk[kRankThreads];
+  __shared__ int32_t sj[kRankThreads];
+  const int c = blockIdx.y;
+  const int64_t t = *d_t;
+  if (t % rounds[c] != 0) return;
+  const int64_t base = off[c], n = off[c + 1] - base;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if ((int64_t)blockIdx.x * blockDim.x >= n) return;      // whole block idle
+  const bool mine = i < n;
+  const uint64_t ki = mine ? keys[base + i] : 0;
+  const int32_t ji = mine ? ids[base + i] : 0;
+  int64_t rank = 0;
+  for (int64_t t0 = 0; t0 < n; t0 += kRankThreads) {
+    const int64_t m = t0 + threadIdx.x;
+    if (m < n) { sk[threadIdx.x] = keys[base + m]; sj[threadIdx.x] = ids[base + m]; }
+    __syncthreads();
+    const int lim = (n - t0) < kRankThreads ? (int)(n - t0) : kRankThreads;
+    for (int q = 0; q < lim; ++q) rank += key_less(sk[q], sj[q], ki, ji);
+    __syncthreads();
+  }
+  if (mine) perm[base + rank] = ji;
+}
+
+// One block per cluster, one thread per batch slot (B <= 1024).
+__global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __restrict__ off,
+                         const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
+                         const int32_t* __restrict__ owner, const int32_t* __restrict__ labels,
+                         int K, int B, int32_t* __restrict__ idx, int32_t* __restrict__ counts,
+                         int32_t* __restrict__ active, int32_t* __restrict__ y) {
+  extern __shared__ int32_t sm[];
+  int32_t* sid = sm;          // [B] ids of the round
+  int32_t* sown = sm + B;     // [B] their owners
+  int32_t* sorted_own = sm + 2 * B;
+  const int c = blockIdx.x;
+  const int b = threadIdx.x;
+  const int64_t s = *d_t % rounds[c];
+  int32_t* cnt = counts + (int64_t)c * K;
+  for (int k = b; k < K; k += blockDim.x) cnt[k] = 0;
+  const int32_t id = perm[off[c] + s * B + b];
+  const int32_t own = owner[id];
+  sid[b] = id;
+  sown[b] = own;
+  __syncthreads();
+  int rank = 0;
+  for (int q = 0; q < B; ++q)
+    rank += (sown[q] < own) || (sown[q] == own && sid[q] < id);
+  idx[(int64_t)c * B + rank] = id;
+  y[(int64_t)c * B + rank] = labels[id];
+  sorted_own[rank] = own;
+  atomicAdd(&cnt[own], 1);
+  __syncthreads();
+  const int first = __syncthreads_count(rank == 0 || sorted_own[rank - 1] != own);
+  if (b == 0) active[c] = first;
+}
+
+// x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w]
+template <typename T>
+__global__ void k_gather(const float* __restrict__ images, const int32_t* __restrict__ idx,
+                         int CB, T* __restrict__ x0) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)CB * 1024) return;
+  const int64_t cb = i >> 10;
+  const int p = (int)(i & 1023);
+  const float* src = images + (int64_t)idx[cb] * 3072 + p;
+  T* dst = x0 + i * 3;
+  dst[0] = from_f<T>(src[0]);
+  dst[1] = from_f<T>(src[1024]);
+  dst[2] = from_f<T>(src[2048]);
+}
+
+}  // namespace
+
+cudaError_t launch_epoch_keys(cudaStream_t s, const int32_t* ids, const int64_t* off,
+                              const int32_t* rounds, const int64_t* d_t, int cluster_base,
+                              uint64_t seed, uint64_t* keys, int C, int64_t max_nc) {
+  dim3 grid((unsigned)((max_nc + 255) / 256), (unsigned)C);
+  k_epoch_keys<<<grid, 256, 0, s>>>(ids, off, rounds, d_t, cluster_base, (uint32_t)seed,
+                                    (uint32_t)(seed >> 32), keys);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_epoch_rank(cudaStream_t s, const int32_t* ids, const int64_t* off,
+                              const int32_t* rounds, const int64_t* d_t, const uint64_t* keys,
+                              int32_t* perm, int C, int64_t max_nc) {
+  dim3 grid((unsigned)((max_nc + kRankThreads - 1) / kRankThreads), (unsigned)C);
+  k_epoch_rank<<<grid, kRankThreads, 0, s>>>(ids, off, rounds, d_t, keys, perm);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* off,
+                          const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
+                          const int32_t* labels, int K, int B, int C, int32_t* idx,
+                          int32_t* counts, int32_t* active, int32_t* y) {
+  k_sample<<<C, B, 3 * B * sizeof(int32_t), s>>>(perm, off, rounds, d_t, owner, labels, K, B,
+                                                  idx, counts, active, y);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_gather(cudaStream_t s, const float* images, const int32_t* idx, int CB, T* x0) {
+  int64_t n = (int64_t)CB * 1024;
+  k_gather<T><<<(unsigned)((n + 255) / 256), 256, 0, s>>>(images, idx, CB, x0);
+  return cudaGetLastError();
+}
+template cudaError_t launch_gather<float>(cudaStream_t, const float*, const int32_t*, int, float*);
+template cudaError_t launch_gather<bf16>(cudaStream_t, const float*, const int32_t*, int, bf16*);
+
+}  // namespace gcpsl
