@@ -83,18 +83,25 @@ def work_per_round(w, esz):
     convs = spec["client"] + spec["server"]
     C, B = w.num_clusters, w.B
     P = synth.num_params(w.arch, "client") + synth.num_params(w.arch, "server")
-    fwd = dgrad = wgrad = 0
+    work = {}
+
+    def add(kind, bound, v):
+        b, old = work.get(kind, (bound, 0.0))
+        work[kind] = (bound, old + v)
+
     for i, (cin, cout, h, ww, _p) in enumerate(convs):
         f = 2.0 * C * B * h * ww * cout * 9 * cin
-        fwd += f
-        wgrad += f
+        # layers with 32k input / 64k output channels run on the tensor cores
+        tc = esz == 2 and cin >= 32 and cin % 32 == 0 and cout % 64 == 0 and ww <= 64
+        sfx = "_tc" if tc else ""
+        add("conv_fwd" + sfx, "tensor", f)
+        add("conv_wgrad" + sfx, "tensor", f)
         if i > 0:
-            dgrad += f
+            add("conv_dgrad" + sfx, "tensor", f)
     fin, fout = spec["fc"]
     fc = 2.0 * C * B * fin * fout
     return {
-        "conv_fwd": ("tensor", fwd), "conv_dgrad": ("tensor", dgrad),
-        "conv_wgrad": ("tensor", wgrad), "fc_fwd": ("tensor", fc),
+        **work, "fc_fwd": ("tensor", fc),
         "fc_bwd": ("tensor", 2 * fc),
         "sgd": ("hbm", C * P * (4 * 5 + (2 if esz == 2 else 0))),
         "fuse": ("hbm", C * P * (4 + 4 + (2 if esz == 2 else 0))),
@@ -103,7 +110,8 @@ def work_per_round(w, esz):
 
 def kernel_source_hash(kind):
     src = {"conv_fwd": "conv_simt.cu", "conv_dgrad": "conv_simt.cu", "conv_wgrad": "conv_simt.cu",
-           "sgd": "optim.cu", "fuse": "optim.cu"}.get(kind)
+           "conv_fwd_tc": "conv_tc.cu", "conv_dgrad_tc": "conv_tc.cu",
+           "conv_wgrad_tc": "conv_tc.cu", "sgd": "optim.cu", "fuse": "optim.cu"}.get(kind)
     if not src:
         return None
     p = os.path.join(ROOT, "paper_2609_29395_gb300", "csrc", src)

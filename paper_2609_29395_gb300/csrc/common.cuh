@@ -1,6 +1,7 @@
 // Internal declarations of libgcpsl.so (not part of the C ABI).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -86,12 +87,15 @@ cudaError_t launch_relu_pool_bwd(cudaStream_t s, const T* dout, const uint8_t* c
 template <typename T>
 cudaError_t launch_conv_dgrad_simt(cudaStream_t s, const T* g, const T* w, int64_t w_rs, T* dx,
                                    int C, int B, const ConvSpec& cs);
+// weight+bias gradient partials of a CUDA-core layer over `splits` pixel
+// ranges (tiles of `tr` image rows): partial[c][split][cout*9*cin + cout]
 template <typename T>
-cudaError_t launch_conv_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* dw,
-                                   int64_t dw_rs, int C, int B, const ConvSpec& cs);
+cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* partial, int C,
+                              int B, const ConvSpec& cs, int tr, int splits, int tiles_per_split);
+// bias-gradient partials over chunks of chunk_px pixels: partial[c][chunk][cout]
 template <typename T>
-cudaError_t launch_bias_grad(cudaStream_t s, const T* g, float* db, int64_t db_rs, int C, int B,
-                             const ConvSpec& cs);
+cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int C, int B,
+                                const ConvSpec& cs, int chunks, int chunk_px);
 
 // head.cu
 template <typename T>
@@ -103,6 +107,42 @@ template <typename T>
 cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const T* h, const T* w,
                           int64_t w_rs, float* dw, float* db, int64_t g_rs, T* dh, int C, int B,
                           int fin, int fout);
+
+// conv_tc.cu (tensor-core convolutions, bf16 operands)
+enum { EPI_POOL = 0, EPI_RELU = 1, EPI_STORE = 2 };
+struct ConvTcArgs {
+  int H, W, B;          // spatial size and batch per replica
+  int kch;              // channels of the activation operand (multiple of the stage width)
+  int hb, bb;           // image rows / images per 128-pixel M tile (W * hb * bb == 128)
+  int tiles_h;          // H / hb
+  int n_total;          // output channels (row length of `out`)
+  const float* bias;    // fp32 bias of replica 0 (EPI_POOL / EPI_RELU)
+  int64_t bias_rs;      // replica stride of the bias
+  bf16* out;            // NHWC output, [C][B][H'][W'][n_total]
+  uint8_t* code;        // max-pool codes, same layout as out (EPI_POOL)
+  int* err;             // error word: bounded waits that gave up
+};
+struct WgradTcArgs {
+  int H, W, B, cout, cin;
+  int hb, bb;           // image rows / images per 64-pixel K block (W * hb * bb == 64)
+  int kb_total;         // K blocks per replica
+  int kb_per_split, splits;
+  float* partial;       // [C][splits][cout][9][cin]
+  int* err;
+};
+bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                     const uint32_t* box, int swizzle_bytes);
+bool tensor_map_bf16_strided(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                             uint64_t outer_stride_bytes, const uint32_t* box, int swizzle_bytes);
+cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                           const ConvTcArgs& p, int bn, int bkc, int epi, int C);
+cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                            const WgradTcArgs& p, int bn, int C);
+// dw[c * dw_rs + i] = sum over s (in order) of partial[c][s][i], i < per
+cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
+                                int splits, int64_t per, int C);
+cudaError_t launch_flip_shadow(cudaStream_t s, const bf16* w, bf16* wt, int64_t rs, int cout,
+                               int cin, int C);
 
 // optim.cu
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,

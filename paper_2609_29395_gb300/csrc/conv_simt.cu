@@ -117,52 +117,80 @@ __global__ void k_conv_dgrad(const T* __restrict__ g, const T* __restrict__ w, i
   dx[i] = from_f<T>(acc);
 }
 
+// Weight and bias gradient partial sums over a range of image-row tiles,
+// staged in shared memory: outputs o < cout*9*cin are dW[co][tap][ci],
+// outputs cout*9*cin + co are db[co] (the bias follows the weight in the
+// parameter store, so one reduction writes both).  Block = 256 threads,
+// grid = (splits, C); partial[c][split][o].  Each thread sums its outputs
+// over the block's pixels in a fixed order.
+constexpr int kWgOut = 32;   // outputs per thread (per <= 256 * kWgOut)
+
 template <typename T>
-__global__ void k_conv_wgrad(const T* __restrict__ x, const T* __restrict__ g,
-                             float* __restrict__ dw, int64_t dw_rs, int C, int B, int cin,
-                             int cout, int H, int W) {
-  const int64_t per = (int64_t)cout * 9 * cin;
-  const int64_t total = (int64_t)C * per;
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= total) return;
-  const int c = (int)(i / per);
-  int64_t r = i % per;
-  const int ci = (int)(r % cin); r /= cin;
-  const int tap = (int)(r % 9);
-  const int co = (int)(r / 9);
-  const int kh = tap / 3, kw = tap % 3;
-  float acc = 0.f;
-  for (int b = 0; b < B; ++b) {
-    const T* gb = g + ((int64_t)c * B + b) * H * W * cout + co;
-    const T* xb = x + ((int64_t)c * B + b) * H * W * cin + ci;
-    for (int h = 0; h < H; ++h) {
-      const int ih = h + kh - 1;
-      if (ih < 0 || ih >= H) continue;
-      for (int w = 0; w < W; ++w) {
-        const int iw = w + kw - 1;
-        if (iw < 0 || iw >= W) continue;
-        acc = fmaf(to_f(gb[((int64_t)h * W + w) * cout]), to_f(xb[((int64_t)ih * W + iw) * cin]), acc);
-      }
+__global__ void __launch_bounds__(256)
+k_wgrad_partial(const T* __restrict__ x, const T* __restrict__ g, float* __restrict__ partial,
+                int B, int cin, int cout, int H, int W, int tr, int tiles_per_split) {
+  extern __shared__ float sm[];
+  const int c = blockIdx.y, split = blockIdx.x;
+  const int per_w = cout * 9 * cin, per = per_w + cout;
+  float* gs = sm;                                   // [tr*W][cout]
+  float* xs = sm + tr * W * cout;                   // [(tr+2)][(W+2)][cin]
+  float acc[kWgOut];
+#pragma unroll
+  for (int j = 0; j < kWgOut; ++j) acc[j] = 0.f;
+  const int tiles_img = H / tr, tiles = B * tiles_img;
+  const int t0 = split * tiles_per_split, t1 = min(t0 + tiles_per_split, tiles);
+  for (int tile = t0; tile < t1; ++tile) {
+    const int b = tile / tiles_img, h0 = (tile % tiles_img) * tr;
+    const T* gb = g + (((int64_t)c * B + b) * H + h0) * W * cout;
+    for (int i = threadIdx.x; i < tr * W * cout; i += blockDim.x) gs[i] = to_f(gb[i]);
+    const T* xb = x + ((int64_t)c * B + b) * H * W * cin;
+    for (int i = threadIdx.x; i < (tr + 2) * (W + 2) * cin; i += blockDim.x) {
+      const int ci = i % cin, ww = (i / cin) % (W + 2) - 1, hh = i / (cin * (W + 2)) + h0 - 1;
+      xs[i] = (hh >= 0 && hh < H && ww >= 0 && ww < W) ? to_f(xb[((int64_t)hh * W + ww) * cin + ci])
+                                                      : 0.f;
     }
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < kWgOut; ++j) {
+      const int o = threadIdx.x + j * 256;
+      if (o >= per) break;
+      float s = acc[j];
+      if (o < per_w) {
+        const int ci = o % cin, tap = (o / cin) % 9, co = o / (9 * cin);
+        const int kh = tap / 3, kw = tap % 3;
+        for (int r = 0; r < tr; ++r)
+          for (int w = 0; w < W; ++w)
+            s = fmaf(gs[(r * W + w) * cout + co], xs[((r + kh) * (W + 2) + w + kw) * cin + ci], s);
+      } else {
+        const int co = o - per_w;
+        for (int q = 0; q < tr * W; ++q) s += gs[q * cout + co];
+      }
+      acc[j] = s;
+    }
+    __syncthreads();
   }
-  dw[(int64_t)c * dw_rs + (int64_t)co * 9 * cin + tap * cin + ci] = acc;
+  float* dst = partial + ((int64_t)c * gridDim.x + split) * per;
+#pragma unroll
+  for (int j = 0; j < kWgOut; ++j) {
+    const int o = threadIdx.x + j * 256;
+    if (o < per) dst[o] = acc[j];
+  }
 }
 
-// db[c][co] = sum over (b, h, w) of g; one warp per (c, co), fixed order:
-// lane l sums pixels l, l+32, ...; then a fixed shuffle tree.
+// Bias-gradient partials: partial[c][chunk][co] = sum of g over the chunk's
+// `chunk_px` pixels (consecutive threads read consecutive channels).
 template <typename T>
-__global__ void k_bias_grad(const T* __restrict__ g, float* __restrict__ db, int64_t db_rs,
-                            int C, int B, int cout, int HW) {
-  const int warp = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-  const int lane = threadIdx.x & 31;
-  if (warp >= C * cout) return;
-  const int c = warp / cout, co = warp % cout;
-  const int64_t npix = (int64_t)B * HW;
-  const T* gc = g + (int64_t)c * npix * cout + co;
-  float s = 0.f;
-  for (int64_t p = lane; p < npix; p += 32) s += to_f(gc[p * cout]);
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if (lane == 0) db[(int64_t)c * db_rs + co] = s;
+__global__ void k_bias_partial(const T* __restrict__ g, float* __restrict__ partial, int64_t npix,
+                               int cout, int chunk_px) {
+  const int c = blockIdx.y, chunk = blockIdx.x;
+  const int64_t p0 = (int64_t)chunk * chunk_px;
+  const int64_t p1 = min(p0 + chunk_px, npix);
+  const T* gc = g + (int64_t)c * npix * cout;
+  for (int co = threadIdx.x; co < cout; co += blockDim.x) {
+    float s = 0.f;
+    for (int64_t p = p0; p < p1; ++p) s += to_f(gc[p * cout + co]);
+    partial[((int64_t)c * gridDim.x + chunk) * cout + co] = s;
+  }
 }
 
 inline unsigned blocks(int64_t n, int t) { return (unsigned)((n + t - 1) / t); }
@@ -199,20 +227,28 @@ cudaError_t launch_conv_dgrad_simt(cudaStream_t s, const T* g, const T* w, int64
 }
 
 template <typename T>
-cudaError_t launch_conv_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* dw,
-                                   int64_t dw_rs, int C, int B, const ConvSpec& cs) {
-  const int64_t n = (int64_t)C * cs.cout * 9 * cs.cin;
-  k_conv_wgrad<T><<<blocks(n, 128), 128, 0, s>>>(x, g, dw, dw_rs, C, B, cs.cin, cs.cout, cs.h,
-                                                  cs.w);
+cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* partial, int C,
+                              int B, const ConvSpec& cs, int tr, int splits, int tiles_per_split) {
+  const int smem = (tr * cs.w * cs.cout + (tr + 2) * (cs.w + 2) * cs.cin) * (int)sizeof(float);
+  if ((int64_t)cs.cout * 9 * cs.cin + cs.cout > 256 * kWgOut) return cudaErrorInvalidValue;
+  static int attr_set = 0;
+  if (smem > 48 * 1024 && attr_set < smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_wgrad_partial<T>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr_set = smem;
+  }
+  k_wgrad_partial<T><<<dim3(splits, C), 256, smem, s>>>(x, g, partial, B, cs.cin, cs.cout, cs.h,
+                                                        cs.w, tr, tiles_per_split);
   return cudaGetLastError();
 }
 
 template <typename T>
-cudaError_t launch_bias_grad(cudaStream_t s, const T* g, float* db, int64_t db_rs, int C, int B,
-                             const ConvSpec& cs) {
-  const int64_t warps = (int64_t)C * cs.cout;
-  k_bias_grad<T><<<blocks(warps * 32, 256), 256, 0, s>>>(g, db, db_rs, C, B, cs.cout,
-                                                          cs.h * cs.w);
+cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int C, int B,
+                                const ConvSpec& cs, int chunks, int chunk_px) {
+  const int64_t npix = (int64_t)B * cs.h * cs.w;
+  const int threads = cs.cout < 256 ? cs.cout : 256;
+  k_bias_partial<T><<<dim3(chunks, C), threads, 0, s>>>(g, partial, npix, cs.cout, chunk_px);
   return cudaGetLastError();
 }
 
@@ -224,10 +260,10 @@ cudaError_t launch_bias_grad(cudaStream_t s, const T* g, float* db, int64_t db_r
                                                const T*, T*, int, int, const ConvSpec&);       \
   template cudaError_t launch_conv_dgrad_simt<T>(cudaStream_t, const T*, const T*, int64_t,    \
                                                  T*, int, int, const ConvSpec&);               \
-  template cudaError_t launch_conv_wgrad_simt<T>(cudaStream_t, const T*, const T*, float*,     \
-                                                 int64_t, int, int, const ConvSpec&);          \
-  template cudaError_t launch_bias_grad<T>(cudaStream_t, const T*, float*, int64_t, int, int,  \
-                                           const ConvSpec&);
+  template cudaError_t launch_wgrad_simt<T>(cudaStream_t, const T*, const T*, float*, int, int, \
+                                            const ConvSpec&, int, int, int);                   \
+  template cudaError_t launch_bias_partial<T>(cudaStream_t, const T*, float*, int, int,        \
+                                              const ConvSpec&, int, int);
 GCPSL_INST(float)
 GCPSL_INST(bf16)
 #undef GCPSL_INST

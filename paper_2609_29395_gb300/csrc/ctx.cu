@@ -141,10 +141,29 @@ struct gcpsl_ctx {
   float* d_q = nullptr;
 
   int64_t P = 0;
-  float* d_theta = nullptr;        // [C][P] fp32 master, kernel layout
+  int64_t P_pad = 0;               // replica stride of every [C][P] array (multiple of 64)
+  float* d_theta = nullptr;        // [C][P_pad] fp32 master, kernel layout
   float* d_mom = nullptr;
   float* d_grad = nullptr;
-  bf16* d_shadow = nullptr;        // [C][P] bf16 operand copy (bf16 mode)
+  bf16* d_shadow = nullptr;        // [C][P_pad] bf16 operand copy (bf16 mode)
+  bf16* d_shadow_t = nullptr;      // conv weights as Wt[ci][8-tap][co] (data-gradient operand)
+  int* d_err = nullptr;            // device error word (bounded waits that gave up)
+
+  // tensor-core layers (bf16 mode): tile shapes and TMA descriptors
+  struct TcLayer {
+    bool on = false;
+    int hb, bb, tiles_h;           // 128-pixel M tile
+    int whb, wbb;                  // 64-pixel K block of the weight gradient
+    int bn_f, bkc_f, bn_d, bkc_d, bn_w;
+    int splits, kb_total, kb_per_split;
+    CUtensorMap fwdA, fwdB, dgrA, dgrB, wgA, wgB;
+  } tc[4];
+  float* d_partial = nullptr;      // weight-gradient split partials (tensor-core layers)
+  // CUDA-core gradient reductions: weight+bias partials of the other layers
+  // (tiles of tr image rows, tiles_per_split tiles per block) and bias
+  // partials of the tensor-core layers (chunks of chunk_px pixels)
+  struct RedLayer { int tr, splits, tiles_per_split, chunks, chunk_px; } red[4];
+  float* d_bpartial = nullptr;
 
   void* d_x0 = nullptr;
   void* d_act[5] = {};             // d_act[i+1] = output of conv i
@@ -204,6 +223,16 @@ gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...) {
     if (_e != cudaSuccess)                                                                 \
       return fail(c, GCPSL_E_CUDA, "kernel %s: %s", name, cudaGetErrorString(_e));        \
   } while (0)
+
+// synchronise the stream, then fail on a device-side timeout
+#define SYNC_CHECK(c)                                        \
+  do {                                                       \
+    CK(cudaStreamSynchronize((c)->stream));                  \
+    gcpsl_status _d = check_device_error(c);                 \
+    if (_d != GCPSL_OK) return _d;                           \
+  } while (0)
+
+gcpsl_status check_device_error(gcpsl_ctx* c);
 
 template <typename P>
 gcpsl_status dalloc(gcpsl_ctx* c, P** p, size_t bytes) {
@@ -297,12 +326,32 @@ int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
 // ---------------------------------------------------------------------------
 // One local round of every cluster
 // ---------------------------------------------------------------------------
+// the data-gradient operand Wt of every tensor-core layer, from the shadow
+gcpsl_status refresh_flipped(gcpsl_ctx* c) {
+  for (int i = 0; i < c->a.L(); ++i) {
+    if (!c->tc[i].on) continue;
+    LAUNCH("flip_shadow", launch_flip_shadow(c->stream, c->d_shadow + c->a.off_w[i],
+                                             c->d_shadow_t + c->a.off_w[i], c->P_pad,
+                                             c->a.conv[i].cout, c->a.conv[i].cin, c->C));
+  }
+  return GCPSL_OK;
+}
+
+// a device-side wait that gave up leaves a nonzero error word; the context
+// then refuses further work
+gcpsl_status check_device_error(gcpsl_ctx* c) {
+  int e = 0;
+  CK(cudaMemcpy(&e, c->d_err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (e) return fail(c, GCPSL_E_TIMEOUT, "device-side wait gave up (error word 0x%x)", e);
+  return GCPSL_OK;
+}
+
 template <typename T>
 gcpsl_status enqueue_round(gcpsl_ctx* c) {
   cudaStream_t s = c->stream;
   const ArchSpec& a = c->a;
   const int C = c->C, B = c->B;
-  const int64_t P = c->P;
+  const int64_t P = c->P_pad;
   const T* wts = c->bf ? (const T*)(const void*)c->d_shadow : (const T*)(const void*)c->d_theta;
   T* act[5];
   T* dact[5];
@@ -321,10 +370,20 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
   LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, act[0]));
 
   // client segment to the cut, then the server segment
-  for (int i = 0; i < a.L(); ++i)
-    LAUNCH("conv_fwd", launch_conv_fwd_simt<T>(s, act[i], wts + a.off_w[i], P,
-                                               c->d_theta + a.off_b[i], P, act[i + 1],
-                                               c->d_code[i], C, B, a.conv[i]));
+  for (int i = 0; i < a.L(); ++i) {
+    const auto& L = c->tc[i];
+    if (L.on) {
+      ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.hb, L.bb, L.tiles_h,
+                   a.conv[i].cout, c->d_theta + a.off_b[i], P, (bf16*)(void*)act[i + 1],
+                   c->d_code[i], c->d_err};
+      LAUNCH("conv_fwd_tc", launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f,
+                                           a.conv[i].pool ? EPI_POOL : EPI_RELU, C));
+    } else {
+      LAUNCH("conv_fwd", launch_conv_fwd_simt<T>(s, act[i], wts + a.off_w[i], P,
+                                                 c->d_theta + a.off_b[i], P, act[i + 1],
+                                                 c->d_code[i], C, B, a.conv[i]));
+    }
+  }
   LAUNCH("fc_fwd", launch_fc_fwd<T>(s, act[a.L()], wts + a.off_fcw, P, c->d_theta + a.off_fcb, P,
                                     c->d_logits, C, B, a.fc_in, a.fc_out));
   LAUNCH("softmax_ce", launch_softmax_ce(s, c->d_logits, c->d_y, c->d_loss, c->d_dlogits, C, B,
@@ -334,24 +393,114 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
                                     C, B, a.fc_in, a.fc_out));
   // backward to the cut gradient (dact[ncl]) and through the client segment
   for (int i = a.L() - 1; i >= 0; --i) {
+    const auto& L = c->tc[i];
+    const ConvSpec& cs = a.conv[i];
     LAUNCH("relu_pool_bwd", launch_relu_pool_bwd<T>(s, dact[i + 1], c->d_code[i], act[i + 1], g,
-                                                    C, B, a.conv[i]));
-    LAUNCH("conv_wgrad", launch_conv_wgrad_simt<T>(s, act[i], g, c->d_grad + a.off_w[i], P, C, B,
-                                                   a.conv[i]));
-    LAUNCH("bias_grad", launch_bias_grad<T>(s, g, c->d_grad + a.off_b[i], P, C, B, a.conv[i]));
-    if (i > 0)
+                                                    C, B, cs));
+    const auto& R = c->red[i];
+    if (L.on) {
+      WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
+                    L.splits, c->d_partial, c->d_err};
+      LAUNCH("conv_wgrad_tc", launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
+      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
+                                                 L.splits, (int64_t)cs.cout * 9 * cs.cin, C));
+      LAUNCH("bias_partial", launch_bias_partial<T>(s, g, c->d_bpartial, C, B, cs, R.chunks,
+                                                    R.chunk_px));
+      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_bpartial, c->d_grad + a.off_b[i], P,
+                                                 R.chunks, cs.cout, C));
+    } else {
+      // weights and bias together (the bias follows the weight in the store)
+      LAUNCH("conv_wgrad", launch_wgrad_simt<T>(s, act[i], g, c->d_bpartial, C, B, cs, R.tr,
+                                                R.splits, R.tiles_per_split));
+      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_bpartial, c->d_grad + a.off_w[i], P,
+                                                 R.splits,
+                                                 (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
+    }
+    if (i == 0) continue;
+    if (L.on) {
+      ConvTcArgs p{cs.h, cs.w, B, cs.cout, L.hb, L.bb, L.tiles_h, cs.cin, nullptr, 0,
+                   (bf16*)(void*)dact[i], nullptr, c->d_err};
+      LAUNCH("conv_dgrad_tc", launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d, EPI_STORE, C));
+    } else {
       LAUNCH("conv_dgrad", launch_conv_dgrad_simt<T>(s, g, wts + a.off_w[i], P, dact[i], C, B,
-                                                     a.conv[i]));
+                                                     cs));
+    }
   }
   LAUNCH("sgd", launch_sgd(s, c->d_theta, c->d_mom, c->d_grad, c->d_shadow, (int64_t)C * P,
                            c->desc.lr, c->desc.momentum, c->desc.weight_decay,
                            c->desc.nesterov, c->d_t));
-  return GCPSL_OK;
+  return refresh_flipped(c);
 }
 
 gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
   if (c->C == 1) return GCPSL_OK;                 // q_1 = 1: the identity
-  LAUNCH("fuse", launch_fuse(c->stream, c->d_theta, c->d_shadow, c->d_q, c->C, c->P));
+  LAUNCH("fuse", launch_fuse(c->stream, c->d_theta, c->d_shadow, c->d_q, c->C, c->P_pad));
+  return refresh_flipped(c);
+}
+
+// Tile shapes, split-K factors and TMA descriptors of every layer that runs on
+// the tensor cores: 3x3 layers with 32k input and 64k output channels and
+// rows of at most 64 pixels.  Layers outside that shape (the 3-channel input
+// layer) stay on the CUDA-core kernels.
+gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
+  const ArchSpec& a = c->a;
+  const int C = c->C, B = c->B;
+  int64_t partial_max = 0;
+  for (int i = 0; i < a.L(); ++i) {
+    const ConvSpec& s = a.conv[i];
+    auto& L = c->tc[i];
+    L.on = false;
+    if (s.cin < 32 || s.cin % 32 || s.cout % 64 || s.w > 64 || 64 % s.w || a.off_w[i] % 8)
+      continue;
+    L.hb = std::min(s.h, 128 / s.w);
+    L.bb = 128 / (s.w * L.hb);
+    L.whb = std::min(s.h, 64 / s.w);
+    L.wbb = 64 / (s.w * L.whb);
+    if (s.w * L.hb * L.bb != 128 || s.h % L.hb || s.w * L.whb * L.wbb != 64 || s.h % L.whb)
+      continue;
+    L.tiles_h = s.h / L.hb;
+    L.bn_f = std::min(s.cout, 256);
+    L.bkc_f = std::min(s.cin, 64);
+    L.bn_d = std::min(s.cin, 256);
+    L.bkc_d = std::min(s.cout, 64);
+    L.bn_w = std::min(s.cin, 128);
+    if (s.cout % L.bn_f || s.cin % L.bn_d || s.cin % L.bkc_f || s.cin % L.bn_w) continue;
+    const int tiles = 9 * (s.cin / L.bn_w) * ((s.cout + 127) / 128);
+    L.kb_total = ((B + L.wbb - 1) / L.wbb) * (s.h / L.whb);
+    // the split (hence the summation order) depends on the per-replica shape
+    // only, so C grouped replicas reproduce C one-replica runs bit for bit
+    int splits = (152 + tiles - 1) / tiles;
+    splits = std::max(1, std::min(splits, L.kb_total));
+    L.kb_per_split = (L.kb_total + splits - 1) / splits;
+    L.splits = (L.kb_total + L.kb_per_split - 1) / L.kb_per_split;
+    partial_max = std::max(partial_max, (int64_t)C * L.splits * s.cout * 9 * s.cin);
+
+    const uint64_t act_in[5] = {(uint64_t)s.cin, (uint64_t)s.w, (uint64_t)s.h, (uint64_t)B,
+                                (uint64_t)C};
+    const uint64_t g_dims[5] = {(uint64_t)s.cout, (uint64_t)s.w, (uint64_t)s.h, (uint64_t)B,
+                                (uint64_t)C};
+    const uint64_t wf[4] = {(uint64_t)s.cin, 9, (uint64_t)s.cout, (uint64_t)C};
+    const uint64_t wd[4] = {(uint64_t)s.cout, 9, (uint64_t)s.cin, (uint64_t)C};
+    const uint64_t rs = (uint64_t)c->P_pad * 2;
+    const uint32_t bA[5] = {(uint32_t)L.bkc_f, (uint32_t)s.w, (uint32_t)L.hb, (uint32_t)L.bb, 1};
+    const uint32_t bB[4] = {(uint32_t)L.bkc_f, 1, (uint32_t)L.bn_f, 1};
+    const uint32_t dA[5] = {(uint32_t)L.bkc_d, (uint32_t)s.w, (uint32_t)L.hb, (uint32_t)L.bb, 1};
+    const uint32_t dB[4] = {(uint32_t)L.bkc_d, 1, (uint32_t)L.bn_d, 1};
+    const uint32_t wA[5] = {64, (uint32_t)s.w, (uint32_t)L.whb, (uint32_t)L.wbb, 1};
+    const int wx = std::min(s.cin, 64);
+    const uint32_t wB[5] = {(uint32_t)wx, (uint32_t)s.w, (uint32_t)L.whb, (uint32_t)L.wbb, 1};
+    bool ok = tensor_map_bf16(&L.fwdA, c->d_act[i], 5, act_in, bA, L.bkc_f * 2) &&
+              tensor_map_bf16_strided(&L.fwdB, c->d_shadow + a.off_w[i], 4, wf, rs, bB,
+                                      L.bkc_f * 2) &&
+              tensor_map_bf16(&L.dgrA, c->d_g, 5, g_dims, dA, L.bkc_d * 2) &&
+              tensor_map_bf16_strided(&L.dgrB, c->d_shadow_t + a.off_w[i], 4, wd, rs, dB,
+                                      L.bkc_d * 2) &&
+              tensor_map_bf16(&L.wgA, c->d_g, 5, g_dims, wA, 128) &&
+              tensor_map_bf16(&L.wgB, c->d_act[i], 5, act_in, wB, wx * 2);
+    if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for layer %d", i);
+    L.on = true;
+  }
+  if (partial_max) DALLOC(c->d_partial, sizeof(float) * partial_max);
   return GCPSL_OK;
 }
 
@@ -439,21 +588,28 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   if (init_params) std::memcpy(can.data(), init_params, sizeof(float) * c->P);
   else seeded_init(a, seed, can.data());
   to_kernel_layout(a, can.data(), ker.data());
-  const size_t pb = sizeof(float) * (size_t)(C * c->P);
+  c->P_pad = (c->P + 63) / 64 * 64;
+  const size_t pb = sizeof(float) * (size_t)(C * c->P_pad);
   DALLOC(c->d_theta, pb);
   DALLOC(c->d_mom, pb);
   DALLOC(c->d_grad, pb);
+  CK(cudaMemset(c->d_theta, 0, pb));
   CK(cudaMemset(c->d_mom, 0, pb));
   CK(cudaMemset(c->d_grad, 0, pb));
   for (int k = 0; k < C; ++k)
-    CK(cudaMemcpy(c->d_theta + (int64_t)k * c->P, ker.data(), sizeof(float) * c->P,
+    CK(cudaMemcpy(c->d_theta + (int64_t)k * c->P_pad, ker.data(), sizeof(float) * c->P,
                   cudaMemcpyHostToDevice));
+  DALLOC(c->d_err, sizeof(int));
+  CK(cudaMemset(c->d_err, 0, sizeof(int)));
   if (c->bf) {
-    DALLOC(c->d_shadow, sizeof(bf16) * (size_t)(C * c->P));
+    DALLOC(c->d_shadow, sizeof(bf16) * (size_t)(C * c->P_pad));
+    DALLOC(c->d_shadow_t, sizeof(bf16) * (size_t)(C * c->P_pad));
+    CK(cudaMemset(c->d_shadow, 0, sizeof(bf16) * (size_t)(C * c->P_pad)));
+    CK(cudaMemset(c->d_shadow_t, 0, sizeof(bf16) * (size_t)(C * c->P_pad)));
     std::vector<bf16> sh(c->P);
     for (int64_t p = 0; p < c->P; ++p) sh[p] = __float2bfloat16_rn(ker[p]);
     for (int k = 0; k < C; ++k)
-      CK(cudaMemcpy(c->d_shadow + (int64_t)k * c->P, sh.data(), sizeof(bf16) * c->P,
+      CK(cudaMemcpy(c->d_shadow + (int64_t)k * c->P_pad, sh.data(), sizeof(bf16) * c->P,
                     cudaMemcpyHostToDevice));
   }
 
@@ -481,6 +637,29 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   CK(cudaMemset(c->d_counts, 0, sizeof(int32_t) * (size_t)C * K));
   CK(cudaHostAlloc((void**)&c->h_loss, sizeof(float) * C, cudaHostAllocDefault));
   CK(cudaHostAlloc((void**)&c->h_active, sizeof(int32_t) * C, cudaHostAllocDefault));
+  // reduction shapes (per replica only, so that the summation order does not
+  // depend on C) and the partial-sum scratch
+  int64_t bpart = 0;
+  for (int i = 0; i < a.L(); ++i) {
+    const ConvSpec& s = a.conv[i];
+    auto& R = c->red[i];
+    R.tr = std::max(1, std::min(s.h, 256 / s.w));
+    while (s.h % R.tr) --R.tr;
+    const int tiles = B * (s.h / R.tr);
+    R.tiles_per_split = std::max(1, (tiles + 127) / 128);
+    R.splits = (tiles + R.tiles_per_split - 1) / R.tiles_per_split;
+    R.chunk_px = 256;
+    R.chunks = (int)(((int64_t)B * s.h * s.w + R.chunk_px - 1) / R.chunk_px);
+    bpart = std::max(bpart, (int64_t)C * R.splits * ((int64_t)s.cout * 9 * s.cin + s.cout));
+    bpart = std::max(bpart, (int64_t)C * R.chunks * s.cout);
+  }
+  DALLOC(c->d_bpartial, sizeof(float) * bpart);
+  if (c->bf) {
+    gcpsl_status st = setup_tensor_core_layers(c);
+    if (st != GCPSL_OK) return st;
+    st = refresh_flipped(c);
+    if (st != GCPSL_OK) return st;
+  }
   CK(cudaDeviceSynchronize());
   return GCPSL_OK;
 }
@@ -560,7 +739,7 @@ gcpsl_status gcpsl_step(gcpsl_ctx* c, gcpsl_step_stats* stats) {
                        c->stream));
     CK(cudaMemcpyAsync(c->h_active, c->d_active, sizeof(int32_t) * c->C, cudaMemcpyDeviceToHost,
                        c->stream));
-    CK(cudaStreamSynchronize(c->stream));
+    SYNC_CHECK(c);
     if (stats->loss) std::memcpy(stats->loss, c->h_loss, sizeof(float) * c->C);
     if (stats->active) std::memcpy(stats->active, c->h_active, sizeof(int32_t) * c->C);
   }
@@ -585,8 +764,8 @@ gcpsl_status gcpsl_get_params(gcpsl_ctx* c, int cluster, int segment, float* dst
   if (!dst) return GCPSL_OK;
   if (len < (size_t)(hi - lo)) return fail(c, GCPSL_E_INVAL, "dst too small");
   std::vector<float> ker(c->P), can(c->P);
-  CK(cudaStreamSynchronize(c->stream));
-  CK(cudaMemcpy(ker.data(), c->d_theta + (int64_t)cluster * c->P, sizeof(float) * c->P,
+  SYNC_CHECK(c);
+  CK(cudaMemcpy(ker.data(), c->d_theta + (int64_t)cluster * c->P_pad, sizeof(float) * c->P,
                 cudaMemcpyDeviceToHost));
   to_canonical_layout(c->a, ker.data(), can.data());
   std::memcpy(dst, can.data() + lo, sizeof(float) * (size_t)(hi - lo));
@@ -600,14 +779,15 @@ gcpsl_status gcpsl_set_params(gcpsl_ctx* c, int cluster, const float* src, size_
     return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
   std::vector<float> ker(c->P);
   to_kernel_layout(c->a, src, ker.data());
-  CK(cudaStreamSynchronize(c->stream));
-  CK(cudaMemcpy(c->d_theta + (int64_t)cluster * c->P, ker.data(), sizeof(float) * c->P,
+  SYNC_CHECK(c);
+  CK(cudaMemcpy(c->d_theta + (int64_t)cluster * c->P_pad, ker.data(), sizeof(float) * c->P,
                 cudaMemcpyHostToDevice));
   if (c->bf) {
     std::vector<bf16> sh(c->P);
     for (int64_t p = 0; p < c->P; ++p) sh[p] = __float2bfloat16_rn(ker[p]);
-    CK(cudaMemcpy(c->d_shadow + (int64_t)cluster * c->P, sh.data(), sizeof(bf16) * c->P,
+    CK(cudaMemcpy(c->d_shadow + (int64_t)cluster * c->P_pad, sh.data(), sizeof(bf16) * c->P,
                   cudaMemcpyHostToDevice));
+    return refresh_flipped(c);
   }
   return GCPSL_OK;
 }
@@ -618,8 +798,8 @@ gcpsl_status gcpsl_get_momentum(gcpsl_ctx* c, int cluster, float* dst, size_t le
   if (cluster < 0 || cluster >= c->C || !dst || len != (size_t)c->P)
     return fail(c, GCPSL_E_INVAL, "bad cluster, dst or len");
   std::vector<float> ker(c->P);
-  CK(cudaStreamSynchronize(c->stream));
-  CK(cudaMemcpy(ker.data(), c->d_mom + (int64_t)cluster * c->P, sizeof(float) * c->P,
+  SYNC_CHECK(c);
+  CK(cudaMemcpy(ker.data(), c->d_mom + (int64_t)cluster * c->P_pad, sizeof(float) * c->P,
                 cudaMemcpyDeviceToHost));
   to_canonical_layout(c->a, ker.data(), dst);
   return GCPSL_OK;
@@ -632,8 +812,8 @@ gcpsl_status gcpsl_set_momentum(gcpsl_ctx* c, int cluster, const float* src, siz
     return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
   std::vector<float> ker(c->P);
   to_kernel_layout(c->a, src, ker.data());
-  CK(cudaStreamSynchronize(c->stream));
-  CK(cudaMemcpy(c->d_mom + (int64_t)cluster * c->P, ker.data(), sizeof(float) * c->P,
+  SYNC_CHECK(c);
+  CK(cudaMemcpy(c->d_mom + (int64_t)cluster * c->P_pad, ker.data(), sizeof(float) * c->P,
                 cudaMemcpyHostToDevice));
   return GCPSL_OK;
 }
@@ -646,7 +826,7 @@ gcpsl_status gcpsl_get_pool_codes(gcpsl_ctx* c, int layer, uint8_t* dst, size_t 
   const int64_t n = act_elems(c, layer + 1);
   if (len < (size_t)n) return fail(c, GCPSL_E_INVAL, "dst too small");
   std::vector<uint8_t> raw(n);
-  CK(cudaStreamSynchronize(c->stream));
+  SYNC_CHECK(c);
   CK(cudaMemcpy(raw.data(), c->d_code[layer], n, cudaMemcpyDeviceToHost));
   const int ch = c->a.conv[layer].cout, hw = c->a.out_h(layer) * c->a.out_w(layer);
   for (int64_t cb = 0; cb < (int64_t)c->C * c->B; ++cb)
@@ -668,7 +848,7 @@ gcpsl_status gcpsl_get_cut(gcpsl_ctx* c, int which, float* dst, size_t len) {
     return fail(c, GCPSL_E_INVAL, "bad dst, len or which");
   const void* src = which == GCPSL_CUT_ACT ? c->d_act[c->a.ncl] : c->d_dact[c->a.ncl];
   std::vector<unsigned char> raw((size_t)n * c->esz);
-  CK(cudaStreamSynchronize(c->stream));
+  SYNC_CHECK(c);
   CK(cudaMemcpy(raw.data(), src, raw.size(), cudaMemcpyDeviceToHost));
   const int l = c->a.ncl - 1;
   const int ch = c->a.conv[l].cout, hw = c->a.out_h(l) * c->a.out_w(l);
@@ -693,7 +873,7 @@ gcpsl_status gcpsl_get_cut(gcpsl_ctx* c, int which, float* dst, size_t len) {
 gcpsl_status gcpsl_get_sample(gcpsl_ctx* c, int32_t* idx, int32_t* counts) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
-  CK(cudaStreamSynchronize(c->stream));
+  SYNC_CHECK(c);
   if (idx) CK(cudaMemcpy(idx, c->d_idx, sizeof(int32_t) * c->C * c->B, cudaMemcpyDeviceToHost));
   if (counts)
     CK(cudaMemcpy(counts, c->d_counts, sizeof(int32_t) * (size_t)c->C * c->K,
@@ -706,7 +886,7 @@ int64_t gcpsl_rounds(const gcpsl_ctx* c) { return c ? c->t : -1; }
 gcpsl_status gcpsl_set_stream(gcpsl_ctx* c, void* stream) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
-  CK(cudaStreamSynchronize(c->stream));
+  SYNC_CHECK(c);
   c->stream = stream ? (cudaStream_t)stream : c->own_stream;
   return GCPSL_OK;
 }
