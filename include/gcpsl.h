@@ -190,6 +190,44 @@ int gcpsl_kernel_times(gcpsl_ctx* ctx, const char** names, int64_t* launches, do
                        int cap);
 void gcpsl_reset_kernel_times(gcpsl_ctx* ctx);
 
+/* gcpsl_sample_round_noalloc -- the GPSL round sampler of gcpsl_step for
+ * callers that cannot allocate device memory.  The paper has no counterpart:
+ * this is a deployment variant.  It is for code that may not call cudaMalloc
+ * while it runs, e.g. a plug-in inside a host framework whose allocator owns
+ * the whole device, or a process that reserves all of its device memory up
+ * front and forbids later allocations.  The caller passes every input and
+ * output; the entry point calls no cudaMalloc, cudaFree or other allocating
+ * routine.  Its working storage is a fixed file-scope device array of about
+ * 3.2 MB, which every GPU that loads the library holds until the process
+ * exits.
+ *
+ * It returns, for round `round` (0-based) of C clusters, the batches that a
+ * context with the same clusters, B, seed and cluster_id_base draws in that
+ * round (gcpsl_get_sample), including the epoch permutation rebuild.
+ *  ids:             device, the clusters' example ids concatenated, each
+ *                   cluster's ids in ascending order (cluster n owns
+ *                   ids[cluster_offsets[n] .. cluster_offsets[n+1]));
+ *  cluster_offsets: host, C+1 entries, cluster_offsets[0] = 0;
+ *  owner, labels:   device, indexed by example id;
+ *  idx:             device out [C][B], ids ordered by (owner, id);
+ *  counts:          device out [C][K], b_{k,t} (Eq. 1);
+ *  active:          device out [C], |A_{n,t}|;
+ *  batch_labels:    device out [C][B], labels of idx;
+ *  stream:          cudaStream_t (NULL = legacy default stream).
+ * Limits: 1 <= C <= 1024, 1 <= B <= 1024, every cluster >= B examples, at most
+ * 262144 examples over all clusters; violations return GCPSL_E_INVAL with a
+ * message in gcpsl_last_error(NULL).  The first call on a device looks up the
+ * array's device address with that device current; make that first call
+ * before any stream capture.  Every call shares the one array and rewrites
+ * all of it that it reads, so calls do not depend on earlier ones, but calls
+ * that overlap on the GPU (other streams, other host threads) race on it.
+ * The call returns after the stream has finished the batch.               */
+gcpsl_status gcpsl_sample_round_noalloc(const int32_t* ids, const int64_t* cluster_offsets,
+                                        const int32_t* owner, const int32_t* labels, int K, int C,
+                                        int B, int64_t round, int cluster_id_base, uint64_t seed,
+                                        int32_t* idx, int32_t* counts, int32_t* active,
+                                        int32_t* batch_labels, void* stream);
+
 /* gcpsl_last_error -- static description of the context's last failure
  * (or of the last failed gcpsl_init when ctx is NULL).                   */
 const char* gcpsl_last_error(const gcpsl_ctx* ctx);

@@ -29,7 +29,8 @@ EXPORTS = ("gcpsl_init", "gcpsl_step", "gcpsl_fuse", "gcpsl_get_params", "gcpsl_
            "gcpsl_get_momentum", "gcpsl_set_momentum", "gcpsl_get_pool_codes",
            "gcpsl_get_cut", "gcpsl_cut_elems", "gcpsl_get_sample", "gcpsl_num_params",
            "gcpsl_rounds", "gcpsl_set_stream", "gcpsl_set_timing", "gcpsl_kernel_times",
-           "gcpsl_reset_kernel_times", "gcpsl_last_error", "gcpsl_destroy")
+           "gcpsl_reset_kernel_times", "gcpsl_sample_round_noalloc", "gcpsl_last_error",
+           "gcpsl_destroy")
 
 
 class gcpsl_model_desc(ct.Structure):
@@ -92,6 +93,10 @@ def load() -> ct.CDLL:
     L.gcpsl_kernel_times.restype = ct.c_int
     L.gcpsl_reset_kernel_times.argtypes = [vp]
     L.gcpsl_reset_kernel_times.restype = None
+    L.gcpsl_sample_round_noalloc.argtypes = [vp, ct.POINTER(ct.c_int64), vp, vp, ct.c_int,
+                                             ct.c_int, ct.c_int, ct.c_int64, ct.c_int,
+                                             ct.c_uint64, vp, vp, vp, vp, vp]
+    L.gcpsl_sample_round_noalloc.restype = ct.c_int
     L.gcpsl_last_error.argtypes = [vp]
     L.gcpsl_last_error.restype = ct.c_char_p
     L.gcpsl_destroy.argtypes = [vp]
@@ -117,6 +122,21 @@ def _check(st, h=None):
 # C-ABI names, argument marshalling only ----------------------------------
 def gcpsl_num_params(arch: int, segment: int) -> int:
     return int(load().gcpsl_num_params(arch, segment))
+
+
+def gcpsl_sample_round_noalloc(ids_dev: int, cluster_offsets, owner_dev: int, labels_dev: int,
+                               K: int, C: int, B: int, round_: int, cluster_id_base: int,
+                               seed: int, idx_dev: int, counts_dev: int, active_dev: int,
+                               batch_labels_dev: int, stream: int | None = None):
+    """The round sampler without device allocation; *_dev are device
+    addresses (e.g. tensor.data_ptr()), cluster_offsets a host int64 array."""
+    off = np.ascontiguousarray(cluster_offsets, dtype=np.int64)
+    st = load().gcpsl_sample_round_noalloc(
+        ct.c_void_p(ids_dev), _p(off, ct.c_int64), ct.c_void_p(owner_dev),
+        ct.c_void_p(labels_dev), K, C, B, round_, cluster_id_base, seed, ct.c_void_p(idx_dev),
+        ct.c_void_p(counts_dev), ct.c_void_p(active_dev), ct.c_void_p(batch_labels_dev),
+        ct.c_void_p(stream) if stream else None)
+    _check(st, None)
 
 
 class Context:

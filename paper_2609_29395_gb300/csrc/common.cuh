@@ -29,6 +29,9 @@ struct ArchSpec {
 };
 bool make_arch(int id, ArchSpec* a);
 
+// message returned by gcpsl_last_error(NULL) for calls without a context
+void set_global_error(const char* msg);
+
 // ---------------------------------------------------------------------------
 // Philox4x32-10 (Salmon et al., SC'11): ten rounds, two 32x32 -> 64-bit
 // products per round, key bumped by the Weyl increments between rounds.

@@ -114,6 +114,8 @@ thread_local std::string g_init_error;
 
 }  // namespace
 
+void gcpsl::set_global_error(const char* msg) { g_init_error = msg; }
+
 struct gcpsl_ctx {
   gcpsl_model_desc desc{};
   ArchSpec a{};
