@@ -91,11 +91,18 @@ def work_per_round(w, esz):
 
     for i, (cin, cout, h, ww, _p) in enumerate(convs):
         f = 2.0 * C * B * h * ww * cout * 9 * cin
-        # layers with 32k input / 64k output channels run on the tensor cores
+        # with bf16 operands every forward runs on the tensor cores (the input
+        # layer through the padded two-taps-per-step kernel); weight and data
+        # gradients do for layers with 32k input / 64k output channels
         tc = esz == 2 and cin >= 32 and cin % 32 == 0 and cout % 64 == 0 and ww <= 64
         sfx = "_tc" if tc else ""
-        add("conv_fwd" + sfx, "tensor", f)
+        add("conv_fwd" + ("_tc" if esz == 2 else ""), "tensor", f)
         add("conv_wgrad" + sfx, "tensor", f)
+        # relu/max-pool backward: read dL/dout (+ codes, or the ReLU output),
+        # write g at full resolution
+        full = C * B * h * ww * cout
+        outp = full // 4 if _p else full
+        add("relu_pool_bwd", "hbm", full * esz + outp * (esz + (1 if _p else esz)))
         if i > 0:
             add("conv_dgrad" + sfx, "tensor", f)
     fin, fout = spec["fc"]

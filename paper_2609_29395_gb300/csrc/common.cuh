@@ -93,8 +93,9 @@ cudaError_t launch_conv_dgrad_simt(cudaStream_t s, const T* g, const T* w, int64
 // weight+bias gradient partials of a CUDA-core layer over `splits` pixel
 // ranges (tiles of `tr` image rows): partial[c][split][cout*9*cin + cout]
 template <typename T>
-cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* partial, int C,
-                              int B, const ConvSpec& cs, int tr, int splits, int tiles_per_split);
+cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, int xc, const T* g, float* partial,
+                              int C, int B, const ConvSpec& cs, int tr, int splits,
+                              int tiles_per_split);
 // bias-gradient partials over chunks of chunk_px pixels: partial[c][chunk][cout]
 template <typename T>
 cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int C, int B,
@@ -141,11 +142,15 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
                            const ConvTcArgs& p, int bn, int bkc, int epi, int C);
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C);
+// input layer (<= 8 input channels, activation padded to 8): two taps per
+// MMA step; b = packed weights [C][10][cout][8]
+cudaError_t launch_conv0_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                            const ConvTcArgs& p, int epi, int C);
+cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout,
+                           int cin, int C);
 // dw[c * dw_rs + i] = sum over s (in order) of partial[c][s][i], i < per
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
                                 int splits, int64_t per, int C);
-cudaError_t launch_flip_shadow(cudaStream_t s, const bf16* w, bf16* wt, int64_t rs, int cout,
-                               int cin, int C);
 
 // optim.cu
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,

@@ -69,26 +69,138 @@ __global__ void k_conv_fwd(const T* __restrict__ x, const T* __restrict__ w, int
   code[i] = (uint8_t)(arg | (best > 0.f ? 4 : 0));
 }
 
+// g = dL/dy from dL/d(out).  One thread per (output pixel, group of V
+// channels), V = 16 bytes of T: for a pooled layer it reads the pooled
+// gradient and codes once and writes the whole 2x2 window (the gradient at
+// the recorded first maximum when it is positive, zero elsewhere); without
+// pooling g = dout where the ReLU output is positive.
 template <typename T>
 __global__ void k_relu_pool_bwd(const T* __restrict__ dout, const uint8_t* __restrict__ code,
                                 const T* __restrict__ act, T* __restrict__ g, int C, int B,
                                 int cout, int H, int W, int pool) {
-  const int64_t total = (int64_t)C * B * H * W * cout;
+  constexpr int V = 16 / sizeof(T);
+  const int Ho = pool ? H / 2 : H, Wo = pool ? W / 2 : W;
+  const int groups = cout / V;
+  const int64_t total = (int64_t)C * B * Ho * Wo * groups;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= total) return;
+  const int grp = (int)(i % groups);
+  const int64_t opix = i / groups;                    // output pixel (pooled grid)
+  const int64_t o = opix * cout + grp * V;
+  const uint4 dv = *reinterpret_cast<const uint4*>(dout + o);
+  const T* d = reinterpret_cast<const T*>(&dv);
   if (!pool) {
-    g[i] = to_f(act[i]) > 0.f ? dout[i] : from_f<T>(0.f);
+    const uint4 av = *reinterpret_cast<const uint4*>(act + o);
+    const T* av_ = reinterpret_cast<const T*>(&av);
+    __align__(16) T out[V];
+#pragma unroll
+    for (int k = 0; k < V; ++k) out[k] = to_f(av_[k]) > 0.f ? d[k] : from_f<T>(0.f);
+    *reinterpret_cast<uint4*>(g + o) = *reinterpret_cast<const uint4*>(out);
     return;
   }
-  const int co = (int)(i % cout);
-  int64_t r = i / cout;
-  const int w = (int)(r % W); r /= W;
-  const int h = (int)(r % H);
-  const int64_t cb = r / H;
-  const int64_t o = ((cb * (H / 2) + h / 2) * (W / 2) + w / 2) * cout + co;
-  const int cd = code[o];
-  const bool hit = (cd & 4) && (cd & 3) == ((h & 1) * 2 + (w & 1));
-  g[i] = hit ? dout[o] : from_f<T>(0.f);
+  uint8_t cd[V];
+  if (V == 8) {
+    const uint2 cv = *reinterpret_cast<const uint2*>(code + o);
+    *reinterpret_cast<uint2*>(cd) = cv;
+  } else {
+    const uint32_t cv = *reinterpret_cast<const uint32_t*>(code + o);
+    *reinterpret_cast<uint32_t*>(cd) = cv;
+  }
+  const int pw = (int)(opix % Wo);
+  const int ph = (int)((opix / Wo) % Ho);
+  const int64_t cb = opix / ((int64_t)Wo * Ho);
+#pragma unroll
+  for (int qd = 0; qd < 4; ++qd) {
+    __align__(16) T out[V];
+#pragma unroll
+    for (int k = 0; k < V; ++k) out[k] = ((cd[k] & 4) && (cd[k] & 3) == qd) ? d[k] : from_f<T>(0.f);
+    const int64_t gi = ((cb * H + 2 * ph + (qd >> 1)) * W + 2 * pw + (qd & 1)) * cout + grp * V;
+    *reinterpret_cast<uint4*>(g + gi) = *reinterpret_cast<const uint4*>(out);
+  }
+}
+
+// Weight and bias gradient partials of an input layer with CIN <= 4 channels
+// (x padded to xc channels per pixel): thread = (4-channel output group q,
+// input channel ci, pixel lane); for each of its pixels it loads g for four
+// output channels and x for nine taps and does 36 FMAs.  The lanes' sums are
+// then added in lane order.  Layout of the partial as in k_wgrad_partial.
+template <typename T, int CIN>
+__global__ void __launch_bounds__(256, 2)
+k_wgrad_small_cin(const T* __restrict__ x, int xc, const T* __restrict__ g,
+                  float* __restrict__ partial, int B, int cout, int H, int W, int tr,
+                  int tiles_per_split) {
+  extern __shared__ float sm[];
+  const int c = blockIdx.y, split = blockIdx.x;
+  const int per_w = cout * 9 * CIN, per = per_w + cout;
+  const int combos = (cout / 4) * CIN, lanes = 256 / combos;
+  const int t = threadIdx.x, combo = t % combos, lane = t / combos;
+  const bool worker = lane < lanes;
+  const int q = combo / CIN, ci = combo % CIN;
+  float* gs = sm;                                   // [tr*W][cout]
+  float* xs = sm + tr * W * cout;                   // [(tr+2)][(W+2)][CIN]
+  float acc[36], bacc[4];
+#pragma unroll
+  for (int k = 0; k < 36; ++k) acc[k] = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) bacc[k] = 0.f;
+  const int tiles_img = H / tr, tiles = B * tiles_img;
+  const int t0 = split * tiles_per_split, t1 = min(t0 + tiles_per_split, tiles);
+  for (int tile = t0; tile < t1; ++tile) {
+    const int b = tile / tiles_img, h0 = (tile % tiles_img) * tr;
+    const T* gb = g + (((int64_t)c * B + b) * H + h0) * W * cout;
+    for (int i = t; i < tr * W * cout; i += blockDim.x) gs[i] = to_f(gb[i]);
+    const T* xb = x + ((int64_t)c * B + b) * H * W * xc;
+    for (int i = t; i < (tr + 2) * (W + 2) * CIN; i += blockDim.x) {
+      const int cc = i % CIN, ww = (i / CIN) % (W + 2) - 1, hh = i / (CIN * (W + 2)) + h0 - 1;
+      xs[i] = (hh >= 0 && hh < H && ww >= 0 && ww < W) ? to_f(xb[((int64_t)hh * W + ww) * xc + cc])
+                                                      : 0.f;
+    }
+    __syncthreads();
+    if (worker) {
+      for (int p = lane; p < tr * W; p += lanes) {
+        const int r = p / W, w = p % W;
+        const float4 gv = *reinterpret_cast<const float4*>(gs + p * cout + 4 * q);
+        const float gq[4] = {gv.x, gv.y, gv.z, gv.w};
+#pragma unroll
+        for (int kh = 0; kh < 3; ++kh)
+#pragma unroll
+          for (int kw = 0; kw < 3; ++kw) {
+            const float xv = xs[((r + kh) * (W + 2) + w + kw) * CIN + ci];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) acc[(kh * 3 + kw) * 4 + j] = fmaf(gq[j], xv, acc[(kh * 3 + kw) * 4 + j]);
+          }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) bacc[j] += gq[j];
+      }
+    }
+    __syncthreads();
+  }
+  // red[lane][combo][40]: 36 weight sums + 4 bias sums
+  float* red = sm;
+  if (worker) {
+    float* dst = red + ((int64_t)lane * combos + combo) * 40;
+#pragma unroll
+    for (int k = 0; k < 36; ++k) dst[k] = acc[k];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) dst[36 + k] = bacc[k];
+  }
+  __syncthreads();
+  float* out = partial + ((int64_t)c * gridDim.x + split) * per;
+  for (int o = t; o < per; o += blockDim.x) {
+    int cmb, k;
+    if (o < per_w) {
+      const int cc = o % CIN, tap = (o / CIN) % 9, co = o / (9 * CIN);
+      cmb = (co / 4) * CIN + cc;
+      k = tap * 4 + co % 4;
+    } else {
+      const int co = o - per_w;
+      cmb = (co / 4) * CIN;                       // the ci == 0 threads hold the bias sums
+      k = 36 + co % 4;
+    }
+    float s = 0.f;
+    for (int l = 0; l < lanes; ++l) s += red[((int64_t)l * combos + cmb) * 40 + k];
+    out[o] = s;
+  }
 }
 
 template <typename T>
@@ -128,7 +240,8 @@ constexpr int kWgOut = 32;   // outputs per thread (per <= 256 * kWgOut)
 template <typename T>
 __global__ void __launch_bounds__(256)
 k_wgrad_partial(const T* __restrict__ x, const T* __restrict__ g, float* __restrict__ partial,
-                int B, int cin, int cout, int H, int W, int tr, int tiles_per_split) {
+                int B, int cin, int xc, int cout, int H, int W, int tr, int tiles_per_split) {
+  // xc = channels per pixel of x in memory (>= cin; the padded input layer)
   extern __shared__ float sm[];
   const int c = blockIdx.y, split = blockIdx.x;
   const int per_w = cout * 9 * cin, per = per_w + cout;
@@ -143,10 +256,10 @@ k_wgrad_partial(const T* __restrict__ x, const T* __restrict__ g, float* __restr
     const int b = tile / tiles_img, h0 = (tile % tiles_img) * tr;
     const T* gb = g + (((int64_t)c * B + b) * H + h0) * W * cout;
     for (int i = threadIdx.x; i < tr * W * cout; i += blockDim.x) gs[i] = to_f(gb[i]);
-    const T* xb = x + ((int64_t)c * B + b) * H * W * cin;
+    const T* xb = x + ((int64_t)c * B + b) * H * W * xc;
     for (int i = threadIdx.x; i < (tr + 2) * (W + 2) * cin; i += blockDim.x) {
       const int ci = i % cin, ww = (i / cin) % (W + 2) - 1, hh = i / (cin * (W + 2)) + h0 - 1;
-      xs[i] = (hh >= 0 && hh < H && ww >= 0 && ww < W) ? to_f(xb[((int64_t)hh * W + ww) * cin + ci])
+      xs[i] = (hh >= 0 && hh < H && ww >= 0 && ww < W) ? to_f(xb[((int64_t)hh * W + ww) * xc + ci])
                                                       : 0.f;
     }
     __syncthreads();
@@ -178,18 +291,39 @@ k_wgrad_partial(const T* __restrict__ x, const T* __restrict__ g, float* __restr
 }
 
 // Bias-gradient partials: partial[c][chunk][co] = sum of g over the chunk's
-// `chunk_px` pixels (consecutive threads read consecutive channels).
+// `chunk_px` pixels.  256 threads = (cout/V channel groups of 16 bytes) x
+// lanes; lane l sums pixels l, l+lanes, ... of the chunk, then the lanes'
+// sums are added in lane order.
 template <typename T>
-__global__ void k_bias_partial(const T* __restrict__ g, float* __restrict__ partial, int64_t npix,
-                               int cout, int chunk_px) {
+__global__ void __launch_bounds__(256)
+k_bias_partial(const T* __restrict__ g, float* __restrict__ partial, int64_t npix, int cout,
+               int chunk_px) {
+  constexpr int V = 16 / sizeof(T);
+  __shared__ float red[256 * V];
   const int c = blockIdx.y, chunk = blockIdx.x;
+  const int groups = cout / V, lanes = 256 / groups;
+  const int t = threadIdx.x, grp = t % groups, lane = t / groups;
   const int64_t p0 = (int64_t)chunk * chunk_px;
   const int64_t p1 = min(p0 + chunk_px, npix);
-  const T* gc = g + (int64_t)c * npix * cout;
-  for (int co = threadIdx.x; co < cout; co += blockDim.x) {
-    float s = 0.f;
-    for (int64_t p = p0; p < p1; ++p) s += to_f(gc[p * cout + co]);
-    partial[((int64_t)c * gridDim.x + chunk) * cout + co] = s;
+  const T* gc = g + (int64_t)c * npix * cout + grp * V;
+  float s[V];
+#pragma unroll
+  for (int k = 0; k < V; ++k) s[k] = 0.f;
+  if (lane < lanes) {
+    for (int64_t p = p0 + lane; p < p1; p += lanes) {
+      const uint4 v = *reinterpret_cast<const uint4*>(gc + p * cout);
+      const T* e = reinterpret_cast<const T*>(&v);
+#pragma unroll
+      for (int k = 0; k < V; ++k) s[k] += to_f(e[k]);
+    }
+#pragma unroll
+    for (int k = 0; k < V; ++k) red[lane * cout + grp * V + k] = s[k];
+  }
+  __syncthreads();
+  for (int co = t; co < cout; co += blockDim.x) {
+    float tot = 0.f;
+    for (int l = 0; l < lanes; ++l) tot += red[l * cout + co];
+    partial[((int64_t)c * gridDim.x + chunk) * cout + co] = tot;
   }
 }
 
@@ -211,7 +345,10 @@ cudaError_t launch_conv_fwd_simt(cudaStream_t s, const T* x, const T* w, int64_t
 template <typename T>
 cudaError_t launch_relu_pool_bwd(cudaStream_t s, const T* dout, const uint8_t* code,
                                  const T* act, T* g, int C, int B, const ConvSpec& cs) {
-  const int64_t n = (int64_t)C * B * cs.h * cs.w * cs.cout;
+  constexpr int V = 16 / sizeof(T);
+  if (cs.cout % V) return cudaErrorInvalidValue;
+  const int64_t opix = (int64_t)C * B * (cs.pool ? cs.h * cs.w / 4 : cs.h * cs.w);
+  const int64_t n = opix * (cs.cout / V);
   k_relu_pool_bwd<T><<<blocks(n, 256), 256, 0, s>>>(dout, code, act, g, C, B, cs.cout, cs.h,
                                                      cs.w, cs.pool);
   return cudaGetLastError();
@@ -227,8 +364,33 @@ cudaError_t launch_conv_dgrad_simt(cudaStream_t s, const T* g, const T* w, int64
 }
 
 template <typename T>
-cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* partial, int C,
-                              int B, const ConvSpec& cs, int tr, int splits, int tiles_per_split) {
+cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, int xc, const T* g, float* partial,
+                              int C, int B, const ConvSpec& cs, int tr, int splits,
+                              int tiles_per_split) {
+  if (cs.cin <= 4 && cs.cout % 4 == 0 && (cs.cout / 4) * cs.cin <= 256) {
+    const int stage = (tr * cs.w * cs.cout + (tr + 2) * (cs.w + 2) * cs.cin) * (int)sizeof(float);
+    const int red = 256 * 40 * (int)sizeof(float);
+    const int sm = stage > red ? stage : red;
+#define GCPSL_SMALL_CIN(CI)                                                                   \
+  if (cs.cin == CI) {                                                                         \
+    static bool attr = false;                                                                 \
+    if (!attr) {                                                                              \
+      cudaError_t e = cudaFuncSetAttribute(k_wgrad_small_cin<T, CI>,                          \
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, 96 << 10); \
+      if (e != cudaSuccess) return e;                                                         \
+      attr = true;                                                                            \
+    }                                                                                         \
+    if (sm > (96 << 10)) return cudaErrorInvalidValue;                                        \
+    k_wgrad_small_cin<T, CI><<<dim3(splits, C), 256, sm, s>>>(x, xc, g, partial, B, cs.cout,  \
+                                                              cs.h, cs.w, tr, tiles_per_split); \
+    return cudaGetLastError();                                                                \
+  }
+    GCPSL_SMALL_CIN(1)
+    GCPSL_SMALL_CIN(2)
+    GCPSL_SMALL_CIN(3)
+    GCPSL_SMALL_CIN(4)
+#undef GCPSL_SMALL_CIN
+  }
   const int smem = (tr * cs.w * cs.cout + (tr + 2) * (cs.w + 2) * cs.cin) * (int)sizeof(float);
   if ((int64_t)cs.cout * 9 * cs.cin + cs.cout > 256 * kWgOut) return cudaErrorInvalidValue;
   static int attr_set = 0;
@@ -238,17 +400,18 @@ cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, const T* g, float* par
     if (e != cudaSuccess) return e;
     attr_set = smem;
   }
-  k_wgrad_partial<T><<<dim3(splits, C), 256, smem, s>>>(x, g, partial, B, cs.cin, cs.cout, cs.h,
-                                                        cs.w, tr, tiles_per_split);
+  k_wgrad_partial<T><<<dim3(splits, C), 256, smem, s>>>(x, g, partial, B, cs.cin, xc, cs.cout,
+                                                        cs.h, cs.w, tr, tiles_per_split);
   return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int C, int B,
                                 const ConvSpec& cs, int chunks, int chunk_px) {
+  constexpr int V = 16 / sizeof(T);
+  if (cs.cout % V || cs.cout / V > 256) return cudaErrorInvalidValue;
   const int64_t npix = (int64_t)B * cs.h * cs.w;
-  const int threads = cs.cout < 256 ? cs.cout : 256;
-  k_bias_partial<T><<<dim3(chunks, C), threads, 0, s>>>(g, partial, npix, cs.cout, chunk_px);
+  k_bias_partial<T><<<dim3(chunks, C), 256, 0, s>>>(g, partial, npix, cs.cout, chunk_px);
   return cudaGetLastError();
 }
 
@@ -260,8 +423,8 @@ cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int 
                                                const T*, T*, int, int, const ConvSpec&);       \
   template cudaError_t launch_conv_dgrad_simt<T>(cudaStream_t, const T*, const T*, int64_t,    \
                                                  T*, int, int, const ConvSpec&);               \
-  template cudaError_t launch_wgrad_simt<T>(cudaStream_t, const T*, const T*, float*, int, int, \
-                                            const ConvSpec&, int, int, int);                   \
+  template cudaError_t launch_wgrad_simt<T>(cudaStream_t, const T*, int, const T*, float*, int, \
+                                            int, const ConvSpec&, int, int, int);              \
   template cudaError_t launch_bias_partial<T>(cudaStream_t, const T*, float*, int, int,        \
                                               const ConvSpec&, int, int);
 GCPSL_INST(float)

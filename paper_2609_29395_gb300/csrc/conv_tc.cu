@@ -14,8 +14,11 @@
 //    B = weights [n][tap][c] (K-major, the bf16 shadow).
 //    fprop: n = cout, B = W[co][tap][ci]; epilogue bias + ReLU (+ 2x2 max-pool
 //      with the first-maximum code, decided on the fp32 values).
-//    dgrad: input = g (gradient w.r.t. the pre-activation), n = cin, B = the
-//      transposed, tap-flipped shadow Wt[ci][8-tap][co]; epilogue stores dx.
+//    dgrad: input = g (gradient w.r.t. the pre-activation), n = cin,
+//      B[ci][tap][co] = W[co][8-tap][ci], read MN-major from the same shadow;
+//      epilogue stores dx.
+//  k_conv0_tc: the input layer (<= 8 channels, images padded to 8): two taps
+//    per K=16 MMA step through the unswizzled layout.
 //  k_wgrad_tc: dW[co][tap][ci] = sum_p g[p][co] x[p + shift(tap)][ci]
 //    M = co, N = ci, K = pixels.  Both operands are MN-major tiles (pixels are
 //    rows, channels contiguous), loaded as 64-pixel boxes.  The pixel range is
@@ -48,6 +51,71 @@ __device__ __forceinline__ void epi_bar() {   // the four epilogue warps only
   asm volatile("bar.sync 1, 128;" ::: "memory");
 }
 
+// Epilogue of a 128-pixel x BN-channel accumulator tile (run by the four
+// epilogue warps; thread `te` in [0,128) reads TMEM row `r` at `trow`).
+//  EPI_POOL : + bias, 2x2 max-pool of relu (first maximum, decided on fp32),
+//             via a [128][BN+1] fp32 staging tile in shared memory `sm`;
+//  EPI_RELU : + bias, relu;   EPI_STORE: plain store.
+template <int BN, int EPI>
+__device__ __forceinline__ void conv_epilogue(uint8_t* sm, uint32_t trow, int r, int te, int n0,
+                                              int b0, int h0, int c, const ConvTcArgs& p) {
+  const int W = p.W, H = p.H;
+  if (EPI == EPI_POOL) {
+    float* st = reinterpret_cast<float*>(sm);
+    const float* bias = p.bias + (int64_t)c * p.bias_rs + n0;
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(trow + c0, v);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 16; ++i) st[r * (BN + 1) + c0 + i] = v[i] + bias[c0 + i];
+    }
+    epi_bar();
+    const int Wo = W / 2, hbo = p.hb / 2, Ho = H / 2;
+#pragma unroll 1
+    for (int idx = te; idx < 32 * BN; idx += 128) {
+      const int pp = idx / BN, co = idx % BN;
+      const int pw = pp % Wo, ph = (pp / Wo) % hbo, bb = pp / (Wo * hbo);
+      if (b0 + bb >= p.B) continue;
+      const int r00 = (bb * p.hb + 2 * ph) * W + 2 * pw;
+      const float* s0 = st + r00 * (BN + 1) + co;
+      float best = s0[0];
+      int arg = 0;
+      const float v1 = s0[BN + 1], v2 = s0[W * (BN + 1)], v3 = s0[(W + 1) * (BN + 1)];
+      if (v1 > best) { best = v1; arg = 1; }
+      if (v2 > best) { best = v2; arg = 2; }
+      if (v3 > best) { best = v3; arg = 3; }
+      const int64_t o =
+          ((((int64_t)c * p.B + b0 + bb) * Ho + h0 / 2 + ph) * Wo + pw) * p.n_total + n0 + co;
+      p.out[o] = __float2bfloat16_rn(best > 0.f ? best : 0.f);
+      p.code[o] = (uint8_t)(arg | (best > 0.f ? 4 : 0));
+    }
+  } else {
+    const int w = r % W, hh = (r / W) % p.hb, bb = r / (W * p.hb);
+    const bool valid = b0 + bb < p.B;
+    const int64_t o = ((((int64_t)c * p.B + b0 + bb) * H + h0 + hh) * W + w) * p.n_total + n0;
+    const float* bias = EPI == EPI_RELU ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(trow + c0, v);
+      tmem_ld_wait();
+      if (!valid) continue;
+      __align__(16) bf16 h[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        float x = v[i];
+        if (EPI == EPI_RELU) { x += bias[c0 + i]; x = x > 0.f ? x : 0.f; }
+        h[i] = __float2bfloat16_rn(x);
+      }
+      uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
+      dst[0] = reinterpret_cast<uint4*>(h)[0];
+      dst[1] = reinterpret_cast<uint4*>(h)[1];
+    }
+  }
+}
+
 template <int BN, int BKC>
 struct ConvCfg {
   static constexpr int A_BYTES = BM * BKC * 2;
@@ -60,7 +128,10 @@ struct ConvCfg {
   static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
 };
 
-template <int BN, int BKC, int EPI>
+// BMN = 0: B tile is K-major [n][tap][k] (fprop: W[co][tap][ci]).
+// BMN = 1: B tile is read MN-major from W[co][tap][ci] itself (dgrad: n = ci,
+//   k = co, tap flipped), as 64-wide (or one 32-wide) N blocks of BKC rows.
+template <int BN, int BKC, int EPI, int BMN>
 __global__ void __launch_bounds__(kThreads, 1)
 k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
           const ConvTcArgs p) {
@@ -100,97 +171,143 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
         const int tap = kb / kper, ch = (kb % kper) * BKC;
         mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
         tma_load_5d(sa, &tA, &full[s], ch, tap % 3 - 1, h0 + tap / 3 - 1, b0, c);
-        tma_load_4d(sa + Cfg::A_BYTES, &tB, &full[s], ch, tap, n0, c);
+        if (!BMN) {
+          tma_load_4d(sa + Cfg::A_BYTES, &tB, &full[s], ch, tap, n0, c);
+        } else {
+          constexpr int NBW = BN < 64 ? BN : 64;           // N block width
+#pragma unroll
+          for (int j = 0; j < BN / NBW; ++j)
+            tma_load_4d(sa + Cfg::A_BYTES + j * NBW * BKC * 2, &tB, &full[s], n0 + j * NBW,
+                        8 - tap, ch, c);
+        }
       }
     }
   } else if (warp == 1) {
     if (elect_one()) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
+      constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, BMN);
       constexpr uint32_t swz = BKC == 64 ? SWZ_128 : SWZ_64;
       constexpr uint32_t sbo = BKC * 2 * 8;
-      bool ok = true;
+      // MN-major B: rows of NBW*2 bytes along K, N blocks BKC rows apart
+      constexpr int NBW = BN < 64 ? BN : 64;
+      constexpr uint32_t b_row = NBW * 2;
+      constexpr uint32_t b_swz = NBW == 64 ? SWZ_128 : SWZ_64;
       for (int kb = 0; kb < KB; ++kb) {
         const int s = kb % S;
-        if (!mbar_wait(&full[s], (kb / S) & 1)) { atomicOr(p.err, 2); ok = false; break; }
+        if (!mbar_wait(&full[s], (kb / S) & 1)) { atomicOr(p.err, 2); break; }
         tc_fence_after();
         const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
 #pragma unroll
-        for (int k = 0; k < BKC / 16; ++k)
-          mma_f16(tmem, smem_desc(a + k * 32, 16, sbo, swz), smem_desc(b + k * 32, 16, sbo, swz),
-                  idesc, (kb | k) != 0);
+        for (int k = 0; k < BKC / 16; ++k) {
+          const uint64_t bd = BMN ? smem_desc(b + k * 16 * b_row, NBW * BKC * 2, 8 * b_row, b_swz)
+                                  : smem_desc(b + k * 32, 16, sbo, swz);
+          mma_f16(tmem, smem_desc(a + k * 32, 16, sbo, swz), bd, idesc, (kb | k) != 0);
+        }
         mma_commit(&empty[s]);
       }
-      (void)ok;
       mma_commit(&done);
     }
   } else {
     // ---------------- epilogue: warps 2..5 ----------------
     const int q = warp & 3;                     // TMEM lane quarter of this warp
-    const int r = q * 32 + lane;                // M row = pixel of the tile
-    const bool ok = mbar_wait(&done, 0);
-    if (!ok) atomicOr(p.err, 4);
+    if (!mbar_wait(&done, 0)) atomicOr(p.err, 4);
     tc_fence_after();
-    const int W = p.W, H = p.H;
-    const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
-    if (EPI == EPI_POOL) {
-      float* st = reinterpret_cast<float*>(sm);
-      const float* bias = p.bias + (int64_t)c * p.bias_rs + n0;
-#pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
-        tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) st[r * (BN + 1) + c0 + i] = v[i] + bias[c0 + i];
-      }
-      epi_bar();
-      const int Wo = W / 2, hbo = p.hb / 2, Ho = H / 2;
-      const int te = threadIdx.x - 64;
-#pragma unroll 1
-      for (int idx = te; idx < 32 * BN; idx += 128) {
-        const int pp = idx / BN, co = idx % BN;
-        const int pw = pp % Wo, ph = (pp / Wo) % hbo, bb = pp / (Wo * hbo);
-        if (b0 + bb >= p.B) continue;
-        const int r00 = (bb * p.hb + 2 * ph) * W + 2 * pw;
-        const float* s0 = st + r00 * (BN + 1) + co;
-        float best = s0[0];
-        int arg = 0;
-        const float v1 = s0[BN + 1], v2 = s0[W * (BN + 1)], v3 = s0[(W + 1) * (BN + 1)];
-        if (v1 > best) { best = v1; arg = 1; }
-        if (v2 > best) { best = v2; arg = 2; }
-        if (v3 > best) { best = v3; arg = 3; }
-        const int64_t o =
-            ((((int64_t)c * p.B + b0 + bb) * Ho + h0 / 2 + ph) * Wo + pw) * p.n_total + n0 + co;
-        p.out[o] = __float2bfloat16_rn(best > 0.f ? best : 0.f);
-        p.code[o] = (uint8_t)(arg | (best > 0.f ? 4 : 0));
-      }
-    } else {
-      const int w = r % W, hh = (r / W) % p.hb, bb = r / (W * p.hb);
-      const bool valid = b0 + bb < p.B;
-      const int64_t o = ((((int64_t)c * p.B + b0 + bb) * H + h0 + hh) * W + w) * p.n_total + n0;
-      const float* bias = EPI == EPI_RELU ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
-#pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
-        tmem_ld_wait();
-        if (!valid) continue;
-        __align__(16) bf16 h[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float x = v[i];
-          if (EPI == EPI_RELU) { x += bias[c0 + i]; x = x > 0.f ? x : 0.f; }
-          h[i] = __float2bfloat16_rn(x);
-        }
-        uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
-        dst[0] = reinterpret_cast<uint4*>(h)[0];
-        dst[1] = reinterpret_cast<uint4*>(h)[1];
-      }
-    }
+    conv_epilogue<BN, EPI>(sm, tmem + ((uint32_t)(q * 32) << 16), q * 32 + lane,
+                           threadIdx.x - 64, n0, b0, h0, c, p);
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
+}
+
+// ---------------------------------------------------------------------------
+// input layer: at most 8 input channels (the gathered images, padded to 8)
+// ---------------------------------------------------------------------------
+// A K=16 MMA step takes two taps: with the unswizzled K-major layout a K=16
+// slice is two 8-element core-matrix columns whose distance is the leading
+// byte offset, so tap t's 128 x 16 B box and tap t+1's box can sit 2 KB apart.
+// Ten tap slots are loaded (slot 9 repeats tap 8); the packed weights
+// [tap][co][8] have zeros for tap 9 and for channels >= cin.
+template <int BN>
+struct Conv0Cfg {
+  static constexpr int SLOT_A = BM * 16;                 // one tap: 128 px x 8 ch
+  static constexpr int A_BYTES = 10 * SLOT_A;
+  static constexpr int B_BYTES = 10 * BN * 16;
+  static constexpr int STAGING = BM * (BN + 1) * 4;
+  static constexpr int SMEM = 1024 + (A_BYTES + B_BYTES > STAGING ? A_BYTES + B_BYTES : STAGING);
+  static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+};
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+k_conv0_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
+           const ConvTcArgs p) {
+  using Cfg = Conv0Cfg<BN>;
+  extern __shared__ uint8_t smraw[];
+  uint8_t* sm = align1024(smraw);
+  __shared__ uint64_t full, done;
+  __shared__ uint32_t tbase;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x, c = blockIdx.z;
+  const int b0 = (mt / p.tiles_h) * p.bb, h0 = (mt % p.tiles_h) * p.hb;
+  if (threadIdx.x == 0) {
+    mbar_init(&full, 1);
+    mbar_init(&done, 1);
+    fence_mbar_init();
+  }
+  if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tbase;
+  if (warp == 0) {
+    if (elect_one()) {
+      mbar_arrive_expect_tx(&full, Cfg::A_BYTES + Cfg::B_BYTES);
+#pragma unroll
+      for (int j = 0; j < 10; ++j) {
+        const int tap = j < 9 ? j : 8;
+        tma_load_5d(sm + j * Cfg::SLOT_A, &tA, &full, 0, tap % 3 - 1, h0 + tap / 3 - 1, b0, c);
+      }
+      tma_load_4d(sm + Cfg::A_BYTES, &tB, &full, 0, 0, 0, c);
+    }
+  } else if (warp == 1) {
+    if (elect_one()) {
+      if (mbar_wait(&full, 0)) {
+        tc_fence_after();
+        constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
+        const uint32_t a = smem_u32(sm), b = a + Cfg::A_BYTES;
+#pragma unroll
+        for (int k = 0; k < 5; ++k)
+          mma_f16(tmem, smem_desc(a + 2 * k * Cfg::SLOT_A, Cfg::SLOT_A, 128, SWZ_NONE),
+                  smem_desc(b + 2 * k * BN * 16, BN * 16, 128, SWZ_NONE), idesc, k != 0);
+      } else {
+        atomicOr(p.err, 64);
+      }
+      mma_commit(&done);
+    }
+  } else {
+    const int q = warp & 3;
+    if (!mbar_wait(&done, 0)) atomicOr(p.err, 128);
+    tc_fence_after();
+    conv_epilogue<BN, EPI>(sm, tmem + ((uint32_t)(q * 32) << 16), q * 32 + lane,
+                           threadIdx.x - 64, 0, b0, h0, c, p);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
+}
+
+// packed input-layer weights: w0p[c][tap][co][8] = W[co][tap][ci] for
+// tap < 9 and ci < cin, else 0
+__global__ void k_pack_w0(const bf16* __restrict__ w, bf16* __restrict__ w0p, int64_t rs,
+                          int cout, int cin) {
+  const int c = blockIdx.y;
+  const int per = 10 * cout * 8;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < per; i += gridDim.x * blockDim.x) {
+    const int ch = i % 8, co = (i / 8) % cout, tap = i / (8 * cout);
+    bf16 v = __float2bfloat16_rn(0.f);
+    if (tap < 9 && ch < cin) v = w[(int64_t)c * rs + ((int64_t)co * 9 + tap) * cin + ch];
+    w0p[(int64_t)c * per + i] = v;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -315,45 +432,50 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
 }
 
-// dw[c][i] = sum over splits (in order) of partial[c][s][i]
-__global__ void k_wgrad_reduce(const float* __restrict__ partial, float* __restrict__ dw,
-                               int64_t dw_rs, int splits, int64_t per) {
+// dw[c][i] = sum_s partial[c][s][i].  A block of 8 warps covers 32 * 8/G
+// consecutive columns; the G warps of a column group split the s range
+// (warp g takes s = g, g+G, ...) and their sums are added in warp order, so
+// the order depends on `splits` only.
+template <int G>
+__global__ void __launch_bounds__(256)
+k_wgrad_reduce(const float* __restrict__ partial, float* __restrict__ dw, int64_t dw_rs,
+               int splits, int64_t per) {
+  __shared__ float red[8][32];
   const int c = blockIdx.y;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < per;
-       i += (int64_t)gridDim.x * blockDim.x) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int grp = w / G, sub = w % G;
+  const int64_t i = ((int64_t)blockIdx.x * (8 / G) + grp) * 32 + lane;
+  float s = 0.f;
+  if (i < per) {
     const float* src = partial + (int64_t)c * splits * per + i;
-    float s = 0.f;
-    for (int k = 0; k < splits; ++k) s += src[(int64_t)k * per];
-    dw[(int64_t)c * dw_rs + i] = s;
+    for (int k = sub; k < splits; k += G) s += src[(int64_t)k * per];
+  }
+  if (G == 1) {
+    if (i < per) dw[(int64_t)c * dw_rs + i] = s;
+    return;
+  }
+  red[w][lane] = s;
+  __syncthreads();
+  if (sub == 0 && i < per) {
+    float t = red[w][lane];
+#pragma unroll
+    for (int q = 1; q < G; ++q) t += red[w + q][lane];
+    dw[(int64_t)c * dw_rs + i] = t;
   }
 }
 
-// Wt[c][ci][8 - tap][co] = W[c][co][tap][ci] (bf16 shadow, conv weights only)
-__global__ void k_flip_shadow(const bf16* __restrict__ w, bf16* __restrict__ wt, int64_t rs,
-                              int cout, int cin) {
-  const int c = blockIdx.y;
-  const int64_t per = (int64_t)cout * 9 * cin;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < per;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int ci = (int)(i % cin);
-    const int tap = (int)((i / cin) % 9);
-    const int co = (int)(i / (9 * (int64_t)cin));
-    wt[(int64_t)c * rs + ((int64_t)ci * 9 + (8 - tap)) * cout + co] = w[(int64_t)c * rs + i];
-  }
-}
-
-template <int BN, int BKC, int EPI>
+template <int BN, int BKC, int EPI, int BMN>
 cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
                              const ConvTcArgs& p, dim3 grid) {
   using Cfg = ConvCfg<BN, BKC>;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_conv_tc<BN, BKC, EPI>,
+    cudaError_t e = cudaFuncSetAttribute(k_conv_tc<BN, BKC, EPI, BMN>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k_conv_tc<BN, BKC, EPI><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p);
+  k_conv_tc<BN, BKC, EPI, BMN><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p);
   return cudaGetLastError();
 }
 
@@ -449,12 +571,15 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
                            const ConvTcArgs& p, int bn, int bkc, int epi, int C) {
   const int tiles_m = p.tiles_h * ((p.B + p.bb - 1) / p.bb);
   dim3 grid(tiles_m, p.n_total / bn, C);
-#define GCPSL_CONV_CASE(BN_, BKC_, EPI_) \
-  if (bn == BN_ && bkc == BKC_ && epi == EPI_) return launch_conv_inst<BN_, BKC_, EPI_>(s, a, b, p, grid);
+  // fprop epilogues read a K-major B; the data gradient (EPI_STORE) reads
+  // the same weights MN-major
+#define GCPSL_CONV_CASE(BN_, BKC_, EPI_, BMN_)             \
+  if (bn == BN_ && bkc == BKC_ && epi == EPI_)             \
+    return launch_conv_inst<BN_, BKC_, EPI_, BMN_>(s, a, b, p, grid);
 #define GCPSL_CONV_EPIS(BN_, BKC_)          \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_POOL)      \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_RELU)      \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_STORE)
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_POOL, 0)   \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_RELU, 0)   \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_STORE, 1)
   GCPSL_CONV_EPIS(32, 64)
   GCPSL_CONV_EPIS(64, 32)
   GCPSL_CONV_EPIS(64, 64)
@@ -464,6 +589,42 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
 #undef GCPSL_CONV_EPIS
 #undef GCPSL_CONV_CASE
   return cudaErrorInvalidValue;
+}
+
+template <int BN, int EPI>
+static cudaError_t launch_conv0_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                                     const ConvTcArgs& p, dim3 grid) {
+  using Cfg = Conv0Cfg<BN>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_conv0_tc<BN, EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  k_conv0_tc<BN, EPI><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_conv0_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                            const ConvTcArgs& p, int epi, int C) {
+  const int tiles_m = p.tiles_h * ((p.B + p.bb - 1) / p.bb);
+  dim3 grid(tiles_m, 1, C);
+  const int bn = p.n_total;
+  if (bn == 16 && epi == EPI_POOL) return launch_conv0_inst<16, EPI_POOL>(s, a, b, p, grid);
+  if (bn == 16 && epi == EPI_RELU) return launch_conv0_inst<16, EPI_RELU>(s, a, b, p, grid);
+  if (bn == 32 && epi == EPI_POOL) return launch_conv0_inst<32, EPI_POOL>(s, a, b, p, grid);
+  if (bn == 32 && epi == EPI_RELU) return launch_conv0_inst<32, EPI_RELU>(s, a, b, p, grid);
+  if (bn == 64 && epi == EPI_POOL) return launch_conv0_inst<64, EPI_POOL>(s, a, b, p, grid);
+  if (bn == 64 && epi == EPI_RELU) return launch_conv0_inst<64, EPI_RELU>(s, a, b, p, grid);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout,
+                           int cin, int C) {
+  const int per = 10 * cout * 8;
+  k_pack_w0<<<dim3((unsigned)((per + 255) / 256), C), 256, 0, s>>>(w, w0p, rs, cout, cin);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
@@ -478,20 +639,15 @@ cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensor
 
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
                                 int splits, int64_t per, int C) {
-  const int threads = 256;
-  int64_t blocks = (per + threads - 1) / threads;
-  if (blocks > 1024) blocks = 1024;
-  k_wgrad_reduce<<<dim3((unsigned)blocks, C), threads, 0, s>>>(partial, dw, dw_rs, splits, per);
+  const int G = splits <= 2 ? 1 : splits <= 8 ? 2 : splits <= 32 ? 4 : 8;
+  const int64_t cols_per_block = 32 * (8 / G);
+  const dim3 grid((unsigned)((per + cols_per_block - 1) / cols_per_block), C);
+  if (G == 1) k_wgrad_reduce<1><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
+  else if (G == 2) k_wgrad_reduce<2><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
+  else if (G == 4) k_wgrad_reduce<4><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
+  else k_wgrad_reduce<8><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
   return cudaGetLastError();
 }
 
-cudaError_t launch_flip_shadow(cudaStream_t s, const bf16* w, bf16* wt, int64_t rs, int cout,
-                               int cin, int C) {
-  const int64_t per = (int64_t)cout * 9 * cin;
-  int64_t blocks = (per + 255) / 256;
-  if (blocks > 512) blocks = 512;
-  k_flip_shadow<<<dim3((unsigned)blocks, C), 256, 0, s>>>(w, wt, rs, cout, cin);
-  return cudaGetLastError();
-}
 
 }  // namespace gcpsl

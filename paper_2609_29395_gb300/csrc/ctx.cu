@@ -148,7 +148,6 @@ struct gcpsl_ctx {
   float* d_mom = nullptr;
   float* d_grad = nullptr;
   bf16* d_shadow = nullptr;        // [C][P_pad] bf16 operand copy (bf16 mode)
-  bf16* d_shadow_t = nullptr;      // conv weights as Wt[ci][8-tap][co] (data-gradient operand)
   int* d_err = nullptr;            // device error word (bounded waits that gave up)
 
   // tensor-core layers (bf16 mode): tile shapes and TMA descriptors
@@ -160,6 +159,15 @@ struct gcpsl_ctx {
     int splits, kb_total, kb_per_split;
     CUtensorMap fwdA, fwdB, dgrA, dgrB, wgA, wgB;
   } tc[4];
+  // input layer on the tensor cores (bf16 mode): the gathered images are
+  // padded to x0c = 8 channels; packed weights [C][10][cout][8]
+  struct Tc0Layer {
+    bool on = false;
+    int hb, bb, tiles_h;
+    CUtensorMap A, B;
+  } tc0;
+  int x0c = 3;
+  bf16* d_w0p = nullptr;
   float* d_partial = nullptr;      // weight-gradient split partials (tensor-core layers)
   // CUDA-core gradient reductions: weight+bias partials of the other layers
   // (tiles of tr image rows, tiles_per_split tiles per block) and bias
@@ -320,7 +328,7 @@ gcpsl_status check_usable(gcpsl_ctx* c) {
 }
 
 int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
-  if (i == 0) return (int64_t)c->C * c->B * 1024 * 3;
+  if (i == 0) return (int64_t)c->C * c->B * 1024 * c->x0c;
   const int l = i - 1;
   return (int64_t)c->C * c->B * c->a.out_h(l) * c->a.out_w(l) * c->a.conv[l].cout;
 }
@@ -328,14 +336,11 @@ int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
 // ---------------------------------------------------------------------------
 // One local round of every cluster
 // ---------------------------------------------------------------------------
-// the data-gradient operand Wt of every tensor-core layer, from the shadow
-gcpsl_status refresh_flipped(gcpsl_ctx* c) {
-  for (int i = 0; i < c->a.L(); ++i) {
-    if (!c->tc[i].on) continue;
-    LAUNCH("flip_shadow", launch_flip_shadow(c->stream, c->d_shadow + c->a.off_w[i],
-                                             c->d_shadow_t + c->a.off_w[i], c->P_pad,
-                                             c->a.conv[i].cout, c->a.conv[i].cin, c->C));
-  }
+// the packed input-layer weights, from the shadow (after every update)
+gcpsl_status refresh_derived(gcpsl_ctx* c) {
+  if (c->tc0.on)
+    LAUNCH("pack_w0", launch_pack_w0(c->stream, c->d_shadow + c->a.off_w[0], c->d_w0p, c->P_pad,
+                                     c->a.conv[0].cout, c->a.conv[0].cin, c->C));
   return GCPSL_OK;
 }
 
@@ -374,7 +379,13 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
   // client segment to the cut, then the server segment
   for (int i = 0; i < a.L(); ++i) {
     const auto& L = c->tc[i];
-    if (L.on) {
+    if (i == 0 && c->tc0.on) {
+      const auto& L0 = c->tc0;
+      ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 8, L0.hb, L0.bb, L0.tiles_h, a.conv[0].cout,
+                   c->d_theta + a.off_b[0], P, (bf16*)(void*)act[1], c->d_code[0], c->d_err};
+      LAUNCH("conv_fwd_tc", launch_conv0_tc(s, L0.A, L0.B, p, a.conv[0].pool ? EPI_POOL : EPI_RELU,
+                                            C));
+    } else if (L.on) {
       ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.hb, L.bb, L.tiles_h,
                    a.conv[i].cout, c->d_theta + a.off_b[i], P, (bf16*)(void*)act[i + 1],
                    c->d_code[i], c->d_err};
@@ -412,8 +423,9 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
                                                  R.chunks, cs.cout, C));
     } else {
       // weights and bias together (the bias follows the weight in the store)
-      LAUNCH("conv_wgrad", launch_wgrad_simt<T>(s, act[i], g, c->d_bpartial, C, B, cs, R.tr,
-                                                R.splits, R.tiles_per_split));
+      LAUNCH("conv_wgrad", launch_wgrad_simt<T>(s, act[i], i == 0 ? c->x0c : cs.cin, g,
+                                                c->d_bpartial, C, B, cs, R.tr, R.splits,
+                                                R.tiles_per_split));
       LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_bpartial, c->d_grad + a.off_w[i], P,
                                                  R.splits,
                                                  (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
@@ -431,13 +443,13 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
   LAUNCH("sgd", launch_sgd(s, c->d_theta, c->d_mom, c->d_grad, c->d_shadow, (int64_t)C * P,
                            c->desc.lr, c->desc.momentum, c->desc.weight_decay,
                            c->desc.nesterov, c->d_t));
-  return refresh_flipped(c);
+  return refresh_derived(c);
 }
 
 gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
   if (c->C == 1) return GCPSL_OK;                 // q_1 = 1: the identity
   LAUNCH("fuse", launch_fuse(c->stream, c->d_theta, c->d_shadow, c->d_q, c->C, c->P_pad));
-  return refresh_flipped(c);
+  return refresh_derived(c);
 }
 
 // Tile shapes, split-K factors and TMA descriptors of every layer that runs on
@@ -472,7 +484,8 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     // the split (hence the summation order) depends on the per-replica shape
     // only, so C grouped replicas reproduce C one-replica runs bit for bit
     int splits = (152 + tiles - 1) / tiles;
-    splits = std::max(1, std::min(splits, L.kb_total));
+    // at least 16 K blocks (1024 pixels) per split: fewer partial bytes
+    splits = std::max(1, std::min(splits, (L.kb_total + 15) / 16));
     L.kb_per_split = (L.kb_total + splits - 1) / splits;
     L.splits = (L.kb_total + L.kb_per_split - 1) / L.kb_per_split;
     partial_max = std::max(partial_max, (int64_t)C * L.splits * s.cout * 9 * s.cin);
@@ -482,12 +495,13 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     const uint64_t g_dims[5] = {(uint64_t)s.cout, (uint64_t)s.w, (uint64_t)s.h, (uint64_t)B,
                                 (uint64_t)C};
     const uint64_t wf[4] = {(uint64_t)s.cin, 9, (uint64_t)s.cout, (uint64_t)C};
-    const uint64_t wd[4] = {(uint64_t)s.cout, 9, (uint64_t)s.cin, (uint64_t)C};
     const uint64_t rs = (uint64_t)c->P_pad * 2;
     const uint32_t bA[5] = {(uint32_t)L.bkc_f, (uint32_t)s.w, (uint32_t)L.hb, (uint32_t)L.bb, 1};
     const uint32_t bB[4] = {(uint32_t)L.bkc_f, 1, (uint32_t)L.bn_f, 1};
     const uint32_t dA[5] = {(uint32_t)L.bkc_d, (uint32_t)s.w, (uint32_t)L.hb, (uint32_t)L.bb, 1};
-    const uint32_t dB[4] = {(uint32_t)L.bkc_d, 1, (uint32_t)L.bn_d, 1};
+    // data gradient: W[co][tap][ci] read MN-major, N blocks of <= 64 ci
+    const int nbw = std::min(L.bn_d, 64);
+    const uint32_t dB[4] = {(uint32_t)nbw, 1, (uint32_t)L.bkc_d, 1};
     const uint32_t wA[5] = {64, (uint32_t)s.w, (uint32_t)L.whb, (uint32_t)L.wbb, 1};
     const int wx = std::min(s.cin, 64);
     const uint32_t wB[5] = {(uint32_t)wx, (uint32_t)s.w, (uint32_t)L.whb, (uint32_t)L.wbb, 1};
@@ -495,14 +509,35 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
               tensor_map_bf16_strided(&L.fwdB, c->d_shadow + a.off_w[i], 4, wf, rs, bB,
                                       L.bkc_f * 2) &&
               tensor_map_bf16(&L.dgrA, c->d_g, 5, g_dims, dA, L.bkc_d * 2) &&
-              tensor_map_bf16_strided(&L.dgrB, c->d_shadow_t + a.off_w[i], 4, wd, rs, dB,
-                                      L.bkc_d * 2) &&
+              tensor_map_bf16_strided(&L.dgrB, c->d_shadow + a.off_w[i], 4, wf, rs, dB,
+                                      nbw * 2) &&
               tensor_map_bf16(&L.wgA, c->d_g, 5, g_dims, wA, 128) &&
               tensor_map_bf16(&L.wgB, c->d_act[i], 5, act_in, wB, wx * 2);
     if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for layer %d", i);
     L.on = true;
   }
   if (partial_max) DALLOC(c->d_partial, sizeof(float) * partial_max);
+
+  // the input layer (<= 8 channels): two taps per MMA step over the padded
+  // images; in bf16 mode it must run here (the input is stored padded)
+  const ConvSpec& s0 = a.conv[0];
+  auto& L0 = c->tc0;
+  L0.on = false;
+  L0.hb = std::min(s0.h, 128 / s0.w);
+  L0.bb = 128 / (s0.w * std::max(1, L0.hb));
+  if (s0.cin > 8 || (s0.cout != 16 && s0.cout != 32 && s0.cout != 64) || s0.w > 128 ||
+      128 % s0.w || s0.w * L0.hb * L0.bb != 128 || s0.h % L0.hb)
+    return fail(c, GCPSL_E_UNSUPPORTED, "input layer shape not supported with bf16 operands");
+  L0.tiles_h = s0.h / L0.hb;
+  DALLOC(c->d_w0p, sizeof(bf16) * (size_t)C * 10 * s0.cout * 8);
+  const uint64_t xdims[5] = {8, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B, (uint64_t)C};
+  const uint32_t xbox[5] = {8, (uint32_t)s0.w, (uint32_t)L0.hb, (uint32_t)L0.bb, 1};
+  const uint64_t wdims[4] = {8, (uint64_t)s0.cout, 10, (uint64_t)C};
+  const uint32_t wbox[4] = {8, (uint32_t)s0.cout, 10, 1};
+  if (!tensor_map_bf16(&L0.A, c->d_act[0], 5, xdims, xbox, 0) ||
+      !tensor_map_bf16(&L0.B, c->d_w0p, 4, wdims, wbox, 0))
+    return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input layer");
+  L0.on = true;
   return GCPSL_OK;
 }
 
@@ -524,6 +559,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   c->K = K; c->C = C; c->B = B; c->F = F; c->seed = seed;
   c->bf = desc->operand_dtype == GCPSL_BF16;
   c->esz = c->bf ? 2 : 4;
+  c->x0c = c->bf ? 8 : 3;
   const ArchSpec& a = c->a;
   c->P = a.p_total;
   c->n = data->n;
@@ -605,9 +641,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   CK(cudaMemset(c->d_err, 0, sizeof(int)));
   if (c->bf) {
     DALLOC(c->d_shadow, sizeof(bf16) * (size_t)(C * c->P_pad));
-    DALLOC(c->d_shadow_t, sizeof(bf16) * (size_t)(C * c->P_pad));
     CK(cudaMemset(c->d_shadow, 0, sizeof(bf16) * (size_t)(C * c->P_pad)));
-    CK(cudaMemset(c->d_shadow_t, 0, sizeof(bf16) * (size_t)(C * c->P_pad)));
     std::vector<bf16> sh(c->P);
     for (int64_t p = 0; p < c->P; ++p) sh[p] = __float2bfloat16_rn(ker[p]);
     for (int k = 0; k < C; ++k)
@@ -650,7 +684,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     const int tiles = B * (s.h / R.tr);
     R.tiles_per_split = std::max(1, (tiles + 127) / 128);
     R.splits = (tiles + R.tiles_per_split - 1) / R.tiles_per_split;
-    R.chunk_px = 256;
+    R.chunk_px = 1024;
     R.chunks = (int)(((int64_t)B * s.h * s.w + R.chunk_px - 1) / R.chunk_px);
     bpart = std::max(bpart, (int64_t)C * R.splits * ((int64_t)s.cout * 9 * s.cin + s.cout));
     bpart = std::max(bpart, (int64_t)C * R.chunks * s.cout);
@@ -659,7 +693,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   if (c->bf) {
     gcpsl_status st = setup_tensor_core_layers(c);
     if (st != GCPSL_OK) return st;
-    st = refresh_flipped(c);
+    st = refresh_derived(c);
     if (st != GCPSL_OK) return st;
   }
   CK(cudaDeviceSynchronize());
@@ -789,7 +823,7 @@ gcpsl_status gcpsl_set_params(gcpsl_ctx* c, int cluster, const float* src, size_
     for (int64_t p = 0; p < c->P; ++p) sh[p] = __float2bfloat16_rn(ker[p]);
     CK(cudaMemcpy(c->d_shadow + (int64_t)cluster * c->P_pad, sh.data(), sizeof(bf16) * c->P,
                   cudaMemcpyHostToDevice));
-    return refresh_flipped(c);
+    return refresh_derived(c);
   }
   return GCPSL_OK;
 }

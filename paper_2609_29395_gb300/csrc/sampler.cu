@@ -99,7 +99,9 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
   if (b == 0) active[c] = first;
 }
 
-// x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w]
+// x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w]; fp32 storage keeps 3
+// channels per pixel, bf16 storage pads each pixel to 8 channels (16 bytes,
+// channels 3..7 zero) for the tensor-core input layer
 template <typename T>
 __global__ void k_gather(const float* __restrict__ images, const int32_t* __restrict__ idx,
                          int CB, T* __restrict__ x0) {
@@ -108,10 +110,21 @@ __global__ void k_gather(const float* __restrict__ images, const int32_t* __rest
   const int64_t cb = i >> 10;
   const int p = (int)(i & 1023);
   const float* src = images + (int64_t)idx[cb] * 3072 + p;
-  T* dst = x0 + i * 3;
-  dst[0] = from_f<T>(src[0]);
-  dst[1] = from_f<T>(src[1024]);
-  dst[2] = from_f<T>(src[2048]);
+  const float r = src[0], g = src[1024], b = src[2048];
+  if (sizeof(T) == 2) {
+    __align__(16) T v[8];
+    v[0] = from_f<T>(r);
+    v[1] = from_f<T>(g);
+    v[2] = from_f<T>(b);
+#pragma unroll
+    for (int k = 3; k < 8; ++k) v[k] = from_f<T>(0.f);
+    reinterpret_cast<uint4*>(x0)[i] = *reinterpret_cast<uint4*>(v);
+  } else {
+    T* dst = x0 + i * 3;
+    dst[0] = from_f<T>(r);
+    dst[1] = from_f<T>(g);
+    dst[2] = from_f<T>(b);
+  }
 }
 
 }  // namespace
