@@ -42,7 +42,11 @@ FLUSH_BYTES = 256 << 20
 
 # DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by
 # kernel kind; valid only while the kernel source hashes to the recorded value.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # profiles/k_conv_tc_fprop_splitcnn_c4_full.md (dram read + write per launch)
+    "conv_fwd_tc.L1": {"bytes": 16.9408e6, "src_hash": "1a7da3a41956111a"},
+    "conv_fwd_tc.L2": {"bytes": 8.99584e6, "src_hash": "1a7da3a41956111a"},
+}
 
 
 def parse():
@@ -95,16 +99,16 @@ def work_per_round(w, esz):
         # layer through the padded two-taps-per-step kernel); weight and data
         # gradients do for layers with 32k input / 64k output channels
         tc = esz == 2 and cin >= 32 and cin % 32 == 0 and cout % 64 == 0 and ww <= 64
-        sfx = "_tc" if tc else ""
-        add("conv_fwd" + ("_tc" if esz == 2 else ""), "tensor", f)
-        add("conv_wgrad" + sfx, "tensor", f)
+        # tensor-core launches are timed per layer (".L<i>")
+        add(f"conv_fwd_tc.L{i}" if esz == 2 else "conv_fwd", "tensor", f)
+        add(f"conv_wgrad_tc.L{i}" if tc else "conv_wgrad", "tensor", f)
         # relu/max-pool backward: read dL/dout (+ codes, or the ReLU output),
         # write g at full resolution
         full = C * B * h * ww * cout
         outp = full // 4 if _p else full
         add("relu_pool_bwd", "hbm", full * esz + outp * (esz + (1 if _p else esz)))
         if i > 0:
-            add("conv_dgrad" + sfx, "tensor", f)
+            add(f"conv_dgrad_tc.L{i}" if tc else "conv_dgrad", "tensor", f)
     fin, fout = spec["fc"]
     fc = 2.0 * C * B * fin * fout
     return {
@@ -116,9 +120,11 @@ def work_per_round(w, esz):
 
 
 def kernel_source_hash(kind):
+    base = kind.split(".")[0]
     src = {"conv_fwd": "conv_simt.cu", "conv_dgrad": "conv_simt.cu", "conv_wgrad": "conv_simt.cu",
            "conv_fwd_tc": "conv_tc.cu", "conv_dgrad_tc": "conv_tc.cu",
-           "conv_wgrad_tc": "conv_tc.cu", "sgd": "optim.cu", "fuse": "optim.cu"}.get(kind)
+           "conv_wgrad_tc": "conv_tc.cu", "relu_pool_bwd": "conv_simt.cu",
+           "sgd": "optim.cu", "fuse": "optim.cu"}.get(base)
     if not src:
         return None
     p = os.path.join(ROOT, "paper_2609_29395_gb300", "csrc", src)

@@ -353,6 +353,14 @@ gcpsl_status check_device_error(gcpsl_ctx* c) {
   return GCPSL_OK;
 }
 
+// per-layer names of the tensor-core launches in the kernel timer
+const char* const kFwdTc[4] = {"conv_fwd_tc.L0", "conv_fwd_tc.L1", "conv_fwd_tc.L2",
+                               "conv_fwd_tc.L3"};
+const char* const kDgradTc[4] = {"conv_dgrad_tc.L0", "conv_dgrad_tc.L1", "conv_dgrad_tc.L2",
+                                 "conv_dgrad_tc.L3"};
+const char* const kWgradTc[4] = {"conv_wgrad_tc.L0", "conv_wgrad_tc.L1", "conv_wgrad_tc.L2",
+                                 "conv_wgrad_tc.L3"};
+
 template <typename T>
 gcpsl_status enqueue_round(gcpsl_ctx* c) {
   cudaStream_t s = c->stream;
@@ -383,13 +391,13 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
       const auto& L0 = c->tc0;
       ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 8, L0.hb, L0.bb, L0.tiles_h, a.conv[0].cout,
                    c->d_theta + a.off_b[0], P, (bf16*)(void*)act[1], c->d_code[0], c->d_err};
-      LAUNCH("conv_fwd_tc", launch_conv0_tc(s, L0.A, L0.B, p, a.conv[0].pool ? EPI_POOL : EPI_RELU,
+      LAUNCH(kFwdTc[0], launch_conv0_tc(s, L0.A, L0.B, p, a.conv[0].pool ? EPI_POOL : EPI_RELU,
                                             C));
     } else if (L.on) {
       ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.hb, L.bb, L.tiles_h,
                    a.conv[i].cout, c->d_theta + a.off_b[i], P, (bf16*)(void*)act[i + 1],
                    c->d_code[i], c->d_err};
-      LAUNCH("conv_fwd_tc", launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f,
+      LAUNCH(kFwdTc[i], launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f,
                                            a.conv[i].pool ? EPI_POOL : EPI_RELU, C));
     } else {
       LAUNCH("conv_fwd", launch_conv_fwd_simt<T>(s, act[i], wts + a.off_w[i], P,
@@ -414,7 +422,7 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
     if (L.on) {
       WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
                     L.splits, c->d_partial, c->d_err};
-      LAUNCH("conv_wgrad_tc", launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
+      LAUNCH(kWgradTc[i], launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
       LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
                                                  L.splits, (int64_t)cs.cout * 9 * cs.cin, C));
       LAUNCH("bias_partial", launch_bias_partial<T>(s, g, c->d_bpartial, C, B, cs, R.chunks,
@@ -434,7 +442,7 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
     if (L.on) {
       ConvTcArgs p{cs.h, cs.w, B, cs.cout, L.hb, L.bb, L.tiles_h, cs.cin, nullptr, 0,
                    (bf16*)(void*)dact[i], nullptr, c->d_err};
-      LAUNCH("conv_dgrad_tc", launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d, EPI_STORE, C));
+      LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d, EPI_STORE, C));
     } else {
       LAUNCH("conv_dgrad", launch_conv_dgrad_simt<T>(s, g, wts + a.off_w[i], P, dact[i], C, B,
                                                      cs));
