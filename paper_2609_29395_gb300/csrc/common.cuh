@@ -117,8 +117,8 @@ enum { EPI_POOL = 0, EPI_RELU = 1, EPI_STORE = 2 };
 struct ConvTcArgs {
   int H, W, B;          // spatial size and batch per replica
   int kch;              // channels of the activation operand (multiple of the stage width)
-  int hb, bb;           // image rows / images per 128-pixel M tile (W * hb * bb == 128)
-  int tiles_h;          // H / hb
+  int bw, hb, bb;       // M tile of 128 pixels: bw columns x hb rows x bb images
+  int tiles_w, tiles_h; // W / bw, H / hb
   int n_total;          // output channels (row length of `out`)
   const float* bias;    // fp32 bias of replica 0 (EPI_POOL / EPI_RELU)
   int64_t bias_rs;      // replica stride of the bias

@@ -47,116 +47,133 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return (uint8_t*)(((uintptr_t)p + 1023) & ~(uintptr_t)1023);
 }
 
-__device__ __forceinline__ void epi_bar() {   // the four epilogue warps only
-  asm volatile("bar.sync 1, 128;" ::: "memory");
-}
-
-// Epilogue of a 128-pixel x BN-channel accumulator tile (run by the four
-// epilogue warps; thread `te` in [0,128) reads TMEM row `r` at `trow`).
-//  EPI_POOL : + bias, 2x2 max-pool of relu (first maximum, decided on fp32),
-//             via a [128][BN+1] fp32 staging tile in shared memory `sm`;
-//  EPI_RELU : + bias, relu;   EPI_STORE: plain store.
+// Epilogue of a 128-pixel x BN-channel accumulator tile, run by the four
+// epilogue warps; the thread of TMEM row r owns pixel (bb, hh, ww) of the
+// tile (r = (bb*hb + hh)*bw + ww, tiles are bw <= 16 pixels wide, so a warp
+// holds whole 2x2 windows: partners at lane^1 and lane^bw).
+//  EPI_POOL : + bias; 2x2 max-pool decided on the fp32 values (the larger
+//             value wins, ties go to the earlier position in row-major
+//             order, i.e. the first maximum); the window's top-left thread
+//             stores relu(max) in bf16 and the code (position | positive<<2).
+//  EPI_RELU : + bias, relu, bf16 store;   EPI_STORE: bf16 store.
+// 16 channels per TMEM load; stores are 16-byte vectors.
 template <int BN, int EPI>
-__device__ __forceinline__ void conv_epilogue(uint8_t* sm, uint32_t trow, int r, int te, int n0,
-                                              int b0, int h0, int c, const ConvTcArgs& p) {
-  const int W = p.W, H = p.H;
+__device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0, int b0, int h0,
+                                                    int w0, int c, const ConvTcArgs& p) {
+  const int W = p.W, H = p.H, bw = p.bw;
+  const int ww = r % bw, hh = (r / bw) % p.hb, bb = r / (bw * p.hb);
+  const bool valid = b0 + bb < p.B;
+  const float* bias = EPI != EPI_STORE ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
+  int64_t o;
+  bool owner = valid;
   if (EPI == EPI_POOL) {
-    float* st = reinterpret_cast<float*>(sm);
-    const float* bias = p.bias + (int64_t)c * p.bias_rs + n0;
-#pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      float v[16];
-      tmem_ld16(trow + c0, v);
-      tmem_ld_wait();
-#pragma unroll
-      for (int i = 0; i < 16; ++i) st[r * (BN + 1) + c0 + i] = v[i] + bias[c0 + i];
-    }
-    epi_bar();
-    const int Wo = W / 2, hbo = p.hb / 2, Ho = H / 2;
-#pragma unroll 1
-    for (int idx = te; idx < 32 * BN; idx += 128) {
-      const int pp = idx / BN, co = idx % BN;
-      const int pw = pp % Wo, ph = (pp / Wo) % hbo, bb = pp / (Wo * hbo);
-      if (b0 + bb >= p.B) continue;
-      const int r00 = (bb * p.hb + 2 * ph) * W + 2 * pw;
-      const float* s0 = st + r00 * (BN + 1) + co;
-      float best = s0[0];
-      int arg = 0;
-      const float v1 = s0[BN + 1], v2 = s0[W * (BN + 1)], v3 = s0[(W + 1) * (BN + 1)];
-      if (v1 > best) { best = v1; arg = 1; }
-      if (v2 > best) { best = v2; arg = 2; }
-      if (v3 > best) { best = v3; arg = 3; }
-      const int64_t o =
-          ((((int64_t)c * p.B + b0 + bb) * Ho + h0 / 2 + ph) * Wo + pw) * p.n_total + n0 + co;
-      p.out[o] = __float2bfloat16_rn(best > 0.f ? best : 0.f);
-      p.code[o] = (uint8_t)(arg | (best > 0.f ? 4 : 0));
-    }
+    o = ((((int64_t)c * p.B + b0 + bb) * (H / 2) + (h0 + hh) / 2) * (W / 2) + (w0 + ww) / 2) *
+            p.n_total + n0;
+    owner = valid && !(hh & 1) && !(ww & 1);
   } else {
-    const int w = r % W, hh = (r / W) % p.hb, bb = r / (W * p.hb);
-    const bool valid = b0 + bb < p.B;
-    const int64_t o = ((((int64_t)c * p.B + b0 + bb) * H + h0 + hh) * W + w) * p.n_total + n0;
-    const float* bias = EPI == EPI_RELU ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
+    o = ((((int64_t)c * p.B + b0 + bb) * H + h0 + hh) * W + w0 + ww) * p.n_total + n0;
+  }
+  const int mypos = (hh & 1) * 2 + (ww & 1);
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      float v[16];
-      tmem_ld16(trow + c0, v);
-      tmem_ld_wait();
-      if (!valid) continue;
-      __align__(16) bf16 h[16];
+  for (int c0 = 0; c0 < BN; c0 += 16) {
+    float v[16];
+    tmem_ld16(trow + c0, v);
+    tmem_ld_wait();
+    __align__(16) bf16 h[16];
+    if (EPI == EPI_POOL) {
+      __align__(16) uint8_t code[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        float val = v[i] + bias[c0 + i];
+        int pos = mypos;
+#pragma unroll
+        for (int step = 0; step < 2; ++step) {
+          const int x = step == 0 ? 1 : bw;
+          const float pv = __shfl_xor_sync(0xffffffffu, val, x);
+          const int pp = __shfl_xor_sync(0xffffffffu, pos, x);
+          if (pv > val || (pv == val && pp < pos)) { val = pv; pos = pp; }
+        }
+        h[i] = __float2bfloat16_rn(val > 0.f ? val : 0.f);
+        code[i] = (uint8_t)(pos | (val > 0.f ? 4 : 0));
+      }
+      if (owner) {
+        uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
+        dst[0] = reinterpret_cast<uint4*>(h)[0];
+        dst[1] = reinterpret_cast<uint4*>(h)[1];
+        *reinterpret_cast<uint4*>(p.code + o + c0) = *reinterpret_cast<uint4*>(code);
+      }
+    } else {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         float x = v[i];
         if (EPI == EPI_RELU) { x += bias[c0 + i]; x = x > 0.f ? x : 0.f; }
         h[i] = __float2bfloat16_rn(x);
       }
-      uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
-      dst[0] = reinterpret_cast<uint4*>(h)[0];
-      dst[1] = reinterpret_cast<uint4*>(h)[1];
+      if (owner) {
+        uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
+        dst[0] = reinterpret_cast<uint4*>(h)[0];
+        dst[1] = reinterpret_cast<uint4*>(h)[1];
+      }
     }
   }
 }
 
-template <int BN, int BKC>
+template <int BN, int BKC, int EPI>
 struct ConvCfg {
   static constexpr int A_BYTES = BM * BKC * 2;
   static constexpr int B_BYTES = BN * BKC * 2;
   static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int S = STAGE >= 24576 ? 3 : (STAGE >= 12288 ? 4 : 6);
-  static constexpr int PIPE = S * STAGE;
-  static constexpr int STAGING = BM * (BN + 1) * 4;      // pooled epilogue
-  static constexpr int SMEM = 1024 + (PIPE > STAGING ? PIPE : STAGING);
   static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  // two CTAs per SM when both fit in TMEM (2 x 2 x TCOLS <= 512 columns)
+  static constexpr int CTAS = 2 * TCOLS <= 256 ? 2 : 1;
+  static constexpr int BUDGET = CTAS == 2 ? 100 * 1024 : 200 * 1024;
+  static constexpr int S0 = BUDGET / STAGE;
+  static constexpr int S = S0 > 8 ? 8 : (S0 < 2 ? 2 : S0);
+  static constexpr int PIPE = S * STAGE;
+  static constexpr int SMEM = 1024 + PIPE;
 };
 
+// (b0, h0, w0) of M tile mt
+__device__ __forceinline__ void tile_origin(int mt, const ConvTcArgs& p, int& b0, int& h0,
+                                            int& w0) {
+  const int wt = mt % p.tiles_w, ht = (mt / p.tiles_w) % p.tiles_h, bt = mt / (p.tiles_w * p.tiles_h);
+  b0 = bt * p.bb;
+  h0 = ht * p.hb;
+  w0 = wt * p.bw;
+}
+
+// Persistent implicit-GEMM convolution.  CTA b takes work items b, b + G,
+// ... of the (replica, M tile, N tile) list (N fastest).  The TMA warp runs
+// ahead through an S-stage ring across item boundaries; the MMA warp
+// alternates between two TMEM accumulators (2 x TCOLS columns), so the
+// epilogue of one item overlaps the MMAs of the next: tfull[b] (MMA ->
+// epilogue) and tempty[b] (epilogue -> MMA, 128 arrivals) hand a buffer over.
 // BMN = 0: B tile is K-major [n][tap][k] (fprop: W[co][tap][ci]).
 // BMN = 1: B tile is read MN-major from W[co][tap][ci] itself (dgrad: n = ci,
 //   k = co, tap flipped), as 64-wide (or one 32-wide) N blocks of BKC rows.
 template <int BN, int BKC, int EPI, int BMN>
 __global__ void __launch_bounds__(kThreads, 1)
 k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
-          const ConvTcArgs p) {
-  using Cfg = ConvCfg<BN, BKC>;
+          const ConvTcArgs p, int tiles_m, int tiles_n, int items) {
+  using Cfg = ConvCfg<BN, BKC, EPI>;
   constexpr int S = Cfg::S;
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = align1024(smraw);
-  __shared__ uint64_t full[S], empty[S], done;
+  __shared__ uint64_t full[S], empty[S], tfull[2], tempty[2];
   __shared__ uint32_t tbase;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = blockIdx.x, c = blockIdx.z;
-  const int n0 = blockIdx.y * BN;
-  const int b0 = (mt / p.tiles_h) * p.bb, h0 = (mt % p.tiles_h) * p.hb;
   const int kper = p.kch / BKC;
   const int KB = 9 * kper;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    mbar_init(&done, 1);
+    for (int b = 0; b < 2; ++b) { mbar_init(&tfull[b], 1); mbar_init(&tempty[b], 128); }
     fence_mbar_init();
     tma_prefetch_desc(&tA);
     tma_prefetch_desc(&tB);
   }
-  if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
+  if (warp == 1) { tmem_alloc(&tbase, 2 * Cfg::TCOLS); tmem_relinquish(); }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -164,21 +181,33 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
 
   if (warp == 0) {
     if (elect_one()) {
-      for (int kb = 0; kb < KB; ++kb) {
-        const int s = kb % S;
-        if (kb >= S && !mbar_wait(&empty[s], ((kb / S) & 1) ^ 1)) { atomicOr(p.err, 1); break; }
-        uint8_t* sa = sm + s * Cfg::STAGE;
-        const int tap = kb / kper, ch = (kb % kper) * BKC;
-        mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
-        tma_load_5d(sa, &tA, &full[s], ch, tap % 3 - 1, h0 + tap / 3 - 1, b0, c);
-        if (!BMN) {
-          tma_load_4d(sa + Cfg::A_BYTES, &tB, &full[s], ch, tap, n0, c);
-        } else {
-          constexpr int NBW = BN < 64 ? BN : 64;           // N block width
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < items && ok; t += gridDim.x) {
+        const int c = t / (tiles_m * tiles_n), r = t % (tiles_m * tiles_n);
+        const int mt = r / tiles_n, n0 = (r % tiles_n) * BN;
+        int b0, h0, w0;
+        tile_origin(mt, p, b0, h0, w0);
+        for (int kb = 0; kb < KB; ++kb, ++it) {
+          const int s = it % S;
+          if (it >= S && !mbar_wait(&empty[s], ((it / S) & 1) ^ 1)) {
+            atomicOr(p.err, 1);
+            ok = false;
+            break;
+          }
+          uint8_t* sa = sm + s * Cfg::STAGE;
+          const int tap = kb / kper, ch = (kb % kper) * BKC;
+          mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
+          tma_load_5d(sa, &tA, &full[s], ch, w0 + tap % 3 - 1, h0 + tap / 3 - 1, b0, c);
+          if (!BMN) {
+            tma_load_4d(sa + Cfg::A_BYTES, &tB, &full[s], ch, tap, n0, c);
+          } else {
+            constexpr int NBW = BN < 64 ? BN : 64;           // N block width
 #pragma unroll
-          for (int j = 0; j < BN / NBW; ++j)
-            tma_load_4d(sa + Cfg::A_BYTES + j * NBW * BKC * 2, &tB, &full[s], n0 + j * NBW,
-                        8 - tap, ch, c);
+            for (int j = 0; j < BN / NBW; ++j)
+              tma_load_4d(sa + Cfg::A_BYTES + j * NBW * BKC * 2, &tB, &full[s], n0 + j * NBW,
+                          8 - tap, ch, c);
+          }
         }
       }
     }
@@ -191,32 +220,62 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
       constexpr int NBW = BN < 64 ? BN : 64;
       constexpr uint32_t b_row = NBW * 2;
       constexpr uint32_t b_swz = NBW == 64 ? SWZ_128 : SWZ_64;
-      for (int kb = 0; kb < KB; ++kb) {
-        const int s = kb % S;
-        if (!mbar_wait(&full[s], (kb / S) & 1)) { atomicOr(p.err, 2); break; }
-        tc_fence_after();
-        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
-#pragma unroll
-        for (int k = 0; k < BKC / 16; ++k) {
-          const uint64_t bd = BMN ? smem_desc(b + k * 16 * b_row, NBW * BKC * 2, 8 * b_row, b_swz)
-                                  : smem_desc(b + k * 32, 16, sbo, swz);
-          mma_f16(tmem, smem_desc(a + k * 32, 16, sbo, swz), bd, idesc, (kb | k) != 0);
+      int it = 0, tl = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < items && ok; t += gridDim.x, ++tl) {
+        const int buf = tl & 1;
+        if (tl >= 2 && !mbar_wait(&tempty[buf], ((tl >> 1) & 1) ^ 1)) {
+          atomicOr(p.err, 2);
+          break;
         }
-        mma_commit(&empty[s]);
+        tc_fence_after();
+        const uint32_t d = tmem + buf * Cfg::TCOLS;
+        for (int kb = 0; kb < KB; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait(&full[s], (it / S) & 1)) {
+            atomicOr(p.err, 2);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BKC / 16; ++k) {
+            const uint64_t bd = BMN ? smem_desc(b + k * 16 * b_row, NBW * BKC * 2, 8 * b_row, b_swz)
+                                    : smem_desc(b + k * 32, 16, sbo, swz);
+            mma_f16(d, smem_desc(a + k * 32, 16, sbo, swz), bd, idesc, (kb | k) != 0);
+          }
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&tfull[buf]);
       }
-      mma_commit(&done);
     }
   } else {
     // ---------------- epilogue: warps 2..5 ----------------
     const int q = warp & 3;                     // TMEM lane quarter of this warp
-    if (!mbar_wait(&done, 0)) atomicOr(p.err, 4);
-    tc_fence_after();
-    conv_epilogue<BN, EPI>(sm, tmem + ((uint32_t)(q * 32) << 16), q * 32 + lane,
-                           threadIdx.x - 64, n0, b0, h0, c, p);
+    const int r = q * 32 + lane;                // M row = pixel of the tile
+    int tl = 0;
+    for (int t = blockIdx.x; t < items; t += gridDim.x, ++tl) {
+      const int buf = tl & 1;
+      // warp-uniform decision: the epilogue shuffles need the whole warp
+      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
+        if (lane == 0) atomicOr(p.err, 4);
+        break;
+      }
+      tc_fence_after();
+      const int c = t / (tiles_m * tiles_n), rr = t % (tiles_m * tiles_n);
+      const int mt = rr / tiles_n, n0 = (rr % tiles_n) * BN;
+      int b0, h0, w0;
+      tile_origin(mt, p, b0, h0, w0);
+      const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
+      conv_epilogue_drain<BN, EPI>(trow, r, n0, b0, h0, w0, c, p);
+      tc_fence_before();
+      mbar_arrive(&tempty[buf]);
+    }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
+  if (warp == 1) tmem_dealloc(tmem, 2 * Cfg::TCOLS);
 }
 
 // ---------------------------------------------------------------------------
@@ -227,73 +286,106 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
 // byte offset, so tap t's 128 x 16 B box and tap t+1's box can sit 2 KB apart.
 // Ten tap slots are loaded (slot 9 repeats tap 8); the packed weights
 // [tap][co][8] have zeros for tap 9 and for channels >= cin.
-template <int BN>
+template <int BN, int EPI>
 struct Conv0Cfg {
   static constexpr int SLOT_A = BM * 16;                 // one tap: 128 px x 8 ch
   static constexpr int A_BYTES = 10 * SLOT_A;
   static constexpr int B_BYTES = 10 * BN * 16;
-  static constexpr int STAGING = BM * (BN + 1) * 4;
-  static constexpr int SMEM = 1024 + (A_BYTES + B_BYTES > STAGING ? A_BYTES + B_BYTES : STAGING);
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int S = 3;
+  static constexpr int PIPE = S * STAGE;
+  static constexpr int SMEM = 1024 + PIPE;
   static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static constexpr int CTAS = 2;                          // 2 x 2 x TCOLS <= 512 for BN <= 64
 };
 
+// Persistent like k_conv_tc: one ring stage holds one work item (ten tap
+// slots and the packed weights), two TMEM accumulators alternate.
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
 k_conv0_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
-           const ConvTcArgs p) {
-  using Cfg = Conv0Cfg<BN>;
+           const ConvTcArgs p, int tiles_m, int items) {
+  using Cfg = Conv0Cfg<BN, EPI>;
+  constexpr int S = Cfg::S;
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = align1024(smraw);
-  __shared__ uint64_t full, done;
+  __shared__ uint64_t full[S], empty[S], tfull[2], tempty[2];
   __shared__ uint32_t tbase;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = blockIdx.x, c = blockIdx.z;
-  const int b0 = (mt / p.tiles_h) * p.bb, h0 = (mt % p.tiles_h) * p.hb;
   if (threadIdx.x == 0) {
-    mbar_init(&full, 1);
-    mbar_init(&done, 1);
+    for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int b = 0; b < 2; ++b) { mbar_init(&tfull[b], 1); mbar_init(&tempty[b], 128); }
     fence_mbar_init();
   }
-  if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
+  if (warp == 1) { tmem_alloc(&tbase, 2 * Cfg::TCOLS); tmem_relinquish(); }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tbase;
   if (warp == 0) {
     if (elect_one()) {
-      mbar_arrive_expect_tx(&full, Cfg::A_BYTES + Cfg::B_BYTES);
+      int it = 0;
+      for (int t = blockIdx.x; t < items; t += gridDim.x, ++it) {
+        const int c = t / tiles_m, mt = t % tiles_m;
+        int b0, h0, w0;
+        tile_origin(mt, p, b0, h0, w0);
+        const int s = it % S;
+        if (it >= S && !mbar_wait(&empty[s], ((it / S) & 1) ^ 1)) { atomicOr(p.err, 64); break; }
+        uint8_t* st = sm + s * Cfg::STAGE;
+        mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
 #pragma unroll
-      for (int j = 0; j < 10; ++j) {
-        const int tap = j < 9 ? j : 8;
-        tma_load_5d(sm + j * Cfg::SLOT_A, &tA, &full, 0, tap % 3 - 1, h0 + tap / 3 - 1, b0, c);
+        for (int j = 0; j < 10; ++j) {
+          const int tap = j < 9 ? j : 8;
+          tma_load_5d(st + j * Cfg::SLOT_A, &tA, &full[s], 0, w0 + tap % 3 - 1, h0 + tap / 3 - 1,
+                      b0, c);
+        }
+        tma_load_4d(st + Cfg::A_BYTES, &tB, &full[s], 0, 0, 0, c);
       }
-      tma_load_4d(sm + Cfg::A_BYTES, &tB, &full, 0, 0, 0, c);
     }
   } else if (warp == 1) {
     if (elect_one()) {
-      if (mbar_wait(&full, 0)) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
+      int tl = 0;
+      for (int t = blockIdx.x; t < items; t += gridDim.x, ++tl) {
+        const int buf = tl & 1, s = tl % S;
+        if (tl >= 2 && !mbar_wait(&tempty[buf], ((tl >> 1) & 1) ^ 1)) {
+          atomicOr(p.err, 64);
+          break;
+        }
+        if (!mbar_wait(&full[s], (tl / S) & 1)) { atomicOr(p.err, 64); break; }
         tc_fence_after();
-        constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
-        const uint32_t a = smem_u32(sm), b = a + Cfg::A_BYTES;
+        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
+        const uint32_t d = tmem + buf * Cfg::TCOLS;
 #pragma unroll
         for (int k = 0; k < 5; ++k)
-          mma_f16(tmem, smem_desc(a + 2 * k * Cfg::SLOT_A, Cfg::SLOT_A, 128, SWZ_NONE),
+          mma_f16(d, smem_desc(a + 2 * k * Cfg::SLOT_A, Cfg::SLOT_A, 128, SWZ_NONE),
                   smem_desc(b + 2 * k * BN * 16, BN * 16, 128, SWZ_NONE), idesc, k != 0);
-      } else {
-        atomicOr(p.err, 64);
+        mma_commit(&empty[s]);
+        mma_commit(&tfull[buf]);
       }
-      mma_commit(&done);
     }
   } else {
-    const int q = warp & 3;
-    if (!mbar_wait(&done, 0)) atomicOr(p.err, 128);
-    tc_fence_after();
-    conv_epilogue<BN, EPI>(sm, tmem + ((uint32_t)(q * 32) << 16), q * 32 + lane,
-                           threadIdx.x - 64, 0, b0, h0, c, p);
+    const int q = warp & 3, r = q * 32 + lane;
+    int tl = 0;
+    for (int t = blockIdx.x; t < items; t += gridDim.x, ++tl) {
+      const int buf = tl & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
+        if (lane == 0) atomicOr(p.err, 128);
+        break;
+      }
+      tc_fence_after();
+      const int c = t / tiles_m, mt = t % tiles_m;
+      int b0, h0, w0;
+      tile_origin(mt, p, b0, h0, w0);
+      const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
+      conv_epilogue_drain<BN, EPI>(trow, r, 0, b0, h0, w0, c, p);
+      tc_fence_before();
+      mbar_arrive(&tempty[buf]);
+    }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
+  if (warp == 1) tmem_dealloc(tmem, 2 * Cfg::TCOLS);
 }
 
 // packed input-layer weights: w0p[c][tap][co][8] = W[co][tap][ci] for
@@ -464,10 +556,22 @@ k_wgrad_reduce(const float* __restrict__ partial, float* __restrict__ dw, int64_
   }
 }
 
+// SMs of the current device (persistent grids use one CTA per SM)
+int sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+  }
+  return n;
+}
+
 template <int BN, int BKC, int EPI, int BMN>
 cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                             const ConvTcArgs& p, dim3 grid) {
-  using Cfg = ConvCfg<BN, BKC>;
+                             const ConvTcArgs& p, int tiles_m, int tiles_n, int items) {
+  using Cfg = ConvCfg<BN, BKC, EPI>;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_conv_tc<BN, BKC, EPI, BMN>,
@@ -475,7 +579,10 @@ cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k_conv_tc<BN, BKC, EPI, BMN><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p);
+  const int cap = sm_count() * Cfg::CTAS;
+  const int grid = items < cap ? items : cap;
+  k_conv_tc<BN, BKC, EPI, BMN><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p, tiles_m, tiles_n,
+                                                                  items);
   return cudaGetLastError();
 }
 
@@ -569,13 +676,14 @@ bool tensor_map_bf16_strided(CUtensorMap* m, const void* base, int rank, const u
 // ---------------------------------------------------------------------------
 cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
                            const ConvTcArgs& p, int bn, int bkc, int epi, int C) {
-  const int tiles_m = p.tiles_h * ((p.B + p.bb - 1) / p.bb);
-  dim3 grid(tiles_m, p.n_total / bn, C);
+  const int tiles_m = p.tiles_w * p.tiles_h * ((p.B + p.bb - 1) / p.bb);
+  const int tiles_n = p.n_total / bn;
+  const int items = tiles_m * tiles_n * C;
   // fprop epilogues read a K-major B; the data gradient (EPI_STORE) reads
   // the same weights MN-major
 #define GCPSL_CONV_CASE(BN_, BKC_, EPI_, BMN_)             \
   if (bn == BN_ && bkc == BKC_ && epi == EPI_)             \
-    return launch_conv_inst<BN_, BKC_, EPI_, BMN_>(s, a, b, p, grid);
+    return launch_conv_inst<BN_, BKC_, EPI_, BMN_>(s, a, b, p, tiles_m, tiles_n, items);
 #define GCPSL_CONV_EPIS(BN_, BKC_)          \
   GCPSL_CONV_CASE(BN_, BKC_, EPI_POOL, 0)   \
   GCPSL_CONV_CASE(BN_, BKC_, EPI_RELU, 0)   \
@@ -585,7 +693,8 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
   GCPSL_CONV_EPIS(64, 64)
   GCPSL_CONV_EPIS(128, 32)
   GCPSL_CONV_EPIS(128, 64)
-  GCPSL_CONV_EPIS(256, 64)
+  GCPSL_CONV_CASE(256, 64, EPI_RELU, 0)     // no staging tile for 256 channels
+  GCPSL_CONV_CASE(256, 64, EPI_STORE, 1)
 #undef GCPSL_CONV_EPIS
 #undef GCPSL_CONV_CASE
   return cudaErrorInvalidValue;
@@ -593,8 +702,8 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
 
 template <int BN, int EPI>
 static cudaError_t launch_conv0_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                                     const ConvTcArgs& p, dim3 grid) {
-  using Cfg = Conv0Cfg<BN>;
+                                     const ConvTcArgs& p, int tiles_m, int items) {
+  using Cfg = Conv0Cfg<BN, EPI>;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_conv0_tc<BN, EPI>,
@@ -602,21 +711,26 @@ static cudaError_t launch_conv0_inst(cudaStream_t s, const CUtensorMap& a, const
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k_conv0_tc<BN, EPI><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p);
+  const int cap = sm_count() * Cfg::CTAS;
+  const int grid = items < cap ? items : cap;
+  k_conv0_tc<BN, EPI><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p, tiles_m, items);
   return cudaGetLastError();
 }
 
 cudaError_t launch_conv0_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
                             const ConvTcArgs& p, int epi, int C) {
-  const int tiles_m = p.tiles_h * ((p.B + p.bb - 1) / p.bb);
-  dim3 grid(tiles_m, 1, C);
+  const int tiles_m = p.tiles_w * p.tiles_h * ((p.B + p.bb - 1) / p.bb);
+  const int items = tiles_m * C;
   const int bn = p.n_total;
-  if (bn == 16 && epi == EPI_POOL) return launch_conv0_inst<16, EPI_POOL>(s, a, b, p, grid);
-  if (bn == 16 && epi == EPI_RELU) return launch_conv0_inst<16, EPI_RELU>(s, a, b, p, grid);
-  if (bn == 32 && epi == EPI_POOL) return launch_conv0_inst<32, EPI_POOL>(s, a, b, p, grid);
-  if (bn == 32 && epi == EPI_RELU) return launch_conv0_inst<32, EPI_RELU>(s, a, b, p, grid);
-  if (bn == 64 && epi == EPI_POOL) return launch_conv0_inst<64, EPI_POOL>(s, a, b, p, grid);
-  if (bn == 64 && epi == EPI_RELU) return launch_conv0_inst<64, EPI_RELU>(s, a, b, p, grid);
+#define GCPSL_CONV0_CASE(BN_, EPI_) \
+  if (bn == BN_ && epi == EPI_) return launch_conv0_inst<BN_, EPI_>(s, a, b, p, tiles_m, items);
+  GCPSL_CONV0_CASE(16, EPI_POOL)
+  GCPSL_CONV0_CASE(16, EPI_RELU)
+  GCPSL_CONV0_CASE(32, EPI_POOL)
+  GCPSL_CONV0_CASE(32, EPI_RELU)
+  GCPSL_CONV0_CASE(64, EPI_POOL)
+  GCPSL_CONV0_CASE(64, EPI_RELU)
+#undef GCPSL_CONV0_CASE
   return cudaErrorInvalidValue;
 }
 

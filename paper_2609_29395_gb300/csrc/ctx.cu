@@ -153,7 +153,7 @@ struct gcpsl_ctx {
   // tensor-core layers (bf16 mode): tile shapes and TMA descriptors
   struct TcLayer {
     bool on = false;
-    int hb, bb, tiles_h;           // 128-pixel M tile
+    int bw, hb, bb, tiles_w, tiles_h;   // 128-pixel M tile
     int whb, wbb;                  // 64-pixel K block of the weight gradient
     int bn_f, bkc_f, bn_d, bkc_d, bn_w;
     int splits, kb_total, kb_per_split;
@@ -163,7 +163,7 @@ struct gcpsl_ctx {
   // padded to x0c = 8 channels; packed weights [C][10][cout][8]
   struct Tc0Layer {
     bool on = false;
-    int hb, bb, tiles_h;
+    int bw, hb, bb, tiles_w, tiles_h;
     CUtensorMap A, B;
   } tc0;
   int x0c = 3;
@@ -389,14 +389,15 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
     const auto& L = c->tc[i];
     if (i == 0 && c->tc0.on) {
       const auto& L0 = c->tc0;
-      ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 8, L0.hb, L0.bb, L0.tiles_h, a.conv[0].cout,
-                   c->d_theta + a.off_b[0], P, (bf16*)(void*)act[1], c->d_code[0], c->d_err};
+      ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 8, L0.bw, L0.hb, L0.bb, L0.tiles_w, L0.tiles_h,
+                   a.conv[0].cout, c->d_theta + a.off_b[0], P, (bf16*)(void*)act[1],
+                   c->d_code[0], c->d_err};
       LAUNCH(kFwdTc[0], launch_conv0_tc(s, L0.A, L0.B, p, a.conv[0].pool ? EPI_POOL : EPI_RELU,
                                             C));
     } else if (L.on) {
-      ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.hb, L.bb, L.tiles_h,
-                   a.conv[i].cout, c->d_theta + a.off_b[i], P, (bf16*)(void*)act[i + 1],
-                   c->d_code[i], c->d_err};
+      ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.bw, L.hb, L.bb, L.tiles_w,
+                   L.tiles_h, a.conv[i].cout, c->d_theta + a.off_b[i], P,
+                   (bf16*)(void*)act[i + 1], c->d_code[i], c->d_err};
       LAUNCH(kFwdTc[i], launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f,
                                            a.conv[i].pool ? EPI_POOL : EPI_RELU, C));
     } else {
@@ -440,8 +441,8 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
     }
     if (i == 0) continue;
     if (L.on) {
-      ConvTcArgs p{cs.h, cs.w, B, cs.cout, L.hb, L.bb, L.tiles_h, cs.cin, nullptr, 0,
-                   (bf16*)(void*)dact[i], nullptr, c->d_err};
+      ConvTcArgs p{cs.h, cs.w, B, cs.cout, L.bw, L.hb, L.bb, L.tiles_w, L.tiles_h, cs.cin,
+                   nullptr, 0, (bf16*)(void*)dact[i], nullptr, c->d_err};
       LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d, EPI_STORE, C));
     } else {
       LAUNCH("conv_dgrad", launch_conv_dgrad_simt<T>(s, g, wts + a.off_w[i], P, dact[i], C, B,
@@ -460,6 +461,16 @@ gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
   return refresh_derived(c);
 }
 
+// 128-pixel M tile of a W x H image: bw <= 16 columns (so a warp holds whole
+// 2x2 pooling windows), hb rows, bb images
+bool m_tile(int W, int H, int& bw, int& hb, int& bb) {
+  bw = std::min(W, 16);
+  if (bw < 2 || W % bw || 128 % bw) return false;
+  hb = std::min(H, 128 / bw);
+  bb = 128 / (bw * hb);
+  return bw * hb * bb == 128 && H % hb == 0 && hb % 2 == 0;
+}
+
 // Tile shapes, split-K factors and TMA descriptors of every layer that runs on
 // the tensor cores: 3x3 layers with 32k input and 64k output channels and
 // rows of at most 64 pixels.  Layers outside that shape (the 3-channel input
@@ -474,12 +485,11 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     L.on = false;
     if (s.cin < 32 || s.cin % 32 || s.cout % 64 || s.w > 64 || 64 % s.w || a.off_w[i] % 8)
       continue;
-    L.hb = std::min(s.h, 128 / s.w);
-    L.bb = 128 / (s.w * L.hb);
+    if (!m_tile(s.w, s.h, L.bw, L.hb, L.bb)) continue;
     L.whb = std::min(s.h, 64 / s.w);
     L.wbb = 64 / (s.w * L.whb);
-    if (s.w * L.hb * L.bb != 128 || s.h % L.hb || s.w * L.whb * L.wbb != 64 || s.h % L.whb)
-      continue;
+    if (s.w * L.whb * L.wbb != 64 || s.h % L.whb) continue;
+    L.tiles_w = s.w / L.bw;
     L.tiles_h = s.h / L.hb;
     L.bn_f = std::min(s.cout, 256);
     L.bkc_f = std::min(s.cin, 64);
@@ -504,9 +514,9 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
                                 (uint64_t)C};
     const uint64_t wf[4] = {(uint64_t)s.cin, 9, (uint64_t)s.cout, (uint64_t)C};
     const uint64_t rs = (uint64_t)c->P_pad * 2;
-    const uint32_t bA[5] = {(uint32_t)L.bkc_f, (uint32_t)s.w, (uint32_t)L.hb, (uint32_t)L.bb, 1};
+    const uint32_t bA[5] = {(uint32_t)L.bkc_f, (uint32_t)L.bw, (uint32_t)L.hb, (uint32_t)L.bb, 1};
     const uint32_t bB[4] = {(uint32_t)L.bkc_f, 1, (uint32_t)L.bn_f, 1};
-    const uint32_t dA[5] = {(uint32_t)L.bkc_d, (uint32_t)s.w, (uint32_t)L.hb, (uint32_t)L.bb, 1};
+    const uint32_t dA[5] = {(uint32_t)L.bkc_d, (uint32_t)L.bw, (uint32_t)L.hb, (uint32_t)L.bb, 1};
     // data gradient: W[co][tap][ci] read MN-major, N blocks of <= 64 ci
     const int nbw = std::min(L.bn_d, 64);
     const uint32_t dB[4] = {(uint32_t)nbw, 1, (uint32_t)L.bkc_d, 1};
@@ -531,15 +541,14 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
   const ConvSpec& s0 = a.conv[0];
   auto& L0 = c->tc0;
   L0.on = false;
-  L0.hb = std::min(s0.h, 128 / s0.w);
-  L0.bb = 128 / (s0.w * std::max(1, L0.hb));
-  if (s0.cin > 8 || (s0.cout != 16 && s0.cout != 32 && s0.cout != 64) || s0.w > 128 ||
-      128 % s0.w || s0.w * L0.hb * L0.bb != 128 || s0.h % L0.hb)
+  if (s0.cin > 8 || (s0.cout != 16 && s0.cout != 32 && s0.cout != 64) ||
+      !m_tile(s0.w, s0.h, L0.bw, L0.hb, L0.bb))
     return fail(c, GCPSL_E_UNSUPPORTED, "input layer shape not supported with bf16 operands");
+  L0.tiles_w = s0.w / L0.bw;
   L0.tiles_h = s0.h / L0.hb;
   DALLOC(c->d_w0p, sizeof(bf16) * (size_t)C * 10 * s0.cout * 8);
   const uint64_t xdims[5] = {8, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B, (uint64_t)C};
-  const uint32_t xbox[5] = {8, (uint32_t)s0.w, (uint32_t)L0.hb, (uint32_t)L0.bb, 1};
+  const uint32_t xbox[5] = {8, (uint32_t)L0.bw, (uint32_t)L0.hb, (uint32_t)L0.bb, 1};
   const uint64_t wdims[4] = {8, (uint64_t)s0.cout, 10, (uint64_t)C};
   const uint32_t wbox[4] = {8, (uint32_t)s0.cout, 10, 1};
   if (!tensor_map_bf16(&L0.A, c->d_act[0], 5, xdims, xbox, 0) ||
