@@ -405,15 +405,23 @@ __global__ void k_pack_w0(const bf16* __restrict__ w, bf16* __restrict__ w0p, in
 // ---------------------------------------------------------------------------
 // weight gradient
 // ---------------------------------------------------------------------------
+// One CTA owns a group of up to TG = 256/BN slots of a (128-co, BN-ci) tile:
+// per K block the g tile is loaded once and multiplied, in one N <= 256 MMA,
+// against the group's tap-shifted x tiles (consecutive N blocks).  Group 0
+// holds taps 0..TG-2 and, in its last slot, a block of ones (written once
+// into every ring stage), so its accumulator also yields the bias gradient
+// sum_p g[p][co]; groups g >= 1 hold TG taps each.  The fp32 partial of a
+// split is laid out like the parameters, [cout][9][cin] then [cout].
 template <int BN>
 struct WgCfg {
   static constexpr int BKP = 64;                         // pixels per stage
+  static constexpr int TG = 256 / BN;                    // taps per CTA
   static constexpr int A_BYTES = 2 * 64 * BKP * 2;       // 128 co (two 64-wide blocks)
-  static constexpr int B_BYTES = BN * BKP * 2;
-  static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int S = STAGE >= 32768 ? 4 : 5;
+  static constexpr int TAP_BYTES = BN * BKP * 2;         // one tap's x tile
+  static constexpr int STAGE = A_BYTES + TG * TAP_BYTES;
+  static constexpr int S = 4;
   static constexpr int SMEM = 1024 + S * STAGE;
-  static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : 128;
+  static constexpr uint32_t TCOLS = 256;
 };
 
 template <int BN>
@@ -421,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tX,
            const WgradTcArgs p) {
   using Cfg = WgCfg<BN>;
-  constexpr int S = Cfg::S;
+  constexpr int S = Cfg::S, TG = Cfg::TG;
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = align1024(smraw);
   __shared__ uint64_t full[S], empty[S], done;
@@ -434,8 +442,12 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   int t = blockIdx.y;
   const int ci0 = (t % ci_tiles) * BN; t /= ci_tiles;
   const int co0 = (t % co_tiles) * 128; t /= co_tiles;
-  const int tap = t;                                 // 0..8
-  const int kh = tap / 3, kw = tap % 3;
+  const int grp = t;                                 // tap group
+  const bool bias_grp = grp == 0;
+  const int tap0 = bias_grp ? 0 : (TG - 1) + (grp - 1) * TG;
+  const int ntaps = bias_grp ? TG - 1 : (9 - tap0 < TG ? 9 - tap0 : TG);
+  const int nslots = bias_grp ? TG : ntaps;          // N = nslots * BN
+  const int per = p.cout * 9 * p.cin + p.cout;       // partial length per split
   const int kb_begin = split * p.kb_per_split;
   const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
   const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
@@ -447,6 +459,16 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     fence_mbar_init();
     tma_prefetch_desc(&tG);
     tma_prefetch_desc(&tX);
+  }
+  if (bias_grp) {
+    // the ones block (bf16 1.0 everywhere, so the swizzle does not matter)
+    const uint4 ones = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    for (int s = 0; s < S; ++s) {
+      uint4* dst = reinterpret_cast<uint4*>(sm + s * Cfg::STAGE + Cfg::A_BYTES +
+                                            (TG - 1) * Cfg::TAP_BYTES);
+      for (int i = threadIdx.x; i < Cfg::TAP_BYTES / 16; i += blockDim.x) dst[i] = ones;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
   tc_fence_before();
@@ -463,26 +485,31 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
         const int b = (kb / rows_blocks) * p.bb, h = (kb % rows_blocks) * p.hb;
         uint8_t* sa = sm + s * Cfg::STAGE;
         uint8_t* sb = sa + Cfg::A_BYTES;
-        mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
+        mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + ntaps * Cfg::TAP_BYTES);
         tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, c);
         // rows 64..127 of the M tile: the next 64 channels, or (cout <= 64) a
         // second copy of the first block whose results the epilogue drops
         tma_load_5d(sa + 64 * Cfg::BKP * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0, 0,
                     h, b, c);
+        for (int tj = 0; tj < ntaps; ++tj) {
+          const int tap = tap0 + tj, kh = tap / 3, kw = tap % 3;
 #pragma unroll
-        for (int j = 0; j < (BN + 63) / 64; ++j)
-          tma_load_5d(sb + j * 64 * Cfg::BKP * 2, &tX, &full[s], ci0 + 64 * j, kw - 1, h + kh - 1,
-                      b, c);
+          for (int j = 0; j < (BN + 63) / 64; ++j)
+            tma_load_5d(sb + tj * Cfg::TAP_BYTES + j * 64 * Cfg::BKP * 2, &tX, &full[s],
+                        ci0 + 64 * j, kw - 1, h + kh - 1, b, c);
+        }
       }
     }
   } else if (warp == 1) {
     if (elect_one()) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN, 1, 1);
-      // A: two 64-co blocks of BKP rows x 128 B; B: 64-ci blocks (SW128) or
-      // one 32-ci block of 64-byte rows (SW64)
+      // one MMA per k step with N = ntaps*BN: the taps' x tiles are the
+      // consecutive MN-major N blocks of one B operand (64-ci blocks, SW128,
+      // or 32-ci blocks of 64-byte rows, SW64), `b_blk` bytes apart
+      const uint32_t idesc = idesc_bf16(BM, nslots * BN, 1, 1);
       constexpr uint32_t a_lbo = 64 * Cfg::BKP * 2;
       constexpr uint32_t b_swz = BN >= 64 ? SWZ_128 : SWZ_64;
       constexpr uint32_t b_row = BN >= 64 ? 128 : 64;
+      constexpr uint32_t b_blk = b_row * Cfg::BKP;
       for (int i = 0; i < nkb; ++i) {
         const int s = i % S;
         if (!mbar_wait(&full[s], (i / S) & 1)) { atomicOr(p.err, 16); break; }
@@ -491,7 +518,7 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
 #pragma unroll
         for (int k = 0; k < Cfg::BKP / 16; ++k)
           mma_f16(tmem, smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128),
-                  smem_desc(b + k * 16 * b_row, a_lbo, 8 * b_row, b_swz), idesc, (i | k) != 0);
+                  smem_desc(b + k * 16 * b_row, b_blk, 8 * b_row, b_swz), idesc, (i | k) != 0);
         mma_commit(&empty[s]);
       }
       mma_commit(&done);
@@ -502,20 +529,28 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     const bool ok = mbar_wait(&done, 0);
     if (!ok) atomicOr(p.err, 32);
     tc_fence_after();
-    float* dst = p.partial + (((int64_t)c * p.splits + split) * p.cout + co) * 9 * p.cin +
-                 (int64_t)tap * p.cin + ci0;
     const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
-#pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
+    float* part = p.partial + ((int64_t)c * p.splits + split) * per;
+    if (bias_grp && ci0 == 0) {
       float v[16];
-      tmem_ld16(trow + c0, v);
+      tmem_ld16(trow + (TG - 1) * BN, v);
       tmem_ld_wait();
-      if (co < p.cout) {
-        float4* d4 = reinterpret_cast<float4*>(dst + c0);
+      if (co < p.cout) part[p.cout * 9 * p.cin + co] = nkb ? v[0] : 0.f;
+    }
+    for (int tj = 0; tj < ntaps; ++tj) {
+      float* dst = part + (int64_t)co * 9 * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        float v[16];
+        tmem_ld16(trow + tj * BN + c0, v);
+        tmem_ld_wait();
+        if (co < p.cout) {
+          float4* d4 = reinterpret_cast<float4*>(dst + c0);
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-          d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
-                      : make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int i = 0; i < 4; ++i)
+            d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
       }
     }
   }
@@ -743,7 +778,9 @@ cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs,
 
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C) {
-  const int tiles = 9 * (p.cin / bn) * ((p.cout + 127) / 128);
+  const int tg = 256 / bn;                            // slots per CTA
+  const int groups = 1 + (9 - (tg - 1) + tg - 1) / tg;
+  const int tiles = groups * (p.cin / bn) * ((p.cout + 127) / 128);
   dim3 grid(p.splits, tiles, C);
   if (bn == 32) return launch_wgrad_inst<32>(s, g, x, p, grid);
   if (bn == 64) return launch_wgrad_inst<64>(s, g, x, p, grid);

@@ -423,13 +423,11 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
     if (L.on) {
       WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
                     L.splits, c->d_partial, c->d_err};
+      // weights and bias together (the bias follows the weight in the store)
       LAUNCH(kWgradTc[i], launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
       LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
-                                                 L.splits, (int64_t)cs.cout * 9 * cs.cin, C));
-      LAUNCH("bias_partial", launch_bias_partial<T>(s, g, c->d_bpartial, C, B, cs, R.chunks,
-                                                    R.chunk_px));
-      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_bpartial, c->d_grad + a.off_b[i], P,
-                                                 R.chunks, cs.cout, C));
+                                                 L.splits,
+                                                 (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
     } else {
       // weights and bias together (the bias follows the weight in the store)
       LAUNCH("conv_wgrad", launch_wgrad_simt<T>(s, act[i], i == 0 ? c->x0c : cs.cin, g,
@@ -497,7 +495,9 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     L.bkc_d = std::min(s.cout, 64);
     L.bn_w = std::min(s.cin, 128);
     if (s.cout % L.bn_f || s.cin % L.bn_d || s.cin % L.bkc_f || s.cin % L.bn_w) continue;
-    const int tiles = 9 * (s.cin / L.bn_w) * ((s.cout + 127) / 128);
+    const int tg = 256 / L.bn_w;                      // slots per weight-gradient CTA
+    const int groups = 1 + (9 - (tg - 1) + tg - 1) / tg;
+    const int tiles = groups * (s.cin / L.bn_w) * ((s.cout + 127) / 128);
     L.kb_total = ((B + L.wbb - 1) / L.wbb) * (s.h / L.whb);
     // the split (hence the summation order) depends on the per-replica shape
     // only, so C grouped replicas reproduce C one-replica runs bit for bit
@@ -506,7 +506,8 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     splits = std::max(1, std::min(splits, (L.kb_total + 15) / 16));
     L.kb_per_split = (L.kb_total + splits - 1) / splits;
     L.splits = (L.kb_total + L.kb_per_split - 1) / L.kb_per_split;
-    partial_max = std::max(partial_max, (int64_t)C * L.splits * s.cout * 9 * s.cin);
+    partial_max = std::max(partial_max,
+                           (int64_t)C * L.splits * ((int64_t)s.cout * 9 * s.cin + s.cout));
 
     const uint64_t act_in[5] = {(uint64_t)s.cin, (uint64_t)s.w, (uint64_t)s.h, (uint64_t)B,
                                 (uint64_t)C};
