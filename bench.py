@@ -101,7 +101,8 @@ def work_per_round(w, esz):
         tc = esz == 2 and cin >= 32 and cin % 32 == 0 and cout % 64 == 0 and ww <= 64
         # tensor-core launches are timed per layer (".L<i>")
         add(f"conv_fwd_tc.L{i}" if esz == 2 else "conv_fwd", "tensor", f)
-        add(f"conv_wgrad_tc.L{i}" if tc else "conv_wgrad", "tensor", f)
+        wg_tc = tc or (esz == 2 and i == 0 and cout in (32, 64) and ww <= 64)
+        add(f"conv_wgrad_tc.L{i}" if wg_tc else "conv_wgrad", "tensor", f)
         # relu/max-pool backward: read dL/dout (+ codes, or the ReLU output),
         # write g at full resolution
         full = C * B * h * ww * cout

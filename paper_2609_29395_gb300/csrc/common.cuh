@@ -148,6 +148,10 @@ cudaError_t launch_conv0_tc(cudaStream_t s, const CUtensorMap& a, const CUtensor
                             const ConvTcArgs& p, int epi, int C);
 cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout,
                            int cin, int C);
+// input-layer weight and bias gradient partials (cout 32 or 64), partial
+// layout [C][splits][cout*9*cin + cout]
+cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                             const WgradTcArgs& p, int C);
 // dw[c * dw_rs + i] = sum over s (in order) of partial[c][s][i], i < per
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
                                 int splits, int64_t per, int C);

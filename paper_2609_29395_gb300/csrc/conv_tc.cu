@@ -559,6 +559,122 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
 }
 
+// Weight and bias gradient of the input layer (x padded to 8 channels, cout
+// 32 or 64): D[co][slot*8 + ch] = sum_p g[p][co] B[p][slot*8 + ch] with slots
+// 0..8 the tap-shifted x tiles (64 pixels x 16 bytes, unswizzled MN-major
+// N blocks 1 KB apart) and slot 9 a block of ones (bias).  The g tile
+// (cout channels, swizzled MN-major) fills the 128 MMA rows 128/cout times;
+// the epilogue keeps rows < cout.  Partial layout as in k_wgrad_tc.
+template <int COUT>
+struct Wg0Cfg {
+  static constexpr int BKP = 64;
+  static constexpr int A_BLK = COUT * BKP * 2;           // one copy of the g tile
+  static constexpr int A_BYTES = 128 * BKP * 2;
+  static constexpr int SLOT = BKP * 16;
+  static constexpr int B_BYTES = 10 * SLOT;
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int S = 4;
+  static constexpr int SMEM = 1024 + S * STAGE;
+};
+
+template <int COUT>
+__global__ void __launch_bounds__(kThreads, 1)
+k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tX,
+            const WgradTcArgs p) {
+  using Cfg = Wg0Cfg<COUT>;
+  constexpr int S = Cfg::S;
+  extern __shared__ uint8_t smraw[];
+  uint8_t* sm = align1024(smraw);
+  __shared__ uint64_t full[S], empty[S], done;
+  __shared__ uint32_t tbase;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, c = blockIdx.z;
+  const int per = COUT * 9 * p.cin + COUT;
+  const int kb_begin = split * p.kb_per_split;
+  const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
+  const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
+  const int rows_blocks = p.H / p.hb;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(&done, 1);
+    fence_mbar_init();
+  }
+  {
+    const uint4 ones = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    for (int s = 0; s < S; ++s) {
+      uint4* dst = reinterpret_cast<uint4*>(sm + s * Cfg::STAGE + Cfg::A_BYTES + 9 * Cfg::SLOT);
+      for (int i = threadIdx.x; i < Cfg::SLOT / 16; i += blockDim.x) dst[i] = ones;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) { tmem_alloc(&tbase, 128); tmem_relinquish(); }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tbase;
+  if (warp == 0) {
+    if (elect_one()) {
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % S;
+        if (i >= S && !mbar_wait(&empty[s], ((i / S) & 1) ^ 1)) { atomicOr(p.err, 256); break; }
+        const int kb = kb_begin + i;
+        const int b = (kb / rows_blocks) * p.bb, h = (kb % rows_blocks) * p.hb;
+        uint8_t* sa = sm + s * Cfg::STAGE;
+        uint8_t* sb = sa + Cfg::A_BYTES;
+        mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + 9 * Cfg::SLOT);
+#pragma unroll
+        for (int j = 0; j < 128 / COUT; ++j) tma_load_5d(sa + j * Cfg::A_BLK, &tG, &full[s], 0, 0, h, b, c);
+#pragma unroll
+        for (int tap = 0; tap < 9; ++tap)
+          tma_load_5d(sb + tap * Cfg::SLOT, &tX, &full[s], 0, tap % 3 - 1, h + tap / 3 - 1, b, c);
+      }
+    }
+  } else if (warp == 1) {
+    if (elect_one()) {
+      constexpr uint32_t idesc = idesc_bf16(BM, 80, 1, 1);
+      constexpr uint32_t a_row = COUT * 2;
+      constexpr uint32_t a_swz = COUT == 64 ? SWZ_128 : SWZ_64;
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % S;
+        if (!mbar_wait(&full[s], (i / S) & 1)) { atomicOr(p.err, 256); break; }
+        tc_fence_after();
+        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
+#pragma unroll
+        for (int k = 0; k < Cfg::BKP / 16; ++k)
+          mma_f16(tmem, smem_desc(a + k * 16 * a_row, Cfg::A_BLK, 8 * a_row, a_swz),
+                  smem_desc(b + k * 16 * 16, 128, Cfg::SLOT, SWZ_NONE), idesc, (i | k) != 0);
+        mma_commit(&empty[s]);
+      }
+      mma_commit(&done);
+    }
+  } else {
+    const int q = warp & 3;
+    const int co = q * 32 + lane;
+    if (!mbar_wait(&done, 0)) atomicOr(p.err, 512);
+    tc_fence_after();
+    if (q * 32 < COUT) {                        // warp-uniform
+      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
+      float* part = p.partial + ((int64_t)c * p.splits + split) * per;
+#pragma unroll 1
+      for (int c0 = 0; c0 < 80; c0 += 16) {
+        float v[16];
+        tmem_ld16(trow + c0, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int col = c0 + i, slot = col / 8, ch = col % 8;
+          const float x = nkb ? v[i] : 0.f;
+          if (slot < 9 && ch < p.cin) part[(co * 9 + slot) * p.cin + ch] = x;
+          else if (slot == 9 && ch == 0) part[COUT * 9 * p.cin + co] = x;
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, 128);
+}
+
 // dw[c][i] = sum_s partial[c][s][i].  A block of 8 warps covers 32 * 8/G
 // consecutive columns; the G warps of a column group split the s range
 // (warp g takes s = g, g+G, ...) and their sums are added in warp order, so
@@ -785,6 +901,27 @@ cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensor
   if (bn == 32) return launch_wgrad_inst<32>(s, g, x, p, grid);
   if (bn == 64) return launch_wgrad_inst<64>(s, g, x, p, grid);
   if (bn == 128) return launch_wgrad_inst<128>(s, g, x, p, grid);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                             const WgradTcArgs& p, int C) {
+#define GCPSL_WG0(CO)                                                                        \
+  if (p.cout == CO) {                                                                        \
+    static bool attr = false;                                                                \
+    if (!attr) {                                                                             \
+      cudaError_t e = cudaFuncSetAttribute(k_wgrad0_tc<CO>,                                  \
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,      \
+                                           Wg0Cfg<CO>::SMEM);                                \
+      if (e != cudaSuccess) return e;                                                        \
+      attr = true;                                                                           \
+    }                                                                                        \
+    k_wgrad0_tc<CO><<<dim3(p.splits, 1, C), kThreads, Wg0Cfg<CO>::SMEM, s>>>(g, x, p);       \
+    return cudaGetLastError();                                                               \
+  }
+  GCPSL_WG0(32)
+  GCPSL_WG0(64)
+#undef GCPSL_WG0
   return cudaErrorInvalidValue;
 }
 

@@ -165,6 +165,9 @@ struct gcpsl_ctx {
     bool on = false;
     int bw, hb, bb, tiles_w, tiles_h;
     CUtensorMap A, B;
+    bool wg_on = false;            // its weight gradient on the tensor cores too
+    int whb, wbb, kb_total, kb_per_split, splits;
+    CUtensorMap wgA, wgB;
   } tc0;
   int x0c = 3;
   bf16* d_w0p = nullptr;
@@ -428,6 +431,14 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
       LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
                                                  L.splits,
                                                  (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
+    } else if (i == 0 && c->tc0.wg_on) {
+      const auto& L0 = c->tc0;
+      WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L0.whb, L0.wbb, L0.kb_total, L0.kb_per_split,
+                    L0.splits, c->d_partial, c->d_err};
+      LAUNCH(kWgradTc[0], launch_wgrad0_tc(s, L0.wgA, L0.wgB, w, C));
+      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[0], P,
+                                                 L0.splits,
+                                                 (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
     } else {
       // weights and bias together (the bias follows the weight in the store)
       LAUNCH("conv_wgrad", launch_wgrad_simt<T>(s, act[i], i == 0 ? c->x0c : cs.cin, g,
@@ -556,6 +567,31 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
       !tensor_map_bf16(&L0.B, c->d_w0p, 4, wdims, wbox, 0))
     return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input layer");
   L0.on = true;
+  // its weight gradient: 64-pixel K blocks, split per replica shape only
+  L0.wg_on = false;
+  L0.whb = std::min(s0.h, 64 / s0.w);
+  L0.wbb = L0.whb > 0 ? 64 / (s0.w * L0.whb) : 0;
+  if ((s0.cout == 32 || s0.cout == 64) && s0.w <= 64 && 64 % s0.w == 0 &&
+      s0.w * L0.whb * L0.wbb == 64 && s0.h % L0.whb == 0) {
+    L0.kb_total = ((B + L0.wbb - 1) / L0.wbb) * (s0.h / L0.whb);
+    const int splits = std::max(1, std::min(64, (L0.kb_total + 15) / 16));
+    L0.kb_per_split = (L0.kb_total + splits - 1) / splits;
+    L0.splits = (L0.kb_total + L0.kb_per_split - 1) / L0.kb_per_split;
+    const uint64_t gd[5] = {(uint64_t)s0.cout, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B,
+                            (uint64_t)C};
+    const uint32_t gb[5] = {(uint32_t)s0.cout, (uint32_t)s0.w, (uint32_t)L0.whb,
+                            (uint32_t)L0.wbb, 1};
+    const uint32_t xb[5] = {8, (uint32_t)s0.w, (uint32_t)L0.whb, (uint32_t)L0.wbb, 1};
+    if (!tensor_map_bf16(&L0.wgA, c->d_g, 5, gd, gb, s0.cout * 2) ||
+        !tensor_map_bf16(&L0.wgB, c->d_act[0], 5, xdims, xb, 0))
+      return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input-layer gradient");
+    const int64_t need = (int64_t)C * L0.splits * ((int64_t)s0.cout * 9 * s0.cin + s0.cout);
+    if (need > partial_max) {
+      partial_max = need;
+      DALLOC(c->d_partial, sizeof(float) * partial_max);
+    }
+    L0.wg_on = true;
+  }
   return GCPSL_OK;
 }
 
