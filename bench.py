@@ -103,17 +103,23 @@ def work_per_round(w, esz):
         add(f"conv_fwd_tc.L{i}" if esz == 2 else "conv_fwd", "tensor", f)
         wg_tc = tc or (esz == 2 and i == 0 and cout in (32, 64) and ww <= 64)
         add(f"conv_wgrad_tc.L{i}" if wg_tc else "conv_wgrad", "tensor", f)
-        # relu/max-pool backward: read dL/dout (+ codes, or the ReLU output),
-        # write g at full resolution
-        full = C * B * h * ww * cout
-        outp = full // 4 if _p else full
-        add("relu_pool_bwd", "hbm", full * esz + outp * (esz + (1 if _p else esz)))
+        # relu/max-pool backward as its own kernel (read dL/dout + codes or
+        # the ReLU output, write g at full resolution) only where no producer
+        # fuses it: the head fuses it for the last layer, a tensor-core data
+        # gradient of layer i+1 for layer i
+        nxt = convs[i + 1] if i + 1 < len(convs) else None
+        fused = nxt is None or (esz == 2 and nxt[0] >= 32 and nxt[0] % 32 == 0
+                                and nxt[1] % 64 == 0 and nxt[3] <= 64)
+        if not fused:
+            full = C * B * h * ww * cout
+            outp = full // 4 if _p else full
+            add("relu_pool_bwd", "hbm", full * esz + outp * (esz + (1 if _p else esz)))
         if i > 0:
             add(f"conv_dgrad_tc.L{i}" if tc else "conv_dgrad", "tensor", f)
     fin, fout = spec["fc"]
     fc = 2.0 * C * B * fin * fout
     return {
-        **work, "fc_fwd": ("tensor", fc),
+        **work, "fc_fwd_ce": ("tensor", fc),
         "fc_bwd": ("tensor", 2 * fc),
         "sgd": ("hbm", C * P * (4 * 5 + (2 if esz == 2 else 0))),
         "fuse": ("hbm", C * P * (4 + 4 + (2 if esz == 2 else 0))),
@@ -273,13 +279,27 @@ def main():
     torch.cuda.synchronize()
 
     K = args.steps
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(K)]
+    # breakdown pass (before the timed region, same rounds): every kernel is
+    # bracketed by events, which finds the dominant kernel kind
     ctx.set_timing(True)
     ctx.reset_kernel_times()
+    for i in range(K):
+        flush.fill_(float(i))
+        ctx.step()
+    torch.cuda.synchronize()
+    all_times = ctx.kernel_times()
+    kind = max(all_times.items(), key=lambda kv: kv[1][1])[0]
+
+    # the timed region: only the dominant kernel carries event records, so
+    # the round runs as it does untimed
+    ctx.set_timing_filter(kind)
+    ctx.reset_kernel_times()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    n0 = ctx.kernels_launched()
     with ClockSampler(local) as clk:
         wall0 = time.perf_counter()
         for i in range(K):
@@ -289,24 +309,24 @@ def main():
             ev[i][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
+    launches = ctx.kernels_launched() - n0
     if world > 1:
         dist.barrier()
-    ctx.set_timing(False)
-    step_ms = sum(a.elapsed_time(b) for a, b in ev)
     ktimes = ctx.kernel_times()
+    ctx.set_timing(False)
+    ctx.set_timing_filter(None)
+    step_ms = sum(a.elapsed_time(b) for a, b in ev)
     if world > 1:
         t = torch.tensor([step_ms], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         step_ms = float(t.item())
     examples = w.num_clusters * w.B * K * world
     value = examples / (step_ms / 1e3)
-    launches = sum(n for n, _ in ktimes.values())
 
     # dominant kernel and its roofline
     peaks = load_peaks()
     work = work_per_round(w, 2 if w.bf16 else 4)
-    top = max(ktimes.items(), key=lambda kv: kv[1][1])
-    kind, (n_launch, k_ms) = top
+    n_launch, k_ms = ktimes.get(kind, (0, 0.0))
     bound, per_round = work.get(kind, ("hbm", None))
     roof = {"kernel": kind, "launches": n_launch, "avg_launch_ms": k_ms / max(n_launch, 1)}
     if per_round is not None:
@@ -330,7 +350,7 @@ def main():
     roof["traffic"] = rec["bytes"] if rec and rec["src_hash"] == kernel_source_hash(kind) else None
 
     breakdown = {k: {"launches": n, "ms_per_round": ms / K} for k, (n, ms) in
-                 sorted(ktimes.items(), key=lambda kv: -kv[1][1])}
+                 sorted(all_times.items(), key=lambda kv: -kv[1][1])}
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
@@ -342,6 +362,7 @@ def main():
                    "global_batch": w.num_clusters * w.B * world, "parallelism": f"replicas{world}",
                    "l2": "flushed between timed steps (256 MiB write)"},
         "roofline": roof, "gpu_launches": launches, "wall_s": wall,
+        # per-kernel device time from the breakdown pass (every kernel timed)
         "kernels": breakdown,
     }
     clocks = clk.summary()

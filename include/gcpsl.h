@@ -180,12 +180,29 @@ int64_t gcpsl_rounds(const gcpsl_ctx* ctx);
  * NULL returns to the context's own stream.  Synchronises the old stream. */
 gcpsl_status gcpsl_set_stream(gcpsl_ctx* ctx, void* cuda_stream);
 
+/* gcpsl_set_graph -- rounds after the first are replayed from CUDA graphs
+ * (default on): each round variant (epoch boundary or not, timed or not) is
+ * captured from the stream on first use and relaunched with one
+ * cudaGraphLaunch.  A replay enqueues exactly the kernels and arguments of
+ * the eager path, so results are identical bit for bit; 0 switches to eager
+ * launches.  Synchronises the stream.  Not part of the paper: a launch-cost
+ * measure for small rounds.                                              */
+gcpsl_status gcpsl_set_graph(gcpsl_ctx* ctx, int enable);
+
 /* Kernel timing: when enabled, every kernel the context launches is
- * bracketed by CUDA events on its stream.  gcpsl_kernel_times fills, for up
+ * bracketed by CUDA events on its stream (event-record nodes in a graph).  gcpsl_kernel_times fills, for up
  * to `cap` kernel kinds, the name (static string), the number of launches
  * and the summed device milliseconds since the last reset, and returns the
  * number of kinds (synchronises).                                        */
 gcpsl_status gcpsl_set_timing(gcpsl_ctx* ctx, int enable);
+/* gcpsl_kernels_launched -- kernels the context has launched so far
+ * (eager launches and the kernel nodes of replayed graphs); -1 for NULL.  */
+int64_t gcpsl_kernels_launched(const gcpsl_ctx* ctx);
+
+/* gcpsl_set_timing_filter -- time only the kernels whose name starts with
+ * `prefix` (NULL or "" = all), so that a timed round carries few event
+ * records.  Synchronises the stream.                                     */
+gcpsl_status gcpsl_set_timing_filter(gcpsl_ctx* ctx, const char* prefix);
 int gcpsl_kernel_times(gcpsl_ctx* ctx, const char** names, int64_t* launches, double* ms,
                        int cap);
 void gcpsl_reset_kernel_times(gcpsl_ctx* ctx);

@@ -28,7 +28,9 @@ STATUS_NAMES = {0: "OK", 1: "E_INVAL", 2: "E_NOMEM", 3: "E_CUDA", 4: "E_STATE", 
 EXPORTS = ("gcpsl_init", "gcpsl_step", "gcpsl_fuse", "gcpsl_get_params", "gcpsl_set_params",
            "gcpsl_get_momentum", "gcpsl_set_momentum", "gcpsl_get_pool_codes",
            "gcpsl_get_cut", "gcpsl_cut_elems", "gcpsl_get_sample", "gcpsl_num_params",
-           "gcpsl_rounds", "gcpsl_set_stream", "gcpsl_set_timing", "gcpsl_kernel_times",
+           "gcpsl_rounds", "gcpsl_set_stream", "gcpsl_set_graph", "gcpsl_set_timing",
+           "gcpsl_set_timing_filter", "gcpsl_kernels_launched",
+           "gcpsl_kernel_times",
            "gcpsl_reset_kernel_times", "gcpsl_sample_round_noalloc", "gcpsl_last_error",
            "gcpsl_destroy")
 
@@ -88,6 +90,10 @@ def load() -> ct.CDLL:
     L.gcpsl_rounds.restype = ct.c_int64
     L.gcpsl_set_stream.argtypes = [vp, vp]
     L.gcpsl_set_timing.argtypes = [vp, ct.c_int]
+    L.gcpsl_set_graph.argtypes = [vp, ct.c_int]
+    L.gcpsl_set_timing_filter.argtypes = [vp, ct.c_char_p]
+    L.gcpsl_kernels_launched.argtypes = [vp]
+    L.gcpsl_kernels_launched.restype = ct.c_int64
     L.gcpsl_kernel_times.argtypes = [vp, ct.POINTER(ct.c_char_p), ct.POINTER(ct.c_int64),
                                      ct.POINTER(ct.c_double), ct.c_int]
     L.gcpsl_kernel_times.restype = ct.c_int
@@ -103,6 +109,7 @@ def load() -> ct.CDLL:
     L.gcpsl_destroy.restype = None
     for name in ("gcpsl_init", "gcpsl_step", "gcpsl_fuse", "gcpsl_get_params", "gcpsl_set_params",
                  "gcpsl_get_cut", "gcpsl_get_sample", "gcpsl_set_stream", "gcpsl_set_timing",
+                 "gcpsl_set_graph", "gcpsl_set_timing_filter",
                  "gcpsl_get_momentum", "gcpsl_set_momentum", "gcpsl_get_pool_codes"):
         getattr(L, name).restype = ct.c_int
     _lib = L
@@ -248,6 +255,19 @@ class Context:
 
     def set_timing(self, on: bool):
         _check(load().gcpsl_set_timing(self._h, int(on)), self._h)
+
+    def kernels_launched(self) -> int:
+        """Kernels launched so far (eager launches and graph kernel nodes)."""
+        return int(load().gcpsl_kernels_launched(self._h))
+
+    def set_timing_filter(self, prefix=None):
+        """Time only kernels whose name starts with prefix (None: all)."""
+        _check(load().gcpsl_set_timing_filter(self._h, prefix.encode() if prefix else None),
+               self._h)
+
+    def set_graph(self, on: bool):
+        """Replay rounds from CUDA graphs (default) or launch them eagerly."""
+        _check(load().gcpsl_set_graph(self._h, int(on)), self._h)
 
     def kernel_times(self):
         """{kernel kind: (launches, total device ms)} since the last reset."""

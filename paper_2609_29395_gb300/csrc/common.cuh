@@ -54,6 +54,36 @@ __host__ __device__ inline void philox4x32_10(uint32_t c[4], uint32_t k0, uint32
 }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch.  Every kernel of the library is launched
+// with programmatic stream serialisation, so it may be scheduled while the
+// previous kernel on the stream drains.  Each kernel therefore runs only
+// set-up that touches no global memory (barrier init, TMEM allocation,
+// descriptor prefetch) before pdl_wait(), which returns once the previous
+// grid has completed and its writes are visible; it then calls
+// pdl_trigger() so that the next kernel can be scheduled in turn.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                            cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+// ---------------------------------------------------------------------------
 // Element conversions for the two storage types
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float to_f(float v) { return v; }
@@ -76,8 +106,17 @@ cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* of
                           const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
                           const int32_t* labels, int K, int B, int C, int32_t* idx,
                           int32_t* counts, int32_t* active, int32_t* y);
+// fp32: x0 = the sampled images, NHWC with 3 channels; bf16: x0 = the input
+// layer's im2col [CB][32][32][32] (27 tap x channel columns, a ones column
+// for the bias gradient, zero padding)
 template <typename T>
 cudaError_t launch_gather(cudaStream_t s, const float* images, const int32_t* idx, int CB, T* x0);
+template <>
+cudaError_t launch_gather<float>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
+                                 float* x0);
+template <>
+cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
+                                bf16* x0);
 
 // conv_simt.cu
 template <typename T>
@@ -96,24 +135,28 @@ template <typename T>
 cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, int xc, const T* g, float* partial,
                               int C, int B, const ConvSpec& cs, int tr, int splits,
                               int tiles_per_split);
-// bias-gradient partials over chunks of chunk_px pixels: partial[c][chunk][cout]
-template <typename T>
-cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int C, int B,
-                                const ConvSpec& cs, int chunks, int chunk_px);
 
 // head.cu
+// forward of the linear layer with the per-example softmax cross-entropy:
+// loss_ex[c][b] = l_b, dlogits[c][b][j]
 template <typename T>
-cudaError_t launch_fc_fwd(cudaStream_t s, const T* h, const T* w, int64_t w_rs, const float* b,
-                          int64_t b_rs, float* logits, int C, int B, int fin, int fout);
-cudaError_t launch_softmax_ce(cudaStream_t s, const float* logits, const int32_t* y, float* loss,
-                              float* dlogits, int C, int B, int fout, float label_smoothing);
+cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_rs,
+                             const float* b, int64_t b_rs, const int32_t* y, float* loss_ex,
+                             float* dlogits, int C, int B, int fin, int fout,
+                             float label_smoothing);
+// backward of the linear layer (dW, db, dh) and loss[c] = mean_b loss_ex[c][b].
+// route: FC_DH_STORE writes dh; FC_DH_POOL writes the last conv layer's g
+// (2Ho x 2Wo x ch) through its max-pool codes; FC_DH_RELU writes g = dh where
+// act > 0.  h is [Ho][Wo][ch] per example.
+enum { FC_DH_STORE = 0, FC_DH_POOL = 1, FC_DH_RELU = 2 };
 template <typename T>
-cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const T* h, const T* w,
-                          int64_t w_rs, float* dw, float* db, int64_t g_rs, T* dh, int C, int B,
-                          int fin, int fout);
+cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* loss_ex,
+                          const T* h, const T* w, int64_t w_rs, float* dw, float* db,
+                          int64_t g_rs, T* dh, float* loss, int C, int B, int fin, int fout,
+                          int route, const uint8_t* code, const T* act, int Ho, int Wo, int ch);
 
 // conv_tc.cu (tensor-core convolutions, bf16 operands)
-enum { EPI_POOL = 0, EPI_RELU = 1, EPI_STORE = 2 };
+enum { EPI_POOL = 0, EPI_RELU = 1, EPI_STORE = 2, EPI_DPOOL = 3, EPI_DRELU = 4 };
 struct ConvTcArgs {
   int H, W, B;          // spatial size and batch per replica
   int kch;              // channels of the activation operand (multiple of the stage width)
@@ -122,9 +165,12 @@ struct ConvTcArgs {
   int n_total;          // output channels (row length of `out`)
   const float* bias;    // fp32 bias of replica 0 (EPI_POOL / EPI_RELU)
   int64_t bias_rs;      // replica stride of the bias
-  bf16* out;            // NHWC output, [C][B][H'][W'][n_total]
-  uint8_t* code;        // max-pool codes, same layout as out (EPI_POOL)
+  bf16* out;            // NHWC output, [C][B][H'][W'][n_total] (may be null for EPI_D*)
+  uint8_t* code;        // max-pool codes, same layout as out (EPI_POOL writes, EPI_DPOOL reads)
   int* err;             // error word: bounded waits that gave up
+  const bf16* act;      // EPI_DRELU: the previous layer's ReLU output, layout of out
+  bf16* gout;           // EPI_DPOOL / EPI_DRELU: the previous layer's g (2H x 2W for DPOOL)
+  int taps = 9;         // 9: 3x3 taps over shifted boxes; 1: the im2col input layer
 };
 struct WgradTcArgs {
   int H, W, B, cout, cin;
@@ -142,14 +188,10 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
                            const ConvTcArgs& p, int bn, int bkc, int epi, int C);
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C);
-// input layer (<= 8 input channels, activation padded to 8): two taps per
-// MMA step; b = packed weights [C][10][cout][8]
-cudaError_t launch_conv0_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                            const ConvTcArgs& p, int epi, int C);
-cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout,
-                           int cin, int C);
-// input-layer weight and bias gradient partials (cout 32 or 64), partial
-// layout [C][splits][cout*9*cin + cout]
+// input layer: b = packed weights w0p[C][cout][32] (k = tap * 3 + ci < 27, else 0)
+cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout, int C);
+// input-layer weight and bias gradient partials from its im2col (cout 32 or
+// 64), partial layout [C][splits][cout*27 + cout]
 cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                              const WgradTcArgs& p, int C);
 // dw[c * dw_rs + i] = sum over s (in order) of partial[c][s][i], i < per

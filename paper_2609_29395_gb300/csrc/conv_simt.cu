@@ -26,6 +26,8 @@ __global__ void k_conv_fwd(const T* __restrict__ x, const T* __restrict__ w, int
                            const float* __restrict__ bias, int64_t b_rs, T* __restrict__ out,
                            uint8_t* __restrict__ code, int C, int B, int cin, int cout, int H,
                            int W, int pool) {
+  pdl_wait();
+  pdl_trigger();
   const int Ho = pool ? H / 2 : H, Wo = pool ? W / 2 : W;
   const int64_t total = (int64_t)C * B * Ho * Wo * cout;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -78,6 +80,8 @@ template <typename T>
 __global__ void k_relu_pool_bwd(const T* __restrict__ dout, const uint8_t* __restrict__ code,
                                 const T* __restrict__ act, T* __restrict__ g, int C, int B,
                                 int cout, int H, int W, int pool) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int V = 16 / sizeof(T);
   const int Ho = pool ? H / 2 : H, Wo = pool ? W / 2 : W;
   const int groups = cout / V;
@@ -129,6 +133,8 @@ __global__ void __launch_bounds__(256, 2)
 k_wgrad_small_cin(const T* __restrict__ x, int xc, const T* __restrict__ g,
                   float* __restrict__ partial, int B, int cout, int H, int W, int tr,
                   int tiles_per_split) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sm[];
   const int c = blockIdx.y, split = blockIdx.x;
   const int per_w = cout * 9 * CIN, per = per_w + cout;
@@ -206,6 +212,8 @@ k_wgrad_small_cin(const T* __restrict__ x, int xc, const T* __restrict__ g,
 template <typename T>
 __global__ void k_conv_dgrad(const T* __restrict__ g, const T* __restrict__ w, int64_t w_rs,
                              T* __restrict__ dx, int C, int B, int cin, int cout, int H, int W) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t total = (int64_t)C * B * H * W * cin;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= total) return;
@@ -241,6 +249,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
 k_wgrad_partial(const T* __restrict__ x, const T* __restrict__ g, float* __restrict__ partial,
                 int B, int cin, int xc, int cout, int H, int W, int tr, int tiles_per_split) {
+  pdl_wait();
+  pdl_trigger();
   // xc = channels per pixel of x in memory (>= cin; the padded input layer)
   extern __shared__ float sm[];
   const int c = blockIdx.y, split = blockIdx.x;
@@ -290,43 +300,6 @@ k_wgrad_partial(const T* __restrict__ x, const T* __restrict__ g, float* __restr
   }
 }
 
-// Bias-gradient partials: partial[c][chunk][co] = sum of g over the chunk's
-// `chunk_px` pixels.  256 threads = (cout/V channel groups of 16 bytes) x
-// lanes; lane l sums pixels l, l+lanes, ... of the chunk, then the lanes'
-// sums are added in lane order.
-template <typename T>
-__global__ void __launch_bounds__(256)
-k_bias_partial(const T* __restrict__ g, float* __restrict__ partial, int64_t npix, int cout,
-               int chunk_px) {
-  constexpr int V = 16 / sizeof(T);
-  __shared__ float red[256 * V];
-  const int c = blockIdx.y, chunk = blockIdx.x;
-  const int groups = cout / V, lanes = 256 / groups;
-  const int t = threadIdx.x, grp = t % groups, lane = t / groups;
-  const int64_t p0 = (int64_t)chunk * chunk_px;
-  const int64_t p1 = min(p0 + chunk_px, npix);
-  const T* gc = g + (int64_t)c * npix * cout + grp * V;
-  float s[V];
-#pragma unroll
-  for (int k = 0; k < V; ++k) s[k] = 0.f;
-  if (lane < lanes) {
-    for (int64_t p = p0 + lane; p < p1; p += lanes) {
-      const uint4 v = *reinterpret_cast<const uint4*>(gc + p * cout);
-      const T* e = reinterpret_cast<const T*>(&v);
-#pragma unroll
-      for (int k = 0; k < V; ++k) s[k] += to_f(e[k]);
-    }
-#pragma unroll
-    for (int k = 0; k < V; ++k) red[lane * cout + grp * V + k] = s[k];
-  }
-  __syncthreads();
-  for (int co = t; co < cout; co += blockDim.x) {
-    float tot = 0.f;
-    for (int l = 0; l < lanes; ++l) tot += red[l * cout + co];
-    partial[((int64_t)c * gridDim.x + chunk) * cout + co] = tot;
-  }
-}
-
 inline unsigned blocks(int64_t n, int t) { return (unsigned)((n + t - 1) / t); }
 
 }  // namespace
@@ -337,9 +310,8 @@ cudaError_t launch_conv_fwd_simt(cudaStream_t s, const T* x, const T* w, int64_t
                                  int B, const ConvSpec& cs) {
   const int Ho = cs.pool ? cs.h / 2 : cs.h, Wo = cs.pool ? cs.w / 2 : cs.w;
   const int64_t n = (int64_t)C * B * Ho * Wo * cs.cout;
-  k_conv_fwd<T><<<blocks(n, 256), 256, 0, s>>>(x, w, w_rs, bias, b_rs, out, code, C, B, cs.cin,
-                                                cs.cout, cs.h, cs.w, cs.pool);
-  return cudaGetLastError();
+  return launch_k(k_conv_fwd<T>, blocks(n, 256), 256, 0, s, x, w, w_rs, bias, b_rs, out, code, C,
+                  B, cs.cin, cs.cout, cs.h, cs.w, cs.pool);
 }
 
 template <typename T>
@@ -349,18 +321,16 @@ cudaError_t launch_relu_pool_bwd(cudaStream_t s, const T* dout, const uint8_t* c
   if (cs.cout % V) return cudaErrorInvalidValue;
   const int64_t opix = (int64_t)C * B * (cs.pool ? cs.h * cs.w / 4 : cs.h * cs.w);
   const int64_t n = opix * (cs.cout / V);
-  k_relu_pool_bwd<T><<<blocks(n, 256), 256, 0, s>>>(dout, code, act, g, C, B, cs.cout, cs.h,
-                                                     cs.w, cs.pool);
-  return cudaGetLastError();
+  return launch_k(k_relu_pool_bwd<T>, blocks(n, 256), 256, 0, s, dout, code, act, g, C, B,
+                  cs.cout, cs.h, cs.w, cs.pool);
 }
 
 template <typename T>
 cudaError_t launch_conv_dgrad_simt(cudaStream_t s, const T* g, const T* w, int64_t w_rs, T* dx,
                                    int C, int B, const ConvSpec& cs) {
   const int64_t n = (int64_t)C * B * cs.h * cs.w * cs.cin;
-  k_conv_dgrad<T><<<blocks(n, 256), 256, 0, s>>>(g, w, w_rs, dx, C, B, cs.cin, cs.cout, cs.h,
-                                                  cs.w);
-  return cudaGetLastError();
+  return launch_k(k_conv_dgrad<T>, blocks(n, 256), 256, 0, s, g, w, w_rs, dx, C, B, cs.cin,
+                  cs.cout, cs.h, cs.w);
 }
 
 template <typename T>
@@ -381,9 +351,8 @@ cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, int xc, const T* g, fl
       attr = true;                                                                            \
     }                                                                                         \
     if (sm > (96 << 10)) return cudaErrorInvalidValue;                                        \
-    k_wgrad_small_cin<T, CI><<<dim3(splits, C), 256, sm, s>>>(x, xc, g, partial, B, cs.cout,  \
-                                                              cs.h, cs.w, tr, tiles_per_split); \
-    return cudaGetLastError();                                                                \
+    return launch_k(k_wgrad_small_cin<T, CI>, dim3(splits, C), 256, sm, s, x, xc, g, partial, \
+                    B, cs.cout, cs.h, cs.w, tr, tiles_per_split);                             \
   }
     GCPSL_SMALL_CIN(1)
     GCPSL_SMALL_CIN(2)
@@ -400,19 +369,8 @@ cudaError_t launch_wgrad_simt(cudaStream_t s, const T* x, int xc, const T* g, fl
     if (e != cudaSuccess) return e;
     attr_set = smem;
   }
-  k_wgrad_partial<T><<<dim3(splits, C), 256, smem, s>>>(x, g, partial, B, cs.cin, xc, cs.cout,
-                                                        cs.h, cs.w, tr, tiles_per_split);
-  return cudaGetLastError();
-}
-
-template <typename T>
-cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int C, int B,
-                                const ConvSpec& cs, int chunks, int chunk_px) {
-  constexpr int V = 16 / sizeof(T);
-  if (cs.cout % V || cs.cout / V > 256) return cudaErrorInvalidValue;
-  const int64_t npix = (int64_t)B * cs.h * cs.w;
-  k_bias_partial<T><<<dim3(chunks, C), 256, 0, s>>>(g, partial, npix, cs.cout, chunk_px);
-  return cudaGetLastError();
+  return launch_k(k_wgrad_partial<T>, dim3(splits, C), 256, smem, s, x, g, partial, B, cs.cin, xc,
+                  cs.cout, cs.h, cs.w, tr, tiles_per_split);
 }
 
 #define GCPSL_INST(T)                                                                          \
@@ -424,9 +382,7 @@ cudaError_t launch_bias_partial(cudaStream_t s, const T* g, float* partial, int 
   template cudaError_t launch_conv_dgrad_simt<T>(cudaStream_t, const T*, const T*, int64_t,    \
                                                  T*, int, int, const ConvSpec&);               \
   template cudaError_t launch_wgrad_simt<T>(cudaStream_t, const T*, int, const T*, float*, int, \
-                                            int, const ConvSpec&, int, int, int);              \
-  template cudaError_t launch_bias_partial<T>(cudaStream_t, const T*, float*, int, int,        \
-                                              const ConvSpec&, int, int);
+                                            int, const ConvSpec&, int, int, int);
 GCPSL_INST(float)
 GCPSL_INST(bf16)
 #undef GCPSL_INST

@@ -16,9 +16,9 @@
 //      with the first-maximum code, decided on the fp32 values).
 //    dgrad: input = g (gradient w.r.t. the pre-activation), n = cin,
 //      B[ci][tap][co] = W[co][8-tap][ci], read MN-major from the same shadow;
-//      epilogue stores dx.
-//  k_conv0_tc: the input layer (<= 8 channels, images padded to 8): two taps
-//    per K=16 MMA step through the unswizzled layout.
+//      the epilogue stores dx, or routes it through the previous layer's
+//      max-pool / ReLU backward into that layer's g.
+//    The input layer runs through it with one tap over its im2col (K = 32).
 //  k_wgrad_tc: dW[co][tap][ci] = sum_p g[p][co] x[p + shift(tap)][ci]
 //    M = co, N = ci, K = pixels.  Both operands are MN-major tiles (pixels are
 //    rows, channels contiguous), loaded as 64-pixel boxes.  The pixel range is
@@ -47,72 +47,181 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return (uint8_t*)(((uintptr_t)p + 1023) & ~(uintptr_t)1023);
 }
 
+// Epilogue scratch of the pooling epilogue: per epilogue warp a 32 x 16
+// fp32 tile, rows padded to 20 words (16-byte accesses conflict-free)
+constexpr int kXsRow = 20;
+constexpr int kEpiScratch = 4 * 32 * kXsRow * 4;
+__host__ __device__ constexpr int epi_scratch(int epi) { return epi == EPI_POOL ? kEpiScratch : 0; }
+
+// wait for this thread's outstanding TMEM loads; the values pass through
+// the asm so that no use of them can be scheduled before the wait
+__device__ __forceinline__ void tmem_wait_regs(float (&v)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]),
+                 "+f"(v[6]), "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]),
+                 "+f"(v[12]), "+f"(v[13]), "+f"(v[14]), "+f"(v[15])
+               :
+               : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
 // Epilogue of a 128-pixel x BN-channel accumulator tile, run by the four
 // epilogue warps; the thread of TMEM row r owns pixel (bb, hh, ww) of the
-// tile (r = (bb*hb + hh)*bw + ww, tiles are bw <= 16 pixels wide, so a warp
-// holds whole 2x2 windows: partners at lane^1 and lane^bw).
-//  EPI_POOL : + bias; 2x2 max-pool decided on the fp32 values (the larger
+// tile (r = (bb*hb + hh)*bw + ww; tiles are bw <= 16 pixels wide and an even
+// number of rows high, so a warp holds whole 2x2 windows).  TMEM is read 16
+// columns at a time, the next load in flight while a chunk is processed.
+//  EPI_POOL : + bias, 2x2 max-pool decided on the fp32 values (the larger
 //             value wins, ties go to the earlier position in row-major
-//             order, i.e. the first maximum); the window's top-left thread
-//             stores relu(max) in bf16 and the code (position | positive<<2).
-//  EPI_RELU : + bias, relu, bf16 store;   EPI_STORE: bf16 store.
-// 16 channels per TMEM load; stores are 16-byte vectors.
+//             order, i.e. the first maximum), bf16 relu(max) and the code
+//             (position | positive << 2).  The warp transposes each chunk
+//             through shared memory so that the window's four threads each
+//             decide 4 of the 16 channels from all four positions.
+//  EPI_RELU : + bias, relu, bf16 store.
+//  EPI_STORE: bf16 store (data gradient).
+//  EPI_DPOOL: data gradient routed through the previous layer's max-pool:
+//             the four pixels of the previous layer's 2x2 window get the
+//             bf16 gradient where the code names that position and the
+//             maximum was positive, else 0 (out, if set, also gets the
+//             gradient itself: the cut).
+//  EPI_DRELU: data gradient times the previous layer's ReLU mask (act > 0),
+//             written to gout (and to out if set).
 template <int BN, int EPI>
 __device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0, int b0, int h0,
-                                                    int w0, int c, const ConvTcArgs& p) {
+                                                    int w0, int c, const ConvTcArgs& p,
+                                                    float* xs) {
   const int W = p.W, H = p.H, bw = p.bw;
+  const int lane = r & 31;
   const int ww = r % bw, hh = (r / bw) % p.hb, bb = r / (bw * p.hb);
   const bool valid = b0 + bb < p.B;
-  const float* bias = EPI != EPI_STORE ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
-  int64_t o;
-  bool owner = valid;
+  const int64_t img = (int64_t)c * p.B + b0 + bb;
+  float v[16];
+  tmem_ld16(trow, v);
   if (EPI == EPI_POOL) {
-    o = ((((int64_t)c * p.B + b0 + bb) * (H / 2) + (h0 + hh) / 2) * (W / 2) + (w0 + ww) / 2) *
-            p.n_total + n0;
-    owner = valid && !(hh & 1) && !(ww & 1);
-  } else {
-    o = ((((int64_t)c * p.B + b0 + bb) * H + h0 + hh) * W + w0 + ww) * p.n_total + n0;
+    const int pos = (hh & 1) * 2 + (ww & 1);        // my position in the window
+    const int l0 = lane - (ww & 1) - (hh & 1) * bw;  // lane of position 0
+    const int64_t o =
+        ((img * (H / 2) + (h0 + hh) / 2) * (W / 2) + (w0 + ww) / 2) * p.n_total + n0 + 4 * pos;
+    const float* bias = p.bias + (int64_t)c * p.bias_rs + n0 + 4 * pos;
+    float4* mine = reinterpret_cast<float4*>(xs + lane * kXsRow);
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float b4[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) b4[i] = bias[c0 + i];
+      tmem_wait_regs(v);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) mine[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+      __syncwarp();
+      if (c0 + 16 < BN) tmem_ld16(trow + c0 + 16, v);
+      float4 wq[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        wq[q] = *reinterpret_cast<const float4*>(xs + (l0 + (q & 1) + (q >> 1) * bw) * kXsRow +
+                                                 4 * pos);
+      __syncwarp();
+      float best[4] = {wq[0].x + b4[0], wq[0].y + b4[1], wq[0].z + b4[2], wq[0].w + b4[3]};
+      int at[4] = {0, 0, 0, 0};
+#pragma unroll
+      for (int q = 1; q < 4; ++q) {
+        const float x4[4] = {wq[q].x + b4[0], wq[q].y + b4[1], wq[q].z + b4[2], wq[q].w + b4[3]};
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (x4[i] > best[i]) { best[i] = x4[i]; at[i] = q; }
+      }
+      uint32_t code = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) code |= (uint32_t)(at[i] | (best[i] > 0.f ? 4 : 0)) << (8 * i);
+      if (valid) {
+        uint2 hv;
+        float rl[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) rl[i] = best[i] > 0.f ? best[i] : 0.f;
+        hv.x = pack_bf16x2(rl[0], rl[1]);
+        hv.y = pack_bf16x2(rl[2], rl[3]);
+        *reinterpret_cast<uint2*>(p.out + o + c0) = hv;
+        *reinterpret_cast<uint32_t*>(p.code + o + c0) = code;
+      }
+    }
+    return;
   }
-  const int mypos = (hh & 1) * 2 + (ww & 1);
+  const int64_t o = ((img * H + h0 + hh) * W + w0 + ww) * p.n_total + n0;
+  const float* bias = EPI == EPI_RELU ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
 #pragma unroll 1
   for (int c0 = 0; c0 < BN; c0 += 16) {
-    float v[16];
-    tmem_ld16(trow + c0, v);
-    tmem_ld_wait();
-    __align__(16) bf16 h[16];
-    if (EPI == EPI_POOL) {
-      __align__(16) uint8_t code[16];
+    float b16[16];
+    if (EPI == EPI_RELU) {
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        float val = v[i] + bias[c0 + i];
-        int pos = mypos;
+      for (int i = 0; i < 16; i += 4) {
+        const float4 t = *reinterpret_cast<const float4*>(bias + c0 + i);
+        b16[i] = t.x; b16[i + 1] = t.y; b16[i + 2] = t.z; b16[i + 3] = t.w;
+      }
+    }
+    uint4 cd;
+    uint4 am[2];
+    if (EPI == EPI_DPOOL && valid) cd = *reinterpret_cast<const uint4*>(p.code + o + c0);
+    if (EPI == EPI_DRELU && valid) {
+      am[0] = *reinterpret_cast<const uint4*>(p.act + o + c0);
+      am[1] = *reinterpret_cast<const uint4*>(p.act + o + c0 + 8);
+    }
+    tmem_wait_regs(v);
+    uint32_t hw[8];
 #pragma unroll
-        for (int step = 0; step < 2; ++step) {
-          const int x = step == 0 ? 1 : bw;
-          const float pv = __shfl_xor_sync(0xffffffffu, val, x);
-          const int pp = __shfl_xor_sync(0xffffffffu, pos, x);
-          if (pv > val || (pv == val && pp < pos)) { val = pv; pos = pp; }
-        }
-        h[i] = __float2bfloat16_rn(val > 0.f ? val : 0.f);
-        code[i] = (uint8_t)(pos | (val > 0.f ? 4 : 0));
+    for (int i = 0; i < 8; ++i) {
+      float x0 = v[2 * i], x1 = v[2 * i + 1];
+      if (EPI == EPI_RELU) {
+        x0 += b16[2 * i];
+        x1 += b16[2 * i + 1];
+        x0 = x0 > 0.f ? x0 : 0.f;
+        x1 = x1 > 0.f ? x1 : 0.f;
       }
-      if (owner) {
-        uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
-        dst[0] = reinterpret_cast<uint4*>(h)[0];
-        dst[1] = reinterpret_cast<uint4*>(h)[1];
-        *reinterpret_cast<uint4*>(p.code + o + c0) = *reinterpret_cast<uint4*>(code);
-      }
+      hw[i] = pack_bf16x2(x0, x1);
+    }
+    if (c0 + 16 < BN) tmem_ld16(trow + c0 + 16, v);
+    if (!valid) continue;
+    if (EPI != EPI_DPOOL && EPI != EPI_DRELU) {
+      uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
+      dst[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+      dst[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+      continue;
+    }
+    if (p.out) {
+      uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
+      dst[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+      dst[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+    }
+    if (EPI == EPI_DRELU) {
+      // act > 0 <=> its bf16 bits are > 0 as a signed 16-bit integer
+      const uint32_t a[8] = {am[0].x, am[0].y, am[0].z, am[0].w, am[1].x, am[1].y, am[1].z, am[1].w};
+      uint32_t gw[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) gw[i] = hw[i] & __vcmpgts2(a[i], 0u);
+      uint4* dst = reinterpret_cast<uint4*>(p.gout + o + c0);
+      dst[0] = make_uint4(gw[0], gw[1], gw[2], gw[3]);
+      dst[1] = make_uint4(gw[4], gw[5], gw[6], gw[7]);
     } else {
+      // byte k of the codes selects the window position that gets channel k
+      const uint32_t cw[4] = {cd.x & 0x07070707u, cd.y & 0x07070707u, cd.z & 0x07070707u,
+                              cd.w & 0x07070707u};
+      const int y = h0 + hh, x = w0 + ww;
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        float x = v[i];
-        if (EPI == EPI_RELU) { x += bias[c0 + i]; x = x > 0.f ? x : 0.f; }
-        h[i] = __float2bfloat16_rn(x);
-      }
-      if (owner) {
-        uint4* dst = reinterpret_cast<uint4*>(p.out + o + c0);
-        dst[0] = reinterpret_cast<uint4*>(h)[0];
-        dst[1] = reinterpret_cast<uint4*>(h)[1];
+      for (int qd = 0; qd < 4; ++qd) {
+        const uint32_t want = (uint32_t)(4 | qd) * 0x01010101u;
+        uint32_t gw[8];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t m = __vcmpeq4(cw[j], want);           // 0xff per selected channel
+          gw[2 * j] = hw[2 * j] & __byte_perm(m, 0, 0x1100);
+          gw[2 * j + 1] = hw[2 * j + 1] & __byte_perm(m, 0, 0x3322);
+        }
+        const int64_t go =
+            ((img * (2 * H) + 2 * y + (qd >> 1)) * (2 * W) + 2 * x + (qd & 1)) * p.n_total + n0 + c0;
+        uint4* dst = reinterpret_cast<uint4*>(p.gout + go);
+        dst[0] = make_uint4(gw[0], gw[1], gw[2], gw[3]);
+        dst[1] = make_uint4(gw[4], gw[5], gw[6], gw[7]);
       }
     }
   }
@@ -126,11 +235,12 @@ struct ConvCfg {
   static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   // two CTAs per SM when both fit in TMEM (2 x 2 x TCOLS <= 512 columns)
   static constexpr int CTAS = 2 * TCOLS <= 256 ? 2 : 1;
-  static constexpr int BUDGET = CTAS == 2 ? 100 * 1024 : 200 * 1024;
+  static constexpr int XS = epi_scratch(EPI);
+  static constexpr int BUDGET = (CTAS == 2 ? 100 * 1024 : 200 * 1024) - XS;
   static constexpr int S0 = BUDGET / STAGE;
   static constexpr int S = S0 > 8 ? 8 : (S0 < 2 ? 2 : S0);
   static constexpr int PIPE = S * STAGE;
-  static constexpr int SMEM = 1024 + PIPE;
+  static constexpr int SMEM = 1024 + PIPE + XS;
 };
 
 // (b0, h0, w0) of M tile mt
@@ -164,7 +274,8 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kper = p.kch / BKC;
-  const int KB = 9 * kper;
+  const int KB = p.taps * kper;
+  const int shift = p.taps == 9 ? 1 : 0;        // 3x3 taps, or one tap (im2col input)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
@@ -178,6 +289,8 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tbase;
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     if (elect_one()) {
@@ -198,7 +311,8 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
           uint8_t* sa = sm + s * Cfg::STAGE;
           const int tap = kb / kper, ch = (kb % kper) * BKC;
           mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
-          tma_load_5d(sa, &tA, &full[s], ch, w0 + tap % 3 - 1, h0 + tap / 3 - 1, b0, c);
+          tma_load_5d(sa, &tA, &full[s], ch, w0 + (tap % 3 - 1) * shift,
+                      h0 + (tap / 3 - 1) * shift, b0, c);
           if (!BMN) {
             tma_load_4d(sa + Cfg::A_BYTES, &tB, &full[s], ch, tap, n0, c);
           } else {
@@ -268,7 +382,8 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
       int b0, h0, w0;
       tile_origin(mt, p, b0, h0, w0);
       const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
-      conv_epilogue_drain<BN, EPI>(trow, r, n0, b0, h0, w0, c, p);
+      conv_epilogue_drain<BN, EPI>(trow, r, n0, b0, h0, w0, c, p,
+                                   reinterpret_cast<float*>(sm + Cfg::PIPE) + q * 32 * kXsRow);
       tc_fence_before();
       mbar_arrive(&tempty[buf]);
     }
@@ -279,126 +394,23 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
 }
 
 // ---------------------------------------------------------------------------
-// input layer: at most 8 input channels (the gathered images, padded to 8)
+// input layer (3 channels): with bf16 operands the gather writes its im2col,
+// x0[p][k] with k = tap * 3 + ch (27 columns), a ones column (k = 27) and
+// zero padding to 32; the forward is then k_conv_tc with one tap and K = 32
+// against weights packed as w0p[c][co][32].
 // ---------------------------------------------------------------------------
-// A K=16 MMA step takes two taps: with the unswizzled K-major layout a K=16
-// slice is two 8-element core-matrix columns whose distance is the leading
-// byte offset, so tap t's 128 x 16 B box and tap t+1's box can sit 2 KB apart.
-// Ten tap slots are loaded (slot 9 repeats tap 8); the packed weights
-// [tap][co][8] have zeros for tap 9 and for channels >= cin.
-template <int BN, int EPI>
-struct Conv0Cfg {
-  static constexpr int SLOT_A = BM * 16;                 // one tap: 128 px x 8 ch
-  static constexpr int A_BYTES = 10 * SLOT_A;
-  static constexpr int B_BYTES = 10 * BN * 16;
-  static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int S = 3;
-  static constexpr int PIPE = S * STAGE;
-  static constexpr int SMEM = 1024 + PIPE;
-  static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
-  static constexpr int CTAS = 2;                          // 2 x 2 x TCOLS <= 512 for BN <= 64
-};
-
-// Persistent like k_conv_tc: one ring stage holds one work item (ten tap
-// slots and the packed weights), two TMEM accumulators alternate.
-template <int BN, int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
-k_conv0_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
-           const ConvTcArgs p, int tiles_m, int items) {
-  using Cfg = Conv0Cfg<BN, EPI>;
-  constexpr int S = Cfg::S;
-  extern __shared__ uint8_t smraw[];
-  uint8_t* sm = align1024(smraw);
-  __shared__ uint64_t full[S], empty[S], tfull[2], tempty[2];
-  __shared__ uint32_t tbase;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    for (int b = 0; b < 2; ++b) { mbar_init(&tfull[b], 1); mbar_init(&tempty[b], 128); }
-    fence_mbar_init();
-  }
-  if (warp == 1) { tmem_alloc(&tbase, 2 * Cfg::TCOLS); tmem_relinquish(); }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = tbase;
-  if (warp == 0) {
-    if (elect_one()) {
-      int it = 0;
-      for (int t = blockIdx.x; t < items; t += gridDim.x, ++it) {
-        const int c = t / tiles_m, mt = t % tiles_m;
-        int b0, h0, w0;
-        tile_origin(mt, p, b0, h0, w0);
-        const int s = it % S;
-        if (it >= S && !mbar_wait(&empty[s], ((it / S) & 1) ^ 1)) { atomicOr(p.err, 64); break; }
-        uint8_t* st = sm + s * Cfg::STAGE;
-        mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
-#pragma unroll
-        for (int j = 0; j < 10; ++j) {
-          const int tap = j < 9 ? j : 8;
-          tma_load_5d(st + j * Cfg::SLOT_A, &tA, &full[s], 0, w0 + tap % 3 - 1, h0 + tap / 3 - 1,
-                      b0, c);
-        }
-        tma_load_4d(st + Cfg::A_BYTES, &tB, &full[s], 0, 0, 0, c);
-      }
-    }
-  } else if (warp == 1) {
-    if (elect_one()) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
-      int tl = 0;
-      for (int t = blockIdx.x; t < items; t += gridDim.x, ++tl) {
-        const int buf = tl & 1, s = tl % S;
-        if (tl >= 2 && !mbar_wait(&tempty[buf], ((tl >> 1) & 1) ^ 1)) {
-          atomicOr(p.err, 64);
-          break;
-        }
-        if (!mbar_wait(&full[s], (tl / S) & 1)) { atomicOr(p.err, 64); break; }
-        tc_fence_after();
-        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
-        const uint32_t d = tmem + buf * Cfg::TCOLS;
-#pragma unroll
-        for (int k = 0; k < 5; ++k)
-          mma_f16(d, smem_desc(a + 2 * k * Cfg::SLOT_A, Cfg::SLOT_A, 128, SWZ_NONE),
-                  smem_desc(b + 2 * k * BN * 16, BN * 16, 128, SWZ_NONE), idesc, k != 0);
-        mma_commit(&empty[s]);
-        mma_commit(&tfull[buf]);
-      }
-    }
-  } else {
-    const int q = warp & 3, r = q * 32 + lane;
-    int tl = 0;
-    for (int t = blockIdx.x; t < items; t += gridDim.x, ++tl) {
-      const int buf = tl & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
-        if (lane == 0) atomicOr(p.err, 128);
-        break;
-      }
-      tc_fence_after();
-      const int c = t / tiles_m, mt = t % tiles_m;
-      int b0, h0, w0;
-      tile_origin(mt, p, b0, h0, w0);
-      const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
-      conv_epilogue_drain<BN, EPI>(trow, r, 0, b0, h0, w0, c, p);
-      tc_fence_before();
-      mbar_arrive(&tempty[buf]);
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, 2 * Cfg::TCOLS);
-}
-
-// packed input-layer weights: w0p[c][tap][co][8] = W[co][tap][ci] for
-// tap < 9 and ci < cin, else 0
+// packed input-layer weights: w0p[c][co][k] = W[co][tap][ci] at k = tap * 3 + ci
+// (k < 27), else 0
 __global__ void k_pack_w0(const bf16* __restrict__ w, bf16* __restrict__ w0p, int64_t rs,
-                          int cout, int cin) {
+                          int cout) {
+  pdl_wait();
+  pdl_trigger();
   const int c = blockIdx.y;
-  const int per = 10 * cout * 8;
+  const int per = cout * 32;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < per; i += gridDim.x * blockDim.x) {
-    const int ch = i % 8, co = (i / 8) % cout, tap = i / (8 * cout);
-    bf16 v = __float2bfloat16_rn(0.f);
-    if (tap < 9 && ch < cin) v = w[(int64_t)c * rs + ((int64_t)co * 9 + tap) * cin + ch];
-    w0p[(int64_t)c * per + i] = v;
+    const int k = i % 32, co = i / 32;
+    w0p[(int64_t)c * per + i] =
+        k < 27 ? w[(int64_t)c * rs + (int64_t)co * 27 + k] : __float2bfloat16_rn(0.f);
   }
 }
 
@@ -475,6 +487,8 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tbase;
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     if (elect_one()) {
@@ -559,21 +573,21 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
 }
 
-// Weight and bias gradient of the input layer (x padded to 8 channels, cout
-// 32 or 64): D[co][slot*8 + ch] = sum_p g[p][co] B[p][slot*8 + ch] with slots
-// 0..8 the tap-shifted x tiles (64 pixels x 16 bytes, unswizzled MN-major
-// N blocks 1 KB apart) and slot 9 a block of ones (bias).  The g tile
-// (cout channels, swizzled MN-major) fills the 128 MMA rows 128/cout times;
-// the epilogue keeps rows < cout.  Partial layout as in k_wgrad_tc.
+// Weight and bias gradient of the input layer from its im2col (cout 32 or
+// 64): D[co][k] = sum_p g[p][co] x0[p][k], a plain GEMM over the pixels;
+// column k < 27 is W[co][tap][ci] (k = tap * 3 + ci), column 27 (the ones
+// column) the bias.  The g tile (cout channels, swizzled MN-major) fills
+// the 128 MMA rows 128/cout times; the epilogue keeps rows < cout.  The x0
+// tile is one MN-major 64-pixel x 32-column box.  Partial layout as in
+// k_wgrad_tc: [cout][27] then [cout].
 template <int COUT>
 struct Wg0Cfg {
   static constexpr int BKP = 64;
   static constexpr int A_BLK = COUT * BKP * 2;           // one copy of the g tile
   static constexpr int A_BYTES = 128 * BKP * 2;
-  static constexpr int SLOT = BKP * 16;
-  static constexpr int B_BYTES = 10 * SLOT;
+  static constexpr int B_BYTES = BKP * 32 * 2;
   static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int S = 4;
+  static constexpr int S = 6;
   static constexpr int SMEM = 1024 + S * STAGE;
 };
 
@@ -589,7 +603,7 @@ k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUte
   __shared__ uint32_t tbase;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, c = blockIdx.z;
-  const int per = COUT * 9 * p.cin + COUT;
+  const int per = COUT * 27 + COUT;
   const int kb_begin = split * p.kb_per_split;
   const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
   const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
@@ -598,20 +612,16 @@ k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUte
     for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(&done, 1);
     fence_mbar_init();
+    tma_prefetch_desc(&tG);
+    tma_prefetch_desc(&tX);
   }
-  {
-    const uint4 ones = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
-    for (int s = 0; s < S; ++s) {
-      uint4* dst = reinterpret_cast<uint4*>(sm + s * Cfg::STAGE + Cfg::A_BYTES + 9 * Cfg::SLOT);
-      for (int i = threadIdx.x; i < Cfg::SLOT / 16; i += blockDim.x) dst[i] = ones;
-    }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  }
-  if (warp == 1) { tmem_alloc(&tbase, 128); tmem_relinquish(); }
+  if (warp == 1) { tmem_alloc(&tbase, 32); tmem_relinquish(); }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tbase;
+  pdl_wait();
+  pdl_trigger();
   if (warp == 0) {
     if (elect_one()) {
       for (int i = 0; i < nkb; ++i) {
@@ -620,18 +630,16 @@ k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUte
         const int kb = kb_begin + i;
         const int b = (kb / rows_blocks) * p.bb, h = (kb % rows_blocks) * p.hb;
         uint8_t* sa = sm + s * Cfg::STAGE;
-        uint8_t* sb = sa + Cfg::A_BYTES;
-        mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + 9 * Cfg::SLOT);
+        mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
 #pragma unroll
-        for (int j = 0; j < 128 / COUT; ++j) tma_load_5d(sa + j * Cfg::A_BLK, &tG, &full[s], 0, 0, h, b, c);
-#pragma unroll
-        for (int tap = 0; tap < 9; ++tap)
-          tma_load_5d(sb + tap * Cfg::SLOT, &tX, &full[s], 0, tap % 3 - 1, h + tap / 3 - 1, b, c);
+        for (int j = 0; j < 128 / COUT; ++j)
+          tma_load_5d(sa + j * Cfg::A_BLK, &tG, &full[s], 0, 0, h, b, c);
+        tma_load_5d(sa + Cfg::A_BYTES, &tX, &full[s], 0, 0, h, b, c);
       }
     }
   } else if (warp == 1) {
     if (elect_one()) {
-      constexpr uint32_t idesc = idesc_bf16(BM, 80, 1, 1);
+      constexpr uint32_t idesc = idesc_bf16(BM, 32, 1, 1);
       constexpr uint32_t a_row = COUT * 2;
       constexpr uint32_t a_swz = COUT == 64 ? SWZ_128 : SWZ_64;
       for (int i = 0; i < nkb; ++i) {
@@ -642,7 +650,7 @@ k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUte
 #pragma unroll
         for (int k = 0; k < Cfg::BKP / 16; ++k)
           mma_f16(tmem, smem_desc(a + k * 16 * a_row, Cfg::A_BLK, 8 * a_row, a_swz),
-                  smem_desc(b + k * 16 * 16, 128, Cfg::SLOT, SWZ_NONE), idesc, (i | k) != 0);
+                  smem_desc(b + k * 16 * 64, Cfg::B_BYTES, 8 * 64, SWZ_64), idesc, (i | k) != 0);
         mma_commit(&empty[s]);
       }
       mma_commit(&done);
@@ -656,23 +664,23 @@ k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUte
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
       float* part = p.partial + ((int64_t)c * p.splits + split) * per;
 #pragma unroll 1
-      for (int c0 = 0; c0 < 80; c0 += 16) {
+      for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
         tmem_ld16(trow + c0, v);
         tmem_ld_wait();
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const int col = c0 + i, slot = col / 8, ch = col % 8;
+          const int k = c0 + i;
           const float x = nkb ? v[i] : 0.f;
-          if (slot < 9 && ch < p.cin) part[(co * 9 + slot) * p.cin + ch] = x;
-          else if (slot == 9 && ch == 0) part[COUT * 9 * p.cin + co] = x;
+          if (k < 27) part[co * 27 + k] = x;
+          else if (k == 27) part[COUT * 27 + co] = x;
         }
       }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, 128);
+  if (warp == 1) tmem_dealloc(tmem, 32);
 }
 
 // dw[c][i] = sum_s partial[c][s][i].  A block of 8 warps covers 32 * 8/G
@@ -684,6 +692,8 @@ __global__ void __launch_bounds__(256)
 k_wgrad_reduce(const float* __restrict__ partial, float* __restrict__ dw, int64_t dw_rs,
                int splits, int64_t per) {
   __shared__ float red[8][32];
+  pdl_wait();
+  pdl_trigger();
   const int c = blockIdx.y;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int grp = w / G, sub = w % G;
@@ -732,9 +742,8 @@ cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
   }
   const int cap = sm_count() * Cfg::CTAS;
   const int grid = items < cap ? items : cap;
-  k_conv_tc<BN, BKC, EPI, BMN><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p, tiles_m, tiles_n,
-                                                                  items);
-  return cudaGetLastError();
+  return launch_k(k_conv_tc<BN, BKC, EPI, BMN>, grid, kThreads, Cfg::SMEM, s, a, b, p, tiles_m,
+                  tiles_n, items);
 }
 
 template <int BN>
@@ -748,8 +757,7 @@ cudaError_t launch_wgrad_inst(cudaStream_t s, const CUtensorMap& g, const CUtens
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k_wgrad_tc<BN><<<grid, kThreads, Cfg::SMEM, s>>>(g, x, p);
-  return cudaGetLastError();
+  return launch_k(k_wgrad_tc<BN>, grid, kThreads, Cfg::SMEM, s, g, x, p);
 }
 
 }  // namespace
@@ -838,58 +846,29 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
 #define GCPSL_CONV_EPIS(BN_, BKC_)          \
   GCPSL_CONV_CASE(BN_, BKC_, EPI_POOL, 0)   \
   GCPSL_CONV_CASE(BN_, BKC_, EPI_RELU, 0)   \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_STORE, 1)
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_STORE, 1)  \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_DPOOL, 1)  \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_DRELU, 1)
+  GCPSL_CONV_CASE(32, 32, EPI_POOL, 0)      // the input layer (im2col, K = 32)
+  GCPSL_CONV_CASE(32, 32, EPI_RELU, 0)
   GCPSL_CONV_EPIS(32, 64)
   GCPSL_CONV_EPIS(64, 32)
   GCPSL_CONV_EPIS(64, 64)
   GCPSL_CONV_EPIS(128, 32)
   GCPSL_CONV_EPIS(128, 64)
-  GCPSL_CONV_CASE(256, 64, EPI_RELU, 0)     // no staging tile for 256 channels
+  GCPSL_CONV_CASE(256, 64, EPI_RELU, 0)
   GCPSL_CONV_CASE(256, 64, EPI_STORE, 1)
+  GCPSL_CONV_CASE(256, 64, EPI_DPOOL, 1)
+  GCPSL_CONV_CASE(256, 64, EPI_DRELU, 1)
 #undef GCPSL_CONV_EPIS
 #undef GCPSL_CONV_CASE
   return cudaErrorInvalidValue;
 }
 
-template <int BN, int EPI>
-static cudaError_t launch_conv0_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                                     const ConvTcArgs& p, int tiles_m, int items) {
-  using Cfg = Conv0Cfg<BN, EPI>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_conv0_tc<BN, EPI>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
-  const int cap = sm_count() * Cfg::CTAS;
-  const int grid = items < cap ? items : cap;
-  k_conv0_tc<BN, EPI><<<grid, kThreads, Cfg::SMEM, s>>>(a, b, p, tiles_m, items);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_conv0_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                            const ConvTcArgs& p, int epi, int C) {
-  const int tiles_m = p.tiles_w * p.tiles_h * ((p.B + p.bb - 1) / p.bb);
-  const int items = tiles_m * C;
-  const int bn = p.n_total;
-#define GCPSL_CONV0_CASE(BN_, EPI_) \
-  if (bn == BN_ && epi == EPI_) return launch_conv0_inst<BN_, EPI_>(s, a, b, p, tiles_m, items);
-  GCPSL_CONV0_CASE(16, EPI_POOL)
-  GCPSL_CONV0_CASE(16, EPI_RELU)
-  GCPSL_CONV0_CASE(32, EPI_POOL)
-  GCPSL_CONV0_CASE(32, EPI_RELU)
-  GCPSL_CONV0_CASE(64, EPI_POOL)
-  GCPSL_CONV0_CASE(64, EPI_RELU)
-#undef GCPSL_CONV0_CASE
-  return cudaErrorInvalidValue;
-}
-
 cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout,
-                           int cin, int C) {
-  const int per = 10 * cout * 8;
-  k_pack_w0<<<dim3((unsigned)((per + 255) / 256), C), 256, 0, s>>>(w, w0p, rs, cout, cin);
-  return cudaGetLastError();
+                           int C) {
+  const int per = cout * 32;
+  return launch_k(k_pack_w0, dim3((unsigned)((per + 255) / 256), C), 256, 0, s, w, w0p, rs, cout);
 }
 
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
@@ -916,8 +895,8 @@ cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtenso
       if (e != cudaSuccess) return e;                                                        \
       attr = true;                                                                           \
     }                                                                                        \
-    k_wgrad0_tc<CO><<<dim3(p.splits, 1, C), kThreads, Wg0Cfg<CO>::SMEM, s>>>(g, x, p);       \
-    return cudaGetLastError();                                                               \
+    return launch_k(k_wgrad0_tc<CO>, dim3(p.splits, 1, C), kThreads, Wg0Cfg<CO>::SMEM, s, g, x, \
+                    p);                                                                      \
   }
   GCPSL_WG0(32)
   GCPSL_WG0(64)
@@ -930,11 +909,10 @@ cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw,
   const int G = splits <= 2 ? 1 : splits <= 8 ? 2 : splits <= 32 ? 4 : 8;
   const int64_t cols_per_block = 32 * (8 / G);
   const dim3 grid((unsigned)((per + cols_per_block - 1) / cols_per_block), C);
-  if (G == 1) k_wgrad_reduce<1><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
-  else if (G == 2) k_wgrad_reduce<2><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
-  else if (G == 4) k_wgrad_reduce<4><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
-  else k_wgrad_reduce<8><<<grid, 256, 0, s>>>(partial, dw, dw_rs, splits, per);
-  return cudaGetLastError();
+  if (G == 1) return launch_k(k_wgrad_reduce<1>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
+  if (G == 2) return launch_k(k_wgrad_reduce<2>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
+  if (G == 4) return launch_k(k_wgrad_reduce<4>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
+  return launch_k(k_wgrad_reduce<8>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
 }
 
 

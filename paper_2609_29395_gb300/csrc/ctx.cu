@@ -64,6 +64,15 @@ struct KernelTimer {
   std::vector<cudaEvent_t> pool;
   int cur_kind = -1;
   cudaEvent_t cur_a = nullptr;
+  // while a round is being captured into a graph, the event pairs become
+  // external event-record nodes of that graph and are listed here
+  std::vector<Pending>* capture = nullptr;
+  // only kernels whose name starts with this prefix are timed (empty: all)
+  std::string filter;
+
+  bool wants(const char* name) const {
+    return filter.empty() || std::strncmp(name, filter.c_str(), filter.size()) == 0;
+  }
 
   int kind(const char* name) {
     for (size_t i = 0; i < names.size(); ++i)
@@ -77,25 +86,33 @@ struct KernelTimer {
     cudaEventCreate(&e);
     return e;
   }
+  void record(cudaEvent_t e, cudaStream_t s) {
+    if (capture) cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+    else cudaEventRecord(e, s);
+  }
   void begin(const char* name, cudaStream_t s) {
     cur_kind = kind(name);
     cur_a = get();
-    cudaEventRecord(cur_a, s);
+    record(cur_a, s);
   }
   void end(cudaStream_t s) {
     cudaEvent_t b = get();
-    cudaEventRecord(b, s);
-    pending.push_back({cur_kind, cur_a, b});
+    record(b, s);
+    (capture ? *capture : pending).push_back({cur_kind, cur_a, b});
   }
-  void collect() {
-    for (auto& p : pending) {
+  // add the elapsed times of recorded pairs (waits for each pair's end)
+  void account(const std::vector<Pending>& v) {
+    for (auto& p : v) {
       float t = 0.f;
       if (cudaEventSynchronize(p.b) == cudaSuccess && cudaEventElapsedTime(&t, p.a, p.b) == cudaSuccess) {
         ms[p.kind] += t;
         launches[p.kind] += 1;
       }
-      pool.push_back(p.a); pool.push_back(p.b);
     }
+  }
+  void collect() {
+    account(pending);
+    for (auto& p : pending) { pool.push_back(p.a); pool.push_back(p.b); }
     pending.clear();
   }
   void reset() {
@@ -159,8 +176,8 @@ struct gcpsl_ctx {
     int splits, kb_total, kb_per_split;
     CUtensorMap fwdA, fwdB, dgrA, dgrB, wgA, wgB;
   } tc[4];
-  // input layer on the tensor cores (bf16 mode): the gathered images are
-  // padded to x0c = 8 channels; packed weights [C][10][cout][8]
+  // input layer on the tensor cores (bf16 mode): the gather writes its
+  // im2col, x0c = 32 columns per pixel; packed weights [C][cout][32]
   struct Tc0Layer {
     bool on = false;
     int bw, hb, bb, tiles_w, tiles_h;
@@ -172,18 +189,22 @@ struct gcpsl_ctx {
   int x0c = 3;
   bf16* d_w0p = nullptr;
   float* d_partial = nullptr;      // weight-gradient split partials (tensor-core layers)
-  // CUDA-core gradient reductions: weight+bias partials of the other layers
-  // (tiles of tr image rows, tiles_per_split tiles per block) and bias
-  // partials of the tensor-core layers (chunks of chunk_px pixels)
-  struct RedLayer { int tr, splits, tiles_per_split, chunks, chunk_px; } red[4];
+  // CUDA-core weight+bias gradient partials of the layers not on the tensor
+  // cores (tiles of tr image rows, tiles_per_split tiles per block)
+  struct RedLayer { int tr, splits, tiles_per_split; } red[4];
   float* d_bpartial = nullptr;
 
   void* d_x0 = nullptr;
   void* d_act[5] = {};             // d_act[i+1] = output of conv i
   void* d_dact[5] = {};
   uint8_t* d_code[4] = {};
+  // g_i, the gradient w.r.t. layer i's pre-activation: layers alternate
+  // between two buffers, since layer i's data gradient reads g_i while its
+  // epilogue writes g_{i-1}
   void* d_g = nullptr;
-  float* d_logits = nullptr;
+  void* d_g2 = nullptr;
+  void* gbuf(int i) const { return (i & 1) ? d_g2 : d_g; }
+  float* d_loss_ex = nullptr;     // [C][B] per-example loss
   float* d_dlogits = nullptr;
   int32_t* d_y = nullptr;
   int32_t* d_idx = nullptr;
@@ -200,6 +221,22 @@ struct gcpsl_ctx {
   std::vector<void*> allocs;
   bool timing = false;
   KernelTimer timer;
+
+  // CUDA graphs of one round: [epoch boundary or not][untimed, timed A, timed B].
+  // The two timed copies alternate so that one copy's event pairs are read
+  // while the other runs.
+  int64_t launched = 0;            // kernels launched so far (eager or graph nodes)
+  int64_t enqueued = 0;            // kernels passed through LAUNCH (eager or captured)
+  bool capturing = false;          // a round is being captured into a graph
+  struct RoundGraph {
+    cudaGraphExec_t exec = nullptr;
+    int64_t kernels = 0;          // kernel nodes of the captured round
+    std::vector<KernelTimer::Pending> marks;
+    bool unread = false;          // marks of the last launch not yet added to the timer
+  };
+  bool use_graph = true;
+  RoundGraph graph[2][3];
+  int timed_phase = 0;
 };
 
 namespace {
@@ -230,9 +267,12 @@ gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...) {
 // launch through the timer when enabled
 #define LAUNCH(name, call)                                                                 \
   do {                                                                                     \
-    if (c->timing) c->timer.begin(name, c->stream);                                        \
+    const bool _t = c->timing && c->timer.wants(name);                                     \
+    ++c->enqueued;                                                                         \
+    if (!c->capturing) ++c->launched;                                                      \
+    if (_t) c->timer.begin(name, c->stream);                                               \
     cudaError_t _e = (call);                                                               \
-    if (c->timing) c->timer.end(c->stream);                                                \
+    if (_t) c->timer.end(c->stream);                                                       \
     if (_e != cudaSuccess)                                                                 \
       return fail(c, GCPSL_E_CUDA, "kernel %s: %s", name, cudaGetErrorString(_e));        \
   } while (0)
@@ -343,7 +383,7 @@ int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
 gcpsl_status refresh_derived(gcpsl_ctx* c) {
   if (c->tc0.on)
     LAUNCH("pack_w0", launch_pack_w0(c->stream, c->d_shadow + c->a.off_w[0], c->d_w0p, c->P_pad,
-                                     c->a.conv[0].cout, c->a.conv[0].cin, c->C));
+                                     c->a.conv[0].cout, c->C));
   return GCPSL_OK;
 }
 
@@ -364,8 +404,15 @@ const char* const kDgradTc[4] = {"conv_dgrad_tc.L0", "conv_dgrad_tc.L1", "conv_d
 const char* const kWgradTc[4] = {"conv_wgrad_tc.L0", "conv_wgrad_tc.L1", "conv_wgrad_tc.L2",
                                  "conv_wgrad_tc.L3"};
 
+// true when some cluster starts an epoch in round c->t (0-based)
+bool epoch_boundary(const gcpsl_ctx* c) {
+  for (int n = 0; n < c->C; ++n)
+    if (c->t % c->h_rounds[n] == 0) return true;
+  return false;
+}
+
 template <typename T>
-gcpsl_status enqueue_round(gcpsl_ctx* c) {
+gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
   cudaStream_t s = c->stream;
   const ArchSpec& a = c->a;
   const int C = c->C, B = c->B;
@@ -374,14 +421,18 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
   T* act[5];
   T* dact[5];
   for (int i = 0; i <= a.L(); ++i) { act[i] = (T*)c->d_act[i]; dact[i] = (T*)c->d_dact[i]; }
-  T* g = (T*)c->d_g;
 
-  // GPSL sampling (Eq. 1) and the gather of the sampled images
-  LAUNCH("epoch_keys", launch_epoch_keys(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
-                                         c->desc.cluster_id_base, c->seed, c->d_keys, C,
-                                         c->max_nc));
-  LAUNCH("epoch_rank", launch_epoch_rank(s, c->d_ids, c->d_off, c->d_rounds, c->d_t, c->d_keys,
-                                         c->d_perm, C, c->max_nc));
+  // GPSL sampling (Eq. 1) and the gather of the sampled images.  The epoch
+  // permutation is rebuilt only when some cluster starts an epoch; the host
+  // round count equals the device one, so other rounds skip those launches
+  // (the kernels also check the device counter themselves).
+  if (boundary) {
+    LAUNCH("epoch_keys", launch_epoch_keys(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
+                                           c->desc.cluster_id_base, c->seed, c->d_keys, C,
+                                           c->max_nc));
+    LAUNCH("epoch_rank", launch_epoch_rank(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
+                                           c->d_keys, c->d_perm, C, c->max_nc));
+  }
   LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_t, c->d_owner,
                                  c->d_labels, c->K, B, C, c->d_idx, c->d_counts, c->d_active,
                                  c->d_y));
@@ -391,12 +442,14 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
   for (int i = 0; i < a.L(); ++i) {
     const auto& L = c->tc[i];
     if (i == 0 && c->tc0.on) {
+      // one tap over the im2col: K = 32 columns
       const auto& L0 = c->tc0;
-      ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 8, L0.bw, L0.hb, L0.bb, L0.tiles_w, L0.tiles_h,
+      ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 32, L0.bw, L0.hb, L0.bb, L0.tiles_w, L0.tiles_h,
                    a.conv[0].cout, c->d_theta + a.off_b[0], P, (bf16*)(void*)act[1],
                    c->d_code[0], c->d_err};
-      LAUNCH(kFwdTc[0], launch_conv0_tc(s, L0.A, L0.B, p, a.conv[0].pool ? EPI_POOL : EPI_RELU,
-                                            C));
+      p.taps = 1;
+      LAUNCH(kFwdTc[0], launch_conv_tc(s, L0.A, L0.B, p, a.conv[0].cout, 32,
+                                       a.conv[0].pool ? EPI_POOL : EPI_RELU, C));
     } else if (L.on) {
       ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.bw, L.hb, L.bb, L.tiles_w,
                    L.tiles_h, a.conv[i].cout, c->d_theta + a.off_b[i], P,
@@ -409,19 +462,32 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
                                                  c->d_code[i], C, B, a.conv[i]));
     }
   }
-  LAUNCH("fc_fwd", launch_fc_fwd<T>(s, act[a.L()], wts + a.off_fcw, P, c->d_theta + a.off_fcb, P,
-                                    c->d_logits, C, B, a.fc_in, a.fc_out));
-  LAUNCH("softmax_ce", launch_softmax_ce(s, c->d_logits, c->d_y, c->d_loss, c->d_dlogits, C, B,
-                                         a.fc_out, c->desc.label_smoothing));
-  LAUNCH("fc_bwd", launch_fc_bwd<T>(s, c->d_dlogits, act[a.L()], wts + a.off_fcw, P,
-                                    c->d_grad + a.off_fcw, c->d_grad + a.off_fcb, P, dact[a.L()],
-                                    C, B, a.fc_in, a.fc_out));
+  LAUNCH("fc_fwd_ce", launch_fc_fwd_ce<T>(s, act[a.L()], wts + a.off_fcw, P,
+                                          c->d_theta + a.off_fcb, P, c->d_y, c->d_loss_ex,
+                                          c->d_dlogits, C, B, a.fc_in, a.fc_out,
+                                          c->desc.label_smoothing));
+  // The head hands dh straight through the last conv layer's max-pool /
+  // ReLU backward into its g; so does every tensor-core data gradient for
+  // the layer below it.  g_ready[i]: g_i has been written.
+  bool g_ready[4] = {};
+  {
+    const int l = a.L() - 1;
+    const ConvSpec& cs = a.conv[l];
+    LAUNCH("fc_bwd", launch_fc_bwd<T>(s, c->d_dlogits, c->d_loss_ex, act[a.L()], wts + a.off_fcw,
+                                      P, c->d_grad + a.off_fcw, c->d_grad + a.off_fcb, P,
+                                      (T*)c->gbuf(l), c->d_loss, C, B, a.fc_in, a.fc_out,
+                                      cs.pool ? FC_DH_POOL : FC_DH_RELU, c->d_code[l], act[a.L()],
+                                      a.out_h(l), a.out_w(l), cs.cout));
+    g_ready[l] = true;
+  }
   // backward to the cut gradient (dact[ncl]) and through the client segment
   for (int i = a.L() - 1; i >= 0; --i) {
     const auto& L = c->tc[i];
     const ConvSpec& cs = a.conv[i];
-    LAUNCH("relu_pool_bwd", launch_relu_pool_bwd<T>(s, dact[i + 1], c->d_code[i], act[i + 1], g,
-                                                    C, B, cs));
+    T* g = (T*)c->gbuf(i);
+    if (!g_ready[i])
+      LAUNCH("relu_pool_bwd", launch_relu_pool_bwd<T>(s, dact[i + 1], c->d_code[i], act[i + 1],
+                                                      g, C, B, cs));
     const auto& R = c->red[i];
     if (L.on) {
       WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
@@ -450,9 +516,16 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
     }
     if (i == 0) continue;
     if (L.on) {
+      // dx of layer i, routed into g_{i-1}; the cut gradient itself is kept
+      const ConvSpec& pv = a.conv[i - 1];
       ConvTcArgs p{cs.h, cs.w, B, cs.cout, L.bw, L.hb, L.bb, L.tiles_w, L.tiles_h, cs.cin,
-                   nullptr, 0, (bf16*)(void*)dact[i], nullptr, c->d_err};
-      LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d, EPI_STORE, C));
+                   nullptr, 0, i == a.ncl ? (bf16*)(void*)dact[i] : nullptr,
+                   pv.pool ? c->d_code[i - 1] : nullptr, c->d_err,
+                   pv.pool ? nullptr : (const bf16*)(const void*)act[i],
+                   (bf16*)c->gbuf(i - 1)};
+      LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d,
+                                         pv.pool ? EPI_DPOOL : EPI_DRELU, C));
+      g_ready[i - 1] = true;
     } else {
       LAUNCH("conv_dgrad", launch_conv_dgrad_simt<T>(s, g, wts + a.off_w[i], P, dact[i], C, B,
                                                      cs));
@@ -462,6 +535,68 @@ gcpsl_status enqueue_round(gcpsl_ctx* c) {
                            c->desc.lr, c->desc.momentum, c->desc.weight_decay,
                            c->desc.nesterov, c->d_t));
   return refresh_derived(c);
+}
+
+// One round through a CUDA graph: captured on first use of its variant
+// (epoch boundary or not; untimed or timed), then replayed.  Every launch
+// parameter is fixed for the context's lifetime (buffers, tensor maps,
+// hyper-parameters) and the round counter lives in device memory, so a
+// replay is the same round the eager path would enqueue.
+gcpsl_status run_round_graph(gcpsl_ctx* c) {
+  const bool boundary = epoch_boundary(c);
+  const int k = c->timing ? 1 + (c->timed_phase ^= 1) : 0;
+  auto& g = c->graph[boundary][k];
+  if (g.unread) {                 // event pairs of this copy's previous launch
+    c->timer.account(g.marks);
+    g.unread = false;
+  }
+  if (!g.exec) {
+    const int64_t before = c->enqueued;
+    CK(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
+    if (c->timing) c->timer.capture = &g.marks;
+    c->capturing = true;
+    gcpsl_status st = c->bf ? enqueue_round<bf16>(c, boundary) : enqueue_round<float>(c, boundary);
+    c->capturing = false;
+    c->timer.capture = nullptr;
+    cudaGraph_t graph = nullptr;
+    cudaError_t e = cudaStreamEndCapture(c->stream, &graph);
+    if (st != GCPSL_OK || e != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      for (auto& m : g.marks) { c->timer.pool.push_back(m.a); c->timer.pool.push_back(m.b); }
+      g.marks.clear();
+      if (st != GCPSL_OK) return st;
+      return fail(c, GCPSL_E_CUDA, "graph capture of a round failed: %s", cudaGetErrorString(e));
+    }
+    e = cudaGraphInstantiate(&g.exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+      g.exec = nullptr;
+      return fail(c, GCPSL_E_CUDA, "graph instantiation failed: %s", cudaGetErrorString(e));
+    }
+    g.kernels = c->enqueued - before;
+  }
+  CK(cudaGraphLaunch(g.exec, c->stream));
+  c->launched += g.kernels;
+  g.unread = c->timing;
+  return GCPSL_OK;
+}
+
+// add the event pairs of every timed graph launch not yet read
+void account_graph_marks(gcpsl_ctx* c) {
+  for (auto& v : c->graph)
+    for (auto& g : v)
+      if (g.unread) { c->timer.account(g.marks); g.unread = false; }
+}
+
+void destroy_graphs(gcpsl_ctx* c) {
+  for (auto& v : c->graph)
+    for (auto& g : v) {
+      if (g.exec) cudaGraphExecDestroy(g.exec);
+      g.exec = nullptr;
+      for (auto& m : g.marks) { cudaEventDestroy(m.a); cudaEventDestroy(m.b); }
+      g.marks.clear();
+      g.unread = false;
+    }
 }
 
 gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
@@ -492,7 +627,9 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     const ConvSpec& s = a.conv[i];
     auto& L = c->tc[i];
     L.on = false;
-    if (s.cin < 32 || s.cin % 32 || s.cout % 64 || s.w > 64 || 64 % s.w || a.off_w[i] % 8)
+    // (16-byte aligned weight rows and bias vectors)
+    if (s.cin < 32 || s.cin % 32 || s.cout % 64 || s.w > 64 || 64 % s.w || a.off_w[i] % 8 ||
+        a.off_b[i] % 4)
       continue;
     if (!m_tile(s.w, s.h, L.bw, L.hb, L.bb)) continue;
     L.whb = std::min(s.h, 64 / s.w);
@@ -538,65 +675,64 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     bool ok = tensor_map_bf16(&L.fwdA, c->d_act[i], 5, act_in, bA, L.bkc_f * 2) &&
               tensor_map_bf16_strided(&L.fwdB, c->d_shadow + a.off_w[i], 4, wf, rs, bB,
                                       L.bkc_f * 2) &&
-              tensor_map_bf16(&L.dgrA, c->d_g, 5, g_dims, dA, L.bkc_d * 2) &&
+              tensor_map_bf16(&L.dgrA, c->gbuf(i), 5, g_dims, dA, L.bkc_d * 2) &&
               tensor_map_bf16_strided(&L.dgrB, c->d_shadow + a.off_w[i], 4, wf, rs, dB,
                                       nbw * 2) &&
-              tensor_map_bf16(&L.wgA, c->d_g, 5, g_dims, wA, 128) &&
+              tensor_map_bf16(&L.wgA, c->gbuf(i), 5, g_dims, wA, 128) &&
               tensor_map_bf16(&L.wgB, c->d_act[i], 5, act_in, wB, wx * 2);
     if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for layer %d", i);
     L.on = true;
   }
   if (partial_max) DALLOC(c->d_partial, sizeof(float) * partial_max);
 
-  // the input layer (<= 8 channels): two taps per MMA step over the padded
-  // images; in bf16 mode it must run here (the input is stored padded)
+  // the input layer (3 channels): with bf16 operands the gather writes its
+  // im2col (32 columns per pixel), so its forward is a one-tap K = 32
+  // convolution and its weight gradient a GEMM over the pixels
   const ConvSpec& s0 = a.conv[0];
   auto& L0 = c->tc0;
   L0.on = false;
-  if (s0.cin > 8 || (s0.cout != 16 && s0.cout != 32 && s0.cout != 64) ||
-      !m_tile(s0.w, s0.h, L0.bw, L0.hb, L0.bb))
+  if (s0.cin != 3 || (s0.cout != 32 && s0.cout != 64) || s0.w != 32 || s0.h != 32 ||
+      a.off_b[0] % 4 || !m_tile(s0.w, s0.h, L0.bw, L0.hb, L0.bb))
     return fail(c, GCPSL_E_UNSUPPORTED, "input layer shape not supported with bf16 operands");
   L0.tiles_w = s0.w / L0.bw;
   L0.tiles_h = s0.h / L0.hb;
-  DALLOC(c->d_w0p, sizeof(bf16) * (size_t)C * 10 * s0.cout * 8);
-  const uint64_t xdims[5] = {8, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B, (uint64_t)C};
-  const uint32_t xbox[5] = {8, (uint32_t)L0.bw, (uint32_t)L0.hb, (uint32_t)L0.bb, 1};
-  const uint64_t wdims[4] = {8, (uint64_t)s0.cout, 10, (uint64_t)C};
-  const uint32_t wbox[4] = {8, (uint32_t)s0.cout, 10, 1};
-  if (!tensor_map_bf16(&L0.A, c->d_act[0], 5, xdims, xbox, 0) ||
-      !tensor_map_bf16(&L0.B, c->d_w0p, 4, wdims, wbox, 0))
+  DALLOC(c->d_w0p, sizeof(bf16) * (size_t)C * s0.cout * 32);
+  const uint64_t xdims[5] = {32, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B, (uint64_t)C};
+  const uint32_t xbox[5] = {32, (uint32_t)L0.bw, (uint32_t)L0.hb, (uint32_t)L0.bb, 1};
+  const uint64_t wdims[4] = {32, 1, (uint64_t)s0.cout, (uint64_t)C};
+  const uint32_t wbox[4] = {32, 1, (uint32_t)s0.cout, 1};
+  if (!tensor_map_bf16(&L0.A, c->d_act[0], 5, xdims, xbox, 64) ||
+      !tensor_map_bf16(&L0.B, c->d_w0p, 4, wdims, wbox, 64))
     return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input layer");
   L0.on = true;
   // its weight gradient: 64-pixel K blocks, split per replica shape only
-  L0.wg_on = false;
-  L0.whb = std::min(s0.h, 64 / s0.w);
-  L0.wbb = L0.whb > 0 ? 64 / (s0.w * L0.whb) : 0;
-  if ((s0.cout == 32 || s0.cout == 64) && s0.w <= 64 && 64 % s0.w == 0 &&
-      s0.w * L0.whb * L0.wbb == 64 && s0.h % L0.whb == 0) {
-    L0.kb_total = ((B + L0.wbb - 1) / L0.wbb) * (s0.h / L0.whb);
+  L0.whb = 64 / s0.w;
+  L0.wbb = 1;
+  L0.kb_total = B * (s0.h / L0.whb);
+  {
     const int splits = std::max(1, std::min(64, (L0.kb_total + 15) / 16));
     L0.kb_per_split = (L0.kb_total + splits - 1) / splits;
     L0.splits = (L0.kb_total + L0.kb_per_split - 1) / L0.kb_per_split;
-    const uint64_t gd[5] = {(uint64_t)s0.cout, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B,
-                            (uint64_t)C};
-    const uint32_t gb[5] = {(uint32_t)s0.cout, (uint32_t)s0.w, (uint32_t)L0.whb,
-                            (uint32_t)L0.wbb, 1};
-    const uint32_t xb[5] = {8, (uint32_t)s0.w, (uint32_t)L0.whb, (uint32_t)L0.wbb, 1};
-    if (!tensor_map_bf16(&L0.wgA, c->d_g, 5, gd, gb, s0.cout * 2) ||
-        !tensor_map_bf16(&L0.wgB, c->d_act[0], 5, xdims, xb, 0))
-      return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input-layer gradient");
-    const int64_t need = (int64_t)C * L0.splits * ((int64_t)s0.cout * 9 * s0.cin + s0.cout);
-    if (need > partial_max) {
-      partial_max = need;
-      DALLOC(c->d_partial, sizeof(float) * partial_max);
-    }
-    L0.wg_on = true;
   }
+  const uint64_t gd[5] = {(uint64_t)s0.cout, (uint64_t)s0.w, (uint64_t)s0.h, (uint64_t)B,
+                          (uint64_t)C};
+  const uint32_t gb[5] = {(uint32_t)s0.cout, (uint32_t)s0.w, (uint32_t)L0.whb, 1, 1};
+  const uint32_t xb[5] = {32, (uint32_t)s0.w, (uint32_t)L0.whb, 1, 1};
+  if (!tensor_map_bf16(&L0.wgA, c->gbuf(0), 5, gd, gb, s0.cout * 2) ||
+      !tensor_map_bf16(&L0.wgB, c->d_act[0], 5, xdims, xb, 64))
+    return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input-layer gradient");
+  const int64_t need = (int64_t)C * L0.splits * ((int64_t)s0.cout * 27 + s0.cout);
+  if (need > partial_max) {
+    partial_max = need;
+    DALLOC(c->d_partial, sizeof(float) * partial_max);
+  }
+  L0.wg_on = true;
   return GCPSL_OK;
 }
 
 void free_all(gcpsl_ctx* c) {
   if (c->stream) cudaStreamSynchronize(c->stream);
+  destroy_graphs(c);
   c->timer.destroy();
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
@@ -613,7 +749,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   c->K = K; c->C = C; c->B = B; c->F = F; c->seed = seed;
   c->bf = desc->operand_dtype == GCPSL_BF16;
   c->esz = c->bf ? 2 : 4;
-  c->x0c = c->bf ? 8 : 3;
+  c->x0c = c->bf ? 32 : 3;
   const ArchSpec& a = c->a;
   c->P = a.p_total;
   c->n = data->n;
@@ -714,7 +850,8 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     gmax = std::max(gmax, (int64_t)C * B * a.conv[i].h * a.conv[i].w * a.conv[i].cout);
   }
   DALLOC(c->d_g, c->esz * gmax);
-  DALLOC(c->d_logits, sizeof(float) * C * B * a.fc_out);
+  DALLOC(c->d_g2, c->esz * gmax);
+  DALLOC(c->d_loss_ex, sizeof(float) * C * B);
   DALLOC(c->d_dlogits, sizeof(float) * C * B * a.fc_out);
   DALLOC(c->d_y, sizeof(int32_t) * C * B);
   DALLOC(c->d_idx, sizeof(int32_t) * C * B);
@@ -738,10 +875,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     const int tiles = B * (s.h / R.tr);
     R.tiles_per_split = std::max(1, (tiles + 127) / 128);
     R.splits = (tiles + R.tiles_per_split - 1) / R.tiles_per_split;
-    R.chunk_px = 1024;
-    R.chunks = (int)(((int64_t)B * s.h * s.w + R.chunk_px - 1) / R.chunk_px);
     bpart = std::max(bpart, (int64_t)C * R.splits * ((int64_t)s.cout * 9 * s.cin + s.cout));
-    bpart = std::max(bpart, (int64_t)C * R.chunks * s.cout);
   }
   DALLOC(c->d_bpartial, sizeof(float) * bpart);
   if (c->bf) {
@@ -817,7 +951,14 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
 gcpsl_status gcpsl_step(gcpsl_ctx* c, gcpsl_step_stats* stats) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
-  st = c->bf ? enqueue_round<bf16>(c) : enqueue_round<float>(c);
+  // the first round runs eagerly (it also sets the kernels' attributes),
+  // later rounds replay captured graphs
+  if (c->use_graph && c->t > 0) {
+    st = run_round_graph(c);
+  } else {
+    st = c->bf ? enqueue_round<bf16>(c, epoch_boundary(c))
+               : enqueue_round<float>(c, epoch_boundary(c));
+  }
   if (st != GCPSL_OK) return st;
   c->t++;
   if (c->F > 0 && c->t % c->F == 0) {
@@ -987,9 +1128,41 @@ gcpsl_status gcpsl_set_timing(gcpsl_ctx* c, int enable) {
   return GCPSL_OK;
 }
 
+int64_t gcpsl_kernels_launched(const gcpsl_ctx* c) { return c ? c->launched : -1; }
+
+gcpsl_status gcpsl_set_timing_filter(gcpsl_ctx* c, const char* prefix) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  const std::string f = prefix ? prefix : "";
+  if (f == c->timer.filter) return GCPSL_OK;
+  // the timed graphs hold event nodes for the old selection: rebuild them
+  SYNC_CHECK(c);
+  account_graph_marks(c);
+  for (auto& v : c->graph)
+    for (int k = 1; k < 3; ++k) {
+      auto& g = v[k];
+      if (g.exec) cudaGraphExecDestroy(g.exec);
+      g.exec = nullptr;
+      for (auto& m : g.marks) { cudaEventDestroy(m.a); cudaEventDestroy(m.b); }
+      g.marks.clear();
+    }
+  c->timer.filter = f;
+  return GCPSL_OK;
+}
+
+gcpsl_status gcpsl_set_graph(gcpsl_ctx* c, int enable) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  SYNC_CHECK(c);
+  account_graph_marks(c);
+  c->use_graph = enable != 0;
+  return GCPSL_OK;
+}
+
 int gcpsl_kernel_times(gcpsl_ctx* c, const char** names, int64_t* launches, double* ms, int cap) {
   if (!c) return -1;
   cudaStreamSynchronize(c->stream);
+  account_graph_marks(c);
   c->timer.collect();
   const int n = (int)c->timer.names.size();
   for (int i = 0; i < n && i < cap; ++i) {
@@ -1003,6 +1176,7 @@ int gcpsl_kernel_times(gcpsl_ctx* c, const char** names, int64_t* launches, doub
 void gcpsl_reset_kernel_times(gcpsl_ctx* c) {
   if (!c) return;
   cudaStreamSynchronize(c->stream);
+  account_graph_marks(c);
   c->timer.reset();
 }
 

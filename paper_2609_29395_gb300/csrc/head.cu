@@ -5,154 +5,336 @@
 // the linear weight is stored in the same (h, w, ch) order, so it equals
 // PyTorch's (ch, h, w) flatten of an NCHW tensor with permuted weights).
 //   logits[b,j] = b_fc[j] + sum_k h[b,k] W[j,k]
-//   loss = (1/B) sum_b ( lse(logits_b) - sum_j t_bj logits_bj ),
+//   loss = (1/B) sum_b l_b,  l_b = lse(logits_b) - sum_j t_bj logits_bj,
 //     t = (1-e) onehot(y) + e/J   (label smoothing e, 0 by default)
 //   dlogits[b,j] = (softmax(logits_b)_j - t_bj) / B
 //   dW[j,k] = sum_b dlogits[b,j] h[b,k];  db[j] = sum_b dlogits[b,j]
 //   dh[b,k] = sum_j dlogits[b,j] W[j,k]
+//
+// Two launches: the forward with the per-example softmax (a block per four
+// examples, its warps on feature slices, 16-byte loads of h and W), and the
+// backward (lanes on feature pairs, warps on example chunks, all J classes
+// in registers), which also sums the per-example losses and the bias
+// gradient in a fixed order, and can hand dh straight through the last conv
+// layer's max-pool / ReLU backward.
 #include "common.cuh"
 
 namespace gcpsl {
 
 namespace {
 
-// one warp per (c, b, j); lanes stride over k; fixed shuffle tree
-template <typename T>
-__global__ void k_fc_fwd(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
-                         const float* __restrict__ bias, int64_t b_rs, float* __restrict__ logits,
-                         int C, int B, int fin, int fout) {
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (warp >= (int64_t)C * B * fout) return;
-  const int j = (int)(warp % fout);
-  const int64_t cb = warp / fout;
-  const int c = (int)(cb / B);
-  const T* hp = h + cb * fin;
-  const T* wp = w + (int64_t)c * w_rs + (int64_t)j * fin;
-  float s = 0.f;
-  for (int k = lane; k < fin; k += 32) s = fmaf(to_f(hp[k]), to_f(wp[k]), s);
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if (lane == 0) logits[warp] = s + bias[(int64_t)c * b_rs + j];
-}
+constexpr int kFwdEx = 4;          // examples per forward block
+constexpr int kFwdSlices = 8;      // warps (feature slices) per forward block
+constexpr int kBwdPairs = 32;      // feature pairs per backward block (one per lane)
+constexpr int kBwdChunks = 8;      // example chunks per backward block (one per warp)
 
-// one block per replica, one thread per example (B <= 1024)
-__global__ void k_softmax_ce(const float* __restrict__ logits, const int32_t* __restrict__ y,
-                             float* __restrict__ loss, float* __restrict__ dlogits, int B,
-                             int fout, float eps) {
-  extern __shared__ float red[];
-  const int c = blockIdx.x, b = threadIdx.x;
-  const float* z = logits + ((int64_t)c * B + b) * fout;
-  float* dz = dlogits + ((int64_t)c * B + b) * fout;
-  const int yb = y[(int64_t)c * B + b];
-  float m = z[0];
-  for (int j = 1; j < fout; ++j) m = fmaxf(m, z[j]);
-  float se = 0.f;
-  for (int j = 0; j < fout; ++j) se += expf(z[j] - m);
-  const float lse = m + logf(se);
-  float l = 0.f;
-  const float invB = 1.f / (float)B;
-  for (int j = 0; j < fout; ++j) {
-    const float t = (j == yb ? 1.f - eps : 0.f) + eps / (float)fout;
-    l += t * (lse - z[j]);
-    dz[j] = (expf(z[j] - lse) - t) * invB;
+// VEC consecutive elements starting at p, as floats (16-byte load for VEC > 1)
+template <typename T, int VEC> struct VecLoad;
+template <> struct VecLoad<bf16, 8> {
+  __device__ static void run(const bf16* p, float* o) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      o[2 * i] = __uint_as_float(w[i] << 16);
+      o[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
   }
-  // deterministic tree over a power-of-two padded block
-  int n2 = 1;
-  while (n2 < blockDim.x) n2 <<= 1;
-  red[b] = l;
-  for (int q = b + blockDim.x; q < n2; q += blockDim.x) red[q] = 0.f;
+};
+template <> struct VecLoad<float, 4> {
+  __device__ static void run(const float* p, float* o) {
+    const float4 u = *reinterpret_cast<const float4*>(p);
+    o[0] = u.x; o[1] = u.y; o[2] = u.z; o[3] = u.w;
+  }
+};
+template <typename T> struct VecLoad<T, 1> {
+  __device__ static void run(const T* p, float* o) { o[0] = to_f(p[0]); }
+};
+
+// Block = (replica c, kFwdEx consecutive examples); warp w takes the k
+// slices w, w + kFwdSlices, ... of VEC * 32 features (one slice each when
+// fin = kFwdSlices * 32 * VEC), so every load of the block is issued at
+// once.  Lane partial sums are reduced by a fixed xor tree, the warps'
+// sums in warp order; then one warp per example takes the softmax.  J is a
+// compile-time constant so the J weight loads of a slice issue together.
+template <typename T, int VEC, int J>
+__global__ void __launch_bounds__(kFwdSlices * 32)
+k_fc_fwd_ce(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
+            const float* __restrict__ bias, int64_t b_rs, const int32_t* __restrict__ y,
+            float* __restrict__ loss_ex, float* __restrict__ dlogits, int C, int B, int fin,
+            float eps) {
+  __shared__ float part[kFwdSlices][kFwdEx * J];
+  __shared__ float logit[kFwdEx][J];
+  pdl_wait();
+  pdl_trigger();
+  const int per_c = (B + kFwdEx - 1) / kFwdEx;
+  const int c = blockIdx.x / per_c, e0 = (blockIdx.x % per_c) * kFwdEx;
+  const int ne = B - e0 < kFwdEx ? B - e0 : kFwdEx;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const T* hp = h + ((int64_t)c * B + e0) * fin;
+  const T* wp = w + (int64_t)c * w_rs;
+  float acc[kFwdEx][J];
+#pragma unroll
+  for (int e = 0; e < kFwdEx; ++e)
+#pragma unroll
+    for (int j = 0; j < J; ++j) acc[e][j] = 0.f;
+  for (int k = (warp * 32 + lane) * VEC; k < fin; k += kFwdSlices * 32 * VEC) {
+    float hv[kFwdEx][VEC], wv[J][VEC];
+#pragma unroll
+    for (int e = 0; e < kFwdEx; ++e) {
+      if (e < ne) VecLoad<T, VEC>::run(hp + (int64_t)e * fin + k, hv[e]);
+      else
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) hv[e][v] = 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < J; ++j) VecLoad<T, VEC>::run(wp + (int64_t)j * fin + k, wv[j]);
+#pragma unroll
+    for (int e = 0; e < kFwdEx; ++e)
+#pragma unroll
+      for (int j = 0; j < J; ++j)
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) acc[e][j] = fmaf(hv[e][v], wv[j][v], acc[e][j]);
+  }
+#pragma unroll
+  for (int e = 0; e < kFwdEx; ++e)
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[e][j] += __shfl_xor_sync(0xffffffffu, acc[e][j], o);
+      if (lane == 0) part[warp][e * J + j] = acc[e][j];
+    }
   __syncthreads();
-  for (int st = n2 >> 1; st > 0; st >>= 1) {
-    for (int q = b; q < st; q += blockDim.x) red[q] += red[q + st];
-    __syncthreads();
+  if (threadIdx.x < kFwdEx * J) {
+    const int e = threadIdx.x / J, j = threadIdx.x % J;
+    float z = 0.f;
+#pragma unroll
+    for (int q = 0; q < kFwdSlices; ++q) z += part[q][threadIdx.x];
+    logit[e][j] = z + bias[(int64_t)c * b_rs + j];
   }
-  if (b == 0) loss[c] = red[0] * invB;
-}
-
-// dW and db: one thread per (c, j, k) (k == fin means the bias), summed over b
-template <typename T>
-__global__ void k_fc_bwd_w(const float* __restrict__ dlogits, const T* __restrict__ h,
-                           float* __restrict__ dw, float* __restrict__ db, int64_t g_rs, int C,
-                           int B, int fin, int fout) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t per = (int64_t)fout * (fin + 1);
-  if (i >= (int64_t)C * per) return;
-  const int c = (int)(i / per);
-  const int64_t r = i % per;
-  const int j = (int)(r / (fin + 1));
-  const int k = (int)(r % (fin + 1));
-  const float* dz = dlogits + (int64_t)c * B * fout + j;
-  float s = 0.f;
-  if (k == fin) {
-    for (int b = 0; b < B; ++b) s += dz[(int64_t)b * fout];
-    db[(int64_t)c * g_rs + j] = s;
-    return;
+  __syncthreads();
+  if (warp >= ne) return;
+  // softmax of example e0 + warp: every lane reads the J logits
+  float z[J];
+#pragma unroll
+  for (int j = 0; j < J; ++j) z[j] = logit[warp][j];
+  float m = z[0];
+#pragma unroll
+  for (int j = 1; j < J; ++j) m = fmaxf(m, z[j]);
+  float se = 0.f;
+#pragma unroll
+  for (int j = 0; j < J; ++j) se += expf(z[j] - m);
+  const float lse = m + logf(se);
+  const int64_t cb = (int64_t)c * B + e0 + warp;
+  const int yb = y[cb];
+  const float invB = 1.f / (float)B;
+  float l = 0.f;
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    const float t = (j == yb ? 1.f - eps : 0.f) + eps / (float)J;
+    l += t * (lse - z[j]);
+    if (lane == j) dlogits[cb * J + j] = (expf(z[j] - lse) - t) * invB;
   }
-  const T* hp = h + (int64_t)c * B * fin + k;
-  for (int b = 0; b < B; ++b) s = fmaf(dz[(int64_t)b * fout], to_f(hp[(int64_t)b * fin]), s);
-  dw[(int64_t)c * g_rs + (int64_t)j * fin + k] = s;
+  if (lane == 0) loss_ex[cb] = l;
 }
 
-// dh: one thread per (c, b, k)
+// two consecutive features as floats
+template <typename T> __device__ __forceinline__ float2 load2(const T* p);
+template <> __device__ __forceinline__ float2 load2<float>(const float* p) {
+  return *reinterpret_cast<const float2*>(p);
+}
+template <> __device__ __forceinline__ float2 load2<bf16>(const bf16* p) {
+  return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+}
+template <typename T> __device__ __forceinline__ void store2(T* p, float a, float b);
+template <> __device__ __forceinline__ void store2<float>(float* p, float a, float b) {
+  *reinterpret_cast<float2*>(p) = make_float2(a, b);
+}
+template <> __device__ __forceinline__ void store2<bf16>(bf16* p, float a, float b) {
+  *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(a, b);
+}
+
+// Where dh goes: stored as is, or routed straight into the previous conv
+// layer's g (the gradient w.r.t. its pre-activation) through that layer's
+// 2x2 max-pool (codes: position | positive << 2) or its ReLU (act > 0).
+struct HeadRoute {
+  int mode;                 // FC_DH_STORE, FC_DH_POOL, FC_DH_RELU
+  const uint8_t* code;      // FC_DH_POOL: codes, layout of h
+  const void* act;          // FC_DH_RELU: ReLU output, layout of h
+  int Ho, Wo, ch;           // h viewed as [Ho][Wo][ch]; g is [2Ho][2Wo][ch] for FC_DH_POOL
+};
+
+// dh of features (k, k+1) of example cb into dh or the routed g
 template <typename T>
-__global__ void k_fc_bwd_x(const float* __restrict__ dlogits, const T* __restrict__ w,
-                           int64_t w_rs, T* __restrict__ dh, int C, int B, int fin, int fout) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (int64_t)C * B * fin) return;
-  const int k = (int)(i % fin);
-  const int64_t cb = i / fin;
-  const int c = (int)(cb / B);
-  const float* dz = dlogits + cb * fout;
-  const T* wp = w + (int64_t)c * w_rs + k;
-  float s = 0.f;
-  for (int j = 0; j < fout; ++j) s = fmaf(dz[j], to_f(wp[(int64_t)j * fin]), s);
-  dh[i] = from_f<T>(s);
+__device__ __forceinline__ void put_dh(T* __restrict__ out, const HeadRoute& rt, int64_t cb,
+                                       int fin, int k, float d0, float d1) {
+  const int64_t o = cb * fin + k;
+  if (rt.mode == FC_DH_STORE) {
+    store2<T>(out + o, d0, d1);
+  } else if (rt.mode == FC_DH_RELU) {
+    const float2 a = load2<T>(reinterpret_cast<const T*>(rt.act) + o);
+    store2<T>(out + o, a.x > 0.f ? d0 : 0.f, a.y > 0.f ? d1 : 0.f);
+  } else {
+    const uint8_t c0 = rt.code[o], c1 = rt.code[o + 1];
+    const int cc = k % rt.ch, pix = k / rt.ch;
+    const int x = pix % rt.Wo, y = pix / rt.Wo;
+#pragma unroll
+    for (int qd = 0; qd < 4; ++qd) {
+      const int64_t go =
+          ((cb * (2 * rt.Ho) + 2 * y + (qd >> 1)) * (2 * rt.Wo) + 2 * x + (qd & 1)) * rt.ch + cc;
+      store2<T>(out + go, c0 == (4 | qd) ? d0 : 0.f, c1 == (4 | qd) ? d1 : 0.f);
+    }
+  }
 }
 
-inline unsigned blocks(int64_t n, int t) { return (unsigned)((n + t - 1) / t); }
+// grid (ceil(fin / (2 * kBwdPairs)), C).  Lane = feature pair (k, k+1),
+// warp = chunk of ceil(B / kBwdChunks) consecutive examples; the warps'
+// dW partial sums are added in warp order through shared memory.  Block
+// x == 0 also writes db (warp 0) and loss[c] (warp 1).
+template <typename T, int J>
+__global__ void __launch_bounds__(kBwdPairs * kBwdChunks)
+k_fc_bwd(const float* __restrict__ dlogits, const float* __restrict__ loss_ex,
+         const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs, float* __restrict__ dw,
+         float* __restrict__ db, int64_t g_rs, T* __restrict__ dh, float* __restrict__ loss,
+         int B, int fin, const HeadRoute rt) {
+  extern __shared__ float sm[];
+  float* sdz = sm;                                 // [B][J]
+  float* red = sm + B * J;                         // [kBwdChunks][kBwdPairs][2J]
+  pdl_wait();
+  pdl_trigger();
+  const int c = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* dz = dlogits + (int64_t)c * B * J;
+  for (int i = threadIdx.x; i < B * J; i += kBwdPairs * kBwdChunks) sdz[i] = dz[i];
+  __syncthreads();
+  const int k = 2 * (blockIdx.x * kBwdPairs + lane);
+  const int bc = (B + kBwdChunks - 1) / kBwdChunks;
+  const int b_lo = warp * bc, b_hi = b_lo + bc < B ? b_lo + bc : B;
+  float a0[J], a1[J];
+#pragma unroll
+  for (int j = 0; j < J; ++j) a0[j] = a1[j] = 0.f;
+  if (k < fin) {
+    const T* wp = w + (int64_t)c * w_rs + k;
+    float w0[J], w1[J];
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+      const float2 v = load2<T>(wp + (int64_t)j * fin);
+      w0[j] = v.x; w1[j] = v.y;
+    }
+    const T* hp = h + (int64_t)c * B * fin + k;
+    constexpr int U = 4;
+    for (int b0 = b_lo; b0 < b_hi; b0 += U) {
+      float2 hv[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        hv[u] = b0 + u < b_hi ? load2<T>(hp + (int64_t)(b0 + u) * fin) : make_float2(0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (b0 + u < b_hi) {
+          const float* g = sdz + (b0 + u) * J;
+          float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+          for (int j = 0; j < J; ++j) {
+            a0[j] = fmaf(g[j], hv[u].x, a0[j]);
+            a1[j] = fmaf(g[j], hv[u].y, a1[j]);
+            d0 = fmaf(g[j], w0[j], d0);
+            d1 = fmaf(g[j], w1[j], d1);
+          }
+          put_dh<T>(dh, rt, (int64_t)c * B + b0 + u, fin, k, d0, d1);
+        }
+      }
+    }
+  }
+  float* mine = red + (warp * kBwdPairs + lane) * 2 * J;
+#pragma unroll
+  for (int j = 0; j < J; ++j) { mine[2 * j] = a0[j]; mine[2 * j + 1] = a1[j]; }
+  __syncthreads();
+  // dW[j][k0 + pair*2 + x] = sum over chunks (in order) of the partials
+  for (int o = threadIdx.x; o < kBwdPairs * 2 * J; o += kBwdPairs * kBwdChunks) {
+    const int pr = o / (2 * J), jj = o % (2 * J);
+    const int kk = 2 * (blockIdx.x * kBwdPairs + pr) + (jj & 1);
+    if (kk >= fin) continue;
+    float sum = 0.f;
+#pragma unroll
+    for (int q = 0; q < kBwdChunks; ++q) sum += red[(q * kBwdPairs + pr) * 2 * J + jj];
+    dw[(int64_t)c * g_rs + (int64_t)(jj >> 1) * fin + kk] = sum;
+  }
+  if (blockIdx.x != 0) return;
+  if (warp == 0 && lane < J) {
+    float sum = 0.f;
+    for (int b = 0; b < B; ++b) sum += sdz[b * J + lane];
+    db[(int64_t)c * g_rs + lane] = sum;
+  } else if (warp == 1) {
+    float sum = 0.f;
+    for (int b = lane; b < B; b += 32) sum += loss_ex[(int64_t)c * B + b];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) loss[c] = sum / (float)B;
+  }
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 
 }  // namespace
 
-template <typename T>
-cudaError_t launch_fc_fwd(cudaStream_t s, const T* h, const T* w, int64_t w_rs, const float* b,
-                          int64_t b_rs, float* logits, int C, int B, int fin, int fout) {
-  const int64_t warps = (int64_t)C * B * fout;
-  k_fc_fwd<T><<<blocks(warps * 32, 256), 256, 0, s>>>(h, w, w_rs, b, b_rs, logits, C, B, fin,
-                                                       fout);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_softmax_ce(cudaStream_t s, const float* logits, const int32_t* y, float* loss,
-                              float* dlogits, int C, int B, int fout, float label_smoothing) {
-  int n2 = 1;
-  while (n2 < B) n2 <<= 1;
-  k_softmax_ce<<<C, B, n2 * sizeof(float), s>>>(logits, y, loss, dlogits, B, fout,
-                                                 label_smoothing);
-  return cudaGetLastError();
-}
+// the class count is a compile-time constant of the kernels; 10 is built
+constexpr int kClasses = 10;
 
 template <typename T>
-cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const T* h, const T* w,
-                          int64_t w_rs, float* dw, float* db, int64_t g_rs, T* dh, int C, int B,
-                          int fin, int fout) {
-  const int64_t nw = (int64_t)C * fout * (fin + 1);
-  k_fc_bwd_w<T><<<blocks(nw, 256), 256, 0, s>>>(dlogits, h, dw, db, g_rs, C, B, fin, fout);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  const int64_t nx = (int64_t)C * B * fin;
-  k_fc_bwd_x<T><<<blocks(nx, 256), 256, 0, s>>>(dlogits, w, w_rs, dh, C, B, fin, fout);
-  return cudaGetLastError();
+cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_rs,
+                             const float* b, int64_t b_rs, const int32_t* y, float* loss_ex,
+                             float* dlogits, int C, int B, int fin, int fout,
+                             float label_smoothing) {
+  if (fout != kClasses) return cudaErrorInvalidValue;
+  constexpr int VEC = 16 / (int)sizeof(T);
+  const unsigned grid = (unsigned)((int64_t)C * ((B + kFwdEx - 1) / kFwdEx));
+  // 16-byte loads need every row of h and of each replica's W on a 16-byte boundary
+  const bool vec = fin % VEC == 0 && (w_rs * (int64_t)sizeof(T)) % 16 == 0 && aligned16(h) &&
+                   aligned16(w);
+  if (vec)
+    return launch_k(k_fc_fwd_ce<T, VEC, kClasses>, grid, kFwdSlices * 32, 0, s, h, w, w_rs, b,
+                    b_rs, y, loss_ex, dlogits, C, B, fin, label_smoothing);
+  return launch_k(k_fc_fwd_ce<T, 1, kClasses>, grid, kFwdSlices * 32, 0, s, h, w, w_rs, b, b_rs,
+                  y, loss_ex, dlogits, C, B, fin, label_smoothing);
 }
 
-template cudaError_t launch_fc_fwd<float>(cudaStream_t, const float*, const float*, int64_t,
-                                          const float*, int64_t, float*, int, int, int, int);
-template cudaError_t launch_fc_fwd<bf16>(cudaStream_t, const bf16*, const bf16*, int64_t,
-                                         const float*, int64_t, float*, int, int, int, int);
+template <typename T>
+cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* loss_ex,
+                          const T* h, const T* w, int64_t w_rs, float* dw, float* db,
+                          int64_t g_rs, T* dh, float* loss, int C, int B, int fin, int fout,
+                          int route, const uint8_t* code, const T* act, int Ho, int Wo, int ch) {
+  // feature pairs: even fin and 2-element alignment of every row
+  if (fout != kClasses || fin % 2 || w_rs % 2 || g_rs % 2 ||
+      ((uintptr_t)w % (2 * sizeof(T))) || ((uintptr_t)dw % (2 * sizeof(float))))
+    return cudaErrorInvalidValue;
+  if (route != FC_DH_STORE && (ch % 2 || (int64_t)Ho * Wo * ch != fin ||
+                               (route == FC_DH_POOL && !code) || (route == FC_DH_RELU && !act)))
+    return cudaErrorInvalidValue;
+  const HeadRoute rt{route, code, act, Ho, Wo, ch};
+  const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C);
+  const size_t smem = sizeof(float) * ((size_t)B * fout + (size_t)kBwdChunks * kBwdPairs * 2 * fout);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_fc_bwd<T, kClasses>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  return launch_k(k_fc_bwd<T, kClasses>, grid, kBwdPairs * kBwdChunks, smem, s, dlogits, loss_ex,
+                  h, w, w_rs, dw, db, g_rs, dh, loss, B, fin, rt);
+}
+
+template cudaError_t launch_fc_fwd_ce<float>(cudaStream_t, const float*, const float*, int64_t,
+                                             const float*, int64_t, const int32_t*, float*,
+                                             float*, int, int, int, int, float);
+template cudaError_t launch_fc_fwd_ce<bf16>(cudaStream_t, const bf16*, const bf16*, int64_t,
+                                            const float*, int64_t, const int32_t*, float*, float*,
+                                            int, int, int, int, float);
 template cudaError_t launch_fc_bwd<float>(cudaStream_t, const float*, const float*, const float*,
-                                          int64_t, float*, float*, int64_t, float*, int, int, int,
-                                          int);
-template cudaError_t launch_fc_bwd<bf16>(cudaStream_t, const float*, const bf16*, const bf16*,
-                                         int64_t, float*, float*, int64_t, bf16*, int, int, int,
-                                         int);
+                                          const float*, int64_t, float*, float*, int64_t, float*,
+                                          float*, int, int, int, int, int, const uint8_t*,
+                                          const float*, int, int, int);
+template cudaError_t launch_fc_bwd<bf16>(cudaStream_t, const float*, const float*, const bf16*,
+                                         const bf16*, int64_t, float*, float*, int64_t, bf16*,
+                                         float*, int, int, int, int, int, const uint8_t*,
+                                         const bf16*, int, int, int);
 
 }  // namespace gcpsl

@@ -17,6 +17,8 @@ namespace {
 __global__ void k_sgd(float* __restrict__ theta, float* __restrict__ mom,
                       const float* __restrict__ grad, bf16* __restrict__ shadow, int64_t n,
                       float lr, float mu, float wd, int nesterov, int64_t* __restrict__ d_t) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
     float th = theta[i];
@@ -38,6 +40,8 @@ __global__ void k_sgd(float* __restrict__ theta, float* __restrict__ mom,
 
 __global__ void k_fuse(float* __restrict__ theta, bf16* __restrict__ shadow,
                        const float* __restrict__ q, int C, int64_t P) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += stride) {
     const float base = theta[p];
@@ -62,15 +66,13 @@ unsigned grid_for(int64_t n, int threads) {
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,
                        bf16* shadow, int64_t n, float lr, float momentum, float wd,
                        int nesterov, int64_t* d_t) {
-  k_sgd<<<grid_for(n, 256), 256, 0, s>>>(theta, mom, grad, shadow, n, lr, momentum, wd, nesterov,
-                                         d_t);
-  return cudaGetLastError();
+  return launch_k(k_sgd, grid_for(n, 256), 256, 0, s, theta, mom, grad, shadow, n, lr, momentum,
+                  wd, nesterov, d_t);
 }
 
 cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,
                         int64_t P) {
-  k_fuse<<<grid_for(P, 256), 256, 0, s>>>(theta, shadow, q, C, P);
-  return cudaGetLastError();
+  return launch_k(k_fuse, grid_for(P, 256), 256, 0, s, theta, shadow, q, C, P);
 }
 
 }  // namespace gcpsl

@@ -1,5 +1,6 @@
 // GPSL global sampling inside each cluster (Eq. 1; epoch rule of
-// Section III-A) and the gather of the sampled images.
+// Section III-A) and the gather of the sampled images (with bf16 operands,
+// straight into the input layer's im2col).
 //
 // Epoch permutation of cluster n: every example id j of the cluster gets the
 // 64-bit key (o0 << 32 | o1) of Philox4x32-10(counter = (j, epoch, n', 0),
@@ -23,6 +24,8 @@ __global__ void k_epoch_keys(const int32_t* __restrict__ ids, const int64_t* __r
                              const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
                              int cluster_base, uint32_t s0, uint32_t s1,
                              uint64_t* __restrict__ keys) {
+  pdl_wait();
+  pdl_trigger();
   const int c = blockIdx.y;
   const int64_t t = *d_t;
   const int64_t r = rounds[c];
@@ -46,6 +49,8 @@ k_epoch_rank(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
              const uint64_t* __restrict__ keys, int32_t* __restrict__ perm) {
   __shared__ uint64_t sk[kRankThreads];
   __shared__ int32_t sj[kRankThreads];
+  pdl_wait();
+  pdl_trigger();
   const int c = blockIdx.y;
   const int64_t t = *d_t;
   if (t % rounds[c] != 0) return;
@@ -77,6 +82,8 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
   int32_t* sid = sm;          // [B] ids of the round
   int32_t* sown = sm + B;     // [B] their owners
   int32_t* sorted_own = sm + 2 * B;
+  pdl_wait();
+  pdl_trigger();
   const int c = blockIdx.x;
   const int b = threadIdx.x;
   const int64_t s = *d_t % rounds[c];
@@ -99,31 +106,57 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
   if (b == 0) active[c] = first;
 }
 
-// x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w]; fp32 storage keeps 3
-// channels per pixel, bf16 storage pads each pixel to 8 channels (16 bytes,
-// channels 3..7 zero) for the tensor-core input layer
-template <typename T>
-__global__ void k_gather(const float* __restrict__ images, const int32_t* __restrict__ idx,
-                         int CB, T* __restrict__ x0) {
+// fp32 storage: x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w] (3 channels).
+__global__ void k_gather_f32(const float* __restrict__ images, const int32_t* __restrict__ idx,
+                             int CB, float* __restrict__ x0) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (int64_t)CB * 1024) return;
   const int64_t cb = i >> 10;
   const int p = (int)(i & 1023);
   const float* src = images + (int64_t)idx[cb] * 3072 + p;
-  const float r = src[0], g = src[1024], b = src[2048];
-  if (sizeof(T) == 2) {
-    __align__(16) T v[8];
-    v[0] = from_f<T>(r);
-    v[1] = from_f<T>(g);
-    v[2] = from_f<T>(b);
+  float* dst = x0 + i * 3;
+  dst[0] = src[0];
+  dst[1] = src[1024];
+  dst[2] = src[2048];
+}
+
+// bf16 storage: the input layer's im2col, x0[c][b][y][x][32] with column
+// k = tap * 3 + ch (tap = 3 ky + kx) = image[ch][y + ky - 1][x + kx - 1]
+// (0 outside the image), k = 27 = 1 (its weight-gradient column is the
+// bias gradient) and k = 28..31 = 0.  One block per sampled image: the
+// image is staged with a zero border in shared memory, then every thread
+// writes 16-byte groups of 8 columns (a warp writes 512 contiguous bytes).
+constexpr int kIm2colThreads = 256;
+__global__ void __launch_bounds__(kIm2colThreads)
+k_gather_im2col(const float* __restrict__ images, const int32_t* __restrict__ idx,
+                bf16* __restrict__ x0) {
+  __shared__ float tile[3][34][34];
+  pdl_wait();
+  pdl_trigger();
+  const int64_t cb = blockIdx.x;
+  const float* src = images + (int64_t)idx[cb] * 3072;
+  for (int i = threadIdx.x; i < 3 * 34 * 34; i += kIm2colThreads) {
+    const int ch = i / (34 * 34), yy = (i / 34) % 34, xx = i % 34;
+    const bool in = yy >= 1 && yy <= 32 && xx >= 1 && xx <= 32;
+    tile[ch][yy][xx] = in ? src[ch * 1024 + (yy - 1) * 32 + (xx - 1)] : 0.f;
+  }
+  __syncthreads();
+  uint4* dst = reinterpret_cast<uint4*>(x0 + cb * 1024 * 32);
+  for (int q = threadIdx.x; q < 1024 * 4; q += kIm2colThreads) {
+    const int pix = q >> 2, g = q & 3, y = pix >> 5, x = pix & 31;
+    float v[8];
 #pragma unroll
-    for (int k = 3; k < 8; ++k) v[k] = from_f<T>(0.f);
-    reinterpret_cast<uint4*>(x0)[i] = *reinterpret_cast<uint4*>(v);
-  } else {
-    T* dst = x0 + i * 3;
-    dst[0] = from_f<T>(r);
-    dst[1] = from_f<T>(g);
-    dst[2] = from_f<T>(b);
+    for (int e = 0; e < 8; ++e) {
+      const int k = 8 * g + e;
+      const int tap = k / 3, ch = k - 3 * tap;
+      v[e] = k < 27 ? tile[ch][y + tap / 3][x + tap % 3] : (k == 27 ? 1.f : 0.f);
+    }
+    __align__(16) bf16 h[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) h[e] = __float2bfloat16_rn(v[e]);
+    dst[q] = *reinterpret_cast<const uint4*>(h);
   }
 }
 
@@ -133,35 +166,35 @@ cudaError_t launch_epoch_keys(cudaStream_t s, const int32_t* ids, const int64_t*
                               const int32_t* rounds, const int64_t* d_t, int cluster_base,
                               uint64_t seed, uint64_t* keys, int C, int64_t max_nc) {
   dim3 grid((unsigned)((max_nc + 255) / 256), (unsigned)C);
-  k_epoch_keys<<<grid, 256, 0, s>>>(ids, off, rounds, d_t, cluster_base, (uint32_t)seed,
-                                    (uint32_t)(seed >> 32), keys);
-  return cudaGetLastError();
+  return launch_k(k_epoch_keys, grid, 256, 0, s, ids, off, rounds, d_t, cluster_base,
+                  (uint32_t)seed, (uint32_t)(seed >> 32), keys);
 }
 
 cudaError_t launch_epoch_rank(cudaStream_t s, const int32_t* ids, const int64_t* off,
                               const int32_t* rounds, const int64_t* d_t, const uint64_t* keys,
                               int32_t* perm, int C, int64_t max_nc) {
   dim3 grid((unsigned)((max_nc + kRankThreads - 1) / kRankThreads), (unsigned)C);
-  k_epoch_rank<<<grid, kRankThreads, 0, s>>>(ids, off, rounds, d_t, keys, perm);
-  return cudaGetLastError();
+  return launch_k(k_epoch_rank, grid, kRankThreads, 0, s, ids, off, rounds, d_t, keys, perm);
 }
 
 cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* off,
                           const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
                           const int32_t* labels, int K, int B, int C, int32_t* idx,
                           int32_t* counts, int32_t* active, int32_t* y) {
-  k_sample<<<C, B, 3 * B * sizeof(int32_t), s>>>(perm, off, rounds, d_t, owner, labels, K, B,
-                                                  idx, counts, active, y);
-  return cudaGetLastError();
+  return launch_k(k_sample, C, B, 3 * B * sizeof(int32_t), s, perm, off, rounds, d_t, owner,
+                  labels, K, B, idx, counts, active, y);
 }
 
-template <typename T>
-cudaError_t launch_gather(cudaStream_t s, const float* images, const int32_t* idx, int CB, T* x0) {
-  int64_t n = (int64_t)CB * 1024;
-  k_gather<T><<<(unsigned)((n + 255) / 256), 256, 0, s>>>(images, idx, CB, x0);
-  return cudaGetLastError();
+template <>
+cudaError_t launch_gather<float>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
+                                 float* x0) {
+  const int64_t n = (int64_t)CB * 1024;
+  return launch_k(k_gather_f32, (unsigned)((n + 255) / 256), 256, 0, s, images, idx, CB, x0);
 }
-template cudaError_t launch_gather<float>(cudaStream_t, const float*, const int32_t*, int, float*);
-template cudaError_t launch_gather<bf16>(cudaStream_t, const float*, const int32_t*, int, bf16*);
+template <>
+cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
+                                bf16* x0) {
+  return launch_k(k_gather_im2col, (unsigned)CB, kIm2colThreads, 0, s, images, idx, x0);
+}
 
 }  // namespace gcpsl

@@ -240,6 +240,28 @@ def test_rerun_is_deterministic():
     assert (runs[0][0] == runs[1][0]).all() and (runs[0][1] == runs[1][1]).all()
 
 
+def test_graph_replay_equals_eager_bit_exact():
+    """Rounds replayed from CUDA graphs (timed and untimed copies, across an
+    epoch boundary and fusions) equal eagerly launched rounds bit for bit."""
+    ds, assign, params = _splitcnn_small(C=2, n=640, K=16)
+    runs = []
+    for graph in (False, True):
+        g = pkg.Context(1, 16, 2, assign, 32, 4, 4, ds.images, ds.labels, ds.owner, params,
+                        bf16=True, momentum=0.9)
+        g.set_graph(graph)
+        losses = []
+        for t in range(11):
+            g.set_timing(t % 3 == 1)        # alternate timed / untimed variants
+            losses.append(g.step(stats=True)[0])
+        kt = g.kernel_times()
+        runs.append((np.stack([g.all_params(n) for n in range(2)]),
+                     np.stack([g.momentum(n) for n in range(2)]), g.cut(1), np.array(losses)))
+        g.close()
+        assert sum(n for n, _ in kt.values()) > 0
+    for a, b in zip(runs[0], runs[1]):
+        assert (a == b).all()
+
+
 def test_fusion_matches_eq5():
     """Explicit fusion of diverged replicas: Eq. 5 with the context's q."""
     ds, assign, params = _splitcnn_small(C=4, n=4096, K=32)
