@@ -424,23 +424,27 @@ __global__ void k_pack_w0(const bf16* __restrict__ w, bf16* __restrict__ w0p, in
 // into every ring stage), so its accumulator also yields the bias gradient
 // sum_p g[p][co]; groups g >= 1 hold TG taps each.  The fp32 partial of a
 // split is laid out like the parameters, [cout][9][cin] then [cout].
-template <int BN>
+// MT = 128 output channels per tile (two 64-wide g blocks), or MT = 64 for
+// layers with 64 output channels (M = 64 MMAs: row r of the accumulator is
+// TMEM lane 32 * (r / 16) + r % 16).
+template <int BN, int MT>
 struct WgCfg {
   static constexpr int BKP = 64;                         // pixels per stage
   static constexpr int TG = 256 / BN;                    // taps per CTA
-  static constexpr int A_BYTES = 2 * 64 * BKP * 2;       // 128 co (two 64-wide blocks)
+  static constexpr int A_BYTES = MT * BKP * 2;           // MT co (64-wide blocks)
   static constexpr int TAP_BYTES = BN * BKP * 2;         // one tap's x tile
   static constexpr int STAGE = A_BYTES + TG * TAP_BYTES;
-  static constexpr int S = 4;
+  static constexpr int S0 = 200 * 1024 / STAGE;
+  static constexpr int S = S0 > 6 ? 6 : S0;
   static constexpr int SMEM = 1024 + S * STAGE;
   static constexpr uint32_t TCOLS = 256;
 };
 
-template <int BN>
+template <int BN, int MT>
 __global__ void __launch_bounds__(kThreads, 1)
 k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tX,
            const WgradTcArgs p) {
-  using Cfg = WgCfg<BN>;
+  using Cfg = WgCfg<BN, MT>;
   constexpr int S = Cfg::S, TG = Cfg::TG;
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = align1024(smraw);
@@ -450,10 +454,10 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, c = blockIdx.z;
   const int ci_tiles = p.cin / BN;
-  const int co_tiles = (p.cout + 127) / 128;
+  const int co_tiles = (p.cout + MT - 1) / MT;
   int t = blockIdx.y;
   const int ci0 = (t % ci_tiles) * BN; t /= ci_tiles;
-  const int co0 = (t % co_tiles) * 128; t /= co_tiles;
+  const int co0 = (t % co_tiles) * MT; t /= co_tiles;
   const int grp = t;                                 // tap group
   const bool bias_grp = grp == 0;
   const int tap0 = bias_grp ? 0 : (TG - 1) + (grp - 1) * TG;
@@ -501,10 +505,12 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
         uint8_t* sb = sa + Cfg::A_BYTES;
         mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + ntaps * Cfg::TAP_BYTES);
         tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, c);
-        // rows 64..127 of the M tile: the next 64 channels, or (cout <= 64) a
-        // second copy of the first block whose results the epilogue drops
-        tma_load_5d(sa + 64 * Cfg::BKP * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0, 0,
-                    h, b, c);
+        // rows 64..127 of an MT = 128 tile: the next 64 channels, or (cout
+        // < co0 + 128) a second copy of the first block whose results the
+        // epilogue drops
+        if (MT == 128)
+          tma_load_5d(sa + 64 * Cfg::BKP * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0,
+                      0, h, b, c);
         for (int tj = 0; tj < ntaps; ++tj) {
           const int tap = tap0 + tj, kh = tap / 3, kw = tap % 3;
 #pragma unroll
@@ -519,7 +525,7 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
       // one MMA per k step with N = ntaps*BN: the taps' x tiles are the
       // consecutive MN-major N blocks of one B operand (64-ci blocks, SW128,
       // or 32-ci blocks of 64-byte rows, SW64), `b_blk` bytes apart
-      const uint32_t idesc = idesc_bf16(BM, nslots * BN, 1, 1);
+      const uint32_t idesc = idesc_bf16(MT, nslots * BN, 1, 1);
       constexpr uint32_t a_lbo = 64 * Cfg::BKP * 2;
       constexpr uint32_t b_swz = BN >= 64 ? SWZ_128 : SWZ_64;
       constexpr uint32_t b_row = BN >= 64 ? 128 : 64;
@@ -539,7 +545,10 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     }
   } else {
     const int q = warp & 3;
-    const int co = co0 + q * 32 + lane;
+    // accumulator row of this thread's TMEM lane (M = 64: lanes 16..31 of
+    // each quarter are unused)
+    const int co = co0 + (MT == 128 ? q * 32 + lane : q * 16 + lane);
+    const bool mine = (MT == 128 || lane < 16) && co < p.cout;
     const bool ok = mbar_wait(&done, 0);
     if (!ok) atomicOr(p.err, 32);
     tc_fence_after();
@@ -549,7 +558,7 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
       float v[16];
       tmem_ld16(trow + (TG - 1) * BN, v);
       tmem_ld_wait();
-      if (co < p.cout) part[p.cout * 9 * p.cin + co] = nkb ? v[0] : 0.f;
+      if (mine) part[p.cout * 9 * p.cin + co] = nkb ? v[0] : 0.f;
     }
     for (int tj = 0; tj < ntaps; ++tj) {
       float* dst = part + (int64_t)co * 9 * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
@@ -558,7 +567,7 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
         float v[16];
         tmem_ld16(trow + tj * BN + c0, v);
         tmem_ld_wait();
-        if (co < p.cout) {
+        if (mine) {
           float4* d4 = reinterpret_cast<float4*>(dst + c0);
 #pragma unroll
           for (int i = 0; i < 4; ++i)
@@ -746,18 +755,18 @@ cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
                   tiles_n, items);
 }
 
-template <int BN>
+template <int BN, int MT>
 cudaError_t launch_wgrad_inst(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                               const WgradTcArgs& p, dim3 grid) {
-  using Cfg = WgCfg<BN>;
+  using Cfg = WgCfg<BN, MT>;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_wgrad_tc<BN>,
+    cudaError_t e = cudaFuncSetAttribute(k_wgrad_tc<BN, MT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  return launch_k(k_wgrad_tc<BN>, grid, kThreads, Cfg::SMEM, s, g, x, p);
+  return launch_k(k_wgrad_tc<BN, MT>, grid, kThreads, Cfg::SMEM, s, g, x, p);
 }
 
 }  // namespace
@@ -875,11 +884,18 @@ cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensor
                             const WgradTcArgs& p, int bn, int C) {
   const int tg = 256 / bn;                            // slots per CTA
   const int groups = 1 + (9 - (tg - 1) + tg - 1) / tg;
-  const int tiles = groups * (p.cin / bn) * ((p.cout + 127) / 128);
+  const int mt = p.cout % 128 == 0 ? 128 : 64;
+  const int tiles = groups * (p.cin / bn) * ((p.cout + mt - 1) / mt);
   dim3 grid(p.splits, tiles, C);
-  if (bn == 32) return launch_wgrad_inst<32>(s, g, x, p, grid);
-  if (bn == 64) return launch_wgrad_inst<64>(s, g, x, p, grid);
-  if (bn == 128) return launch_wgrad_inst<128>(s, g, x, p, grid);
+  if (mt == 64) {
+    if (bn == 32) return launch_wgrad_inst<32, 64>(s, g, x, p, grid);
+    if (bn == 64) return launch_wgrad_inst<64, 64>(s, g, x, p, grid);
+    if (bn == 128) return launch_wgrad_inst<128, 64>(s, g, x, p, grid);
+    return cudaErrorInvalidValue;
+  }
+  if (bn == 32) return launch_wgrad_inst<32, 128>(s, g, x, p, grid);
+  if (bn == 64) return launch_wgrad_inst<64, 128>(s, g, x, p, grid);
+  if (bn == 128) return launch_wgrad_inst<128, 128>(s, g, x, p, grid);
   return cudaErrorInvalidValue;
 }
 

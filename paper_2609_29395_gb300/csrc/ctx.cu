@@ -645,7 +645,8 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     if (s.cout % L.bn_f || s.cin % L.bn_d || s.cin % L.bkc_f || s.cin % L.bn_w) continue;
     const int tg = 256 / L.bn_w;                      // slots per weight-gradient CTA
     const int groups = 1 + (9 - (tg - 1) + tg - 1) / tg;
-    const int tiles = groups * (s.cin / L.bn_w) * ((s.cout + 127) / 128);
+    const int mt = s.cout % 128 == 0 ? 128 : 64;      // output channels per tile
+    const int tiles = groups * (s.cin / L.bn_w) * ((s.cout + mt - 1) / mt);
     L.kb_total = ((B + L.wbb - 1) / L.wbb) * (s.h / L.whb);
     // the split (hence the summation order) depends on the per-replica shape
     // only, so C grouped replicas reproduce C one-replica runs bit for bit

@@ -302,3 +302,50 @@ def test_splitcnn_c4_full_size():
         perm = oracle.epoch_perm(ids, m, 0, 4)
         idx, counts, act = oracle.sample_round(perm, 1, w.B, ds.owner, w.num_clients)
         assert (gi[m] == idx).all() and (gc[m] == counts).all() and active[m] == act
+
+
+def _first_round_per_cluster(name, clusters):
+    """A full-size workload in the benchmarked launch configuration: the
+    GPU takes its first round with every cluster; selected clusters are
+    re-run alone by the oracle (a one-cluster context with the same cluster
+    id, so the same Philox stream) and compared slice by slice."""
+    w = configs.WORKLOADS[name]
+    ds, assign, params = configs.build_inputs(w)
+    gpu = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
+                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=True)
+    loss, active = gpu.step(stats=True)
+    gi, gc = gpu.sample()
+    assert (gc.sum(1) == w.B).all()
+    cut_act = gpu.cut(pkg.binding.GCPSL_CUT_ACT)
+    cut_grad = gpu.cut(pkg.binding.GCPSL_CUT_GRAD)
+    for m in clusters:
+        sub = np.where(assign == m, 0, -1).astype(np.int32)
+        orc = oracle.Oracle(w.arch, w.num_clients, 1, sub, w.B, w.F, 4, ds.images, ds.labels,
+                            ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=True,
+                            cluster_base=m)
+        orc.set_tie_tol(DECISION_TOL[True])
+        orc.step()
+        oi, oc = orc.sample()
+        assert (gi[m] == oi[0]).all() and (gc[m] == oc[0]).all(), f"cluster {m}: sample"
+        ol, oa = orc.stats()
+        assert active[m] == oa[0]
+        assert abs(loss[m] - ol[0]) < LOSS_ABS, (m, loss[m], ol[0])
+        assert rel_l2(cut_act[m], orc.cut(0).reshape(cut_act[m].shape)) < REL_L2
+        assert check_decisions(gpu, orc, w.arch, gpu_clusters=[m]) > 0.9
+        assert rel_l2(cut_grad[m], orc.cut(1).reshape(cut_grad[m].shape)) < REL_L2
+        gp, op = gpu.all_params(m), orc.all_params(0)
+        assert rel_l2(gp, op) < REL_L2, ("params", m)
+        assert rel_l2(gp - params, op - params) < REL_L2, ("update", m)
+        del orc
+    gpu.close()
+
+
+def test_splitcnn_c16_full_size_sampled_clusters():
+    """C=16 size-balanced clusters (50,000 images, K=256, B=64)."""
+    _first_round_per_cluster("splitcnn_c16", [0, 7, 15])
+
+
+def test_splitcnn_c64_full_size_sampled_clusters():
+    """C=64 label-aware clusters (50,000 images, K=256, B=64): many small
+    replica GEMMs in one grouped launch."""
+    _first_round_per_cluster("splitcnn_c64", [0, 21, 42, 63])
