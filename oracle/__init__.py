@@ -1,4 +1,4 @@
-"""ctypes wrapper of the CPU oracle (``gcpsl_oracle.c``).
+"""ctypes wrapper of the CPU oracle (``gcpsl_oracle.c``, ``gcpsl_resnet.c``).
 
 TEST INFRASTRUCTURE ONLY: imported by the tests, the smoke check and the CPU
 baseline leg of the benchmark, never by the product package.  The oracle is a
@@ -17,16 +17,17 @@ import numpy as np
 HERE = Path(__file__).resolve().parent
 LIBDIR = HERE / "lib"
 LIB = LIBDIR / "libgcpsl_oracle.so"
-SRC = HERE / "gcpsl_oracle.c"
+SRCS = [HERE / "gcpsl_oracle.c", HERE / "gcpsl_resnet.c"]
 
 
 def build(force: bool = False) -> Path:
     """Compile the oracle with gcc (OpenMP when available)."""
-    if LIB.exists() and not force and LIB.stat().st_mtime >= SRC.stat().st_mtime:
+    if LIB.exists() and not force and all(LIB.stat().st_mtime >= s.stat().st_mtime for s in SRCS):
         return LIB
     LIBDIR.mkdir(exist_ok=True)
     tmp = LIBDIR / f".tmp_{os.getpid()}.so"
-    base = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", str(SRC), "-o", str(tmp), "-lm"]
+    base = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared"] + [str(s) for s in SRCS] + [
+        "-o", str(tmp), "-lm"]
     try:
         subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True, capture_output=True)
     except subprocess.CalledProcessError:
@@ -84,6 +85,11 @@ def _declare(L):
     L.orc_get_pool_cand.restype = ct.c_int64
     L.orc_get_ties.argtypes = [ct.c_void_p, i32p]
     L.orc_get_ties.restype = None
+    L.orc_set_bn_state.argtypes = [ct.c_void_p, ct.c_int, f64p]
+    L.orn_forward_backward.argtypes = [ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p, i32p,
+                                       f64p, f64p, f64p, f64p, f64p]
+    L.orn_init_bn_state.argtypes = [f64p]
+    L.orn_init_bn_state.restype = None
     L.orc_set_threads.argtypes = [ct.c_int]
     L.orc_get_threads.restype = ct.c_int
 
@@ -121,6 +127,47 @@ def num_params(arch: int, segment: int) -> int:
     return int(lib().orc_num_params(arch, segment))
 
 
+RESNET18 = 2
+
+
+def bn_state_size() -> int:
+    """BatchNorm running statistics per replica of the ResNet-18 split."""
+    return num_params(RESNET18, 2)
+
+
+def initial_bn_state():
+    out = np.zeros(bn_state_size())
+    lib().orn_init_bn_state(_ptr(out, ct.c_double))
+    return out
+
+
+def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False,
+                            label_smoothing: float = 0.0, want_grad: bool = True):
+    """ResNet-18 split: (loss, grad[P] or None, cut_act, cut_grad, logits, bn_state
+    after this batch's update of the running statistics)."""
+    params = np.ascontiguousarray(params, dtype=np.float64)
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    labels = np.ascontiguousarray(labels, dtype=np.int32)
+    B = labels.size
+    P = num_params(RESNET18, 0) + num_params(RESNET18, 1)
+    bn = np.ascontiguousarray(initial_bn_state() if bn_state is None else bn_state,
+                              dtype=np.float64).copy()
+    loss = np.zeros(1)
+    grad = np.zeros(P) if want_grad else None
+    ncut = _cut_elems(RESNET18, B)
+    ca, cg = np.zeros(ncut), np.zeros(ncut)
+    logits = np.zeros(B * 10)
+    rc = lib().orn_forward_backward(int(bf16), label_smoothing, _ptr(params, ct.c_double),
+                                    _ptr(bn, ct.c_double), B, _ptr(x, ct.c_double),
+                                    _ptr(labels, ct.c_int32), _ptr(loss, ct.c_double),
+                                    _ptr(grad, ct.c_double) if want_grad else None,
+                                    _ptr(ca, ct.c_double), _ptr(cg, ct.c_double),
+                                    _ptr(logits, ct.c_double))
+    if rc:
+        raise RuntimeError(f"oracle resnet forward_backward failed: {rc}")
+    return float(loss[0]), grad, ca, cg, logits.reshape(B, 10), bn
+
+
 def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smoothing: float = 0.0,
                      want_grad: bool = True):
     """(loss, grad[P] or None, cut_act, cut_grad, logits) for one replica."""
@@ -146,11 +193,11 @@ def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smo
 
 
 def _cut_elems(arch: int, B: int) -> int:
-    return B * {0: 16 * 16 * 16, 1: 64 * 16 * 16}[arch]
+    return B * {0: 16 * 16 * 16, 1: 64 * 16 * 16, 2: 64 * 32 * 32}[arch]
 
 
 def cut_shape(arch: int):
-    return {0: (16, 16, 16), 1: (64, 16, 16)}[arch]
+    return {0: (16, 16, 16), 1: (64, 16, 16), 2: (64, 32, 32)}[arch]
 
 
 def fuse_arrays(q, theta):
@@ -220,6 +267,19 @@ class Oracle:
     def set_params(self, cluster: int, blob):
         blob = np.ascontiguousarray(blob, dtype=np.float64)
         lib().orc_set_params(self._h, cluster, _ptr(blob, ct.c_double))
+
+    def bn_state(self, cluster: int):
+        """BatchNorm running statistics of one replica (ResNet-18 split)."""
+        out = np.zeros(bn_state_size())
+        rc = lib().orc_get_params(self._h, cluster, 2, _ptr(out, ct.c_double))
+        if rc:
+            raise ValueError("no BatchNorm state for this architecture")
+        return out
+
+    def set_bn_state(self, cluster: int, v):
+        v = np.ascontiguousarray(v, dtype=np.float64)
+        if lib().orc_set_bn_state(self._h, cluster, _ptr(v, ct.c_double)):
+            raise ValueError("no BatchNorm state for this architecture")
 
     def momentum(self, cluster: int):
         out = np.zeros(self.P_client + self.P_server)

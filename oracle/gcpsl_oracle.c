@@ -40,6 +40,15 @@
 #include <omp.h>
 #endif
 
+/* the CIFAR ResNet-18 split model (architecture 2), gcpsl_resnet.c */
+int64_t orn_num_params(int segment);
+int orn_forward_backward(int bf16, double label_smoothing, const double* params,
+                         double* bn_state, int B, const double* x, const int32_t* labels,
+                         double* loss_out, double* grad, double* cut_act, double* cut_grad,
+                         double* logits_out);
+void orn_init_bn_state(double* state);
+#define ORC_RESNET18 2
+
 #define ORC_OK 0
 #define ORC_EINVAL 1
 #define ORC_ENOMEM 2
@@ -165,6 +174,7 @@ static void get_offs(const arch_t* a, offs_t* o) {
 }
 
 int64_t orc_num_params(int arch, int segment) {
+  if (arch == ORC_RESNET18) return orn_num_params(segment);
   arch_t a; offs_t o;
   if (get_arch(arch, &a)) return -1;
   get_offs(&a, &o);
@@ -528,6 +538,9 @@ typedef struct {
   int64_t ncut;
   work_t w;
   double* xbuf; int32_t* ybuf;
+  int resnet;                                 /* architecture 2 */
+  int64_t S;                                  /* BatchNorm state per replica (resnet) */
+  double* bn;                                 /* [C][S] running mean / var */
   double tie_tol;                             /* see relu_pool_fwd */
   uint8_t* cand[4];                           /* [C][B][cout][Ho][Wo] of the last round */
   int32_t* ties;                              /* [C][B] ambiguous windows per example */
@@ -541,7 +554,9 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
              const int32_t* owner, int64_t n, const float* init_params, orc_ctx** out) {
   *out = NULL;
   arch_t a;
-  if (get_arch(arch, &a)) return ORC_EUNSUPPORTED;
+  memset(&a, 0, sizeof(a));
+  const int resnet = arch == ORC_RESNET18;
+  if (!resnet && get_arch(arch, &a)) return ORC_EUNSUPPORTED;
   if (K <= 0 || C <= 0 || B <= 0 || F < 0 || n <= 0 || !assignment || !images || !labels ||
       !owner || !init_params)
     return ORC_EINVAL;
@@ -552,7 +567,16 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   c->arch = arch; c->bf16 = bf16; c->K = K; c->C = C; c->B = B; c->F = F;
   c->nesterov = nesterov; c->cluster_base = cluster_base;
   c->lr = lr; c->momentum = momentum; c->wd = wd; c->ls = label_smoothing; c->seed = seed;
-  c->a = a; get_offs(&a, &c->o);
+  c->a = a;
+  c->resnet = resnet;
+  if (resnet) {
+    memset(&c->o, 0, sizeof(c->o));
+    c->o.p_client = orn_num_params(0);
+    c->o.p_total = c->o.p_client + orn_num_params(1);
+    c->S = orn_num_params(2);
+  } else {
+    get_offs(&a, &c->o);
+  }
   c->n = n;
   c->images_src = images;        /* read-only, caller keeps it alive */
   c->labels = (int32_t*)malloc(sizeof(int32_t) * (size_t)n);
@@ -590,7 +614,7 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   c->counts = (int32_t*)calloc((size_t)C * K, sizeof(int32_t));
   c->loss = (double*)calloc((size_t)C, sizeof(double));
   c->active = (int32_t*)calloc((size_t)C, sizeof(int32_t));
-  c->ncut = conv_out_elems(&a.conv[a.ncl - 1], B);
+  c->ncut = resnet ? (int64_t)B * 64 * 1024 : conv_out_elems(&a.conv[a.ncl - 1], B);
   c->cut_act = (double*)calloc((size_t)(C * c->ncut), sizeof(double));
   c->cut_grad = (double*)calloc((size_t)(C * c->ncut), sizeof(double));
   c->ybuf = (int32_t*)calloc((size_t)B, sizeof(int32_t));
@@ -599,8 +623,14 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
     if (a.conv[i].pool)
       c->cand[i] = (uint8_t*)calloc((size_t)C * conv_out_elems(&a.conv[i], B), 1);
   c->ties = (int32_t*)calloc((size_t)C * B, sizeof(int32_t));
+  if (resnet) {
+    c->xbuf = (double*)calloc((size_t)B * 3072, sizeof(double));
+    c->bn = (double*)calloc((size_t)(C * c->S > 0 ? C * c->S : 1), sizeof(double));
+    if (!c->xbuf || !c->bn) { orc_destroy(c); return ORC_ENOMEM; }
+    for (int k = 0; k < C; ++k) orn_init_bn_state(c->bn + k * c->S);
+  }
   if (!c->theta || !c->mom || !c->grad || !c->cut_act || !c->cut_grad ||
-      work_alloc(&c->w, &a, &c->o, B)) { orc_destroy(c); return ORC_ENOMEM; }
+      (!resnet && work_alloc(&c->w, &a, &c->o, B))) { orc_destroy(c); return ORC_ENOMEM; }
   *out = c;
   return ORC_OK;
 }
@@ -611,7 +641,7 @@ void orc_destroy(orc_ctx* c) {
   free(c->ids); free(c->perm); free(c->nc); free(c->cur_epoch); free(c->q);
   free(c->labels); free(c->owner); free(c->theta); free(c->mom); free(c->grad);
   free(c->idx); free(c->counts); free(c->loss); free(c->active);
-  free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties);
+  free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties); free(c->xbuf); free(c->bn);
   for (int i = 0; i < 4; ++i) free(c->cand[i]);
   work_free(&c->w);
   free(c);
@@ -625,6 +655,13 @@ int orc_fuse(orc_ctx* c) {
   orc_fuse_arrays(c->C, P, c->q, c->theta, f);
   for (int k = 0; k < c->C; ++k) memcpy(c->theta + k * P, f, sizeof(double) * (size_t)P);
   free(f);
+  if (c->resnet && c->S > 0) {            /* BatchNorm running statistics, same q */
+    double* g = (double*)malloc(sizeof(double) * (size_t)c->S);
+    if (!g) return ORC_ENOMEM;
+    orc_fuse_arrays(c->C, c->S, c->q, c->bn, g);
+    for (int k = 0; k < c->C; ++k) memcpy(c->bn + k * c->S, g, sizeof(double) * (size_t)c->S);
+    free(g);
+  }
   return ORC_OK;
 }
 
@@ -657,6 +694,19 @@ int orc_step(orc_ctx* c) {
     int32_t* idx = c->idx + (int64_t)k * B;
     c->active[k] = orc_sample_round(c->perm[k], s, B, c->owner, c->K, idx,
                                     c->counts + (int64_t)k * c->K);
+    if (c->resnet) {
+      for (int b = 0; b < B; ++b) {
+        const float* src = c->images_src + (int64_t)idx[b] * 3072;
+        for (int i = 0; i < 3072; ++i) c->xbuf[(int64_t)b * 3072 + i] = (double)src[i];
+        c->ybuf[b] = c->labels[idx[b]];
+      }
+      int64_t P = c->o.p_total;
+      int rc = orn_forward_backward(c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B,
+                                    c->xbuf, c->ybuf, &c->loss[k], c->grad + k * P,
+                                    c->cut_act + k * c->ncut, c->cut_grad + k * c->ncut, NULL);
+      if (rc) return rc;
+      continue;
+    }
     for (int b = 0; b < B; ++b) {
       const float* src = c->images_src + (int64_t)idx[b] * 3072;
       for (int i = 0; i < 3072; ++i) c->w.act[0][(int64_t)b * 3072 + i] = (double)src[i];
@@ -686,9 +736,15 @@ int orc_step(orc_ctx* c) {
   return ORC_OK;
 }
 
-/* segment 0 = client, 1 = server; dst gets fp64 canonical-order values */
+/* segment 0 = client, 1 = server, 2 = BatchNorm state (resnet); dst gets
+ * fp64 canonical-order values */
 int orc_get_params(const orc_ctx* c, int cluster, int segment, double* dst) {
   if (cluster < 0 || cluster >= c->C) return ORC_EINVAL;
+  if (segment == 2) {
+    if (!c->resnet) return ORC_EINVAL;
+    memcpy(dst, c->bn + (int64_t)cluster * c->S, sizeof(double) * (size_t)c->S);
+    return ORC_OK;
+  }
   int64_t P = c->o.p_total, pc = c->o.p_client;
   const double* th = c->theta + (int64_t)cluster * P;
   if (segment == 0) memcpy(dst, th, sizeof(double) * (size_t)pc);
@@ -700,6 +756,12 @@ int orc_get_params(const orc_ctx* c, int cluster, int segment, double* dst) {
 int orc_set_params(orc_ctx* c, int cluster, const double* blob) {
   if (cluster < 0 || cluster >= c->C) return ORC_EINVAL;
   memcpy(c->theta + (int64_t)cluster * c->o.p_total, blob, sizeof(double) * (size_t)c->o.p_total);
+  return ORC_OK;
+}
+
+int orc_set_bn_state(orc_ctx* c, int cluster, const double* src) {
+  if (!c->resnet || cluster < 0 || cluster >= c->C) return ORC_EINVAL;
+  memcpy(c->bn + (int64_t)cluster * c->S, src, sizeof(double) * (size_t)c->S);
   return ORC_OK;
 }
 

@@ -108,8 +108,43 @@ ARCHS = {
 }
 
 
+# The CIFAR ResNet-18 split: client = conv 3->64 stem + GroupNorm + stage 1,
+# server = stages 2-4 with BatchNorm, global average pool, linear 512->10.
+# Basic blocks (conv1, norm1, conv2, norm2[, shortcut conv 1x1, norm]);
+# convolutions have no bias.  Names and order follow PyTorch's
+# named_parameters() of the usual CIFAR ResNet-18 module layout.
+RESNET_STAGES = ((64, 1), (128, 2), (256, 2), (512, 2))     # (width, first stride)
+
+
+def _resnet_shapes(segment: str):
+    out = []
+    if segment == "client":
+        out += [("conv1.weight", (64, 3, 3, 3)), ("bn1.weight", (64,)), ("bn1.bias", (64,))]
+    cin = 64
+    for st, (width, stride) in enumerate(RESNET_STAGES):
+        for j in range(2):
+            s = stride if j == 0 else 1
+            in_client = st == 0
+            if (segment == "client") == in_client:
+                pre = f"layer{st + 1}.{j}"
+                out += [(f"{pre}.conv1.weight", (width, cin, 3, 3)),
+                        (f"{pre}.bn1.weight", (width,)), (f"{pre}.bn1.bias", (width,)),
+                        (f"{pre}.conv2.weight", (width, width, 3, 3)),
+                        (f"{pre}.bn2.weight", (width,)), (f"{pre}.bn2.bias", (width,))]
+                if s != 1 or cin != width:
+                    out += [(f"{pre}.shortcut.0.weight", (width, cin, 1, 1)),
+                            (f"{pre}.shortcut.1.weight", (width,)),
+                            (f"{pre}.shortcut.1.bias", (width,))]
+            cin = width
+    if segment == "server":
+        out += [("linear.weight", (10, 512)), ("linear.bias", (10,))]
+    return out
+
+
 def param_shapes(arch: int, segment: str):
     """[(name, shape)] for one segment ('client' or 'server')."""
+    if arch == ARCH_RESNET18:
+        return _resnet_shapes(segment)
     spec = ARCHS[arch]
     out = []
     for i, (cin, cout, _h, _w, _p) in enumerate(spec[segment]):
@@ -135,6 +170,12 @@ def init_params(arch: int, seed: int = SEED_INIT) -> np.ndarray:
     for seg in ("client", "server"):
         shapes = param_shapes(arch, seg)
         for (name, shape) in shapes:
+            if len(shape) == 1 and (".bn" in name or "shortcut.1" in name or
+                                    name.startswith("bn1")):
+                # norm affine: weight 1, bias 0 (PyTorch's default)
+                val = 1.0 if name.endswith(".weight") else 0.0
+                parts.append(np.full(shape, val, dtype=np.float32))
+                continue
             if name.endswith(".weight"):
                 fan_in = int(np.prod(shape[1:]))
             bound = 1.0 / np.sqrt(fan_in)
