@@ -156,9 +156,12 @@ cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* los
                           int route, const uint8_t* code, const T* act, int Ho, int Wo, int ch);
 
 // conv_tc.cu (tensor-core convolutions, bf16 operands)
-enum { EPI_POOL = 0, EPI_RELU = 1, EPI_STORE = 2, EPI_DPOOL = 3, EPI_DRELU = 4 };
+enum {
+  EPI_POOL = 0, EPI_RELU = 1, EPI_STORE = 2, EPI_DPOOL = 3, EPI_DRELU = 4, EPI_ADD = 5,
+  EPI_DSTORE = 6
+};
 struct ConvTcArgs {
-  int H, W, B;          // spatial size and batch per replica
+  int H, W, B;          // M grid (the GEMM's output pixels) and batch per replica
   int kch;              // channels of the activation operand (multiple of the stage width)
   int bw, hb, bb;       // M tile of 128 pixels: bw columns x hb rows x bb images
   int tiles_w, tiles_h; // W / bw, H / hb
@@ -170,22 +173,45 @@ struct ConvTcArgs {
   int* err;             // error word: bounded waits that gave up
   const bf16* act;      // EPI_DRELU: the previous layer's ReLU output, layout of out
   bf16* gout;           // EPI_DPOOL / EPI_DRELU: the previous layer's g (2H x 2W for DPOOL)
-  int taps = 9;         // 9: 3x3 taps over shifted boxes; 1: the im2col input layer
+  // K taps: A box origin = (M pixel) * stride + (tdy, tdx); B tap index tw;
+  // tsrc selects the operand pair (0: a/b, 1: a2/b2).  Filled by the
+  // conv_taps_* helpers.
+  int stride = 1;
+  int ntaps = 9;
+  int8_t tdy[9] = {}, tdx[9] = {}, tw[9] = {}, tsrc[9] = {};
+  // output pixel of M pixel (y, x): (y * osy + ooy, x * osx + oox) in an
+  // out_H x out_W grid (0: the M grid) -- EPI_STORE / EPI_ADD / EPI_DRELU
+  int out_H = 0, out_W = 0, osy = 1, osx = 1, ooy = 0, oox = 0;
+  const bf16* res = nullptr;  // EPI_ADD: out = bf16(acc + res), layout of out
 };
+// 3x3 forward taps (kernel row/col ky, kx -> shift (ky-1, kx-1), tap ky*3+kx)
+void conv_taps_fwd3(ConvTcArgs& p);
+// one tap without shift (1x1 convolutions, the im2col input layer)
+void conv_taps_one(ConvTcArgs& p);
+// 3x3 stride-1 data gradient: shift (sy, sx), weight tap (1-sy)*3 + (1-sx)
+void conv_taps_dgrad3(ConvTcArgs& p);
+// 3x3 stride-2 data gradient for the input pixels of parity (py, px): the
+// taps with (p+1-k) even, shift (p+1-k)/2; with_sc adds the 1x1 stride-2
+// shortcut (operand pair 1) to parity (0, 0)
+void conv_taps_dgrad3_s2(ConvTcArgs& p, int py, int px, bool with_sc);
 struct WgradTcArgs {
-  int H, W, B, cout, cin;
+  int H, W, B, cout, cin;   // H, W: the output grid (g)
   int hb, bb;           // image rows / images per 64-pixel K block (W * hb * bb == 64)
   int kb_total;         // K blocks per replica
   int kb_per_split, splits;
-  float* partial;       // [C][splits][cout][9][cin]
+  float* partial;       // [C][splits][cout][taps][cin] (+ [cout] bias)
   int* err;
+  int taps = 9;         // 9 (3x3) or 1 (1x1)
+  int bias = 1;         // also the bias gradient (a block of ones)
+  int stride = 1, pad = 1;  // x pixel of output pixel p and tap (kh, kw): p*stride + k - pad
 };
 bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                      const uint32_t* box, int swizzle_bytes);
 bool tensor_map_bf16_strided(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                              uint64_t outer_stride_bytes, const uint32_t* box, int swizzle_bytes);
 cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                           const ConvTcArgs& p, int bn, int bkc, int epi, int C);
+                           const ConvTcArgs& p, int bn, int bkc, int epi, int C,
+                           const CUtensorMap* a2 = nullptr, const CUtensorMap* b2 = nullptr);
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C);
 // input layer: b = packed weights w0p[C][cout][32] (k = tap * 3 + ci < 27, else 0)
@@ -194,9 +220,10 @@ cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs,
 // 64), partial layout [C][splits][cout*27 + cout]
 cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                              const WgradTcArgs& p, int C);
-// dw[c * dw_rs + i] = sum over s (in order) of partial[c][s][i], i < per
+// dw[c * dw_rs + i] = sum over s (in order) of partial[c][s][i], i < count
+// (partials `per` apart)
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
-                                int splits, int64_t per, int C);
+                                int splits, int64_t per, int C, int64_t count = -1);
 
 // optim.cu
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,

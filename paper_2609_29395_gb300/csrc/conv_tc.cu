@@ -81,7 +81,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 //             through shared memory so that the window's four threads each
 //             decide 4 of the 16 channels from all four positions.
 //  EPI_RELU : + bias, relu, bf16 store.
-//  EPI_STORE: bf16 store (data gradient).
+//  EPI_STORE / EPI_DSTORE: bf16 store (bias-free forward / data gradient).
 //  EPI_DPOOL: data gradient routed through the previous layer's max-pool:
 //             the four pixels of the previous layer's 2x2 window get the
 //             bf16 gradient where the code names that position and the
@@ -89,6 +89,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 //             gradient itself: the cut).
 //  EPI_DRELU: data gradient times the previous layer's ReLU mask (act > 0),
 //             written to gout (and to out if set).
+//  EPI_ADD  : bf16(acc + res) (a data gradient plus the residual path's).
+//  Outside EPI_POOL the output pixel is mapped by (osy, ooy, osx, oox).
 template <int BN, int EPI>
 __device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0, int b0, int h0,
                                                     int w0, int c, const ConvTcArgs& p,
@@ -148,7 +150,9 @@ __device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0
     }
     return;
   }
-  const int64_t o = ((img * H + h0 + hh) * W + w0 + ww) * p.n_total + n0;
+  const int oH = p.out_H ? p.out_H : H, oW = p.out_W ? p.out_W : W;
+  const int64_t o = ((img * oH + (h0 + hh) * p.osy + p.ooy) * oW + (w0 + ww) * p.osx + p.oox) *
+                        p.n_total + n0;
   const float* bias = EPI == EPI_RELU ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
 #pragma unroll 1
   for (int c0 = 0; c0 < BN; c0 += 16) {
@@ -163,6 +167,10 @@ __device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0
     uint4 cd;
     uint4 am[2];
     if (EPI == EPI_DPOOL && valid) cd = *reinterpret_cast<const uint4*>(p.code + o + c0);
+    if (EPI == EPI_ADD && valid) {
+      am[0] = *reinterpret_cast<const uint4*>(p.res + o + c0);
+      am[1] = *reinterpret_cast<const uint4*>(p.res + o + c0 + 8);
+    }
     if (EPI == EPI_DRELU && valid) {
       am[0] = *reinterpret_cast<const uint4*>(p.act + o + c0);
       am[1] = *reinterpret_cast<const uint4*>(p.act + o + c0 + 8);
@@ -177,6 +185,11 @@ __device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0
         x1 += b16[2 * i + 1];
         x0 = x0 > 0.f ? x0 : 0.f;
         x1 = x1 > 0.f ? x1 : 0.f;
+      }
+      if (EPI == EPI_ADD) {
+        const uint32_t r = (&am[0].x)[i];
+        x0 += __uint_as_float(r << 16);
+        x1 += __uint_as_float(r & 0xffff0000u);
       }
       hw[i] = pack_bf16x2(x0, x1);
     }
@@ -264,6 +277,7 @@ __device__ __forceinline__ void tile_origin(int mt, const ConvTcArgs& p, int& b0
 template <int BN, int BKC, int EPI, int BMN>
 __global__ void __launch_bounds__(kThreads, 1)
 k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
+          const __grid_constant__ CUtensorMap tA2, const __grid_constant__ CUtensorMap tB2,
           const ConvTcArgs p, int tiles_m, int tiles_n, int items) {
   using Cfg = ConvCfg<BN, BKC, EPI>;
   constexpr int S = Cfg::S;
@@ -274,8 +288,9 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kper = p.kch / BKC;
-  const int KB = p.taps * kper;
-  const int shift = p.taps == 9 ? 1 : 0;        // 3x3 taps, or one tap (im2col input)
+  const int KB = p.ntaps * kper;
+  bool two = false;                              // a second operand pair in the tap list
+  for (int t = 0; t < p.ntaps; ++t) two |= p.tsrc[t] != 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
@@ -283,6 +298,7 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
     fence_mbar_init();
     tma_prefetch_desc(&tA);
     tma_prefetch_desc(&tB);
+    if (two) { tma_prefetch_desc(&tA2); tma_prefetch_desc(&tB2); }
   }
   if (warp == 1) { tmem_alloc(&tbase, 2 * Cfg::TCOLS); tmem_relinquish(); }
   tc_fence_before();
@@ -310,17 +326,19 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
           }
           uint8_t* sa = sm + s * Cfg::STAGE;
           const int tap = kb / kper, ch = (kb % kper) * BKC;
+          const CUtensorMap* ma = p.tsrc[tap] ? &tA2 : &tA;
+          const CUtensorMap* mb = p.tsrc[tap] ? &tB2 : &tB;
           mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
-          tma_load_5d(sa, &tA, &full[s], ch, w0 + (tap % 3 - 1) * shift,
-                      h0 + (tap / 3 - 1) * shift, b0, c);
+          tma_load_5d(sa, ma, &full[s], ch, w0 * p.stride + p.tdx[tap],
+                      h0 * p.stride + p.tdy[tap], b0, c);
           if (!BMN) {
-            tma_load_4d(sa + Cfg::A_BYTES, &tB, &full[s], ch, tap, n0, c);
+            tma_load_4d(sa + Cfg::A_BYTES, mb, &full[s], ch, p.tw[tap], n0, c);
           } else {
             constexpr int NBW = BN < 64 ? BN : 64;           // N block width
 #pragma unroll
             for (int j = 0; j < BN / NBW; ++j)
-              tma_load_4d(sa + Cfg::A_BYTES + j * NBW * BKC * 2, &tB, &full[s], n0 + j * NBW,
-                          8 - tap, ch, c);
+              tma_load_4d(sa + Cfg::A_BYTES + j * NBW * BKC * 2, mb, &full[s], n0 + j * NBW,
+                          p.tw[tap], ch, c);
           }
         }
       }
@@ -458,12 +476,15 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   int t = blockIdx.y;
   const int ci0 = (t % ci_tiles) * BN; t /= ci_tiles;
   const int co0 = (t % co_tiles) * MT; t /= co_tiles;
-  const int grp = t;                                 // tap group
-  const bool bias_grp = grp == 0;
-  const int tap0 = bias_grp ? 0 : (TG - 1) + (grp - 1) * TG;
-  const int ntaps = bias_grp ? TG - 1 : (9 - tap0 < TG ? 9 - tap0 : TG);
-  const int nslots = bias_grp ? TG : ntaps;          // N = nslots * BN
-  const int per = p.cout * 9 * p.cin + p.cout;       // partial length per split
+  // slot group t: slots [t*TG, t*TG + nslots) of taps 0..taps-1 and, with
+  // the bias, one last slot of ones
+  const int total = p.taps + p.bias;
+  const int tap0 = t * TG;
+  const int nslots = total - tap0 < TG ? total - tap0 : TG;  // N = nslots * BN
+  const bool bias_grp = p.bias && p.taps >= tap0 && p.taps < tap0 + nslots;
+  const int ntaps = bias_grp ? nslots - 1 : nslots;
+  const int ksz = p.taps == 9 ? 3 : 1;
+  const int per = p.cout * p.taps * p.cin + (p.bias ? p.cout : 0);   // partial length per split
   const int kb_begin = split * p.kb_per_split;
   const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
   const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
@@ -481,7 +502,7 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     const uint4 ones = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
     for (int s = 0; s < S; ++s) {
       uint4* dst = reinterpret_cast<uint4*>(sm + s * Cfg::STAGE + Cfg::A_BYTES +
-                                            (TG - 1) * Cfg::TAP_BYTES);
+                                            ntaps * Cfg::TAP_BYTES);
       for (int i = threadIdx.x; i < Cfg::TAP_BYTES / 16; i += blockDim.x) dst[i] = ones;
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -512,11 +533,11 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
           tma_load_5d(sa + 64 * Cfg::BKP * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0,
                       0, h, b, c);
         for (int tj = 0; tj < ntaps; ++tj) {
-          const int tap = tap0 + tj, kh = tap / 3, kw = tap % 3;
+          const int tap = tap0 + tj, kh = tap / ksz, kw = tap % ksz;
 #pragma unroll
           for (int j = 0; j < (BN + 63) / 64; ++j)
             tma_load_5d(sb + tj * Cfg::TAP_BYTES + j * 64 * Cfg::BKP * 2, &tX, &full[s],
-                        ci0 + 64 * j, kw - 1, h + kh - 1, b, c);
+                        ci0 + 64 * j, kw - p.pad, h * p.stride + kh - p.pad, b, c);
         }
       }
     }
@@ -556,12 +577,12 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     float* part = p.partial + ((int64_t)c * p.splits + split) * per;
     if (bias_grp && ci0 == 0) {
       float v[16];
-      tmem_ld16(trow + (TG - 1) * BN, v);
+      tmem_ld16(trow + ntaps * BN, v);
       tmem_ld_wait();
-      if (mine) part[p.cout * 9 * p.cin + co] = nkb ? v[0] : 0.f;
+      if (mine) part[p.cout * p.taps * p.cin + co] = nkb ? v[0] : 0.f;
     }
     for (int tj = 0; tj < ntaps; ++tj) {
-      float* dst = part + (int64_t)co * 9 * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
+      float* dst = part + (int64_t)co * p.taps * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 16) {
         float v[16];
@@ -692,14 +713,14 @@ k_wgrad0_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUte
   if (warp == 1) tmem_dealloc(tmem, 32);
 }
 
-// dw[c][i] = sum_s partial[c][s][i].  A block of 8 warps covers 32 * 8/G
+// dw[c][i] = sum_s partial[c][s][i] for i < count (partials `per` apart).  A block of 8 warps covers 32 * 8/G
 // consecutive columns; the G warps of a column group split the s range
 // (warp g takes s = g, g+G, ...) and their sums are added in warp order, so
 // the order depends on `splits` only.
 template <int G>
 __global__ void __launch_bounds__(256)
 k_wgrad_reduce(const float* __restrict__ partial, float* __restrict__ dw, int64_t dw_rs,
-               int splits, int64_t per) {
+               int splits, int64_t per, int64_t count) {
   __shared__ float red[8][32];
   pdl_wait();
   pdl_trigger();
@@ -708,17 +729,17 @@ k_wgrad_reduce(const float* __restrict__ partial, float* __restrict__ dw, int64_
   const int grp = w / G, sub = w % G;
   const int64_t i = ((int64_t)blockIdx.x * (8 / G) + grp) * 32 + lane;
   float s = 0.f;
-  if (i < per) {
+  if (i < count) {
     const float* src = partial + (int64_t)c * splits * per + i;
     for (int k = sub; k < splits; k += G) s += src[(int64_t)k * per];
   }
   if (G == 1) {
-    if (i < per) dw[(int64_t)c * dw_rs + i] = s;
+    if (i < count) dw[(int64_t)c * dw_rs + i] = s;
     return;
   }
   red[w][lane] = s;
   __syncthreads();
-  if (sub == 0 && i < per) {
+  if (sub == 0 && i < count) {
     float t = red[w][lane];
 #pragma unroll
     for (int q = 1; q < G; ++q) t += red[w + q][lane];
@@ -740,7 +761,8 @@ int sm_count() {
 
 template <int BN, int BKC, int EPI, int BMN>
 cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                             const ConvTcArgs& p, int tiles_m, int tiles_n, int items) {
+                             const CUtensorMap& a2, const CUtensorMap& b2, const ConvTcArgs& p,
+                             int tiles_m, int tiles_n, int items) {
   using Cfg = ConvCfg<BN, BKC, EPI>;
   static bool attr = false;
   if (!attr) {
@@ -751,8 +773,8 @@ cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
   }
   const int cap = sm_count() * Cfg::CTAS;
   const int grid = items < cap ? items : cap;
-  return launch_k(k_conv_tc<BN, BKC, EPI, BMN>, grid, kThreads, Cfg::SMEM, s, a, b, p, tiles_m,
-                  tiles_n, items);
+  return launch_k(k_conv_tc<BN, BKC, EPI, BMN>, grid, kThreads, Cfg::SMEM, s, a, b, a2, b2, p,
+                  tiles_m, tiles_n, items);
 }
 
 template <int BN, int MT>
@@ -770,6 +792,63 @@ cudaError_t launch_wgrad_inst(cudaStream_t s, const CUtensorMap& g, const CUtens
 }
 
 }  // namespace
+
+// ---------------------------------------------------------------------------
+// host: tap tables
+// ---------------------------------------------------------------------------
+void conv_taps_fwd3(ConvTcArgs& p) {
+  p.ntaps = 9;
+  for (int t = 0; t < 9; ++t) {
+    p.tdy[t] = (int8_t)(t / 3 - 1);
+    p.tdx[t] = (int8_t)(t % 3 - 1);
+    p.tw[t] = (int8_t)t;
+    p.tsrc[t] = 0;
+  }
+}
+
+void conv_taps_one(ConvTcArgs& p) {
+  p.ntaps = 1;
+  p.tdy[0] = p.tdx[0] = p.tw[0] = p.tsrc[0] = 0;
+}
+
+// dx[y][x] = sum_{sy,sx} g[y+sy][x+sx] W[1-sy][1-sx] (correlation with the
+// flipped kernel)
+void conv_taps_dgrad3(ConvTcArgs& p) {
+  p.ntaps = 9;
+  for (int t = 0; t < 9; ++t) {
+    const int sy = t / 3 - 1, sx = t % 3 - 1;
+    p.tdy[t] = (int8_t)sy;
+    p.tdx[t] = (int8_t)sx;
+    p.tw[t] = (int8_t)((1 - sy) * 3 + (1 - sx));
+    p.tsrc[t] = 0;
+  }
+}
+
+// input pixel (2Y+py, 2X+px) of a stride-2 3x3 convolution receives
+// g[Y + (py+1-ky)/2][X + (px+1-kx)/2] W[ky][kx] for the taps with py+1-ky
+// and px+1-kx even
+void conv_taps_dgrad3_s2(ConvTcArgs& p, int py, int px, bool with_sc) {
+  int n = 0;
+  for (int ky = 0; ky < 3; ++ky)
+    for (int kx = 0; kx < 3; ++kx) {
+      if ((py + 1 - ky) % 2 != 0 || (px + 1 - kx) % 2 != 0) continue;
+      p.tdy[n] = (int8_t)((py + 1 - ky) / 2);
+      p.tdx[n] = (int8_t)((px + 1 - kx) / 2);
+      p.tw[n] = (int8_t)(ky * 3 + kx);
+      p.tsrc[n] = 0;
+      ++n;
+    }
+  if (with_sc && py == 0 && px == 0) {
+    p.tdy[n] = p.tdx[n] = p.tw[n] = 0;
+    p.tsrc[n] = 1;
+    ++n;
+  }
+  p.ntaps = n;
+  p.stride = 1;
+  p.osy = p.osx = 2;
+  p.ooy = py;
+  p.oox = px;
+}
 
 // ---------------------------------------------------------------------------
 // host: tensor maps
@@ -843,21 +922,31 @@ bool tensor_map_bf16_strided(CUtensorMap* m, const void* base, int rank, const u
 // launchers
 // ---------------------------------------------------------------------------
 cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
-                           const ConvTcArgs& p, int bn, int bkc, int epi, int C) {
+                           const ConvTcArgs& p, int bn, int bkc, int epi, int C,
+                           const CUtensorMap* a2, const CUtensorMap* b2) {
+  if (p.ntaps < 1 || p.ntaps > 9 || p.stride < 1) return cudaErrorInvalidValue;
+  for (int t = 0; t < p.ntaps; ++t)
+    if (p.tsrc[t] && (!a2 || !b2)) return cudaErrorInvalidValue;
+  const CUtensorMap& A2 = a2 ? *a2 : a;
+  const CUtensorMap& B2 = b2 ? *b2 : b;
   const int tiles_m = p.tiles_w * p.tiles_h * ((p.B + p.bb - 1) / p.bb);
   const int tiles_n = p.n_total / bn;
   const int items = tiles_m * tiles_n * C;
-  // fprop epilogues read a K-major B; the data gradient (EPI_STORE) reads
+  // forward epilogues read a K-major B; the data-gradient epilogues read
   // the same weights MN-major
 #define GCPSL_CONV_CASE(BN_, BKC_, EPI_, BMN_)             \
   if (bn == BN_ && bkc == BKC_ && epi == EPI_)             \
-    return launch_conv_inst<BN_, BKC_, EPI_, BMN_>(s, a, b, p, tiles_m, tiles_n, items);
-#define GCPSL_CONV_EPIS(BN_, BKC_)          \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_POOL, 0)   \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_RELU, 0)   \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_STORE, 1)  \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_DPOOL, 1)  \
-  GCPSL_CONV_CASE(BN_, BKC_, EPI_DRELU, 1)
+    return launch_conv_inst<BN_, BKC_, EPI_, BMN_>(s, a, b, A2, B2, p, tiles_m, tiles_n, items);
+// EPI_STORE: the bias-free forward (pre-norm output, K-major B);
+// EPI_DSTORE: the same store for a data gradient (MN-major B)
+#define GCPSL_CONV_EPIS(BN_, BKC_)           \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_POOL, 0)    \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_RELU, 0)    \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_STORE, 0)   \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_DSTORE, 1)  \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_DPOOL, 1)   \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_DRELU, 1)   \
+  GCPSL_CONV_CASE(BN_, BKC_, EPI_ADD, 1)
   GCPSL_CONV_CASE(32, 32, EPI_POOL, 0)      // the input layer (im2col, K = 32)
   GCPSL_CONV_CASE(32, 32, EPI_RELU, 0)
   GCPSL_CONV_EPIS(32, 64)
@@ -866,9 +955,11 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
   GCPSL_CONV_EPIS(128, 32)
   GCPSL_CONV_EPIS(128, 64)
   GCPSL_CONV_CASE(256, 64, EPI_RELU, 0)
-  GCPSL_CONV_CASE(256, 64, EPI_STORE, 1)
+  GCPSL_CONV_CASE(256, 64, EPI_STORE, 0)
+  GCPSL_CONV_CASE(256, 64, EPI_DSTORE, 1)
   GCPSL_CONV_CASE(256, 64, EPI_DPOOL, 1)
   GCPSL_CONV_CASE(256, 64, EPI_DRELU, 1)
+  GCPSL_CONV_CASE(256, 64, EPI_ADD, 1)
 #undef GCPSL_CONV_EPIS
 #undef GCPSL_CONV_CASE
   return cudaErrorInvalidValue;
@@ -883,7 +974,8 @@ cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs,
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C) {
   const int tg = 256 / bn;                            // slots per CTA
-  const int groups = 1 + (9 - (tg - 1) + tg - 1) / tg;
+  if ((p.taps != 9 && p.taps != 1) || (p.taps == 1 && p.pad != 0)) return cudaErrorInvalidValue;
+  const int groups = (p.taps + p.bias + tg - 1) / tg;
   const int mt = p.cout % 128 == 0 ? 128 : 64;
   const int tiles = groups * (p.cin / bn) * ((p.cout + mt - 1) / mt);
   dim3 grid(p.splits, tiles, C);
@@ -921,14 +1013,18 @@ cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtenso
 }
 
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
-                                int splits, int64_t per, int C) {
+                                int splits, int64_t per, int C, int64_t count) {
+  if (count < 0) count = per;
   const int G = splits <= 2 ? 1 : splits <= 8 ? 2 : splits <= 32 ? 4 : 8;
   const int64_t cols_per_block = 32 * (8 / G);
-  const dim3 grid((unsigned)((per + cols_per_block - 1) / cols_per_block), C);
-  if (G == 1) return launch_k(k_wgrad_reduce<1>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
-  if (G == 2) return launch_k(k_wgrad_reduce<2>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
-  if (G == 4) return launch_k(k_wgrad_reduce<4>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
-  return launch_k(k_wgrad_reduce<8>, grid, 256, 0, s, partial, dw, dw_rs, splits, per);
+  const dim3 grid((unsigned)((count + cols_per_block - 1) / cols_per_block), C);
+  if (G == 1)
+    return launch_k(k_wgrad_reduce<1>, grid, 256, 0, s, partial, dw, dw_rs, splits, per, count);
+  if (G == 2)
+    return launch_k(k_wgrad_reduce<2>, grid, 256, 0, s, partial, dw, dw_rs, splits, per, count);
+  if (G == 4)
+    return launch_k(k_wgrad_reduce<4>, grid, 256, 0, s, partial, dw, dw_rs, splits, per, count);
+  return launch_k(k_wgrad_reduce<8>, grid, 256, 0, s, partial, dw, dw_rs, splits, per, count);
 }
 
 

@@ -8,14 +8,8 @@
 // cluster (Algorithm 2's inner loop body) as grouped kernels on one stream.
 #include <algorithm>
 #include <cmath>
-#include <cstdarg>
-#include <cstdio>
-#include <cstring>
-#include <string>
-#include <vector>
 
-#include "common.cuh"
-#include "gcpsl.h"
+#include "ctx.h"
 
 using namespace gcpsl;
 
@@ -50,82 +44,7 @@ bool gcpsl::make_arch(int id, ArchSpec* a) {
   return true;
 }
 
-// ---------------------------------------------------------------------------
-// Kernel timing with CUDA events on the context's stream
-// ---------------------------------------------------------------------------
 namespace {
-
-struct KernelTimer {
-  std::vector<const char*> names;
-  std::vector<int64_t> launches;
-  std::vector<double> ms;
-  struct Pending { int kind; cudaEvent_t a, b; };
-  std::vector<Pending> pending;
-  std::vector<cudaEvent_t> pool;
-  int cur_kind = -1;
-  cudaEvent_t cur_a = nullptr;
-  // while a round is being captured into a graph, the event pairs become
-  // external event-record nodes of that graph and are listed here
-  std::vector<Pending>* capture = nullptr;
-  // only kernels whose name starts with this prefix are timed (empty: all)
-  std::string filter;
-
-  bool wants(const char* name) const {
-    return filter.empty() || std::strncmp(name, filter.c_str(), filter.size()) == 0;
-  }
-
-  int kind(const char* name) {
-    for (size_t i = 0; i < names.size(); ++i)
-      if (names[i] == name || std::strcmp(names[i], name) == 0) return (int)i;
-    names.push_back(name); launches.push_back(0); ms.push_back(0.0);
-    return (int)names.size() - 1;
-  }
-  cudaEvent_t get() {
-    if (!pool.empty()) { cudaEvent_t e = pool.back(); pool.pop_back(); return e; }
-    cudaEvent_t e = nullptr;
-    cudaEventCreate(&e);
-    return e;
-  }
-  void record(cudaEvent_t e, cudaStream_t s) {
-    if (capture) cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
-    else cudaEventRecord(e, s);
-  }
-  void begin(const char* name, cudaStream_t s) {
-    cur_kind = kind(name);
-    cur_a = get();
-    record(cur_a, s);
-  }
-  void end(cudaStream_t s) {
-    cudaEvent_t b = get();
-    record(b, s);
-    (capture ? *capture : pending).push_back({cur_kind, cur_a, b});
-  }
-  // add the elapsed times of recorded pairs (waits for each pair's end)
-  void account(const std::vector<Pending>& v) {
-    for (auto& p : v) {
-      float t = 0.f;
-      if (cudaEventSynchronize(p.b) == cudaSuccess && cudaEventElapsedTime(&t, p.a, p.b) == cudaSuccess) {
-        ms[p.kind] += t;
-        launches[p.kind] += 1;
-      }
-    }
-  }
-  void collect() {
-    account(pending);
-    for (auto& p : pending) { pool.push_back(p.a); pool.push_back(p.b); }
-    pending.clear();
-  }
-  void reset() {
-    collect();
-    std::fill(launches.begin(), launches.end(), 0);
-    std::fill(ms.begin(), ms.end(), 0.0);
-  }
-  void destroy() {
-    collect();
-    for (auto e : pool) cudaEventDestroy(e);
-    pool.clear();
-  }
-};
 
 thread_local std::string g_init_error;
 
@@ -133,115 +52,7 @@ thread_local std::string g_init_error;
 
 void gcpsl::set_global_error(const char* msg) { g_init_error = msg; }
 
-struct gcpsl_ctx {
-  gcpsl_model_desc desc{};
-  ArchSpec a{};
-  int K = 0, C = 0, B = 0, F = 0;
-  uint64_t seed = 0;
-  bool bf = false;
-  size_t esz = 4;
-  cudaStream_t own_stream = nullptr, stream = nullptr;
-
-  int64_t n = 0;
-  float* d_images = nullptr;       // device copy, or device view of h_images
-  float* h_images = nullptr;       // pinned mapped host copy (data_on_host)
-  int32_t* d_labels = nullptr;
-  int32_t* d_owner = nullptr;
-
-  std::vector<int64_t> h_off;      // [C+1] offsets of the clusters' id lists
-  std::vector<int32_t> h_rounds;   // r_n = n_c / B
-  std::vector<float> h_q;          // fusion weights
-  int64_t max_nc = 0;
-  int64_t* d_off = nullptr;
-  int32_t* d_rounds = nullptr;
-  int32_t* d_ids = nullptr;
-  int32_t* d_perm = nullptr;
-  uint64_t* d_keys = nullptr;
-  float* d_q = nullptr;
-
-  int64_t P = 0;
-  int64_t P_pad = 0;               // replica stride of every [C][P] array (multiple of 64)
-  float* d_theta = nullptr;        // [C][P_pad] fp32 master, kernel layout
-  float* d_mom = nullptr;
-  float* d_grad = nullptr;
-  bf16* d_shadow = nullptr;        // [C][P_pad] bf16 operand copy (bf16 mode)
-  int* d_err = nullptr;            // device error word (bounded waits that gave up)
-
-  // tensor-core layers (bf16 mode): tile shapes and TMA descriptors
-  struct TcLayer {
-    bool on = false;
-    int bw, hb, bb, tiles_w, tiles_h;   // 128-pixel M tile
-    int whb, wbb;                  // 64-pixel K block of the weight gradient
-    int bn_f, bkc_f, bn_d, bkc_d, bn_w;
-    int splits, kb_total, kb_per_split;
-    CUtensorMap fwdA, fwdB, dgrA, dgrB, wgA, wgB;
-  } tc[4];
-  // input layer on the tensor cores (bf16 mode): the gather writes its
-  // im2col, x0c = 32 columns per pixel; packed weights [C][cout][32]
-  struct Tc0Layer {
-    bool on = false;
-    int bw, hb, bb, tiles_w, tiles_h;
-    CUtensorMap A, B;
-    bool wg_on = false;            // its weight gradient on the tensor cores too
-    int whb, wbb, kb_total, kb_per_split, splits;
-    CUtensorMap wgA, wgB;
-  } tc0;
-  int x0c = 3;
-  bf16* d_w0p = nullptr;
-  float* d_partial = nullptr;      // weight-gradient split partials (tensor-core layers)
-  // CUDA-core weight+bias gradient partials of the layers not on the tensor
-  // cores (tiles of tr image rows, tiles_per_split tiles per block)
-  struct RedLayer { int tr, splits, tiles_per_split; } red[4];
-  float* d_bpartial = nullptr;
-
-  void* d_x0 = nullptr;
-  void* d_act[5] = {};             // d_act[i+1] = output of conv i
-  void* d_dact[5] = {};
-  uint8_t* d_code[4] = {};
-  // g_i, the gradient w.r.t. layer i's pre-activation: layers alternate
-  // between two buffers, since layer i's data gradient reads g_i while its
-  // epilogue writes g_{i-1}
-  void* d_g = nullptr;
-  void* d_g2 = nullptr;
-  void* gbuf(int i) const { return (i & 1) ? d_g2 : d_g; }
-  float* d_loss_ex = nullptr;     // [C][B] per-example loss
-  float* d_dlogits = nullptr;
-  int32_t* d_y = nullptr;
-  int32_t* d_idx = nullptr;
-  int32_t* d_counts = nullptr;
-  int32_t* d_active = nullptr;
-  float* d_loss = nullptr;
-  int64_t* d_t = nullptr;
-  float* h_loss = nullptr;         // pinned staging
-  int32_t* h_active = nullptr;
-
-  int64_t t = 0;
-  gcpsl_status sticky = GCPSL_OK;
-  std::string err;
-  std::vector<void*> allocs;
-  bool timing = false;
-  KernelTimer timer;
-
-  // CUDA graphs of one round: [epoch boundary or not][untimed, timed A, timed B].
-  // The two timed copies alternate so that one copy's event pairs are read
-  // while the other runs.
-  int64_t launched = 0;            // kernels launched so far (eager or graph nodes)
-  int64_t enqueued = 0;            // kernels passed through LAUNCH (eager or captured)
-  bool capturing = false;          // a round is being captured into a graph
-  struct RoundGraph {
-    cudaGraphExec_t exec = nullptr;
-    int64_t kernels = 0;          // kernel nodes of the captured round
-    std::vector<KernelTimer::Pending> marks;
-    bool unread = false;          // marks of the last launch not yet added to the timer
-  };
-  bool use_graph = true;
-  RoundGraph graph[2][3];
-  int timed_phase = 0;
-};
-
-namespace {
-
-gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...) {
+gcpsl_status gcpsl::fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...) {
   char buf[512];
   va_list ap;
   va_start(ap, fmt);
@@ -256,52 +67,8 @@ gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...) {
   return st;
 }
 
-#define CK(call)                                                                           \
-  do {                                                                                     \
-    cudaError_t _e = (call);                                                               \
-    if (_e != cudaSuccess)                                                                 \
-      return fail(c, _e == cudaErrorMemoryAllocation ? GCPSL_E_NOMEM : GCPSL_E_CUDA,       \
-                  "%s failed: %s (%s:%d)", #call, cudaGetErrorString(_e), __FILE__, __LINE__); \
-  } while (0)
 
-// launch through the timer when enabled
-#define LAUNCH(name, call)                                                                 \
-  do {                                                                                     \
-    const bool _t = c->timing && c->timer.wants(name);                                     \
-    ++c->enqueued;                                                                         \
-    if (!c->capturing) ++c->launched;                                                      \
-    if (_t) c->timer.begin(name, c->stream);                                               \
-    cudaError_t _e = (call);                                                               \
-    if (_t) c->timer.end(c->stream);                                                       \
-    if (_e != cudaSuccess)                                                                 \
-      return fail(c, GCPSL_E_CUDA, "kernel %s: %s", name, cudaGetErrorString(_e));        \
-  } while (0)
-
-// synchronise the stream, then fail on a device-side timeout
-#define SYNC_CHECK(c)                                        \
-  do {                                                       \
-    CK(cudaStreamSynchronize((c)->stream));                  \
-    gcpsl_status _d = check_device_error(c);                 \
-    if (_d != GCPSL_OK) return _d;                           \
-  } while (0)
-
-gcpsl_status check_device_error(gcpsl_ctx* c);
-
-template <typename P>
-gcpsl_status dalloc(gcpsl_ctx* c, P** p, size_t bytes) {
-  void* q = nullptr;
-  cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
-  if (e != cudaSuccess)
-    return fail(c, GCPSL_E_NOMEM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
-  c->allocs.push_back(q);
-  *p = (P*)q;
-  return GCPSL_OK;
-}
-#define DALLOC(p, bytes)                                   \
-  do {                                                     \
-    gcpsl_status _s = dalloc(c, &(p), (size_t)(bytes));    \
-    if (_s != GCPSL_OK) return _s;                         \
-  } while (0)
+namespace {
 
 // canonical (PyTorch) <-> kernel layout of one replica's parameters.
 // conv weight: OIHW <-> [co][kh][kw][ci]; linear weight: input index
@@ -364,11 +131,15 @@ void seeded_init(const ArchSpec& a, uint64_t seed, float* can) {
   fill(a.off_fcb, a.fc_out, a.fc_in);
 }
 
-gcpsl_status check_usable(gcpsl_ctx* c) {
+}  // namespace
+
+gcpsl_status gcpsl::check_usable(gcpsl_ctx* c) {
   if (!c) return GCPSL_E_INVAL;
   if (c->sticky != GCPSL_OK) return GCPSL_E_STATE;
   return GCPSL_OK;
 }
+
+namespace {
 
 int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
   if (i == 0) return (int64_t)c->C * c->B * 1024 * c->x0c;
@@ -387,14 +158,18 @@ gcpsl_status refresh_derived(gcpsl_ctx* c) {
   return GCPSL_OK;
 }
 
+}  // namespace
+
 // a device-side wait that gave up leaves a nonzero error word; the context
 // then refuses further work
-gcpsl_status check_device_error(gcpsl_ctx* c) {
+gcpsl_status gcpsl::check_device_error(gcpsl_ctx* c) {
   int e = 0;
   CK(cudaMemcpy(&e, c->d_err, sizeof(int), cudaMemcpyDeviceToHost));
   if (e) return fail(c, GCPSL_E_TIMEOUT, "device-side wait gave up (error word 0x%x)", e);
   return GCPSL_OK;
 }
+
+namespace {
 
 // per-layer names of the tensor-core launches in the kernel timer
 const char* const kFwdTc[4] = {"conv_fwd_tc.L0", "conv_fwd_tc.L1", "conv_fwd_tc.L2",
@@ -447,13 +222,14 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
       ConvTcArgs p{a.conv[0].h, a.conv[0].w, B, 32, L0.bw, L0.hb, L0.bb, L0.tiles_w, L0.tiles_h,
                    a.conv[0].cout, c->d_theta + a.off_b[0], P, (bf16*)(void*)act[1],
                    c->d_code[0], c->d_err};
-      p.taps = 1;
+      conv_taps_one(p);
       LAUNCH(kFwdTc[0], launch_conv_tc(s, L0.A, L0.B, p, a.conv[0].cout, 32,
                                        a.conv[0].pool ? EPI_POOL : EPI_RELU, C));
     } else if (L.on) {
       ConvTcArgs p{a.conv[i].h, a.conv[i].w, B, a.conv[i].cin, L.bw, L.hb, L.bb, L.tiles_w,
                    L.tiles_h, a.conv[i].cout, c->d_theta + a.off_b[i], P,
                    (bf16*)(void*)act[i + 1], c->d_code[i], c->d_err};
+      conv_taps_fwd3(p);
       LAUNCH(kFwdTc[i], launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f,
                                            a.conv[i].pool ? EPI_POOL : EPI_RELU, C));
     } else {
@@ -523,6 +299,7 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
                    pv.pool ? c->d_code[i - 1] : nullptr, c->d_err,
                    pv.pool ? nullptr : (const bf16*)(const void*)act[i],
                    (bf16*)c->gbuf(i - 1)};
+      conv_taps_dgrad3(p);
       LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d,
                                          pv.pool ? EPI_DPOOL : EPI_DRELU, C));
       g_ready[i - 1] = true;
@@ -605,15 +382,19 @@ gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
   return refresh_derived(c);
 }
 
+}  // namespace
+
 // 128-pixel M tile of a W x H image: bw <= 16 columns (so a warp holds whole
 // 2x2 pooling windows), hb rows, bb images
-bool m_tile(int W, int H, int& bw, int& hb, int& bb) {
+bool gcpsl::m_tile(int W, int H, int& bw, int& hb, int& bb) {
   bw = std::min(W, 16);
   if (bw < 2 || W % bw || 128 % bw) return false;
   hb = std::min(H, 128 / bw);
   bb = 128 / (bw * hb);
   return bw * hb * bb == 128 && H % hb == 0 && hb % 2 == 0;
 }
+
+namespace {
 
 // Tile shapes, split-K factors and TMA descriptors of every layer that runs on
 // the tensor cores: 3x3 layers with 32k input and 64k output channels and
@@ -644,7 +425,7 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     L.bn_w = std::min(s.cin, 128);
     if (s.cout % L.bn_f || s.cin % L.bn_d || s.cin % L.bkc_f || s.cin % L.bn_w) continue;
     const int tg = 256 / L.bn_w;                      // slots per weight-gradient CTA
-    const int groups = 1 + (9 - (tg - 1) + tg - 1) / tg;
+    const int groups = (9 + 1 + tg - 1) / tg;          // 9 taps + the bias slot
     const int mt = s.cout % 128 == 0 ? 128 : 64;      // output channels per tile
     const int tiles = groups * (s.cin / L.bn_w) * ((s.cout + mt - 1) / mt);
     L.kb_total = ((B + L.wbb - 1) / L.wbb) * (s.h / L.whb);
