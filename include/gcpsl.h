@@ -48,7 +48,7 @@ typedef enum {
  *             server conv 64->128 pool, conv 128->128 pool, FC 2048->10   */
 enum { GCPSL_TINY_CNN = 0, GCPSL_SPLIT_CNN = 1, GCPSL_RESNET18 = 2 };
 enum { GCPSL_F32 = 0, GCPSL_BF16 = 1 };
-enum { GCPSL_CLIENT = 0, GCPSL_SERVER = 1 };
+enum { GCPSL_CLIENT = 0, GCPSL_SERVER = 1, GCPSL_BN_STATE = 2 };
 enum { GCPSL_CUT_ACT = 0, GCPSL_CUT_GRAD = 1 };
 
 /* Model and optimiser description.
@@ -134,6 +134,9 @@ gcpsl_status gcpsl_fuse(gcpsl_ctx* ctx);
 
 /* gcpsl_get_params -- copy replica `cluster`'s parameters of `segment`
  * (GCPSL_CLIENT / GCPSL_SERVER) as fp32 in the init_params order into dst.
+ * With the ResNet-18 split, segment GCPSL_BN_STATE gives the BatchNorm
+ * running statistics (per BatchNorm layer in module order: running_mean
+ * then running_var; fused with q like the parameters, Eq. 5).
  * dst == NULL (or len too small) only reports the needed count in *needed
  * (and returns GCPSL_E_INVAL if dst is non-NULL but too small).          */
 gcpsl_status gcpsl_get_params(gcpsl_ctx* ctx, int cluster, int segment, float* dst, size_t len,
@@ -142,6 +145,11 @@ gcpsl_status gcpsl_get_params(gcpsl_ctx* ctx, int cluster, int segment, float* d
 /* gcpsl_set_params -- overwrite replica `cluster`'s parameters (both
  * segments, init_params order and length).  Momentum is left unchanged.  */
 gcpsl_status gcpsl_set_params(gcpsl_ctx* ctx, int cluster, const float* src, size_t len);
+
+/* gcpsl_set_bn_state -- overwrite replica `cluster`'s BatchNorm running
+ * statistics (ResNet-18 split only; len = gcpsl_num_params(arch,
+ * GCPSL_BN_STATE)).                                                       */
+gcpsl_status gcpsl_set_bn_state(gcpsl_ctx* ctx, int cluster, const float* src, size_t len);
 
 /* gcpsl_get_momentum / gcpsl_set_momentum -- replica `cluster`'s SGD
  * momentum buffer (Section IV-C: optimiser state stays per replica), both
@@ -156,6 +164,15 @@ gcpsl_status gcpsl_set_momentum(gcpsl_ctx* ctx, int cluster, const float* src, s
  * the window position of the first maximum in row-major order, bit 2 is set
  * when that maximum is positive (the output then carries a gradient).     */
 gcpsl_status gcpsl_get_pool_codes(gcpsl_ctx* ctx, int layer, uint8_t* dst, size_t len);
+
+/* gcpsl_get_relu_masks -- ResNet-18 split only: the last round's ReLU
+ * decisions, one byte per activation (1: the ReLU output is positive),
+ * laid out [C][B][E] with, per example, the stem's decisions, then for
+ * each of the 8 blocks those of its inner ReLU (a1) and of its output, each
+ * in [channels][h][w] order (E = 64*32*32 + sum over blocks of 2*ch*h*w).
+ * A test's record of which branch of every ReLU the round took.
+ * dst == NULL only reports the count in *needed.                          */
+gcpsl_status gcpsl_get_relu_masks(gcpsl_ctx* ctx, uint8_t* dst, size_t len, size_t* needed);
 
 /* gcpsl_get_cut -- the last round's cut activation z (GCPSL_CUT_ACT) or cut
  * gradient dL/dz (GCPSL_CUT_GRAD) of every cluster as fp32, laid out

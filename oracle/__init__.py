@@ -88,6 +88,14 @@ def _declare(L):
     L.orc_set_bn_state.argtypes = [ct.c_void_p, ct.c_int, f64p]
     L.orn_forward_backward.argtypes = [ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p, i32p,
                                        f64p, f64p, f64p, f64p, f64p]
+    L.orn_forward_backward_masks.argtypes = [ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p,
+                                             i32p, f64p, f64p, f64p, f64p, f64p,
+                                             _p(ct.c_uint8), _p(ct.c_uint8)]
+    L.orn_mask_elems.restype = ct.c_int64
+    L.orn_set_relu_tol.argtypes = [ct.c_double]
+    L.orn_set_relu_tol.restype = None
+    L.orc_set_relu_masks.argtypes = [ct.c_void_p, _p(ct.c_uint8)]
+    L.orc_get_relu_masks.argtypes = [ct.c_void_p, _p(ct.c_uint8)]
     L.orn_init_bn_state.argtypes = [f64p]
     L.orn_init_bn_state.restype = None
     L.orc_set_threads.argtypes = [ct.c_int]
@@ -141,10 +149,24 @@ def initial_bn_state():
     return out
 
 
+def set_relu_tol(tol: float):
+    """Width, in units of a layer's RMS pre-ReLU value, under which a ReLU
+    decision is recorded as ambiguous (ResNet-18 split)."""
+    lib().orn_set_relu_tol(tol)
+
+
+def resnet_mask_elems() -> int:
+    """ReLU decisions per example of the ResNet-18 split (see masks below)."""
+    return int(lib().orn_mask_elems())
+
+
 def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False,
-                            label_smoothing: float = 0.0, want_grad: bool = True):
+                            label_smoothing: float = 0.0, want_grad: bool = True,
+                            masks_in=None, want_masks: bool = False):
     """ResNet-18 split: (loss, grad[P] or None, cut_act, cut_grad, logits, bn_state
-    after this batch's update of the running statistics)."""
+    after this batch's update of the running statistics[, masks]).  masks:
+    [B][resnet_mask_elems()] uint8 ReLU decisions (stem, then per block those
+    of a1 and of the output, NCHW); masks_in replays given decisions."""
     params = np.ascontiguousarray(params, dtype=np.float64)
     x = np.ascontiguousarray(x, dtype=np.float64)
     labels = np.ascontiguousarray(labels, dtype=np.int32)
@@ -157,15 +179,22 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
     ncut = _cut_elems(RESNET18, B)
     ca, cg = np.zeros(ncut), np.zeros(ncut)
     logits = np.zeros(B * 10)
-    rc = lib().orn_forward_backward(int(bf16), label_smoothing, _ptr(params, ct.c_double),
-                                    _ptr(bn, ct.c_double), B, _ptr(x, ct.c_double),
-                                    _ptr(labels, ct.c_int32), _ptr(loss, ct.c_double),
-                                    _ptr(grad, ct.c_double) if want_grad else None,
-                                    _ptr(ca, ct.c_double), _ptr(cg, ct.c_double),
-                                    _ptr(logits, ct.c_double))
+    mo = np.zeros((B, resnet_mask_elems()), dtype=np.uint8) if want_masks else None
+    mi = None
+    if masks_in is not None:
+        mi = np.ascontiguousarray(masks_in, dtype=np.uint8)
+        assert mi.size == B * resnet_mask_elems()
+    rc = lib().orn_forward_backward_masks(
+        int(bf16), label_smoothing, _ptr(params, ct.c_double), _ptr(bn, ct.c_double), B,
+        _ptr(x, ct.c_double), _ptr(labels, ct.c_int32), _ptr(loss, ct.c_double),
+        _ptr(grad, ct.c_double) if want_grad else None, _ptr(ca, ct.c_double),
+        _ptr(cg, ct.c_double), _ptr(logits, ct.c_double),
+        _ptr(mi, ct.c_uint8) if mi is not None else None,
+        _ptr(mo, ct.c_uint8) if mo is not None else None)
     if rc:
         raise RuntimeError(f"oracle resnet forward_backward failed: {rc}")
-    return float(loss[0]), grad, ca, cg, logits.reshape(B, 10), bn
+    out = (float(loss[0]), grad, ca, cg, logits.reshape(B, 10), bn)
+    return out + (mo,) if want_masks else out
 
 
 def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smoothing: float = 0.0,
@@ -280,6 +309,23 @@ class Oracle:
         v = np.ascontiguousarray(v, dtype=np.float64)
         if lib().orc_set_bn_state(self._h, cluster, _ptr(v, ct.c_double)):
             raise ValueError("no BatchNorm state for this architecture")
+
+    def set_relu_masks(self, masks):
+        """ResNet-18 split: ReLU decisions ([C][B][resnet_mask_elems()], bit 0)
+        that the next round follows instead of its own sign tests."""
+        m = np.ascontiguousarray(masks, dtype=np.uint8)
+        assert m.size == self.C * self.B * resnet_mask_elems()
+        if lib().orc_set_relu_masks(self._h, _ptr(m, ct.c_uint8)):
+            raise ValueError("no ReLU records for this architecture")
+
+    def relu_masks(self):
+        """[C][B][E] ReLU records of the last round: bit 0 decision used, bit 1
+        own sign, bit 2 within the tolerance of 0 (set_relu_tol), bit 3
+        within five times it."""
+        out = np.zeros((self.C, self.B, resnet_mask_elems()), dtype=np.uint8)
+        if lib().orc_get_relu_masks(self._h, _ptr(out, ct.c_uint8)):
+            raise ValueError("no ReLU records for this architecture")
+        return out
 
     def momentum(self, cluster: int):
         out = np.zeros(self.P_client + self.P_server)

@@ -42,10 +42,12 @@
 
 /* the CIFAR ResNet-18 split model (architecture 2), gcpsl_resnet.c */
 int64_t orn_num_params(int segment);
-int orn_forward_backward(int bf16, double label_smoothing, const double* params,
-                         double* bn_state, int B, const double* x, const int32_t* labels,
-                         double* loss_out, double* grad, double* cut_act, double* cut_grad,
-                         double* logits_out);
+int orn_forward_backward_masks(int bf16, double label_smoothing, const double* params,
+                               double* bn_state, int B, const double* x,
+                               const int32_t* labels, double* loss_out, double* grad,
+                               double* cut_act, double* cut_grad, double* logits_out,
+                               const uint8_t* masks_in, uint8_t* masks_out);
+int64_t orn_mask_elems(void);
 void orn_init_bn_state(double* state);
 #define ORC_RESNET18 2
 
@@ -539,6 +541,9 @@ typedef struct {
   work_t w;
   double* xbuf; int32_t* ybuf;
   int resnet;                                 /* architecture 2 */
+  uint8_t* relu_rec;                          /* [C][B][E] ReLU records of the last round */
+  uint8_t* relu_in;                           /* [C][B][E] decisions to replay next round */
+  int replay;
   int64_t S;                                  /* BatchNorm state per replica (resnet) */
   double* bn;                                 /* [C][S] running mean / var */
   double tie_tol;                             /* see relu_pool_fwd */
@@ -626,7 +631,10 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   if (resnet) {
     c->xbuf = (double*)calloc((size_t)B * 3072, sizeof(double));
     c->bn = (double*)calloc((size_t)(C * c->S > 0 ? C * c->S : 1), sizeof(double));
-    if (!c->xbuf || !c->bn) { orc_destroy(c); return ORC_ENOMEM; }
+    const int64_t E = orn_mask_elems();
+    c->relu_rec = (uint8_t*)calloc((size_t)(C * B * E), 1);
+    c->relu_in = (uint8_t*)calloc((size_t)(C * B * E), 1);
+    if (!c->xbuf || !c->bn || !c->relu_rec || !c->relu_in) { orc_destroy(c); return ORC_ENOMEM; }
     for (int k = 0; k < C; ++k) orn_init_bn_state(c->bn + k * c->S);
   }
   if (!c->theta || !c->mom || !c->grad || !c->cut_act || !c->cut_grad ||
@@ -641,7 +649,7 @@ void orc_destroy(orc_ctx* c) {
   free(c->ids); free(c->perm); free(c->nc); free(c->cur_epoch); free(c->q);
   free(c->labels); free(c->owner); free(c->theta); free(c->mom); free(c->grad);
   free(c->idx); free(c->counts); free(c->loss); free(c->active);
-  free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties); free(c->xbuf); free(c->bn);
+  free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties); free(c->xbuf); free(c->bn); free(c->relu_rec); free(c->relu_in);
   for (int i = 0; i < 4; ++i) free(c->cand[i]);
   work_free(&c->w);
   free(c);
@@ -701,9 +709,11 @@ int orc_step(orc_ctx* c) {
         c->ybuf[b] = c->labels[idx[b]];
       }
       int64_t P = c->o.p_total;
-      int rc = orn_forward_backward(c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B,
-                                    c->xbuf, c->ybuf, &c->loss[k], c->grad + k * P,
-                                    c->cut_act + k * c->ncut, c->cut_grad + k * c->ncut, NULL);
+      const int64_t E = orn_mask_elems();
+      int rc = orn_forward_backward_masks(
+          c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B, c->xbuf, c->ybuf, &c->loss[k],
+          c->grad + k * P, c->cut_act + k * c->ncut, c->cut_grad + k * c->ncut, NULL,
+          c->replay ? c->relu_in + (int64_t)k * B * E : NULL, c->relu_rec + (int64_t)k * B * E);
       if (rc) return rc;
       continue;
     }
@@ -731,6 +741,7 @@ int orc_step(orc_ctx* c) {
     memcpy(c->cut_grad + k * c->ncut, c->w.dact[c->a.ncl], sizeof(double) * (size_t)c->ncut);
   }
   for (int k = 0; k < c->C; ++k) sgd(c, k);
+  c->replay = 0;
   c->t++;
   if (c->F > 0 && c->t % c->F == 0) return orc_fuse(c);
   return ORC_OK;
@@ -762,6 +773,21 @@ int orc_set_params(orc_ctx* c, int cluster, const double* blob) {
 int orc_set_bn_state(orc_ctx* c, int cluster, const double* src) {
   if (!c->resnet || cluster < 0 || cluster >= c->C) return ORC_EINVAL;
   memcpy(c->bn + (int64_t)cluster * c->S, src, sizeof(double) * (size_t)c->S);
+  return ORC_OK;
+}
+
+/* ResNet-18 split: ReLU decisions to replay in the next round ([C][B][E],
+ * bit 0 used), and the records of the last round (bits as in
+ * gcpsl_resnet.c's norm_fwd); E = orn_mask_elems() */
+int orc_set_relu_masks(orc_ctx* c, const uint8_t* src) {
+  if (!c->resnet) return ORC_EINVAL;
+  memcpy(c->relu_in, src, (size_t)(c->C * c->B * orn_mask_elems()));
+  c->replay = 1;
+  return ORC_OK;
+}
+int orc_get_relu_masks(const orc_ctx* c, uint8_t* dst) {
+  if (!c->resnet) return ORC_EINVAL;
+  memcpy(dst, c->relu_rec, (size_t)(c->C * c->B * orn_mask_elems()));
   return ORC_OK;
 }
 

@@ -210,9 +210,18 @@ static int64_t nset_elem(const nset* q, int i, int64_t e, int* ch) {
 }
 
 /* out = gamma * x_hat + beta (+ res), then ReLU when relu; mean / rstd per set */
+/* With relu, mask[k] records the decision: bit 0 = the output passes the
+ * ReLU (the decision used), bit 1 = the pre-ReLU value is positive (this
+ * run's own sign), bit 2 = ambiguous: |value| <= relu_tol * RMS of the
+ * layer's pre-ReLU values, bit 3 = |value| <= 5 relu_tol * RMS.  When mask_in is set, its bit 0 replaces the
+ * sign test (replaying another run's decisions; the output is then the
+ * value wherever the given decision passes). */
+static double g_relu_tol = 0.0;
+void orn_set_relu_tol(double tol) { g_relu_tol = tol; }
+
 static void norm_fwd(const nset* q, const double* y, const double* gamma, const double* beta,
                      const double* res, int relu, double* out, double* mean, double* rstd,
-                     double* var_biased) {
+                     double* var_biased, uint8_t* mask, const uint8_t* mask_in) {
   const int ns = nset_count(q);
   const int64_t n = nset_size(q);
 #pragma omp parallel for schedule(static)
@@ -231,8 +240,20 @@ static void norm_fwd(const nset* q, const double* y, const double* gamma, const 
       const int64_t k = nset_elem(q, i, e, &ch);
       double o = gamma[ch] * (y[k] - mu) * r + beta[ch];
       if (res) o += res[k];
-      out[k] = relu ? (o > 0.0 ? o : 0.0) : o;
+      out[k] = o;                     /* pre-ReLU value; decisions below */
     }
+  }
+  if (!relu) return;
+  const int64_t total = (int64_t)ns * n;
+  double ss = 0.0;
+  for (int64_t k = 0; k < total; ++k) ss += out[k] * out[k];
+  const double thr = g_relu_tol * sqrt(ss / (double)total);
+  for (int64_t k = 0; k < total; ++k) {
+    const double o = out[k];
+    const uint8_t own = (uint8_t)(o > 0.0);
+    const uint8_t pass = mask_in ? (uint8_t)(mask_in[k] & 1u) : own;
+    mask[k] = (uint8_t)(pass | (own << 1) | ((fabs(o) <= thr) << 2) | ((fabs(o) <= 5.0 * thr) << 3));
+    out[k] = pass ? o : 0.0;
   }
 }
 
@@ -280,6 +301,7 @@ typedef struct { double* y; double* mean; double* rstd; double* var; } rn_nsave;
 typedef struct {
   double* x;                       /* block input (a view of the previous output) */
   double* y1; double* a1; double* y2; double* ys; double* out;
+  uint8_t* m1; uint8_t* m2;        /* ReLU decisions of a1 and out */
   rn_nsave n1, n2, ns;
 } rn_bsave;
 
@@ -303,14 +325,58 @@ static void bn_running(const rn_norm* nm, const rn_nsave* sv, int64_t count, dou
   }
 }
 
+/* one ReLU's decisions between the per-example records [B][tot] and a
+ * [B][per] array (the ReLU's NCHW layout) */
+static void mask_gather(const uint8_t* rec, int64_t tot, int64_t off, int64_t per, int B,
+                        uint8_t* dst) {
+  for (int b = 0; b < B; ++b) memcpy(dst + (int64_t)b * per, rec + (int64_t)b * tot + off, (size_t)per);
+}
+static void mask_scatter(uint8_t* rec, int64_t tot, int64_t off, int64_t per, int B,
+                         const uint8_t* src) {
+  for (int b = 0; b < B; ++b) memcpy(rec + (int64_t)b * tot + off, src + (int64_t)b * per, (size_t)per);
+}
+
 /* One forward (and, with grad != NULL, backward) pass of the split model on
  * B examples x [B][3][32][32].  bn_state (nullable) is updated with this
  * batch's statistics.  cut_act / cut_grad (nullable) receive the client
  * output [B][64][32][32] and the gradient with respect to it. */
+int orn_forward_backward_masks(int bf16, double label_smoothing, const double* params,
+                               double* bn_state, int B, const double* x,
+                               const int32_t* labels, double* loss_out, double* grad,
+                               double* cut_act, double* cut_grad, double* logits_out,
+                               const uint8_t* masks_in, uint8_t* masks_out);
+
 int orn_forward_backward(int bf16, double label_smoothing, const double* params,
                          double* bn_state, int B, const double* x, const int32_t* labels,
                          double* loss_out, double* grad, double* cut_act, double* cut_grad,
                          double* logits_out) {
+  return orn_forward_backward_masks(bf16, label_smoothing, params, bn_state, B, x, labels,
+                                    loss_out, grad, cut_act, cut_grad, logits_out, NULL, NULL);
+}
+
+/* ReLU decisions per example: the stem's then, per block, those of a1 and of
+ * the block output, NCHW; returns the byte count per example. */
+int64_t orn_mask_elems(void) {
+  rn_net n;
+  rn_build(&n);
+  int64_t e = 64 * 1024;
+  for (int i = 0; i < 8; ++i) {
+    const int ho = out_hw(&n.blk[i].c1);
+    e += 2 * (int64_t)n.blk[i].c1.cout * ho * ho;
+  }
+  return e;
+}
+
+/* As orn_forward_backward; masks_out (nullable) receives every ReLU
+ * decision record ([B][orn_mask_elems()] in the order stem, block 0 a1,
+ * block 0 out, ...; bits as in norm_fwd), and masks_in (nullable) replaces
+ * the sign tests by the given decisions (bit 0), so that a run can follow
+ * another run's (e.g. the GPU's) branches exactly. */
+int orn_forward_backward_masks(int bf16, double label_smoothing, const double* params,
+                               double* bn_state, int B, const double* x,
+                               const int32_t* labels, double* loss_out, double* grad,
+                               double* cut_act, double* cut_grad, double* logits_out,
+                               const uint8_t* masks_in, uint8_t* masks_out) {
   rn_net n;
   rn_build(&n);
   if (B <= 0) return 1;
@@ -340,12 +406,31 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
   double* ystem = (double*)zal(stem_n);
   double* astem = (double*)zal(stem_n);
   rn_nsave sstem; nsave_alloc(&sstem, &n.stem_n, B);
+  uint8_t* mstem = (uint8_t*)calloc((size_t)stem_n, 1);
+  /* offsets of each ReLU's decisions within one example's mask record */
+  int64_t moff[17], mper[17];
+  {
+    int64_t o = 0;
+    mper[0] = 64 * 1024; moff[0] = o; o += mper[0];
+    for (int i = 0; i < 8; ++i) {
+      const int ho = out_hw(&n.blk[i].c1);
+      mper[1 + 2 * i] = mper[2 + 2 * i] = (int64_t)n.blk[i].c1.cout * ho * ho;
+      moff[1 + 2 * i] = o; o += mper[1 + 2 * i];
+      moff[2 + 2 * i] = o; o += mper[2 + 2 * i];
+    }
+  }
+  const int64_t mtot = moff[16] + mper[16];
+  /* gather / scatter one ReLU's [B][per] decisions from / to the records */
+  uint8_t* mtmp = (uint8_t*)calloc((size_t)B * 512 * 1024, 1);
+#define MASK_IN(r, dst)                                                          \
+  (masks_in ? (mask_gather(masks_in, mtot, moff[r], mper[r], B, dst), (const uint8_t*)(dst)) \
+            : (const uint8_t*)NULL)
   conv_fwd(&n.stem, B, x0, wr + n.stem.w, ystem);
   rn_round(ystem, stem_n, bf16);
   {
     nset q = nset_of(&n.stem_n, B, 1024);
     norm_fwd(&q, ystem, wr + n.stem_n.g, wr + n.stem_n.b, NULL, 1, astem, sstem.mean, sstem.rstd,
-             sstem.var);
+             sstem.var, mstem, MASK_IN(0, mtmp));
   }
   rn_round(astem, stem_n, bf16);
   rn_bsave sv[8];
@@ -359,12 +444,13 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
     s->x = (double*)cur;
     s->y1 = (double*)zal(on); s->a1 = (double*)zal(on); s->y2 = (double*)zal(on);
     s->out = (double*)zal(on);
+    s->m1 = (uint8_t*)calloc((size_t)on, 1); s->m2 = (uint8_t*)calloc((size_t)on, 1);
     nsave_alloc(&s->n1, &bk->n1, B); nsave_alloc(&s->n2, &bk->n2, B);
     conv_fwd(&bk->c1, B, cur, wr + bk->c1.w, s->y1);
     rn_round(s->y1, on, bf16);
     nset q1 = nset_of(&bk->n1, B, hw);
     norm_fwd(&q1, s->y1, wr + bk->n1.g, wr + bk->n1.b, NULL, 1, s->a1, s->n1.mean, s->n1.rstd,
-             s->n1.var);
+             s->n1.var, s->m1, MASK_IN(1 + 2 * i, mtmp));
     rn_round(s->a1, on, bf16);
     conv_fwd(&bk->c2, B, s->a1, wr + bk->c2.w, s->y2);
     rn_round(s->y2, on, bf16);
@@ -378,12 +464,12 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
       nset qs = nset_of(&bk->ns, B, hw);
       scv = (double*)zal(on);
       norm_fwd(&qs, s->ys, wr + bk->ns.g, wr + bk->ns.b, NULL, 0, scv, s->ns.mean, s->ns.rstd,
-               s->ns.var);
+               s->ns.var, NULL, NULL);
       res = scv;
     }
     nset q2 = nset_of(&bk->n2, B, hw);
     norm_fwd(&q2, s->y2, wr + bk->n2.g, wr + bk->n2.b, res, 1, s->out, s->n2.mean, s->n2.rstd,
-             s->n2.var);
+             s->n2.var, s->m2, MASK_IN(2 + 2 * i, mtmp));
     rn_round(s->out, on, bf16);
     free(scv);
     cur = s->out;
@@ -426,6 +512,13 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
     }
   }
   *loss_out = loss / B;
+  if (masks_out) {
+    mask_scatter(masks_out, mtot, moff[0], mper[0], B, mstem);
+    for (int i = 0; i < 8; ++i) {
+      mask_scatter(masks_out, mtot, moff[1 + 2 * i], mper[1 + 2 * i], B, sv[i].m1);
+      mask_scatter(masks_out, mtot, moff[2 + 2 * i], mper[2 + 2 * i], B, sv[i].m2);
+    }
+  }
   if (logits_out) memcpy(logits_out, logits, sizeof(double) * (size_t)B * RN_CLASSES);
   if (cut_act) memcpy(cut_act, sv[1].out, sizeof(double) * (size_t)stem_n);
 
@@ -460,7 +553,7 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
       const int64_t in_e = (int64_t)B * bk->c1.cin * bk->c1.hin * bk->c1.win;
       /* through the output ReLU */
       double* dz = (double*)zal(on);
-      for (int64_t k = 0; k < on; ++k) dz[k] = s->out[k] > 0.0 ? dout[k] : 0.0;
+      for (int64_t k = 0; k < on; ++k) dz[k] = (s->m2[k] & 1u) ? dout[k] : 0.0;
       double* dy2 = (double*)zal(on);
       nset q2 = nset_of(&bk->n2, B, hw);
       norm_bwd(&q2, s->y2, dz, wr + bk->n2.g, s->n2.mean, s->n2.rstd, dy2, grad + bk->n2.g,
@@ -470,7 +563,7 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
       double* da1 = (double*)zal(on);
       conv_dgrad_add(&bk->c2, B, dy2, wr + bk->c2.w, da1);
       rn_round(da1, on, bf16);
-      for (int64_t k = 0; k < on; ++k) if (!(s->a1[k] > 0.0)) da1[k] = 0.0;
+      for (int64_t k = 0; k < on; ++k) if (!(s->m1[k] & 1u)) da1[k] = 0.0;
       double* dy1 = (double*)zal(on);
       nset q1 = nset_of(&bk->n1, B, hw);
       norm_bwd(&q1, s->y1, da1, wr + bk->n1.g, s->n1.mean, s->n1.rstd, dy1, grad + bk->n1.g,
@@ -499,7 +592,7 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
     }
     /* stem: through its ReLU and GroupNorm, then the weight gradient */
     double* dz = (double*)zal(stem_n);
-    for (int64_t k = 0; k < stem_n; ++k) dz[k] = astem[k] > 0.0 ? dout[k] : 0.0;
+    for (int64_t k = 0; k < stem_n; ++k) dz[k] = (mstem[k] & 1u) ? dout[k] : 0.0;
     double* dy = (double*)zal(stem_n);
     nset q = nset_of(&n.stem_n, B, 1024);
     norm_bwd(&q, ystem, dz, wr + n.stem_n.g, sstem.mean, sstem.rstd, dy, grad + n.stem_n.g,
@@ -510,11 +603,13 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
   }
   for (int i = 0; i < 8; ++i) {
     rn_bsave* s = &sv[i];
-    free(s->y1); free(s->a1); free(s->y2); free(s->ys); free(s->out);
+    free(s->y1); free(s->a1); free(s->y2); free(s->ys); free(s->out); free(s->m1); free(s->m2);
     nsave_free(&s->n1); nsave_free(&s->n2);
     if (n.blk[i].sc) nsave_free(&s->ns);
   }
   nsave_free(&sstem);
+  free(mstem); free(mtmp);
+#undef MASK_IN
   free(ystem); free(astem); free(x0); free(h); free(logits); free(dlog); free(wr);
   return rc;
 }

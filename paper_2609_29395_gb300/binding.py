@@ -18,7 +18,7 @@ GCPSL_OK, GCPSL_E_INVAL, GCPSL_E_NOMEM, GCPSL_E_CUDA, GCPSL_E_STATE, GCPSL_E_TIM
     GCPSL_E_UNSUPPORTED = range(7)
 GCPSL_TINY_CNN, GCPSL_SPLIT_CNN, GCPSL_RESNET18 = 0, 1, 2
 GCPSL_F32, GCPSL_BF16 = 0, 1
-GCPSL_CLIENT, GCPSL_SERVER = 0, 1
+GCPSL_CLIENT, GCPSL_SERVER, GCPSL_BN_STATE = 0, 1, 2
 GCPSL_CUT_ACT, GCPSL_CUT_GRAD = 0, 1
 
 STATUS_NAMES = {0: "OK", 1: "E_INVAL", 2: "E_NOMEM", 3: "E_CUDA", 4: "E_STATE", 5: "E_TIMEOUT",
@@ -26,6 +26,7 @@ STATUS_NAMES = {0: "OK", 1: "E_INVAL", 2: "E_NOMEM", 3: "E_CUDA", 4: "E_STATE", 
 
 # every entry point declared in include/gcpsl.h
 EXPORTS = ("gcpsl_init", "gcpsl_step", "gcpsl_fuse", "gcpsl_get_params", "gcpsl_set_params",
+           "gcpsl_set_bn_state", "gcpsl_get_relu_masks",
            "gcpsl_get_momentum", "gcpsl_set_momentum", "gcpsl_get_pool_codes",
            "gcpsl_get_cut", "gcpsl_cut_elems", "gcpsl_get_sample", "gcpsl_num_params",
            "gcpsl_rounds", "gcpsl_set_stream", "gcpsl_set_graph", "gcpsl_set_timing",
@@ -91,6 +92,9 @@ def load() -> ct.CDLL:
     L.gcpsl_set_stream.argtypes = [vp, vp]
     L.gcpsl_set_timing.argtypes = [vp, ct.c_int]
     L.gcpsl_set_graph.argtypes = [vp, ct.c_int]
+    L.gcpsl_set_bn_state.argtypes = [vp, ct.c_int, f32p, ct.c_size_t]
+    L.gcpsl_get_relu_masks.argtypes = [vp, ct.POINTER(ct.c_uint8), ct.c_size_t,
+                                       ct.POINTER(ct.c_size_t)]
     L.gcpsl_set_timing_filter.argtypes = [vp, ct.c_char_p]
     L.gcpsl_kernels_launched.argtypes = [vp]
     L.gcpsl_kernels_launched.restype = ct.c_int64
@@ -109,7 +113,8 @@ def load() -> ct.CDLL:
     L.gcpsl_destroy.restype = None
     for name in ("gcpsl_init", "gcpsl_step", "gcpsl_fuse", "gcpsl_get_params", "gcpsl_set_params",
                  "gcpsl_get_cut", "gcpsl_get_sample", "gcpsl_set_stream", "gcpsl_set_timing",
-                 "gcpsl_set_graph", "gcpsl_set_timing_filter",
+                 "gcpsl_set_graph", "gcpsl_set_timing_filter", "gcpsl_set_bn_state",
+                 "gcpsl_get_relu_masks",
                  "gcpsl_get_momentum", "gcpsl_set_momentum", "gcpsl_get_pool_codes"):
         getattr(L, name).restype = ct.c_int
     _lib = L
@@ -214,6 +219,26 @@ class Context:
     def set_params(self, cluster: int, blob):
         blob = np.ascontiguousarray(blob, dtype=np.float32)
         _check(load().gcpsl_set_params(self._h, cluster, _p(blob, ct.c_float), blob.size), self._h)
+
+    def bn_state(self, cluster: int):
+        """BatchNorm running statistics of one replica (ResNet-18 split)."""
+        n = gcpsl_num_params(self.arch, GCPSL_BN_STATE)
+        out = np.empty(n, dtype=np.float32)
+        _check(load().gcpsl_get_params(self._h, cluster, GCPSL_BN_STATE, _p(out, ct.c_float), n,
+                                       None), self._h)
+        return out
+
+    def relu_masks(self):
+        """[C][B][E] ReLU decisions of the last round (ResNet-18 split)."""
+        n = ct.c_size_t(0)
+        _check(load().gcpsl_get_relu_masks(self._h, None, 0, ct.byref(n)), self._h)
+        out = np.empty(n.value, dtype=np.uint8)
+        _check(load().gcpsl_get_relu_masks(self._h, _p(out, ct.c_uint8), n.value, None), self._h)
+        return out.reshape(self.C, self.B, -1)
+
+    def set_bn_state(self, cluster: int, v):
+        v = np.ascontiguousarray(v, dtype=np.float32)
+        _check(load().gcpsl_set_bn_state(self._h, cluster, _p(v, ct.c_float), v.size), self._h)
 
     def momentum(self, cluster: int):
         n = self.P_client + self.P_server

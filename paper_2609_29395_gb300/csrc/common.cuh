@@ -147,8 +147,9 @@ cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_r
 // backward of the linear layer (dW, db, dh) and loss[c] = mean_b loss_ex[c][b].
 // route: FC_DH_STORE writes dh; FC_DH_POOL writes the last conv layer's g
 // (2Ho x 2Wo x ch) through its max-pool codes; FC_DH_RELU writes g = dh where
-// act > 0.  h is [Ho][Wo][ch] per example.
-enum { FC_DH_STORE = 0, FC_DH_POOL = 1, FC_DH_RELU = 2 };
+// act > 0; FC_DH_AVG writes dh / (Ho Wo) to every pixel of an Ho x Wo x ch
+// map (global average pool backward, h = [ch]).  Otherwise h is [Ho][Wo][ch].
+enum { FC_DH_STORE = 0, FC_DH_POOL = 1, FC_DH_RELU = 2, FC_DH_AVG = 3 };
 template <typename T>
 cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* loss_ex,
                           const T* h, const T* w, int64_t w_rs, float* dw, float* db,
@@ -205,8 +206,11 @@ struct WgradTcArgs {
   int bias = 1;         // also the bias gradient (a block of ones)
   int stride = 1, pad = 1;  // x pixel of output pixel p and tap (kh, kw): p*stride + k - pad
 };
+// elem_strides (nullable): traversal stride per dimension; a box then
+// loads ceil(box[i] / elem_strides[i]) elements along dimension i
 bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
-                     const uint32_t* box, int swizzle_bytes);
+                     const uint32_t* box, int swizzle_bytes,
+                     const uint32_t* elem_strides = nullptr);
 bool tensor_map_bf16_strided(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                              uint64_t outer_stride_bytes, const uint32_t* box, int swizzle_bytes);
 cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
@@ -224,6 +228,38 @@ cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtenso
 // (partials `per` apart)
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
                                 int splits, int64_t per, int C, int64_t count = -1);
+
+// norm.cu (GroupNorm with 32 groups / train-mode BatchNorm on [C][B][HW][ch]
+// bf16 tensors; statistics per set: GroupNorm (c, b, group), BatchNorm (c, ch))
+// per-(c, b, ch) pixel sums: forward (sum y, sum y^2); backward (sum dz,
+// sum dz x_hat) with dz = d (times [mask > 0], written to dz_out if set)
+cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16* d,
+                             const bf16* mask, const float* mean, const float* rstd, bf16* dz_out,
+                             float* sums, int C, int B, int HW, int ch, int gn);
+// per set: mean, rstd; BatchNorm also updates run ([C] x run_rs: mean[ch], var[ch])
+cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, float* mean, float* rstd,
+                                     float* run, int64_t run_rs, int C, int B, int HW, int ch,
+                                     int gn);
+// per set: m1 = mean(dz gamma), m2 = mean(dz gamma x_hat); per channel dgamma, dbeta
+cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,
+                                     int64_t g_rs, float* m1, float* m2, float* dgamma,
+                                     float* dbeta, int64_t d_rs, int C, int B, int HW, int ch,
+                                     int gn);
+// out = relu?(gamma x_hat + beta + r): r = res (bf16), or the second
+// normalised tensor y2 (its stats / affine), or 0
+cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float* mean,
+                                  const float* rstd, const float* gamma, const float* beta,
+                                  int64_t g_rs, const bf16* res, const bf16* y2,
+                                  const float* mean2, const float* rstd2, const float* gamma2,
+                                  const float* beta2, bf16* out, int C, int B, int HW, int ch,
+                                  int gn, int relu);
+// out = rstd (dz gamma - m1 - x_hat m2), dz = d (times [mask > 0])
+cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float* mean,
+                                  const float* rstd, const float* gamma, int64_t g_rs,
+                                  const float* m1, const float* m2, const bf16* d,
+                                  const bf16* mask, bf16* out, int C, int B, int HW, int ch,
+                                  int gn);
+cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch);
 
 // optim.cu
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,

@@ -872,7 +872,7 @@ static EncodeTiledFn encode_fn() {
 }
 
 bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
-                     const uint32_t* box, int swizzle_bytes) {
+                     const uint32_t* box, int swizzle_bytes, const uint32_t* elem_strides) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t gd[5], gs[4];
@@ -881,7 +881,7 @@ bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t*
   for (int i = 0; i < rank; ++i) {
     gd[i] = dims[i];
     bx[i] = box[i];
-    es[i] = 1;
+    es[i] = elem_strides ? elem_strides[i] : 1;
     if (i > 0) gs[i - 1] = stride;
     stride *= dims[i];
   }

@@ -152,10 +152,20 @@ int64_t act_elems(const gcpsl_ctx* c, int i) {   // elements of d_act[i]
 // ---------------------------------------------------------------------------
 // the packed input-layer weights, from the shadow (after every update)
 gcpsl_status refresh_derived(gcpsl_ctx* c) {
-  if (c->tc0.on)
-    LAUNCH("pack_w0", launch_pack_w0(c->stream, c->d_shadow + c->a.off_w[0], c->d_w0p, c->P_pad,
-                                     c->a.conv[0].cout, c->C));
+  if (c->tc0.on || c->rn)
+    LAUNCH("pack_w0", launch_pack_w0(c->stream, c->d_shadow + c->w0_off, c->d_w0p, c->P_pad,
+                                     c->w0_cout, c->C));
   return GCPSL_OK;
+}
+
+// canonical <-> kernel parameter layout of the context's architecture
+void to_kernel(const gcpsl_ctx* c, const float* can, float* ker) {
+  if (c->rn) rn_to_kernel_layout(can, ker);
+  else to_kernel_layout(c->a, can, ker);
+}
+void to_canonical(const gcpsl_ctx* c, const float* ker, float* can) {
+  if (c->rn) rn_to_canonical_layout(ker, can);
+  else to_canonical_layout(c->a, ker, can);
 }
 
 }  // namespace
@@ -186,21 +196,14 @@ bool epoch_boundary(const gcpsl_ctx* c) {
   return false;
 }
 
+// GPSL sampling (Eq. 1) and the gather of the sampled images.  The epoch
+// permutation is rebuilt only when some cluster starts an epoch; the host
+// round count equals the device one, so other rounds skip those launches
+// (the kernels also check the device counter themselves).
 template <typename T>
-gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
+gcpsl_status enqueue_sample(gcpsl_ctx* c, bool boundary) {
   cudaStream_t s = c->stream;
-  const ArchSpec& a = c->a;
   const int C = c->C, B = c->B;
-  const int64_t P = c->P_pad;
-  const T* wts = c->bf ? (const T*)(const void*)c->d_shadow : (const T*)(const void*)c->d_theta;
-  T* act[5];
-  T* dact[5];
-  for (int i = 0; i <= a.L(); ++i) { act[i] = (T*)c->d_act[i]; dact[i] = (T*)c->d_dact[i]; }
-
-  // GPSL sampling (Eq. 1) and the gather of the sampled images.  The epoch
-  // permutation is rebuilt only when some cluster starts an epoch; the host
-  // round count equals the device one, so other rounds skip those launches
-  // (the kernels also check the device counter themselves).
   if (boundary) {
     LAUNCH("epoch_keys", launch_epoch_keys(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
                                            c->desc.cluster_id_base, c->seed, c->d_keys, C,
@@ -211,7 +214,34 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
   LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_t, c->d_owner,
                                  c->d_labels, c->K, B, C, c->d_idx, c->d_counts, c->d_active,
                                  c->d_y));
-  LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, act[0]));
+  LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, (T*)c->d_act[0]));
+  return GCPSL_OK;
+}
+
+gcpsl_status enqueue_sgd(gcpsl_ctx* c) {
+  LAUNCH("sgd", launch_sgd(c->stream, c->d_theta, c->d_mom, c->d_grad, c->d_shadow,
+                           (int64_t)c->C * c->P_pad, c->desc.lr, c->desc.momentum,
+                           c->desc.weight_decay, c->desc.nesterov, c->d_t));
+  return refresh_derived(c);
+}
+
+template <typename T>
+gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
+  gcpsl_status st0 = enqueue_sample<T>(c, boundary);
+  if (st0 != GCPSL_OK) return st0;
+  if (c->rn) {
+    st0 = rn_enqueue_round(c);
+    if (st0 != GCPSL_OK) return st0;
+    return enqueue_sgd(c);
+  }
+  cudaStream_t s = c->stream;
+  const ArchSpec& a = c->a;
+  const int C = c->C, B = c->B;
+  const int64_t P = c->P_pad;
+  const T* wts = c->bf ? (const T*)(const void*)c->d_shadow : (const T*)(const void*)c->d_theta;
+  T* act[5];
+  T* dact[5];
+  for (int i = 0; i <= a.L(); ++i) { act[i] = (T*)c->d_act[i]; dact[i] = (T*)c->d_dact[i]; }
 
   // client segment to the cut, then the server segment
   for (int i = 0; i < a.L(); ++i) {
@@ -308,10 +338,7 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
                                                      cs));
     }
   }
-  LAUNCH("sgd", launch_sgd(s, c->d_theta, c->d_mom, c->d_grad, c->d_shadow, (int64_t)C * P,
-                           c->desc.lr, c->desc.momentum, c->desc.weight_decay,
-                           c->desc.nesterov, c->d_t));
-  return refresh_derived(c);
+  return enqueue_sgd(c);
 }
 
 // One round through a CUDA graph: captured on first use of its variant
@@ -379,6 +406,11 @@ void destroy_graphs(gcpsl_ctx* c) {
 gcpsl_status enqueue_fuse(gcpsl_ctx* c) {
   if (c->C == 1) return GCPSL_OK;                 // q_1 = 1: the identity
   LAUNCH("fuse", launch_fuse(c->stream, c->d_theta, c->d_shadow, c->d_q, c->C, c->P_pad));
+  if (c->rn) {                                    // BatchNorm running statistics, same q
+    int64_t S, S_pad;
+    float* bn = rn_bn_state(c, &S, &S_pad);
+    LAUNCH("fuse", launch_fuse(c->stream, bn, nullptr, c->d_q, c->C, S_pad));
+  }
   return refresh_derived(c);
 }
 
@@ -515,6 +547,7 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
 void free_all(gcpsl_ctx* c) {
   if (c->stream) cudaStreamSynchronize(c->stream);
   destroy_graphs(c);
+  rn_free(c);
   c->timer.destroy();
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
@@ -533,7 +566,8 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   c->esz = c->bf ? 2 : 4;
   c->x0c = c->bf ? 32 : 3;
   const ArchSpec& a = c->a;
-  c->P = a.p_total;
+  const bool resnet = desc->arch == GCPSL_RESNET18;
+  c->P = resnet ? rn_num_params(GCPSL_CLIENT) + rn_num_params(GCPSL_SERVER) : a.p_total;
   c->n = data->n;
 
   // clusters: ascending example ids per cluster, r_n, q_n (Eq. 5)
@@ -596,8 +630,10 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   // parameters: C identical replicas
   std::vector<float> can(c->P), ker(c->P);
   if (init_params) std::memcpy(can.data(), init_params, sizeof(float) * c->P);
+  else if (resnet) rn_seeded_init(seed, can.data());
   else seeded_init(a, seed, can.data());
-  to_kernel_layout(a, can.data(), ker.data());
+  if (resnet) rn_to_kernel_layout(can.data(), ker.data());
+  else to_kernel_layout(a, can.data(), ker.data());
   c->P_pad = (c->P + 63) / 64 * 64;
   const size_t pb = sizeof(float) * (size_t)(C * c->P_pad);
   DALLOC(c->d_theta, pb);
@@ -619,6 +655,33 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     for (int k = 0; k < C; ++k)
       CK(cudaMemcpy(c->d_shadow + (int64_t)k * c->P_pad, sh.data(), sizeof(bf16) * c->P,
                     cudaMemcpyHostToDevice));
+  }
+
+  if (resnet) {
+    // shared per-round buffers; the layers' own come from rn_setup
+    DALLOC(c->d_act[0], sizeof(bf16) * (size_t)C * B * 1024 * 32);
+    DALLOC(c->d_w0p, sizeof(bf16) * (size_t)C * 64 * 32);
+    DALLOC(c->d_loss_ex, sizeof(float) * C * B);
+    DALLOC(c->d_dlogits, sizeof(float) * C * B * 10);
+    DALLOC(c->d_y, sizeof(int32_t) * C * B);
+    DALLOC(c->d_idx, sizeof(int32_t) * C * B);
+    DALLOC(c->d_counts, sizeof(int32_t) * (size_t)C * K);
+    DALLOC(c->d_active, sizeof(int32_t) * C);
+    DALLOC(c->d_loss, sizeof(float) * C);
+    DALLOC(c->d_t, sizeof(int64_t));
+    CK(cudaMemset(c->d_t, 0, sizeof(int64_t)));
+    CK(cudaMemset(c->d_idx, 0, sizeof(int32_t) * C * B));
+    CK(cudaMemset(c->d_counts, 0, sizeof(int32_t) * (size_t)C * K));
+    CK(cudaHostAlloc((void**)&c->h_loss, sizeof(float) * C, cudaHostAllocDefault));
+    CK(cudaHostAlloc((void**)&c->h_active, sizeof(int32_t) * C, cudaHostAllocDefault));
+    c->w0_off = 0;                                // the stem convolution
+    c->w0_cout = 64;
+    gcpsl_status st = rn_setup(c);
+    if (st != GCPSL_OK) return st;
+    st = refresh_derived(c);
+    if (st != GCPSL_OK) return st;
+    CK(cudaDeviceSynchronize());
+    return GCPSL_OK;
   }
 
   // activations of one round
@@ -660,6 +723,8 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     bpart = std::max(bpart, (int64_t)C * R.splits * ((int64_t)s.cout * 9 * s.cin + s.cout));
   }
   DALLOC(c->d_bpartial, sizeof(float) * bpart);
+  c->w0_off = a.off_w[0];
+  c->w0_cout = a.conv[0].cout;
   if (c->bf) {
     gcpsl_status st = setup_tensor_core_layers(c);
     if (st != GCPSL_OK) return st;
@@ -678,6 +743,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
 extern "C" {
 
 int64_t gcpsl_num_params(int arch, int segment) {
+  if (arch == GCPSL_RESNET18) return rn_num_params(segment);
   ArchSpec a;
   if (!make_arch(arch, &a)) return -1;
   if (segment == GCPSL_CLIENT) return a.p_client;
@@ -703,8 +769,13 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
   if (!(desc->lr >= 0.f) || !(desc->label_smoothing >= 0.f && desc->label_smoothing < 1.f))
     return fail(nullptr, GCPSL_E_INVAL, "bad lr or label_smoothing");
   ArchSpec a;
-  if (!make_arch(desc->arch, &a))
+  std::memset(&a, 0, sizeof(a));
+  if (desc->arch == GCPSL_RESNET18) {
+    if (desc->operand_dtype != GCPSL_BF16)
+      return fail(nullptr, GCPSL_E_UNSUPPORTED, "the ResNet-18 split runs with bf16 operands");
+  } else if (!make_arch(desc->arch, &a)) {
     return fail(nullptr, GCPSL_E_UNSUPPORTED, "architecture %d is not built", desc->arch);
+  }
   for (int k = 0; k < K; ++k)
     if (assignment[k] < -1 || assignment[k] >= C)
       return fail(nullptr, GCPSL_E_INVAL, "assignment[%d]=%d outside [-1, %d)", k, assignment[k], C);
@@ -769,10 +840,22 @@ gcpsl_status gcpsl_get_params(gcpsl_ctx* c, int cluster, int segment, float* dst
                               size_t* needed) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
-  if (cluster < 0 || cluster >= c->C || (segment != GCPSL_CLIENT && segment != GCPSL_SERVER))
+  if (cluster < 0 || cluster >= c->C ||
+      (segment != GCPSL_CLIENT && segment != GCPSL_SERVER && !(segment == GCPSL_BN_STATE && c->rn)))
     return fail(c, GCPSL_E_INVAL, "bad cluster %d or segment %d", cluster, segment);
-  const int64_t lo = segment == GCPSL_CLIENT ? 0 : c->a.p_client;
-  const int64_t hi = segment == GCPSL_CLIENT ? c->a.p_client : c->a.p_total;
+  if (segment == GCPSL_BN_STATE) {
+    int64_t S, S_pad;
+    const float* bn = rn_bn_state(c, &S, &S_pad);
+    if (needed) *needed = (size_t)S;
+    if (!dst) return GCPSL_OK;
+    if (len < (size_t)S) return fail(c, GCPSL_E_INVAL, "dst too small");
+    SYNC_CHECK(c);
+    CK(cudaMemcpy(dst, bn + (int64_t)cluster * S_pad, sizeof(float) * S, cudaMemcpyDeviceToHost));
+    return GCPSL_OK;
+  }
+  const int64_t pc = c->rn ? rn_num_params(GCPSL_CLIENT) : c->a.p_client;
+  const int64_t lo = segment == GCPSL_CLIENT ? 0 : pc;
+  const int64_t hi = segment == GCPSL_CLIENT ? pc : c->P;
   if (needed) *needed = (size_t)(hi - lo);
   if (!dst) return GCPSL_OK;
   if (len < (size_t)(hi - lo)) return fail(c, GCPSL_E_INVAL, "dst too small");
@@ -780,7 +863,7 @@ gcpsl_status gcpsl_get_params(gcpsl_ctx* c, int cluster, int segment, float* dst
   SYNC_CHECK(c);
   CK(cudaMemcpy(ker.data(), c->d_theta + (int64_t)cluster * c->P_pad, sizeof(float) * c->P,
                 cudaMemcpyDeviceToHost));
-  to_canonical_layout(c->a, ker.data(), can.data());
+  to_canonical(c, ker.data(), can.data());
   std::memcpy(dst, can.data() + lo, sizeof(float) * (size_t)(hi - lo));
   return GCPSL_OK;
 }
@@ -791,7 +874,7 @@ gcpsl_status gcpsl_set_params(gcpsl_ctx* c, int cluster, const float* src, size_
   if (cluster < 0 || cluster >= c->C || !src || len != (size_t)c->P)
     return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
   std::vector<float> ker(c->P);
-  to_kernel_layout(c->a, src, ker.data());
+  to_kernel(c, src, ker.data());
   SYNC_CHECK(c);
   CK(cudaMemcpy(c->d_theta + (int64_t)cluster * c->P_pad, ker.data(), sizeof(float) * c->P,
                 cudaMemcpyHostToDevice));
@@ -805,6 +888,19 @@ gcpsl_status gcpsl_set_params(gcpsl_ctx* c, int cluster, const float* src, size_
   return GCPSL_OK;
 }
 
+gcpsl_status gcpsl_set_bn_state(gcpsl_ctx* c, int cluster, const float* src, size_t len) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (!c->rn) return fail(c, GCPSL_E_INVAL, "this architecture has no BatchNorm state");
+  int64_t S, S_pad;
+  float* bn = rn_bn_state(c, &S, &S_pad);
+  if (cluster < 0 || cluster >= c->C || !src || len != (size_t)S)
+    return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
+  SYNC_CHECK(c);
+  CK(cudaMemcpy(bn + (int64_t)cluster * S_pad, src, sizeof(float) * S, cudaMemcpyHostToDevice));
+  return GCPSL_OK;
+}
+
 gcpsl_status gcpsl_get_momentum(gcpsl_ctx* c, int cluster, float* dst, size_t len) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
@@ -814,7 +910,7 @@ gcpsl_status gcpsl_get_momentum(gcpsl_ctx* c, int cluster, float* dst, size_t le
   SYNC_CHECK(c);
   CK(cudaMemcpy(ker.data(), c->d_mom + (int64_t)cluster * c->P_pad, sizeof(float) * c->P,
                 cudaMemcpyDeviceToHost));
-  to_canonical_layout(c->a, ker.data(), dst);
+  to_canonical(c, ker.data(), dst);
   return GCPSL_OK;
 }
 
@@ -824,7 +920,7 @@ gcpsl_status gcpsl_set_momentum(gcpsl_ctx* c, int cluster, const float* src, siz
   if (cluster < 0 || cluster >= c->C || !src || len != (size_t)c->P)
     return fail(c, GCPSL_E_INVAL, "bad cluster, src or len");
   std::vector<float> ker(c->P);
-  to_kernel_layout(c->a, src, ker.data());
+  to_kernel(c, src, ker.data());
   SYNC_CHECK(c);
   CK(cudaMemcpy(c->d_mom + (int64_t)cluster * c->P_pad, ker.data(), sizeof(float) * c->P,
                 cudaMemcpyHostToDevice));
@@ -834,7 +930,7 @@ gcpsl_status gcpsl_set_momentum(gcpsl_ctx* c, int cluster, const float* src, siz
 gcpsl_status gcpsl_get_pool_codes(gcpsl_ctx* c, int layer, uint8_t* dst, size_t len) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
-  if (layer < 0 || layer >= c->a.L() || !c->a.conv[layer].pool || !dst)
+  if (c->rn || layer < 0 || layer >= c->a.L() || !c->a.conv[layer].pool || !dst)
     return fail(c, GCPSL_E_INVAL, "layer %d has no pooling or dst is NULL", layer);
   const int64_t n = act_elems(c, layer + 1);
   if (len < (size_t)n) return fail(c, GCPSL_E_INVAL, "dst too small");
@@ -848,23 +944,37 @@ gcpsl_status gcpsl_get_pool_codes(gcpsl_ctx* c, int layer, uint8_t* dst, size_t 
   return GCPSL_OK;
 }
 
+gcpsl_status gcpsl_get_relu_masks(gcpsl_ctx* c, uint8_t* dst, size_t len, size_t* needed) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (!c->rn) return fail(c, GCPSL_E_INVAL, "ReLU decisions are kept for the ResNet-18 split");
+  return rn_relu_masks(c, dst, len, needed);
+}
+
 size_t gcpsl_cut_elems(const gcpsl_ctx* c) {
   if (!c) return 0;
+  if (c->rn) return (size_t)c->C * c->B * 64 * 1024;
   return (size_t)act_elems(c, c->a.ncl);
 }
 
 gcpsl_status gcpsl_get_cut(gcpsl_ctx* c, int which, float* dst, size_t len) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;
-  const int64_t n = act_elems(c, c->a.ncl);
+  const int64_t n = (int64_t)gcpsl_cut_elems(c);
   if (!dst || len < (size_t)n || (which != GCPSL_CUT_ACT && which != GCPSL_CUT_GRAD))
     return fail(c, GCPSL_E_INVAL, "bad dst, len or which");
-  const void* src = which == GCPSL_CUT_ACT ? c->d_act[c->a.ncl] : c->d_dact[c->a.ncl];
+  const void* src = c->rn ? (const void*)rn_cut(c, which)
+                          : (which == GCPSL_CUT_ACT ? c->d_act[c->a.ncl] : c->d_dact[c->a.ncl]);
   std::vector<unsigned char> raw((size_t)n * c->esz);
   SYNC_CHECK(c);
   CK(cudaMemcpy(raw.data(), src, raw.size(), cudaMemcpyDeviceToHost));
-  const int l = c->a.ncl - 1;
-  const int ch = c->a.conv[l].cout, hw = c->a.out_h(l) * c->a.out_w(l);
+  int ch, hw;
+  if (c->rn) {
+    ch = 64; hw = 1024;
+  } else {
+    const int l = c->a.ncl - 1;
+    ch = c->a.conv[l].cout; hw = c->a.out_h(l) * c->a.out_w(l);
+  }
   for (int64_t cb = 0; cb < (int64_t)c->C * c->B; ++cb)
     for (int p = 0; p < hw; ++p)
       for (int k = 0; k < ch; ++k) {

@@ -151,6 +151,11 @@ struct gcpsl_ctx {
     CUtensorMap wgA, wgB;
   } tc0;
   int x0c = 3;
+  // the ResNet-18 split (architecture 2), else null
+  gcpsl::RnState* rn = nullptr;
+  // the input layer's packed weights: offset and output channels
+  int64_t w0_off = 0;
+  int w0_cout = 0;
   bf16* d_w0p = nullptr;
   float* d_partial = nullptr;      // weight-gradient split partials (tensor-core layers)
   // CUDA-core weight+bias gradient partials of the layers not on the tensor
@@ -207,6 +212,18 @@ struct gcpsl_ctx {
 namespace gcpsl {
 
 gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...);
+
+// resnet.cu: the ResNet-18 split (architecture 2)
+int64_t rn_num_params(int segment);              // GCPSL_CLIENT / SERVER / BN_STATE
+void rn_to_kernel_layout(const float* can, float* ker);
+void rn_to_canonical_layout(const float* ker, float* can);
+void rn_seeded_init(uint64_t seed, float* can);
+gcpsl_status rn_setup(gcpsl_ctx* c);
+void rn_free(gcpsl_ctx* c);
+gcpsl_status rn_enqueue_round(gcpsl_ctx* c);
+const bf16* rn_cut(const gcpsl_ctx* c, int which);
+gcpsl_status rn_relu_masks(gcpsl_ctx* c, uint8_t* dst, size_t len, size_t* needed);
+float* rn_bn_state(const gcpsl_ctx* c, int64_t* S, int64_t* S_pad);
 gcpsl_status check_device_error(gcpsl_ctx* c);
 gcpsl_status check_usable(gcpsl_ctx* c);
 // 128-pixel M tile of a W x H image: bw <= 16 columns, hb rows, bb images

@@ -171,6 +171,10 @@ __device__ __forceinline__ void put_dh(T* __restrict__ out, const HeadRoute& rt,
   const int64_t o = cb * fin + k;
   if (rt.mode == FC_DH_STORE) {
     store2<T>(out + o, d0, d1);
+  } else if (rt.mode == FC_DH_AVG) {
+    const int hw = rt.Ho * rt.Wo;
+    const float inv = 1.f / (float)hw;
+    for (int p = 0; p < hw; ++p) store2<T>(out + (cb * hw + p) * rt.ch + k, d0 * inv, d1 * inv);
   } else if (rt.mode == FC_DH_RELU) {
     const float2 a = load2<T>(reinterpret_cast<const T*>(rt.act) + o);
     store2<T>(out + o, a.x > 0.f ? d0 : 0.f, a.y > 0.f ? d1 : 0.f);
@@ -307,8 +311,10 @@ cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* los
   if (fout != kClasses || fin % 2 || w_rs % 2 || g_rs % 2 ||
       ((uintptr_t)w % (2 * sizeof(T))) || ((uintptr_t)dw % (2 * sizeof(float))))
     return cudaErrorInvalidValue;
-  if (route != FC_DH_STORE && (ch % 2 || (int64_t)Ho * Wo * ch != fin ||
-                               (route == FC_DH_POOL && !code) || (route == FC_DH_RELU && !act)))
+  if (route == FC_DH_AVG && (ch != fin || Ho * Wo < 1)) return cudaErrorInvalidValue;
+  if (route != FC_DH_STORE && route != FC_DH_AVG &&
+      (ch % 2 || (int64_t)Ho * Wo * ch != fin || (route == FC_DH_POOL && !code) ||
+       (route == FC_DH_RELU && !act)))
     return cudaErrorInvalidValue;
   const HeadRoute rt{route, code, act, Ho, Wo, ch};
   const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C);
