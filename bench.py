@@ -82,8 +82,68 @@ def load_peaks():
 # algorithmic work per kernel kind and round (FLOPs for contractions, bytes
 # for the elementwise/bandwidth kernels)
 # ---------------------------------------------------------------------------
+def work_per_round_resnet(w):
+    """Kernel kinds of the ResNet-18 split (per stage) and their FLOPs per
+    round: 2*C*B*Ho*Wo*cout*cin*k*k per convolution and pass (the stem has
+    no data gradient); the norm and pooling kernels as HBM bytes."""
+    from paper_2609_29395_gb300 import synth
+    C, B = w.num_clusters, w.B
+    work = {}
+
+    def add(kind, bound, v):
+        b, old = work.get(kind, (bound, 0.0))
+        work[kind] = (bound, old + v)
+
+    def conv(stage, cin, cout, k, stride, hin):
+        ho = hin // stride
+        f = 2.0 * C * B * ho * ho * cout * cin * k * k
+        name = "stem" if stage == 0 else f"s{stage}"
+        add(f"rn_conv_fwd.{name}", "tensor", f)
+        add(f"rn_conv_wgrad.{name}", "tensor", f)
+        if stage > 0:
+            add(f"rn_conv_dgrad.{name}", "tensor", f)
+
+    def norm(e, kind):
+        """HBM bytes of the norm kernels for one norm over E bf16 elements:
+        forward sums read y; apply reads y (+ the residual or the shortcut's
+        y) and writes out; backward sums read d, y (+ the ReLU output) and
+        may write dz; backward apply reads y, dz (+ mask) and writes dy."""
+        b = 2.0 * e
+        fwd_apply = {"n1": 2, "n2": 3, "stem": 2, "ns": 0}[kind]
+        bwd_sums = {"n1": 2, "n2": 4, "stem": 3, "ns": 2}[kind]
+        bwd_apply = {"n1": 3, "n2": 3, "stem": 4, "ns": 3}[kind]
+        add("rn_norm_sums", "hbm", b)
+        if fwd_apply:
+            add("rn_norm_apply", "hbm", fwd_apply * b)
+        add("rn_norm_bwd_sums", "hbm", bwd_sums * b)
+        add("rn_norm_bwd_apply", "hbm", bwd_apply * b)
+
+    conv(0, 3, 64, 3, 1, 32)
+    norm(C * B * 1024 * 64, "stem")
+    cin, hw = 64, 32
+    for st, (width, stride) in enumerate(synth.RESNET_STAGES):
+        for j in range(2):
+            s_ = stride if j == 0 else 1
+            ho = hw // s_
+            e = C * B * ho * ho * width
+            conv(st + 1, cin, width, 3, s_, hw)
+            conv(st + 1, width, width, 3, 1, ho)
+            norm(e, "n1")
+            norm(e, "n2")
+            if s_ != 1 or cin != width:
+                conv(st + 1, cin, width, 1, s_, hw)
+                norm(e, "ns")
+            cin, hw = width, ho
+    P = synth.num_params(w.arch, "client") + synth.num_params(w.arch, "server")
+    work["sgd"] = ("hbm", C * P * (4 * 5 + 2))
+    work["fuse"] = ("hbm", C * P * (4 + 4 + 2))
+    return work
+
+
 def work_per_round(w, esz):
     from paper_2609_29395_gb300 import synth
+    if w.arch == synth.ARCH_RESNET18:
+        return work_per_round_resnet(w)
     spec = synth.ARCHS[w.arch]
     convs = spec["client"] + spec["server"]
     C, B = w.num_clusters, w.B
@@ -187,6 +247,15 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------
+def _oracle_pass(oracle, w, blob, x, y):
+    """One forward+backward of the oracle on one replica's batch."""
+    from paper_2609_29395_gb300 import synth
+    if w.arch == synth.ARCH_RESNET18:
+        oracle.resnet_forward_backward(blob, x, y, bf16=w.bf16)
+    else:
+        oracle.forward_backward(w.arch, blob, x, y, bf16=w.bf16)
+
+
 def cpu_baseline(w, ds, assign, params, budget_s=15.0):
     """The oracle as it stands, on this host's cores: repeated forward/
     backward of a small batch of cluster-0 examples (bf16-operand mode when
@@ -197,7 +266,7 @@ def cpu_baseline(w, ds, assign, params, budget_s=15.0):
     y = ds.labels[ids]
     done, t0 = 0, time.perf_counter()
     while True:
-        oracle.forward_backward(w.arch, params.astype(np.float64), x, y, bf16=w.bf16)
+        _oracle_pass(oracle, w, params.astype(np.float64), x, y)
         done += len(ids)
         if time.perf_counter() - t0 > budget_s:
             break
@@ -221,7 +290,7 @@ def run_reference(args, w):
     blob = params.astype(np.float64)
 
     def one():
-        oracle.forward_backward(w.arch, blob, x, y, bf16=w.bf16)
+        _oracle_pass(oracle, w, blob, x, y)
     for _ in range(args.warmup):
         one()
     t0 = time.perf_counter()
@@ -291,13 +360,15 @@ def main():
         ctx.step()
     kinds = sorted(ctx.kernel_times())
     all_times = {}
+    kb = max(3, min(K, 10))                      # rounds per kind
     for kd in kinds:
         ctx.set_timing_filter(kd)
         ctx.reset_kernel_times()
-        for i in range(K):
+        for i in range(kb):
             flush.fill_(float(i))
             ctx.step()
-        all_times[kd] = ctx.kernel_times().get(kd, (0, 0.0))
+        n_, ms_ = ctx.kernel_times().get(kd, (0, 0.0))
+        all_times[kd] = (n_ * K / kb, ms_ * K / kb)  # per K rounds
     kind = max(all_times.items(), key=lambda kv: kv[1][1])[0]
 
     # the timed region: only the dominant kernel carries event records, so
@@ -368,7 +439,8 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.bf16 else "f32",
         "data": "synthetic",
         "config": {"workload": f"{w.name}: n={w.n} K={w.num_clients} C={w.num_clusters} "
-                               f"B={w.B} F={w.F} SplitCNN" if w.arch == 1 else w.name,
+                               f"B={w.B} F={w.F} "
+                               f"{ {1: 'SplitCNN', 2: 'ResNet-18 split'}.get(w.arch, '')}",
                    "global_batch": w.num_clusters * w.B * world, "parallelism": f"replicas{world}",
                    "l2": "flushed between timed steps (256 MiB write)"},
         "roofline": roof, "gpu_launches": launches, "wall_s": wall,

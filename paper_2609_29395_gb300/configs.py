@@ -42,6 +42,10 @@ WORKLOADS = {
                              synth.ARCH_SPLIT_CNN, True, 0.05, 0.9),
     "splitcnn_c64": Workload("splitcnn_c64", 50_000, 256, 0.3, True, 64, "label_greedy", 64, 25,
                              synth.ARCH_SPLIT_CNN, True, 0.05, 0.9),
+    # 200,000 images (20,000 per class), K = 1024, Dir(0.1), C = 8 random,
+    # B = 128, F = 100, the ResNet-18 split
+    "resnet18_c8": Workload("resnet18_c8", 200_000, 1024, 0.1, True, 8, "random", 128, 100,
+                            synth.ARCH_RESNET18, True, 0.05, 0.9),
 }
 
 

@@ -236,29 +236,27 @@ cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw,
 cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16* d,
                              const bf16* mask, const float* mean, const float* rstd, bf16* dz_out,
                              float* sums, int C, int B, int HW, int ch, int gn);
-// per set: mean, rstd; BatchNorm also updates run ([C] x run_rs: mean[ch], var[ch])
-cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, float* mean, float* rstd,
-                                     float* run, int64_t run_rs, int C, int B, int HW, int ch,
-                                     int gn);
-// per set: m1 = mean(dz gamma), m2 = mean(dz gamma x_hat); per channel dgamma, dbeta
+// per set: mean, rstd, and per (c, [b,] ch) the affine form ss = (gamma rstd,
+// beta - mean gamma rstd) (GroupNorm per example, BatchNorm shared over the
+// batch); BatchNorm also updates run ([C] x run_rs: mean[ch], var[ch])
+cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const float* gamma,
+                                     const float* beta, int64_t g_rs, float* mean, float* rstd,
+                                     float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
+                                     int ch, int gn);
+// backward affine form kk = (k1, k2, k3, 0): dy = k1 dz + k2 y + k3 per
+// (c, [b,] ch); per channel dgamma, dbeta
 cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,
-                                     int64_t g_rs, float* m1, float* m2, float* dgamma,
-                                     float* dbeta, int64_t d_rs, int C, int B, int HW, int ch,
-                                     int gn);
-// out = relu?(gamma x_hat + beta + r): r = res (bf16), or the second
-// normalised tensor y2 (its stats / affine), or 0
-cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float* mean,
-                                  const float* rstd, const float* gamma, const float* beta,
-                                  int64_t g_rs, const bf16* res, const bf16* y2,
-                                  const float* mean2, const float* rstd2, const float* gamma2,
-                                  const float* beta2, bf16* out, int C, int B, int HW, int ch,
-                                  int gn, int relu);
-// out = rstd (dz gamma - m1 - x_hat m2), dz = d (times [mask > 0])
-cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float* mean,
-                                  const float* rstd, const float* gamma, int64_t g_rs,
-                                  const float* m1, const float* m2, const bf16* d,
-                                  const bf16* mask, bf16* out, int C, int B, int HW, int ch,
-                                  int gn);
+                                     int64_t g_rs, const float* mean, const float* rstd,
+                                     float4* kk, float* dgamma, float* dbeta, int64_t d_rs, int C,
+                                     int B, int HW, int ch, int gn);
+// out = relu?(y scale + shift + r): r = res (bf16), or y2 scale2 + shift2, or 0
+cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float2* ss, int gn,
+                                  const bf16* res, const bf16* y2, const float2* ss2, int gn2,
+                                  bf16* out, int C, int B, int HW, int ch, int relu);
+// out = k1 dz + k2 y + k3, dz = d (times [mask > 0])
+cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* kk, int gn,
+                                  const bf16* d, const bf16* mask, bf16* out, int C, int B, int HW,
+                                  int ch);
 cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch);
 
 // optim.cu

@@ -11,7 +11,8 @@
 //
 // Both directions go through per-(example, channel) partial sums over the
 // pixels (fp32, pixels in a fixed order), combined per set in fp64 by a
-// small finalize kernel, then an elementwise apply.  Every sum has a fixed
+// small finalize kernel (which also folds the normalisation into a
+// per-channel affine form), then an elementwise apply.  Every sum has a fixed
 // order, so results do not depend on C or on launch geometry.
 #include "common.cuh"
 
@@ -113,187 +114,235 @@ k_chan_sums(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* 
   }
 }
 
-// Forward statistics per set from the (b, channel) sums, in fp64; BatchNorm
-// also updates its running statistics (momentum 0.1, unbiased variance).
-__global__ void k_norm_finalize_fwd(const float* __restrict__ sums, float* __restrict__ mean,
-                                    float* __restrict__ rstd, float* __restrict__ run,
+// One warp per (replica, set) [GroupNorm (b, group) / BatchNorm channel]:
+// the set's sums in a fixed lane order (xor tree), in fp64.
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Forward statistics per set, and per (replica, [example,] channel) the
+// affine form of the normalisation: scale = gamma * rstd, shift = beta -
+// mean * scale (GroupNorm: per example; BatchNorm: shared over the batch).
+// BatchNorm also updates its running statistics (momentum 0.1, unbiased
+// variance).
+__global__ void k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ gamma,
+                                    const float* __restrict__ beta, int64_t g_rs,
+                                    float* __restrict__ mean, float* __restrict__ rstd,
+                                    float2* __restrict__ ss, float* __restrict__ run,
                                     int64_t run_rs, int C, int B, int HW, int ch, int gn) {
   pdl_wait();
   pdl_trigger();
-  const int sets = gn ? B * 32 : ch;
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (int64_t)C * sets) return;
-  const int c = (int)(i / sets), s = (int)(i % sets);
-  double s1 = 0.0, s2 = 0.0, n;
+  const int cpg = ch / 32;
   if (gn) {
-    const int b = s / 32, g = s % 32, cpg = ch / 32;
+    // GroupNorm: one thread per (replica, example, group)
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)C * B * 32) return;
+    const int64_t cbv = i / 32;                     // c * B + b
+    const int g = (int)(i % 32), c = (int)(cbv / B);
+    double s1 = 0.0, s2 = 0.0;
     for (int k = 0; k < cpg; ++k) {
-      const int64_t o = (((int64_t)c * B + b) * ch + g * cpg + k) * 2;
+      const int64_t o = (cbv * ch + g * cpg + k) * 2;
       s1 += sums[o]; s2 += sums[o + 1];
     }
-    n = (double)cpg * HW;
-  } else {
-    for (int b = 0; b < B; ++b) {
-      const int64_t o = (((int64_t)c * B + b) * ch + s) * 2;
-      s1 += sums[o]; s2 += sums[o + 1];
+    const double n = (double)cpg * HW, mu = s1 / n;
+    double var = s2 / n - mu * mu;
+    var = var > 0.0 ? var : 0.0;
+    const double r = 1.0 / sqrt(var + kEps);
+    mean[i] = (float)mu;
+    rstd[i] = (float)r;
+    const float* gm = gamma + (int64_t)c * g_rs;
+    const float* bt = beta + (int64_t)c * g_rs;
+    for (int k = 0; k < cpg; ++k) {
+      const int chn = g * cpg + k;
+      const float sc = (float)((double)gm[chn] * r);
+      ss[cbv * ch + chn] = make_float2(sc, (float)((double)bt[chn] - mu * sc));
     }
-    n = (double)B * HW;
+    return;
   }
-  const double mu = s1 / n;
+  // BatchNorm: one warp per (replica, channel), lanes over the batch
+  const int lane = threadIdx.x & 31;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (w >= (int64_t)C * ch) return;
+  const int c = (int)(w / ch), s = (int)(w % ch);
+  double s1 = 0.0, s2 = 0.0;
+  for (int b = lane; b < B; b += 32) {
+    const int64_t o = (((int64_t)c * B + b) * ch + s) * 2;
+    s1 += sums[o]; s2 += sums[o + 1];
+  }
+  s1 = warp_sum(s1);
+  s2 = warp_sum(s2);
+  if (lane != 0) return;
+  const double n = (double)B * HW, mu = s1 / n;
   double var = s2 / n - mu * mu;
   var = var > 0.0 ? var : 0.0;
-  mean[i] = (float)mu;
-  rstd[i] = (float)(1.0 / sqrt(var + kEps));
-  if (!gn && run) {
+  const double r = 1.0 / sqrt(var + kEps);
+  mean[w] = (float)mu;
+  rstd[w] = (float)r;
+  if (run) {
     float* rm = run + (int64_t)c * run_rs;
     float* rv = rm + ch;
     rm[s] = (float)(0.9 * (double)rm[s] + 0.1 * mu);
     rv[s] = (float)(0.9 * (double)rv[s] + 0.1 * var * n / (n - 1.0));
   }
+  const float gsv = gamma[(int64_t)c * g_rs + s], bsv = beta[(int64_t)c * g_rs + s];
+  const float sc = (float)((double)gsv * r);
+  ss[(int64_t)c * ch + s] = make_float2(sc, (float)((double)bsv - mu * sc));
 }
 
-// Backward set constants m1, m2 and the affine gradients.
-//   GroupNorm set (b, g): m1 = sum_{c in g} gamma_c S1[b][c] / n,
-//                         m2 = sum_{c in g} gamma_c S2[b][c] / n;
-//   BatchNorm set c:      m1 = gamma_c sum_b S1[b][c] / n, m2 likewise;
-//   dgamma_c = sum_b S2[b][c], dbeta_c = sum_b S1[b][c].
+// Backward: per set m1 = mean(dz gamma), m2 = mean(dz gamma x_hat), and the
+// affine form dy = k1 dz + k2 y + k3 with k1 = gamma rstd, k2 = -rstd^2 m2,
+// k3 = rstd^2 m2 mean - rstd m1 (GroupNorm per example, BatchNorm shared);
+// per channel dgamma = sum_b S2[b][c], dbeta = sum_b S1[b][c].
+//   GroupNorm set (b, g): m1 = sum_{c in g} gamma_c S1[b][c] / n (m2 with S2);
+//   BatchNorm set c:      m1 = gamma_c sum_b S1[b][c] / n.
 __global__ void k_norm_finalize_bwd(const float* __restrict__ sums,
                                     const float* __restrict__ gamma, int64_t g_rs,
-                                    float* __restrict__ m1, float* __restrict__ m2,
-                                    float* __restrict__ dgamma, float* __restrict__ dbeta,
-                                    int64_t d_rs, int C, int B, int HW, int ch, int gn) {
+                                    const float* __restrict__ mean, const float* __restrict__ rstd,
+                                    float4* __restrict__ kk, float* __restrict__ dgamma,
+                                    float* __restrict__ dbeta, int64_t d_rs, int C, int B, int HW,
+                                    int ch, int gn) {
   pdl_wait();
   pdl_trigger();
-  const int sets = gn ? B * 32 : ch;
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t total = (int64_t)C * (sets > ch ? sets : ch);
-  if (i >= total) return;
-  const int c = (int)(i / (sets > ch ? sets : ch)), s = (int)(i % (sets > ch ? sets : ch));
-  const float* gm = gamma + (int64_t)c * g_rs;
-  if (s < sets) {
-    double a = 0.0, b2 = 0.0, n;
-    if (gn) {
-      const int b = s / 32, g = s % 32, cpg = ch / 32;
-      for (int k = 0; k < cpg; ++k) {
-        const int chn = g * cpg + k;
-        const int64_t o = (((int64_t)c * B + b) * ch + chn) * 2;
-        a += (double)gm[chn] * sums[o];
-        b2 += (double)gm[chn] * sums[o + 1];
-      }
-      n = (double)cpg * HW;
-    } else {
-      for (int b = 0; b < B; ++b) {
-        const int64_t o = (((int64_t)c * B + b) * ch + s) * 2;
-        a += sums[o]; b2 += sums[o + 1];
-      }
-      a *= gm[s]; b2 *= gm[s];
-      n = (double)B * HW;
+  const int cpg = ch / 32;
+  // warps [0, C*ch): per channel over the batch (dgamma, dbeta; the whole
+  // BatchNorm set); GroupNorm sets follow, one thread each
+  const int64_t nw = (int64_t)C * ch;
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t w = t >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w < nw) {
+    const int c = (int)(w / ch), chn = (int)(w % ch);
+    double a = 0.0, b2 = 0.0;
+    for (int b = lane; b < B; b += 32) {
+      const int64_t o = (((int64_t)c * B + b) * ch + chn) * 2;
+      a += sums[o]; b2 += sums[o + 1];
     }
-    m1[(int64_t)c * sets + s] = (float)(a / n);
-    m2[(int64_t)c * sets + s] = (float)(b2 / n);
+    a = warp_sum(a);
+    b2 = warp_sum(b2);
+    if (lane != 0) return;
+    dgamma[(int64_t)c * d_rs + chn] = (float)b2;
+    dbeta[(int64_t)c * d_rs + chn] = (float)a;
+    if (!gn) {
+      const double g = gamma[(int64_t)c * g_rs + chn];
+      const double n = (double)B * HW;
+      const double m1 = g * a / n, m2 = g * b2 / n;
+      const double mu = mean[w], r = rstd[w];
+      kk[w] = make_float4((float)(g * r), (float)(-r * r * m2), (float)(r * r * m2 * mu - r * m1),
+                          0.f);
+    }
+    return;
   }
-  if (s < ch) {
-    double dg = 0.0, db = 0.0;
-    for (int b = 0; b < B; ++b) {
-      const int64_t o = (((int64_t)c * B + b) * ch + s) * 2;
-      db += sums[o]; dg += sums[o + 1];
-    }
-    dgamma[(int64_t)c * d_rs + s] = (float)dg;
-    dbeta[(int64_t)c * d_rs + s] = (float)db;
+  if (!gn) return;
+  const int64_t i = t - nw * 32;                   // GroupNorm set (c, b, g)
+  if (i < 0 || i >= (int64_t)C * B * 32) return;
+  const int64_t cbv = i / 32;
+  const int g = (int)(i % 32), c = (int)(cbv / B);
+  const float* gm = gamma + (int64_t)c * g_rs;
+  double a = 0.0, b2 = 0.0;
+  for (int k = 0; k < cpg; ++k) {
+    const int chn = g * cpg + k;
+    const int64_t o = (cbv * ch + chn) * 2;
+    a += (double)gm[chn] * sums[o];
+    b2 += (double)gm[chn] * sums[o + 1];
+  }
+  const double n = (double)cpg * HW;
+  const double m1 = a / n, m2 = b2 / n;
+  const double mu = mean[i], r = rstd[i];
+  for (int k = 0; k < cpg; ++k) {
+    const int chn = g * cpg + k;
+    kk[cbv * ch + chn] = make_float4((float)(gm[chn] * r), (float)(-r * r * m2),
+                                     (float)(r * r * m2 * mu - r * m1), 0.f);
   }
 }
 
-// Elementwise, one thread per 8 channels of one pixel.
-//   forward: out = relu?(gamma (y - mu) rstd + beta + r), with r = 0, the
-//            bf16 tensor res, or a second normalised tensor y2 (its own
-//            stats and affine);
-//   backward: out = rstd (dz gamma - m1 - x_hat m2), dz = d (times
-//            [mask > 0] when mask is set).
-struct NormTerm {
-  const bf16* y;
-  const float* mean;
-  const float* rstd;
-  const float* gamma;       // replica 0; replica stride g_rs
-  const float* beta;
-  int64_t g_rs;
-};
-
+// Elementwise with the per-channel affine forms of the finalize kernels
+// (GroupNorm: per example, BatchNorm: shared over the batch).  A block per
+// (replica, example, pixel chunk): thread = 8 channels x a pixel lane, so
+// each thread loads its affine coefficients once.
+//   forward:  out = relu?(y scale + shift + r), r = res (bf16), or
+//             y2 scale2 + shift2 (the shortcut's norm), or 0;
+//   backward: out = k1 dz + k2 y + k3, dz = d (times [mask > 0]).
+constexpr int kApplyPixels = 256;        // pixels per block at most
 template <bool BWD>
 __global__ void __launch_bounds__(kThreads)
-k_norm_apply(NormTerm t, NormTerm t2, const bf16* __restrict__ res, const bf16* __restrict__ d,
+k_norm_apply(const bf16* __restrict__ y, const void* __restrict__ aff, int aff_gn,
+             const bf16* __restrict__ y2, const float2* __restrict__ aff2, int aff2_gn,
+             const bf16* __restrict__ res, const bf16* __restrict__ d,
              const bf16* __restrict__ mask, bf16* __restrict__ out, int C, int B, int HW, int ch,
-             int gn, int relu) {
+             int relu) {
   pdl_wait();
   pdl_trigger();
   const int V = ch / 8;
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (int64_t)C * B * HW * V) return;
-  const int v = (int)(i % V);
-  const int64_t pix = i / V;
-  const int64_t cb = pix / HW;
-  const int c = (int)(cb / B), b = (int)(cb % B);
-  const int cpg = ch / 32;
-  const int64_t o = pix * ch + v * 8;
-  float y[8];
-  unpack8(*reinterpret_cast<const uint4*>(t.y + o), y);
-  float r[8];
-  auto stats = [&](const NormTerm& q, int chn, float& mu, float& rs) {
-    const int64_t set = gn ? ((int64_t)c * B + b) * 32 + chn / cpg : (int64_t)c * ch + chn;
-    mu = q.mean[set];
-    rs = q.rstd[set];
-  };
+  const int L = kThreads / V;
+  const int chunks = (HW + kApplyPixels - 1) / kApplyPixels;
+  const int64_t cb = blockIdx.x / chunks;
+  const int p0 = (int)(blockIdx.x % chunks) * kApplyPixels;
+  const int p1 = p0 + kApplyPixels < HW ? p0 + kApplyPixels : HW;
+  const int c = (int)(cb / B);
+  const int v = threadIdx.x % V, l = threadIdx.x / V;
+  if (l >= L) return;
+  const int64_t arow = (aff_gn ? cb : (int64_t)c) * ch + v * 8;
   if (!BWD) {
-    if (res) {
-      unpack8(*reinterpret_cast<const uint4*>(res + o), r);
-    } else if (t2.y) {
-      float y2[8];
-      unpack8(*reinterpret_cast<const uint4*>(t2.y + o), y2);
+    float sc[8], sh[8], sc2[8], sh2[8];
+    const float4* a4 = reinterpret_cast<const float4*>(reinterpret_cast<const float2*>(aff) + arow);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float4 q = a4[k];
+      sc[2 * k] = q.x; sh[2 * k] = q.y; sc[2 * k + 1] = q.z; sh[2 * k + 1] = q.w;
+    }
+    if (y2) {
+      const float4* b4 =
+          reinterpret_cast<const float4*>(aff2 + (aff2_gn ? cb : (int64_t)c) * ch + v * 8);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float4 q = b4[k];
+        sc2[2 * k] = q.x; sh2[2 * k] = q.y; sc2[2 * k + 1] = q.z; sh2[2 * k + 1] = q.w;
+      }
+    }
+    for (int p = p0 + l; p < p1; p += L) {
+      const int64_t o = (cb * HW + p) * ch + v * 8;
+      float yy[8], r[8] = {0, 0, 0, 0, 0, 0, 0, 0}, o8[8];
+      unpack8(*reinterpret_cast<const uint4*>(y + o), yy);
+      if (res) {
+        unpack8(*reinterpret_cast<const uint4*>(res + o), r);
+      } else if (y2) {
+        float z[8];
+        unpack8(*reinterpret_cast<const uint4*>(y2 + o), z);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) r[k] = fmaf(z[k], sc2[k], sh2[k]);
+      }
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
-        const int chn = v * 8 + k;
-        float mu, rs;
-        stats(t2, chn, mu, rs);
-        r[k] = fmaf(t2.gamma[(int64_t)c * t2.g_rs + chn], (y2[k] - mu) * rs,
-                    t2.beta[(int64_t)c * t2.g_rs + chn]);
+        const float x = fmaf(yy[k], sc[k], sh[k]) + r[k];
+        o8[k] = relu ? (x > 0.f ? x : 0.f) : x;
       }
-    } else {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) r[k] = 0.f;
+      *reinterpret_cast<uint4*>(out + o) = pack8(o8);
     }
-    float o8[8];
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const int chn = v * 8 + k;
-      float mu, rs;
-      stats(t, chn, mu, rs);
-      float x = fmaf(t.gamma[(int64_t)c * t.g_rs + chn], (y[k] - mu) * rs,
-                     t.beta[(int64_t)c * t.g_rs + chn]) + r[k];
-      o8[k] = relu ? (x > 0.f ? x : 0.f) : x;
-    }
-    *reinterpret_cast<uint4*>(out + o) = pack8(o8);
   } else {
-    float dz[8];
-    unpack8(*reinterpret_cast<const uint4*>(d + o), dz);
-    if (mask) {
-      float m[8];
-      unpack8(*reinterpret_cast<const uint4*>(mask + o), m);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) dz[k] = m[k] > 0.f ? dz[k] : 0.f;
-    }
-    float o8[8];
+    float k1[8], k2[8], k3[8];
+    const float4* k4 = reinterpret_cast<const float4*>(aff) + arow;
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-      const int chn = v * 8 + k;
-      float rs, mu;
-      stats(t, chn, mu, rs);
-      // backward: t.mean / t.rstd are the forward stats, t2.mean / t2.rstd
-      // carry m1 / m2 of the same sets
-      float m1, m2;
-      stats(t2, chn, m1, m2);
-      const float xh = (y[k] - mu) * rs;
-      o8[k] = rs * (dz[k] * t.gamma[(int64_t)c * t.g_rs + chn] - m1 - xh * m2);
+      const float4 q = k4[k];
+      k1[k] = q.x; k2[k] = q.y; k3[k] = q.z;
     }
-    *reinterpret_cast<uint4*>(out + o) = pack8(o8);
+    for (int p = p0 + l; p < p1; p += L) {
+      const int64_t o = (cb * HW + p) * ch + v * 8;
+      float yy[8], dz[8], o8[8];
+      unpack8(*reinterpret_cast<const uint4*>(y + o), yy);
+      unpack8(*reinterpret_cast<const uint4*>(d + o), dz);
+      if (mask) {
+        float m[8];
+        unpack8(*reinterpret_cast<const uint4*>(mask + o), m);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) dz[k] = m[k] > 0.f ? dz[k] : 0.f;
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) o8[k] = fmaf(k1[k], dz[k], fmaf(k2[k], yy[k], k3[k]));
+      *reinterpret_cast<uint4*>(out + o) = pack8(o8);
+    }
   }
 }
 
@@ -328,47 +377,42 @@ cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16
                   rstd, dz_out, sums, B, HW, ch, gn);
 }
 
-cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, float* mean, float* rstd,
-                                     float* run, int64_t run_rs, int C, int B, int HW, int ch,
-                                     int gn) {
-  const int sets = gn ? B * 32 : ch;
-  return launch_k(k_norm_finalize_fwd, nblk((int64_t)C * sets, 128), 128, 0, s, sums, mean, rstd,
-                  run, run_rs, C, B, HW, ch, gn);
+cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const float* gamma,
+                                     const float* beta, int64_t g_rs, float* mean, float* rstd,
+                                     float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
+                                     int ch, int gn) {
+  const int64_t threads = gn ? (int64_t)C * B * 32 : (int64_t)C * ch * 32;
+  return launch_k(k_norm_finalize_fwd, nblk(threads, 256), 256, 0, s, sums, gamma, beta, g_rs,
+                  mean, rstd, ss, run, run_rs, C, B, HW, ch, gn);
 }
 
 cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,
-                                     int64_t g_rs, float* m1, float* m2, float* dgamma,
-                                     float* dbeta, int64_t d_rs, int C, int B, int HW, int ch,
-                                     int gn) {
-  const int sets = gn ? B * 32 : ch;
-  const int64_t n = (int64_t)C * (sets > ch ? sets : ch);
-  return launch_k(k_norm_finalize_bwd, nblk(n, 128), 128, 0, s, sums, gamma, g_rs, m1, m2,
-                  dgamma, dbeta, d_rs, C, B, HW, ch, gn);
+                                     int64_t g_rs, const float* mean, const float* rstd,
+                                     float4* kk, float* dgamma, float* dbeta, int64_t d_rs, int C,
+                                     int B, int HW, int ch, int gn) {
+  const int64_t threads = (int64_t)C * ch * 32 + (gn ? (int64_t)C * B * 32 : 0);
+  return launch_k(k_norm_finalize_bwd, nblk(threads, 256), 256, 0, s, sums, gamma, g_rs, mean,
+                  rstd, kk, dgamma, dbeta, d_rs, C, B, HW, ch, gn);
 }
 
-cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float* mean,
-                                  const float* rstd, const float* gamma, const float* beta,
-                                  int64_t g_rs, const bf16* res, const bf16* y2,
-                                  const float* mean2, const float* rstd2, const float* gamma2,
-                                  const float* beta2, bf16* out, int C, int B, int HW, int ch,
-                                  int gn, int relu) {
-  const NormTerm t{y, mean, rstd, gamma, beta, g_rs};
-  const NormTerm t2{y2, mean2, rstd2, gamma2, beta2, g_rs};
-  const int64_t n = (int64_t)C * B * HW * (ch / 8);
-  return launch_k(k_norm_apply<false>, nblk(n, kThreads), kThreads, 0, s, t, t2, res,
-                  (const bf16*)nullptr, (const bf16*)nullptr, out, C, B, HW, ch, gn, relu);
+cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float2* ss, int gn,
+                                  const bf16* res, const bf16* y2, const float2* ss2, int gn2,
+                                  bf16* out, int C, int B, int HW, int ch, int relu) {
+  if (ch % 8 || ch / 8 > kThreads) return cudaErrorInvalidValue;
+  const int64_t n = (int64_t)C * B * ((HW + kApplyPixels - 1) / kApplyPixels);
+  return launch_k(k_norm_apply<false>, (unsigned)n, kThreads, 0, s, y, (const void*)ss, gn,
+                  y2, ss2, gn2, res, (const bf16*)nullptr, (const bf16*)nullptr, out, C, B, HW,
+                  ch, relu);
 }
 
-cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float* mean,
-                                  const float* rstd, const float* gamma, int64_t g_rs,
-                                  const float* m1, const float* m2, const bf16* d,
-                                  const bf16* mask, bf16* out, int C, int B, int HW, int ch,
-                                  int gn) {
-  const NormTerm t{y, mean, rstd, gamma, nullptr, g_rs};
-  const NormTerm t2{nullptr, m1, m2, nullptr, nullptr, g_rs};
-  const int64_t n = (int64_t)C * B * HW * (ch / 8);
-  return launch_k(k_norm_apply<true>, nblk(n, kThreads), kThreads, 0, s, t, t2,
-                  (const bf16*)nullptr, d, mask, out, C, B, HW, ch, gn, 0);
+cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* kk, int gn,
+                                  const bf16* d, const bf16* mask, bf16* out, int C, int B, int HW,
+                                  int ch) {
+  if (ch % 8 || ch / 8 > kThreads) return cudaErrorInvalidValue;
+  const int64_t n = (int64_t)C * B * ((HW + kApplyPixels - 1) / kApplyPixels);
+  return launch_k(k_norm_apply<true>, (unsigned)n, kThreads, 0, s, y, (const void*)kk, gn,
+                  (const bf16*)nullptr, (const float2*)nullptr, 0, (const bf16*)nullptr, d, mask,
+                  out, C, B, HW, ch, 0);
 }
 
 cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch) {

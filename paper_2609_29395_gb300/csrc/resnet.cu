@@ -51,6 +51,7 @@ struct RnNorm {
   int64_t off_g, off_b, s_off;      // affine offsets in the blob; BatchNorm state offset
   float* mean;                      // [C][sets]
   float* rstd;
+  float2* ss;                       // [C][B or 1][ch] forward affine form
 };
 
 struct RnBlock {
@@ -68,7 +69,8 @@ struct RnState {
   bf16* h;                          // pooled features [C][B][512]
   bf16 *gin[2], *cutg;              // block gradients (ping-pong) and the cut gradient
   bf16 *dz, *dy, *dys, *dt;
-  float *sums, *m1, *m2;
+  float* sums;
+  float4* kk;                       // backward affine form of the norm being differentiated
   float* bn;                        // [C][S_pad] running mean / var per BatchNorm
   int64_t S, S_pad;
   int64_t fcw, fcb, p_client, p_total;
@@ -240,12 +242,11 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
   RN_ACT(r.gin[0], big); RN_ACT(r.gin[1], big); RN_ACT(r.cutg, big);
   RN_ACT(r.dz, big); RN_ACT(r.dy, big); RN_ACT(r.dys, big); RN_ACT(r.dt, big);
 #undef RN_ACT
-  int64_t max_sets = 0;
   auto stats = [&](RnNorm& n) -> gcpsl_status {
     const int64_t sets = sets_of(n, B);
-    max_sets = std::max(max_sets, sets);
     DALLOC(n.mean, sizeof(float) * (size_t)(C * sets));
     DALLOC(n.rstd, sizeof(float) * (size_t)(C * sets));
+    DALLOC(n.ss, sizeof(float2) * (size_t)C * (n.gn ? B : 1) * n.ch);
     return GCPSL_OK;
   };
   if ((st = stats(r.stem_n)) != GCPSL_OK) return st;
@@ -254,8 +255,7 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
     if ((st = stats(b.n2)) != GCPSL_OK) return st;
     if (b.sc && (st = stats(b.ns)) != GCPSL_OK) return st;
   }
-  DALLOC(r.m1, sizeof(float) * (size_t)(C * max_sets));
-  DALLOC(r.m2, sizeof(float) * (size_t)(C * max_sets));
+  DALLOC(r.kk, sizeof(float4) * (size_t)C * B * 512);
   DALLOC(r.sums, sizeof(float) * (size_t)C * B * 512 * 2);
   // BatchNorm running statistics: mean 0, variance 1
   DALLOC(r.bn, sizeof(float) * (size_t)(C * r.S_pad));
@@ -398,12 +398,14 @@ gcpsl_status conv_wgrad(gcpsl_ctx* c, const RnConv& v) {
 
 gcpsl_status norm_stats(gcpsl_ctx* c, const RnNorm& n, const bf16* y) {
   RnState& r = *c->rn;
+  const float* th = c->d_theta;
   LAUNCH("rn_norm_sums", launch_norm_sums(c->stream, false, y, nullptr, nullptr, nullptr,
                                           nullptr, nullptr, r.sums, c->C, c->B, n.hw, n.ch,
                                           n.gn));
-  LAUNCH("rn_norm_finalize", launch_norm_finalize_fwd(c->stream, r.sums, n.mean, n.rstd,
-                                                      n.gn ? nullptr : r.bn + n.s_off, r.S_pad,
-                                                      c->C, c->B, n.hw, n.ch, n.gn));
+  LAUNCH("rn_norm_finalize",
+         launch_norm_finalize_fwd(c->stream, r.sums, th + n.off_g, th + n.off_b, c->P_pad, n.mean,
+                                  n.rstd, n.ss, n.gn ? nullptr : r.bn + n.s_off, r.S_pad, c->C,
+                                  c->B, n.hw, n.ch, n.gn));
   return GCPSL_OK;
 }
 
@@ -416,13 +418,12 @@ gcpsl_status norm_bwd(gcpsl_ctx* c, const RnNorm& n, const bf16* y, const bf16* 
   LAUNCH("rn_norm_bwd_sums", launch_norm_sums(c->stream, true, y, d, mask, n.mean, n.rstd,
                                               dz_out, r.sums, c->C, c->B, n.hw, n.ch, n.gn));
   LAUNCH("rn_norm_bwd_finalize",
-         launch_norm_finalize_bwd(c->stream, r.sums, th + n.off_g, c->P_pad, r.m1, r.m2,
+         launch_norm_finalize_bwd(c->stream, r.sums, th + n.off_g, c->P_pad, n.mean, n.rstd, r.kk,
                                   c->d_grad + n.off_g, c->d_grad + n.off_b, c->P_pad, c->C, c->B,
                                   n.hw, n.ch, n.gn));
   LAUNCH("rn_norm_bwd_apply",
-         launch_norm_apply_bwd(c->stream, y, n.mean, n.rstd, th + n.off_g, c->P_pad, r.m1, r.m2,
-                               dz_out ? dz_out : d, dz_out ? nullptr : mask, dy, c->C, c->B, n.hw,
-                               n.ch, n.gn));
+         launch_norm_apply_bwd(c->stream, y, r.kk, n.gn, dz_out ? dz_out : d,
+                               dz_out ? nullptr : mask, dy, c->C, c->B, n.hw, n.ch));
   return GCPSL_OK;
 }
 
@@ -441,17 +442,13 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
   // ---- forward ----
   RN(conv_fwd(c, r.stem, true));
   RN(norm_stats(c, r.stem_n, r.ystem));
-  LAUNCH("rn_norm_apply",
-         launch_norm_apply_fwd(s, r.ystem, r.stem_n.mean, r.stem_n.rstd, th + r.stem_n.off_g,
-                               th + r.stem_n.off_b, P, nullptr, nullptr, nullptr, nullptr,
-                               nullptr, nullptr, r.astem, C, B, 1024, 64, 1, 1));
+  LAUNCH("rn_norm_apply", launch_norm_apply_fwd(s, r.ystem, r.stem_n.ss, 1, nullptr, nullptr,
+                                                nullptr, 0, r.astem, C, B, 1024, 64, 1));
   for (auto& b : r.blk) {
     RN(conv_fwd(c, b.c1, false));
     RN(norm_stats(c, b.n1, b.y1));
-    LAUNCH("rn_norm_apply",
-           launch_norm_apply_fwd(s, b.y1, b.n1.mean, b.n1.rstd, th + b.n1.off_g, th + b.n1.off_b,
-                                 P, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, b.a1, C,
-                                 B, b.n1.hw, b.n1.ch, b.n1.gn, 1));
+    LAUNCH("rn_norm_apply", launch_norm_apply_fwd(s, b.y1, b.n1.ss, b.n1.gn, nullptr, nullptr,
+                                                  nullptr, 0, b.a1, C, B, b.n1.hw, b.n1.ch, 1));
     RN(conv_fwd(c, b.c2, false));
     RN(norm_stats(c, b.n2, b.y2));
     if (b.sc) {
@@ -459,12 +456,9 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
       RN(norm_stats(c, b.ns, b.ys));
     }
     LAUNCH("rn_norm_apply",
-           launch_norm_apply_fwd(s, b.y2, b.n2.mean, b.n2.rstd, th + b.n2.off_g, th + b.n2.off_b,
-                                 P, b.sc ? nullptr : b.c1.x, b.sc ? b.ys : nullptr,
-                                 b.sc ? b.ns.mean : nullptr, b.sc ? b.ns.rstd : nullptr,
-                                 b.sc ? th + b.ns.off_g : nullptr,
-                                 b.sc ? th + b.ns.off_b : nullptr, b.out, C, B, b.n2.hw, b.n2.ch,
-                                 b.n2.gn, 1));
+           launch_norm_apply_fwd(s, b.y2, b.n2.ss, b.n2.gn, b.sc ? nullptr : b.c1.x,
+                                 b.sc ? b.ys : nullptr, b.sc ? b.ns.ss : nullptr, b.ns.gn, b.out, C,
+                                 B, b.n2.hw, b.n2.ch, 1));
   }
   LAUNCH("rn_avgpool", launch_avgpool(s, r.blk[7].out, r.h, C * B, 16, 512));
   LAUNCH("fc_fwd_ce", launch_fc_fwd_ce<bf16>(s, r.h, c->d_shadow + r.fcw, P, th + r.fcb, P,
