@@ -141,3 +141,50 @@ def test_resnet18_grouped_equals_serialized_and_graph_equals_eager():
         assert (one.bn_state(0) == both.bn_state(m)).all()
         assert (eager.all_params(m) == both.all_params(m)).all()
         one.close()
+
+
+def test_resnet18_c8_full_size_sampled_cluster():
+    """The 200,000-image, K=1024, C=8, B=128 workload in the benchmarked
+    launch configuration: the GPU takes its first round with all eight
+    clusters; cluster 5 is re-run alone by the oracle (one-cluster context,
+    same cluster id, so the same Philox stream) replaying that cluster's
+    ReLU decisions, and compared slice by slice."""
+    from paper_2609_29395_gb300 import configs
+    w = configs.WORKLOADS["resnet18_c8"]
+    ds, assign, params = configs.build_inputs(w)
+    gpu = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
+                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=True)
+    bn0 = gpu.bn_state(0)
+    loss, active = gpu.step(stats=True)
+    gi, gc = gpu.sample()
+    assert (gc.sum(1) == w.B).all()
+    masks = gpu.relu_masks()
+    cut_act = gpu.cut(pkg.binding.GCPSL_CUT_ACT)
+    cut_grad = gpu.cut(pkg.binding.GCPSL_CUT_GRAD)
+    m = 5
+    sub = np.where(assign == m, 0, -1).astype(np.int32)
+    orc = oracle.Oracle(w.arch, w.num_clients, 1, sub, w.B, w.F, 4, ds.images, ds.labels,
+                        ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=True,
+                        cluster_base=m)
+    orc.set_bn_state(0, bn0.astype(np.float64))
+    oracle.set_relu_tol(RELU_TOL)
+    orc.set_relu_masks(masks[m:m + 1])
+    orc.step()
+    rec = orc.relu_masks()
+    used, own = rec & 1, (rec >> 1) & 1
+    deep = 64 * 1024 + 2 * (2 * 64 * 1024)
+    amb = np.concatenate([(rec[:, :, :deep] >> 2) & 1, (rec[:, :, deep:] >> 3) & 1], axis=2)
+    assert not ((amb == 0) & (used != own)).any()
+    assert amb.mean() < 0.1
+    oi, oc = orc.sample()
+    assert (gi[m] == oi[0]).all() and (gc[m] == oc[0]).all()
+    ol, oa = orc.stats()
+    assert active[m] == oa[0]
+    assert abs(loss[m] - ol[0]) < LOSS_ABS, (loss[m], ol[0])
+    assert rel_l2(cut_act[m], orc.cut(0).reshape(cut_act[m].shape)) < REL_L2
+    assert rel_l2(cut_grad[m], orc.cut(1).reshape(cut_grad[m].shape)) < REL_L2
+    gp, op = gpu.all_params(m), orc.all_params(0)
+    assert rel_l2(gp, op) < REL_L2
+    assert rel_l2(gp - params, op - params) < REL_L2, "update"
+    assert rel_l2(gpu.bn_state(m), orc.bn_state(0)) < REL_L2
+    gpu.close()
