@@ -11,6 +11,7 @@ This is also the small, fixed program that kernel profilers are pointed at:
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import time
 
 import numpy as np
@@ -23,8 +24,16 @@ def main() -> int:
     ap.add_argument("--workload", default="splitcnn_c4", choices=sorted(configs.WORKLOADS))
     ap.add_argument("--rounds", type=int, default=5)
     ap.add_argument("--eager", action="store_true", help="launch kernels one by one, no graphs")
+    ap.add_argument("--images", type=int, default=0,
+                    help="dataset size (default: the workload's); the round shapes stay")
+    ap.add_argument("--clusters", type=int, default=0,
+                    help="number of clusters C (default: the workload's)")
     args = ap.parse_args()
     w = configs.WORKLOADS[args.workload]
+    if args.images:
+        w = dataclasses.replace(w, n=args.images)
+    if args.clusters:
+        w = dataclasses.replace(w, num_clusters=args.clusters)
     ds, assign, params = configs.build_inputs(w)
     ctx = Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
                   ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=w.bf16)

@@ -205,7 +205,13 @@ struct WgradTcArgs {
   int taps = 9;         // 9 (3x3) or 1 (1x1)
   int bias = 1;         // also the bias gradient (a block of ones)
   int stride = 1, pad = 1;  // x pixel of output pixel p and tap (kh, kw): p*stride + k - pad
+  // non-null: the splits (<= kWgradClusterMax) run as one thread-block
+  // cluster per tile and write the summed gradient to out[c * out_rs + ...]
+  // (same layout as a partial; 16-byte aligned); `partial` is then unused
+  float* out = nullptr;
+  int64_t out_rs = 0;
 };
+constexpr int kWgradClusterMax = 8;   // portable cluster size
 // elem_strides (nullable): traversal stride per dimension; a box then
 // loads ceil(box[i] / elem_strides[i]) elements along dimension i
 bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
@@ -218,6 +224,14 @@ cudaError_t launch_conv_tc(cudaStream_t s, const CUtensorMap& a, const CUtensorM
                            const CUtensorMap* a2 = nullptr, const CUtensorMap* b2 = nullptr);
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C);
+// 3x3 stride-1 convolution (forward, or data gradient with the dgrad3 tap
+// table) on 8 x 16-pixel M tiles of one image, weights resident in shared
+// memory: `a` maps the activation operand with a box of BKC channels x 10
+// x 18 pixels, `b` the weights as for launch_conv_tc with an N box of
+// min(bn, 64).  p.bw = 8, p.hb = 16, p.bb = 1.
+bool halo_supported(int H, int W, int kch, int bn, int bkc, int epi);
+cudaError_t launch_conv_halo(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                             const ConvTcArgs& p, int bn, int bkc, int epi, int C);
 // input layer: b = packed weights w0p[C][cout][32] (k = tap * 3 + ci < 27, else 0)
 cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs, int cout, int C);
 // input-layer weight and bias gradient partials from its im2col (cout 32 or

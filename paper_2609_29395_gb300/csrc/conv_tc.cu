@@ -22,8 +22,10 @@
 //  k_wgrad_tc: dW[co][tap][ci] = sum_p g[p][co] x[p + shift(tap)][ci]
 //    M = co, N = ci, K = pixels.  Both operands are MN-major tiles (pixels are
 //    rows, channels contiguous), loaded as 64-pixel boxes.  The pixel range is
-//    split across CTAs; each writes an fp32 partial tile and k_wgrad_reduce
-//    sums the partials in split order (deterministic).
+//    split across CTAs.  Up to kWgradClusterMax splits form one thread-block
+//    cluster and sum their fp32 tiles through distributed shared memory in
+//    rank order; with more splits each writes an fp32 partial tile and
+//    k_wgrad_reduce sums the partials in split order (deterministic).
 //
 // Warp roles (192 threads): warp 0 issues TMA, warp 1 allocates TMEM and
 // issues MMAs, warps 2-5 run the epilogue (warp w reads TMEM lanes
@@ -240,6 +242,149 @@ __device__ __forceinline__ void conv_epilogue_drain(uint32_t trow, int r, int n0
   }
 }
 
+// 32 lanes x 32 consecutive columns, waited for in one go (the values pass
+// through the wait so that no use is scheduled before it)
+__device__ __forceinline__ void tmem_ld32_wait(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Epilogue of the non-pooling kinds over NC columns (a multiple of 16), in
+// groups of G = min(32, NC) columns: the operands the epilogue reads (res,
+// act, codes) of the first group are loaded before the accumulator is
+// waited for, and those of the next group while the current one is
+// processed; each group's TMEM columns come in one load and one wait.
+// Results are those of conv_epilogue_drain.  Returns false if the wait for
+// the accumulator gave up.
+template <int NC, int EPI>
+__device__ __forceinline__ bool conv_epilogue_stream(uint64_t* tfull, uint32_t parity,
+                                                     uint32_t trow, int r, int n0, int b0, int h0,
+                                                     int w0, int c, const ConvTcArgs& p) {
+  static_assert(EPI != EPI_POOL, "pooling epilogue: conv_epilogue_drain");
+  constexpr int G = NC < 32 ? NC : 32;
+  constexpr int NA = G / 8;                        // uint4 of bf16 aux per group
+  const int W = p.W, H = p.H, bw = p.bw;
+  const int ww = r % bw, hh = (r / bw) % p.hb, bb = r / (bw * p.hb);
+  const bool valid = b0 + bb < p.B;
+  const int64_t img = (int64_t)c * p.B + b0 + bb;
+  const int oH = p.out_H ? p.out_H : H, oW = p.out_W ? p.out_W : W;
+  const int64_t o = ((img * oH + (h0 + hh) * p.osy + p.ooy) * oW + (w0 + ww) * p.osx + p.oox) *
+                        p.n_total + n0;
+  const float* bias = EPI == EPI_RELU ? p.bias + (int64_t)c * p.bias_rs + n0 : nullptr;
+  const bf16* aux_src = EPI == EPI_ADD ? p.res : EPI == EPI_DRELU ? p.act : nullptr;
+  uint4 aux[NA];
+  uint4 cd[(G + 15) / 16];
+  auto load_aux = [&](int g0) {
+    if (!valid) return;
+    if (aux_src) {
+#pragma unroll
+      for (int i = 0; i < NA; ++i) aux[i] = *reinterpret_cast<const uint4*>(aux_src + o + g0 + 8 * i);
+    }
+    if (EPI == EPI_DPOOL) {
+#pragma unroll
+      for (int i = 0; i < (G + 15) / 16; ++i)
+        cd[i] = *reinterpret_cast<const uint4*>(p.code + o + g0 + 16 * i);
+    }
+  };
+  load_aux(0);
+  if (!__all_sync(0xffffffffu, mbar_wait(tfull, parity))) return false;
+  tc_fence_after();
+#pragma unroll 1
+  for (int g0 = 0; g0 < NC; g0 += G) {
+    float v[32];
+    if (G == 32) {
+      tmem_ld32_wait(trow + g0, v);
+    } else {
+      float h[16];
+      tmem_ld16(trow + g0, h);
+      tmem_wait_regs(h);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = h[i];
+    }
+    uint4 am[NA];
+    uint4 cw[(G + 15) / 16];
+#pragma unroll
+    for (int i = 0; i < NA; ++i) am[i] = aux[i];
+#pragma unroll
+    for (int i = 0; i < (G + 15) / 16; ++i) cw[i] = cd[i];
+    if (g0 + G < NC) load_aux(g0 + G);
+    if (!valid) continue;
+    uint32_t hw[G / 2];
+#pragma unroll
+    for (int i = 0; i < G / 2; ++i) {
+      float x0 = v[2 * i], x1 = v[2 * i + 1];
+      if (EPI == EPI_RELU) {
+        x0 += bias[g0 + 2 * i];
+        x1 += bias[g0 + 2 * i + 1];
+        x0 = x0 > 0.f ? x0 : 0.f;
+        x1 = x1 > 0.f ? x1 : 0.f;
+      }
+      if (EPI == EPI_ADD) {
+        const uint32_t rr = (&am[0].x)[i];
+        x0 += __uint_as_float(rr << 16);
+        x1 += __uint_as_float(rr & 0xffff0000u);
+      }
+      hw[i] = pack_bf16x2(x0, x1);
+    }
+    if (EPI != EPI_DPOOL && EPI != EPI_DRELU) {
+      uint4* dst = reinterpret_cast<uint4*>(p.out + o + g0);
+#pragma unroll
+      for (int i = 0; i < G / 8; ++i)
+        dst[i] = make_uint4(hw[4 * i], hw[4 * i + 1], hw[4 * i + 2], hw[4 * i + 3]);
+      continue;
+    }
+    if (p.out) {
+      uint4* dst = reinterpret_cast<uint4*>(p.out + o + g0);
+#pragma unroll
+      for (int i = 0; i < G / 8; ++i)
+        dst[i] = make_uint4(hw[4 * i], hw[4 * i + 1], hw[4 * i + 2], hw[4 * i + 3]);
+    }
+    if (EPI == EPI_DRELU) {
+      // act > 0 <=> its bf16 bits are > 0 as a signed 16-bit integer
+      uint32_t gw[G / 2];
+#pragma unroll
+      for (int i = 0; i < G / 2; ++i) gw[i] = hw[i] & __vcmpgts2((&am[0].x)[i], 0u);
+      uint4* dst = reinterpret_cast<uint4*>(p.gout + o + g0);
+#pragma unroll
+      for (int i = 0; i < G / 8; ++i)
+        dst[i] = make_uint4(gw[4 * i], gw[4 * i + 1], gw[4 * i + 2], gw[4 * i + 3]);
+    } else {
+      // byte k of the codes selects the window position that gets channel k
+      const int y = h0 + hh, x = w0 + ww;
+#pragma unroll
+      for (int qd = 0; qd < 4; ++qd) {
+        const uint32_t want = (uint32_t)(4 | qd) * 0x01010101u;
+        uint32_t gw[G / 2];
+#pragma unroll
+        for (int j = 0; j < G / 4; ++j) {
+          const uint32_t m = __vcmpeq4((&cw[0].x)[j] & 0x07070707u, want);
+          gw[2 * j] = hw[2 * j] & __byte_perm(m, 0, 0x1100);
+          gw[2 * j + 1] = hw[2 * j + 1] & __byte_perm(m, 0, 0x3322);
+        }
+        const int64_t go =
+            ((img * (2 * H) + 2 * y + (qd >> 1)) * (2 * W) + 2 * x + (qd & 1)) * p.n_total + n0 + g0;
+        uint4* dst = reinterpret_cast<uint4*>(p.gout + go);
+#pragma unroll
+        for (int i = 0; i < G / 8; ++i)
+          dst[i] = make_uint4(gw[4 * i], gw[4 * i + 1], gw[4 * i + 2], gw[4 * i + 3]);
+      }
+    }
+  }
+  return true;
+}
+
 template <int BN, int BKC, int EPI>
 struct ConvCfg {
   static constexpr int A_BYTES = BM * BKC * 2;
@@ -389,19 +534,242 @@ k_conv_tc(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtens
     int tl = 0;
     for (int t = blockIdx.x; t < items; t += gridDim.x, ++tl) {
       const int buf = tl & 1;
-      // warp-uniform decision: the epilogue shuffles need the whole warp
-      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
-        if (lane == 0) atomicOr(p.err, 4);
-        break;
-      }
-      tc_fence_after();
       const int c = t / (tiles_m * tiles_n), rr = t % (tiles_m * tiles_n);
       const int mt = rr / tiles_n, n0 = (rr % tiles_n) * BN;
       int b0, h0, w0;
       tile_origin(mt, p, b0, h0, w0);
       const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
-      conv_epilogue_drain<BN, EPI>(trow, r, n0, b0, h0, w0, c, p,
-                                   reinterpret_cast<float*>(sm + Cfg::PIPE) + q * 32 * kXsRow);
+      if (EPI == EPI_POOL) {
+        // warp-uniform decision: the epilogue shuffles need the whole warp
+        if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
+          if (lane == 0) atomicOr(p.err, 4);
+          break;
+        }
+        tc_fence_after();
+        conv_epilogue_drain<BN, EPI>(trow, r, n0, b0, h0, w0, c, p,
+                                     reinterpret_cast<float*>(sm + Cfg::PIPE) + q * 32 * kXsRow);
+      } else if (!conv_epilogue_stream<BN, EPI == EPI_POOL ? EPI_STORE : EPI>(
+                     &tfull[buf], (tl >> 1) & 1, trow, r, n0, b0, h0, w0, c, p)) {
+        if (lane == 0) atomicOr(p.err, 4);
+        break;
+      }
+      tc_fence_before();
+      mbar_arrive(&tempty[buf]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, 2 * Cfg::TCOLS);
+}
+
+// ---------------------------------------------------------------------------
+// Halo-tiled 3x3 stride-1 convolution (forward or data gradient) with the
+// weights resident in shared memory.
+//
+// An M tile is 8 columns x 16 rows of one image.  Per K block of BKC channels
+// the TMA warp loads ONE box of (8+2) x (16+2) pixels around it (zero fill
+// outside the image is the padding), and the nine taps read it in place: the
+// tap with shift (sy, sx) is the K-major operand that starts (sy+1)*10 +
+// (sx+1) pixel rows into the box, its 16 groups of 8 pixels 10 rows apart.
+// (The operand swizzle is a function of the shared-memory address, so a
+// start that is not aligned to the swizzle repeat reads the TMA-written
+// rows correctly.)  The weights of the current (replica, N tile) -- 9 taps x
+// K blocks, loaded once -- stay in shared memory while the CTA works through
+// a contiguous range of items (replica, N tile, M tile; M fastest), and are
+// reloaded only when the replica or N tile changes.  Accumulators, epilogue
+// and TMEM double buffering as in k_conv_tc.
+// ---------------------------------------------------------------------------
+constexpr int kHaloW = 10, kHaloH = 18, kHaloMaxStages = 8;
+// warps: 0 TMA, 1 MMA, 2..9 epilogue (two per TMEM lane quarter, each
+// draining half of the N columns)
+constexpr int kHaloThreads = 320, kHaloEpiThreads = 256;
+template <int BN, int BKC, int EPI>
+struct HaloCfg {
+  static constexpr int ROWB = BKC * 2;                        // bytes per pixel row
+  static constexpr int A_RAW = kHaloW * kHaloH * ROWB;        // bytes of one halo box
+  static constexpr int A_BYTES = (A_RAW + 1023) / 1024 * 1024;
+  static constexpr int B_TILE = BN * BKC * 2;                 // one (tap, K block) weight tile
+  static constexpr uint32_t TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static constexpr int XS = 2 * epi_scratch(EPI);            // eight epilogue warps
+  // dynamic shared memory at most: the opt-in maximum per CTA (227 KB) less
+  // 1 KB for the static barriers
+  static constexpr int SMEM_MAX = 232448 - 1024;
+};
+__host__ __device__ inline int halo_item_begin(int cta, int ctas, int items) {
+  return (int)((int64_t)items * cta / ctas);
+}
+
+template <int BN, int BKC, int EPI, int BMN>
+__global__ void __launch_bounds__(kHaloThreads, 1)
+k_conv_halo(const __grid_constant__ CUtensorMap tA, const __grid_constant__ CUtensorMap tB,
+            const ConvTcArgs p, int tiles_m, int tiles_n, int items, int S) {
+  using Cfg = HaloCfg<BN, BKC, EPI>;
+  extern __shared__ uint8_t smraw[];
+  uint8_t* sm = align1024(smraw);
+  const int kper = p.kch / BKC;
+  uint8_t* sB = sm;                                           // 9 * kper weight tiles
+  uint8_t* sA = sm + 9 * kper * Cfg::B_TILE;                  // S halo stages
+  float* xs = reinterpret_cast<float*>(sA + S * Cfg::A_BYTES);
+  __shared__ uint64_t full[kHaloMaxStages], empty[kHaloMaxStages], tfull[2], tempty[2];
+  __shared__ uint64_t wfull, wempty;
+  __shared__ uint32_t tbase;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t_begin = halo_item_begin(blockIdx.x, gridDim.x, items);
+  const int t_end = halo_item_begin(blockIdx.x + 1, gridDim.x, items);
+  const int per_c = tiles_m * tiles_n;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], kHaloEpiThreads);
+    }
+    mbar_init(&wfull, 1);
+    mbar_init(&wempty, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tA);
+    tma_prefetch_desc(&tB);
+  }
+  if (warp == 1) { tmem_alloc(&tbase, 2 * Cfg::TCOLS); tmem_relinquish(); }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tbase;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (elect_one()) {
+      int it = 0, wl = 0, prev = -1;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t) {
+        const int c = t / per_c, r = t % per_c;
+        const int nt = r / tiles_m, mt = r % tiles_m;
+        const int key = c * tiles_n + nt, n0 = nt * BN;
+        if (key != prev) {
+          // new (replica, N tile): its weights, once the MMAs on the old ones are done
+          if (wl > 0 && !mbar_wait(&wempty, (wl - 1) & 1)) { atomicOr(p.err, 1); break; }
+          mbar_arrive_expect_tx(&wfull, 9 * kper * Cfg::B_TILE);
+          for (int tap = 0; tap < 9; ++tap)
+            for (int kb = 0; kb < kper; ++kb) {
+              uint8_t* dst = sB + (tap * kper + kb) * Cfg::B_TILE;
+              if (!BMN) {
+                tma_load_4d(dst, &tB, &wfull, kb * BKC, p.tw[tap], n0, c);
+              } else {
+                constexpr int NBW = BN < 64 ? BN : 64;
+#pragma unroll
+                for (int j = 0; j < BN / NBW; ++j)
+                  tma_load_4d(dst + j * NBW * BKC * 2, &tB, &wfull, n0 + j * NBW, p.tw[tap],
+                              kb * BKC, c);
+              }
+            }
+          ++wl;
+          prev = key;
+        }
+        int b0, h0, w0;
+        tile_origin(mt, p, b0, h0, w0);
+        for (int kb = 0; kb < kper; ++kb, ++it) {
+          const int s = it % S;
+          if (it >= S && !mbar_wait(&empty[s], ((it / S) & 1) ^ 1)) {
+            atomicOr(p.err, 1);
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], Cfg::A_RAW);
+          tma_load_5d(sA + s * Cfg::A_BYTES, &tA, &full[s], kb * BKC, w0 - 1, h0 - 1, b0, c);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (elect_one()) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN, 0, BMN);
+      constexpr uint32_t swz = BKC == 64 ? SWZ_128 : SWZ_64;
+      constexpr uint32_t a_sbo = kHaloW * Cfg::ROWB;           // 8-pixel groups one row apart
+      constexpr int NBW = BN < 64 ? BN : 64;
+      constexpr uint32_t b_row = NBW * 2;
+      constexpr uint32_t b_swz = NBW == 64 ? SWZ_128 : SWZ_64;
+      // descriptors are built once; an operand at byte offset o from its base
+      // is the base descriptor plus o >> 4 (the start-address field)
+      uint32_t aoff[9];
+#pragma unroll
+      for (int tap = 0; tap < 9; ++tap)
+        aoff[tap] = (uint32_t)(((p.tdy[tap] + 1) * kHaloW + p.tdx[tap] + 1) * Cfg::ROWB) >> 4;
+      const uint64_t a_desc0 = smem_desc(smem_u32(sA), 16, a_sbo, swz);
+      const uint64_t b_desc0 = BMN ? smem_desc(smem_u32(sB), NBW * BKC * 2, 8 * b_row, b_swz)
+                                   : smem_desc(smem_u32(sB), 16, BKC * 2 * 8, swz);
+      constexpr uint32_t b_kstep = (BMN ? 16 * b_row : 32) >> 4;   // per K = 16 step
+      const uint32_t b_tapstep = (uint32_t)(kper * Cfg::B_TILE) >> 4;
+      int it = 0, tl = 0, wl = 0, prev = -1;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t, ++tl) {
+        const int c = t / per_c, nt = (t % per_c) / tiles_m;
+        const int key = c * tiles_n + nt;
+        if (key != prev) {
+          if (!mbar_wait(&wfull, wl & 1)) { atomicOr(p.err, 2); break; }
+          ++wl;
+          prev = key;
+        }
+        const int buf = tl & 1;
+        if (tl >= 2 && !mbar_wait(&tempty[buf], ((tl >> 1) & 1) ^ 1)) {
+          atomicOr(p.err, 2);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + buf * Cfg::TCOLS;
+        for (int kb = 0; kb < kper; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait(&full[s], (it / S) & 1)) {
+            atomicOr(p.err, 2);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t da = a_desc0 + (uint32_t)((s * Cfg::A_BYTES) >> 4);
+          const uint64_t db = b_desc0 + (uint32_t)((kb * Cfg::B_TILE) >> 4);
+#pragma unroll
+          for (int tap = 0; tap < 9; ++tap) {
+#pragma unroll
+            for (int k = 0; k < BKC / 16; ++k)
+              mma_f16(d, da + aoff[tap] + 2 * k, db + tap * b_tapstep + k * b_kstep, idesc,
+                      (kb | tap | k) != 0);
+          }
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&tfull[buf]);
+        // the last item on these weights: release them to the TMA warp
+        const int nx = t + 1;
+        const int nkey = nx < t_end ? (nx / per_c) * tiles_n + (nx % per_c) / tiles_m : -1;
+        if (nkey != key) mma_commit(&wempty);
+      }
+    }
+  } else {
+    // ---------------- epilogue: warps 2..9 ----------------
+    const int q = warp & 3;                      // TMEM lane quarter
+    const int half = (warp - 2) >> 2;            // columns [half * BN/2, (half + 1) * BN/2)
+    const int r = q * 32 + lane;
+    constexpr int NH = BN / 2;
+    int tl = 0;
+    for (int t = t_begin; t < t_end; ++t, ++tl) {
+      const int buf = tl & 1;
+      const int c = t / per_c, rr = t % per_c;
+      const int n0 = (rr / tiles_m) * BN, mt = rr % tiles_m;
+      int b0, h0, w0;
+      tile_origin(mt, p, b0, h0, w0);
+      const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16) + half * NH;
+      if (EPI == EPI_POOL) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
+          if (lane == 0) atomicOr(p.err, 4);
+          break;
+        }
+        tc_fence_after();
+        conv_epilogue_drain<NH, EPI>(trow, r, n0 + half * NH, b0, h0, w0, c, p,
+                                     xs + (warp - 2) * 32 * kXsRow);
+      } else if (!conv_epilogue_stream<NH, EPI == EPI_POOL ? EPI_STORE : EPI>(
+                     &tfull[buf], (tl >> 1) & 1, trow, r, n0 + half * NH, b0, h0, w0, c, p)) {
+        if (lane == 0) atomicOr(p.err, 4);
+        break;
+      }
       tc_fence_before();
       mbar_arrive(&tempty[buf]);
     }
@@ -456,6 +824,8 @@ struct WgCfg {
   static constexpr int S = S0 > 6 ? 6 : S0;
   static constexpr int SMEM = 1024 + S * STAGE;
   static constexpr uint32_t TCOLS = 256;
+  // the cluster reduction's fp32 tile reuses the operand ring
+  static_assert(MT * (TG * BN + 4) * 4 <= S * STAGE, "accumulator tile exceeds the ring");
 };
 
 template <int BN, int MT>
@@ -568,32 +938,54 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     const int q = warp & 3;
     // accumulator row of this thread's TMEM lane (M = 64: lanes 16..31 of
     // each quarter are unused)
-    const int co = co0 + (MT == 128 ? q * 32 + lane : q * 16 + lane);
+    const int row = MT == 128 ? q * 32 + lane : q * 16 + lane;
+    const int co = co0 + row;
     const bool mine = (MT == 128 || lane < 16) && co < p.cout;
     const bool ok = mbar_wait(&done, 0);
     if (!ok) atomicOr(p.err, 32);
     tc_fence_after();
     const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
-    float* part = p.partial + ((int64_t)c * p.splits + split) * per;
-    if (bias_grp && ci0 == 0) {
-      float v[16];
-      tmem_ld16(trow + ntaps * BN, v);
-      tmem_ld_wait();
-      if (mine) part[p.cout * p.taps * p.cin + co] = nkb ? v[0] : 0.f;
-    }
-    for (int tj = 0; tj < ntaps; ++tj) {
-      float* dst = part + (int64_t)co * p.taps * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
+    if (p.out) {
+      // cluster reduction: the accumulator goes to this CTA's shared memory
+      // (the operand ring is free once `done` has fired: every MMA, hence
+      // every TMA load, has completed), rows padded by 4 words
+      float* acc = reinterpret_cast<float*>(sm);
+      const int ld = nslots * BN + 4;
 #pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 16) {
+      for (int c0 = 0; c0 < nslots * BN; c0 += 16) {
         float v[16];
-        tmem_ld16(trow + tj * BN + c0, v);
+        tmem_ld16(trow + c0, v);
         tmem_ld_wait();
-        if (mine) {
-          float4* d4 = reinterpret_cast<float4*>(dst + c0);
+        if (MT == 128 || lane < 16) {
+          float4* d4 = reinterpret_cast<float4*>(acc + (int64_t)row * ld + c0);
 #pragma unroll
           for (int i = 0; i < 4; ++i)
             d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
                         : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+    } else {
+      float* part = p.partial + ((int64_t)c * p.splits + split) * per;
+      if (bias_grp && ci0 == 0) {
+        float v[16];
+        tmem_ld16(trow + ntaps * BN, v);
+        tmem_ld_wait();
+        if (mine) part[p.cout * p.taps * p.cin + co] = nkb ? v[0] : 0.f;
+      }
+      for (int tj = 0; tj < ntaps; ++tj) {
+        float* dst = part + (int64_t)co * p.taps * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 16) {
+          float v[16];
+          tmem_ld16(trow + tj * BN + c0, v);
+          tmem_ld_wait();
+          if (mine) {
+            float4* d4 = reinterpret_cast<float4*>(dst + c0);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
         }
       }
     }
@@ -601,6 +993,38 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
+  if (p.out) {
+    // The splits of this tile are the CTAs of one cluster (rank = split).
+    // Rank k sums the k-th 1/splits of the tile over every rank's shared
+    // memory, in rank order, and writes the gradient itself.
+    cluster_sync();
+    const int N = nslots * BN, ld = N + 4, upr = N / 4;
+    const int rows = p.cout - co0 < MT ? p.cout - co0 : MT;
+    const int U = rows * upr, S = p.splits, k = (int)cluster_rank();
+    const int ub = (int)((int64_t)U * k / S), ue = (int)((int64_t)U * (k + 1) / S);
+    const uint32_t base = smem_u32(sm);
+    float* out = p.out + (int64_t)c * p.out_rs;
+    for (int u = ub + (int)threadIdx.x; u < ue; u += blockDim.x) {
+      const int rw = u / upr, col = (u % upr) * 4;
+      const uint32_t off = base + (uint32_t)(rw * ld + col) * 4u;
+      // every rank's value in flight at once, then summed in rank order
+      float4 v[kWgradClusterMax];
+#pragma unroll
+      for (int j = 0; j < kWgradClusterMax; ++j)
+        if (j < S) v[j] = ld_peer_f4(peer_smem(off, (uint32_t)j));
+      float4 sum = v[0];
+#pragma unroll
+      for (int j = 1; j < kWgradClusterMax; ++j)
+        if (j < S) { sum.x += v[j].x; sum.y += v[j].y; sum.z += v[j].z; sum.w += v[j].w; }
+      const int slot = col / BN, ci = col % BN, co = co0 + rw;
+      if (slot < ntaps)
+        *reinterpret_cast<float4*>(out + (int64_t)co * p.taps * p.cin +
+                                   (int64_t)(tap0 + slot) * p.cin + ci0 + ci) = sum;
+      else if (ci == 0 && ci0 == 0)
+        out[(int64_t)p.cout * p.taps * p.cin + co] = sum.x;     // the ones slot: bias
+    }
+    cluster_sync();   // the peers have finished reading this CTA's shared memory
+  }
 }
 
 // Weight and bias gradient of the input layer from its im2col (cout 32 or
@@ -788,7 +1212,46 @@ cudaError_t launch_wgrad_inst(cudaStream_t s, const CUtensorMap& g, const CUtens
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  return launch_k(k_wgrad_tc<BN, MT>, grid, kThreads, Cfg::SMEM, s, g, x, p);
+  if (!p.out) return launch_k(k_wgrad_tc<BN, MT>, grid, kThreads, Cfg::SMEM, s, g, x, p);
+  // the splits of a tile as one cluster (grid.x == splits)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute la[2];
+  la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  la[0].val.programmaticStreamSerializationAllowed = 1;
+  la[1].id = cudaLaunchAttributeClusterDimension;
+  la[1].val.clusterDim.x = grid.x;
+  la[1].val.clusterDim.y = 1;
+  la[1].val.clusterDim.z = 1;
+  cfg.attrs = la;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, k_wgrad_tc<BN, MT>, g, x, p);
+}
+
+template <int BN, int BKC, int EPI, int BMN>
+cudaError_t launch_halo_inst(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                             const ConvTcArgs& p, int tiles_m, int tiles_n, int items) {
+  using Cfg = HaloCfg<BN, BKC, EPI>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_conv_halo<BN, BKC, EPI, BMN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Cfg::SMEM_MAX);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int kper = p.kch / BKC;
+  const int fixed = 1024 + 9 * kper * Cfg::B_TILE + Cfg::XS;
+  int S = (Cfg::SMEM_MAX - fixed) / Cfg::A_BYTES;
+  if (S > 6) S = 6;
+  if (S < 2) return cudaErrorInvalidValue;
+  const int smem = fixed + S * Cfg::A_BYTES;
+  const int grid = items < sm_count() ? items : sm_count();
+  return launch_k(k_conv_halo<BN, BKC, EPI, BMN>, grid, kHaloThreads, smem, s, a, b, p, tiles_m,
+                  tiles_n, items, S);
 }
 
 }  // namespace
@@ -971,10 +1434,55 @@ cudaError_t launch_pack_w0(cudaStream_t s, const bf16* w, bf16* w0p, int64_t rs,
   return launch_k(k_pack_w0, dim3((unsigned)((per + 255) / 256), C), 256, 0, s, w, w0p, rs, cout);
 }
 
+// the instantiated (BN, BKC, epilogue) combinations of k_conv_halo
+static const int kHaloKinds[][3] = {{64, 64, EPI_STORE}, {64, 64, EPI_DRELU}, {64, 64, EPI_ADD},
+                                    {64, 32, EPI_POOL},  {128, 64, EPI_POOL}, {32, 64, EPI_DRELU},
+                                    {64, 64, EPI_DPOOL}};
+
+bool halo_supported(int H, int W, int kch, int bn, int bkc, int epi) {
+  if (H % 16 || W % 8 || kch % bkc) return false;
+  // resident weights and at least two halo stages within the shared memory
+  const int a_bytes = ((kHaloW * kHaloH * bkc * 2) + 1023) / 1024 * 1024;
+  const int need = 1024 + 9 * kch * bn * 2 + (epi == EPI_POOL ? 2 * kEpiScratch : 0) + 2 * a_bytes;
+  if (need > 232448 - 1024) return false;
+  for (const auto& k : kHaloKinds)
+    if (k[0] == bn && k[1] == bkc && k[2] == epi) return true;
+  return false;
+}
+
+cudaError_t launch_conv_halo(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
+                             const ConvTcArgs& p, int bn, int bkc, int epi, int C) {
+  if (p.ntaps != 9 || p.stride != 1 || p.bw != 8 || p.hb != 16 || p.bb != 1 ||
+      !halo_supported(p.H, p.W, p.kch, bn, bkc, epi) || p.tiles_w * 8 != p.W ||
+      p.tiles_h * 16 != p.H ||
+      p.n_total % bn)
+    return cudaErrorInvalidValue;
+  for (int t = 0; t < 9; ++t)
+    if (p.tsrc[t] || p.tdy[t] < -1 || p.tdy[t] > 1 || p.tdx[t] < -1 || p.tdx[t] > 1)
+      return cudaErrorInvalidValue;
+  const int tiles_m = p.tiles_w * p.tiles_h * p.B;
+  const int tiles_n = p.n_total / bn;
+  const int items = C * tiles_m * tiles_n;
+#define GCPSL_HALO(BN_, BKC_, EPI_, BMN_)                                                  \
+  if (bn == BN_ && bkc == BKC_ && epi == EPI_ && (BMN_ == (epi >= EPI_DPOOL)))            \
+    return launch_halo_inst<BN_, BKC_, EPI_, BMN_>(s, a, b, p, tiles_m, tiles_n, items);
+  GCPSL_HALO(64, 64, EPI_STORE, 0)
+  GCPSL_HALO(64, 64, EPI_DRELU, 1)
+  GCPSL_HALO(64, 64, EPI_ADD, 1)
+  GCPSL_HALO(64, 32, EPI_POOL, 0)
+  GCPSL_HALO(128, 64, EPI_POOL, 0)
+  GCPSL_HALO(32, 64, EPI_DRELU, 1)
+  GCPSL_HALO(64, 64, EPI_DPOOL, 1)
+#undef GCPSL_HALO
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C) {
   const int tg = 256 / bn;                            // slots per CTA
   if ((p.taps != 9 && p.taps != 1) || (p.taps == 1 && p.pad != 0)) return cudaErrorInvalidValue;
+  if (p.out && (p.splits > kWgradClusterMax || (uintptr_t)p.out % 16 || p.out_rs % 4))
+    return cudaErrorInvalidValue;
   const int groups = (p.taps + p.bias + tg - 1) / tg;
   const int mt = p.cout % 128 == 0 ? 128 : 64;
   const int tiles = groups * (p.cin / bn) * ((p.cout + mt - 1) / mt);

@@ -260,8 +260,15 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
                    L.tiles_h, a.conv[i].cout, c->d_theta + a.off_b[i], P,
                    (bf16*)(void*)act[i + 1], c->d_code[i], c->d_err};
       conv_taps_fwd3(p);
-      LAUNCH(kFwdTc[i], launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f,
-                                           a.conv[i].pool ? EPI_POOL : EPI_RELU, C));
+      const int epi = a.conv[i].pool ? EPI_POOL : EPI_RELU;
+      if (L.halo_f) {
+        p.bw = 8; p.hb = 16; p.bb = 1;
+        p.tiles_w = a.conv[i].w / 8;
+        p.tiles_h = a.conv[i].h / 16;
+        LAUNCH(kFwdTc[i], launch_conv_halo(s, L.hfA, L.fwdB, p, L.bn_f, L.bkc_f, epi, C));
+      } else {
+        LAUNCH(kFwdTc[i], launch_conv_tc(s, L.fwdA, L.fwdB, p, L.bn_f, L.bkc_f, epi, C));
+      }
     } else {
       LAUNCH("conv_fwd", launch_conv_fwd_simt<T>(s, act[i], wts + a.off_w[i], P,
                                                  c->d_theta + a.off_b[i], P, act[i + 1],
@@ -298,11 +305,18 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
     if (L.on) {
       WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
                     L.splits, c->d_partial, c->d_err};
-      // weights and bias together (the bias follows the weight in the store)
+      // weights and bias together (the bias follows the weight in the store);
+      // few splits reduce inside a cluster and write the gradient directly
+      const bool direct = L.splits <= kWgradClusterMax && a.off_w[i] % 4 == 0;
+      if (direct) {
+        w.out = c->d_grad + a.off_w[i];
+        w.out_rs = P;
+      }
       LAUNCH(kWgradTc[i], launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
-      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
-                                                 L.splits,
-                                                 (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
+      if (!direct)
+        LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
+                                                   L.splits,
+                                                   (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
     } else if (i == 0 && c->tc0.wg_on) {
       const auto& L0 = c->tc0;
       WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L0.whb, L0.wbb, L0.kb_total, L0.kb_per_split,
@@ -330,8 +344,16 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
                    pv.pool ? nullptr : (const bf16*)(const void*)act[i],
                    (bf16*)c->gbuf(i - 1)};
       conv_taps_dgrad3(p);
-      LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d,
-                                         pv.pool ? EPI_DPOOL : EPI_DRELU, C));
+      const int epi = pv.pool ? EPI_DPOOL : EPI_DRELU;
+      if (L.halo_d) {
+        p.bw = 8; p.hb = 16; p.bb = 1;
+        p.tiles_w = cs.w / 8;
+        p.tiles_h = cs.h / 16;
+        LAUNCH(kDgradTc[i], launch_conv_halo(s, L.hdA, L.dgrB, p, std::min(L.bn_d, 64),
+                                             L.bkc_d, epi, C));
+      } else {
+        LAUNCH(kDgradTc[i], launch_conv_tc(s, L.dgrA, L.dgrB, p, L.bn_d, L.bkc_d, epi, C));
+      }
       g_ready[i - 1] = true;
     } else {
       LAUNCH("conv_dgrad", launch_conv_dgrad_simt<T>(s, g, wts + a.off_w[i], P, dact[i], C, B,
@@ -494,6 +516,15 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
                                       nbw * 2) &&
               tensor_map_bf16(&L.wgA, c->gbuf(i), 5, g_dims, wA, 128) &&
               tensor_map_bf16(&L.wgB, c->d_act[i], 5, act_in, wB, wx * 2);
+    // halo-tiled forward / data gradient where the shape allows: one box of
+    // 10 x 18 pixels per K block
+    L.halo_f = halo_supported(s.h, s.w, s.cin, L.bn_f, L.bkc_f, s.pool ? EPI_POOL : EPI_RELU);
+    L.halo_d = i > 0 && halo_supported(s.h, s.w, s.cout, std::min(L.bn_d, 64), L.bkc_d,
+                                       a.conv[i - 1].pool ? EPI_DPOOL : EPI_DRELU);
+    const uint32_t hbf[5] = {(uint32_t)L.bkc_f, 10, 18, 1, 1};
+    const uint32_t hbd[5] = {(uint32_t)L.bkc_d, 10, 18, 1, 1};
+    if (L.halo_f) ok = ok && tensor_map_bf16(&L.hfA, c->d_act[i], 5, act_in, hbf, L.bkc_f * 2);
+    if (L.halo_d) ok = ok && tensor_map_bf16(&L.hdA, c->gbuf(i), 5, g_dims, hbd, L.bkc_d * 2);
     if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for layer %d", i);
     L.on = true;
   }

@@ -139,6 +139,9 @@ struct gcpsl_ctx {
     int bn_f, bkc_f, bn_d, bkc_d, bn_w;
     int splits, kb_total, kb_per_split;
     CUtensorMap fwdA, fwdB, dgrA, dgrB, wgA, wgB;
+    // halo-tiled forward / data gradient (3x3 stride 1, resident weights)
+    bool halo_f = false, halo_d = false;
+    CUtensorMap hfA, hdA;
   } tc[4];
   // input layer on the tensor cores (bf16 mode): the gather writes its
   // im2col, x0c = 32 columns per pixel; packed weights [C][cout][32]

@@ -114,29 +114,49 @@ k_chan_sums(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* 
   }
 }
 
-// One warp per (replica, set) [GroupNorm (b, group) / BatchNorm channel]:
-// the set's sums in a fixed lane order (xor tree), in fp64.
-__device__ __forceinline__ double warp_sum(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
+// Per-channel sums over the batch: a block of 8 warps per (replica, chunk of
+// 32 channels); lane = channel (coalesced loads of the [b][ch][2] sums), warp
+// w takes the examples b = w, w + 8, ... in fp64, and the eight warp partials
+// are added in warp order.  Fixed order, independent of C.
+constexpr int kChanWarps = 8;
+__device__ __forceinline__ void batch_sums(const float* __restrict__ sums, int c, int chn, int B,
+                                           int ch, double* red, double& s1, double& s2) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  double a = 0.0, q = 0.0;
+  for (int b = w; b < B; b += kChanWarps) {
+    const float2 v = *reinterpret_cast<const float2*>(sums + (((int64_t)c * B + b) * ch + chn) * 2);
+    a += v.x;
+    q += v.y;
+  }
+  red[(w * 32 + lane) * 2] = a;
+  red[(w * 32 + lane) * 2 + 1] = q;
+  __syncthreads();
+  s1 = 0.0;
+  s2 = 0.0;
+  if (w == 0) {
+    for (int k = 0; k < kChanWarps; ++k) {
+      s1 += red[(k * 32 + lane) * 2];
+      s2 += red[(k * 32 + lane) * 2 + 1];
+    }
+  }
 }
 
 // Forward statistics per set, and per (replica, [example,] channel) the
 // affine form of the normalisation: scale = gamma * rstd, shift = beta -
 // mean * scale (GroupNorm: per example; BatchNorm: shared over the batch).
 // BatchNorm also updates its running statistics (momentum 0.1, unbiased
-// variance).
-__global__ void k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ gamma,
-                                    const float* __restrict__ beta, int64_t g_rs,
-                                    float* __restrict__ mean, float* __restrict__ rstd,
-                                    float2* __restrict__ ss, float* __restrict__ run,
-                                    int64_t run_rs, int C, int B, int HW, int ch, int gn) {
+// variance).  GroupNorm: one thread per (replica, example, group);
+// BatchNorm: batch_sums blocks.
+__global__ void __launch_bounds__(kChanWarps * 32)
+k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ gamma,
+                    const float* __restrict__ beta, int64_t g_rs, float* __restrict__ mean,
+                    float* __restrict__ rstd, float2* __restrict__ ss, float* __restrict__ run,
+                    int64_t run_rs, int C, int B, int HW, int ch, int gn) {
+  __shared__ double red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
   const int cpg = ch / 32;
   if (gn) {
-    // GroupNorm: one thread per (replica, example, group)
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= (int64_t)C * B * 32) return;
     const int64_t cbv = i / 32;                     // c * B + b
@@ -161,23 +181,16 @@ __global__ void k_norm_finalize_fwd(const float* __restrict__ sums, const float*
     }
     return;
   }
-  // BatchNorm: one warp per (replica, channel), lanes over the batch
-  const int lane = threadIdx.x & 31;
-  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  if (w >= (int64_t)C * ch) return;
-  const int c = (int)(w / ch), s = (int)(w % ch);
-  double s1 = 0.0, s2 = 0.0;
-  for (int b = lane; b < B; b += 32) {
-    const int64_t o = (((int64_t)c * B + b) * ch + s) * 2;
-    s1 += sums[o]; s2 += sums[o + 1];
-  }
-  s1 = warp_sum(s1);
-  s2 = warp_sum(s2);
-  if (lane != 0) return;
+  const int chunks = ch / 32;
+  const int c = blockIdx.x / chunks, s = (blockIdx.x % chunks) * 32 + (threadIdx.x & 31);
+  double s1, s2;
+  batch_sums(sums, c, s, B, ch, red, s1, s2);
+  if (threadIdx.x >= 32) return;
   const double n = (double)B * HW, mu = s1 / n;
   double var = s2 / n - mu * mu;
   var = var > 0.0 ? var : 0.0;
   const double r = 1.0 / sqrt(var + kEps);
+  const int64_t w = (int64_t)c * ch + s;
   mean[w] = (float)mu;
   rstd[w] = (float)r;
   if (run) {
@@ -188,7 +201,7 @@ __global__ void k_norm_finalize_fwd(const float* __restrict__ sums, const float*
   }
   const float gsv = gamma[(int64_t)c * g_rs + s], bsv = beta[(int64_t)c * g_rs + s];
   const float sc = (float)((double)gsv * r);
-  ss[(int64_t)c * ch + s] = make_float2(sc, (float)((double)bsv - mu * sc));
+  ss[w] = make_float2(sc, (float)((double)bsv - mu * sc));
 }
 
 // Backward: per set m1 = mean(dz gamma), m2 = mean(dz gamma x_hat), and the
@@ -197,34 +210,29 @@ __global__ void k_norm_finalize_fwd(const float* __restrict__ sums, const float*
 // per channel dgamma = sum_b S2[b][c], dbeta = sum_b S1[b][c].
 //   GroupNorm set (b, g): m1 = sum_{c in g} gamma_c S1[b][c] / n (m2 with S2);
 //   BatchNorm set c:      m1 = gamma_c sum_b S1[b][c] / n.
-__global__ void k_norm_finalize_bwd(const float* __restrict__ sums,
-                                    const float* __restrict__ gamma, int64_t g_rs,
-                                    const float* __restrict__ mean, const float* __restrict__ rstd,
-                                    float4* __restrict__ kk, float* __restrict__ dgamma,
-                                    float* __restrict__ dbeta, int64_t d_rs, int C, int B, int HW,
-                                    int ch, int gn) {
+// Blocks [0, C ch / 32): batch_sums per channel chunk (dgamma, dbeta and
+// the whole BatchNorm set); GroupNorm sets follow, one thread each.
+__global__ void __launch_bounds__(kChanWarps * 32)
+k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ gamma,
+                    int64_t g_rs, const float* __restrict__ mean, const float* __restrict__ rstd,
+                    float4* __restrict__ kk, float* __restrict__ dgamma,
+                    float* __restrict__ dbeta, int64_t d_rs, int C, int B, int HW, int ch,
+                    int gn) {
+  __shared__ double red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
   const int cpg = ch / 32;
-  // warps [0, C*ch): per channel over the batch (dgamma, dbeta; the whole
-  // BatchNorm set); GroupNorm sets follow, one thread each
-  const int64_t nw = (int64_t)C * ch;
-  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t w = t >> 5;
-  const int lane = threadIdx.x & 31;
-  if (w < nw) {
-    const int c = (int)(w / ch), chn = (int)(w % ch);
-    double a = 0.0, b2 = 0.0;
-    for (int b = lane; b < B; b += 32) {
-      const int64_t o = (((int64_t)c * B + b) * ch + chn) * 2;
-      a += sums[o]; b2 += sums[o + 1];
-    }
-    a = warp_sum(a);
-    b2 = warp_sum(b2);
-    if (lane != 0) return;
+  const int chunks = ch / 32;
+  const int nb = C * chunks;
+  if ((int)blockIdx.x < nb) {
+    const int c = blockIdx.x / chunks, chn = (blockIdx.x % chunks) * 32 + (threadIdx.x & 31);
+    double a, b2;
+    batch_sums(sums, c, chn, B, ch, red, a, b2);
+    if (threadIdx.x >= 32) return;
     dgamma[(int64_t)c * d_rs + chn] = (float)b2;
     dbeta[(int64_t)c * d_rs + chn] = (float)a;
     if (!gn) {
+      const int64_t w = (int64_t)c * ch + chn;
       const double g = gamma[(int64_t)c * g_rs + chn];
       const double n = (double)B * HW;
       const double m1 = g * a / n, m2 = g * b2 / n;
@@ -235,8 +243,8 @@ __global__ void k_norm_finalize_bwd(const float* __restrict__ sums,
     return;
   }
   if (!gn) return;
-  const int64_t i = t - nw * 32;                   // GroupNorm set (c, b, g)
-  if (i < 0 || i >= (int64_t)C * B * 32) return;
+  const int64_t i = (int64_t)(blockIdx.x - nb) * blockDim.x + threadIdx.x;  // set (c, b, g)
+  if (i >= (int64_t)C * B * 32) return;
   const int64_t cbv = i / 32;
   const int g = (int)(i % 32), c = (int)(cbv / B);
   const float* gm = gamma + (int64_t)c * g_rs;
@@ -381,8 +389,9 @@ cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const fl
                                      const float* beta, int64_t g_rs, float* mean, float* rstd,
                                      float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
                                      int ch, int gn) {
-  const int64_t threads = gn ? (int64_t)C * B * 32 : (int64_t)C * ch * 32;
-  return launch_k(k_norm_finalize_fwd, nblk(threads, 256), 256, 0, s, sums, gamma, beta, g_rs,
+  if (ch % 32) return cudaErrorInvalidValue;
+  const unsigned blocks = gn ? nblk((int64_t)C * B * 32, 256) : (unsigned)(C * (ch / 32));
+  return launch_k(k_norm_finalize_fwd, blocks, 256, 0, s, sums, gamma, beta, g_rs,
                   mean, rstd, ss, run, run_rs, C, B, HW, ch, gn);
 }
 
@@ -390,8 +399,9 @@ cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const fl
                                      int64_t g_rs, const float* mean, const float* rstd,
                                      float4* kk, float* dgamma, float* dbeta, int64_t d_rs, int C,
                                      int B, int HW, int ch, int gn) {
-  const int64_t threads = (int64_t)C * ch * 32 + (gn ? (int64_t)C * B * 32 : 0);
-  return launch_k(k_norm_finalize_bwd, nblk(threads, 256), 256, 0, s, sums, gamma, g_rs, mean,
+  if (ch % 32) return cudaErrorInvalidValue;
+  const unsigned blocks = (unsigned)(C * (ch / 32)) + (gn ? nblk((int64_t)C * B * 32, 256) : 0u);
+  return launch_k(k_norm_finalize_bwd, blocks, 256, 0, s, sums, gamma, g_rs, mean,
                   rstd, kk, dgamma, dbeta, d_rs, C, B, HW, ch, gn);
 }
 

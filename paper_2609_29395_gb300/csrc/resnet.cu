@@ -40,6 +40,10 @@ struct RnConv {
   int bn_f, bkc_f, bn_d, bkc_d, bn_w;
   int whb, wbb, kb_total, kb_per_split, splits;
   CUtensorMap fA, fB, dA, dB, wA, wB;
+  // halo-tiled forward / data gradient (3x3 stride 1 on 8 x 16 M tiles,
+  // resident weights, N tiles of 64): activation boxes of 10 x 18 pixels
+  bool halo_f, halo_d;
+  CUtensorMap hfA, hfB, hdA;
   const bf16* x;                    // input activation
   bf16* y;                          // output (pre-norm)
   bf16* g;                          // its gradient dL/dy (scratch shared with other layers)
@@ -355,6 +359,18 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
       ok = ok && tensor_map_bf16(&v.wA, v.g, 5, gd, wa, 128) &&
            tensor_map_bf16(&v.wB, v.x, 5, xd, wb, wx * 2, es);
     }
+    v.halo_f = v.halo_d = false;
+    if (!im2col && v.k == 3 && v.stride == 1) {
+      v.halo_f = halo_supported(v.hout, v.wout, v.cin, 64, 64, EPI_STORE);
+      v.halo_d = halo_supported(v.hout, v.wout, v.cout, 64, 64, EPI_DRELU) &&
+                 halo_supported(v.hout, v.wout, v.cout, 64, 64, EPI_ADD);
+      const uint32_t hb[5] = {64, 10, 18, 1, 1};
+      const uint32_t hw[4] = {64, 1, 64, 1};
+      if (v.halo_f)
+        ok = ok && tensor_map_bf16(&v.hfA, v.x, 5, xd, hb, 128) &&
+             tensor_map_bf16_strided(&v.hfB, c->d_shadow + v.off_w, 4, wd, rs, hw, 128);
+      if (v.halo_d) ok = ok && tensor_map_bf16(&v.hdA, v.g, 5, gd, hb, 128);
+    }
     if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed (stage %d conv)", v.stage);
     return GCPSL_OK;
   };
@@ -370,6 +386,15 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
 
 namespace {
 
+// M tiles of the halo-tiled kernel: 8 columns x 16 rows of one image
+void halo_tiles(ConvTcArgs& p, const RnConv& v) {
+  p.bw = 8;
+  p.hb = 16;
+  p.bb = 1;
+  p.tiles_w = v.wout / 8;
+  p.tiles_h = v.hout / 16;
+}
+
 // forward convolution: raw bf16 output (the norm follows)
 gcpsl_status conv_fwd(gcpsl_ctx* c, const RnConv& v, bool im2col) {
   ConvTcArgs p{v.hout, v.wout, c->B, im2col ? 32 : v.cin, v.bw, v.hb, v.bb, v.tiles_w,
@@ -377,6 +402,12 @@ gcpsl_status conv_fwd(gcpsl_ctx* c, const RnConv& v, bool im2col) {
   if (v.k == 3 && !im2col) conv_taps_fwd3(p);
   else conv_taps_one(p);                         // 1x1, or the stem's im2col (K = 32)
   p.stride = v.stride;
+  if (v.halo_f) {
+    halo_tiles(p, v);
+    LAUNCH(kFwdName[v.stage], launch_conv_halo(c->stream, v.hfA, v.hfB, p, 64, 64, EPI_STORE,
+                                               c->C));
+    return GCPSL_OK;
+  }
   LAUNCH(kFwdName[v.stage], launch_conv_tc(c->stream, v.fA, v.fB, p, v.bn_f, v.bkc_f, EPI_STORE,
                                            c->C));
   return GCPSL_OK;
@@ -390,9 +421,16 @@ gcpsl_status conv_wgrad(gcpsl_ctx* c, const RnConv& v) {
   w.stride = v.stride;
   w.pad = v.k / 2;
   const int64_t per = (int64_t)v.cout * v.k * v.k * v.cin;
+  // few splits reduce inside a cluster and write the gradient directly
+  const bool direct = v.splits <= kWgradClusterMax && v.off_w % 4 == 0;
+  if (direct) {
+    w.out = c->d_grad + v.off_w;
+    w.out_rs = c->P_pad;
+  }
   LAUNCH(kWgradName[v.stage], launch_wgrad_tc(c->stream, v.wA, v.wB, w, v.bn_w, c->C));
-  LAUNCH("rn_wgrad_reduce", launch_wgrad_reduce(c->stream, c->d_partial, c->d_grad + v.off_w,
-                                                c->P_pad, v.splits, per, c->C));
+  if (!direct)
+    LAUNCH("rn_wgrad_reduce", launch_wgrad_reduce(c->stream, c->d_partial, c->d_grad + v.off_w,
+                                                  c->P_pad, v.splits, per, c->C));
   return GCPSL_OK;
 }
 
@@ -483,8 +521,14 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
       ConvTcArgs p{b.c2.hout, b.c2.wout, B, b.c2.cout, b.c2.bw, b.c2.hb, b.c2.bb, b.c2.tiles_w,
                    b.c2.tiles_h, b.c2.cin, nullptr, 0, nullptr, nullptr, c->d_err, b.a1, r.dt};
       conv_taps_dgrad3(p);
-      LAUNCH(kDgradName[b.c2.stage], launch_conv_tc(s, b.c2.dA, b.c2.dB, p, b.c2.bn_d,
-                                                    b.c2.bkc_d, EPI_DRELU, C));
+      if (b.c2.halo_d) {
+        halo_tiles(p, b.c2);
+        LAUNCH(kDgradName[b.c2.stage], launch_conv_halo(s, b.c2.hdA, b.c2.dB, p, 64, 64,
+                                                        EPI_DRELU, C));
+      } else {
+        LAUNCH(kDgradName[b.c2.stage], launch_conv_tc(s, b.c2.dA, b.c2.dB, p, b.c2.bn_d,
+                                                      b.c2.bkc_d, EPI_DRELU, C));
+      }
     }
     RN(norm_bwd(c, b.n1, b.y1, r.dt, nullptr, nullptr, r.dy));
     RN(conv_wgrad(c, b.c1));
@@ -494,7 +538,13 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
                    nullptr, 0, dx, nullptr, c->d_err};
       conv_taps_dgrad3(p);
       p.res = r.dz;
-      LAUNCH(kDgradName[v.stage], launch_conv_tc(s, v.dA, v.dB, p, v.bn_d, v.bkc_d, EPI_ADD, C));
+      if (v.halo_d) {
+        halo_tiles(p, v);
+        LAUNCH(kDgradName[v.stage], launch_conv_halo(s, v.hdA, v.dB, p, 64, 64, EPI_ADD, C));
+      } else {
+        LAUNCH(kDgradName[v.stage], launch_conv_tc(s, v.dA, v.dB, p, v.bn_d, v.bkc_d, EPI_ADD,
+                                                   C));
+      }
     } else {
       for (int py = 0; py < 2; ++py)
         for (int px = 0; px < 2; ++px) {
