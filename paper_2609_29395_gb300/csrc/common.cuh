@@ -229,6 +229,16 @@ cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensor
 // memory: `a` maps the activation operand with a box of BKC channels x 10
 // x 18 pixels, `b` the weights as for launch_conv_tc with an N box of
 // min(bn, 64).  p.bw = 8, p.hb = 16, p.bb = 1.
+// weight gradient of a 3x3 stride-1 convolution from halo tiles of x:
+// `x` maps the input with a box of CB = (cin == 32 ? 32 : 64) channels x
+// (W + 2) columns x (hb + 2) rows (cin == 32) or hb rows (otherwise); `g`
+// as for launch_wgrad_tc.  p.hb * W == 64, p.bb == 1; tiles per replica
+// from wgrad_halo_tiles.
+bool wgrad_halo_supported(int H, int W, int cin, int cout, int taps, int stride);
+int wgrad_halo_rows(int cin);     // kernel rows per CTA (3 or 1)
+int wgrad_halo_tiles(int cin, int cout);
+cudaError_t launch_wgrad_halo(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                              const WgradTcArgs& p, int C);
 bool halo_supported(int H, int W, int kch, int bn, int bkc, int epi);
 cudaError_t launch_conv_halo(cudaStream_t s, const CUtensorMap& a, const CUtensorMap& b,
                              const ConvTcArgs& p, int bn, int bkc, int epi, int C);

@@ -1027,6 +1027,218 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
   }
 }
 
+// Weight gradient of a 3x3 stride-1 convolution from halo tiles.
+//
+// Per K block (64 output pixels: hb rows x W columns of one image, W = 16,
+// 32 or 64) the TMA warp loads the g tile and ONE box of x around the block:
+// (W + 2) columns x (hb + 2) rows (ND = 3: all three kernel rows dy) or hb
+// rows shifted by dy (ND = 1: one kernel row per CTA).  For a K step of 16
+// pixels (within one image row) and a kernel row dy, the three taps dx =
+// -1, 0, 1 are one MN-major B operand of N = 3 x CB: its N blocks of CB
+// channels start one pixel row apart (LBO = row bytes), i.e. block j reads
+// the x rows of block 0 shifted by j pixels.  So a K step is ND MMAs of
+// N = 3 CB (+ one N = 32 MMA against a block of ones for the bias), with
+// no per-tap loads.  Accumulator columns: [dy group][dx][ci] then the bias.
+// Splits, partials and the cluster reduction as in k_wgrad_tc; the partial
+// layout is the parameter layout [cout][9][cin] (+ [cout]).
+template <int CB, int MT, int ND>
+struct WhCfg {
+  static constexpr int ROWB = CB * 2;
+  static constexpr int A_BYTES = MT * 64 * 2;               // MT co x 64 pixels
+  // halo rows at most: (hb + 2)(W + 2) <= 3 * 66 (ND = 3), hb (W + 2) <= 4 * 18 (ND = 1)
+  static constexpr int HMAX = ND == 3 ? 3 * 66 : 4 * 18;
+  static constexpr int H_BYTES = (HMAX * ROWB + 1023) / 1024 * 1024;
+  static constexpr int STAGE = A_BYTES + H_BYTES;
+  static constexpr int S0 = 190 * 1024 / STAGE;
+  static constexpr int S = S0 > 6 ? 6 : S0;
+  static constexpr int NT = ND * 3 * CB;                     // tap columns
+  static constexpr int ONES = 16 * 64;                       // 16 K rows x 32 ones (64 B rows)
+  static constexpr int SMEM = 1024 + S * STAGE + ONES;
+  static constexpr uint32_t TCOLS = NT + 32 <= 256 ? 256 : 512;
+  static_assert(MT * (NT + 32 + 4) * 4 <= S * STAGE, "accumulator tile exceeds the ring");
+};
+
+template <int CB, int MT, int ND>
+__global__ void __launch_bounds__(kThreads, 1)
+k_wgrad_halo(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tX,
+             const WgradTcArgs p) {
+  using Cfg = WhCfg<CB, MT, ND>;
+  constexpr int S = Cfg::S, NT = Cfg::NT;
+  extern __shared__ uint8_t smraw[];
+  uint8_t* sm = align1024(smraw);
+  uint8_t* ones = sm + S * Cfg::STAGE;
+  __shared__ uint64_t full[S], empty[S], done;
+  __shared__ uint32_t tbase;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, c = blockIdx.z;
+  constexpr int DG = 3 / ND;                                 // dy groups
+  const int ci_tiles = p.cin / CB;
+  int t = blockIdx.y;
+  const int dyg = t % DG; t /= DG;
+  const int ci0 = (t % ci_tiles) * CB; t /= ci_tiles;
+  const int co0 = t * MT;
+  const bool bias_cta = p.bias && ci0 == 0 && dyg == 0;
+  const int ncols = NT + (bias_cta ? 32 : 0);
+  const int per = p.cout * 9 * p.cin + (p.bias ? p.cout : 0);
+  const int kb_begin = split * p.kb_per_split;
+  const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
+  const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
+  const int rows_blocks = p.H / p.hb;
+  const int HW2 = p.W + 2;
+  const int hrows = ND == 3 ? p.hb + 2 : p.hb;
+  const uint32_t h_tx = (uint32_t)(HW2 * hrows * Cfg::ROWB);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(&done, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tG);
+    tma_prefetch_desc(&tX);
+  }
+  if (bias_cta) {
+    const uint4 one = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    for (int i = threadIdx.x; i < Cfg::ONES / 16; i += blockDim.x) reinterpret_cast<uint4*>(ones)[i] = one;
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tbase;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (elect_one()) {
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % S;
+        if (i >= S && !mbar_wait(&empty[s], ((i / S) & 1) ^ 1)) { atomicOr(p.err, 8); break; }
+        const int kb = kb_begin + i;
+        const int b = kb / rows_blocks, h = (kb % rows_blocks) * p.hb;
+        uint8_t* sa = sm + s * Cfg::STAGE;
+        mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + h_tx);
+        tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, c);
+        if (MT == 128)
+          tma_load_5d(sa + 64 * 64 * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0, 0, h, b,
+                      c);
+        tma_load_5d(sa + Cfg::A_BYTES, &tX, &full[s], ci0, -1, ND == 3 ? h - 1 : h + dyg - 1, b,
+                    c);
+      }
+    }
+  } else if (warp == 1) {
+    if (elect_one()) {
+      constexpr uint32_t swz = CB == 64 ? SWZ_128 : SWZ_64;
+      const uint32_t idesc = idesc_bf16(MT, 3 * CB, 1, 1);
+      const uint32_t idesc_b = idesc_bf16(MT, 32, 1, 1);
+      constexpr uint32_t a_lbo = 64 * 64 * 2;                 // the two 64-co blocks (MT = 128)
+      const uint64_t ones_desc = smem_desc(smem_u32(ones), 64 * 16, 8 * 64, SWZ_64);
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % S;
+        if (!mbar_wait(&full[s], (i / S) & 1)) { atomicOr(p.err, 16); break; }
+        tc_fence_after();
+        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), hb0 = a + Cfg::A_BYTES;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int y = (16 * k) / p.W, x0 = (16 * k) % p.W;
+          const uint64_t ad = smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128);
+#pragma unroll
+          for (int d = 0; d < ND; ++d) {
+            const uint32_t start = hb0 + (uint32_t)(((y + d) * HW2 + x0) * Cfg::ROWB);
+            mma_f16(tmem + d * 3 * CB, ad,
+                    smem_desc(start, Cfg::ROWB, 8 * Cfg::ROWB, swz), idesc, (i | k) != 0);
+          }
+          if (bias_cta) mma_f16(tmem + NT, ad, ones_desc, idesc_b, (i | k) != 0);
+        }
+        mma_commit(&empty[s]);
+      }
+      mma_commit(&done);
+    }
+  } else {
+    const int q = warp & 3;
+    const int row = MT == 128 ? q * 32 + lane : q * 16 + lane;
+    const int co = co0 + row;
+    const bool mine = (MT == 128 || lane < 16) && co < p.cout;
+    const bool ok = mbar_wait(&done, 0);
+    if (!ok) atomicOr(p.err, 32);
+    tc_fence_after();
+    const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
+    if (p.out) {
+      float* acc = reinterpret_cast<float*>(sm);
+      const int ld = ncols + 4;
+#pragma unroll 1
+      for (int c0 = 0; c0 < ncols; c0 += 16) {
+        float v[16];
+        tmem_ld16(trow + c0, v);
+        tmem_ld_wait();
+        if (MT == 128 || lane < 16) {
+          float4* d4 = reinterpret_cast<float4*>(acc + (int64_t)row * ld + c0);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+    } else {
+      float* part = p.partial + ((int64_t)c * p.splits + split) * per;
+#pragma unroll 1
+      for (int c0 = 0; c0 < ncols; c0 += 16) {
+        float v[16];
+        tmem_ld16(trow + c0, v);
+        tmem_ld_wait();
+        if (!mine) continue;
+        if (c0 >= NT) {                                       // the ones block: bias
+          if (c0 == NT) part[p.cout * 9 * p.cin + co] = nkb ? v[0] : 0.f;
+          continue;
+        }
+        const int dd = c0 / (3 * CB), j = (c0 % (3 * CB)) / CB, ci = c0 % CB;
+        const int tap = (ND == 3 ? dd : dyg) * 3 + j;
+        float4* d4 = reinterpret_cast<float4*>(part + (int64_t)co * 9 * p.cin +
+                                               (int64_t)tap * p.cin + ci0 + ci);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
+  if (p.out) {
+    // splits of this tile = the CTAs of one cluster; rank k sums its slice
+    cluster_sync();
+    const int ld = ncols + 4, upr = ncols / 4;
+    const int rows = p.cout - co0 < MT ? p.cout - co0 : MT;
+    const int U = rows * upr, S_ = p.splits, k = (int)cluster_rank();
+    const int ub = (int)((int64_t)U * k / S_), ue = (int)((int64_t)U * (k + 1) / S_);
+    const uint32_t base = smem_u32(sm);
+    float* out = p.out + (int64_t)c * p.out_rs;
+    for (int u = ub + (int)threadIdx.x; u < ue; u += blockDim.x) {
+      const int rw = u / upr, col = (u % upr) * 4;
+      const uint32_t off = base + (uint32_t)(rw * ld + col) * 4u;
+      float4 v[kWgradClusterMax];
+#pragma unroll
+      for (int j = 0; j < kWgradClusterMax; ++j)
+        if (j < S_) v[j] = ld_peer_f4(peer_smem(off, (uint32_t)j));
+      float4 sum = v[0];
+#pragma unroll
+      for (int j = 1; j < kWgradClusterMax; ++j)
+        if (j < S_) { sum.x += v[j].x; sum.y += v[j].y; sum.z += v[j].z; sum.w += v[j].w; }
+      const int co = co0 + rw;
+      if (col >= NT) {
+        if (col == NT) out[(int64_t)p.cout * 9 * p.cin + co] = sum.x;
+        continue;
+      }
+      const int dd = col / (3 * CB), j = (col % (3 * CB)) / CB, ci = col % CB;
+      const int tap = (ND == 3 ? dd : dyg) * 3 + j;
+      *reinterpret_cast<float4*>(out + (int64_t)co * 9 * p.cin + (int64_t)tap * p.cin + ci0 + ci) =
+          sum;
+    }
+    cluster_sync();
+  }
+}
+
 // Weight and bias gradient of the input layer from its im2col (cout 32 or
 // 64): D[co][k] = sum_p g[p][co] x0[p][k], a plain GEMM over the pixels;
 // column k < 27 is W[co][tap][ci] (k = tap * 3 + ci), column 27 (the ones
@@ -1254,6 +1466,34 @@ cudaError_t launch_halo_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
                   tiles_n, items, S);
 }
 
+template <int CB, int MT, int ND>
+cudaError_t launch_wgrad_halo_inst(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                                   const WgradTcArgs& p, dim3 grid) {
+  using Cfg = WhCfg<CB, MT, ND>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_wgrad_halo<CB, MT, ND>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute la[2];
+  la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  la[0].val.programmaticStreamSerializationAllowed = 1;
+  la[1].id = cudaLaunchAttributeClusterDimension;
+  la[1].val.clusterDim.x = p.out ? grid.x : 1;
+  la[1].val.clusterDim.y = 1;
+  la[1].val.clusterDim.z = 1;
+  cfg.attrs = la;
+  cfg.numAttrs = p.out ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, k_wgrad_halo<CB, MT, ND>, g, x, p);
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -1475,6 +1715,37 @@ cudaError_t launch_conv_halo(cudaStream_t s, const CUtensorMap& a, const CUtenso
   GCPSL_HALO(64, 64, EPI_DPOOL, 1)
 #undef GCPSL_HALO
   return cudaErrorInvalidValue;
+}
+
+int wgrad_halo_rows(int cin) { return cin == 32 ? 3 : 1; }
+
+bool wgrad_halo_supported(int H, int W, int cin, int cout, int taps, int stride) {
+  // ND = 1 holds hb (W + 2) <= 72 halo rows: W = 16 or 32
+  const bool w_ok = cin == 32 ? (W == 16 || W == 32 || W == 64) : (W == 16 || W == 32);
+  return taps == 9 && stride == 1 && w_ok && H % (64 / W) == 0 &&
+         (cin == 32 || cin % 64 == 0) && (cout == 64 || cout % 128 == 0);
+}
+
+int wgrad_halo_tiles(int cin, int cout) {
+  const int cb = cin == 32 ? 32 : 64;
+  const int mt = cout % 128 == 0 ? 128 : 64;
+  return (cout / mt) * (cin / cb) * (3 / wgrad_halo_rows(cin));
+}
+
+cudaError_t launch_wgrad_halo(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                              const WgradTcArgs& p, int C) {
+  if (!wgrad_halo_supported(p.H, p.W, p.cin, p.cout, p.taps, p.stride) || p.hb * p.W != 64 ||
+      p.bb != 1 || p.pad != 1)
+    return cudaErrorInvalidValue;
+  if (p.out && (p.splits > kWgradClusterMax || (uintptr_t)p.out % 16 || p.out_rs % 4))
+    return cudaErrorInvalidValue;
+  const dim3 grid(p.splits, wgrad_halo_tiles(p.cin, p.cout), C);
+  const bool m64 = p.cout % 128 != 0;
+  if (p.cin == 32)
+    return m64 ? launch_wgrad_halo_inst<32, 64, 3>(s, g, x, p, grid)
+               : launch_wgrad_halo_inst<32, 128, 3>(s, g, x, p, grid);
+  return m64 ? launch_wgrad_halo_inst<64, 64, 1>(s, g, x, p, grid)
+             : launch_wgrad_halo_inst<64, 128, 1>(s, g, x, p, grid);
 }
 
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,

@@ -312,7 +312,10 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
         w.out = c->d_grad + a.off_w[i];
         w.out_rs = P;
       }
-      LAUNCH(kWgradTc[i], launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
+      if (L.wg_halo)
+        LAUNCH(kWgradTc[i], launch_wgrad_halo(s, L.wgA, L.wgH, w, C));
+      else
+        LAUNCH(kWgradTc[i], launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
       if (!direct)
         LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
                                                    L.splits,
@@ -481,7 +484,9 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     const int tg = 256 / L.bn_w;                      // slots per weight-gradient CTA
     const int groups = (9 + 1 + tg - 1) / tg;          // 9 taps + the bias slot
     const int mt = s.cout % 128 == 0 ? 128 : 64;      // output channels per tile
-    const int tiles = groups * (s.cin / L.bn_w) * ((s.cout + mt - 1) / mt);
+    L.wg_halo = wgrad_halo_supported(s.h, s.w, s.cin, s.cout, 9, 1) && L.whb * s.w == 64;
+    const int tiles = L.wg_halo ? wgrad_halo_tiles(s.cin, s.cout)
+                                : groups * (s.cin / L.bn_w) * ((s.cout + mt - 1) / mt);
     L.kb_total = ((B + L.wbb - 1) / L.wbb) * (s.h / L.whb);
     // the split (hence the summation order) depends on the per-replica shape
     // only, so C grouped replicas reproduce C one-replica runs bit for bit
@@ -525,6 +530,12 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     const uint32_t hbd[5] = {(uint32_t)L.bkc_d, 10, 18, 1, 1};
     if (L.halo_f) ok = ok && tensor_map_bf16(&L.hfA, c->d_act[i], 5, act_in, hbf, L.bkc_f * 2);
     if (L.halo_d) ok = ok && tensor_map_bf16(&L.hdA, c->gbuf(i), 5, g_dims, hbd, L.bkc_d * 2);
+    if (L.wg_halo) {
+      const int cb = s.cin == 32 ? 32 : 64;
+      const int hrows = wgrad_halo_rows(s.cin) == 3 ? L.whb + 2 : L.whb;
+      const uint32_t hx[5] = {(uint32_t)cb, (uint32_t)s.w + 2, (uint32_t)hrows, 1, 1};
+      ok = ok && tensor_map_bf16(&L.wgH, c->d_act[i], 5, act_in, hx, cb * 2);
+    }
     if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for layer %d", i);
     L.on = true;
   }

@@ -142,6 +142,8 @@ struct gcpsl_ctx {
     // halo-tiled forward / data gradient (3x3 stride 1, resident weights)
     bool halo_f = false, halo_d = false;
     CUtensorMap hfA, hdA;
+    bool wg_halo = false;          // weight gradient from halo tiles of x
+    CUtensorMap wgH;
   } tc[4];
   // input layer on the tensor cores (bf16 mode): the gather writes its
   // im2col, x0c = 32 columns per pixel; packed weights [C][cout][32]

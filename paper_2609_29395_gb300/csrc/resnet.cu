@@ -44,6 +44,8 @@ struct RnConv {
   // resident weights, N tiles of 64): activation boxes of 10 x 18 pixels
   bool halo_f, halo_d;
   CUtensorMap hfA, hfB, hdA;
+  bool wg_halo;                     // weight gradient from halo tiles of x
+  CUtensorMap wH;
   const bf16* x;                    // input activation
   bf16* y;                          // output (pre-norm)
   bf16* g;                          // its gradient dL/dy (scratch shared with other layers)
@@ -331,8 +333,12 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
       return fail(c, GCPSL_E_UNSUPPORTED, "no weight-gradient K block for %dx%d", v.wout, v.hout);
     v.kb_total = ((B + v.wbb - 1) / v.wbb) * (v.hout / v.whb);
     int tiles;
+    v.wg_halo = !im2col && v.whb * v.wout == 64 &&
+                wgrad_halo_supported(v.hout, v.wout, v.cin, v.cout, v.k * v.k, v.stride);
     if (im2col) {
       tiles = 1;
+    } else if (v.wg_halo) {
+      tiles = wgrad_halo_tiles(v.cin, v.cout);
     } else {
       const int tg = 256 / v.bn_w, taps = v.k * v.k;
       const int mt = v.cout % 128 == 0 ? 128 : 64;
@@ -354,6 +360,12 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
       ok = ok && tensor_map_bf16(&v.wA, v.g, 5, gd, wa0, v.cout * 2) &&
            tensor_map_bf16(&v.wB, v.x, 5, xd, xb0, 64);
     } else {
+      if (v.wg_halo) {
+        const int cb = v.cin == 32 ? 32 : 64;
+        const int hrows = wgrad_halo_rows(v.cin) == 3 ? v.whb + 2 : v.whb;
+        const uint32_t hx[5] = {(uint32_t)cb, (uint32_t)v.wout + 2, (uint32_t)hrows, 1, 1};
+        ok = ok && tensor_map_bf16(&v.wH, v.x, 5, xd, hx, cb * 2);
+      }
       const int wx = std::min(v.cin, 64);
       const uint32_t wb[5] = {(uint32_t)wx, s * v.wout, s * v.whb, (uint32_t)v.wbb, 1};
       ok = ok && tensor_map_bf16(&v.wA, v.g, 5, gd, wa, 128) &&
@@ -427,7 +439,10 @@ gcpsl_status conv_wgrad(gcpsl_ctx* c, const RnConv& v) {
     w.out = c->d_grad + v.off_w;
     w.out_rs = c->P_pad;
   }
-  LAUNCH(kWgradName[v.stage], launch_wgrad_tc(c->stream, v.wA, v.wB, w, v.bn_w, c->C));
+  if (v.wg_halo)
+    LAUNCH(kWgradName[v.stage], launch_wgrad_halo(c->stream, v.wA, v.wH, w, c->C));
+  else
+    LAUNCH(kWgradName[v.stage], launch_wgrad_tc(c->stream, v.wA, v.wB, w, v.bn_w, c->C));
   if (!direct)
     LAUNCH("rn_wgrad_reduce", launch_wgrad_reduce(c->stream, c->d_partial, c->d_grad + v.off_w,
                                                   c->P_pad, v.splits, per, c->C));
