@@ -70,7 +70,9 @@ def build(force: bool = False, verbose: bool = False, extra=()) -> Path:
     if LIB.exists() and not force and LIB.stat().st_mtime >= max(o.stat().st_mtime for o in objs):
         return LIB
     tmp = LIBDIR / f".libgcpsl.{os.getpid()}.so"
-    cmd = [nvcc()] + ARCH + ["-shared", "-o", str(tmp)] + [str(o) for o in objs] + ["-lcuda"]
+    # every symbol resolved at link time: an undefined one fails the build, not the load
+    cmd = [nvcc()] + ARCH + ["-shared", "-Xlinker", "--no-undefined", "-o", str(tmp)] + \
+        [str(o) for o in objs] + ["-lcuda"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         # libcuda is resolved at run time through the runtime's entry points

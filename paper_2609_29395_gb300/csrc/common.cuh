@@ -205,13 +205,16 @@ struct WgradTcArgs {
   int taps = 9;         // 9 (3x3) or 1 (1x1)
   int bias = 1;         // also the bias gradient (a block of ones)
   int stride = 1, pad = 1;  // x pixel of output pixel p and tap (kh, kw): p*stride + k - pad
-  // non-null: the splits (<= kWgradClusterMax) run as one thread-block
-  // cluster per tile and write the summed gradient to out[c * out_rs + ...]
-  // (same layout as a partial; 16-byte aligned); `partial` is then unused
+  // non-null (one split only): the gradient is written to out[c * out_rs +
+  // ...] directly (same layout as a partial; 16-byte aligned) and `partial`
+  // is unused
   float* out = nullptr;
   int64_t out_rs = 0;
 };
-constexpr int kWgradClusterMax = 8;   // portable cluster size
+// splits of a weight gradient with `tiles` tiles and kb_total K blocks per
+// replica (a function of the per-replica shape only)
+int wgrad_splits(int tiles, int kb_total, int64_t per);
+int wgrad_tc_tiles(int cin, int cout, int taps, int bn);
 // elem_strides (nullable): traversal stride per dimension; a box then
 // loads ceil(box[i] / elem_strides[i]) elements along dimension i
 bool tensor_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
@@ -284,6 +287,30 @@ cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* k
 cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch);
 
 // optim.cu
+// A range of every replica's parameters [off, off + count) whose gradient
+// the update reads from src: element j of replica c is the sum over s <
+// splits of src[(c * splits + s) * per + j] (split partials of a weight
+// gradient), or src[c * per + j] with splits = 1 (the gradient store).
+// total = C * count elements, in (replica, element) order.
+struct SgdSeg {
+  const float* src;
+  int64_t off, count, per, total;
+  int splits;
+};
+constexpr int kSgdThreads = 256, kSgdPer = 2;
+// quads (4 parameters) per update block of a segment with `splits` sources:
+// about the same bytes per block whatever the split count
+inline int sgd_chunk(int splits) {
+  const int n = kSgdThreads * kSgdPer * 2 / (splits + 1);
+  return n < kSgdThreads ? kSgdThreads : n;
+}
+// SGD over the segments (they tile [0, P_pad) of each replica; offsets,
+// counts and strides multiples of 4), then the bf16 shadow; one launch for
+// all replicas.  blocks[b] = {segment, first quad of the block in it, quads
+// (<= kSgdThreads * kSgdPer), 0}.
+cudaError_t launch_sgd_seg(cudaStream_t s, float* theta, float* mom, bf16* shadow,
+                           const SgdSeg* segs, const int4* blocks, int nblocks, int64_t P_pad,
+                           float lr, float momentum, float wd, int nesterov, int64_t* d_t);
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,
                        bf16* shadow, int64_t n, float lr, float momentum, float wd,
                        int nesterov, int64_t* d_t);

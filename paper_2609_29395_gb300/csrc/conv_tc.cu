@@ -21,11 +21,14 @@
 //    The input layer runs through it with one tap over its im2col (K = 32).
 //  k_wgrad_tc: dW[co][tap][ci] = sum_p g[p][co] x[p + shift(tap)][ci]
 //    M = co, N = ci, K = pixels.  Both operands are MN-major tiles (pixels are
-//    rows, channels contiguous), loaded as 64-pixel boxes.  The pixel range is
-//    split across CTAs.  Up to kWgradClusterMax splits form one thread-block
-//    cluster and sum their fp32 tiles through distributed shared memory in
-//    rank order; with more splits each writes an fp32 partial tile and
-//    k_wgrad_reduce sums the partials in split order (deterministic).
+//    rows, channels contiguous), loaded as 64-pixel boxes.  Persistent: a
+//    CTA works through a contiguous range of (replica, tile, pixel split)
+//    items; a single split writes the gradient, several write fp32 partials
+//    that k_wgrad_reduce sums in split order (deterministic).
+//  k_wgrad_halo: the same for 3x3 stride-1 layers from one halo box of x per
+//    K block.
+//  k_conv_halo: 3x3 stride-1 fprop / dgrad from one halo box per K block,
+//    weights resident in shared memory.
 //
 // Warp roles (192 threads): warp 0 issues TMA, warp 1 allocates TMEM and
 // issues MMAs, warps 2-5 run the epilogue (warp w reads TMEM lanes
@@ -801,83 +804,137 @@ __global__ void k_pack_w0(const bf16* __restrict__ w, bf16* __restrict__ w0p, in
 }
 
 // ---------------------------------------------------------------------------
-// weight gradient
+// weight gradient (persistent)
 // ---------------------------------------------------------------------------
-// One CTA owns a group of up to TG = 256/BN slots of a (128-co, BN-ci) tile:
-// per K block the g tile is loaded once and multiplied, in one N <= 256 MMA,
-// against the group's tap-shifted x tiles (consecutive N blocks).  Group 0
-// holds taps 0..TG-2 and, in its last slot, a block of ones (written once
-// into every ring stage), so its accumulator also yields the bias gradient
-// sum_p g[p][co]; groups g >= 1 hold TG taps each.  The fp32 partial of a
-// split is laid out like the parameters, [cout][9][cin] then [cout].
-// MT = 128 output channels per tile (two 64-wide g blocks), or MT = 64 for
-// layers with 64 output channels (M = 64 MMAs: row r of the accumulator is
-// TMEM lane 32 * (r / 16) + r % 16).
+// A work item is (replica, tile, split): one tile of dW over one K range (a
+// split of the output pixels).  CTA b of G takes the contiguous item range
+// [b items / G, (b+1) items / G) (splits fastest).  The TMA warp runs
+// through an S-stage ring across items; the MMA warp alternates between
+// NBUF TMEM accumulators, so one item's epilogue overlaps the next item's
+// MMAs.  An item's fp32 result goes to the gradient itself (one split) or
+// to its split's partial, laid out like the parameters ([cout][taps][cin]
+// then [cout]), summed in split order by k_wgrad_reduce.  The bias gradient
+// sum_p g[p][co] is one extra N = 32 MMA per K step against a block of
+// ones, in the items of the last tap group with ci0 = 0.  MT = 128 output
+// channels per tile (two 64-wide g blocks), or MT = 64 for layers with 64
+// output channels (M = 64 MMAs: row r of the accumulator is TMEM lane
+// 32 * (r / 16) + r % 16).
+constexpr int kOnesBytes = 16 * 64;            // 16 K rows x 32 ones (64-byte rows)
+
+struct WgItem {
+  int c, tile, split, kb0, nkb;
+};
+__device__ __forceinline__ WgItem wg_item(int t, int tiles, const WgradTcArgs& p) {
+  WgItem it;
+  it.c = t / (tiles * p.splits);
+  const int r = t % (tiles * p.splits);
+  it.tile = r / p.splits;
+  it.split = r % p.splits;
+  it.kb0 = it.split * p.kb_per_split;
+  const int kb1 = min(it.kb0 + p.kb_per_split, p.kb_total);
+  it.nkb = kb1 > it.kb0 ? kb1 - it.kb0 : 0;
+  return it;
+}
+
+// Drain one accumulator (rows = output channels co0 + row) to the fp32
+// store of its replica and split: columns [0, ncols) in chunks of 16 that
+// stay inside one (tap, channel block); dst_col(col) gives the offset of a
+// column in a row ([tap][cin] order) and bias_col (if >= 0) the column that
+// holds the bias.
+template <int MT, typename ColFn>
+__device__ __forceinline__ void wgrad_drain(uint32_t trow, int q, int lane, int co0, int ncols,
+                                            int bias_col, bool zero, float* dst, int row_len,
+                                            int cout, ColFn dst_col) {
+  const int co = co0 + (MT == 128 ? q * 32 + lane : q * 16 + lane);
+  const bool mine = (MT == 128 || lane < 16) && co < cout;
+#pragma unroll 1
+  for (int c0 = 0; c0 < ncols; c0 += 16) {
+    float v[16];
+    tmem_ld16(trow + c0, v);
+    tmem_wait_regs(v);
+    if (!mine) continue;
+    if (c0 == bias_col) {
+      dst[(int64_t)cout * row_len + co] = zero ? 0.f : v[0];
+      continue;
+    }
+    if (bias_col >= 0 && c0 > bias_col) continue;
+    float4* d4 = reinterpret_cast<float4*>(dst + (int64_t)co * row_len + dst_col(c0));
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      d4[i] = zero ? make_float4(0.f, 0.f, 0.f, 0.f)
+                   : make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+  }
+}
+
+__device__ __forceinline__ float* wgrad_dst(const WgradTcArgs& p, const WgItem& it, int per) {
+  return p.out ? p.out + (int64_t)it.c * p.out_rs
+               : p.partial + ((int64_t)it.c * p.splits + it.split) * per;
+}
+
+// k_wgrad_tc: any 3x3 / 1x1 layer (stride 1 or 2).  A tile is a group of up
+// to TG = 256/BN taps of a (MT-co, BN-ci) block: per K block the g tile is
+// loaded once and multiplied, in one N <= 256 MMA, against the group's
+// tap-shifted x tiles (consecutive MN-major N blocks).
 template <int BN, int MT>
 struct WgCfg {
   static constexpr int BKP = 64;                         // pixels per stage
-  static constexpr int TG = 256 / BN;                    // taps per CTA
+  static constexpr int TG = 256 / BN;                    // taps per tile
   static constexpr int A_BYTES = MT * BKP * 2;           // MT co (64-wide blocks)
   static constexpr int TAP_BYTES = BN * BKP * 2;         // one tap's x tile
   static constexpr int STAGE = A_BYTES + TG * TAP_BYTES;
   static constexpr int S0 = 200 * 1024 / STAGE;
   static constexpr int S = S0 > 6 ? 6 : S0;
-  static constexpr int SMEM = 1024 + S * STAGE;
-  static constexpr uint32_t TCOLS = 256;
-  // the cluster reduction's fp32 tile reuses the operand ring
-  static_assert(MT * (TG * BN + 4) * 4 <= S * STAGE, "accumulator tile exceeds the ring");
+  static constexpr int SMEM = 1024 + S * STAGE + kOnesBytes;
+  static constexpr uint32_t TCOLS = 256;                 // per accumulator; two of them
+  static_assert(BN + 32 <= TCOLS, "last tap group and bias exceed the accumulator");
+  // all 512 TMEM columns per CTA: one CTA per SM
+  static_assert(SMEM > 116 * 1024, "a second CTA per SM would wait for TMEM");
 };
 
 template <int BN, int MT>
 __global__ void __launch_bounds__(kThreads, 1)
 k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tX,
-           const WgradTcArgs p) {
+           const WgradTcArgs p, int C) {
   using Cfg = WgCfg<BN, MT>;
   constexpr int S = Cfg::S, TG = Cfg::TG;
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = align1024(smraw);
-  __shared__ uint64_t full[S], empty[S], done;
+  uint8_t* ones = sm + S * Cfg::STAGE;
+  __shared__ uint64_t full[S], empty[S], tfull[2], tempty[2];
   __shared__ uint32_t tbase;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x, c = blockIdx.z;
   const int ci_tiles = p.cin / BN;
   const int co_tiles = (p.cout + MT - 1) / MT;
-  int t = blockIdx.y;
-  const int ci0 = (t % ci_tiles) * BN; t /= ci_tiles;
-  const int co0 = (t % co_tiles) * MT; t /= co_tiles;
-  // slot group t: slots [t*TG, t*TG + nslots) of taps 0..taps-1 and, with
-  // the bias, one last slot of ones
-  const int total = p.taps + p.bias;
-  const int tap0 = t * TG;
-  const int nslots = total - tap0 < TG ? total - tap0 : TG;  // N = nslots * BN
-  const bool bias_grp = p.bias && p.taps >= tap0 && p.taps < tap0 + nslots;
-  const int ntaps = bias_grp ? nslots - 1 : nslots;
+  const int groups = (p.taps + TG - 1) / TG;
+  const int tiles = groups * ci_tiles * co_tiles;
+  const int items = C * tiles * p.splits;
+  const int t_begin = (int)((int64_t)items * blockIdx.x / gridDim.x);
+  const int t_end = (int)((int64_t)items * (blockIdx.x + 1) / gridDim.x);
   const int ksz = p.taps == 9 ? 3 : 1;
-  const int per = p.cout * p.taps * p.cin + (p.bias ? p.cout : 0);   // partial length per split
-  const int kb_begin = split * p.kb_per_split;
-  const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
-  const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
+  const int per = p.cout * p.taps * p.cin + (p.bias ? p.cout : 0);
   const int rows_blocks = p.H / p.hb;               // pixel blocks per image group
+  // tile -> (tap group, ci0, co0); the bias rides on the last group at ci0 = 0
+  auto tile_of = [&](int tile, int& g, int& ci0, int& co0) {
+    ci0 = (tile % ci_tiles) * BN; tile /= ci_tiles;
+    co0 = (tile % co_tiles) * MT; tile /= co_tiles;
+    g = tile;
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    mbar_init(&done, 1);
+    for (int b = 0; b < 2; ++b) { mbar_init(&tfull[b], 1); mbar_init(&tempty[b], 128); }
     fence_mbar_init();
     tma_prefetch_desc(&tG);
     tma_prefetch_desc(&tX);
   }
-  if (bias_grp) {
-    // the ones block (bf16 1.0 everywhere, so the swizzle does not matter)
-    const uint4 ones = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
-    for (int s = 0; s < S; ++s) {
-      uint4* dst = reinterpret_cast<uint4*>(sm + s * Cfg::STAGE + Cfg::A_BYTES +
-                                            ntaps * Cfg::TAP_BYTES);
-      for (int i = threadIdx.x; i < Cfg::TAP_BYTES / 16; i += blockDim.x) dst[i] = ones;
-    }
+  {
+    const uint4 one = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    for (int i = threadIdx.x; i < kOnesBytes / 16; i += blockDim.x)
+      reinterpret_cast<uint4*>(ones)[i] = one;
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
+  if (warp == 1) { tmem_alloc(&tbase, 2 * Cfg::TCOLS); tmem_relinquish(); }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -887,160 +944,123 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
 
   if (warp == 0) {
     if (elect_one()) {
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % S;
-        if (i >= S && !mbar_wait(&empty[s], ((i / S) & 1) ^ 1)) { atomicOr(p.err, 8); break; }
-        const int kb = kb_begin + i;
-        const int b = (kb / rows_blocks) * p.bb, h = (kb % rows_blocks) * p.hb;
-        uint8_t* sa = sm + s * Cfg::STAGE;
-        uint8_t* sb = sa + Cfg::A_BYTES;
-        mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + ntaps * Cfg::TAP_BYTES);
-        tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, c);
-        // rows 64..127 of an MT = 128 tile: the next 64 channels, or (cout
-        // < co0 + 128) a second copy of the first block whose results the
-        // epilogue drops
-        if (MT == 128)
-          tma_load_5d(sa + 64 * Cfg::BKP * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0,
-                      0, h, b, c);
-        for (int tj = 0; tj < ntaps; ++tj) {
-          const int tap = tap0 + tj, kh = tap / ksz, kw = tap % ksz;
+      int it = 0;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t) {
+        const WgItem w = wg_item(t, tiles, p);
+        int g, ci0, co0;
+        tile_of(w.tile, g, ci0, co0);
+        const int tap0 = g * TG, ntaps = min(TG, p.taps - tap0);
+        for (int i = 0; i < w.nkb; ++i, ++it) {
+          const int s = it % S;
+          if (it >= S && !mbar_wait(&empty[s], ((it / S) & 1) ^ 1)) {
+            atomicOr(p.err, 8);
+            ok = false;
+            break;
+          }
+          const int kb = w.kb0 + i;
+          const int b = (kb / rows_blocks) * p.bb, h = (kb % rows_blocks) * p.hb;
+          uint8_t* sa = sm + s * Cfg::STAGE;
+          uint8_t* sb = sa + Cfg::A_BYTES;
+          mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + ntaps * Cfg::TAP_BYTES);
+          tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, w.c);
+          // rows 64..127 of an MT = 128 tile: the next 64 channels, or (cout
+          // < co0 + 128) a second copy of the first block whose results the
+          // epilogue drops
+          if (MT == 128)
+            tma_load_5d(sa + 64 * Cfg::BKP * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0,
+                        0, h, b, w.c);
+          for (int tj = 0; tj < ntaps; ++tj) {
+            const int tap = tap0 + tj, kh = tap / ksz, kw = tap % ksz;
 #pragma unroll
-          for (int j = 0; j < (BN + 63) / 64; ++j)
-            tma_load_5d(sb + tj * Cfg::TAP_BYTES + j * 64 * Cfg::BKP * 2, &tX, &full[s],
-                        ci0 + 64 * j, kw - p.pad, h * p.stride + kh - p.pad, b, c);
+            for (int j = 0; j < (BN + 63) / 64; ++j)
+              tma_load_5d(sb + tj * Cfg::TAP_BYTES + j * 64 * Cfg::BKP * 2, &tX, &full[s],
+                          ci0 + 64 * j, kw - p.pad, h * p.stride + kh - p.pad, b, w.c);
+          }
         }
       }
     }
   } else if (warp == 1) {
     if (elect_one()) {
-      // one MMA per k step with N = ntaps*BN: the taps' x tiles are the
-      // consecutive MN-major N blocks of one B operand (64-ci blocks, SW128,
-      // or 32-ci blocks of 64-byte rows, SW64), `b_blk` bytes apart
-      const uint32_t idesc = idesc_bf16(MT, nslots * BN, 1, 1);
+      // MN-major B: the taps' x tiles are consecutive N blocks (64-ci blocks,
+      // SW128, or 32-ci blocks of 64-byte rows, SW64), `b_blk` bytes apart
       constexpr uint32_t a_lbo = 64 * Cfg::BKP * 2;
       constexpr uint32_t b_swz = BN >= 64 ? SWZ_128 : SWZ_64;
       constexpr uint32_t b_row = BN >= 64 ? 128 : 64;
       constexpr uint32_t b_blk = b_row * Cfg::BKP;
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % S;
-        if (!mbar_wait(&full[s], (i / S) & 1)) { atomicOr(p.err, 16); break; }
+      const uint32_t idesc_b = idesc_bf16(MT, 32, 1, 1);
+      const uint64_t ones_desc = smem_desc(smem_u32(ones), 64 * 16, 8 * 64, SWZ_64);
+      int it = 0, tl = 0;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t, ++tl) {
+        const WgItem w = wg_item(t, tiles, p);
+        int g, ci0, co0;
+        tile_of(w.tile, g, ci0, co0);
+        const int ntaps = min(TG, p.taps - g * TG);
+        const bool bias = p.bias && ci0 == 0 && g == groups - 1;
+        const uint32_t idesc = idesc_bf16(MT, ntaps * BN, 1, 1);
+        const int buf = tl & 1;
+        if (tl >= 2 && !mbar_wait(&tempty[buf], ((tl >> 1) & 1) ^ 1)) { atomicOr(p.err, 16); break; }
         tc_fence_after();
-        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
+        const uint32_t d = tmem + buf * Cfg::TCOLS;
+        for (int i = 0; i < w.nkb; ++i, ++it) {
+          const int s = it % S;
+          if (!mbar_wait(&full[s], (it / S) & 1)) { atomicOr(p.err, 16); ok = false; break; }
+          tc_fence_after();
+          const uint32_t a = smem_u32(sm + s * Cfg::STAGE), b = a + Cfg::A_BYTES;
 #pragma unroll
-        for (int k = 0; k < Cfg::BKP / 16; ++k)
-          mma_f16(tmem, smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128),
-                  smem_desc(b + k * 16 * b_row, b_blk, 8 * b_row, b_swz), idesc, (i | k) != 0);
-        mma_commit(&empty[s]);
+          for (int k = 0; k < Cfg::BKP / 16; ++k) {
+            const uint64_t ad = smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128);
+            mma_f16(d, ad, smem_desc(b + k * 16 * b_row, b_blk, 8 * b_row, b_swz), idesc,
+                    (i | k) != 0);
+            if (bias) mma_f16(d + ntaps * BN, ad, ones_desc, idesc_b, (i | k) != 0);
+          }
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&tfull[buf]);
       }
-      mma_commit(&done);
     }
   } else {
     const int q = warp & 3;
-    // accumulator row of this thread's TMEM lane (M = 64: lanes 16..31 of
-    // each quarter are unused)
-    const int row = MT == 128 ? q * 32 + lane : q * 16 + lane;
-    const int co = co0 + row;
-    const bool mine = (MT == 128 || lane < 16) && co < p.cout;
-    const bool ok = mbar_wait(&done, 0);
-    if (!ok) atomicOr(p.err, 32);
-    tc_fence_after();
-    const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
-    if (p.out) {
-      // cluster reduction: the accumulator goes to this CTA's shared memory
-      // (the operand ring is free once `done` has fired: every MMA, hence
-      // every TMA load, has completed), rows padded by 4 words
-      float* acc = reinterpret_cast<float*>(sm);
-      const int ld = nslots * BN + 4;
-#pragma unroll 1
-      for (int c0 = 0; c0 < nslots * BN; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
-        tmem_ld_wait();
-        if (MT == 128 || lane < 16) {
-          float4* d4 = reinterpret_cast<float4*>(acc + (int64_t)row * ld + c0);
-#pragma unroll
-          for (int i = 0; i < 4; ++i)
-            d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
+    int tl = 0;
+    for (int t = t_begin; t < t_end; ++t, ++tl) {
+      const int buf = tl & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl >> 1) & 1))) {
+        if (lane == 0) atomicOr(p.err, 32);
+        break;
       }
-    } else {
-      float* part = p.partial + ((int64_t)c * p.splits + split) * per;
-      if (bias_grp && ci0 == 0) {
-        float v[16];
-        tmem_ld16(trow + ntaps * BN, v);
-        tmem_ld_wait();
-        if (mine) part[p.cout * p.taps * p.cin + co] = nkb ? v[0] : 0.f;
-      }
-      for (int tj = 0; tj < ntaps; ++tj) {
-        float* dst = part + (int64_t)co * p.taps * p.cin + (int64_t)(tap0 + tj) * p.cin + ci0;
-#pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          float v[16];
-          tmem_ld16(trow + tj * BN + c0, v);
-          tmem_ld_wait();
-          if (mine) {
-            float4* d4 = reinterpret_cast<float4*>(dst + c0);
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-              d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
-          }
-        }
-      }
+      tc_fence_after();
+      const WgItem w = wg_item(t, tiles, p);
+      int g, ci0, co0;
+      tile_of(w.tile, g, ci0, co0);
+      const int tap0 = g * TG, ntaps = min(TG, p.taps - tap0);
+      const bool bias = p.bias && ci0 == 0 && g == groups - 1;
+      const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
+      const int cin = p.cin;
+      wgrad_drain<MT>(trow, q, lane, co0, ntaps * BN + (bias ? 32 : 0), bias ? ntaps * BN : -1,
+                      w.nkb == 0, wgrad_dst(p, w, per), p.taps * p.cin, p.cout,
+                      [&](int col) { return (tap0 + col / BN) * cin + ci0 + col % BN; });
+      tc_fence_before();
+      mbar_arrive(&tempty[buf]);
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
-  if (p.out) {
-    // The splits of this tile are the CTAs of one cluster (rank = split).
-    // Rank k sums the k-th 1/splits of the tile over every rank's shared
-    // memory, in rank order, and writes the gradient itself.
-    cluster_sync();
-    const int N = nslots * BN, ld = N + 4, upr = N / 4;
-    const int rows = p.cout - co0 < MT ? p.cout - co0 : MT;
-    const int U = rows * upr, S = p.splits, k = (int)cluster_rank();
-    const int ub = (int)((int64_t)U * k / S), ue = (int)((int64_t)U * (k + 1) / S);
-    const uint32_t base = smem_u32(sm);
-    float* out = p.out + (int64_t)c * p.out_rs;
-    for (int u = ub + (int)threadIdx.x; u < ue; u += blockDim.x) {
-      const int rw = u / upr, col = (u % upr) * 4;
-      const uint32_t off = base + (uint32_t)(rw * ld + col) * 4u;
-      // every rank's value in flight at once, then summed in rank order
-      float4 v[kWgradClusterMax];
-#pragma unroll
-      for (int j = 0; j < kWgradClusterMax; ++j)
-        if (j < S) v[j] = ld_peer_f4(peer_smem(off, (uint32_t)j));
-      float4 sum = v[0];
-#pragma unroll
-      for (int j = 1; j < kWgradClusterMax; ++j)
-        if (j < S) { sum.x += v[j].x; sum.y += v[j].y; sum.z += v[j].z; sum.w += v[j].w; }
-      const int slot = col / BN, ci = col % BN, co = co0 + rw;
-      if (slot < ntaps)
-        *reinterpret_cast<float4*>(out + (int64_t)co * p.taps * p.cin +
-                                   (int64_t)(tap0 + slot) * p.cin + ci0 + ci) = sum;
-      else if (ci == 0 && ci0 == 0)
-        out[(int64_t)p.cout * p.taps * p.cin + co] = sum.x;     // the ones slot: bias
-    }
-    cluster_sync();   // the peers have finished reading this CTA's shared memory
-  }
+  if (warp == 1) tmem_dealloc(tmem, 2 * Cfg::TCOLS);
 }
 
-// Weight gradient of a 3x3 stride-1 convolution from halo tiles.
+// k_wgrad_halo: 3x3 stride-1 layers from halo tiles.
 //
-// Per K block (64 output pixels: hb rows x W columns of one image, W = 16,
-// 32 or 64) the TMA warp loads the g tile and ONE box of x around the block:
-// (W + 2) columns x (hb + 2) rows (ND = 3: all three kernel rows dy) or hb
-// rows shifted by dy (ND = 1: one kernel row per CTA).  For a K step of 16
+// Per K block (64 output pixels: hb rows x W columns of one image) the TMA
+// warp loads the g tile and ONE box of x around the block: (W + 2) columns
+// x (hb + 2) rows (ND = 3: all three kernel rows dy per tile) or hb rows
+// shifted by dy (ND = 1: one kernel row per tile).  For a K step of 16
 // pixels (within one image row) and a kernel row dy, the three taps dx =
-// -1, 0, 1 are one MN-major B operand of N = 3 x CB: its N blocks of CB
-// channels start one pixel row apart (LBO = row bytes), i.e. block j reads
-// the x rows of block 0 shifted by j pixels.  So a K step is ND MMAs of
-// N = 3 CB (+ one N = 32 MMA against a block of ones for the bias), with
-// no per-tap loads.  Accumulator columns: [dy group][dx][ci] then the bias.
-// Splits, partials and the cluster reduction as in k_wgrad_tc; the partial
-// layout is the parameter layout [cout][9][cin] (+ [cout]).
+// -1, 0, 1 are one MN-major B operand of N = 3 CB: its N blocks of CB
+// channels start one pixel row apart (LBO = row bytes), so block j reads
+// the x rows of block 0 shifted by j pixels.  A K step is ND MMAs of
+// N = 3 CB, with no per-tap loads.  Accumulator columns: [dy][dx][ci], then
+// the bias.  Tiles: (dy group, ci block, co block), dy fastest.
 template <int CB, int MT, int ND>
 struct WhCfg {
   static constexpr int ROWB = CB * 2;
@@ -1049,59 +1069,64 @@ struct WhCfg {
   static constexpr int HMAX = ND == 3 ? 3 * 66 : 4 * 18;
   static constexpr int H_BYTES = (HMAX * ROWB + 1023) / 1024 * 1024;
   static constexpr int STAGE = A_BYTES + H_BYTES;
-  static constexpr int S0 = 190 * 1024 / STAGE;
-  static constexpr int S = S0 > 6 ? 6 : S0;
   static constexpr int NT = ND * 3 * CB;                     // tap columns
-  static constexpr int ONES = 16 * 64;                       // 16 K rows x 32 ones (64 B rows)
-  static constexpr int SMEM = 1024 + S * STAGE + ONES;
+  static constexpr int S0 = (NT + 32 <= 256 ? 110 : 200) * 1024 / STAGE;
+  static constexpr int S = S0 > 8 ? 8 : S0;
+  // one accumulator per CTA; with at most 256 columns two CTAs share an SM
+  // (one's epilogue overlaps the other's MMAs), else one CTA holds all 512
+  static constexpr int NBUF = 1;
   static constexpr uint32_t TCOLS = NT + 32 <= 256 ? 256 : 512;
-  static_assert(MT * (NT + 32 + 4) * 4 <= S * STAGE, "accumulator tile exceeds the ring");
+  static constexpr int CTAS = TCOLS == 256 ? 2 : 1;
+  static constexpr int SMEM0 = 1024 + S * STAGE + kOnesBytes;
+  // a lone CTA keeps at least 116 KB so that no second one lands on its SM
+  static constexpr int SMEM = CTAS == 2 ? SMEM0 : (SMEM0 > 116 * 1024 ? SMEM0 : 116 * 1024);
+  static_assert(CTAS == 1 || SMEM0 <= 113 * 1024, "two CTAs per SM do not fit");
 };
 
 template <int CB, int MT, int ND>
 __global__ void __launch_bounds__(kThreads, 1)
 k_wgrad_halo(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tX,
-             const WgradTcArgs p) {
+             const WgradTcArgs p, int C) {
   using Cfg = WhCfg<CB, MT, ND>;
-  constexpr int S = Cfg::S, NT = Cfg::NT;
+  constexpr int S = Cfg::S, NT = Cfg::NT, NBUF = Cfg::NBUF;
+  constexpr int DG = 3 / ND;                                 // dy groups
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = align1024(smraw);
   uint8_t* ones = sm + S * Cfg::STAGE;
-  __shared__ uint64_t full[S], empty[S], done;
+  __shared__ uint64_t full[S], empty[S], tfull[2], tempty[2];
   __shared__ uint32_t tbase;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x, c = blockIdx.z;
-  constexpr int DG = 3 / ND;                                 // dy groups
   const int ci_tiles = p.cin / CB;
-  int t = blockIdx.y;
-  const int dyg = t % DG; t /= DG;
-  const int ci0 = (t % ci_tiles) * CB; t /= ci_tiles;
-  const int co0 = t * MT;
-  const bool bias_cta = p.bias && ci0 == 0 && dyg == 0;
-  const int ncols = NT + (bias_cta ? 32 : 0);
+  const int tiles = ((p.cout + MT - 1) / MT) * ci_tiles * DG;
+  const int items = C * tiles * p.splits;
+  const int t_begin = (int)((int64_t)items * blockIdx.x / gridDim.x);
+  const int t_end = (int)((int64_t)items * (blockIdx.x + 1) / gridDim.x);
   const int per = p.cout * 9 * p.cin + (p.bias ? p.cout : 0);
-  const int kb_begin = split * p.kb_per_split;
-  const int kb_end = min(kb_begin + p.kb_per_split, p.kb_total);
-  const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
   const int rows_blocks = p.H / p.hb;
   const int HW2 = p.W + 2;
   const int hrows = ND == 3 ? p.hb + 2 : p.hb;
   const uint32_t h_tx = (uint32_t)(HW2 * hrows * Cfg::ROWB);
+  auto tile_of = [&](int tile, int& dyg, int& ci0, int& co0) {
+    dyg = tile % DG; tile /= DG;
+    ci0 = (tile % ci_tiles) * CB; tile /= ci_tiles;
+    co0 = tile * MT;
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    mbar_init(&done, 1);
+    for (int b = 0; b < 2; ++b) { mbar_init(&tfull[b], 1); mbar_init(&tempty[b], 128); }
     fence_mbar_init();
     tma_prefetch_desc(&tG);
     tma_prefetch_desc(&tX);
   }
-  if (bias_cta) {
+  {
     const uint4 one = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
-    for (int i = threadIdx.x; i < Cfg::ONES / 16; i += blockDim.x) reinterpret_cast<uint4*>(ones)[i] = one;
+    for (int i = threadIdx.x; i < kOnesBytes / 16; i += blockDim.x)
+      reinterpret_cast<uint4*>(ones)[i] = one;
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == 1) { tmem_alloc(&tbase, Cfg::TCOLS); tmem_relinquish(); }
+  if (warp == 1) { tmem_alloc(&tbase, NBUF * Cfg::TCOLS); tmem_relinquish(); }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -1111,132 +1136,103 @@ k_wgrad_halo(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUt
 
   if (warp == 0) {
     if (elect_one()) {
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % S;
-        if (i >= S && !mbar_wait(&empty[s], ((i / S) & 1) ^ 1)) { atomicOr(p.err, 8); break; }
-        const int kb = kb_begin + i;
-        const int b = kb / rows_blocks, h = (kb % rows_blocks) * p.hb;
-        uint8_t* sa = sm + s * Cfg::STAGE;
-        mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + h_tx);
-        tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, c);
-        if (MT == 128)
-          tma_load_5d(sa + 64 * 64 * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0, 0, h, b,
-                      c);
-        tma_load_5d(sa + Cfg::A_BYTES, &tX, &full[s], ci0, -1, ND == 3 ? h - 1 : h + dyg - 1, b,
-                    c);
+      int it = 0;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t) {
+        const WgItem w = wg_item(t, tiles, p);
+        int dyg, ci0, co0;
+        tile_of(w.tile, dyg, ci0, co0);
+        for (int i = 0; i < w.nkb; ++i, ++it) {
+          const int s = it % S;
+          if (it >= S && !mbar_wait(&empty[s], ((it / S) & 1) ^ 1)) {
+            atomicOr(p.err, 8);
+            ok = false;
+            break;
+          }
+          const int kb = w.kb0 + i;
+          const int b = kb / rows_blocks, h = (kb % rows_blocks) * p.hb;
+          uint8_t* sa = sm + s * Cfg::STAGE;
+          mbar_arrive_expect_tx(&full[s], Cfg::A_BYTES + h_tx);
+          tma_load_5d(sa, &tG, &full[s], co0, 0, h, b, w.c);
+          if (MT == 128)
+            tma_load_5d(sa + 64 * 64 * 2, &tG, &full[s], p.cout > co0 + 64 ? co0 + 64 : co0, 0, h,
+                        b, w.c);
+          tma_load_5d(sa + Cfg::A_BYTES, &tX, &full[s], ci0, -1, ND == 3 ? h - 1 : h + dyg - 1, b,
+                      w.c);
+        }
       }
     }
   } else if (warp == 1) {
     if (elect_one()) {
       constexpr uint32_t swz = CB == 64 ? SWZ_128 : SWZ_64;
-      const uint32_t idesc = idesc_bf16(MT, 3 * CB, 1, 1);
-      const uint32_t idesc_b = idesc_bf16(MT, 32, 1, 1);
+      constexpr uint32_t idesc = idesc_bf16(MT, 3 * CB, 1, 1);
+      constexpr uint32_t idesc_b = idesc_bf16(MT, 32, 1, 1);
       constexpr uint32_t a_lbo = 64 * 64 * 2;                 // the two 64-co blocks (MT = 128)
       const uint64_t ones_desc = smem_desc(smem_u32(ones), 64 * 16, 8 * 64, SWZ_64);
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % S;
-        if (!mbar_wait(&full[s], (i / S) & 1)) { atomicOr(p.err, 16); break; }
-        tc_fence_after();
-        const uint32_t a = smem_u32(sm + s * Cfg::STAGE), hb0 = a + Cfg::A_BYTES;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int y = (16 * k) / p.W, x0 = (16 * k) % p.W;
-          const uint64_t ad = smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128);
-#pragma unroll
-          for (int d = 0; d < ND; ++d) {
-            const uint32_t start = hb0 + (uint32_t)(((y + d) * HW2 + x0) * Cfg::ROWB);
-            mma_f16(tmem + d * 3 * CB, ad,
-                    smem_desc(start, Cfg::ROWB, 8 * Cfg::ROWB, swz), idesc, (i | k) != 0);
-          }
-          if (bias_cta) mma_f16(tmem + NT, ad, ones_desc, idesc_b, (i | k) != 0);
+      int it = 0, tl = 0;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t, ++tl) {
+        const WgItem w = wg_item(t, tiles, p);
+        int dyg, ci0, co0;
+        tile_of(w.tile, dyg, ci0, co0);
+        const bool bias = p.bias && ci0 == 0 && dyg == 0;
+        const int buf = tl % NBUF;
+        if (tl >= NBUF && !mbar_wait(&tempty[buf], ((tl / NBUF) & 1) ^ 1)) {
+          atomicOr(p.err, 16);
+          break;
         }
-        mma_commit(&empty[s]);
+        tc_fence_after();
+        const uint32_t d = tmem + buf * Cfg::TCOLS;
+        for (int i = 0; i < w.nkb; ++i, ++it) {
+          const int s = it % S;
+          if (!mbar_wait(&full[s], (it / S) & 1)) { atomicOr(p.err, 16); ok = false; break; }
+          tc_fence_after();
+          const uint32_t a = smem_u32(sm + s * Cfg::STAGE), hb0 = a + Cfg::A_BYTES;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int y = (16 * k) / p.W, x0 = (16 * k) % p.W;
+            const uint64_t ad = smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128);
+#pragma unroll
+            for (int dd = 0; dd < ND; ++dd) {
+              const uint32_t start = hb0 + (uint32_t)(((y + dd) * HW2 + x0) * Cfg::ROWB);
+              mma_f16(d + dd * 3 * CB, ad, smem_desc(start, Cfg::ROWB, 8 * Cfg::ROWB, swz), idesc,
+                      (i | k) != 0);
+            }
+            if (bias) mma_f16(d + NT, ad, ones_desc, idesc_b, (i | k) != 0);
+          }
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&tfull[buf]);
       }
-      mma_commit(&done);
     }
   } else {
     const int q = warp & 3;
-    const int row = MT == 128 ? q * 32 + lane : q * 16 + lane;
-    const int co = co0 + row;
-    const bool mine = (MT == 128 || lane < 16) && co < p.cout;
-    const bool ok = mbar_wait(&done, 0);
-    if (!ok) atomicOr(p.err, 32);
-    tc_fence_after();
-    const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
-    if (p.out) {
-      float* acc = reinterpret_cast<float*>(sm);
-      const int ld = ncols + 4;
-#pragma unroll 1
-      for (int c0 = 0; c0 < ncols; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
-        tmem_ld_wait();
-        if (MT == 128 || lane < 16) {
-          float4* d4 = reinterpret_cast<float4*>(acc + (int64_t)row * ld + c0);
-#pragma unroll
-          for (int i = 0; i < 4; ++i)
-            d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
+    int tl = 0;
+    for (int t = t_begin; t < t_end; ++t, ++tl) {
+      const int buf = tl % NBUF;
+      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[buf], (tl / NBUF) & 1))) {
+        if (lane == 0) atomicOr(p.err, 32);
+        break;
       }
-    } else {
-      float* part = p.partial + ((int64_t)c * p.splits + split) * per;
-#pragma unroll 1
-      for (int c0 = 0; c0 < ncols; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
-        tmem_ld_wait();
-        if (!mine) continue;
-        if (c0 >= NT) {                                       // the ones block: bias
-          if (c0 == NT) part[p.cout * 9 * p.cin + co] = nkb ? v[0] : 0.f;
-          continue;
-        }
-        const int dd = c0 / (3 * CB), j = (c0 % (3 * CB)) / CB, ci = c0 % CB;
-        const int tap = (ND == 3 ? dd : dyg) * 3 + j;
-        float4* d4 = reinterpret_cast<float4*>(part + (int64_t)co * 9 * p.cin +
-                                               (int64_t)tap * p.cin + ci0 + ci);
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          d4[i] = nkb ? make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3])
-                      : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
+      tc_fence_after();
+      const WgItem w = wg_item(t, tiles, p);
+      int dyg, ci0, co0;
+      tile_of(w.tile, dyg, ci0, co0);
+      const bool bias = p.bias && ci0 == 0 && dyg == 0;
+      const uint32_t trow = tmem + buf * Cfg::TCOLS + ((uint32_t)(q * 32) << 16);
+      const int cin = p.cin;
+      wgrad_drain<MT>(trow, q, lane, co0, NT + (bias ? 32 : 0), bias ? NT : -1, w.nkb == 0,
+                      wgrad_dst(p, w, per), 9 * p.cin, p.cout, [&](int col) {
+                        const int dd = col / (3 * CB), j = (col % (3 * CB)) / CB;
+                        return ((ND == 3 ? dd : dyg) * 3 + j) * cin + ci0 + col % CB;
+                      });
+      tc_fence_before();
+      mbar_arrive(&tempty[buf]);
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, Cfg::TCOLS);
-  if (p.out) {
-    // splits of this tile = the CTAs of one cluster; rank k sums its slice
-    cluster_sync();
-    const int ld = ncols + 4, upr = ncols / 4;
-    const int rows = p.cout - co0 < MT ? p.cout - co0 : MT;
-    const int U = rows * upr, S_ = p.splits, k = (int)cluster_rank();
-    const int ub = (int)((int64_t)U * k / S_), ue = (int)((int64_t)U * (k + 1) / S_);
-    const uint32_t base = smem_u32(sm);
-    float* out = p.out + (int64_t)c * p.out_rs;
-    for (int u = ub + (int)threadIdx.x; u < ue; u += blockDim.x) {
-      const int rw = u / upr, col = (u % upr) * 4;
-      const uint32_t off = base + (uint32_t)(rw * ld + col) * 4u;
-      float4 v[kWgradClusterMax];
-#pragma unroll
-      for (int j = 0; j < kWgradClusterMax; ++j)
-        if (j < S_) v[j] = ld_peer_f4(peer_smem(off, (uint32_t)j));
-      float4 sum = v[0];
-#pragma unroll
-      for (int j = 1; j < kWgradClusterMax; ++j)
-        if (j < S_) { sum.x += v[j].x; sum.y += v[j].y; sum.z += v[j].z; sum.w += v[j].w; }
-      const int co = co0 + rw;
-      if (col >= NT) {
-        if (col == NT) out[(int64_t)p.cout * 9 * p.cin + co] = sum.x;
-        continue;
-      }
-      const int dd = col / (3 * CB), j = (col % (3 * CB)) / CB, ci = col % CB;
-      const int tap = (ND == 3 ? dd : dyg) * 3 + j;
-      *reinterpret_cast<float4*>(out + (int64_t)co * 9 * p.cin + (int64_t)tap * p.cin + ci0 + ci) =
-          sum;
-    }
-    cluster_sync();
-  }
+  if (warp == 1) tmem_dealloc(tmem, NBUF * Cfg::TCOLS);
 }
 
 // Weight and bias gradient of the input layer from its im2col (cout 32 or
@@ -1413,34 +1409,37 @@ cudaError_t launch_conv_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
                   tiles_m, tiles_n, items);
 }
 
-template <int BN, int MT>
-cudaError_t launch_wgrad_inst(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
-                              const WgradTcArgs& p, dim3 grid) {
-  using Cfg = WgCfg<BN, MT>;
-  static bool attr = false;
+// persistent weight-gradient launch: one CTA per SM at most
+template <typename KernelT>
+cudaError_t launch_wgrad_persistent(KernelT* kernel, int smem, int ctas, bool& attr,
+                                    cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                                    const WgradTcArgs& p, int C, int tiles) {
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_wgrad_tc<BN, MT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  if (!p.out) return launch_k(k_wgrad_tc<BN, MT>, grid, kThreads, Cfg::SMEM, s, g, x, p);
-  // the splits of a tile as one cluster (grid.x == splits)
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = Cfg::SMEM;
-  cfg.stream = s;
-  cudaLaunchAttribute la[2];
-  la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  la[0].val.programmaticStreamSerializationAllowed = 1;
-  la[1].id = cudaLaunchAttributeClusterDimension;
-  la[1].val.clusterDim.x = grid.x;
-  la[1].val.clusterDim.y = 1;
-  la[1].val.clusterDim.z = 1;
-  cfg.attrs = la;
-  cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, k_wgrad_tc<BN, MT>, g, x, p);
+  const int items = C * tiles * p.splits;
+  const int cap = ctas * sm_count();
+  const int grid = items < cap ? items : cap;
+  return launch_k(kernel, grid, kThreads, smem, s, g, x, p, C);
+}
+
+template <int BN, int MT>
+cudaError_t launch_wgrad_inst(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                              const WgradTcArgs& p, int C, int tiles) {
+  static bool attr = false;
+  return launch_wgrad_persistent(k_wgrad_tc<BN, MT>, WgCfg<BN, MT>::SMEM, 1, attr, s, g, x, p, C,
+                                 tiles);
+}
+
+template <int CB, int MT, int ND>
+cudaError_t launch_wgrad_halo_inst(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
+                                   const WgradTcArgs& p, int C, int tiles) {
+  static bool attr = false;
+  using Cfg = WhCfg<CB, MT, ND>;
+  return launch_wgrad_persistent(k_wgrad_halo<CB, MT, ND>, Cfg::SMEM, Cfg::CTAS, attr, s, g, x,
+                                 p, C, tiles);
 }
 
 template <int BN, int BKC, int EPI, int BMN>
@@ -1464,34 +1463,6 @@ cudaError_t launch_halo_inst(cudaStream_t s, const CUtensorMap& a, const CUtenso
   const int grid = items < sm_count() ? items : sm_count();
   return launch_k(k_conv_halo<BN, BKC, EPI, BMN>, grid, kHaloThreads, smem, s, a, b, p, tiles_m,
                   tiles_n, items, S);
-}
-
-template <int CB, int MT, int ND>
-cudaError_t launch_wgrad_halo_inst(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
-                                   const WgradTcArgs& p, dim3 grid) {
-  using Cfg = WhCfg<CB, MT, ND>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_wgrad_halo<CB, MT, ND>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = Cfg::SMEM;
-  cfg.stream = s;
-  cudaLaunchAttribute la[2];
-  la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  la[0].val.programmaticStreamSerializationAllowed = 1;
-  la[1].id = cudaLaunchAttributeClusterDimension;
-  la[1].val.clusterDim.x = p.out ? grid.x : 1;
-  la[1].val.clusterDim.y = 1;
-  la[1].val.clusterDim.z = 1;
-  cfg.attrs = la;
-  cfg.numAttrs = p.out ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, k_wgrad_halo<CB, MT, ND>, g, x, p);
 }
 
 }  // namespace
@@ -1732,41 +1703,59 @@ int wgrad_halo_tiles(int cin, int cout) {
   return (cout / mt) * (cin / cb) * (3 / wgrad_halo_rows(cin));
 }
 
+int wgrad_splits(int tiles, int kb_total, int64_t per) {
+  // about 64 items per replica (a few per SM once several replicas are
+  // grouped), at least 8 K blocks each, and at most 16 MB of partials per
+  // replica; the per-replica shape alone decides the split, hence the
+  // summation order, so C grouped replicas reproduce C one-replica runs bit
+  // for bit
+  int splits = (64 + tiles - 1) / tiles;
+  splits = std::min(splits, std::max(1, kb_total / 8));
+  splits = (int)std::min<int64_t>(splits, std::max<int64_t>(1, (4 << 20) / per));
+  return std::max(1, splits);
+}
+
+static cudaError_t check_wgrad_out(const WgradTcArgs& p) {
+  if (p.out && (p.splits != 1 || (uintptr_t)p.out % 16 || p.out_rs % 4))
+    return cudaErrorInvalidValue;
+  return cudaSuccess;
+}
+
 cudaError_t launch_wgrad_halo(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                               const WgradTcArgs& p, int C) {
   if (!wgrad_halo_supported(p.H, p.W, p.cin, p.cout, p.taps, p.stride) || p.hb * p.W != 64 ||
-      p.bb != 1 || p.pad != 1)
+      p.bb != 1 || p.pad != 1 || check_wgrad_out(p) != cudaSuccess)
     return cudaErrorInvalidValue;
-  if (p.out && (p.splits > kWgradClusterMax || (uintptr_t)p.out % 16 || p.out_rs % 4))
-    return cudaErrorInvalidValue;
-  const dim3 grid(p.splits, wgrad_halo_tiles(p.cin, p.cout), C);
+  const int tiles = wgrad_halo_tiles(p.cin, p.cout);
   const bool m64 = p.cout % 128 != 0;
   if (p.cin == 32)
-    return m64 ? launch_wgrad_halo_inst<32, 64, 3>(s, g, x, p, grid)
-               : launch_wgrad_halo_inst<32, 128, 3>(s, g, x, p, grid);
-  return m64 ? launch_wgrad_halo_inst<64, 64, 1>(s, g, x, p, grid)
-             : launch_wgrad_halo_inst<64, 128, 1>(s, g, x, p, grid);
+    return m64 ? launch_wgrad_halo_inst<32, 64, 3>(s, g, x, p, C, tiles)
+               : launch_wgrad_halo_inst<32, 128, 3>(s, g, x, p, C, tiles);
+  return m64 ? launch_wgrad_halo_inst<64, 64, 1>(s, g, x, p, C, tiles)
+             : launch_wgrad_halo_inst<64, 128, 1>(s, g, x, p, C, tiles);
+}
+
+int wgrad_tc_tiles(int cin, int cout, int taps, int bn) {
+  const int tg = 256 / bn;
+  const int mt = cout % 128 == 0 ? 128 : 64;
+  return ((taps + tg - 1) / tg) * (cin / bn) * ((cout + mt - 1) / mt);
 }
 
 cudaError_t launch_wgrad_tc(cudaStream_t s, const CUtensorMap& g, const CUtensorMap& x,
                             const WgradTcArgs& p, int bn, int C) {
-  const int tg = 256 / bn;                            // slots per CTA
-  if ((p.taps != 9 && p.taps != 1) || (p.taps == 1 && p.pad != 0)) return cudaErrorInvalidValue;
-  if (p.out && (p.splits > kWgradClusterMax || (uintptr_t)p.out % 16 || p.out_rs % 4))
+  if ((p.taps != 9 && p.taps != 1) || (p.taps == 1 && p.pad != 0) ||
+      check_wgrad_out(p) != cudaSuccess)
     return cudaErrorInvalidValue;
-  const int groups = (p.taps + p.bias + tg - 1) / tg;
-  const int mt = p.cout % 128 == 0 ? 128 : 64;
-  const int tiles = groups * (p.cin / bn) * ((p.cout + mt - 1) / mt);
-  dim3 grid(p.splits, tiles, C);
-  if (mt == 64) {
-    if (bn == 32) return launch_wgrad_inst<32, 64>(s, g, x, p, grid);
-    if (bn == 64) return launch_wgrad_inst<64, 64>(s, g, x, p, grid);
-    if (bn == 128) return launch_wgrad_inst<128, 64>(s, g, x, p, grid);
+  const int tiles = wgrad_tc_tiles(p.cin, p.cout, p.taps, bn);
+  if (p.cout % 128 != 0) {
+    if (bn == 32) return launch_wgrad_inst<32, 64>(s, g, x, p, C, tiles);
+    if (bn == 64) return launch_wgrad_inst<64, 64>(s, g, x, p, C, tiles);
+    if (bn == 128) return launch_wgrad_inst<128, 64>(s, g, x, p, C, tiles);
     return cudaErrorInvalidValue;
   }
-  if (bn == 32) return launch_wgrad_inst<32, 128>(s, g, x, p, grid);
-  if (bn == 64) return launch_wgrad_inst<64, 128>(s, g, x, p, grid);
-  if (bn == 128) return launch_wgrad_inst<128, 128>(s, g, x, p, grid);
+  if (bn == 32) return launch_wgrad_inst<32, 128>(s, g, x, p, C, tiles);
+  if (bn == 64) return launch_wgrad_inst<64, 128>(s, g, x, p, C, tiles);
+  if (bn == 128) return launch_wgrad_inst<128, 128>(s, g, x, p, C, tiles);
   return cudaErrorInvalidValue;
 }
 

@@ -179,6 +179,50 @@ gcpsl_status gcpsl::check_device_error(gcpsl_ctx* c) {
   return GCPSL_OK;
 }
 
+float* gcpsl::partial_range(gcpsl_ctx* c, int64_t off, int64_t count, int64_t per, int splits) {
+  float* buf = nullptr;
+  if (dalloc(c, &buf, sizeof(float) * (size_t)c->C * splits * per) != GCPSL_OK) return nullptr;
+  c->pranges.push_back({off, count, per, splits, buf});
+  return buf;
+}
+
+gcpsl_status gcpsl::build_sgd_segments(gcpsl_ctx* c) {
+  if (c->pranges.empty()) return GCPSL_OK;
+  std::vector<gcpsl_ctx::PartialRange> r = c->pranges;
+  std::sort(r.begin(), r.end(), [](const auto& a, const auto& b) { return a.off < b.off; });
+  std::vector<SgdSeg> segs;
+  std::vector<int4> blocks;
+  int64_t at = 0;
+  bool aligned = true;
+  auto add = [&](const float* src, int64_t off, int64_t count, int64_t per, int splits) {
+    aligned = aligned && off % 4 == 0 && count % 4 == 0 && per % 4 == 0 &&
+              (uintptr_t)src % 16 == 0;
+    const int64_t quads = (int64_t)c->C * count / 4;
+    const int chunk = sgd_chunk(splits);
+    for (int64_t e = 0; e < quads; e += chunk)
+      blocks.push_back(make_int4((int)segs.size(), (int)e, (int)std::min<int64_t>(chunk, quads - e),
+                                 0));
+    segs.push_back({src, off, count, per, (int64_t)c->C * count, splits});
+  };
+  for (const auto& q : r) {
+    if (q.off < at || q.off + q.count > c->P_pad)
+      return fail(c, GCPSL_E_INVAL, "overlapping weight-gradient partial ranges");
+    if (q.off > at) add(c->d_grad + at, at, q.off - at, c->P_pad, 1);
+    add(q.buf, q.off, q.count, q.per, q.splits);
+    at = q.off + q.count;
+  }
+  if (at < c->P_pad) add(c->d_grad + at, at, c->P_pad - at, c->P_pad, 1);
+  if ((int64_t)c->C * c->P_pad >= ((int64_t)1 << 31) || !aligned)
+    return fail(c, GCPSL_E_UNSUPPORTED, "parameter segments not supported by the update");
+  DALLOC(c->d_sgd_segs, sizeof(SgdSeg) * segs.size());
+  DALLOC(c->d_sgd_blocks, sizeof(int4) * blocks.size());
+  CK(cudaMemcpy(c->d_sgd_segs, segs.data(), sizeof(SgdSeg) * segs.size(), cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(c->d_sgd_blocks, blocks.data(), sizeof(int4) * blocks.size(),
+                cudaMemcpyHostToDevice));
+  c->n_sgd_blocks = (int)blocks.size();
+  return GCPSL_OK;
+}
+
 namespace {
 
 // per-layer names of the tensor-core launches in the kernel timer
@@ -219,11 +263,18 @@ gcpsl_status enqueue_sample(gcpsl_ctx* c, bool boundary) {
 }
 
 gcpsl_status enqueue_sgd(gcpsl_ctx* c) {
-  LAUNCH("sgd", launch_sgd(c->stream, c->d_theta, c->d_mom, c->d_grad, c->d_shadow,
-                           (int64_t)c->C * c->P_pad, c->desc.lr, c->desc.momentum,
-                           c->desc.weight_decay, c->desc.nesterov, c->d_t));
+  if (c->n_sgd_blocks)
+    LAUNCH("sgd", launch_sgd_seg(c->stream, c->d_theta, c->d_mom, c->d_shadow, c->d_sgd_segs,
+                                 c->d_sgd_blocks, c->n_sgd_blocks, c->P_pad, c->desc.lr,
+                                 c->desc.momentum, c->desc.weight_decay, c->desc.nesterov,
+                                 c->d_t));
+  else
+    LAUNCH("sgd", launch_sgd(c->stream, c->d_theta, c->d_mom, c->d_grad, c->d_shadow,
+                             (int64_t)c->C * c->P_pad, c->desc.lr, c->desc.momentum,
+                             c->desc.weight_decay, c->desc.nesterov, c->d_t));
   return refresh_derived(c);
 }
+
 
 template <typename T>
 gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
@@ -303,12 +354,12 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
                                                       g, C, B, cs));
     const auto& R = c->red[i];
     if (L.on) {
-      WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
-                    L.splits, c->d_partial, c->d_err};
       // weights and bias together (the bias follows the weight in the store);
-      // few splits reduce inside a cluster and write the gradient directly
-      const bool direct = L.splits <= kWgradClusterMax && a.off_w[i] % 4 == 0;
-      if (direct) {
+      // a single split writes the gradient directly, several write the
+      // layer's partials, which the update sums
+      WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L.whb, L.wbb, L.kb_total, L.kb_per_split,
+                    L.splits, L.part, c->d_err};
+      if (!L.part) {
         w.out = c->d_grad + a.off_w[i];
         w.out_rs = P;
       }
@@ -316,18 +367,11 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
         LAUNCH(kWgradTc[i], launch_wgrad_halo(s, L.wgA, L.wgH, w, C));
       else
         LAUNCH(kWgradTc[i], launch_wgrad_tc(s, L.wgA, L.wgB, w, L.bn_w, C));
-      if (!direct)
-        LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[i], P,
-                                                   L.splits,
-                                                   (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
     } else if (i == 0 && c->tc0.wg_on) {
       const auto& L0 = c->tc0;
       WgradTcArgs w{cs.h, cs.w, B, cs.cout, cs.cin, L0.whb, L0.wbb, L0.kb_total, L0.kb_per_split,
-                    L0.splits, c->d_partial, c->d_err};
+                    L0.splits, L0.part, c->d_err};
       LAUNCH(kWgradTc[0], launch_wgrad0_tc(s, L0.wgA, L0.wgB, w, C));
-      LAUNCH("wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + a.off_w[0], P,
-                                                 L0.splits,
-                                                 (int64_t)cs.cout * 9 * cs.cin + cs.cout, C));
     } else {
       // weights and bias together (the bias follows the weight in the store)
       LAUNCH("conv_wgrad", launch_wgrad_simt<T>(s, act[i], i == 0 ? c->x0c : cs.cin, g,
@@ -460,7 +504,6 @@ namespace {
 gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
   const ArchSpec& a = c->a;
   const int C = c->C, B = c->B;
-  int64_t partial_max = 0;
   for (int i = 0; i < a.L(); ++i) {
     const ConvSpec& s = a.conv[i];
     auto& L = c->tc[i];
@@ -481,22 +524,19 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     L.bkc_d = std::min(s.cout, 64);
     L.bn_w = std::min(s.cin, 128);
     if (s.cout % L.bn_f || s.cin % L.bn_d || s.cin % L.bkc_f || s.cin % L.bn_w) continue;
-    const int tg = 256 / L.bn_w;                      // slots per weight-gradient CTA
-    const int groups = (9 + 1 + tg - 1) / tg;          // 9 taps + the bias slot
-    const int mt = s.cout % 128 == 0 ? 128 : 64;      // output channels per tile
     L.wg_halo = wgrad_halo_supported(s.h, s.w, s.cin, s.cout, 9, 1) && L.whb * s.w == 64;
     const int tiles = L.wg_halo ? wgrad_halo_tiles(s.cin, s.cout)
-                                : groups * (s.cin / L.bn_w) * ((s.cout + mt - 1) / mt);
+                                : wgrad_tc_tiles(s.cin, s.cout, 9, L.bn_w);
     L.kb_total = ((B + L.wbb - 1) / L.wbb) * (s.h / L.whb);
-    // the split (hence the summation order) depends on the per-replica shape
-    // only, so C grouped replicas reproduce C one-replica runs bit for bit
-    int splits = (152 + tiles - 1) / tiles;
-    // at least 16 K blocks (1024 pixels) per split: fewer partial bytes
-    splits = std::max(1, std::min(splits, (L.kb_total + 15) / 16));
+    const int64_t per = (int64_t)s.cout * 9 * s.cin + s.cout;
+    const int splits = wgrad_splits(tiles, L.kb_total, per);
     L.kb_per_split = (L.kb_total + splits - 1) / splits;
     L.splits = (L.kb_total + L.kb_per_split - 1) / L.kb_per_split;
-    partial_max = std::max(partial_max,
-                           (int64_t)C * L.splits * ((int64_t)s.cout * 9 * s.cin + s.cout));
+    L.part = nullptr;
+    if (L.splits > 1 || a.off_w[i] % 4) {
+      L.part = partial_range(c, a.off_w[i], per, per, L.splits);
+      if (!L.part) return fail(c, GCPSL_E_NOMEM, "device allocation failed");
+    }
 
     const uint64_t act_in[5] = {(uint64_t)s.cin, (uint64_t)s.w, (uint64_t)s.h, (uint64_t)B,
                                 (uint64_t)C};
@@ -539,7 +579,6 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
     if (!ok) return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for layer %d", i);
     L.on = true;
   }
-  if (partial_max) DALLOC(c->d_partial, sizeof(float) * partial_max);
 
   // the input layer (3 channels): with bf16 operands the gather writes its
   // im2col (32 columns per pixel), so its forward is a one-tap K = 32
@@ -577,11 +616,9 @@ gcpsl_status setup_tensor_core_layers(gcpsl_ctx* c) {
   if (!tensor_map_bf16(&L0.wgA, c->gbuf(0), 5, gd, gb, s0.cout * 2) ||
       !tensor_map_bf16(&L0.wgB, c->d_act[0], 5, xdims, xb, 64))
     return fail(c, GCPSL_E_CUDA, "cuTensorMapEncodeTiled failed for the input-layer gradient");
-  const int64_t need = (int64_t)C * L0.splits * ((int64_t)s0.cout * 27 + s0.cout);
-  if (need > partial_max) {
-    partial_max = need;
-    DALLOC(c->d_partial, sizeof(float) * partial_max);
-  }
+  const int64_t per0 = (int64_t)s0.cout * 27 + s0.cout;
+  L0.part = partial_range(c, a.off_w[0], per0, per0, L0.splits);
+  if (!L0.part) return fail(c, GCPSL_E_NOMEM, "device allocation failed");
   L0.wg_on = true;
   return GCPSL_OK;
 }
@@ -720,6 +757,8 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     c->w0_cout = 64;
     gcpsl_status st = rn_setup(c);
     if (st != GCPSL_OK) return st;
+    st = build_sgd_segments(c);
+    if (st != GCPSL_OK) return st;
     st = refresh_derived(c);
     if (st != GCPSL_OK) return st;
     CK(cudaDeviceSynchronize());
@@ -769,6 +808,8 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   c->w0_cout = a.conv[0].cout;
   if (c->bf) {
     gcpsl_status st = setup_tensor_core_layers(c);
+    if (st != GCPSL_OK) return st;
+    st = build_sgd_segments(c);
     if (st != GCPSL_OK) return st;
     st = refresh_derived(c);
     if (st != GCPSL_OK) return st;

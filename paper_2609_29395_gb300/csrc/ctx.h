@@ -144,6 +144,7 @@ struct gcpsl_ctx {
     CUtensorMap hfA, hdA;
     bool wg_halo = false;          // weight gradient from halo tiles of x
     CUtensorMap wgH;
+    float* part = nullptr;         // its split partials (null: written to the gradient)
   } tc[4];
   // input layer on the tensor cores (bf16 mode): the gather writes its
   // im2col, x0c = 32 columns per pixel; packed weights [C][cout][32]
@@ -154,6 +155,7 @@ struct gcpsl_ctx {
     bool wg_on = false;            // its weight gradient on the tensor cores too
     int whb, wbb, kb_total, kb_per_split, splits;
     CUtensorMap wgA, wgB;
+    float* part = nullptr;         // its split partials
   } tc0;
   int x0c = 3;
   // the ResNet-18 split (architecture 2), else null
@@ -162,7 +164,15 @@ struct gcpsl_ctx {
   int64_t w0_off = 0;
   int w0_cout = 0;
   bf16* d_w0p = nullptr;
-  float* d_partial = nullptr;      // weight-gradient split partials (tensor-core layers)
+  // weight-gradient split partials of the tensor-core layers, one buffer
+  // per layer ([C][splits][per]), summed by the update itself (k_sgd_seg);
+  // the update's segments tile [0, P_pad) with these ranges and the
+  // gradient store
+  struct PartialRange { int64_t off, count, per; int splits; float* buf; };
+  std::vector<PartialRange> pranges;
+  gcpsl::SgdSeg* d_sgd_segs = nullptr;
+  int4* d_sgd_blocks = nullptr;    // per update block: {segment, first element, count, 0}
+  int n_sgd_blocks = 0;
   // CUDA-core weight+bias gradient partials of the layers not on the tensor
   // cores (tiles of tr image rows, tiles_per_split tiles per block)
   struct RedLayer { int tr, splits, tiles_per_split; } red[4];
@@ -273,6 +283,12 @@ gcpsl_status dalloc(gcpsl_ctx* c, P** p, size_t bytes) {
   *p = (P*)q;
   return GCPSL_OK;
 }
+// a [C][splits][per] partial buffer for parameters [off, off + count) of
+// every replica, summed by the update (null on allocation failure)
+float* partial_range(gcpsl_ctx* c, int64_t off, int64_t count, int64_t per, int splits);
+// the update's segments from the partial ranges (after every setup)
+gcpsl_status build_sgd_segments(gcpsl_ctx* c);
+
 #define DALLOC(p, bytes)                                   \
   do {                                                     \
     gcpsl_status _s = dalloc(c, &(p), (size_t)(bytes));    \

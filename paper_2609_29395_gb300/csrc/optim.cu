@@ -38,6 +38,80 @@ __global__ void k_sgd(float* __restrict__ theta, float* __restrict__ mom,
   if (blockIdx.x == 0 && threadIdx.x == 0) *d_t += 1;
 }
 
+// k_sgd over parameter segments (see SgdSeg): the split partials of a
+// weight gradient are summed here, in split order, instead of in a separate
+// reduction pass.  Everything is in units of 4 parameters (segment offsets,
+// counts, strides and the replica stride are multiples of 4), 32-bit
+// indices.  Block b takes blocks[b] = {segment, first quad, quads}: fewer
+// quads per block where a segment has more splits, so that every block
+// reads about the same number of bytes; a thread keeps the loads of its
+// kSgdPer quads in flight together.
+__device__ __forceinline__ float4 f4add(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float sgd1(float& th, float& m, float g, float lr, float mu, float wd,
+                                      int nesterov) {
+  if (wd != 0.f) g = fmaf(wd, th, g);
+  if (mu != 0.f) {
+    const float v = fmaf(mu, m, g);
+    m = v;
+    g = nesterov ? fmaf(mu, v, g) : v;
+  }
+  th = fmaf(-lr, g, th);
+  return th;
+}
+
+__global__ void __launch_bounds__(kSgdThreads)
+k_sgd_seg(float4* __restrict__ theta, float4* __restrict__ mom, uint2* __restrict__ shadow,
+          const SgdSeg* __restrict__ segs, const int4* __restrict__ blocks, uint32_t P4,
+          float lr, float mu, float wd, int nesterov, int64_t* __restrict__ d_t) {
+  pdl_wait();
+  pdl_trigger();
+  const int4 bk = blocks[blockIdx.x];
+  const SgdSeg& sq = segs[bk.x];
+  const float4* src = reinterpret_cast<const float4*>(sq.src);
+  const uint32_t cnt4 = (uint32_t)(sq.count >> 2), per4 = (uint32_t)(sq.per >> 2);
+  const uint32_t off4 = (uint32_t)(sq.off >> 2);
+  const int splits = sq.splits;
+  float4 g[kSgdPer];
+  uint32_t at[kSgdPer], sa[kSgdPer];
+  bool ok[kSgdPer];
+#pragma unroll
+  for (int k = 0; k < kSgdPer; ++k) {
+    const uint32_t r = (uint32_t)(k * kSgdThreads) + threadIdx.x;
+    const uint32_t local = (uint32_t)bk.y + r;
+    const uint32_t c = local / cnt4, j = local - c * cnt4;
+    ok[k] = r < (uint32_t)bk.z;
+    at[k] = c * P4 + off4 + j;
+    sa[k] = c * (uint32_t)splits * per4 + j;
+    g[k] = ok[k] ? src[sa[k]] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  for (int sp = 1; sp < splits; ++sp) {
+#pragma unroll
+    for (int k = 0; k < kSgdPer; ++k)
+      if (ok[k]) g[k] = f4add(g[k], src[sa[k] + (uint32_t)sp * per4]);
+  }
+#pragma unroll
+  for (int k = 0; k < kSgdPer; ++k) {
+    if (!ok[k]) continue;
+    float4 th = theta[at[k]];
+    float4 m = mu != 0.f ? mom[at[k]] : make_float4(0.f, 0.f, 0.f, 0.f);
+    sgd1(th.x, m.x, g[k].x, lr, mu, wd, nesterov);
+    sgd1(th.y, m.y, g[k].y, lr, mu, wd, nesterov);
+    sgd1(th.z, m.z, g[k].z, lr, mu, wd, nesterov);
+    sgd1(th.w, m.w, g[k].w, lr, mu, wd, nesterov);
+    theta[at[k]] = th;
+    if (mu != 0.f) mom[at[k]] = m;
+    if (shadow) {
+      const __nv_bfloat162 lo = __floats2bfloat162_rn(th.x, th.y);
+      const __nv_bfloat162 hi = __floats2bfloat162_rn(th.z, th.w);
+      shadow[at[k]] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                                 *reinterpret_cast<const uint32_t*>(&hi));
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) *d_t += 1;
+}
+
 __global__ void k_fuse(float* __restrict__ theta, bf16* __restrict__ shadow,
                        const float* __restrict__ q, int C, int64_t P) {
   pdl_wait();
@@ -68,6 +142,18 @@ cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* gr
                        int nesterov, int64_t* d_t) {
   return launch_k(k_sgd, grid_for(n, 256), 256, 0, s, theta, mom, grad, shadow, n, lr, momentum,
                   wd, nesterov, d_t);
+}
+
+cudaError_t launch_sgd_seg(cudaStream_t s, float* theta, float* mom, bf16* shadow,
+                           const SgdSeg* segs, const int4* blocks, int nblocks, int64_t P_pad,
+                           float lr, float momentum, float wd, int nesterov, int64_t* d_t) {
+  if (nblocks < 1 || P_pad % 4 || (uintptr_t)theta % 16 || (uintptr_t)mom % 16 ||
+      (uintptr_t)shadow % 8)
+    return cudaErrorInvalidValue;
+  return launch_k(k_sgd_seg, (unsigned)nblocks, kSgdThreads, 0, s,
+                  reinterpret_cast<float4*>(theta), reinterpret_cast<float4*>(mom),
+                  reinterpret_cast<uint2*>(shadow), segs, blocks, (uint32_t)(P_pad / 4), lr,
+                  momentum, wd, nesterov, d_t);
 }
 
 cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,

@@ -46,6 +46,7 @@ struct RnConv {
   CUtensorMap hfA, hfB, hdA;
   bool wg_halo;                     // weight gradient from halo tiles of x
   CUtensorMap wH;
+  float* part;                      // weight-gradient split partials (null: direct)
   const bf16* x;                    // input activation
   bf16* y;                          // output (pre-norm)
   bf16* g;                          // its gradient dL/dy (scratch shared with other layers)
@@ -289,7 +290,6 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
   }
 
   // tensor maps
-  int64_t partial_max = 0;
   auto setup = [&](RnConv& v, bool im2col) -> gcpsl_status {
     if (!m_tile(v.wout, v.hout, v.bw, v.hb, v.bb))
       return fail(c, GCPSL_E_UNSUPPORTED, "no M tile for a %dx%d output", v.wout, v.hout);
@@ -340,19 +340,23 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
     } else if (v.wg_halo) {
       tiles = wgrad_halo_tiles(v.cin, v.cout);
     } else {
-      const int tg = 256 / v.bn_w, taps = v.k * v.k;
-      const int mt = v.cout % 128 == 0 ? 128 : 64;
-      tiles = ((taps + tg - 1) / tg) * (v.cin / v.bn_w) * (v.cout / mt);
+      tiles = wgrad_tc_tiles(v.cin, v.cout, v.k * v.k, v.bn_w);
     }
     // per-replica shape only: C grouped replicas equal C one-replica runs
-    int splits = (152 + tiles - 1) / tiles;
-    splits = std::max(1, std::min(splits, (v.kb_total + 15) / 16));
+    const int64_t per = im2col ? (int64_t)v.cout * 27 + v.cout
+                               : (int64_t)v.cout * v.k * v.k * v.cin;
+    int splits = wgrad_splits(tiles, v.kb_total, per);
     if (im2col) splits = std::max(1, std::min(64, (v.kb_total + 15) / 16));
     v.kb_per_split = (v.kb_total + splits - 1) / splits;
     v.splits = (v.kb_total + v.kb_per_split - 1) / v.kb_per_split;
-    const int64_t per = im2col ? (int64_t)v.cout * 27 + v.cout
-                               : (int64_t)v.cout * v.k * v.k * v.cin;
-    partial_max = std::max(partial_max, (int64_t)C * v.splits * per);
+    // several splits write partials that the update sums; the stem's
+    // partial also holds its ones-column sums (no parameter), so it always
+    // goes through one
+    v.part = nullptr;
+    if (im2col || v.splits > 1 || v.off_w % 4) {
+      v.part = partial_range(c, v.off_w, im2col ? (int64_t)v.cout * 27 : per, per, v.splits);
+      if (!v.part) return fail(c, GCPSL_E_NOMEM, "device allocation failed");
+    }
     const uint32_t wa[5] = {64, (uint32_t)v.wout, (uint32_t)v.whb, (uint32_t)v.wbb, 1};
     if (im2col) {
       const uint32_t wa0[5] = {(uint32_t)v.cout, (uint32_t)v.wout, (uint32_t)v.whb, 1, 1};
@@ -392,7 +396,6 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
     if ((st = setup(b.c2, false)) != GCPSL_OK) return st;
     if (b.sc && (st = setup(b.cs, false)) != GCPSL_OK) return st;
   }
-  DALLOC(c->d_partial, sizeof(float) * (size_t)partial_max);
   return GCPSL_OK;
 }
 
@@ -427,15 +430,14 @@ gcpsl_status conv_fwd(gcpsl_ctx* c, const RnConv& v, bool im2col) {
 
 gcpsl_status conv_wgrad(gcpsl_ctx* c, const RnConv& v) {
   WgradTcArgs w{v.hout, v.wout, c->B, v.cout, v.cin, v.whb, v.wbb, v.kb_total, v.kb_per_split,
-                v.splits, c->d_partial, c->d_err};
+                v.splits, v.part, c->d_err};
   w.taps = v.k * v.k;
   w.bias = 0;
   w.stride = v.stride;
   w.pad = v.k / 2;
-  const int64_t per = (int64_t)v.cout * v.k * v.k * v.cin;
-  // few splits reduce inside a cluster and write the gradient directly
-  const bool direct = v.splits <= kWgradClusterMax && v.off_w % 4 == 0;
-  if (direct) {
+  // a single split writes the gradient directly; several write the layer's
+  // partials, which the update sums
+  if (!v.part) {
     w.out = c->d_grad + v.off_w;
     w.out_rs = c->P_pad;
   }
@@ -443,9 +445,6 @@ gcpsl_status conv_wgrad(gcpsl_ctx* c, const RnConv& v) {
     LAUNCH(kWgradName[v.stage], launch_wgrad_halo(c->stream, v.wA, v.wH, w, c->C));
   else
     LAUNCH(kWgradName[v.stage], launch_wgrad_tc(c->stream, v.wA, v.wB, w, v.bn_w, c->C));
-  if (!direct)
-    LAUNCH("rn_wgrad_reduce", launch_wgrad_reduce(c->stream, c->d_partial, c->d_grad + v.off_w,
-                                                  c->P_pad, v.splits, per, c->C));
   return GCPSL_OK;
 }
 
@@ -579,12 +578,10 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
   {
     const RnConv& v = r.stem;
     WgradTcArgs w{v.hout, v.wout, B, v.cout, 3, v.whb, v.wbb, v.kb_total, v.kb_per_split, v.splits,
-                  c->d_partial, c->d_err};
+                  v.part, c->d_err};
+    // weights only: the update skips the ones column's sums (a bias
+    // gradient, not a parameter here)
     LAUNCH(kWgradName[0], launch_wgrad0_tc(s, v.wA, v.wB, w, C));
-    // weights only: the ones column's sums (a bias gradient) are not a parameter here
-    LAUNCH("rn_wgrad_reduce", launch_wgrad_reduce(s, c->d_partial, c->d_grad + v.off_w, P,
-                                                  v.splits, (int64_t)v.cout * 27 + v.cout, C,
-                                                  (int64_t)v.cout * 27));
   }
 #undef RN
   return GCPSL_OK;

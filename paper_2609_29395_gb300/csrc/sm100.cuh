@@ -178,35 +178,6 @@ __device__ __forceinline__ void tmem_ld_wait() {
 }
 
 // ---------------------------------------------------------------------------
-// Thread-block clusters: barrier over every thread of the cluster (release /
-// acquire orders shared-memory writes before the peers' reads), and loads
-// from a peer CTA's shared memory at the same offset as a local address.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
-               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ uint32_t peer_smem(uint32_t saddr, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
-  return r;
-}
-// (no memory clobber: several loads can be in flight before their first use;
-// callers order them after a cluster_sync, whose asm is volatile with one)
-__device__ __forceinline__ float4 ld_peer_f4(uint32_t caddr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(caddr));
-  return v;
-}
-
-// ---------------------------------------------------------------------------
 // Descriptors
 // ---------------------------------------------------------------------------
 // Swizzle modes of the shared-memory descriptor (bits 61-63).
