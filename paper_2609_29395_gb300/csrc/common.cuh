@@ -284,6 +284,21 @@ cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float2* s
 cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* kk, int gn,
                                   const bf16* d, const bf16* mask, bf16* out, int C, int B, int HW,
                                   int ch);
+// GroupNorm (32 groups) of one example per block, statistics and apply in
+// one launch: forward out = relu?(norm(y) + res) (res nullable), writing the
+// per-set mean / rstd; backward dy from d (times [mask > 0], kept in dz_out
+// when set) with the per-(example, channel) sums for dgamma / dbeta, which
+// launch_norm_finalize_bwd_channels then reduces over the batch.
+cudaError_t launch_gn_fused_fwd(cudaStream_t s, const bf16* y, const bf16* res,
+                                const float* gamma, const float* beta, int64_t g_rs, float* mean,
+                                float* rstd, bf16* out, int C, int B, int HW, int ch, int relu,
+                                int* err);
+cudaError_t launch_gn_fused_bwd(cudaStream_t s, const bf16* y, const bf16* d, const bf16* mask,
+                                bf16* dz_out, const float* gamma, int64_t g_rs, const float* mean,
+                                const float* rstd, float* sums, bf16* out, int C, int B, int HW,
+                                int ch, int* err);
+cudaError_t launch_norm_finalize_bwd_channels(cudaStream_t s, const float* sums, float* dgamma,
+                                              float* dbeta, int64_t d_rs, int C, int B, int ch);
 cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch);
 
 // optim.cu

@@ -15,6 +15,7 @@
 // per-channel affine form), then an elementwise apply.  Every sum has a fixed
 // order, so results do not depend on C or on launch geometry.
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace gcpsl {
 
@@ -354,6 +355,188 @@ k_norm_apply(const bf16* __restrict__ y, const void* __restrict__ aff, int aff_g
   }
 }
 
+// GroupNorm of one example in one kernel: a GroupNorm set (example, group)
+// never leaves its example, so one block per (replica, example) computes the
+// statistics and applies them, with the example's tensor (y forward, dz
+// backward; HW x ch bf16 <= 128 KB) staged in shared memory between the two
+// passes: one block per SM, 512 threads.  The staged tensor (y, or d) comes
+// in by one bulk copy.
+//   FWD: per-channel fp32 sums (pixels in lane order, lanes combined by a
+//        fixed shuffle tree and then in warp order), per group mean / rstd
+//        in fp64 (written for the backward), then
+//        out = relu?(gamma x_hat + beta + res).
+//   BWD: dz = d [mask > 0] (kept in dz_out when set), per-channel S1 = sum
+//        dz and S2 = sum dz x_hat (written to sums for dgamma / dbeta), per
+//        group m1, m2 and the affine form, then dy = k1 dz + k2 y + k3.
+// Threads: V = ch / 8 channel vectors x L pixel lanes (thread = l V + v).
+constexpr int kGnThreads = 512, kGnStageBytes = 128 * 1024;
+template <bool BWD>
+__global__ void __launch_bounds__(kGnThreads, 1)
+k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* __restrict__ mask,
+           const bf16* __restrict__ res, const float* __restrict__ gamma,
+           const float* __restrict__ beta, int64_t g_rs, float* __restrict__ mean,
+           float* __restrict__ rstd, float* __restrict__ sums, bf16* __restrict__ dz_out,
+           bf16* __restrict__ out, int B, int HW, int ch, int relu, int* err) {
+  extern __shared__ uint4 gsm4[];
+  __shared__ uint64_t bar;
+  uint8_t* stage = reinterpret_cast<uint8_t*>(gsm4);             // HW x ch bf16
+  float* red = reinterpret_cast<float*>(stage + kGnStageBytes);  // [warps][V][16]
+  const int V = ch / 8, L = kGnThreads / V;
+  const int nw = kGnThreads / 32;
+  float* csum = red + nw * V * 16;                               // [ch][2]
+  float4* aff = reinterpret_cast<float4*>(csum + 2 * ch);        // [ch]
+  const int64_t cb = blockIdx.x;                     // c * B + b
+  if (threadIdx.x == 0) {
+    sm100::mbar_init(&bar, 1);
+    sm100::fence_mbar_init();
+  }
+  __syncthreads();
+  pdl_wait();
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    const uint32_t bytes = (uint32_t)(HW * ch * 2);
+    sm100::mbar_arrive_expect_tx(&bar, bytes);
+    sm100::bulk_load(stage, (BWD ? d : y) + cb * HW * ch, bytes, &bar);
+  }
+  const int c = (int)(cb / B);
+  const int v = threadIdx.x % V, l = threadIdx.x / V;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int cpg = ch / 32;
+  const int64_t base = cb * HW * ch + v * 8;
+  const float* gm = gamma + (int64_t)c * g_rs;
+  float mu[8], rs[8];
+  if (BWD) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int64_t set = cb * 32 + (v * 8 + i) / cpg;
+      mu[i] = mean[set];
+      rs[i] = rstd[set];
+    }
+  }
+  if (!sm100::mbar_wait(&bar, 0) && threadIdx.x == 0) atomicOr(err, 64);
+  // pass 1: per-lane channel sums; the backward turns the staged d into dz
+  float s1[8] = {0, 0, 0, 0, 0, 0, 0, 0}, s2[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll 4
+  for (int p = l; p < HW; p += L) {
+    const int64_t o = base + (int64_t)p * ch;
+    uint4* st = reinterpret_cast<uint4*>(stage + ((int64_t)p * ch + v * 8) * 2);
+    float a[8];
+    if (!BWD) {
+      unpack8(*st, a);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { s1[i] += a[i]; s2[i] = fmaf(a[i], a[i], s2[i]); }
+    } else {
+      unpack8(*st, a);
+      if (mask) {
+        float m[8];
+        unpack8(*reinterpret_cast<const uint4*>(mask + o), m);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a[i] = m[i] > 0.f ? a[i] : 0.f;
+      }
+      const uint4 dzr = pack8(a);
+      *st = dzr;
+      if (dz_out) *reinterpret_cast<uint4*>(dz_out + o) = dzr;
+      unpack8(dzr, a);                                 // the stored (bf16) dz
+      float yy[8];
+      unpack8(*reinterpret_cast<const uint4*>(y + o), yy);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        s1[i] += a[i];
+        s2[i] = fmaf(a[i], (yy[i] - mu[i]) * rs[i], s2[i]);
+      }
+    }
+  }
+  // lanes of a warp with the same v (32 / V of them) by a fixed xor tree,
+  // then the warps in order
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    for (int o = 16; o >= V; o >>= 1) {
+      s1[i] += __shfl_xor_sync(0xffffffffu, s1[i], o);
+      s2[i] += __shfl_xor_sync(0xffffffffu, s2[i], o);
+    }
+  }
+  if (lane < V) {
+    float* mine = red + ((int64_t)warp * V + v) * 16;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { mine[i] = s1[i]; mine[8 + i] = s2[i]; }
+  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < V * 16; q += kGnThreads) {
+    const int vv = q / 16, k = q % 16;
+    float t = 0.f;
+    for (int w = 0; w < nw; ++w) t += red[((int64_t)w * V + vv) * 16 + k];
+    const int chn = vv * 8 + (k & 7);
+    csum[chn * 2 + (k >> 3)] = t;
+    if (BWD) sums[(cb * ch + chn) * 2 + (k >> 3)] = t;
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int g = threadIdx.x;
+    const double n = (double)cpg * HW;
+    if (!BWD) {
+      double a = 0.0, q2 = 0.0;
+      for (int k = 0; k < cpg; ++k) { a += csum[(g * cpg + k) * 2]; q2 += csum[(g * cpg + k) * 2 + 1]; }
+      const double m = a / n;
+      double var = q2 / n - m * m;
+      var = var > 0.0 ? var : 0.0;
+      const double r = 1.0 / sqrt(var + kEps);
+      mean[cb * 32 + g] = (float)m;
+      rstd[cb * 32 + g] = (float)r;
+      const float* bt = beta + (int64_t)c * g_rs;
+      for (int k = 0; k < cpg; ++k) {
+        const int chn = g * cpg + k;
+        const float sc = (float)((double)gm[chn] * r);
+        aff[chn] = make_float4(sc, (float)((double)bt[chn] - m * sc), 0.f, 0.f);
+      }
+    } else {
+      double a = 0.0, b2 = 0.0;
+      for (int k = 0; k < cpg; ++k) {
+        const int chn = g * cpg + k;
+        a += (double)gm[chn] * csum[chn * 2];
+        b2 += (double)gm[chn] * csum[chn * 2 + 1];
+      }
+      const double m1 = a / n, m2 = b2 / n;
+      const double m = mean[cb * 32 + g], r = rstd[cb * 32 + g];
+      for (int k = 0; k < cpg; ++k) {
+        const int chn = g * cpg + k;
+        aff[chn] = make_float4((float)(gm[chn] * r), (float)(-r * r * m2),
+                               (float)(r * r * m2 * m - r * m1), 0.f);
+      }
+    }
+  }
+  __syncthreads();
+  // pass 2 from the staged tensor
+  float k1[8], k2[8], k3[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 q = aff[v * 8 + i];
+    k1[i] = q.x; k2[i] = q.y; k3[i] = q.z;
+  }
+#pragma unroll 4
+  for (int p = l; p < HW; p += L) {
+    const int64_t o = base + (int64_t)p * ch;
+    const uint4 sv = *reinterpret_cast<const uint4*>(stage + ((int64_t)p * ch + v * 8) * 2);
+    float o8[8];
+    if (!BWD) {
+      float yy[8], r8[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      unpack8(sv, yy);
+      if (res) unpack8(*reinterpret_cast<const uint4*>(res + o), r8);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float x = fmaf(yy[i], k1[i], k2[i]) + r8[i];
+        o8[i] = relu ? (x > 0.f ? x : 0.f) : x;
+      }
+    } else {
+      float dz[8], yy[8];
+      unpack8(sv, dz);
+      unpack8(*reinterpret_cast<const uint4*>(y + o), yy);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o8[i] = fmaf(k1[i], dz[i], fmaf(k2[i], yy[i], k3[i]));
+    }
+    *reinterpret_cast<uint4*>(out + o) = pack8(o8);
+  }
+}
+
 // h[c][b][ch] = mean over the HW pixels (fixed order), bf16
 __global__ void k_avgpool(const bf16* __restrict__ x, bf16* __restrict__ h, int CB, int HW,
                           int ch) {
@@ -423,6 +606,57 @@ cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* k
   return launch_k(k_norm_apply<true>, (unsigned)n, kThreads, 0, s, y, (const void*)kk, gn,
                   (const bf16*)nullptr, (const float2*)nullptr, 0, (const bf16*)nullptr, d, mask,
                   out, C, B, HW, ch, 0);
+}
+
+static size_t gn_smem(int ch) {
+  const int V = ch / 8;
+  return kGnStageBytes + sizeof(float) * ((size_t)(kGnThreads / 32) * V * 16 + 2 * ch) +
+         sizeof(float4) * ch;
+}
+
+template <bool BWD>
+static bool gn_attr() {
+  static bool done = false;
+  if (!done)
+    done = cudaFuncSetAttribute(k_gn_fused<BWD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)gn_smem(256)) == cudaSuccess;
+  return done;
+}
+
+static bool gn_shape_ok(int HW, int ch) {
+  // V = ch / 8 lanes of a warp share the xor tree: V divides 32
+  return ch % 32 == 0 && ch <= 256 && (int64_t)HW * ch * 2 <= kGnStageBytes;
+}
+
+cudaError_t launch_gn_fused_fwd(cudaStream_t s, const bf16* y, const bf16* res,
+                                const float* gamma, const float* beta, int64_t g_rs, float* mean,
+                                float* rstd, bf16* out, int C, int B, int HW, int ch, int relu,
+                                int* err) {
+  if (!gn_shape_ok(HW, ch) || !gn_attr<false>()) return cudaErrorInvalidValue;
+  return launch_k(k_gn_fused<false>, (unsigned)(C * B), kGnThreads, gn_smem(ch), s, y,
+                  (const bf16*)nullptr, (const bf16*)nullptr, res, gamma, beta, g_rs, mean, rstd,
+                  (float*)nullptr, (bf16*)nullptr, out, B, HW, ch, relu, err);
+}
+
+cudaError_t launch_gn_fused_bwd(cudaStream_t s, const bf16* y, const bf16* d, const bf16* mask,
+                                bf16* dz_out, const float* gamma, int64_t g_rs, const float* mean,
+                                const float* rstd, float* sums, bf16* out, int C, int B, int HW,
+                                int ch, int* err) {
+  if (!gn_shape_ok(HW, ch) || (dz_out && !mask) || !gn_attr<true>()) return cudaErrorInvalidValue;
+  return launch_k(k_gn_fused<true>, (unsigned)(C * B), kGnThreads, gn_smem(ch), s, y, d, mask,
+                  (const bf16*)nullptr, gamma, (const float*)nullptr, g_rs,
+                  const_cast<float*>(mean), const_cast<float*>(rstd), sums, dz_out, out, B, HW,
+                  ch, 0, err);
+}
+
+cudaError_t launch_norm_finalize_bwd_channels(cudaStream_t s, const float* sums, float* dgamma,
+                                              float* dbeta, int64_t d_rs, int C, int B, int ch) {
+  if (ch % 32) return cudaErrorInvalidValue;
+  // the channel blocks of k_norm_finalize_bwd only (gn = 1: no BatchNorm
+  // form; the GroupNorm sets are left to the caller)
+  return launch_k(k_norm_finalize_bwd, (unsigned)(C * (ch / 32)), 256, 0, s, sums,
+                  (const float*)nullptr, (int64_t)0, (const float*)nullptr, (const float*)nullptr,
+                  (float4*)nullptr, dgamma, dbeta, d_rs, C, B, 1, ch, 1);
 }
 
 cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch) {

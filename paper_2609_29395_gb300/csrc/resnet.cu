@@ -461,12 +461,32 @@ gcpsl_status norm_stats(gcpsl_ctx* c, const RnNorm& n, const bf16* y) {
   return GCPSL_OK;
 }
 
+// GroupNorm forward in one launch per layer: out = relu(norm(y) + res)
+gcpsl_status gn_fwd(gcpsl_ctx* c, const RnNorm& n, const bf16* y, const bf16* res, bf16* out) {
+  const float* th = c->d_theta;
+  LAUNCH("rn_norm_gn", launch_gn_fused_fwd(c->stream, y, res, th + n.off_g, th + n.off_b,
+                                           c->P_pad, n.mean, n.rstd, out, c->C, c->B, n.hw, n.ch,
+                                           1, c->d_err));
+  return GCPSL_OK;
+}
+
 // dy = N'(dz) for dz = d [mask > 0] (mask nullable); dz_out (nullable)
 // keeps dz; affine gradients go to the gradient store
 gcpsl_status norm_bwd(gcpsl_ctx* c, const RnNorm& n, const bf16* y, const bf16* d,
                       const bf16* mask, bf16* dz_out, bf16* dy) {
   RnState& r = *c->rn;
   const float* th = c->d_theta;
+  if (n.gn) {
+    // one example per block: sums, the per-set affine form and dy together;
+    // then dgamma / dbeta over the batch
+    LAUNCH("rn_norm_gn_bwd",
+           launch_gn_fused_bwd(c->stream, y, d, mask, dz_out, th + n.off_g, c->P_pad, n.mean,
+                               n.rstd, r.sums, dy, c->C, c->B, n.hw, n.ch, c->d_err));
+    LAUNCH("rn_norm_bwd_finalize",
+           launch_norm_finalize_bwd_channels(c->stream, r.sums, c->d_grad + n.off_g,
+                                             c->d_grad + n.off_b, c->P_pad, c->C, c->B, n.ch));
+    return GCPSL_OK;
+  }
   LAUNCH("rn_norm_bwd_sums", launch_norm_sums(c->stream, true, y, d, mask, n.mean, n.rstd,
                                               dz_out, r.sums, c->C, c->B, n.hw, n.ch, n.gn));
   LAUNCH("rn_norm_bwd_finalize",
@@ -493,15 +513,21 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
 
   // ---- forward ----
   RN(conv_fwd(c, r.stem, true));
-  RN(norm_stats(c, r.stem_n, r.ystem));
-  LAUNCH("rn_norm_apply", launch_norm_apply_fwd(s, r.ystem, r.stem_n.ss, 1, nullptr, nullptr,
-                                                nullptr, 0, r.astem, C, B, 1024, 64, 1));
+  RN(gn_fwd(c, r.stem_n, r.ystem, nullptr, r.astem));
   for (auto& b : r.blk) {
     RN(conv_fwd(c, b.c1, false));
-    RN(norm_stats(c, b.n1, b.y1));
-    LAUNCH("rn_norm_apply", launch_norm_apply_fwd(s, b.y1, b.n1.ss, b.n1.gn, nullptr, nullptr,
-                                                  nullptr, 0, b.a1, C, B, b.n1.hw, b.n1.ch, 1));
+    if (b.n1.gn) {
+      RN(gn_fwd(c, b.n1, b.y1, nullptr, b.a1));
+    } else {
+      RN(norm_stats(c, b.n1, b.y1));
+      LAUNCH("rn_norm_apply", launch_norm_apply_fwd(s, b.y1, b.n1.ss, 0, nullptr, nullptr,
+                                                    nullptr, 0, b.a1, C, B, b.n1.hw, b.n1.ch, 1));
+    }
     RN(conv_fwd(c, b.c2, false));
+    if (b.n2.gn && !b.sc) {
+      RN(gn_fwd(c, b.n2, b.y2, b.c1.x, b.out));       // + the identity shortcut
+      continue;
+    }
     RN(norm_stats(c, b.n2, b.y2));
     if (b.sc) {
       RN(conv_fwd(c, b.cs, false));
