@@ -103,15 +103,22 @@ def work_per_round_resnet(w):
         if stage > 0:
             add(f"rn_conv_dgrad.{name}", "tensor", f)
 
-    def norm(e, kind):
-        """HBM bytes of the norm kernels for one norm over E bf16 elements:
+    def norm(e, kind, gn):
+        """HBM bytes of the norm kernels for one norm over E bf16 elements.
+        GroupNorm (one launch per direction, the example staged on chip):
+        forward reads y (+ the residual) and writes out; backward reads d,
+        y (+ the ReLU output) and writes dy (+ dz when kept).  BatchNorm:
         forward sums read y; apply reads y (+ the residual or the shortcut's
         y) and writes out; backward sums read d, y (+ the ReLU output) and
         may write dz; backward apply reads y, dz (+ mask) and writes dy."""
         b = 2.0 * e
-        fwd_apply = {"n1": 2, "n2": 3, "stem": 2, "ns": 0}[kind]
-        bwd_sums = {"n1": 2, "n2": 4, "stem": 3, "ns": 2}[kind]
-        bwd_apply = {"n1": 3, "n2": 3, "stem": 4, "ns": 3}[kind]
+        if gn:
+            add("rn_norm_gn", "hbm", {"n1": 2, "n2": 3, "stem": 2}[kind] * b)
+            add("rn_norm_gn_bwd", "hbm", {"n1": 3, "n2": 5, "stem": 4}[kind] * b)
+            return
+        fwd_apply = {"n1": 2, "n2": 3, "ns": 0}[kind]
+        bwd_sums = {"n1": 2, "n2": 4, "ns": 2}[kind]
+        bwd_apply = {"n1": 3, "n2": 3, "ns": 3}[kind]
         add("rn_norm_sums", "hbm", b)
         if fwd_apply:
             add("rn_norm_apply", "hbm", fwd_apply * b)
@@ -119,7 +126,7 @@ def work_per_round_resnet(w):
         add("rn_norm_bwd_apply", "hbm", bwd_apply * b)
 
     conv(0, 3, 64, 3, 1, 32)
-    norm(C * B * 1024 * 64, "stem")
+    norm(C * B * 1024 * 64, "stem", True)
     cin, hw = 64, 32
     for st, (width, stride) in enumerate(synth.RESNET_STAGES):
         for j in range(2):
@@ -128,11 +135,12 @@ def work_per_round_resnet(w):
             e = C * B * ho * ho * width
             conv(st + 1, cin, width, 3, s_, hw)
             conv(st + 1, width, width, 3, 1, ho)
-            norm(e, "n1")
-            norm(e, "n2")
+            gn = st == 0                    # the client's stage 1 uses GroupNorm
+            norm(e, "n1", gn)
+            norm(e, "n2", gn)
             if s_ != 1 or cin != width:
                 conv(st + 1, cin, width, 1, s_, hw)
-                norm(e, "ns")
+                norm(e, "ns", gn)
             cin, hw = width, ho
     P = synth.num_params(w.arch, "client") + synth.num_params(w.arch, "server")
     work["sgd"] = ("hbm", C * P * (4 * 5 + 2))

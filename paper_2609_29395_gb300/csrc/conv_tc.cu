@@ -1688,11 +1688,13 @@ cudaError_t launch_conv_halo(cudaStream_t s, const CUtensorMap& a, const CUtenso
   return cudaErrorInvalidValue;
 }
 
-int wgrad_halo_rows(int cin) { return cin == 32 ? 3 : 1; }
+// one kernel row per tile: at most 3 x 64 + 32 accumulator columns, so two
+// CTAs share an SM and the partials stay few
+int wgrad_halo_rows(int) { return 1; }
 
 bool wgrad_halo_supported(int H, int W, int cin, int cout, int taps, int stride) {
-  // ND = 1 holds hb (W + 2) <= 72 halo rows: W = 16 or 32
-  const bool w_ok = cin == 32 ? (W == 16 || W == 32 || W == 64) : (W == 16 || W == 32);
+  // hb (W + 2) <= 72 halo rows: W = 16 or 32
+  const bool w_ok = W == 16 || W == 32;
   return taps == 9 && stride == 1 && w_ok && H % (64 / W) == 0 &&
          (cin == 32 || cin % 64 == 0) && (cout == 64 || cout % 128 == 0);
 }
@@ -1729,8 +1731,8 @@ cudaError_t launch_wgrad_halo(cudaStream_t s, const CUtensorMap& g, const CUtens
   const int tiles = wgrad_halo_tiles(p.cin, p.cout);
   const bool m64 = p.cout % 128 != 0;
   if (p.cin == 32)
-    return m64 ? launch_wgrad_halo_inst<32, 64, 3>(s, g, x, p, C, tiles)
-               : launch_wgrad_halo_inst<32, 128, 3>(s, g, x, p, C, tiles);
+    return m64 ? launch_wgrad_halo_inst<32, 64, 1>(s, g, x, p, C, tiles)
+               : launch_wgrad_halo_inst<32, 128, 1>(s, g, x, p, C, tiles);
   return m64 ? launch_wgrad_halo_inst<64, 64, 1>(s, g, x, p, C, tiles)
              : launch_wgrad_halo_inst<64, 128, 1>(s, g, x, p, C, tiles);
 }
