@@ -53,7 +53,7 @@ NCU_TRAFFIC = {
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="splitcnn_c4")
@@ -200,7 +200,10 @@ def kernel_source_hash(kind):
     src = {"conv_fwd": "conv_simt.cu", "conv_dgrad": "conv_simt.cu", "conv_wgrad": "conv_simt.cu",
            "conv_fwd_tc": "conv_tc.cu", "conv_dgrad_tc": "conv_tc.cu",
            "conv_wgrad_tc": "conv_tc.cu", "relu_pool_bwd": "conv_simt.cu",
-           "sgd": "optim.cu", "fuse": "optim.cu"}.get(base)
+           "rn_conv_fwd": "conv_tc.cu", "rn_conv_dgrad": "conv_tc.cu",
+           "rn_conv_wgrad": "conv_tc.cu", "rn_norm_gn": "norm.cu", "rn_norm_gn_bwd": "norm.cu",
+           "rn_norm_sums": "norm.cu", "rn_norm_apply": "norm.cu", "rn_norm_bwd_sums": "norm.cu",
+           "rn_norm_bwd_apply": "norm.cu", "sgd": "optim.cu", "fuse": "optim.cu"}.get(base)
     if not src:
         return None
     p = os.path.join(ROOT, "paper_2609_29395_gb300", "csrc", src)
@@ -221,7 +224,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={q}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
         return self
