@@ -1051,11 +1051,13 @@ k_wgrad_tc(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
 
 // k_wgrad_halo: 3x3 stride-1 layers from halo tiles.
 //
-// Per K block (64 output pixels: hb rows x W columns of one image) the TMA
-// warp loads the g tile and ONE box of x around the block: (W + 2) columns
-// x (hb + 2) rows (ND = 3: all three kernel rows dy per tile) or hb rows
-// shifted by dy (ND = 1: one kernel row per tile).  For a K step of 16
-// pixels (within one image row) and a kernel row dy, the three taps dx =
+// Per K block (64 output pixels: hb rows x W columns of one image, W = 8,
+// 16 or 32) the TMA warp loads the g tile and ONE box of x around the
+// block: (W + 2) columns x (hb + 2) rows (ND = 3: all three kernel rows dy
+// per tile) or hb rows shifted by dy (ND = 1: one kernel row per tile; the
+// instantiated form).  For a K step of 16
+// pixels (two 8-pixel groups: in one image row, or for W = 8 in two rows,
+// one halo row apart) and a kernel row dy, the three taps dx =
 // -1, 0, 1 are one MN-major B operand of N = 3 CB: its N blocks of CB
 // channels start one pixel row apart (LBO = row bytes), so block j reads
 // the x rows of block 0 shifted by j pixels.  A K step is ND MMAs of
@@ -1065,8 +1067,8 @@ template <int CB, int MT, int ND>
 struct WhCfg {
   static constexpr int ROWB = CB * 2;
   static constexpr int A_BYTES = MT * 64 * 2;               // MT co x 64 pixels
-  // halo rows at most: (hb + 2)(W + 2) <= 3 * 66 (ND = 3), hb (W + 2) <= 4 * 18 (ND = 1)
-  static constexpr int HMAX = ND == 3 ? 3 * 66 : 4 * 18;
+  // halo rows at most: (hb + 2)(W + 2) <= 3 * 66 (ND = 3), hb (W + 2) <= 8 * 10 (ND = 1)
+  static constexpr int HMAX = ND == 3 ? 3 * 66 : 8 * 10;
   static constexpr int H_BYTES = (HMAX * ROWB + 1023) / 1024 * 1024;
   static constexpr int STAGE = A_BYTES + H_BYTES;
   static constexpr int NT = ND * 3 * CB;                     // tap columns
@@ -1169,6 +1171,7 @@ k_wgrad_halo(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUt
       constexpr uint32_t idesc_b = idesc_bf16(MT, 32, 1, 1);
       constexpr uint32_t a_lbo = 64 * 64 * 2;                 // the two 64-co blocks (MT = 128)
       const uint64_t ones_desc = smem_desc(smem_u32(ones), 64 * 16, 8 * 64, SWZ_64);
+      const uint32_t b_sbo = (uint32_t)((p.W >= 16 ? 8 : HW2) * Cfg::ROWB);
       int it = 0, tl = 0;
       bool ok = true;
       for (int t = t_begin; t < t_end && ok; ++t, ++tl) {
@@ -1190,12 +1193,14 @@ k_wgrad_halo(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUt
           const uint32_t a = smem_u32(sm + s * Cfg::STAGE), hb0 = a + Cfg::A_BYTES;
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
+            // a K step of 16 pixels: two 8-pixel groups, consecutive in one
+            // image row (W >= 16) or the same columns of two rows (W = 8)
             const int y = (16 * k) / p.W, x0 = (16 * k) % p.W;
             const uint64_t ad = smem_desc(a + k * 16 * 128, a_lbo, 1024, SWZ_128);
 #pragma unroll
             for (int dd = 0; dd < ND; ++dd) {
               const uint32_t start = hb0 + (uint32_t)(((y + dd) * HW2 + x0) * Cfg::ROWB);
-              mma_f16(d + dd * 3 * CB, ad, smem_desc(start, Cfg::ROWB, 8 * Cfg::ROWB, swz), idesc,
+              mma_f16(d + dd * 3 * CB, ad, smem_desc(start, Cfg::ROWB, b_sbo, swz), idesc,
                       (i | k) != 0);
             }
             if (bias) mma_f16(d + NT, ad, ones_desc, idesc_b, (i | k) != 0);
@@ -1693,8 +1698,8 @@ cudaError_t launch_conv_halo(cudaStream_t s, const CUtensorMap& a, const CUtenso
 int wgrad_halo_rows(int) { return 1; }
 
 bool wgrad_halo_supported(int H, int W, int cin, int cout, int taps, int stride) {
-  // hb (W + 2) <= 72 halo rows: W = 16 or 32
-  const bool w_ok = W == 16 || W == 32;
+  // hb (W + 2) <= 80 halo rows: W = 8, 16 or 32
+  const bool w_ok = W == 8 || W == 16 || W == 32;
   return taps == 9 && stride == 1 && w_ok && H % (64 / W) == 0 &&
          (cin == 32 || cin % 64 == 0) && (cout == 64 || cout % 128 == 0);
 }
