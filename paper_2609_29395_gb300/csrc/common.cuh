@@ -311,6 +311,10 @@ struct SgdSeg {
   const float* src;
   int64_t off, count, per, total;
   int splits;
+  // the input layer's weights: also written packed as w0p[c][co][32]
+  // (column k = tap * 3 + ci < 27) for its one-tap forward; else null
+  bf16* w0p;
+  int w0_cout;
 };
 constexpr int kSgdThreads = 256, kSgdPer = 2;
 // quads (4 parameters) per update block of a segment with `splits` sources:

@@ -202,7 +202,11 @@ gcpsl_status gcpsl::build_sgd_segments(gcpsl_ctx* c) {
     for (int64_t e = 0; e < quads; e += chunk)
       blocks.push_back(make_int4((int)segs.size(), (int)e, (int)std::min<int64_t>(chunk, quads - e),
                                  0));
-    segs.push_back({src, off, count, per, (int64_t)c->C * count, splits});
+    // the input layer's weights also go packed to w0p (bf16 mode)
+    const bool w0 = c->d_w0p && off == c->w0_off;
+    segs.push_back({src, off, count, per, (int64_t)c->C * count, splits, w0 ? c->d_w0p : nullptr,
+                    w0 ? c->w0_cout : 0});
+    if (w0) c->sgd_packs_w0 = true;
   };
   for (const auto& q : r) {
     if (q.off < at || q.off + q.count > c->P_pad)
@@ -272,7 +276,8 @@ gcpsl_status enqueue_sgd(gcpsl_ctx* c) {
     LAUNCH("sgd", launch_sgd(c->stream, c->d_theta, c->d_mom, c->d_grad, c->d_shadow,
                              (int64_t)c->C * c->P_pad, c->desc.lr, c->desc.momentum,
                              c->desc.weight_decay, c->desc.nesterov, c->d_t));
-  return refresh_derived(c);
+  // the segment update also rewrites the packed input-layer weights
+  return c->sgd_packs_w0 ? GCPSL_OK : refresh_derived(c);
 }
 
 

@@ -173,6 +173,7 @@ struct gcpsl_ctx {
   gcpsl::SgdSeg* d_sgd_segs = nullptr;
   int4* d_sgd_blocks = nullptr;    // per update block: {segment, first element, count, 0}
   int n_sgd_blocks = 0;
+  bool sgd_packs_w0 = false;       // the update also writes d_w0p
   // CUDA-core weight+bias gradient partials of the layers not on the tensor
   // cores (tiles of tr image rows, tiles_per_split tiles per block)
   struct RedLayer { int tr, splits, tiles_per_split; } red[4];

@@ -108,6 +108,21 @@ k_sgd_seg(float4* __restrict__ theta, float4* __restrict__ mom, uint2* __restric
       shadow[at[k]] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
                                  *reinterpret_cast<const uint32_t*>(&hi));
     }
+    if (sq.w0p) {
+      // element j of the input layer's weights [co][27] -> w0p[c][co][j % 27]
+      const uint32_t local = (uint32_t)bk.y + (uint32_t)(k * kSgdThreads) + threadIdx.x;
+      const uint32_t c = local / cnt4, j0 = (local - c * cnt4) * 4;
+      const uint32_t n27 = (uint32_t)sq.w0_cout * 27;
+      const float t4[4] = {th.x, th.y, th.z, th.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t j = j0 + e;
+        if (j < n27) {
+          const uint32_t co = j / 27;
+          sq.w0p[((int64_t)c * sq.w0_cout + co) * 32 + (j - co * 27)] = __float2bfloat16_rn(t4[e]);
+        }
+      }
+    }
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) *d_t += 1;
 }
