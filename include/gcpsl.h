@@ -64,7 +64,15 @@ enum { GCPSL_CUT_ACT = 0, GCPSL_CUT_GRAD = 1 };
  *    C-cluster context exactly).
  *  data_on_host: 0 = images copied to device memory at init; 1 = images stay
  *    in pinned, device-mapped host memory owned by the context and each round
- *    gathers its B sampled images per cluster from there.               */
+ *    gathers its B sampled images per cluster from there.
+ *  augment: 0 = the sampled images as stored; 1 = the training augmentation
+ *    of Section V-A (random crop from the 4-pixel zero-padded image, then a
+ *    random horizontal flip), drawn per round, cluster and batch position
+ *    from Philox4x32-10 with counter (b, t, cluster_id_base + n, 1) and key
+ *    `seed`: dy = (o0 * 9) >> 32, dx = (o1 * 9) >> 32, flip = o2 & 1, and
+ *    out[ch][y][x] = img[ch][y + dy - 4][x' + dx - 4], x' = flip ? 31 - x : x,
+ *    0 outside the image.  (The synthetic images are N(0,1) already, so the
+ *    dataset normalisation of Section V-A is the identity.)              */
 typedef struct {
   int arch;
   int operand_dtype;
@@ -73,6 +81,7 @@ typedef struct {
   float label_smoothing;
   int cluster_id_base;
   int data_on_host;
+  int augment;
 } gcpsl_model_desc;
 
 /* Training data of all K clients (Section III-A: client k owns D_k).

@@ -66,6 +66,12 @@ def _declare(L):
                            ct.c_double, ct.c_int, ct.c_int, i32p, ct.c_int, ct.c_int, ct.c_uint64,
                            ct.c_int, f32p, i32p, i32p, ct.c_int64, f32p, _p(ct.c_void_p)]
     L.orc_destroy.argtypes = [ct.c_void_p]
+    L.orc_augment_params.argtypes = [ct.c_uint64, ct.c_uint32, ct.c_uint32, ct.c_uint32, i32p]
+    L.orc_augment_params.restype = None
+    L.orc_augment_image.argtypes = [f32p, ct.c_int, ct.c_int, ct.c_int, f64p]
+    L.orc_augment_image.restype = None
+    L.orc_set_augment.argtypes = [ct.c_void_p, ct.c_int]
+    L.orc_set_augment.restype = None
     L.orc_step.argtypes = [ct.c_void_p]
     L.orc_fuse.argtypes = [ct.c_void_p]
     L.orc_get_params.argtypes = [ct.c_void_p, ct.c_int, ct.c_int, f64p]
@@ -129,6 +135,23 @@ def sample_round(perm, s: int, B: int, owner, K: int):
     act = lib().orc_sample_round(_ptr(perm, ct.c_int32), s, B, _ptr(owner, ct.c_int32), K,
                                  _ptr(idx, ct.c_int32), _ptr(counts, ct.c_int32))
     return idx, counts, act
+
+
+def augment_params(seed: int, t: int, cluster: int, pos: int):
+    """(dy, dx, flip) of the sampled image at batch position `pos` of
+    cluster `cluster` in round `t` (Section V-A crop + flip; Philox draw)."""
+    out = np.zeros(3, dtype=np.int32)
+    lib().orc_augment_params(seed, t, cluster, pos, _ptr(out, ct.c_int32))
+    return int(out[0]), int(out[1]), int(out[2])
+
+
+def augment_image(img, dy: int, dx: int, flip: int):
+    """The crop at (dy, dx) of the 4-pixel zero-padded CHW image, mirrored
+    when flip (fp64)."""
+    src = np.ascontiguousarray(img, dtype=np.float32).reshape(3, 32, 32)
+    out = np.zeros((3, 32, 32))
+    lib().orc_augment_image(_ptr(src, ct.c_float), dy, dx, flip, _ptr(out, ct.c_double))
+    return out
 
 
 def num_params(arch: int, segment: int) -> int:
@@ -251,7 +274,7 @@ class Oracle:
 
     def __init__(self, arch, K, C, assignment, B, F, seed, images, labels, owner, init_params,
                  lr=0.05, momentum=0.0, weight_decay=0.0, nesterov=False, label_smoothing=0.0,
-                 bf16=False, cluster_base=0):
+                 bf16=False, cluster_base=0, augment=False):
         self.arch, self.K, self.C, self.B = arch, K, C, B
         # the context reads the images in place: keep them alive here
         self._images = np.ascontiguousarray(images, dtype=np.float32)
@@ -268,6 +291,7 @@ class Oracle:
         if rc:
             raise ValueError(f"oracle init failed: {rc}")
         self._h = h
+        lib().orc_set_augment(h, int(augment))
         self.P_client = num_params(arch, 0)
         self.P_server = num_params(arch, 1)
 

@@ -549,6 +549,7 @@ typedef struct {
   double tie_tol;                             /* see relu_pool_fwd */
   uint8_t* cand[4];                           /* [C][B][cout][Ho][Wo] of the last round */
   int32_t* ties;                              /* [C][B] ambiguous windows per example */
+  int augment;                                /* crop + flip of the sampled images */
 } orc_ctx;
 
 void orc_destroy(orc_ctx* c);
@@ -688,6 +689,56 @@ static void sgd(orc_ctx* c, int k) {
   }
 }
 
+/* Training augmentation (Section V-A: random crops and horizontal flips),
+ * as torchvision's RandomCrop(32, padding=4) followed by
+ * RandomHorizontalFlip, with the random draws taken from Philox4x32-10:
+ * counter (position in the batch, round, cluster id, 1), key = seed;
+ * dy = floor(o0 * 9 / 2^32), dx = floor(o1 * 9 / 2^32) (crop offsets into the
+ * 40 x 40 zero-padded image), flip = o2 mod 2.                            */
+void orc_augment_params(uint64_t seed, uint32_t t, uint32_t cluster, uint32_t pos,
+                        int32_t out[3]) {
+  const uint32_t ctr[4] = {pos, t, cluster, 1u};
+  const uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  uint32_t o[4];
+  orc_philox4x32_10(ctr, key, o);
+  out[0] = (int32_t)(((uint64_t)o[0] * 9u) >> 32);
+  out[1] = (int32_t)(((uint64_t)o[1] * 9u) >> 32);
+  out[2] = (int32_t)(o[2] & 1u);
+}
+
+/* dst[ch][y][x] (CHW, 3 x 32 x 32) = the crop of the zero-padded image at
+ * rows dy..dy+31, columns dx..dx+31, mirrored left-right when flip:
+ * padded[ch][Y][X] = src[ch][Y - 4][X - 4] inside the image, else 0.      */
+void orc_augment_image(const float* src, int dy, int dx, int flip, double* dst) {
+  for (int ch = 0; ch < 3; ++ch)
+    for (int y = 0; y < 32; ++y)
+      for (int x = 0; x < 32; ++x) {
+        const int cx = flip ? 31 - x : x;             /* column of the crop */
+        const int Y = y + dy, X = cx + dx;            /* in the padded image */
+        const int sy = Y - 4, sx = X - 4;
+        const int in = sy >= 0 && sy < 32 && sx >= 0 && sx < 32;
+        dst[(ch * 32 + y) * 32 + x] = in ? (double)src[(ch * 32 + sy) * 32 + sx] : 0.0;
+      }
+}
+
+void orc_set_augment(orc_ctx* c, int on) { c->augment = on != 0; }
+
+/* the batch's images of cluster k in round t (augmented when set) */
+static void batch_images(const orc_ctx* c, int k, const int32_t* idx, double* dst) {
+  for (int b = 0; b < c->B; ++b) {
+    const float* src = c->images_src + (int64_t)idx[b] * 3072;
+    double* d = dst + (int64_t)b * 3072;
+    if (c->augment) {
+      int32_t a[3];
+      orc_augment_params(c->seed, (uint32_t)c->t, (uint32_t)(c->cluster_base + k), (uint32_t)b,
+                         a);
+      orc_augment_image(src, a[0], a[1], a[2], d);
+    } else {
+      for (int i = 0; i < 3072; ++i) d[i] = (double)src[i];
+    }
+  }
+}
+
 /* One local round of every cluster, then fusion when (t+1) mod F == 0. */
 int orc_step(orc_ctx* c) {
   int B = c->B;
@@ -703,11 +754,8 @@ int orc_step(orc_ctx* c) {
     c->active[k] = orc_sample_round(c->perm[k], s, B, c->owner, c->K, idx,
                                     c->counts + (int64_t)k * c->K);
     if (c->resnet) {
-      for (int b = 0; b < B; ++b) {
-        const float* src = c->images_src + (int64_t)idx[b] * 3072;
-        for (int i = 0; i < 3072; ++i) c->xbuf[(int64_t)b * 3072 + i] = (double)src[i];
-        c->ybuf[b] = c->labels[idx[b]];
-      }
+      batch_images(c, k, idx, c->xbuf);
+      for (int b = 0; b < B; ++b) c->ybuf[b] = c->labels[idx[b]];
       int64_t P = c->o.p_total;
       const int64_t E = orn_mask_elems();
       int rc = orn_forward_backward_masks(
@@ -717,11 +765,8 @@ int orc_step(orc_ctx* c) {
       if (rc) return rc;
       continue;
     }
-    for (int b = 0; b < B; ++b) {
-      const float* src = c->images_src + (int64_t)idx[b] * 3072;
-      for (int i = 0; i < 3072; ++i) c->w.act[0][(int64_t)b * 3072 + i] = (double)src[i];
-      c->ybuf[b] = c->labels[idx[b]];
-    }
+    batch_images(c, k, idx, c->w.act[0]);
+    for (int b = 0; b < B; ++b) c->ybuf[b] = c->labels[idx[b]];
     int64_t P = c->o.p_total;
     int rc = fwd_bwd(&c->a, &c->o, c->bf16, c->ls, c->theta + k * P, B, c->ybuf, &c->w,
                      &c->loss[k], c->grad + k * P, c->tie_tol);

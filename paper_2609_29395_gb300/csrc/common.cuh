@@ -106,17 +106,32 @@ cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* of
                           const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
                           const int32_t* labels, int K, int B, int C, int32_t* idx,
                           int32_t* counts, int32_t* active, int32_t* y);
+// Training augmentation of the gathered images (Sec. V-A: random crops and
+// horizontal flips): sampled image b of cluster n in round t is cropped
+// from its 4-pixel zero-padded version at offset (dy, dx) in [0, 8]^2 and
+// then mirrored when flip = 1, i.e. out[ch][y][x] = img[ch][y + dy - 4]
+// [x' + dx - 4] with x' = flip ? 31 - x : x (0 outside).  With Philox4x32-10
+// (counter = (b, t, n', 1), key = seed), n' = cluster_base + n:
+// dy = (o0 * 9) >> 32, dx = (o1 * 9) >> 32, flip = o2 & 1.  Off: dy = dx = 4,
+// flip = 0 (the image itself).
+struct AugArgs {
+  int on;
+  uint32_t s0, s1;              // the seed's low and high words
+  const int64_t* d_t;           // the device round counter
+  int cluster_base, B;
+};
 // fp32: x0 = the sampled images, NHWC with 3 channels; bf16: x0 = the input
 // layer's im2col [CB][32][32][32] (27 tap x channel columns, a ones column
 // for the bias gradient, zero padding)
 template <typename T>
-cudaError_t launch_gather(cudaStream_t s, const float* images, const int32_t* idx, int CB, T* x0);
+cudaError_t launch_gather(cudaStream_t s, const float* images, const int32_t* idx, int CB, T* x0,
+                          const AugArgs& aug);
 template <>
 cudaError_t launch_gather<float>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
-                                 float* x0);
+                                 float* x0, const AugArgs& aug);
 template <>
 cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
-                                bf16* x0);
+                                bf16* x0, const AugArgs& aug);
 
 // conv_simt.cu
 template <typename T>

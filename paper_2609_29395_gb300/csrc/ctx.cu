@@ -262,7 +262,9 @@ gcpsl_status enqueue_sample(gcpsl_ctx* c, bool boundary) {
   LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_t, c->d_owner,
                                  c->d_labels, c->K, B, C, c->d_idx, c->d_counts, c->d_active,
                                  c->d_y));
-  LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, (T*)c->d_act[0]));
+  const AugArgs aug{c->desc.augment, (uint32_t)c->seed, (uint32_t)(c->seed >> 32), c->d_t,
+                    c->desc.cluster_id_base, B};
+  LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, (T*)c->d_act[0], aug));
   return GCPSL_OK;
 }
 
@@ -854,6 +856,8 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
     return fail(nullptr, GCPSL_E_INVAL, "num_classes must be 10");
   if (desc->operand_dtype != GCPSL_F32 && desc->operand_dtype != GCPSL_BF16)
     return fail(nullptr, GCPSL_E_INVAL, "unknown operand_dtype %d", desc->operand_dtype);
+  if (desc->augment != 0 && desc->augment != 1)
+    return fail(nullptr, GCPSL_E_INVAL, "augment must be 0 or 1");
   if (!(desc->lr >= 0.f) || !(desc->label_smoothing >= 0.f && desc->label_smoothing < 1.f))
     return fail(nullptr, GCPSL_E_INVAL, "bad lr or label_smoothing");
   ArchSpec a;

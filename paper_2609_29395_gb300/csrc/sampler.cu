@@ -1,6 +1,7 @@
 // GPSL global sampling inside each cluster (Eq. 1; epoch rule of
 // Section III-A) and the gather of the sampled images (with bf16 operands,
-// straight into the input layer's im2col).
+// straight into the input layer's im2col), optionally with the crop and
+// flip augmentation of Section V-A (see AugArgs).
 //
 // Epoch permutation of cluster n: every example id j of the cluster gets the
 // 64-bit key (o0 << 32 | o1) of Philox4x32-10(counter = (j, epoch, n', 0),
@@ -107,19 +108,37 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
 }
 
 // fp32 storage: x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w] (3 channels).
+// crop offsets and flip of sampled image cb = c * B + b (see AugArgs)
+__device__ __forceinline__ void aug_params(const AugArgs& a, int64_t cb, int& dy, int& dx,
+                                           int& flip) {
+  dy = dx = 4;
+  flip = 0;
+  if (!a.on) return;
+  const int c = (int)(cb / a.B), b = (int)(cb % a.B);
+  uint32_t ctr[4] = {(uint32_t)b, (uint32_t)*a.d_t, (uint32_t)(a.cluster_base + c), 1u};
+  philox4x32_10(ctr, a.s0, a.s1);
+  dy = (int)(((uint64_t)ctr[0] * 9u) >> 32);
+  dx = (int)(((uint64_t)ctr[1] * 9u) >> 32);
+  flip = (int)(ctr[2] & 1u);
+}
+
 __global__ void k_gather_f32(const float* __restrict__ images, const int32_t* __restrict__ idx,
-                             int CB, float* __restrict__ x0) {
+                             int CB, float* __restrict__ x0, const AugArgs aug) {
   pdl_wait();
   pdl_trigger();
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (int64_t)CB * 1024) return;
   const int64_t cb = i >> 10;
-  const int p = (int)(i & 1023);
-  const float* src = images + (int64_t)idx[cb] * 3072 + p;
+  const int p = (int)(i & 1023), y = p >> 5, x = p & 31;
+  int dy, dx, flip;
+  aug_params(aug, cb, dy, dx, flip);
+  const int sy = y + dy - 4, sx = (flip ? 31 - x : x) + dx - 4;
+  const bool in = sy >= 0 && sy < 32 && sx >= 0 && sx < 32;
+  const float* src = images + (int64_t)idx[cb] * 3072 + (in ? sy * 32 + sx : 0);
   float* dst = x0 + i * 3;
-  dst[0] = src[0];
-  dst[1] = src[1024];
-  dst[2] = src[2048];
+  dst[0] = in ? src[0] : 0.f;
+  dst[1] = in ? src[1024] : 0.f;
+  dst[2] = in ? src[2048] : 0.f;
 }
 
 // bf16 storage: the input layer's im2col, x0[c][b][y][x][32] with column
@@ -131,16 +150,22 @@ __global__ void k_gather_f32(const float* __restrict__ images, const int32_t* __
 constexpr int kIm2colThreads = 256;
 __global__ void __launch_bounds__(kIm2colThreads)
 k_gather_im2col(const float* __restrict__ images, const int32_t* __restrict__ idx,
-                bf16* __restrict__ x0) {
+                bf16* __restrict__ x0, const AugArgs aug) {
   __shared__ float tile[3][34][34];
   pdl_wait();
   pdl_trigger();
   const int64_t cb = blockIdx.x;
   const float* src = images + (int64_t)idx[cb] * 3072;
+  int dy, dx, flip;
+  aug_params(aug, cb, dy, dx, flip);
   for (int i = threadIdx.x; i < 3 * 34 * 34; i += kIm2colThreads) {
     const int ch = i / (34 * 34), yy = (i / 34) % 34, xx = i % 34;
-    const bool in = yy >= 1 && yy <= 32 && xx >= 1 && xx <= 32;
-    tile[ch][yy][xx] = in ? src[ch * 1024 + (yy - 1) * 32 + (xx - 1)] : 0.f;
+    // (yy - 1, xx - 1): the augmented image's pixel, zero around it
+    const int y = yy - 1, x = xx - 1;
+    const int sy = y + dy - 4, sx = (flip ? 31 - x : x) + dx - 4;
+    const bool in = y >= 0 && y < 32 && x >= 0 && x < 32 && sy >= 0 && sy < 32 && sx >= 0 &&
+                    sx < 32;
+    tile[ch][yy][xx] = in ? src[ch * 1024 + sy * 32 + sx] : 0.f;
   }
   __syncthreads();
   uint4* dst = reinterpret_cast<uint4*>(x0 + cb * 1024 * 32);
@@ -187,14 +212,15 @@ cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* of
 
 template <>
 cudaError_t launch_gather<float>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
-                                 float* x0) {
+                                 float* x0, const AugArgs& aug) {
   const int64_t n = (int64_t)CB * 1024;
-  return launch_k(k_gather_f32, (unsigned)((n + 255) / 256), 256, 0, s, images, idx, CB, x0);
+  return launch_k(k_gather_f32, (unsigned)((n + 255) / 256), 256, 0, s, images, idx, CB, x0,
+                  aug);
 }
 template <>
 cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
-                                bf16* x0) {
-  return launch_k(k_gather_im2col, (unsigned)CB, kIm2colThreads, 0, s, images, idx, x0);
+                                bf16* x0, const AugArgs& aug) {
+  return launch_k(k_gather_im2col, (unsigned)CB, kIm2colThreads, 0, s, images, idx, x0, aug);
 }
 
 }  // namespace gcpsl

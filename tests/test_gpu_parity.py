@@ -170,6 +170,34 @@ def test_splitcnn_bf16_rounds_with_fusion():
         check_round(gpu, orc, synth.ARCH_SPLIT_CNN)
 
 
+def test_augmented_rounds_bf16_and_fp32():
+    """The crop + flip augmentation of Section V-A fused into the gather (the
+    bf16 path's im2col gather and the fp32 path's gather): every round's
+    batch is the oracle's augmented batch, so the usual bars hold; and the
+    round differs from the unaugmented one."""
+    ds, assign, params = _splitcnn_small(C=4, n=4096)
+    kw = dict(lr=0.05, momentum=0.9, augment=True)
+    gpu, orc = pair(synth.ARCH_SPLIT_CNN, 32, 4, assign, 32, 2, ds, params, True, **kw)
+    for _ in range(3):
+        check_round(gpu, orc, synth.ARCH_SPLIT_CNN)
+    plain = pkg.Context(synth.ARCH_SPLIT_CNN, 32, 4, assign, 32, 2, 4, ds.images, ds.labels,
+                        ds.owner, params, lr=0.05, momentum=0.9)
+    aug = pkg.Context(synth.ARCH_SPLIT_CNN, 32, 4, assign, 32, 2, 4, ds.images, ds.labels,
+                      ds.owner, params, **kw)
+    plain.step()
+    aug.step()
+    assert (plain.sample()[0] == aug.sample()[0]).all()
+    assert not np.array_equal(plain.cut(pkg.binding.GCPSL_CUT_ACT), aug.cut(pkg.binding.GCPSL_CUT_ACT))
+    plain.close()
+    aug.close()
+    w = configs.WORKLOADS["tiny"]
+    ds, assign, params = configs.build_inputs(w)
+    gpu, orc = pair(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, ds, params, False,
+                    lr=w.lr, momentum=w.momentum, augment=True)
+    for _ in range(3):
+        check_round(gpu, orc, w.arch, tol=1e-3, loss_tol=1e-4, fwd_tol=1e-5)
+
+
 def test_ragged_batch_nesterov_wd_label_smoothing():
     """B = 24 (not a power of two), C = 6, Nesterov, weight decay, label
     smoothing."""

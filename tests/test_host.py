@@ -65,7 +65,7 @@ def test_init_rejects_bad_arguments(lib, case):
         kw["arch"] = 9
     with pytest.raises(binding.GcpslError) as e:
         if case == "bad_dtype":
-            desc = binding.gcpsl_model_desc(0, 7, 0.05, 0, 0, 0, 0, 0, 0)
+            desc = binding.gcpsl_model_desc(0, 7, 0.05, 0, 0, 0, 0, 0, 0, 0)
             ds_c = binding.gcpsl_dataset(binding._p(ds.images, ct.c_float),
                                          binding._p(ds.labels, ct.c_int32),
                                          binding._p(ds.owner, ct.c_int32), ds.images.shape[0], 10)

@@ -334,3 +334,66 @@ def test_init_rejects_bad_inputs():
     with pytest.raises(ValueError):   # assignment out of range
         oracle.Oracle(arch, K, 2, np.full(K, 2, np.int32), 8, 0, 4, ds.images, ds.labels,
                       ds.owner, blob)
+
+
+# --------------------------------------------------------------------------
+# Training augmentation (Section V-A: random crop + horizontal flip)
+# --------------------------------------------------------------------------
+def test_augment_image_is_padded_crop_then_flip():
+    """The oracle's augmentation equals numpy's zero-pad by 4, crop at
+    (dy, dx), then left-right mirror, for every offset and both flips."""
+    rng = np.random.default_rng(3)
+    img = rng.normal(size=(3, 32, 32)).astype(np.float32)
+    padded = np.pad(img.astype(np.float64), ((0, 0), (4, 4), (4, 4)))
+    for dy in range(9):
+        for dx in range(9):
+            for flip in (0, 1):
+                ref = padded[:, dy:dy + 32, dx:dx + 32]
+                if flip:
+                    ref = ref[:, :, ::-1]
+                got = oracle.augment_image(img, dy, dx, flip)
+                assert np.array_equal(got, ref), (dy, dx, flip)
+
+
+def test_augment_params_range_uniformity_and_stream():
+    """Offsets in [0, 8], flips in {0, 1}, each close to uniform (chi^2 over
+    many draws); draws differ between rounds, clusters and positions, and
+    equal the Philox definition (counter (pos, t, cluster, 1), key = seed)."""
+    seed = 0x1234ABCD5678
+    n = 9 * 800
+    draws = np.array([oracle.augment_params(seed, t, c, p)
+                      for t in range(20) for c in range(4) for p in range(n // 80)])
+    assert draws.shape[0] == n
+    assert draws[:, :2].min() == 0 and draws[:, :2].max() == 8
+    assert set(np.unique(draws[:, 2])) == {0, 1}
+    for col in (0, 1):
+        cnt = np.bincount(draws[:, col], minlength=9)
+        chi2 = ((cnt - n / 9) ** 2 / (n / 9)).sum()
+        assert chi2 < 30.0, (col, cnt)            # 8 dof: p(chi2 > 30) < 3e-4
+    assert abs(draws[:, 2].mean() - 0.5) < 0.03
+    o = [int(v) for v in oracle.philox4x32_10([5, 7, 3, 1], [seed & 0xFFFFFFFF, seed >> 32])]
+    assert oracle.augment_params(seed, 7, 3, 5) == ((o[0] * 9) >> 32, (o[1] * 9) >> 32, o[2] & 1)
+
+
+def test_oracle_round_uses_the_augmented_batch():
+    """With augmentation, a round's loss equals the forward pass on the
+    sampled images augmented with that round's draws (and differs from the
+    plain batch)."""
+    ds = synth.make_dataset(256, 10, 8, 0.5, balanced=False, seed_data=1, seed_split=2)
+    assign = clustering.random_clustering(8, 2, 3)
+    arch = synth.ARCH_TINY_CNN
+    params = synth.init_params(arch, seed=4).astype(np.float64)
+    B, seed = 16, 9
+    for aug in (True, False):
+        orc = oracle.Oracle(arch, 8, 2, assign, B, 0, seed, ds.images, ds.labels, ds.owner,
+                            params, augment=aug)
+        orc.step()
+        idx, _ = orc.sample()
+        loss, _ = orc.stats()
+        for m in range(2):
+            x = ds.images[idx[m]].astype(np.float64)
+            if aug:
+                x = np.stack([oracle.augment_image(ds.images[i], *oracle.augment_params(seed, 0, m, b))
+                              for b, i in enumerate(idx[m])])
+            ref = oracle.forward_backward(arch, params, x, ds.labels[idx[m]])[0]
+            assert abs(ref - loss[m]) < 1e-12 * max(1.0, abs(ref))
