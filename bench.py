@@ -327,7 +327,7 @@ def run_reference(args, w):
 
 def main():
     args = parse()
-    from paper_2609_29395_gb300 import configs
+    from paper_2609_29395_gb300 import clustering, configs
     w = configs.WORKLOADS[args.workload]
     if args.impl == "reference":
         return run_reference(args, w)
@@ -460,6 +460,11 @@ def main():
     }
     clocks = clk.summary()
     line["clocks"] = clocks
+    # Eq. 6 for this workload's clusters: the ideal speedup of the concurrent
+    # epoch schedule over running the clusters one after another
+    s_ideal, e_ideal = clustering.ideal_schedule_speedup(
+        configs.cluster_sizes(ds.owner, assign, w.num_clusters), w.B)
+    line["schedule"] = {"S_ideal": s_ideal, "E_ideal": e_ideal}
 
     if rank == 0 and not args.no_extras:
         line["e2e"] = e2e_leg(pkg, w, ds, assign, params, torch, flush, max(10, K // 3))

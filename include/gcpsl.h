@@ -111,7 +111,14 @@ typedef struct gcpsl_ctx gcpsl_ctx;
  *  assignment[K]: cluster of each client (Algorithm 1's fixed map), in
  *    [0, C), or -1 for a client this context does not serve;
  *  B: per-cluster batch (Eq. 1, sum_k b_{k,t} = B); F: fuse after every F-th
- *    round (0 = never; gcpsl_fuse can still be called);
+ *    round (0 = never; gcpsl_fuse can still be called), every cluster taking
+ *    a local round every round (lockstep); or F = -1: the epoch schedule of
+ *    Section IV-C -- a system epoch is R = max_n r_n rounds (r_n = n_c / B),
+ *    cluster n takes local rounds 0 .. r_n - 1 of it and then waits at the
+ *    fusion barrier (no padded optimizer step, no BatchNorm-state update;
+ *    its batch in a waiting round is its last one, computed but not
+ *    applied, reported with loss 0 and |A| = 0), and the replicas are fused
+ *    after every system epoch;
  *  seed: sampler seed (Philox4x32-10 key);
  *  data: the dataset (see gcpsl_dataset);
  *  init_params: NULL or the initial parameters of one replica as fp32, client
@@ -119,7 +126,7 @@ typedef struct gcpsl_ctx gcpsl_ctx;
  *    weights OIHW, linear weight [out][in]); NULL draws them from a fixed
  *    Philox stream as U(-1/sqrt(fan_in), 1/sqrt(fan_in));
  *  out: receives the context.
- * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < 0, assignment
+ * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < -1, assignment
  * outside [-1, C), owner outside [0, K), labels outside [0, classes), a
  * cluster with fewer than B examples.  Fusion weights are
  * q_n = n_c / sum_m n_m over this context's clusters (Eq. 5).            */

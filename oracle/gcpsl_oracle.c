@@ -550,6 +550,8 @@ typedef struct {
   uint8_t* cand[4];                           /* [C][B][cout][Ho][Wo] of the last round */
   int32_t* ties;                              /* [C][B] ambiguous windows per example */
   int augment;                                /* crop + flip of the sampled images */
+  int64_t R;                                  /* F = -1: rounds per system epoch, else 0 */
+  int32_t* upd;                               /* [C] the cluster updated in the last round */
 } orc_ctx;
 
 void orc_destroy(orc_ctx* c);
@@ -563,7 +565,7 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   memset(&a, 0, sizeof(a));
   const int resnet = arch == ORC_RESNET18;
   if (!resnet && get_arch(arch, &a)) return ORC_EUNSUPPORTED;
-  if (K <= 0 || C <= 0 || B <= 0 || F < 0 || n <= 0 || !assignment || !images || !labels ||
+  if (K <= 0 || C <= 0 || B <= 0 || F < -1 || n <= 0 || !assignment || !images || !labels ||
       !owner || !init_params)
     return ORC_EINVAL;
   for (int k = 0; k < K; ++k) if (assignment[k] < -1 || assignment[k] >= C) return ORC_EINVAL;
@@ -610,6 +612,13 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   }
   free(fill);
   for (int k = 0; k < C; ++k) c->q[k] = (double)c->nc[k] / (double)total;
+  c->upd = (int32_t*)malloc(sizeof(int32_t) * (size_t)C);
+  if (!c->upd) { orc_destroy(c); return ORC_ENOMEM; }
+  c->R = 0;
+  for (int k = 0; k < C; ++k) {
+    c->upd[k] = 1;
+    if (F == -1 && c->nc[k] / B > c->R) c->R = c->nc[k] / B;
+  }
   int64_t P = c->o.p_total;
   c->theta = (double*)malloc(sizeof(double) * (size_t)(C * P));
   c->mom = (double*)calloc((size_t)(C * P), sizeof(double));
@@ -647,7 +656,7 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
 void orc_destroy(orc_ctx* c) {
   if (!c) return;
   for (int k = 0; k < c->C; ++k) { if (c->ids) free(c->ids[k]); if (c->perm) free(c->perm[k]); }
-  free(c->ids); free(c->perm); free(c->nc); free(c->cur_epoch); free(c->q);
+  free(c->ids); free(c->perm); free(c->nc); free(c->cur_epoch); free(c->q); free(c->upd);
   free(c->labels); free(c->owner); free(c->theta); free(c->mom); free(c->grad);
   free(c->idx); free(c->counts); free(c->loss); free(c->active);
   free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties); free(c->xbuf); free(c->bn); free(c->relu_rec); free(c->relu_in);
@@ -740,11 +749,21 @@ static void batch_images(const orc_ctx* c, int k, const int32_t* idx, double* ds
 }
 
 /* One local round of every cluster, then fusion when (t+1) mod F == 0. */
+/* Schedule (Section IV-C; Eq. 6).  Lockstep (F >= 0): every cluster takes
+ * a local round every round, its own epoch after r_n = n_c / B of them.
+ * Epoch schedule (F = -1): a system epoch is R = max_n r_n rounds; cluster
+ * n takes local rounds 0..r_n-1 of it and then waits at the fusion barrier
+ * (its batch in a waiting round is its last one, computed but not applied:
+ * no padded optimizer step, no normalisation-state update, loss and |A|
+ * reported as 0); the replicas are fused after every system epoch.        */
 int orc_step(orc_ctx* c) {
   int B = c->B;
   for (int k = 0; k < c->C; ++k) {
     int64_t r = c->nc[k] / B;
-    int64_t e = c->t / r, s = c->t % r;
+    int64_t period = c->R ? c->R : r;
+    int64_t e = c->t / period, s = c->t % period;
+    c->upd[k] = s < r;
+    if (s >= r) s = r - 1;
     if (e != c->cur_epoch[k]) {
       orc_epoch_perm(c->ids[k], c->nc[k], (uint32_t)(c->cluster_base + k), (uint32_t)e, c->seed,
                      c->perm[k]);
@@ -758,10 +777,21 @@ int orc_step(orc_ctx* c) {
       for (int b = 0; b < B; ++b) c->ybuf[b] = c->labels[idx[b]];
       int64_t P = c->o.p_total;
       const int64_t E = orn_mask_elems();
+      /* a waiting cluster keeps its BatchNorm running statistics */
+      double* bn_keep = NULL;
+      if (!c->upd[k]) {
+        bn_keep = (double*)malloc(sizeof(double) * (size_t)c->S);
+        if (!bn_keep) return ORC_ENOMEM;
+        memcpy(bn_keep, c->bn + k * c->S, sizeof(double) * (size_t)c->S);
+      }
       int rc = orn_forward_backward_masks(
           c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B, c->xbuf, c->ybuf, &c->loss[k],
           c->grad + k * P, c->cut_act + k * c->ncut, c->cut_grad + k * c->ncut, NULL,
           c->replay ? c->relu_in + (int64_t)k * B * E : NULL, c->relu_rec + (int64_t)k * B * E);
+      if (bn_keep) {
+        memcpy(c->bn + k * c->S, bn_keep, sizeof(double) * (size_t)c->S);
+        free(bn_keep);
+      }
       if (rc) return rc;
       continue;
     }
@@ -785,10 +815,18 @@ int orc_step(orc_ctx* c) {
     memcpy(c->cut_act + k * c->ncut, c->w.act[c->a.ncl], sizeof(double) * (size_t)c->ncut);
     memcpy(c->cut_grad + k * c->ncut, c->w.dact[c->a.ncl], sizeof(double) * (size_t)c->ncut);
   }
-  for (int k = 0; k < c->C; ++k) sgd(c, k);
+  for (int k = 0; k < c->C; ++k) {
+    if (c->upd[k]) {
+      sgd(c, k);
+    } else {
+      c->loss[k] = 0.0;
+      c->active[k] = 0;
+    }
+  }
   c->replay = 0;
   c->t++;
-  if (c->F > 0 && c->t % c->F == 0) return orc_fuse(c);
+  const int64_t every = c->R ? c->R : c->F;
+  if (every > 0 && c->t % every == 0) return orc_fuse(c);
   return ORC_OK;
 }
 

@@ -138,3 +138,18 @@ def label_aware_local_search(hist: np.ndarray, num_clusters: int,
         cur, cl, n = best
         assign[cl] = n
     return assign
+
+
+def schedule_rounds(sizes: np.ndarray, B: int) -> np.ndarray:
+    """r_n = n_c // B local rounds per epoch of each cluster (Section IV-C)."""
+    return np.asarray(sizes, dtype=np.int64) // B
+
+
+def ideal_schedule_speedup(sizes: np.ndarray, B: int):
+    """Eq. 6: S_ideal = sum_n r_n / max_n r_n and E_ideal = S_ideal / N for
+    one epoch of the concurrent schedule (clusters with fewer rounds wait at
+    the fusion barrier)."""
+    r = schedule_rounds(sizes, B)
+    s = float(r.sum()) / float(r.max())
+    return s, s / r.size
+

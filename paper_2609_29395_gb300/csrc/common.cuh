@@ -96,16 +96,24 @@ template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __flo
 // Kernel launchers (each enqueues on `s`; return the launch error)
 // ---------------------------------------------------------------------------
 // sampler.cu
+// period[n]: rounds per epoch of cluster n's sampler (r_n in lockstep, the
+// system epoch's max_m r_m under the epoch schedule); the permutation of
+// epoch t / period[n] is built when t % period[n] == 0.
 cudaError_t launch_epoch_keys(cudaStream_t s, const int32_t* ids, const int64_t* off,
-                              const int32_t* rounds, const int64_t* d_t, int cluster_base,
+                              const int32_t* period, const int64_t* d_t, int cluster_base,
                               uint64_t seed, uint64_t* keys, int C, int64_t max_nc);
 cudaError_t launch_epoch_rank(cudaStream_t s, const int32_t* ids, const int64_t* off,
-                              const int32_t* rounds, const int64_t* d_t, const uint64_t* keys,
+                              const int32_t* period, const int64_t* d_t, const uint64_t* keys,
                               int32_t* perm, int C, int64_t max_nc);
+// The round's batch of every cluster: local round s = t % period[n] of its
+// epoch when s < rounds[n]; a cluster past its r_n rounds (epoch schedule)
+// waits at the fusion barrier: upd[n] = 0 (nullable), its batch is its last
+// one (s = r_n - 1) and active[n] = 0.
 cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* off,
-                          const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
-                          const int32_t* labels, int K, int B, int C, int32_t* idx,
-                          int32_t* counts, int32_t* active, int32_t* y);
+                          const int32_t* rounds, const int32_t* period, const int64_t* d_t,
+                          const int32_t* owner, const int32_t* labels, int K, int B, int C,
+                          int32_t* idx, int32_t* counts, int32_t* active, int32_t* y,
+                          int32_t* upd);
 // Training augmentation of the gathered images (Sec. V-A: random crops and
 // horizontal flips): sampled image b of cluster n in round t is cropped
 // from its 4-pixel zero-padded version at offset (dy, dx) in [0, 8]^2 and
@@ -280,11 +288,12 @@ cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16
                              float* sums, int C, int B, int HW, int ch, int gn);
 // per set: mean, rstd, and per (c, [b,] ch) the affine form ss = (gamma rstd,
 // beta - mean gamma rstd) (GroupNorm per example, BatchNorm shared over the
-// batch); BatchNorm also updates run ([C] x run_rs: mean[ch], var[ch])
+// batch); BatchNorm also updates run ([C] x run_rs: mean[ch], var[ch]) of the
+// replicas with upd[c] (upd nullable: all)
 cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const float* gamma,
                                      const float* beta, int64_t g_rs, float* mean, float* rstd,
                                      float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
-                                     int ch, int gn);
+                                     int ch, int gn, const int32_t* upd = nullptr);
 // backward affine form kk = (k1, k2, k3, 0): dy = k1 dz + k2 y + k3 per
 // (c, [b,] ch); per channel dgamma, dbeta
 cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,
@@ -344,10 +353,12 @@ inline int sgd_chunk(int splits) {
 // (<= kSgdThreads * kSgdPer), 0}.
 cudaError_t launch_sgd_seg(cudaStream_t s, float* theta, float* mom, bf16* shadow,
                            const SgdSeg* segs, const int4* blocks, int nblocks, int64_t P_pad,
-                           float lr, float momentum, float wd, int nesterov, int64_t* d_t);
+                           float lr, float momentum, float wd, int nesterov, const int32_t* upd,
+                           int64_t* d_t);
+// upd (nullable): replica c = i / P_pad takes the update only when upd[c]
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,
-                       bf16* shadow, int64_t n, float lr, float momentum, float wd,
-                       int nesterov, int64_t* d_t);
+                       bf16* shadow, int64_t n, int64_t P_pad, float lr, float momentum, float wd,
+                       int nesterov, const int32_t* upd, int64_t* d_t);
 cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,
                         int64_t P);
 

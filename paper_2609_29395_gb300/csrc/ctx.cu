@@ -240,7 +240,7 @@ const char* const kWgradTc[4] = {"conv_wgrad_tc.L0", "conv_wgrad_tc.L1", "conv_w
 // true when some cluster starts an epoch in round c->t (0-based)
 bool epoch_boundary(const gcpsl_ctx* c) {
   for (int n = 0; n < c->C; ++n)
-    if (c->t % c->h_rounds[n] == 0) return true;
+    if (c->t % c->h_period[n] == 0) return true;
   return false;
 }
 
@@ -253,15 +253,15 @@ gcpsl_status enqueue_sample(gcpsl_ctx* c, bool boundary) {
   cudaStream_t s = c->stream;
   const int C = c->C, B = c->B;
   if (boundary) {
-    LAUNCH("epoch_keys", launch_epoch_keys(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
+    LAUNCH("epoch_keys", launch_epoch_keys(s, c->d_ids, c->d_off, c->d_period, c->d_t,
                                            c->desc.cluster_id_base, c->seed, c->d_keys, C,
                                            c->max_nc));
-    LAUNCH("epoch_rank", launch_epoch_rank(s, c->d_ids, c->d_off, c->d_rounds, c->d_t,
+    LAUNCH("epoch_rank", launch_epoch_rank(s, c->d_ids, c->d_off, c->d_period, c->d_t,
                                            c->d_keys, c->d_perm, C, c->max_nc));
   }
-  LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_t, c->d_owner,
-                                 c->d_labels, c->K, B, C, c->d_idx, c->d_counts, c->d_active,
-                                 c->d_y));
+  LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_period, c->d_t,
+                                 c->d_owner, c->d_labels, c->K, B, C, c->d_idx, c->d_counts,
+                                 c->d_active, c->d_y, c->d_upd));
   const AugArgs aug{c->desc.augment, (uint32_t)c->seed, (uint32_t)(c->seed >> 32), c->d_t,
                     c->desc.cluster_id_base, B};
   LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, (T*)c->d_act[0], aug));
@@ -273,11 +273,11 @@ gcpsl_status enqueue_sgd(gcpsl_ctx* c) {
     LAUNCH("sgd", launch_sgd_seg(c->stream, c->d_theta, c->d_mom, c->d_shadow, c->d_sgd_segs,
                                  c->d_sgd_blocks, c->n_sgd_blocks, c->P_pad, c->desc.lr,
                                  c->desc.momentum, c->desc.weight_decay, c->desc.nesterov,
-                                 c->d_t));
+                                 c->d_upd, c->d_t));
   else
     LAUNCH("sgd", launch_sgd(c->stream, c->d_theta, c->d_mom, c->d_grad, c->d_shadow,
-                             (int64_t)c->C * c->P_pad, c->desc.lr, c->desc.momentum,
-                             c->desc.weight_decay, c->desc.nesterov, c->d_t));
+                             (int64_t)c->C * c->P_pad, c->P_pad, c->desc.lr, c->desc.momentum,
+                             c->desc.weight_decay, c->desc.nesterov, c->d_upd, c->d_t));
   // the segment update also rewrites the packed input-layer weights
   return c->sgd_packs_w0 ? GCPSL_OK : refresh_derived(c);
 }
@@ -710,6 +710,18 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   DALLOC(c->d_keys, sizeof(uint64_t) * total);
   CK(cudaMemcpy(c->d_off, c->h_off.data(), sizeof(int64_t) * (C + 1), cudaMemcpyHostToDevice));
   CK(cudaMemcpy(c->d_rounds, c->h_rounds.data(), sizeof(int32_t) * C, cudaMemcpyHostToDevice));
+  c->R = 0;
+  if (F == -1)
+    for (int k = 0; k < C; ++k) c->R = std::max<int64_t>(c->R, c->h_rounds[k]);
+  c->h_period.assign(C, 0);
+  for (int k = 0; k < C; ++k) c->h_period[k] = c->R ? (int32_t)c->R : c->h_rounds[k];
+  DALLOC(c->d_period, sizeof(int32_t) * C);
+  DALLOC(c->d_upd, sizeof(int32_t) * C);
+  CK(cudaMemcpy(c->d_period, c->h_period.data(), sizeof(int32_t) * C, cudaMemcpyHostToDevice));
+  {
+    const std::vector<int32_t> ones((size_t)C, 1);
+    CK(cudaMemcpy(c->d_upd, ones.data(), sizeof(int32_t) * C, cudaMemcpyHostToDevice));
+  }
   CK(cudaMemcpy(c->d_q, c->h_q.data(), sizeof(float) * C, cudaMemcpyHostToDevice));
   CK(cudaMemcpy(c->d_ids, ids.data(), sizeof(int32_t) * total, cudaMemcpyHostToDevice));
 
@@ -849,7 +861,7 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
   *out = nullptr;
   if (!desc || !assignment || !data || !data->images || !data->labels || !data->owner)
     return fail(nullptr, GCPSL_E_INVAL, "NULL argument");
-  if (K <= 0 || C <= 0 || B <= 0 || B > 1024 || F < 0 || data->n <= 0 || data->n > INT32_MAX)
+  if (K <= 0 || C <= 0 || B <= 0 || B > 1024 || F < -1 || data->n <= 0 || data->n > INT32_MAX)
     return fail(nullptr, GCPSL_E_INVAL, "bad size (K=%d C=%d B=%d F=%d n=%lld)", K, C, B, F,
                 (long long)data->n);
   if (data->num_classes != 10)
@@ -906,7 +918,8 @@ gcpsl_status gcpsl_step(gcpsl_ctx* c, gcpsl_step_stats* stats) {
   }
   if (st != GCPSL_OK) return st;
   c->t++;
-  if (c->F > 0 && c->t % c->F == 0) {
+  const int64_t every = c->R ? c->R : c->F;       // fusion interval in rounds
+  if (every > 0 && c->t % every == 0) {
     st = enqueue_fuse(c);
     if (st != GCPSL_OK) return st;
   }
@@ -916,6 +929,9 @@ gcpsl_status gcpsl_step(gcpsl_ctx* c, gcpsl_step_stats* stats) {
     CK(cudaMemcpyAsync(c->h_active, c->d_active, sizeof(int32_t) * c->C, cudaMemcpyDeviceToHost,
                        c->stream));
     SYNC_CHECK(c);
+    // a cluster waiting at the fusion barrier took no update: loss 0
+    for (int n = 0; n < c->C; ++n)
+      if ((c->t - 1) % c->h_period[n] >= c->h_rounds[n]) c->h_loss[n] = 0.f;
     if (stats->loss) std::memcpy(stats->loss, c->h_loss, sizeof(float) * c->C);
     if (stats->active) std::memcpy(stats->active, c->h_active, sizeof(int32_t) * c->C);
   }

@@ -114,6 +114,13 @@ struct gcpsl_ctx {
 
   std::vector<int64_t> h_off;      // [C+1] offsets of the clusters' id lists
   std::vector<int32_t> h_rounds;   // r_n = n_c / B
+  // schedule: lockstep (F >= 0): period_n = r_n; epoch schedule (F = -1):
+  // period_n = R = max_n r_n, fuse every R rounds, cluster n updates in the
+  // first r_n rounds of each system epoch (d_upd[n] of the current round)
+  std::vector<int32_t> h_period;
+  int64_t R = 0;
+  int32_t* d_period = nullptr;
+  int32_t* d_upd = nullptr;
   std::vector<float> h_q;          // fusion weights
   int64_t max_nc = 0;
   int64_t* d_off = nullptr;

@@ -164,8 +164,8 @@ extern "C" gcpsl_status gcpsl_sample_round_noalloc(
     e = cudaGetLastError();
   }
   if (e == cudaSuccess)
-    e = launch_sample(s, perm, off, rounds, t, owner, labels, K, B, C, idx, counts, active,
-                      batch_labels);
+    e = launch_sample(s, perm, off, rounds, rounds, t, owner, labels, K, B, C, idx, counts,
+                      active, batch_labels, nullptr);
   // the host copies above read pageable memory; finish them before the
   // vectors go out of scope
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);

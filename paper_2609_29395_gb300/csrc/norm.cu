@@ -152,7 +152,8 @@ __global__ void __launch_bounds__(kChanWarps * 32)
 k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ gamma,
                     const float* __restrict__ beta, int64_t g_rs, float* __restrict__ mean,
                     float* __restrict__ rstd, float2* __restrict__ ss, float* __restrict__ run,
-                    int64_t run_rs, int C, int B, int HW, int ch, int gn) {
+                    int64_t run_rs, int C, int B, int HW, int ch, int gn,
+                    const int32_t* __restrict__ upd) {
   __shared__ double red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
@@ -194,7 +195,7 @@ k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ ga
   const int64_t w = (int64_t)c * ch + s;
   mean[w] = (float)mu;
   rstd[w] = (float)r;
-  if (run) {
+  if (run && (!upd || upd[c])) {          // replicas at the fusion barrier keep theirs
     float* rm = run + (int64_t)c * run_rs;
     float* rv = rm + ch;
     rm[s] = (float)(0.9 * (double)rm[s] + 0.1 * mu);
@@ -571,11 +572,11 @@ cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16
 cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const float* gamma,
                                      const float* beta, int64_t g_rs, float* mean, float* rstd,
                                      float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
-                                     int ch, int gn) {
+                                     int ch, int gn, const int32_t* upd) {
   if (ch % 32) return cudaErrorInvalidValue;
   const unsigned blocks = gn ? nblk((int64_t)C * B * 32, 256) : (unsigned)(C * (ch / 32));
   return launch_k(k_norm_finalize_fwd, blocks, 256, 0, s, sums, gamma, beta, g_rs,
-                  mean, rstd, ss, run, run_rs, C, B, HW, ch, gn);
+                  mean, rstd, ss, run, run_rs, C, B, HW, ch, gn, upd);
 }
 
 cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,

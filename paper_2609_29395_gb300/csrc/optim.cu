@@ -16,11 +16,13 @@ namespace {
 
 __global__ void k_sgd(float* __restrict__ theta, float* __restrict__ mom,
                       const float* __restrict__ grad, bf16* __restrict__ shadow, int64_t n,
-                      float lr, float mu, float wd, int nesterov, int64_t* __restrict__ d_t) {
+                      int64_t P_pad, float lr, float mu, float wd, int nesterov,
+                      const int32_t* __restrict__ upd, int64_t* __restrict__ d_t) {
   pdl_wait();
   pdl_trigger();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    if (upd && !upd[i / P_pad]) continue;          // waiting at the fusion barrier
     float th = theta[i];
     float g = grad[i];
     if (wd != 0.f) g = fmaf(wd, th, g);
@@ -64,7 +66,8 @@ __device__ __forceinline__ float sgd1(float& th, float& m, float g, float lr, fl
 __global__ void __launch_bounds__(kSgdThreads)
 k_sgd_seg(float4* __restrict__ theta, float4* __restrict__ mom, uint2* __restrict__ shadow,
           const SgdSeg* __restrict__ segs, const int4* __restrict__ blocks, uint32_t P4,
-          float lr, float mu, float wd, int nesterov, int64_t* __restrict__ d_t) {
+          float lr, float mu, float wd, int nesterov, const int32_t* __restrict__ upd,
+          int64_t* __restrict__ d_t) {
   pdl_wait();
   pdl_trigger();
   const int4 bk = blocks[blockIdx.x];
@@ -81,7 +84,7 @@ k_sgd_seg(float4* __restrict__ theta, float4* __restrict__ mom, uint2* __restric
     const uint32_t r = (uint32_t)(k * kSgdThreads) + threadIdx.x;
     const uint32_t local = (uint32_t)bk.y + r;
     const uint32_t c = local / cnt4, j = local - c * cnt4;
-    ok[k] = r < (uint32_t)bk.z;
+    ok[k] = r < (uint32_t)bk.z && (!upd || upd[c]);   // skip replicas at the fusion barrier
     at[k] = c * P4 + off4 + j;
     sa[k] = c * (uint32_t)splits * per4 + j;
     g[k] = ok[k] ? src[sa[k]] : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -153,22 +156,23 @@ unsigned grid_for(int64_t n, int threads) {
 }  // namespace
 
 cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* grad,
-                       bf16* shadow, int64_t n, float lr, float momentum, float wd,
-                       int nesterov, int64_t* d_t) {
-  return launch_k(k_sgd, grid_for(n, 256), 256, 0, s, theta, mom, grad, shadow, n, lr, momentum,
-                  wd, nesterov, d_t);
+                       bf16* shadow, int64_t n, int64_t P_pad, float lr, float momentum, float wd,
+                       int nesterov, const int32_t* upd, int64_t* d_t) {
+  return launch_k(k_sgd, grid_for(n, 256), 256, 0, s, theta, mom, grad, shadow, n, P_pad, lr,
+                  momentum, wd, nesterov, upd, d_t);
 }
 
 cudaError_t launch_sgd_seg(cudaStream_t s, float* theta, float* mom, bf16* shadow,
                            const SgdSeg* segs, const int4* blocks, int nblocks, int64_t P_pad,
-                           float lr, float momentum, float wd, int nesterov, int64_t* d_t) {
+                           float lr, float momentum, float wd, int nesterov, const int32_t* upd,
+                           int64_t* d_t) {
   if (nblocks < 1 || P_pad % 4 || (uintptr_t)theta % 16 || (uintptr_t)mom % 16 ||
       (uintptr_t)shadow % 8)
     return cudaErrorInvalidValue;
   return launch_k(k_sgd_seg, (unsigned)nblocks, kSgdThreads, 0, s,
                   reinterpret_cast<float4*>(theta), reinterpret_cast<float4*>(mom),
                   reinterpret_cast<uint2*>(shadow), segs, blocks, (uint32_t)(P_pad / 4), lr,
-                  momentum, wd, nesterov, d_t);
+                  momentum, wd, nesterov, upd, d_t);
 }
 
 cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,

@@ -457,7 +457,7 @@ gcpsl_status norm_stats(gcpsl_ctx* c, const RnNorm& n, const bf16* y) {
   LAUNCH("rn_norm_finalize",
          launch_norm_finalize_fwd(c->stream, r.sums, th + n.off_g, th + n.off_b, c->P_pad, n.mean,
                                   n.rstd, n.ss, n.gn ? nullptr : r.bn + n.s_off, r.S_pad, c->C,
-                                  c->B, n.hw, n.ch, n.gn));
+                                  c->B, n.hw, n.ch, n.gn, c->d_upd));
   return GCPSL_OK;
 }
 

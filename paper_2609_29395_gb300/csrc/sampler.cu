@@ -22,14 +22,14 @@ namespace {
 constexpr int kRankThreads = 256;
 
 __global__ void k_epoch_keys(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
-                             const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
+                             const int32_t* __restrict__ period, const int64_t* __restrict__ d_t,
                              int cluster_base, uint32_t s0, uint32_t s1,
                              uint64_t* __restrict__ keys) {
   pdl_wait();
   pdl_trigger();
   const int c = blockIdx.y;
   const int64_t t = *d_t;
-  const int64_t r = rounds[c];
+  const int64_t r = period[c];
   if (t % r != 0) return;                       // not an epoch boundary
   const uint32_t epoch = (uint32_t)(t / r);
   const int64_t base = off[c], n = off[c + 1] - base;
@@ -46,7 +46,7 @@ __device__ __forceinline__ bool key_less(uint64_t ka, int32_t ja, uint64_t kb, i
 
 __global__ void __launch_bounds__(kRankThreads)
 k_epoch_rank(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
-             const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
+             const int32_t* __restrict__ period, const int64_t* __restrict__ d_t,
              const uint64_t* __restrict__ keys, int32_t* __restrict__ perm) {
   __shared__ uint64_t sk[kRankThreads];
   __shared__ int32_t sj[kRankThreads];
@@ -54,7 +54,7 @@ k_epoch_rank(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
   pdl_trigger();
   const int c = blockIdx.y;
   const int64_t t = *d_t;
-  if (t % rounds[c] != 0) return;
+  if (t % period[c] != 0) return;
   const int64_t base = off[c], n = off[c + 1] - base;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if ((int64_t)blockIdx.x * blockDim.x >= n) return;      // whole block idle
@@ -75,10 +75,12 @@ k_epoch_rank(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
 
 // One block per cluster, one thread per batch slot (B <= 1024).
 __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __restrict__ off,
-                         const int32_t* __restrict__ rounds, const int64_t* __restrict__ d_t,
-                         const int32_t* __restrict__ owner, const int32_t* __restrict__ labels,
-                         int K, int B, int32_t* __restrict__ idx, int32_t* __restrict__ counts,
-                         int32_t* __restrict__ active, int32_t* __restrict__ y) {
+                         const int32_t* __restrict__ rounds, const int32_t* __restrict__ period,
+                         const int64_t* __restrict__ d_t, const int32_t* __restrict__ owner,
+                         const int32_t* __restrict__ labels, int K, int B,
+                         int32_t* __restrict__ idx, int32_t* __restrict__ counts,
+                         int32_t* __restrict__ active, int32_t* __restrict__ y,
+                         int32_t* __restrict__ upd) {
   extern __shared__ int32_t sm[];
   int32_t* sid = sm;          // [B] ids of the round
   int32_t* sown = sm + B;     // [B] their owners
@@ -87,7 +89,9 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
   pdl_trigger();
   const int c = blockIdx.x;
   const int b = threadIdx.x;
-  const int64_t s = *d_t % rounds[c];
+  int64_t s = *d_t % period[c];
+  const bool updates = s < rounds[c];          // else waiting at the fusion barrier
+  if (!updates) s = rounds[c] - 1;
   int32_t* cnt = counts + (int64_t)c * K;
   for (int k = b; k < K; k += blockDim.x) cnt[k] = 0;
   const int32_t id = perm[off[c] + s * B + b];
@@ -104,10 +108,12 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
   atomicAdd(&cnt[own], 1);
   __syncthreads();
   const int first = __syncthreads_count(rank == 0 || sorted_own[rank - 1] != own);
-  if (b == 0) active[c] = first;
+  if (b == 0) {
+    active[c] = updates ? first : 0;
+    if (upd) upd[c] = updates;
+  }
 }
 
-// fp32 storage: x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w] (3 channels).
 // crop offsets and flip of sampled image cb = c * B + b (see AugArgs)
 __device__ __forceinline__ void aug_params(const AugArgs& a, int64_t cb, int& dy, int& dx,
                                            int& flip) {
@@ -122,6 +128,7 @@ __device__ __forceinline__ void aug_params(const AugArgs& a, int64_t cb, int& dy
   flip = (int)(ctr[2] & 1u);
 }
 
+// fp32 storage: x0[c][b][h][w][ch] = images[idx[c][b]][ch][h][w] (3 channels).
 __global__ void k_gather_f32(const float* __restrict__ images, const int32_t* __restrict__ idx,
                              int CB, float* __restrict__ x0, const AugArgs aug) {
   pdl_wait();
@@ -188,26 +195,27 @@ k_gather_im2col(const float* __restrict__ images, const int32_t* __restrict__ id
 }  // namespace
 
 cudaError_t launch_epoch_keys(cudaStream_t s, const int32_t* ids, const int64_t* off,
-                              const int32_t* rounds, const int64_t* d_t, int cluster_base,
+                              const int32_t* period, const int64_t* d_t, int cluster_base,
                               uint64_t seed, uint64_t* keys, int C, int64_t max_nc) {
   dim3 grid((unsigned)((max_nc + 255) / 256), (unsigned)C);
-  return launch_k(k_epoch_keys, grid, 256, 0, s, ids, off, rounds, d_t, cluster_base,
+  return launch_k(k_epoch_keys, grid, 256, 0, s, ids, off, period, d_t, cluster_base,
                   (uint32_t)seed, (uint32_t)(seed >> 32), keys);
 }
 
 cudaError_t launch_epoch_rank(cudaStream_t s, const int32_t* ids, const int64_t* off,
-                              const int32_t* rounds, const int64_t* d_t, const uint64_t* keys,
+                              const int32_t* period, const int64_t* d_t, const uint64_t* keys,
                               int32_t* perm, int C, int64_t max_nc) {
   dim3 grid((unsigned)((max_nc + kRankThreads - 1) / kRankThreads), (unsigned)C);
-  return launch_k(k_epoch_rank, grid, kRankThreads, 0, s, ids, off, rounds, d_t, keys, perm);
+  return launch_k(k_epoch_rank, grid, kRankThreads, 0, s, ids, off, period, d_t, keys, perm);
 }
 
 cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* off,
-                          const int32_t* rounds, const int64_t* d_t, const int32_t* owner,
-                          const int32_t* labels, int K, int B, int C, int32_t* idx,
-                          int32_t* counts, int32_t* active, int32_t* y) {
-  return launch_k(k_sample, C, B, 3 * B * sizeof(int32_t), s, perm, off, rounds, d_t, owner,
-                  labels, K, B, idx, counts, active, y);
+                          const int32_t* rounds, const int32_t* period, const int64_t* d_t,
+                          const int32_t* owner, const int32_t* labels, int K, int B, int C,
+                          int32_t* idx, int32_t* counts, int32_t* active, int32_t* y,
+                          int32_t* upd) {
+  return launch_k(k_sample, C, B, 3 * B * sizeof(int32_t), s, perm, off, rounds, period, d_t,
+                  owner, labels, K, B, idx, counts, active, y, upd);
 }
 
 template <>

@@ -198,6 +198,29 @@ def test_augmented_rounds_bf16_and_fp32():
         check_round(gpu, orc, w.arch, tol=1e-3, loss_tol=1e-4, fwd_tol=1e-5)
 
 
+def test_epoch_schedule_with_fusion_barrier():
+    """F = -1 (Section IV-C): clusters of unequal size take r_n local rounds
+    per system epoch of R = max r_n rounds and wait at the fusion barrier
+    (no update, loss and |A| 0), then all replicas are fused; the GPU matches
+    the oracle round by round through one system epoch and into the next."""
+    ds = synth.make_dataset(3072, 10, 24, 0.3, balanced=False, seed_data=2, seed_split=3)
+    assign = (np.arange(24) % 6 > 2).astype(np.int32) + (np.arange(24) % 6 > 4).astype(np.int32)
+    params = synth.init_params(synth.ARCH_SPLIT_CNN)
+    B = 64
+    r = np.bincount(assign[ds.owner], minlength=3) // B
+    R = int(r.max())
+    assert len(set(r.tolist())) == 3 and R <= 24, r
+    gpu, orc = pair(synth.ARCH_SPLIT_CNN, 24, 3, assign, B, -1, ds, params, True, lr=0.05,
+                    momentum=0.9)
+    for t in range(R + 2):
+        check_round(gpu, orc, synth.ARCH_SPLIT_CNN)
+        active = orc.stats()[1]                 # equal to the GPU's (check_round)
+        for n in range(3):
+            assert (active[n] == 0) == (t % R >= r[n])
+        if t == R - 1:
+            assert all((gpu.all_params(n) == gpu.all_params(0)).all() for n in range(3))
+
+
 def test_ragged_batch_nesterov_wd_label_smoothing():
     """B = 24 (not a power of two), C = 6, Nesterov, weight decay, label
     smoothing."""

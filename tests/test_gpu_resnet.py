@@ -132,6 +132,32 @@ def test_resnet18_rounds_against_oracle():
     assert (gpu.bn_state(0) == gpu.bn_state(1)).all()
 
 
+def test_resnet18_epoch_schedule_keeps_waiting_batchnorm_state():
+    """F = -1 with unequal clusters: a cluster waiting at the fusion barrier
+    keeps its parameters, momentum and BatchNorm running statistics (its
+    round is computed, not applied); fusion after the system epoch."""
+    ds = synth.make_dataset(200, 10, 8, 0.5, balanced=False, seed_data=7, seed_split=8)
+    assign = np.array([0, 0, 0, 0, 0, 1, 1, 1], dtype=np.int32)
+    params = synth.init_params(RES, seed=9)
+    B = 16
+    r = np.bincount(assign[ds.owner], minlength=2) // B
+    R = int(r.max())
+    assert r.min() < R <= 10, r
+    kw = dict(lr=0.05, momentum=0.9)
+    gpu = pkg.Context(RES, 8, 2, assign, B, -1, 4, ds.images, ds.labels, ds.owner, params,
+                      bf16=True, **kw)
+    orc = oracle.Oracle(RES, 8, 2, assign, B, -1, 4, ds.images, ds.labels, ds.owner, params,
+                        bf16=True, **kw)
+    short = int(np.argmin(r))
+    for t in range(R):
+        bn_before = orc.bn_state(short).astype(np.float32)     # what _round loads
+        _round(gpu, orc)
+        if r[short] <= t < R - 1:
+            assert (gpu.bn_state(short) == bn_before).all()
+    assert (gpu.all_params(0) == gpu.all_params(1)).all()
+    assert (gpu.bn_state(0) == gpu.bn_state(1)).all()
+
+
 def test_resnet18_grouped_equals_serialized_and_graph_equals_eager():
     """Two clusters in one context == each cluster alone (same cluster id),
     and graph replay == eager launches, bit for bit, over three rounds."""

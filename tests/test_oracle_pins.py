@@ -397,3 +397,66 @@ def test_oracle_round_uses_the_augmented_batch():
                               for b, i in enumerate(idx[m])])
             ref = oracle.forward_backward(arch, params, x, ds.labels[idx[m]])[0]
             assert abs(ref - loss[m]) < 1e-12 * max(1.0, abs(ref))
+
+
+# --------------------------------------------------------------------------
+# Epoch schedule with the fusion barrier (Section IV-C, Eq. 6)
+# --------------------------------------------------------------------------
+def test_epoch_schedule_barrier_and_fusion():
+    """F = -1: cluster n takes r_n = n_c / B local rounds per system epoch of
+    R = max r_n rounds, then waits (parameters, momentum and sample frozen,
+    loss and |A| reported 0); after R rounds the replicas are fused with q
+    (Eq. 5).  Its first min r_n rounds equal the lockstep schedule's."""
+    ds = synth.make_dataset(600, 10, 12, 0.5, balanced=False, seed_data=5, seed_split=6)
+    rng = np.random.default_rng(7)
+    assign = rng.choice(3, size=12, p=[0.55, 0.3, 0.15]).astype(np.int32)
+    assign[:3] = [0, 1, 2]
+    arch = synth.ARCH_TINY_CNN
+    params = synth.init_params(arch, seed=8)
+    B = 16
+    sizes = np.bincount(assign[ds.owner], minlength=3)
+    r = clustering.schedule_rounds(sizes, B)
+    R = int(r.max())
+    assert len(set(r.tolist())) > 1, r          # unequal epochs
+    kw = dict(lr=0.05, momentum=0.9)
+    ep = oracle.Oracle(arch, 12, 3, assign, B, -1, 4, ds.images, ds.labels, ds.owner, params, **kw)
+    ls = oracle.Oracle(arch, 12, 3, assign, B, 0, 4, ds.images, ds.labels, ds.owner, params, **kw)
+    seen = [set() for _ in range(3)]
+    for t in range(R):
+        before = [ep.all_params(n) for n in range(3)]
+        ep.step()
+        ls.step()
+        idx, counts = ep.sample()
+        loss, active = ep.stats()
+        last = t == R - 1
+        for n in range(3):
+            if t < r[n]:
+                assert loss[n] > 0 and active[n] > 0
+                seen[n].update(idx[n].tolist())
+                if t < r.min():
+                    li, _ = ls.sample()
+                    assert (idx[n] == li[n]).all()
+                if not last:
+                    assert not np.array_equal(ep.all_params(n), before[n])
+            else:
+                assert loss[n] == 0 and active[n] == 0
+                if not last:
+                    assert np.array_equal(ep.all_params(n), before[n])
+        if t == R - 2:
+            pre_fuse = [ep.all_params(n) for n in range(3)]
+    for n in range(3):
+        assert len(seen[n]) == r[n] * B                 # each example at most once
+    q = ep.q()
+    fused = ep.all_params(0)
+    for n in range(3):
+        assert np.array_equal(ep.all_params(n), fused)
+    # every cluster but the longest waited in round R - 1 (its parameters
+    # before the fusion are those after round R - 2); the longest one's
+    # trajectory is the lockstep run's (same batches, no fusion yet)
+    longest = int(np.argmax(r))
+    assert sorted(r.tolist()).count(R) == 1
+    expect = sum(q[n] * pre_fuse[n] for n in range(3) if n != longest) + \
+        q[longest] * ls.all_params(longest)
+    np.testing.assert_allclose(fused, expect, rtol=0, atol=1e-12 * np.abs(expect).max())
+    s, e = clustering.ideal_schedule_speedup(sizes, B)
+    assert abs(s - r.sum() / R) < 1e-12 and abs(e - s / 3) < 1e-12
