@@ -43,10 +43,24 @@ FLUSH_BYTES = 256 << 20
 # DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by
 # kernel kind; valid only while the kernel source hashes to the recorded value.
 NCU_TRAFFIC = {
-    # profiles/k_wgrad_tc_and_k_conv_tc_fprop_layer1_splitcnn_c4_full.md (dram read + write
-    # per launch)
-    "conv_wgrad_tc.L1": {"bytes": 50.35264e6 + 0.963328e6, "src_hash": "b78caee8c7041e7d"},
-    "conv_fwd_tc.L1": {"bytes": 16.9472e6, "src_hash": "b78caee8c7041e7d"},
+    # DRAM read + write per launch (ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,
+    # one pass); SplitCNN kinds from the full C=4 workload, the ResNet-18 GroupNorm kinds
+    # from C=2 (20,000 images) scaled x4 to C=8 (per-example kernels): see
+    # profiles/splitcnn_c4_and_resnet18_traffic.md
+    "conv_fwd_tc.L0": {"bytes": 1.681e+07, "src_hash": "9edb62919210128c"},
+    "conv_fwd_tc.L1": {"bytes": 1.697e+07, "src_hash": "9edb62919210128c"},
+    "conv_fwd_tc.L2": {"bytes": 9.02e+06, "src_hash": "9edb62919210128c"},
+    "conv_fwd_tc.L3": {"bytes": 5.4e+06, "src_hash": "9edb62919210128c"},
+    "conv_dgrad_tc.L1": {"bytes": 5.051e+07, "src_hash": "9edb62919210128c"},
+    "conv_dgrad_tc.L2": {"bytes": 2.178e+07, "src_hash": "9edb62919210128c"},
+    "conv_dgrad_tc.L3": {"bytes": 7.5e+06, "src_hash": "9edb62919210128c"},
+    "conv_wgrad_tc.L0": {"bytes": 3.357e+07, "src_hash": "9edb62919210128c"},
+    "conv_wgrad_tc.L1": {"bytes": 5.036e+07, "src_hash": "9edb62919210128c"},
+    "conv_wgrad_tc.L2": {"bytes": 2.523e+07, "src_hash": "9edb62919210128c"},
+    "conv_wgrad_tc.L3": {"bytes": 8.43e+06, "src_hash": "9edb62919210128c"},
+    "sgd": {"bytes": 6.11e+07, "src_hash": "483ce6954d2d1468"},
+    "rn_norm_gn_bwd": {"bytes": 3.93448e+08, "src_hash": "d7895818885460a1"},
+    "rn_norm_gn": {"bytes": 1.88496e+08, "src_hash": "d7895818885460a1"},
 }
 
 
