@@ -92,9 +92,9 @@ def _declare(L):
     L.orc_get_ties.argtypes = [ct.c_void_p, i32p]
     L.orc_get_ties.restype = None
     L.orc_set_bn_state.argtypes = [ct.c_void_p, ct.c_int, f64p]
-    L.orn_forward_backward.argtypes = [ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p, i32p,
+    L.orn_forward_backward.argtypes = [ct.c_int, ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p, i32p,
                                        f64p, f64p, f64p, f64p, f64p]
-    L.orn_forward_backward_masks.argtypes = [ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p,
+    L.orn_forward_backward_masks.argtypes = [ct.c_int, ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p,
                                              i32p, f64p, f64p, f64p, f64p, f64p,
                                              _p(ct.c_uint8), _p(ct.c_uint8)]
     L.orn_mask_elems.restype = ct.c_int64
@@ -159,6 +159,7 @@ def num_params(arch: int, segment: int) -> int:
 
 
 RESNET18 = 2
+RESNET18_C100 = 3          # the same split with a 100-class head
 
 
 def bn_state_size() -> int:
@@ -185,8 +186,8 @@ def resnet_mask_elems() -> int:
 
 def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False,
                             label_smoothing: float = 0.0, want_grad: bool = True,
-                            masks_in=None, want_masks: bool = False):
-    """ResNet-18 split: (loss, grad[P] or None, cut_act, cut_grad, logits, bn_state
+                            masks_in=None, want_masks: bool = False, classes: int = 10):
+    """ResNet-18 split with a `classes`-way head (10 or 100): (loss, grad[P] or None, cut_act, cut_grad, logits, bn_state
     after this batch's update of the running statistics[, masks]).  masks:
     [B][resnet_mask_elems()] uint8 ReLU decisions (stem, then per block those
     of a1 and of the output, NCHW); masks_in replays given decisions."""
@@ -194,21 +195,22 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
     x = np.ascontiguousarray(x, dtype=np.float64)
     labels = np.ascontiguousarray(labels, dtype=np.int32)
     B = labels.size
-    P = num_params(RESNET18, 0) + num_params(RESNET18, 1)
+    arch = {10: RESNET18, 100: RESNET18_C100}[classes]
+    P = num_params(arch, 0) + num_params(arch, 1)
     bn = np.ascontiguousarray(initial_bn_state() if bn_state is None else bn_state,
                               dtype=np.float64).copy()
     loss = np.zeros(1)
     grad = np.zeros(P) if want_grad else None
     ncut = _cut_elems(RESNET18, B)
     ca, cg = np.zeros(ncut), np.zeros(ncut)
-    logits = np.zeros(B * 10)
+    logits = np.zeros(B * classes)
     mo = np.zeros((B, resnet_mask_elems()), dtype=np.uint8) if want_masks else None
     mi = None
     if masks_in is not None:
         mi = np.ascontiguousarray(masks_in, dtype=np.uint8)
         assert mi.size == B * resnet_mask_elems()
     rc = lib().orn_forward_backward_masks(
-        int(bf16), label_smoothing, _ptr(params, ct.c_double), _ptr(bn, ct.c_double), B,
+        classes, int(bf16), label_smoothing, _ptr(params, ct.c_double), _ptr(bn, ct.c_double), B,
         _ptr(x, ct.c_double), _ptr(labels, ct.c_int32), _ptr(loss, ct.c_double),
         _ptr(grad, ct.c_double) if want_grad else None, _ptr(ca, ct.c_double),
         _ptr(cg, ct.c_double), _ptr(logits, ct.c_double),
@@ -216,7 +218,7 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
         _ptr(mo, ct.c_uint8) if mo is not None else None)
     if rc:
         raise RuntimeError(f"oracle resnet forward_backward failed: {rc}")
-    out = (float(loss[0]), grad, ca, cg, logits.reshape(B, 10), bn)
+    out = (float(loss[0]), grad, ca, cg, logits.reshape(B, classes), bn)
     return out + (mo,) if want_masks else out
 
 
@@ -245,11 +247,11 @@ def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smo
 
 
 def _cut_elems(arch: int, B: int) -> int:
-    return B * {0: 16 * 16 * 16, 1: 64 * 16 * 16, 2: 64 * 32 * 32}[arch]
+    return B * {0: 16 * 16 * 16, 1: 64 * 16 * 16, 2: 64 * 32 * 32, 3: 64 * 32 * 32}[arch]
 
 
 def cut_shape(arch: int):
-    return {0: (16, 16, 16), 1: (64, 16, 16), 2: (64, 32, 32)}[arch]
+    return {0: (16, 16, 16), 1: (64, 16, 16), 2: (64, 32, 32), 3: (64, 32, 32)}[arch]
 
 
 def fuse_arrays(q, theta):

@@ -40,9 +40,10 @@
 #include <omp.h>
 #endif
 
-/* the CIFAR ResNet-18 split model (architecture 2), gcpsl_resnet.c */
-int64_t orn_num_params(int segment);
-int orn_forward_backward_masks(int bf16, double label_smoothing, const double* params,
+/* the CIFAR ResNet-18 split model (architectures 2 and 3: 10 and 100
+ * classes), gcpsl_resnet.c */
+int64_t orn_num_params(int J, int segment);
+int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const double* params,
                                double* bn_state, int B, const double* x,
                                const int32_t* labels, double* loss_out, double* grad,
                                double* cut_act, double* cut_grad, double* logits_out,
@@ -50,6 +51,7 @@ int orn_forward_backward_masks(int bf16, double label_smoothing, const double* p
 int64_t orn_mask_elems(void);
 void orn_init_bn_state(double* state);
 #define ORC_RESNET18 2
+#define ORC_RESNET18_C100 3
 
 #define ORC_OK 0
 #define ORC_EINVAL 1
@@ -175,8 +177,13 @@ static void get_offs(const arch_t* a, offs_t* o) {
   o->p_total = p;
 }
 
+/* classes of a ResNet-18 architecture id, 0 for any other id */
+static int resnet_classes(int arch) {
+  return arch == ORC_RESNET18 ? 10 : arch == ORC_RESNET18_C100 ? 100 : 0;
+}
+
 int64_t orc_num_params(int arch, int segment) {
-  if (arch == ORC_RESNET18) return orn_num_params(segment);
+  if (resnet_classes(arch)) return orn_num_params(resnet_classes(arch), segment);
   arch_t a; offs_t o;
   if (get_arch(arch, &a)) return -1;
   get_offs(&a, &o);
@@ -540,7 +547,8 @@ typedef struct {
   int64_t ncut;
   work_t w;
   double* xbuf; int32_t* ybuf;
-  int resnet;                                 /* architecture 2 */
+  int resnet;                                 /* architecture 2 or 3 */
+  int J;                                      /* classes */
   uint8_t* relu_rec;                          /* [C][B][E] ReLU records of the last round */
   uint8_t* relu_in;                           /* [C][B][E] decisions to replay next round */
   int replay;
@@ -563,13 +571,15 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   *out = NULL;
   arch_t a;
   memset(&a, 0, sizeof(a));
-  const int resnet = arch == ORC_RESNET18;
+  const int resnet = resnet_classes(arch) != 0;
   if (!resnet && get_arch(arch, &a)) return ORC_EUNSUPPORTED;
+  const int J = resnet ? resnet_classes(arch) : a.fc_out;
   if (K <= 0 || C <= 0 || B <= 0 || F < -1 || n <= 0 || !assignment || !images || !labels ||
       !owner || !init_params)
     return ORC_EINVAL;
   for (int k = 0; k < K; ++k) if (assignment[k] < -1 || assignment[k] >= C) return ORC_EINVAL;
-  for (int64_t i = 0; i < n; ++i) if (owner[i] < 0 || owner[i] >= K) return ORC_EINVAL;
+  for (int64_t i = 0; i < n; ++i)
+    if (owner[i] < 0 || owner[i] >= K || labels[i] < 0 || labels[i] >= J) return ORC_EINVAL;
   orc_ctx* c = (orc_ctx*)calloc(1, sizeof(orc_ctx));
   if (!c) return ORC_ENOMEM;
   c->arch = arch; c->bf16 = bf16; c->K = K; c->C = C; c->B = B; c->F = F;
@@ -577,11 +587,12 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   c->lr = lr; c->momentum = momentum; c->wd = wd; c->ls = label_smoothing; c->seed = seed;
   c->a = a;
   c->resnet = resnet;
+  c->J = J;
   if (resnet) {
     memset(&c->o, 0, sizeof(c->o));
-    c->o.p_client = orn_num_params(0);
-    c->o.p_total = c->o.p_client + orn_num_params(1);
-    c->S = orn_num_params(2);
+    c->o.p_client = orn_num_params(J, 0);
+    c->o.p_total = c->o.p_client + orn_num_params(J, 1);
+    c->S = orn_num_params(J, 2);
   } else {
     get_offs(&a, &c->o);
   }
@@ -785,7 +796,7 @@ int orc_step(orc_ctx* c) {
         memcpy(bn_keep, c->bn + k * c->S, sizeof(double) * (size_t)c->S);
       }
       int rc = orn_forward_backward_masks(
-          c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B, c->xbuf, c->ybuf, &c->loss[k],
+          c->J, c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B, c->xbuf, c->ybuf, &c->loss[k],
           c->grad + k * P, c->cut_act + k * c->ncut, c->cut_grad + k * c->ncut, NULL,
           c->replay ? c->relu_in + (int64_t)k * B * E : NULL, c->relu_rec + (int64_t)k * B * E);
       if (bn_keep) {

@@ -2,7 +2,7 @@
  * gcpsl_resnet.c -- the CIFAR ResNet-18 split model of the CPU oracle.
  *
  * TEST INFRASTRUCTURE ONLY, like gcpsl_oracle.c (which calls into this file
- * for architecture 2).  Plain fp64 loops in PyTorch's NCHW / OIHW layouts.
+ * for architectures 2 and 3).  Plain fp64 loops in PyTorch's NCHW / OIHW layouts.
  *
  * Model (the workload's split of the CIFAR ResNet-18):
  *   client: stem conv3x3 3->64 (stride 1, pad 1, no bias), GroupNorm(32), ReLU;
@@ -10,7 +10,8 @@
  *   server: stages 2-4 (128 / 256 / 512 channels, two basic blocks each, the
  *           first with stride 2 and a 1x1 stride-2 convolution + norm on the
  *           shortcut), train-mode BatchNorm; global average pool over 4x4;
- *           linear 512 -> 10 with bias.
+ *           linear 512 -> J with bias (J = 10 classes for architecture 2,
+ *           100 for architecture 3, the CIFAR-100 shape of Section V-A).
  *   basic block: out = relu(N2(conv2(relu(N1(conv1(x))))) + s),
  *                s = x, or Ns(conv_s(x)) when the shape changes.
  *   norms: x_hat = (y - mean) / sqrt(var + 1e-5), var biased, then
@@ -39,7 +40,6 @@
 #define RN_EPS 1e-5
 #define RN_BN_MOMENTUM 0.1
 #define RN_GROUPS 32
-#define RN_CLASSES 10
 
 typedef struct { int cin, cout, k, stride, hin, win; int64_t w; } rn_conv;
 typedef struct { int ch, gn; int64_t g, b; int64_t s; } rn_norm;   /* s: BN state offset */
@@ -47,6 +47,7 @@ typedef struct { rn_conv c1, c2, cs; rn_norm n1, n2, ns; int sc; } rn_block;
 typedef struct {
   rn_conv stem; rn_norm stem_n; rn_block blk[8];
   int64_t fcw, fcb, p_client, p_total, s_total;
+  int J;                                   /* classes: outputs of the linear head */
 } rn_net;
 
 static void rn_norm_at(rn_norm* n, int ch, int gn, int64_t* p, int64_t* s) {
@@ -56,8 +57,9 @@ static void rn_norm_at(rn_norm* n, int ch, int gn, int64_t* p, int64_t* s) {
   if (!gn) { n->s = *s; *s += 2 * ch; }
 }
 
-static void rn_build(rn_net* n) {
+static void rn_build(rn_net* n, int J) {
   int64_t p = 0, s = 0;
+  n->J = J;
   n->stem = (rn_conv){3, 64, 3, 1, 32, 32, p}; p += 64 * 3 * 9;
   rn_norm_at(&n->stem_n, 64, 1, &p, &s);
   const int widths[4] = {64, 128, 256, 512};
@@ -79,15 +81,16 @@ static void rn_build(rn_net* n) {
       if (st == 0 && j == 1) n->p_client = p;
       cin = cout; hw = ho;
     }
-  n->fcw = p; p += RN_CLASSES * 512;
-  n->fcb = p; p += RN_CLASSES;
+  n->fcw = p; p += (int64_t)J * 512;
+  n->fcb = p; p += J;
   n->p_total = p;
   n->s_total = s;
 }
 
-int64_t orn_num_params(int segment) {
+int64_t orn_num_params(int J, int segment) {
   rn_net n;
-  rn_build(&n);
+  if (J < 2) return -1;
+  rn_build(&n, J);
   if (segment == 0) return n.p_client;
   if (segment == 1) return n.p_total - n.p_client;
   if (segment == 2) return n.s_total;
@@ -340,17 +343,17 @@ static void mask_scatter(uint8_t* rec, int64_t tot, int64_t off, int64_t per, in
  * B examples x [B][3][32][32].  bn_state (nullable) is updated with this
  * batch's statistics.  cut_act / cut_grad (nullable) receive the client
  * output [B][64][32][32] and the gradient with respect to it. */
-int orn_forward_backward_masks(int bf16, double label_smoothing, const double* params,
+int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const double* params,
                                double* bn_state, int B, const double* x,
                                const int32_t* labels, double* loss_out, double* grad,
                                double* cut_act, double* cut_grad, double* logits_out,
                                const uint8_t* masks_in, uint8_t* masks_out);
 
-int orn_forward_backward(int bf16, double label_smoothing, const double* params,
+int orn_forward_backward(int J, int bf16, double label_smoothing, const double* params,
                          double* bn_state, int B, const double* x, const int32_t* labels,
                          double* loss_out, double* grad, double* cut_act, double* cut_grad,
                          double* logits_out) {
-  return orn_forward_backward_masks(bf16, label_smoothing, params, bn_state, B, x, labels,
+  return orn_forward_backward_masks(J, bf16, label_smoothing, params, bn_state, B, x, labels,
                                     loss_out, grad, cut_act, cut_grad, logits_out, NULL, NULL);
 }
 
@@ -358,7 +361,7 @@ int orn_forward_backward(int bf16, double label_smoothing, const double* params,
  * the block output, NCHW; returns the byte count per example. */
 int64_t orn_mask_elems(void) {
   rn_net n;
-  rn_build(&n);
+  rn_build(&n, 10);   /* the ReLU layers do not depend on the class count */
   int64_t e = 64 * 1024;
   for (int i = 0; i < 8; ++i) {
     const int ho = out_hw(&n.blk[i].c1);
@@ -372,14 +375,16 @@ int64_t orn_mask_elems(void) {
  * block 0 out, ...; bits as in norm_fwd), and masks_in (nullable) replaces
  * the sign tests by the given decisions (bit 0), so that a run can follow
  * another run's (e.g. the GPU's) branches exactly. */
-int orn_forward_backward_masks(int bf16, double label_smoothing, const double* params,
+int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const double* params,
                                double* bn_state, int B, const double* x,
                                const int32_t* labels, double* loss_out, double* grad,
                                double* cut_act, double* cut_grad, double* logits_out,
                                const uint8_t* masks_in, uint8_t* masks_out) {
   rn_net n;
-  rn_build(&n);
-  if (B <= 0) return 1;
+  if (B <= 0 || J < 2) return 1;
+  rn_build(&n, J);
+  for (int b = 0; b < B; ++b)
+    if (labels[b] < 0 || labels[b] >= J) return 1;
   const int64_t P = n.p_total;
   double* wr = (double*)malloc(sizeof(double) * (size_t)P);
   if (!wr) return 2;
@@ -394,7 +399,7 @@ int orn_forward_backward_masks(int bf16, double label_smoothing, const double* p
     }
     for (int i = 0; i < nc; ++i)
       rn_round(wr + cs[i]->w, (int64_t)cs[i]->cout * cs[i]->cin * cs[i]->k * cs[i]->k, bf16);
-    rn_round(wr + n.fcw, RN_CLASSES * 512, bf16);
+    rn_round(wr + n.fcw, (int64_t)J * 512, bf16);
   }
   const int64_t in_n = (int64_t)B * 3 * 1024;
   double* x0 = (double*)zal(in_n);
@@ -490,25 +495,25 @@ int orn_forward_backward_masks(int bf16, double label_smoothing, const double* p
   rn_round(h, (int64_t)B * 512, bf16);
   const double* Wfc = wr + n.fcw;
   const double* bfc = wr + n.fcb;
-  double* logits = (double*)zal((int64_t)B * RN_CLASSES);
-  double* dlog = (double*)zal((int64_t)B * RN_CLASSES);
+  double* logits = (double*)zal((int64_t)B * J);
+  double* dlog = (double*)zal((int64_t)B * J);
   double loss = 0.0;
   for (int b = 0; b < B; ++b) {
-    double* z = logits + b * RN_CLASSES;
-    for (int j = 0; j < RN_CLASSES; ++j) {
+    double* z = logits + b * J;
+    for (int j = 0; j < J; ++j) {
       double s = bfc[j];
       for (int k = 0; k < 512; ++k) s += h[b * 512 + k] * Wfc[j * 512 + k];
       z[j] = s;
     }
     double m = z[0];
-    for (int j = 1; j < RN_CLASSES; ++j) m = z[j] > m ? z[j] : m;
+    for (int j = 1; j < J; ++j) m = z[j] > m ? z[j] : m;
     double se = 0.0;
-    for (int j = 0; j < RN_CLASSES; ++j) se += exp(z[j] - m);
+    for (int j = 0; j < J; ++j) se += exp(z[j] - m);
     const double lse = m + log(se);
-    for (int j = 0; j < RN_CLASSES; ++j) {
-      const double t = (j == labels[b] ? 1.0 - label_smoothing : 0.0) + label_smoothing / RN_CLASSES;
+    for (int j = 0; j < J; ++j) {
+      const double t = (j == labels[b] ? 1.0 - label_smoothing : 0.0) + label_smoothing / J;
       loss += t * (lse - z[j]);
-      dlog[b * RN_CLASSES + j] = (exp(z[j] - lse) - t) / B;
+      dlog[b * J + j] = (exp(z[j] - lse) - t) / B;
     }
   }
   *loss_out = loss / B;
@@ -519,19 +524,19 @@ int orn_forward_backward_masks(int bf16, double label_smoothing, const double* p
       mask_scatter(masks_out, mtot, moff[2 + 2 * i], mper[2 + 2 * i], B, sv[i].m2);
     }
   }
-  if (logits_out) memcpy(logits_out, logits, sizeof(double) * (size_t)B * RN_CLASSES);
+  if (logits_out) memcpy(logits_out, logits, sizeof(double) * (size_t)B * J);
   if (cut_act) memcpy(cut_act, sv[1].out, sizeof(double) * (size_t)stem_n);
 
   int rc = 0;
   if (grad) {
     memset(grad, 0, sizeof(double) * (size_t)P);
-    for (int j = 0; j < RN_CLASSES; ++j) {
+    for (int j = 0; j < J; ++j) {
       double sb = 0.0;
-      for (int b = 0; b < B; ++b) sb += dlog[b * RN_CLASSES + j];
+      for (int b = 0; b < B; ++b) sb += dlog[b * J + j];
       grad[n.fcb + j] = sb;
       for (int k = 0; k < 512; ++k) {
         double s = 0.0;
-        for (int b = 0; b < B; ++b) s += dlog[b * RN_CLASSES + j] * h[b * 512 + k];
+        for (int b = 0; b < B; ++b) s += dlog[b * J + j] * h[b * 512 + k];
         grad[n.fcw + j * 512 + k] = s;
       }
     }
@@ -541,7 +546,7 @@ int orn_forward_backward_masks(int bf16, double label_smoothing, const double* p
     for (int b = 0; b < B; ++b)
       for (int c = 0; c < 512; ++c) {
         double s = 0.0;
-        for (int j = 0; j < RN_CLASSES; ++j) s += dlog[b * RN_CLASSES + j] * Wfc[j * 512 + c];
+        for (int j = 0; j < J; ++j) s += dlog[b * J + j] * Wfc[j * 512 + c];
         for (int p = 0; p < 16; ++p) dout[((int64_t)b * 512 + c) * 16 + p] = s / 16.0;
       }
     rn_round(dout, last_n, bf16);
@@ -617,7 +622,7 @@ int orn_forward_backward_masks(int bf16, double label_smoothing, const double* p
 /* initial BatchNorm state: running_mean 0, running_var 1 (PyTorch) */
 void orn_init_bn_state(double* state) {
   rn_net n;
-  rn_build(&n);
+  rn_build(&n, 10);   /* the BatchNorm layers do not depend on the class count */
   const rn_norm* all[3 * 8];
   int k = 0;
   for (int i = 0; i < 8; ++i) {

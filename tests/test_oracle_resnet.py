@@ -1,4 +1,5 @@
-"""Pins of the oracle's ResNet-18 split (architecture 2) against PyTorch's
+"""Pins of the oracle's ResNet-18 split (architectures 2 and 3, 10- and
+100-way heads) against PyTorch's
 fp64 autograd, written here from the module definitions (conv2d,
 group_norm, batch_norm in training mode, relu, avg_pool2d, linear,
 cross_entropy) -- none of the oracle's code.  CPU only."""
@@ -11,14 +12,15 @@ import oracle
 from paper_2609_29395_gb300 import synth
 
 RES = synth.ARCH_RESNET18
+RES100 = synth.ARCH_RESNET18_C100
 
 
-def torch_model(blob, x, y, bn_state, label_smoothing=0.0):
+def torch_model(blob, x, y, bn_state, label_smoothing=0.0, arch=RES):
     """Loss, parameter tensors (requires_grad), cut activation (retained
     grad), logits and the BatchNorm state after the batch, with the blob in
     PyTorch's named_parameters() order."""
-    names = [n for n, _ in synth.param_shapes(RES, "client") + synth.param_shapes(RES, "server")]
-    shapes = [s for _, s in synth.param_shapes(RES, "client") + synth.param_shapes(RES, "server")]
+    names = [n for n, _ in synth.param_shapes(arch, "client") + synth.param_shapes(arch, "server")]
+    shapes = [s for _, s in synth.param_shapes(arch, "client") + synth.param_shapes(arch, "server")]
     prm, off = {}, 0
     for n, s in zip(names, shapes):
         k = int(np.prod(s))
@@ -67,23 +69,33 @@ def torch_model(blob, x, y, bn_state, label_smoothing=0.0):
     return loss, [prm[n] for n in names], cut, logits, state.numpy()
 
 
-@pytest.fixture(scope="module")
-def case():
+def make_case(arch, labels):
     rng = np.random.default_rng(11)
-    blob = synth.init_params(RES, seed=7).astype(np.float64)
+    blob = synth.init_params(arch, seed=7).astype(np.float64)
     # non-trivial norm affine parameters
     off = 0
-    for name, shape in synth.param_shapes(RES, "client") + synth.param_shapes(RES, "server"):
+    for name, shape in synth.param_shapes(arch, "client") + synth.param_shapes(arch, "server"):
         k = int(np.prod(shape))
         if len(shape) == 1 and name != "linear.bias":
             blob[off:off + k] += rng.normal(0, 0.2, k)
         off += k
-    B = 3
+    B = len(labels)
     x = rng.normal(size=(B, 3, 32, 32))
-    y = rng.integers(0, 10, size=B).astype(np.int32)
+    y = np.asarray(labels, dtype=np.int32)
     bn0 = oracle.initial_bn_state()
     bn0[:] += rng.uniform(0.0, 0.5, bn0.size)
     return blob, x, y, bn0
+
+
+@pytest.fixture(scope="module")
+def case():
+    return make_case(RES, [3, 9, 0])
+
+
+@pytest.fixture(scope="module")
+def case100():
+    # labels beyond the first ten rows of the head
+    return make_case(RES100, [57, 3, 99])
 
 
 def test_resnet_param_count_and_state_size():
@@ -110,6 +122,58 @@ def test_resnet_matches_torch_fp64_autograd(case, ls):
     scale = np.abs(tgrad).max()
     np.testing.assert_allclose(grad, tgrad, rtol=0, atol=1e-10 * scale)
     np.testing.assert_allclose(bn1, tstate, rtol=0, atol=1e-12)
+
+
+def test_resnet100_param_count():
+    assert oracle.num_params(RES100, 0) == oracle.num_params(RES, 0) == 149824
+    assert oracle.num_params(RES100, 1) == synth.num_params(RES100, "server") == \
+        oracle.num_params(RES, 1) + 90 * 512 + 90
+
+
+@pytest.mark.parametrize("ls", [0.0, 0.1])
+def test_resnet100_matches_torch_fp64_autograd(case100, ls):
+    """The 100-way head (architecture 3) against PyTorch's linear +
+    cross_entropy with its 100 classes, label smoothing spread over all 100."""
+    blob, x, y, bn0 = case100
+    loss, grad, ca, cg, logits, bn1 = oracle.resnet_forward_backward(
+        blob, x, y, bn_state=bn0, label_smoothing=ls, classes=100)
+    tl, tparams, tcut, tlogits, tstate = torch_model(blob, torch.tensor(x), y, bn0, ls,
+                                                     arch=RES100)
+    tl.backward()
+    tgrad = np.concatenate([p.grad.numpy().ravel() for p in tparams])
+    assert logits.shape == (3, 100)
+    assert abs(loss - tl.item()) < 1e-12 * max(1.0, abs(loss))
+    np.testing.assert_allclose(logits, tlogits.detach().numpy(), rtol=0, atol=1e-11)
+    np.testing.assert_allclose(cg, tcut.grad.numpy().ravel(), rtol=0,
+                               atol=1e-12 * np.abs(cg).max())
+    np.testing.assert_allclose(grad, tgrad, rtol=0, atol=1e-10 * np.abs(tgrad).max())
+    np.testing.assert_allclose(bn1, tstate, rtol=0, atol=1e-12)
+
+
+def test_resnet100_zero_head_closed_form(case100):
+    """Zero head weights and bias: every logit 0, so the loss is ln 100 with
+    or without label smoothing, the bias gradient is 1/100 - mean_b t_b (t
+    the smoothed target), and the cut gradient vanishes."""
+    blob, x, y, bn0 = case100
+    z = blob.copy()
+    off = oracle.num_params(RES100, 0) + oracle.num_params(RES100, 1) - 100 * 512 - 100
+    z[off:] = 0.0
+    for ls in (0.0, 0.1):
+        l0, g, _ca, cg, logits, _ = oracle.resnet_forward_backward(
+            z, x, y, bn_state=bn0, label_smoothing=ls, classes=100)
+        assert abs(l0 - np.log(100.0)) < 1e-13     # a 100-term fp64 sum
+        assert np.abs(logits).max() == 0.0
+        assert np.abs(cg).max() == 0.0
+        want_db = np.full(100, 1.0 / 100) - np.bincount(y, minlength=100) * (1.0 - ls) / len(y) \
+            - ls / 100
+        np.testing.assert_allclose(g[-100:], want_db, rtol=0, atol=1e-15)
+
+
+def test_resnet100_rejects_labels_outside_the_head(case100):
+    blob, x, y, bn0 = case100
+    with pytest.raises(RuntimeError):
+        oracle.resnet_forward_backward(blob[:oracle.num_params(RES, 0) + oracle.num_params(RES, 1)],
+                                       x, y, bn_state=bn0, classes=10)
 
 
 def test_resnet_finite_differences(case):
