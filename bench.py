@@ -96,6 +96,9 @@ def load_peaks():
 # algorithmic work per kernel kind and round (FLOPs for contractions, bytes
 # for the elementwise/bandwidth kernels)
 # ---------------------------------------------------------------------------
+ARCH_NAMES = {1: "SplitCNN", 2: "ResNet-18 split", 3: "ResNet-18 split, 100 classes"}
+
+
 def work_per_round_resnet(w):
     """Kernel kinds of the ResNet-18 split (per stage) and their FLOPs per
     round: 2*C*B*Ho*Wo*cout*cin*k*k per convolution and pass (the stem has
@@ -164,7 +167,7 @@ def work_per_round_resnet(w):
 
 def work_per_round(w, esz):
     from paper_2609_29395_gb300 import synth
-    if w.arch == synth.ARCH_RESNET18:
+    if w.arch in synth.RESNET_ARCHS:
         return work_per_round_resnet(w)
     spec = synth.ARCHS[w.arch]
     convs = spec["client"] + spec["server"]
@@ -275,10 +278,12 @@ class ClockSampler:
 def _oracle_pass(oracle, w, blob, x, y):
     """One forward+backward of the oracle on one replica's batch."""
     from paper_2609_29395_gb300 import synth
-    if w.arch == synth.ARCH_RESNET18:
-        oracle.resnet_forward_backward(blob, x, y, bf16=w.bf16)
+    if w.arch in synth.RESNET_ARCHS:
+        oracle.resnet_forward_backward(blob, x, y, bf16=w.bf16, classes=w.num_classes,
+                                       label_smoothing=w.label_smoothing)
     else:
-        oracle.forward_backward(w.arch, blob, x, y, bf16=w.bf16)
+        oracle.forward_backward(w.arch, blob, x, y, bf16=w.bf16,
+                                label_smoothing=w.label_smoothing)
 
 
 def cpu_baseline(w, ds, assign, params, budget_s=15.0):
@@ -362,7 +367,7 @@ def main():
 
     ds, assign, params = configs.build_inputs(w)
     ctx = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
-                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=w.bf16)
+                      ds.labels, ds.owner, params, bf16=w.bf16, **w.options())
     # a dedicated stream: the library, the events and the L2 flush all use it
     stream = torch.cuda.Stream()
     torch.cuda.set_stream(stream)
@@ -465,7 +470,7 @@ def main():
         "data": "synthetic",
         "config": {"workload": f"{w.name}: n={w.n} K={w.num_clients} C={w.num_clusters} "
                                f"B={w.B} F={w.F} "
-                               f"{ {1: 'SplitCNN', 2: 'ResNet-18 split'}.get(w.arch, '')}",
+                               f"{ARCH_NAMES.get(w.arch, '')}",
                    "global_batch": w.num_clusters * w.B * world, "parallelism": f"replicas{world}",
                    "l2": "flushed between timed steps (256 MiB write)"},
         "roofline": roof, "gpu_launches": launches, "wall_s": wall,
@@ -503,8 +508,8 @@ def e2e_leg(pkg, w, ds, assign, params, torch, flush, K):
     host memory over NVLink-C2C and returns the per-cluster loss and |A| to
     the host (gcpsl_step with stats, which synchronises)."""
     ctx = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
-                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=w.bf16,
-                      data_on_host=True)
+                      ds.labels, ds.owner, params, bf16=w.bf16, data_on_host=True,
+                      **w.options())
     for _ in range(3):
         ctx.step(stats=True)
     tot = 0.0
@@ -525,8 +530,8 @@ def serialized_leg(pkg, w, ds, assign, params, torch, flush, K, grouped_value):
     """The paper's sequential control on one GPU: the C workloads as C
     one-cluster contexts stepped one after another (same kernels)."""
     ctxs = [pkg.Context(w.arch, w.num_clients, 1, np.where(assign == n, 0, -1).astype(np.int32),
-                        w.B, 0, 4, ds.images, ds.labels, ds.owner, params, lr=w.lr,
-                        momentum=w.momentum, bf16=w.bf16, cluster_id_base=n)
+                        w.B, 0, 4, ds.images, ds.labels, ds.owner, params, bf16=w.bf16,
+                        cluster_id_base=n, **w.options())
             for n in range(w.num_clusters)]
     stream = torch.cuda.current_stream()
     for c in ctxs:

@@ -45,8 +45,14 @@ typedef enum {
  * bias, each followed by ReLU; "pool" is a 2x2 stride-2 max-pool.
  *  TINY_CNN : client conv 3->16 pool | server conv 16->32 pool, FC 2048->10
  *  SPLIT_CNN: client conv 3->32, conv 32->64 pool (cut 64x16x16) |
- *             server conv 64->128 pool, conv 128->128 pool, FC 2048->10   */
-enum { GCPSL_TINY_CNN = 0, GCPSL_SPLIT_CNN = 1, GCPSL_RESNET18 = 2 };
+ *             server conv 64->128 pool, conv 128->128 pool, FC 2048->10
+ *  RESNET18 : the CIFAR ResNet-18 split after stage 1 (Section V-A): client
+ *             conv3x3 3->64 stem + GroupNorm(32) + ReLU, stage 1 (two basic
+ *             blocks of 64 channels, GroupNorm) (cut 64x32x32) | server
+ *             stages 2-4 (128/256/512 channels, stride 2, train-mode
+ *             BatchNorm), global average pool, FC 512->10; no conv bias
+ *  RESNET18_C100: the same split with FC 512->100 (the CIFAR-100 shape)   */
+enum { GCPSL_TINY_CNN = 0, GCPSL_SPLIT_CNN = 1, GCPSL_RESNET18 = 2, GCPSL_RESNET18_C100 = 3 };
 enum { GCPSL_F32 = 0, GCPSL_BF16 = 1 };
 enum { GCPSL_CLIENT = 0, GCPSL_SERVER = 1, GCPSL_BN_STATE = 2 };
 enum { GCPSL_CUT_ACT = 0, GCPSL_CUT_GRAD = 1 };
@@ -92,7 +98,7 @@ typedef struct {
   const int32_t* labels;
   const int32_t* owner;
   int64_t n;
-  int num_classes;        /* must be 10 for the built architectures */
+  int num_classes;        /* the architecture's: 100 for RESNET18_C100, else 10 */
 } gcpsl_dataset;
 
 /* Per-round statistics, written by gcpsl_step when non-NULL (forces a sync).
@@ -127,8 +133,9 @@ typedef struct gcpsl_ctx gcpsl_ctx;
  *    Philox stream as U(-1/sqrt(fan_in), 1/sqrt(fan_in));
  *  out: receives the context.
  * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < -1, assignment
- * outside [-1, C), owner outside [0, K), labels outside [0, classes), a
- * cluster with fewer than B examples.  Fusion weights are
+ * outside [-1, C), owner outside [0, K), num_classes other than the
+ * architecture's, labels outside [0, num_classes), a cluster with fewer
+ * than B examples.  Fusion weights are
  * q_n = n_c / sum_m n_m over this context's clusters (Eq. 5).            */
 gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_t* assignment,
                         int B, int F, uint64_t seed, const gcpsl_dataset* data,

@@ -36,7 +36,7 @@ def main() -> int:
         w = dataclasses.replace(w, num_clusters=args.clusters)
     ds, assign, params = configs.build_inputs(w)
     ctx = Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
-                  ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=w.bf16)
+                  ds.labels, ds.owner, params, bf16=w.bf16, **w.options())
     if args.eager:
         ctx.set_graph(False)
     t0 = time.perf_counter()

@@ -16,7 +16,7 @@ LIB_PATH = Path(__file__).resolve().parent / "lib" / "libgcpsl.so"
 
 GCPSL_OK, GCPSL_E_INVAL, GCPSL_E_NOMEM, GCPSL_E_CUDA, GCPSL_E_STATE, GCPSL_E_TIMEOUT, \
     GCPSL_E_UNSUPPORTED = range(7)
-GCPSL_TINY_CNN, GCPSL_SPLIT_CNN, GCPSL_RESNET18 = 0, 1, 2
+GCPSL_TINY_CNN, GCPSL_SPLIT_CNN, GCPSL_RESNET18, GCPSL_RESNET18_C100 = 0, 1, 2, 3
 GCPSL_F32, GCPSL_BF16 = 0, 1
 GCPSL_CLIENT, GCPSL_SERVER, GCPSL_BN_STATE = 0, 1, 2
 GCPSL_CUT_ACT, GCPSL_CUT_GRAD = 0, 1
@@ -132,6 +132,11 @@ def _check(st, h=None):
 
 
 # C-ABI names, argument marshalling only ----------------------------------
+def num_classes(arch: int) -> int:
+    """Classes of an architecture's linear head (the dataset's num_classes)."""
+    return 100 if arch == GCPSL_RESNET18_C100 else 10
+
+
 def gcpsl_num_params(arch: int, segment: int) -> int:
     return int(load().gcpsl_num_params(arch, segment))
 
@@ -168,7 +173,7 @@ class Context:
         owner = np.ascontiguousarray(owner, dtype=np.int32)
         assignment = np.ascontiguousarray(assignment, dtype=np.int32)
         ds = gcpsl_dataset(_p(images, ct.c_float), _p(labels, ct.c_int32),
-                           _p(owner, ct.c_int32), images.shape[0], 10)
+                           _p(owner, ct.c_int32), images.shape[0], num_classes(arch))
         init = None
         if init_params is not None:
             init = np.ascontiguousarray(init_params, dtype=np.float32)

@@ -167,7 +167,9 @@ cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_r
                              const float* b, int64_t b_rs, const int32_t* y, float* loss_ex,
                              float* dlogits, int C, int B, int fin, int fout,
                              float label_smoothing);
-// backward of the linear layer (dW, db, dh) and loss[c] = mean_b loss_ex[c][b].
+// backward of the linear layer (dW, db, dh) and loss[c] = mean_b loss_ex[c][b];
+// fout = 10 or 100 classes.  When fc_bwd_split_dh(fout), this launch writes
+// dW, db and loss only, and launch_fc_bwd_dh (same route arguments) writes dh.
 // route: FC_DH_STORE writes dh; FC_DH_POOL writes the last conv layer's g
 // (2Ho x 2Wo x ch) through its max-pool codes; FC_DH_RELU writes g = dh where
 // act > 0; FC_DH_AVG writes dh / (Ho Wo) to every pixel of an Ho x Wo x ch
@@ -178,6 +180,11 @@ cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* los
                           const T* h, const T* w, int64_t w_rs, float* dw, float* db,
                           int64_t g_rs, T* dh, float* loss, int C, int B, int fin, int fout,
                           int route, const uint8_t* code, const T* act, int Ho, int Wo, int ch);
+bool fc_bwd_split_dh(int fout);
+template <typename T>
+cudaError_t launch_fc_bwd_dh(cudaStream_t s, const float* dlogits, const T* w, int64_t w_rs,
+                             T* dh, int C, int B, int fin, int fout, int route,
+                             const uint8_t* code, const T* act, int Ho, int Wo, int ch);
 
 // conv_tc.cu (tensor-core convolutions, bf16 operands)
 enum {

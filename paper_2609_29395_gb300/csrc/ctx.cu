@@ -46,6 +46,18 @@ bool gcpsl::make_arch(int id, ArchSpec* a) {
 
 namespace {
 
+// classes of a ResNet-18 split architecture, 0 for any other id
+int resnet_classes(int arch) {
+  return arch == GCPSL_RESNET18 ? 10 : arch == GCPSL_RESNET18_C100 ? 100 : 0;
+}
+
+// classes of any built architecture, 0 for an unknown id
+int arch_classes(int arch) {
+  if (resnet_classes(arch)) return resnet_classes(arch);
+  ArchSpec a;
+  return make_arch(arch, &a) ? a.fc_out : 0;
+}
+
 thread_local std::string g_init_error;
 
 }  // namespace
@@ -160,11 +172,11 @@ gcpsl_status refresh_derived(gcpsl_ctx* c) {
 
 // canonical <-> kernel parameter layout of the context's architecture
 void to_kernel(const gcpsl_ctx* c, const float* can, float* ker) {
-  if (c->rn) rn_to_kernel_layout(can, ker);
+  if (c->rn) rn_to_kernel_layout(c->J, can, ker);
   else to_kernel_layout(c->a, can, ker);
 }
 void to_canonical(const gcpsl_ctx* c, const float* ker, float* can) {
-  if (c->rn) rn_to_canonical_layout(ker, can);
+  if (c->rn) rn_to_canonical_layout(c->J, ker, can);
   else to_canonical_layout(c->a, ker, can);
 }
 
@@ -652,8 +664,10 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   c->esz = c->bf ? 2 : 4;
   c->x0c = c->bf ? 32 : 3;
   const ArchSpec& a = c->a;
-  const bool resnet = desc->arch == GCPSL_RESNET18;
-  c->P = resnet ? rn_num_params(GCPSL_CLIENT) + rn_num_params(GCPSL_SERVER) : a.p_total;
+  const bool resnet = resnet_classes(desc->arch) != 0;
+  c->J = data->num_classes;
+  c->P = resnet ? rn_num_params(c->J, GCPSL_CLIENT) + rn_num_params(c->J, GCPSL_SERVER)
+                : a.p_total;
   c->n = data->n;
 
   // clusters: ascending example ids per cluster, r_n, q_n (Eq. 5)
@@ -728,9 +742,9 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   // parameters: C identical replicas
   std::vector<float> can(c->P), ker(c->P);
   if (init_params) std::memcpy(can.data(), init_params, sizeof(float) * c->P);
-  else if (resnet) rn_seeded_init(seed, can.data());
+  else if (resnet) rn_seeded_init(c->J, seed, can.data());
   else seeded_init(a, seed, can.data());
-  if (resnet) rn_to_kernel_layout(can.data(), ker.data());
+  if (resnet) rn_to_kernel_layout(c->J, can.data(), ker.data());
   else to_kernel_layout(a, can.data(), ker.data());
   c->P_pad = (c->P + 63) / 64 * 64;
   const size_t pb = sizeof(float) * (size_t)(C * c->P_pad);
@@ -760,7 +774,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     DALLOC(c->d_act[0], sizeof(bf16) * (size_t)C * B * 1024 * 32);
     DALLOC(c->d_w0p, sizeof(bf16) * (size_t)C * 64 * 32);
     DALLOC(c->d_loss_ex, sizeof(float) * C * B);
-    DALLOC(c->d_dlogits, sizeof(float) * C * B * 10);
+    DALLOC(c->d_dlogits, sizeof(float) * C * B * c->J);
     DALLOC(c->d_y, sizeof(int32_t) * C * B);
     DALLOC(c->d_idx, sizeof(int32_t) * C * B);
     DALLOC(c->d_counts, sizeof(int32_t) * (size_t)C * K);
@@ -845,7 +859,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
 extern "C" {
 
 int64_t gcpsl_num_params(int arch, int segment) {
-  if (arch == GCPSL_RESNET18) return rn_num_params(segment);
+  if (resnet_classes(arch)) return rn_num_params(resnet_classes(arch), segment);
   ArchSpec a;
   if (!make_arch(arch, &a)) return -1;
   if (segment == GCPSL_CLIENT) return a.p_client;
@@ -864,8 +878,6 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
   if (K <= 0 || C <= 0 || B <= 0 || B > 1024 || F < -1 || data->n <= 0 || data->n > INT32_MAX)
     return fail(nullptr, GCPSL_E_INVAL, "bad size (K=%d C=%d B=%d F=%d n=%lld)", K, C, B, F,
                 (long long)data->n);
-  if (data->num_classes != 10)
-    return fail(nullptr, GCPSL_E_INVAL, "num_classes must be 10");
   if (desc->operand_dtype != GCPSL_F32 && desc->operand_dtype != GCPSL_BF16)
     return fail(nullptr, GCPSL_E_INVAL, "unknown operand_dtype %d", desc->operand_dtype);
   if (desc->augment != 0 && desc->augment != 1)
@@ -874,12 +886,15 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
     return fail(nullptr, GCPSL_E_INVAL, "bad lr or label_smoothing");
   ArchSpec a;
   std::memset(&a, 0, sizeof(a));
-  if (desc->arch == GCPSL_RESNET18) {
+  if (resnet_classes(desc->arch)) {
     if (desc->operand_dtype != GCPSL_BF16)
       return fail(nullptr, GCPSL_E_UNSUPPORTED, "the ResNet-18 split runs with bf16 operands");
   } else if (!make_arch(desc->arch, &a)) {
     return fail(nullptr, GCPSL_E_UNSUPPORTED, "architecture %d is not built", desc->arch);
   }
+  if (data->num_classes != arch_classes(desc->arch))
+    return fail(nullptr, GCPSL_E_INVAL, "num_classes=%d, architecture %d has %d", data->num_classes,
+                desc->arch, arch_classes(desc->arch));
   for (int k = 0; k < K; ++k)
     if (assignment[k] < -1 || assignment[k] >= C)
       return fail(nullptr, GCPSL_E_INVAL, "assignment[%d]=%d outside [-1, %d)", k, assignment[k], C);
@@ -961,7 +976,7 @@ gcpsl_status gcpsl_get_params(gcpsl_ctx* c, int cluster, int segment, float* dst
     CK(cudaMemcpy(dst, bn + (int64_t)cluster * S_pad, sizeof(float) * S, cudaMemcpyDeviceToHost));
     return GCPSL_OK;
   }
-  const int64_t pc = c->rn ? rn_num_params(GCPSL_CLIENT) : c->a.p_client;
+  const int64_t pc = c->rn ? rn_num_params(c->J, GCPSL_CLIENT) : c->a.p_client;
   const int64_t lo = segment == GCPSL_CLIENT ? 0 : pc;
   const int64_t hi = segment == GCPSL_CLIENT ? pc : c->P;
   if (needed) *needed = (size_t)(hi - lo);

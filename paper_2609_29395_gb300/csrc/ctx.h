@@ -101,6 +101,7 @@ struct gcpsl_ctx {
   gcpsl_model_desc desc{};
   ArchSpec a{};
   int K = 0, C = 0, B = 0, F = 0;
+  int J = 10;                       // classes (outputs of the linear head)
   uint64_t seed = 0;
   bool bf = false;
   size_t esz = 4;
@@ -237,10 +238,11 @@ namespace gcpsl {
 gcpsl_status fail(gcpsl_ctx* c, gcpsl_status st, const char* fmt, ...);
 
 // resnet.cu: the ResNet-18 split (architecture 2)
-int64_t rn_num_params(int segment);              // GCPSL_CLIENT / SERVER / BN_STATE
-void rn_to_kernel_layout(const float* can, float* ker);
-void rn_to_canonical_layout(const float* ker, float* can);
-void rn_seeded_init(uint64_t seed, float* can);
+// the ResNet-18 split with a J-way linear head (J = 10: GCPSL_RESNET18, 100: GCPSL_RESNET18_C100)
+int64_t rn_num_params(int J, int segment);       // GCPSL_CLIENT / SERVER / BN_STATE
+void rn_to_kernel_layout(int J, const float* can, float* ker);
+void rn_to_canonical_layout(int J, const float* ker, float* can);
+void rn_seeded_init(int J, uint64_t seed, float* can);
 gcpsl_status rn_setup(gcpsl_ctx* c);
 void rn_free(gcpsl_ctx* c);
 gcpsl_status rn_enqueue_round(gcpsl_ctx* c);

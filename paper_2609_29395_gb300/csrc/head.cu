@@ -54,15 +54,18 @@ template <typename T> struct VecLoad<T, 1> {
 // Block = (replica c, kFwdEx consecutive examples); warp w takes the k
 // slices w, w + kFwdSlices, ... of VEC * 32 features (one slice each when
 // fin = kFwdSlices * 32 * VEC), so every load of the block is issued at
-// once.  Lane partial sums are reduced by a fixed xor tree, the warps'
-// sums in warp order; then one warp per example takes the softmax.  J is a
-// compile-time constant so the J weight loads of a slice issue together.
-template <typename T, int VEC, int J>
+// once.  The classes are taken JC at a time (JC weight rows in registers);
+// lane partial sums are reduced by a fixed xor tree, the warps' sums in
+// warp order; then one warp per example takes the softmax: with J <= 32
+// every lane reads all J logits, otherwise lane l holds the logits
+// l, l + 32, ... and max, sum and loss are xor-tree warp reductions.
+template <typename T, int VEC, int J, int JC>
 __global__ void __launch_bounds__(kFwdSlices * 32)
 k_fc_fwd_ce(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
             const float* __restrict__ bias, int64_t b_rs, const int32_t* __restrict__ y,
             float* __restrict__ loss_ex, float* __restrict__ dlogits, int C, int B, int fin,
             float eps) {
+  static_assert(J % JC == 0, "class chunks must tile J");
   __shared__ float part[kFwdSlices][kFwdEx * J];
   __shared__ float logit[kFwdEx][J];
   pdl_wait();
@@ -73,69 +76,105 @@ k_fc_fwd_ce(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const T* hp = h + ((int64_t)c * B + e0) * fin;
   const T* wp = w + (int64_t)c * w_rs;
-  float acc[kFwdEx][J];
-#pragma unroll
-  for (int e = 0; e < kFwdEx; ++e)
-#pragma unroll
-    for (int j = 0; j < J; ++j) acc[e][j] = 0.f;
-  for (int k = (warp * 32 + lane) * VEC; k < fin; k += kFwdSlices * 32 * VEC) {
-    float hv[kFwdEx][VEC], wv[J][VEC];
-#pragma unroll
-    for (int e = 0; e < kFwdEx; ++e) {
-      if (e < ne) VecLoad<T, VEC>::run(hp + (int64_t)e * fin + k, hv[e]);
-      else
-#pragma unroll
-        for (int v = 0; v < VEC; ++v) hv[e][v] = 0.f;
-    }
-#pragma unroll
-    for (int j = 0; j < J; ++j) VecLoad<T, VEC>::run(wp + (int64_t)j * fin + k, wv[j]);
+  for (int j0 = 0; j0 < J; j0 += JC) {
+    float acc[kFwdEx][JC];
 #pragma unroll
     for (int e = 0; e < kFwdEx; ++e)
 #pragma unroll
-      for (int j = 0; j < J; ++j)
+      for (int j = 0; j < JC; ++j) acc[e][j] = 0.f;
+    for (int k = (warp * 32 + lane) * VEC; k < fin; k += kFwdSlices * 32 * VEC) {
+      float hv[kFwdEx][VEC], wv[JC][VEC];
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) acc[e][j] = fmaf(hv[e][v], wv[j][v], acc[e][j]);
-  }
+      for (int e = 0; e < kFwdEx; ++e) {
+        if (e < ne) VecLoad<T, VEC>::run(hp + (int64_t)e * fin + k, hv[e]);
+        else
 #pragma unroll
-  for (int e = 0; e < kFwdEx; ++e)
+          for (int v = 0; v < VEC; ++v) hv[e][v] = 0.f;
+      }
 #pragma unroll
-    for (int j = 0; j < J; ++j) {
+      for (int j = 0; j < JC; ++j) VecLoad<T, VEC>::run(wp + (int64_t)(j0 + j) * fin + k, wv[j]);
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc[e][j] += __shfl_xor_sync(0xffffffffu, acc[e][j], o);
-      if (lane == 0) part[warp][e * J + j] = acc[e][j];
+      for (int e = 0; e < kFwdEx; ++e)
+#pragma unroll
+        for (int j = 0; j < JC; ++j)
+#pragma unroll
+          for (int v = 0; v < VEC; ++v) acc[e][j] = fmaf(hv[e][v], wv[j][v], acc[e][j]);
     }
+#pragma unroll
+    for (int e = 0; e < kFwdEx; ++e)
+#pragma unroll
+      for (int j = 0; j < JC; ++j) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc[e][j] += __shfl_xor_sync(0xffffffffu, acc[e][j], o);
+        if (lane == 0) part[warp][e * J + j0 + j] = acc[e][j];
+      }
+  }
   __syncthreads();
-  if (threadIdx.x < kFwdEx * J) {
-    const int e = threadIdx.x / J, j = threadIdx.x % J;
+  for (int i = threadIdx.x; i < kFwdEx * J; i += kFwdSlices * 32) {
+    const int e = i / J, j = i % J;
     float z = 0.f;
 #pragma unroll
-    for (int q = 0; q < kFwdSlices; ++q) z += part[q][threadIdx.x];
+    for (int q = 0; q < kFwdSlices; ++q) z += part[q][i];
     logit[e][j] = z + bias[(int64_t)c * b_rs + j];
   }
   __syncthreads();
   if (warp >= ne) return;
-  // softmax of example e0 + warp: every lane reads the J logits
-  float z[J];
-#pragma unroll
-  for (int j = 0; j < J; ++j) z[j] = logit[warp][j];
-  float m = z[0];
-#pragma unroll
-  for (int j = 1; j < J; ++j) m = fmaxf(m, z[j]);
-  float se = 0.f;
-#pragma unroll
-  for (int j = 0; j < J; ++j) se += expf(z[j] - m);
-  const float lse = m + logf(se);
   const int64_t cb = (int64_t)c * B + e0 + warp;
   const int yb = y[cb];
   const float invB = 1.f / (float)B;
-  float l = 0.f;
+  if constexpr (J <= 32) {
+    // softmax of example e0 + warp: every lane reads the J logits
+    float z[J];
 #pragma unroll
-  for (int j = 0; j < J; ++j) {
-    const float t = (j == yb ? 1.f - eps : 0.f) + eps / (float)J;
-    l += t * (lse - z[j]);
-    if (lane == j) dlogits[cb * J + j] = (expf(z[j] - lse) - t) * invB;
+    for (int j = 0; j < J; ++j) z[j] = logit[warp][j];
+    float m = z[0];
+#pragma unroll
+    for (int j = 1; j < J; ++j) m = fmaxf(m, z[j]);
+    float se = 0.f;
+#pragma unroll
+    for (int j = 0; j < J; ++j) se += expf(z[j] - m);
+    const float lse = m + logf(se);
+    float l = 0.f;
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+      const float t = (j == yb ? 1.f - eps : 0.f) + eps / (float)J;
+      l += t * (lse - z[j]);
+      if (lane == j) dlogits[cb * J + j] = (expf(z[j] - lse) - t) * invB;
+    }
+    if (lane == 0) loss_ex[cb] = l;
+  } else {
+    constexpr int NJ = (J + 31) / 32;
+    float z[NJ];
+    float m = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < NJ; ++i) {
+      const int j = lane + 32 * i;
+      z[i] = j < J ? logit[warp][j] : -INFINITY;
+      m = fmaxf(m, z[i]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    float se = 0.f;
+#pragma unroll
+    for (int i = 0; i < NJ; ++i)
+      if (lane + 32 * i < J) se += expf(z[i] - m);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+    const float lse = m + logf(se);
+    float l = 0.f;
+#pragma unroll
+    for (int i = 0; i < NJ; ++i) {
+      const int j = lane + 32 * i;
+      if (j < J) {
+        const float t = (j == yb ? 1.f - eps : 0.f) + eps / (float)J;
+        l += t * (lse - z[i]);
+        dlogits[cb * J + j] = (expf(z[i] - lse) - t) * invB;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    if (lane == 0) loss_ex[cb] = l;
   }
-  if (lane == 0) loss_ex[cb] = l;
 }
 
 // two consecutive features as floats
@@ -191,39 +230,45 @@ __device__ __forceinline__ void put_dh(T* __restrict__ out, const HeadRoute& rt,
   }
 }
 
-// grid (ceil(fin / (2 * kBwdPairs)), C).  Lane = feature pair (k, k+1),
-// warp = chunk of ceil(B / kBwdChunks) consecutive examples; the warps'
-// dW partial sums are added in warp order through shared memory.  Block
-// x == 0 also writes db (warp 0) and loss[c] (warp 1).
-template <typename T, int J>
+// grid (ceil(fin / (2 * kBwdPairs)), C, J / JC).  Lane = feature pair
+// (k, k+1), warp = chunk of ceil(B / kBwdChunks) consecutive examples,
+// blockIdx.z = the classes j0 .. j0 + JC - 1; the warps' dW partial sums are
+// added in warp order through shared memory.  Blocks with x == 0 also write
+// db of their classes (warp 0); block (0, c, 0) writes loss[c] (warp 1).
+// With DH (only when JC = J) the block also forms dh, all J classes of a
+// feature pair being in its registers; otherwise k_fc_bwd_dh does.
+template <typename T, int JC, bool DH>
 __global__ void __launch_bounds__(kBwdPairs * kBwdChunks)
 k_fc_bwd(const float* __restrict__ dlogits, const float* __restrict__ loss_ex,
          const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs, float* __restrict__ dw,
          float* __restrict__ db, int64_t g_rs, T* __restrict__ dh, float* __restrict__ loss,
-         int B, int fin, const HeadRoute rt) {
+         int B, int fin, int J, const HeadRoute rt) {
   extern __shared__ float sm[];
-  float* sdz = sm;                                 // [B][J]
-  float* red = sm + B * J;                         // [kBwdChunks][kBwdPairs][2J]
+  float* sdz = sm;                                 // [B][JC]
+  float* red = sm + B * JC;                        // [kBwdChunks][kBwdPairs][2JC]
   pdl_wait();
   pdl_trigger();
-  const int c = blockIdx.y;
+  const int c = blockIdx.y, j0 = blockIdx.z * JC;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* dz = dlogits + (int64_t)c * B * J;
-  for (int i = threadIdx.x; i < B * J; i += kBwdPairs * kBwdChunks) sdz[i] = dz[i];
+  for (int i = threadIdx.x; i < B * JC; i += kBwdPairs * kBwdChunks)
+    sdz[i] = dz[(i / JC) * J + j0 + i % JC];
   __syncthreads();
   const int k = 2 * (blockIdx.x * kBwdPairs + lane);
   const int bc = (B + kBwdChunks - 1) / kBwdChunks;
   const int b_lo = warp * bc, b_hi = b_lo + bc < B ? b_lo + bc : B;
-  float a0[J], a1[J];
+  float a0[JC], a1[JC];
 #pragma unroll
-  for (int j = 0; j < J; ++j) a0[j] = a1[j] = 0.f;
+  for (int j = 0; j < JC; ++j) a0[j] = a1[j] = 0.f;
   if (k < fin) {
-    const T* wp = w + (int64_t)c * w_rs + k;
-    float w0[J], w1[J];
+    float w0[JC], w1[JC];
+    if constexpr (DH) {
+      const T* wp = w + (int64_t)c * w_rs + k;
 #pragma unroll
-    for (int j = 0; j < J; ++j) {
-      const float2 v = load2<T>(wp + (int64_t)j * fin);
-      w0[j] = v.x; w1[j] = v.y;
+      for (int j = 0; j < JC; ++j) {
+        const float2 v = load2<T>(wp + (int64_t)j * fin);
+        w0[j] = v.x; w1[j] = v.y;
+      }
     }
     const T* hp = h + (int64_t)c * B * fin + k;
     constexpr int U = 4;
@@ -235,40 +280,42 @@ k_fc_bwd(const float* __restrict__ dlogits, const float* __restrict__ loss_ex,
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         if (b0 + u < b_hi) {
-          const float* g = sdz + (b0 + u) * J;
+          const float* g = sdz + (b0 + u) * JC;
           float d0 = 0.f, d1 = 0.f;
 #pragma unroll
-          for (int j = 0; j < J; ++j) {
+          for (int j = 0; j < JC; ++j) {
             a0[j] = fmaf(g[j], hv[u].x, a0[j]);
             a1[j] = fmaf(g[j], hv[u].y, a1[j]);
-            d0 = fmaf(g[j], w0[j], d0);
-            d1 = fmaf(g[j], w1[j], d1);
+            if constexpr (DH) {
+              d0 = fmaf(g[j], w0[j], d0);
+              d1 = fmaf(g[j], w1[j], d1);
+            }
           }
-          put_dh<T>(dh, rt, (int64_t)c * B + b0 + u, fin, k, d0, d1);
+          if constexpr (DH) put_dh<T>(dh, rt, (int64_t)c * B + b0 + u, fin, k, d0, d1);
         }
       }
     }
   }
-  float* mine = red + (warp * kBwdPairs + lane) * 2 * J;
+  float* mine = red + (warp * kBwdPairs + lane) * 2 * JC;
 #pragma unroll
-  for (int j = 0; j < J; ++j) { mine[2 * j] = a0[j]; mine[2 * j + 1] = a1[j]; }
+  for (int j = 0; j < JC; ++j) { mine[2 * j] = a0[j]; mine[2 * j + 1] = a1[j]; }
   __syncthreads();
-  // dW[j][k0 + pair*2 + x] = sum over chunks (in order) of the partials
-  for (int o = threadIdx.x; o < kBwdPairs * 2 * J; o += kBwdPairs * kBwdChunks) {
-    const int pr = o / (2 * J), jj = o % (2 * J);
+  // dW[j0 + j][k0 + pair*2 + x] = sum over chunks (in order) of the partials
+  for (int o = threadIdx.x; o < kBwdPairs * 2 * JC; o += kBwdPairs * kBwdChunks) {
+    const int pr = o / (2 * JC), jj = o % (2 * JC);
     const int kk = 2 * (blockIdx.x * kBwdPairs + pr) + (jj & 1);
     if (kk >= fin) continue;
     float sum = 0.f;
 #pragma unroll
-    for (int q = 0; q < kBwdChunks; ++q) sum += red[(q * kBwdPairs + pr) * 2 * J + jj];
-    dw[(int64_t)c * g_rs + (int64_t)(jj >> 1) * fin + kk] = sum;
+    for (int q = 0; q < kBwdChunks; ++q) sum += red[(q * kBwdPairs + pr) * 2 * JC + jj];
+    dw[(int64_t)c * g_rs + (int64_t)(j0 + (jj >> 1)) * fin + kk] = sum;
   }
   if (blockIdx.x != 0) return;
-  if (warp == 0 && lane < J) {
+  if (warp == 0 && lane < JC) {
     float sum = 0.f;
-    for (int b = 0; b < B; ++b) sum += sdz[b * J + lane];
-    db[(int64_t)c * g_rs + lane] = sum;
-  } else if (warp == 1) {
+    for (int b = 0; b < B; ++b) sum += sdz[b * JC + lane];
+    db[(int64_t)c * g_rs + j0 + lane] = sum;
+  } else if (warp == 1 && blockIdx.z == 0) {
     float sum = 0.f;
     for (int b = lane; b < B; b += 32) sum += loss_ex[(int64_t)c * B + b];
 #pragma unroll
@@ -277,30 +324,95 @@ k_fc_bwd(const float* __restrict__ dlogits, const float* __restrict__ loss_ex,
   }
 }
 
+// dh[b][k] = sum_j dlogits[b][j] W[j][k] for heads too wide for k_fc_bwd's
+// registers.  grid (ceil(fin / (2 * kBwdPairs)), C): the block stages its
+// J x 2 kBwdPairs slice of W in shared memory as fp32; lane = feature pair,
+// warp = chunk of examples, each dlogits row read as float4 (a broadcast:
+// every lane reads the same row), classes summed in order 0 .. J-1.
+template <typename T, int J>
+__global__ void __launch_bounds__(kBwdPairs * kBwdChunks)
+k_fc_bwd_dh(const float* __restrict__ dlogits, const T* __restrict__ w, int64_t w_rs,
+            T* __restrict__ dh, int B, int fin, const HeadRoute rt) {
+  static_assert(J % 4 == 0, "dlogits rows are read as float4");
+  __shared__ float2 ws[J][kBwdPairs];
+  pdl_wait();
+  pdl_trigger();
+  const int c = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < J * kBwdPairs; i += kBwdPairs * kBwdChunks) {
+    const int j = i / kBwdPairs, pr = i % kBwdPairs;
+    const int kk = 2 * (blockIdx.x * kBwdPairs + pr);
+    ws[j][pr] = kk < fin ? load2<T>(w + (int64_t)c * w_rs + (int64_t)j * fin + kk)
+                         : make_float2(0.f, 0.f);
+  }
+  __syncthreads();
+  const int k = 2 * (blockIdx.x * kBwdPairs + lane);
+  if (k >= fin) return;
+  const int bc = (B + kBwdChunks - 1) / kBwdChunks;
+  const int b_lo = warp * bc, b_hi = b_lo + bc < B ? b_lo + bc : B;
+  for (int b = b_lo; b < b_hi; ++b) {
+    const float4* g4 = reinterpret_cast<const float4*>(dlogits + ((int64_t)c * B + b) * J);
+    float d0 = 0.f, d1 = 0.f;
+#pragma unroll 5
+    for (int q = 0; q < J / 4; ++q) {
+      const float4 g = g4[q];
+      const float gv[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float2 wv = ws[4 * q + u][lane];
+        d0 = fmaf(gv[u], wv.x, d0);
+        d1 = fmaf(gv[u], wv.y, d1);
+      }
+    }
+    put_dh<T>(dh, rt, (int64_t)c * B + b, fin, k, d0, d1);
+  }
+}
+
 bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 
 }  // namespace
 
-// the class count is a compile-time constant of the kernels; 10 is built
-constexpr int kClasses = 10;
+// The class count is a compile-time constant of the kernels: 10 and 100 are
+// built.  The 100-way head takes its classes 10 at a time in the forward and
+// the weight gradient and forms dh in k_fc_bwd_dh.
+constexpr int kClassChunk = 10;
+
+bool fc_bwd_split_dh(int fout) { return fout > kClassChunk; }
 
 template <typename T>
 cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_rs,
                              const float* b, int64_t b_rs, const int32_t* y, float* loss_ex,
                              float* dlogits, int C, int B, int fin, int fout,
                              float label_smoothing) {
-  if (fout != kClasses) return cudaErrorInvalidValue;
+  if (fout != 10 && fout != 100) return cudaErrorInvalidValue;
   constexpr int VEC = 16 / (int)sizeof(T);
   const unsigned grid = (unsigned)((int64_t)C * ((B + kFwdEx - 1) / kFwdEx));
   // 16-byte loads need every row of h and of each replica's W on a 16-byte boundary
   const bool vec = fin % VEC == 0 && (w_rs * (int64_t)sizeof(T)) % 16 == 0 && aligned16(h) &&
                    aligned16(w);
-  if (vec)
-    return launch_k(k_fc_fwd_ce<T, VEC, kClasses>, grid, kFwdSlices * 32, 0, s, h, w, w_rs, b,
-                    b_rs, y, loss_ex, dlogits, C, B, fin, label_smoothing);
-  return launch_k(k_fc_fwd_ce<T, 1, kClasses>, grid, kFwdSlices * 32, 0, s, h, w, w_rs, b, b_rs,
-                  y, loss_ex, dlogits, C, B, fin, label_smoothing);
+#define FWD_ARGS s, h, w, w_rs, b, b_rs, y, loss_ex, dlogits, C, B, fin, label_smoothing
+  if (fout == 10)
+    return vec ? launch_k(k_fc_fwd_ce<T, VEC, 10, 10>, grid, kFwdSlices * 32, 0, FWD_ARGS)
+               : launch_k(k_fc_fwd_ce<T, 1, 10, 10>, grid, kFwdSlices * 32, 0, FWD_ARGS);
+  return vec ? launch_k(k_fc_fwd_ce<T, VEC, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS)
+             : launch_k(k_fc_fwd_ce<T, 1, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS);
+#undef FWD_ARGS
 }
+
+namespace {
+
+bool head_route(int route, const uint8_t* code, const void* act, int Ho, int Wo, int ch, int fin,
+                HeadRoute* rt) {
+  if (route == FC_DH_AVG && (ch != fin || Ho * Wo < 1)) return false;
+  if (route != FC_DH_STORE && route != FC_DH_AVG &&
+      (ch % 2 || (int64_t)Ho * Wo * ch != fin || (route == FC_DH_POOL && !code) ||
+       (route == FC_DH_RELU && !act)))
+    return false;
+  *rt = HeadRoute{route, code, act, Ho, Wo, ch};
+  return true;
+}
+
+}  // namespace
 
 template <typename T>
 cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* loss_ex,
@@ -308,24 +420,37 @@ cudaError_t launch_fc_bwd(cudaStream_t s, const float* dlogits, const float* los
                           int64_t g_rs, T* dh, float* loss, int C, int B, int fin, int fout,
                           int route, const uint8_t* code, const T* act, int Ho, int Wo, int ch) {
   // feature pairs: even fin and 2-element alignment of every row
-  if (fout != kClasses || fin % 2 || w_rs % 2 || g_rs % 2 ||
+  if ((fout != 10 && fout != 100) || fin % 2 || w_rs % 2 || g_rs % 2 ||
       ((uintptr_t)w % (2 * sizeof(T))) || ((uintptr_t)dw % (2 * sizeof(float))))
     return cudaErrorInvalidValue;
-  if (route == FC_DH_AVG && (ch != fin || Ho * Wo < 1)) return cudaErrorInvalidValue;
-  if (route != FC_DH_STORE && route != FC_DH_AVG &&
-      (ch % 2 || (int64_t)Ho * Wo * ch != fin || (route == FC_DH_POOL && !code) ||
-       (route == FC_DH_RELU && !act)))
-    return cudaErrorInvalidValue;
-  const HeadRoute rt{route, code, act, Ho, Wo, ch};
-  const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C);
-  const size_t smem = sizeof(float) * ((size_t)B * fout + (size_t)kBwdChunks * kBwdPairs * 2 * fout);
+  HeadRoute rt;
+  if (!head_route(route, code, act, Ho, Wo, ch, fin, &rt)) return cudaErrorInvalidValue;
+  const int JC = fout == 10 ? 10 : kClassChunk;
+  const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C,
+                  (unsigned)(fout / JC));
+  const size_t smem = sizeof(float) * ((size_t)B * JC + (size_t)kBwdChunks * kBwdPairs * 2 * JC);
+  auto kern = fc_bwd_split_dh(fout) ? k_fc_bwd<T, kClassChunk, false> : k_fc_bwd<T, 10, true>;
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(k_fc_bwd<T, kClasses>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  return launch_k(k_fc_bwd<T, kClasses>, grid, kBwdPairs * kBwdChunks, smem, s, dlogits, loss_ex,
-                  h, w, w_rs, dw, db, g_rs, dh, loss, B, fin, rt);
+  return launch_k(kern, grid, kBwdPairs * kBwdChunks, smem, s, dlogits, loss_ex, h, w, w_rs, dw,
+                  db, g_rs, dh, loss, B, fin, fout, rt);
+}
+
+template <typename T>
+cudaError_t launch_fc_bwd_dh(cudaStream_t s, const float* dlogits, const T* w, int64_t w_rs,
+                             T* dh, int C, int B, int fin, int fout, int route,
+                             const uint8_t* code, const T* act, int Ho, int Wo, int ch) {
+  if (fout != 100 || fin % 2 || w_rs % 2 || ((uintptr_t)w % (2 * sizeof(T))) ||
+      !aligned16(dlogits))
+    return cudaErrorInvalidValue;
+  HeadRoute rt;
+  if (!head_route(route, code, act, Ho, Wo, ch, fin, &rt)) return cudaErrorInvalidValue;
+  const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C);
+  return launch_k(k_fc_bwd_dh<T, 100>, grid, kBwdPairs * kBwdChunks, 0, s, dlogits, w, w_rs, dh,
+                  B, fin, rt);
 }
 
 template cudaError_t launch_fc_fwd_ce<float>(cudaStream_t, const float*, const float*, int64_t,
@@ -342,5 +467,12 @@ template cudaError_t launch_fc_bwd<bf16>(cudaStream_t, const float*, const float
                                          const bf16*, int64_t, float*, float*, int64_t, bf16*,
                                          float*, int, int, int, int, int, const uint8_t*,
                                          const bf16*, int, int, int);
+
+template cudaError_t launch_fc_bwd_dh<float>(cudaStream_t, const float*, const float*, int64_t,
+                                             float*, int, int, int, int, int, const uint8_t*,
+                                             const float*, int, int, int);
+template cudaError_t launch_fc_bwd_dh<bf16>(cudaStream_t, const float*, const bf16*, int64_t,
+                                            bf16*, int, int, int, int, int, const uint8_t*,
+                                            const bf16*, int, int, int);
 
 }  // namespace gcpsl

@@ -81,6 +81,7 @@ struct RnState {
   float* bn;                        // [C][S_pad] running mean / var per BatchNorm
   int64_t S, S_pad;
   int64_t fcw, fcb, p_client, p_total;
+  int J;                            // classes
 };
 
 namespace {
@@ -88,8 +89,9 @@ namespace {
 constexpr int kStages[4][2] = {{64, 1}, {128, 2}, {256, 2}, {512, 2}};
 
 // parameter and state offsets in the order of PyTorch's named_parameters()
-void rn_layout(RnState& r) {
+void rn_layout(RnState& r, int J) {
   int64_t p = 0, s = 0;
+  r.J = J;
   auto conv = [&](RnConv& c, int cin, int cout, int k, int stride, int hin, int stage) {
     c = RnConv{};
     c.cin = cin; c.cout = cout; c.k = k; c.stride = stride;
@@ -124,8 +126,8 @@ void rn_layout(RnState& r) {
       if (st == 0 && j == 1) r.p_client = p;
       cin = cout; hw = ho;
     }
-  r.fcw = p; p += 10 * 512;
-  r.fcb = p; p += 10;
+  r.fcw = p; p += (int64_t)J * 512;
+  r.fcb = p; p += J;
   r.p_total = p;
   r.S = s;
   r.S_pad = (s + 63) / 64 * 64;
@@ -151,9 +153,9 @@ int64_t sets_of(const RnNorm& n, int B) { return n.gn ? (int64_t)B * 32 : n.ch; 
 
 }  // namespace
 
-int64_t rn_num_params(int segment) {
+int64_t rn_num_params(int J, int segment) {
   RnState r;
-  rn_layout(r);
+  rn_layout(r, J);
   if (segment == GCPSL_CLIENT) return r.p_client;
   if (segment == GCPSL_SERVER) return r.p_total - r.p_client;
   if (segment == GCPSL_BN_STATE) return r.S;
@@ -162,9 +164,9 @@ int64_t rn_num_params(int segment) {
 
 // canonical (OIHW) <-> kernel ([co][ky][kx][ci]) conv weights; the rest is
 // copied unchanged
-void rn_to_kernel_layout(const float* can, float* ker) {
+void rn_to_kernel_layout(int J, const float* can, float* ker) {
   RnState r;
-  rn_layout(r);
+  rn_layout(r, J);
   std::memcpy(ker, can, sizeof(float) * (size_t)r.p_total);
   for_each_conv(r, [&](RnConv& c) {
     const int kk = c.k * c.k;
@@ -176,9 +178,9 @@ void rn_to_kernel_layout(const float* can, float* ker) {
   });
 }
 
-void rn_to_canonical_layout(const float* ker, float* can) {
+void rn_to_canonical_layout(int J, const float* ker, float* can) {
   RnState r;
-  rn_layout(r);
+  rn_layout(r, J);
   std::memcpy(can, ker, sizeof(float) * (size_t)r.p_total);
   for_each_conv(r, [&](RnConv& c) {
     const int kk = c.k * c.k;
@@ -192,9 +194,9 @@ void rn_to_canonical_layout(const float* ker, float* can) {
 
 // PyTorch-style initial parameters: conv / linear weights U(+-1/sqrt(fan_in)),
 // linear bias likewise, norm weight 1 and bias 0 (deterministic LCG stream)
-void rn_seeded_init(uint64_t seed, float* can) {
+void rn_seeded_init(int J, uint64_t seed, float* can) {
   RnState r;
-  rn_layout(r);
+  rn_layout(r, J);
   uint64_t st = seed * 6364136223846793005ull + 1442695040888963407ull;
   auto uni = [&](float bound) {
     st = st * 6364136223846793005ull + 1442695040888963407ull;
@@ -213,8 +215,8 @@ void rn_seeded_init(uint64_t seed, float* can) {
     if (b.sc) ones(b.ns);
   }
   const float bf = 1.f / std::sqrt(512.f);
-  for (int i = 0; i < 10 * 512; ++i) can[r.fcw + i] = uni(bf);
-  for (int i = 0; i < 10; ++i) can[r.fcb + i] = uni(bf);
+  for (int i = 0; i < J * 512; ++i) can[r.fcw + i] = uni(bf);
+  for (int i = 0; i < J; ++i) can[r.fcb + i] = uni(bf);
 }
 
 void rn_free(gcpsl_ctx* c) {
@@ -227,7 +229,7 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
   c->rn = new (std::nothrow) RnState();
   if (!c->rn) return fail(c, GCPSL_E_NOMEM, "host allocation failed");
   RnState& r = *c->rn;
-  rn_layout(r);
+  rn_layout(r, c->J);
   const int C = c->C, B = c->B;
   const int64_t P = c->P_pad;
   auto act = [&](bf16*& p, int64_t elems) -> gcpsl_status {
@@ -540,13 +542,16 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
   }
   LAUNCH("rn_avgpool", launch_avgpool(s, r.blk[7].out, r.h, C * B, 16, 512));
   LAUNCH("fc_fwd_ce", launch_fc_fwd_ce<bf16>(s, r.h, c->d_shadow + r.fcw, P, th + r.fcb, P,
-                                              c->d_y, c->d_loss_ex, c->d_dlogits, C, B, 512, 10,
+                                              c->d_y, c->d_loss_ex, c->d_dlogits, C, B, 512, r.J,
                                               c->desc.label_smoothing));
   // ---- backward ----
   bf16* d = r.gin[1];
   LAUNCH("fc_bwd", launch_fc_bwd<bf16>(s, c->d_dlogits, c->d_loss_ex, r.h, c->d_shadow + r.fcw, P,
                                         c->d_grad + r.fcw, c->d_grad + r.fcb, P, d, c->d_loss, C,
-                                        B, 512, 10, FC_DH_AVG, nullptr, nullptr, 4, 4, 512));
+                                        B, 512, r.J, FC_DH_AVG, nullptr, nullptr, 4, 4, 512));
+  if (fc_bwd_split_dh(r.J))
+    LAUNCH("fc_bwd_dh", launch_fc_bwd_dh<bf16>(s, c->d_dlogits, c->d_shadow + r.fcw, P, d, C, B,
+                                                512, r.J, FC_DH_AVG, nullptr, nullptr, 4, 4, 512));
   for (int i = 7; i >= 0; --i) {
     RnBlock& b = r.blk[i];
     bf16* dx = i == 2 ? r.cutg : (d == r.gin[1] ? r.gin[0] : r.gin[1]);

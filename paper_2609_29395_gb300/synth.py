@@ -5,11 +5,11 @@ split and the initial split-model parameters.  It holds none of the method's
 arithmetic (no sampling, no forward/backward, no update, no fusion), so that
 both the CUDA library and the CPU oracle can take their inputs from it.
 
-Stand-in for CIFAR-10 (Section V-A uses CIFAR-10/100, which are not available
-here): 32x32x3 images with N(0,1) pixels and 10 classes.  The client split is a
-per-class Dirichlet draw (the paper's Section V-A uses an extended-Dirichlet
-protocol with two classes per client; the plain per-class Dirichlet(alpha) is
-the recipe these workloads use instead).
+Stand-in for CIFAR-10 and CIFAR-100 (Section V-A; the datasets are not
+available here): 32x32x3 images with N(0,1) pixels and 10 or 100 classes.  Two
+client splits: a per-class Dirichlet(alpha) draw over all clients, and the
+extended-Dirichlet protocol of Section V-A (each client holds two classes,
+each class is spread over its holders by a Dirichlet(alpha) draw).
 """
 from __future__ import annotations
 
@@ -82,12 +82,62 @@ def dirichlet_split(labels: np.ndarray, num_clients: int, alpha: float,
     return owner
 
 
+def class_support(num_clients: int, num_classes: int, per_client: int,
+                  seed: int = SEED_SPLIT) -> np.ndarray:
+    """[K][per_client] distinct classes of each client: client k's first is
+    k mod num_classes (so every class has a holder once K >= num_classes),
+    the others are drawn uniformly without replacement from the rest."""
+    if not 1 <= per_client <= num_classes:
+        raise ValueError("per_client must lie in [1, num_classes]")
+    rng = np.random.default_rng(seed)
+    sup = np.empty((num_clients, per_client), dtype=np.int32)
+    for k in range(num_clients):
+        first = k % num_classes
+        rest = np.delete(np.arange(num_classes), first)
+        sup[k, 0] = first
+        sup[k, 1:] = rng.choice(rest, size=per_client - 1, replace=False)
+    return sup
+
+
+def extended_dirichlet_split(labels: np.ndarray, num_clients: int, per_client: int,
+                             alpha: float, seed: int = SEED_SPLIT) -> np.ndarray:
+    """Owner of every example under the extended-Dirichlet protocol of
+    Section V-A: each client holds `per_client` classes (class_support), and
+    each class's examples go to its holders in Dirichlet(alpha) proportions,
+    dealt as in dirichlet_split (floor, largest remainders, shuffled deal).
+    A class no client holds (K < num_classes) keeps owner -1 and is rejected."""
+    num_classes = int(labels.max()) + 1 if labels.size else 0
+    sup = class_support(num_clients, num_classes, per_client, seed)
+    rng = np.random.default_rng(seed + 7_919)
+    owner = np.full(labels.shape[0], -1, dtype=np.int32)
+    for c in range(num_classes):
+        holders = np.flatnonzero((sup == c).any(axis=1)).astype(np.int32)
+        ex = np.flatnonzero(labels == c)
+        if holders.size == 0:
+            raise ValueError(f"class {c} has no holder")
+        p = rng.dirichlet(np.full(holders.size, alpha))
+        raw = p * ex.size
+        cnt = np.floor(raw).astype(np.int64)
+        rem = ex.size - int(cnt.sum())
+        order = np.lexsort((np.arange(holders.size), -(raw - cnt)))
+        cnt[order[:rem]] += 1
+        rng.shuffle(ex)
+        owner[ex] = np.repeat(holders, cnt)
+    return owner
+
+
 def make_dataset(n: int, num_classes: int, num_clients: int, alpha: float,
                  balanced: bool, seed_data: int = SEED_DATA,
-                 seed_split: int = SEED_SPLIT) -> Dataset:
+                 seed_split: int = SEED_SPLIT, classes_per_client: int = 0) -> Dataset:
+    """classes_per_client = 0: per-class Dirichlet(alpha) over all clients;
+    m > 0: the extended-Dirichlet split with m classes per client."""
     images = make_images(n, seed_data)
     labels = make_labels(n, num_classes, balanced, seed_data)
-    owner = dirichlet_split(labels, num_clients, alpha, seed_split)
+    if classes_per_client:
+        owner = extended_dirichlet_split(labels, num_clients, classes_per_client, alpha,
+                                         seed_split)
+    else:
+        owner = dirichlet_split(labels, num_clients, alpha, seed_split)
     return Dataset(images, labels, owner, num_classes, num_clients)
 
 
@@ -96,7 +146,8 @@ def make_dataset(n: int, num_classes: int, num_clients: int, alpha: float,
 # OIHW), client segment first.  Conv layers are 3x3, stride 1, padding 1,
 # with bias; every conv is followed by ReLU; `pool` adds a 2x2/2 max-pool.
 # ---------------------------------------------------------------------------
-ARCH_TINY_CNN, ARCH_SPLIT_CNN, ARCH_RESNET18 = 0, 1, 2
+ARCH_TINY_CNN, ARCH_SPLIT_CNN, ARCH_RESNET18, ARCH_RESNET18_C100 = 0, 1, 2, 3
+RESNET_ARCHS = {ARCH_RESNET18: 10, ARCH_RESNET18_C100: 100}     # arch -> classes
 
 ARCHS = {
     # (cin, cout, H, W, pool) per conv layer; fc (in, out)
@@ -109,14 +160,15 @@ ARCHS = {
 
 
 # The CIFAR ResNet-18 split: client = conv 3->64 stem + GroupNorm + stage 1,
-# server = stages 2-4 with BatchNorm, global average pool, linear 512->10.
+# server = stages 2-4 with BatchNorm, global average pool, linear 512->J
+# (J = 10, or 100 for ARCH_RESNET18_C100).
 # Basic blocks (conv1, norm1, conv2, norm2[, shortcut conv 1x1, norm]);
 # convolutions have no bias.  Names and order follow PyTorch's
 # named_parameters() of the usual CIFAR ResNet-18 module layout.
 RESNET_STAGES = ((64, 1), (128, 2), (256, 2), (512, 2))     # (width, first stride)
 
 
-def _resnet_shapes(segment: str):
+def _resnet_shapes(segment: str, classes: int):
     out = []
     if segment == "client":
         out += [("conv1.weight", (64, 3, 3, 3)), ("bn1.weight", (64,)), ("bn1.bias", (64,))]
@@ -137,14 +189,14 @@ def _resnet_shapes(segment: str):
                             (f"{pre}.shortcut.1.bias", (width,))]
             cin = width
     if segment == "server":
-        out += [("linear.weight", (10, 512)), ("linear.bias", (10,))]
+        out += [("linear.weight", (classes, 512)), ("linear.bias", (classes,))]
     return out
 
 
 def param_shapes(arch: int, segment: str):
     """[(name, shape)] for one segment ('client' or 'server')."""
-    if arch == ARCH_RESNET18:
-        return _resnet_shapes(segment)
+    if arch in RESNET_ARCHS:
+        return _resnet_shapes(segment, RESNET_ARCHS[arch])
     spec = ARCHS[arch]
     out = []
     for i, (cin, cout, _h, _w, _p) in enumerate(spec[segment]):
@@ -155,6 +207,10 @@ def param_shapes(arch: int, segment: str):
         out.append(("server.fc.weight", (fout, fin)))
         out.append(("server.fc.bias", (fout,)))
     return out
+
+
+def num_classes(arch: int) -> int:
+    return RESNET_ARCHS.get(arch, 10)
 
 
 def num_params(arch: int, segment: str) -> int:

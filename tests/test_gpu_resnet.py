@@ -1,5 +1,6 @@
-"""GPU parity of the ResNet-18 split (architecture 2): the CUDA library
-against the CPU oracle in its bf16-operand mode, through the C ABI.
+"""GPU parity of the ResNet-18 split (architecture 2, and architecture 3
+with its 100-way head): the CUDA library against the CPU oracle in its
+bf16-operand mode, through the C ABI.
 
 Each round both sides start from the same state (parameters, momentum and
 BatchNorm running statistics of the oracle, rounded to fp32).
@@ -33,6 +34,7 @@ from paper_2609_29395_gb300 import clustering, synth
 pytestmark = pytest.mark.gpu
 
 RES = synth.ARCH_RESNET18
+RES100 = synth.ARCH_RESNET18_C100
 REL_L2 = 2e-2
 LOSS_ABS = 1e-2
 # forward values of the two sides differ by well under 1% of a layer's RMS
@@ -51,10 +53,11 @@ def rel_l2(a, b):
     return np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30)
 
 
-def _small(C=2, n=160, K=8, seed=3):
-    ds = synth.make_dataset(n, 10, K, 0.5, balanced=False, seed_data=seed, seed_split=seed + 1)
+def _small(C=2, n=160, K=8, seed=3, arch=RES):
+    ds = synth.make_dataset(n, synth.num_classes(arch), K, 0.5, balanced=False, seed_data=seed,
+                            seed_split=seed + 1)
     assign = clustering.random_clustering(K, C, seed + 2)
-    return ds, assign, synth.init_params(RES, seed=seed + 6)
+    return ds, assign, synth.init_params(arch, seed=seed + 6)
 
 
 def _sync(gpu, orc):
@@ -158,14 +161,15 @@ def test_resnet18_epoch_schedule_keeps_waiting_batchnorm_state():
     assert (gpu.bn_state(0) == gpu.bn_state(1)).all()
 
 
-def test_resnet18_grouped_equals_serialized_and_graph_equals_eager():
+@pytest.mark.parametrize("arch", [RES, RES100])
+def test_resnet18_grouped_equals_serialized_and_graph_equals_eager(arch):
     """Two clusters in one context == each cluster alone (same cluster id),
     and graph replay == eager launches, bit for bit, over three rounds."""
-    ds, assign, params = _small(seed=5)
+    ds, assign, params = _small(seed=5, arch=arch)
     kw = dict(lr=0.05, momentum=0.9)
-    both = pkg.Context(RES, 8, 2, assign, 4, 0, 4, ds.images, ds.labels, ds.owner, params,
+    both = pkg.Context(arch, 8, 2, assign, 4, 0, 4, ds.images, ds.labels, ds.owner, params,
                        bf16=True, **kw)
-    eager = pkg.Context(RES, 8, 2, assign, 4, 0, 4, ds.images, ds.labels, ds.owner, params,
+    eager = pkg.Context(arch, 8, 2, assign, 4, 0, 4, ds.images, ds.labels, ds.owner, params,
                         bf16=True, **kw)
     eager.set_graph(False)
     for _ in range(3):
@@ -173,7 +177,7 @@ def test_resnet18_grouped_equals_serialized_and_graph_equals_eager():
         eager.step()
     for m in range(2):
         sub = np.where(assign == m, 0, -1).astype(np.int32)
-        one = pkg.Context(RES, 8, 1, sub, 4, 0, 4, ds.images, ds.labels, ds.owner, params,
+        one = pkg.Context(arch, 8, 1, sub, 4, 0, 4, ds.images, ds.labels, ds.owner, params,
                           bf16=True, cluster_id_base=m, **kw)
         for _ in range(3):
             one.step()
@@ -183,17 +187,38 @@ def test_resnet18_grouped_equals_serialized_and_graph_equals_eager():
         one.close()
 
 
-def test_resnet18_c8_full_size_sampled_cluster():
-    """The 200,000-image, K=1024, C=8, B=128 workload in the benchmarked
-    launch configuration: the GPU takes its first round with all eight
-    clusters; cluster 5 is re-run alone by the oracle (one-cluster context,
+def test_resnet18_c100_rounds_against_oracle():
+    """The 100-way head with the paper's training recipe (Nesterov momentum
+    0.9, weight decay 5e-4, label smoothing 0.1 over 100 classes, random crop
+    + flip), two clusters, B = 8, labels over all 100 classes, two rounds and
+    a fusion."""
+    ds, assign, params = _small(n=400, seed=11, arch=RES100)
+    assert ds.labels.max() > 90
+    kw = dict(lr=0.01, momentum=0.9, weight_decay=5e-4, nesterov=True, label_smoothing=0.1,
+              augment=True)
+    gpu = pkg.Context(RES100, 8, 2, assign, 8, 2, 4, ds.images, ds.labels, ds.owner, params,
+                      bf16=True, **kw)
+    orc = oracle.Oracle(RES100, 8, 2, assign, 8, 2, 4, ds.images, ds.labels, ds.owner, params,
+                        bf16=True, **kw)
+    for _ in range(2):
+        print("cut grad, update:", _round(gpu, orc))
+    assert (gpu.all_params(0) == gpu.all_params(1)).all()
+
+
+@pytest.mark.parametrize("name,m", [("resnet18_c8", 5), ("resnet18_c100_c4", 2)])
+def test_resnet18_full_size_sampled_cluster(name, m):
+    """A full ResNet-18 workload in the benchmarked launch configuration
+    (200,000 images, K=1024, C=8, B=128; or the CIFAR-100 shape: 50,000
+    images, 100 classes, K=256 two-class clients, C=4 label-aware clusters,
+    B=128, the paper's recipe): the GPU takes its first round with all
+    clusters; cluster m is re-run alone by the oracle (one-cluster context,
     same cluster id, so the same Philox stream) replaying that cluster's
     ReLU decisions, and compared slice by slice."""
     from paper_2609_29395_gb300 import configs
-    w = configs.WORKLOADS["resnet18_c8"]
+    w = configs.WORKLOADS[name]
     ds, assign, params = configs.build_inputs(w)
     gpu = pkg.Context(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, 4, ds.images,
-                      ds.labels, ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=True)
+                      ds.labels, ds.owner, params, bf16=True, **w.options())
     bn0 = gpu.bn_state(0)
     loss, active = gpu.step(stats=True)
     gi, gc = gpu.sample()
@@ -201,11 +226,9 @@ def test_resnet18_c8_full_size_sampled_cluster():
     masks = gpu.relu_masks()
     cut_act = gpu.cut(pkg.binding.GCPSL_CUT_ACT)
     cut_grad = gpu.cut(pkg.binding.GCPSL_CUT_GRAD)
-    m = 5
     sub = np.where(assign == m, 0, -1).astype(np.int32)
     orc = oracle.Oracle(w.arch, w.num_clients, 1, sub, w.B, w.F, 4, ds.images, ds.labels,
-                        ds.owner, params, lr=w.lr, momentum=w.momentum, bf16=True,
-                        cluster_base=m)
+                        ds.owner, params, bf16=True, cluster_base=m, **w.options())
     orc.set_bn_state(0, bn0.astype(np.float64))
     oracle.set_relu_tol(RELU_TOL)
     orc.set_relu_masks(masks[m:m + 1])

@@ -37,6 +37,14 @@ def test_num_params(lib):
         pkg.gcpsl_num_params(binding.GCPSL_TINY_CNN, 1) == 25_578
     assert pkg.gcpsl_num_params(binding.GCPSL_SPLIT_CNN, 0) == synth.num_params(1, "client")
     assert pkg.gcpsl_num_params(7, 0) == -1
+    # the 100-way head adds 90 rows of 512 weights and 90 biases to the server
+    for seg in (0, 1):
+        assert pkg.gcpsl_num_params(binding.GCPSL_RESNET18_C100, seg) == \
+            synth.num_params(synth.ARCH_RESNET18_C100, ("client", "server")[seg])
+    assert pkg.gcpsl_num_params(binding.GCPSL_RESNET18_C100, 1) - \
+        pkg.gcpsl_num_params(binding.GCPSL_RESNET18, 1) == 90 * 513
+    assert pkg.gcpsl_num_params(binding.GCPSL_RESNET18_C100, 0) == \
+        pkg.gcpsl_num_params(binding.GCPSL_RESNET18, 0)
 
 
 def _ds(n=256, K=8):
@@ -44,7 +52,7 @@ def _ds(n=256, K=8):
 
 
 @pytest.mark.parametrize("case", ["small_cluster", "assign_range", "owner_range", "label_range",
-                                  "bad_B", "bad_arch", "bad_dtype"])
+                                  "bad_B", "bad_arch", "bad_dtype", "class_count"])
 def test_init_rejects_bad_arguments(lib, case):
     ds = _ds()
     K, C, B = 8, 2, 16
@@ -64,7 +72,18 @@ def test_init_rejects_bad_arguments(lib, case):
     elif case == "bad_arch":
         kw["arch"] = 9
     with pytest.raises(binding.GcpslError) as e:
-        if case == "bad_dtype":
+        if case == "class_count":
+            # a 10-class dataset declared to a 100-class architecture
+            desc = binding.gcpsl_model_desc(binding.GCPSL_RESNET18_C100, 1, 0.05, 0, 0, 0, 0, 0,
+                                            0, 0)
+            ds_c = binding.gcpsl_dataset(binding._p(ds.images, ct.c_float),
+                                         binding._p(ds.labels, ct.c_int32),
+                                         binding._p(ds.owner, ct.c_int32), ds.images.shape[0], 10)
+            h = ct.c_void_p()
+            st = lib.gcpsl_init(ct.byref(desc), K, C, binding._p(assign, ct.c_int32), B, 0, 1,
+                                ct.byref(ds_c), None, ct.byref(h))
+            binding._check(st)
+        elif case == "bad_dtype":
             desc = binding.gcpsl_model_desc(0, 7, 0.05, 0, 0, 0, 0, 0, 0, 0)
             ds_c = binding.gcpsl_dataset(binding._p(ds.images, ct.c_float),
                                          binding._p(ds.labels, ct.c_int32),
@@ -169,4 +188,67 @@ def test_workloads_fit_their_batch():
     ds, assign, params = configs.build_inputs(w)
     sizes = configs.cluster_sizes(ds.owner, assign, w.num_clusters)
     assert (sizes >= w.B).all()
+    assert params.size == synth.num_params(w.arch, "client") + synth.num_params(w.arch, "server")
+
+
+# --------------------------------------------------------------------------
+# Extended-Dirichlet client split (Section V-A)
+# --------------------------------------------------------------------------
+def test_class_support_covers_every_class():
+    sup = synth.class_support(256, 100, 2, seed=5)
+    assert sup.shape == (256, 2)
+    assert (sup[:, 0] == np.arange(256) % 100).all()
+    assert (sup[:, 0] != sup[:, 1]).all()
+    assert set(np.unique(sup)) == set(range(100))
+    # the second class is uniform over the other 99: chi-square over 256 draws
+    # is loose, so check only the range and that many classes appear
+    assert len(np.unique(sup[:, 1])) > 80
+    with pytest.raises(ValueError):
+        synth.class_support(8, 10, 0)
+
+
+def test_extended_dirichlet_split_invariants():
+    n, J, K, m = 20_000, 100, 256, 2
+    labels = synth.make_labels(n, J, True)
+    owner = synth.extended_dirichlet_split(labels, K, m, 3.0, seed=9)
+    sup = synth.class_support(K, J, m, seed=9)
+    assert owner.shape == labels.shape and owner.min() >= 0 and owner.max() < K
+    # every example's class is one of its owner's classes
+    assert (sup[owner] == labels[:, None]).any(axis=1).all()
+    # every class's examples all went to its holders, and were all dealt
+    for c in (0, 17, 99):
+        holders = set(np.flatnonzero((sup == c).any(axis=1)))
+        assert set(np.unique(owner[labels == c])) <= holders
+    assert np.bincount(labels, minlength=J).sum() == n
+    # deterministic
+    assert (owner == synth.extended_dirichlet_split(labels, K, m, 3.0, seed=9)).all()
+
+
+def test_extended_dirichlet_concentration():
+    """Large alpha spreads a class evenly over its holders; small alpha
+    concentrates it (Dirichlet concentration)."""
+    labels = synth.make_labels(100_000, 10, True)
+    spread = {}
+    for alpha in (1000.0, 0.05):
+        owner = synth.extended_dirichlet_split(labels, 40, 2, alpha, seed=3)
+        sup = synth.class_support(40, 10, 2, seed=3)
+        cv = []
+        for c in range(10):
+            holders = np.flatnonzero((sup == c).any(axis=1))
+            cnt = np.bincount(owner[labels == c], minlength=40)[holders]
+            cv.append(cnt.std() / cnt.mean())
+        spread[alpha] = float(np.mean(cv))
+    assert spread[1000.0] < 0.1 < 1.0 < spread[0.05]
+
+
+def test_cifar100_workload_inputs():
+    w = configs.WORKLOADS["resnet18_c100_c4"]
+    assert w.num_classes == 100
+    ds, assign, params = configs.build_inputs(w)
+    assert ds.num_classes == 100 and ds.labels.max() == 99
+    assert np.bincount(ds.labels).min() == np.bincount(ds.labels).max() == 500
+    per_client = [np.unique(ds.labels[ds.owner == k]).size for k in range(w.num_clients)]
+    assert max(per_client) <= 2
+    sizes = configs.cluster_sizes(ds.owner, assign, w.num_clusters)
+    assert (sizes >= w.B).all() and sizes.sum() == w.n
     assert params.size == synth.num_params(w.arch, "client") + synth.num_params(w.arch, "server")
