@@ -44,9 +44,12 @@ FLUSH_BYTES = 256 << 20
 # kernel kind; valid only while the kernel source hashes to the recorded value.
 NCU_TRAFFIC = {
     # DRAM read + write per launch (ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,
-    # one pass); SplitCNN kinds from the full C=4 workload, the ResNet-18 GroupNorm kinds
-    # from C=2 (20,000 images) scaled x4 to C=8 (per-example kernels): see
-    # profiles/splitcnn_c4_and_resnet18_traffic.md
+    # one pass), with the examples per round (C*B) of the capture: the SplitCNN kinds from
+    # the full C=4 workload, the ResNet-18 GroupNorm kinds (per-example kernels, the same
+    # 64x32x32 map in all five layers) from C=2, B=128, 20,000 images; see
+    # profiles/splitcnn_c4_and_resnet18_traffic.md.  A conv / norm kernel's traffic scales
+    # with the examples of a round; the update's with C*P, so it is taken only at the
+    # captured C.
     "conv_fwd_tc.L0": {"bytes": 1.681e+07, "src_hash": "9edb62919210128c"},
     "conv_fwd_tc.L1": {"bytes": 1.697e+07, "src_hash": "9edb62919210128c"},
     "conv_fwd_tc.L2": {"bytes": 9.02e+06, "src_hash": "9edb62919210128c"},
@@ -58,10 +61,32 @@ NCU_TRAFFIC = {
     "conv_wgrad_tc.L1": {"bytes": 5.036e+07, "src_hash": "9edb62919210128c"},
     "conv_wgrad_tc.L2": {"bytes": 2.523e+07, "src_hash": "9edb62919210128c"},
     "conv_wgrad_tc.L3": {"bytes": 8.43e+06, "src_hash": "9edb62919210128c"},
-    "sgd": {"bytes": 6.11e+07, "src_hash": "483ce6954d2d1468"},
-    "rn_norm_gn_bwd": {"bytes": 3.93448e+08, "src_hash": "d7895818885460a1"},
-    "rn_norm_gn": {"bytes": 1.88496e+08, "src_hash": "d7895818885460a1"},
+    "sgd": {"bytes": 6.11e+07, "src_hash": "483ce6954d2d1468", "per": "C", "C": 4},
+    "rn_norm_gn_bwd": {"bytes": 9.8362e+07, "src_hash": "d7895818885460a1", "family": "resnet",
+                       "examples": 256},
+    "rn_norm_gn": {"bytes": 4.7124e+07, "src_hash": "d7895818885460a1", "family": "resnet",
+                   "examples": 256},
 }
+for _k, _v in NCU_TRAFFIC.items():
+    _v.setdefault("family", "splitcnn")
+    _v.setdefault("examples", 256)          # SplitCNN C=4 x B=64
+    _v.setdefault("per", "examples")
+
+
+def ncu_traffic(kind, w):
+    """Recorded DRAM bytes per launch of `kind` for workload w, or None when
+    the kernel's source changed since the capture or the figure does not
+    carry over to w's model or cluster count."""
+    from paper_2609_29395_gb300 import synth
+    rec = NCU_TRAFFIC.get(kind)
+    if not rec or rec["src_hash"] != kernel_source_hash(kind):
+        return None
+    family = "resnet" if w.arch in synth.RESNET_ARCHS else "splitcnn"
+    if rec["family"] != family:
+        return None
+    if rec["per"] == "C":
+        return rec["bytes"] if w.num_clusters == rec["C"] else None
+    return rec["bytes"] * w.num_clusters * w.B / rec["examples"]
 
 
 def parse():
@@ -457,8 +482,7 @@ def main():
             ach = total_work / secs / 1e9
             roof.update(bound="hbm", achieved=ach, unit="GB/s", peak=peaks["hbm"],
                         frac=ach / peaks["hbm"], peak_src=f"HBM copy, {peaks['src']}")
-    rec = NCU_TRAFFIC.get(kind)
-    roof["traffic"] = rec["bytes"] if rec and rec["src_hash"] == kernel_source_hash(kind) else None
+    roof["traffic"] = ncu_traffic(kind, w)
 
     breakdown = {k: {"launches": n, "ms_per_round": ms / K} for k, (n, ms) in
                  sorted(all_times.items(), key=lambda kv: -kv[1][1])}

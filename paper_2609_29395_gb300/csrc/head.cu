@@ -47,6 +47,19 @@ template <> struct VecLoad<float, 4> {
     o[0] = u.x; o[1] = u.y; o[2] = u.z; o[3] = u.w;
   }
 };
+template <> struct VecLoad<bf16, 2> {
+  __device__ static void run(const bf16* p, float* o) {
+    const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+    o[0] = __uint_as_float(u << 16);
+    o[1] = __uint_as_float(u & 0xffff0000u);
+  }
+};
+template <> struct VecLoad<float, 2> {
+  __device__ static void run(const float* p, float* o) {
+    const float2 u = *reinterpret_cast<const float2*>(p);
+    o[0] = u.x; o[1] = u.y;
+  }
+};
 template <typename T> struct VecLoad<T, 1> {
   __device__ static void run(const T* p, float* o) { o[0] = to_f(p[0]); }
 };
@@ -325,10 +338,13 @@ k_fc_bwd(const float* __restrict__ dlogits, const float* __restrict__ loss_ex,
 }
 
 // dh[b][k] = sum_j dlogits[b][j] W[j][k] for heads too wide for k_fc_bwd's
-// registers.  grid (ceil(fin / (2 * kBwdPairs)), C): the block stages its
-// J x 2 kBwdPairs slice of W in shared memory as fp32; lane = feature pair,
-// warp = chunk of examples, each dlogits row read as float4 (a broadcast:
-// every lane reads the same row), classes summed in order 0 .. J-1.
+// registers.  grid (ceil(fin / (2 * kBwdPairs)), C, ceil(B / kDhExamples)):
+// the block stages its J x 2 kBwdPairs slice of W in shared memory as fp32;
+// lane = feature pair, warp = kDhExamples / kBwdChunks consecutive examples
+// of the block's chunk, each dlogits row read as float4 (a broadcast: every
+// lane reads the same row), classes summed in order 0 .. J-1.
+constexpr int kDhExamples = 16;   // examples per k_fc_bwd_dh block
+
 template <typename T, int J>
 __global__ void __launch_bounds__(kBwdPairs * kBwdChunks)
 k_fc_bwd_dh(const float* __restrict__ dlogits, const T* __restrict__ w, int64_t w_rs,
@@ -348,8 +364,9 @@ k_fc_bwd_dh(const float* __restrict__ dlogits, const T* __restrict__ w, int64_t 
   __syncthreads();
   const int k = 2 * (blockIdx.x * kBwdPairs + lane);
   if (k >= fin) return;
-  const int bc = (B + kBwdChunks - 1) / kBwdChunks;
-  const int b_lo = warp * bc, b_hi = b_lo + bc < B ? b_lo + bc : B;
+  constexpr int per_warp = kDhExamples / kBwdChunks;
+  const int b_lo = blockIdx.z * kDhExamples + warp * per_warp;
+  const int b_hi = b_lo + per_warp < B ? b_lo + per_warp : B;
   for (int b = b_lo; b < b_hi; ++b) {
     const float4* g4 = reinterpret_cast<const float4*>(dlogits + ((int64_t)c * B + b) * J);
     float d0 = 0.f, d1 = 0.f;
@@ -394,8 +411,11 @@ cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_r
   if (fout == 10)
     return vec ? launch_k(k_fc_fwd_ce<T, VEC, 10, 10>, grid, kFwdSlices * 32, 0, FWD_ARGS)
                : launch_k(k_fc_fwd_ce<T, 1, 10, 10>, grid, kFwdSlices * 32, 0, FWD_ARGS);
-  return vec ? launch_k(k_fc_fwd_ce<T, VEC, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS)
-             : launch_k(k_fc_fwd_ce<T, 1, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS);
+  // the 100-way head loads pairs, so that all eight warps share fin = 512
+  const bool vec2 = fin % 2 == 0 && w_rs % 2 == 0 && (uintptr_t)h % (2 * sizeof(T)) == 0 &&
+                    (uintptr_t)w % (2 * sizeof(T)) == 0;
+  return vec2 ? launch_k(k_fc_fwd_ce<T, 2, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS)
+              : launch_k(k_fc_fwd_ce<T, 1, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS);
 #undef FWD_ARGS
 }
 
@@ -448,7 +468,8 @@ cudaError_t launch_fc_bwd_dh(cudaStream_t s, const float* dlogits, const T* w, i
     return cudaErrorInvalidValue;
   HeadRoute rt;
   if (!head_route(route, code, act, Ho, Wo, ch, fin, &rt)) return cudaErrorInvalidValue;
-  const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C);
+  const dim3 grid((unsigned)((fin / 2 + kBwdPairs - 1) / kBwdPairs), (unsigned)C,
+                  (unsigned)((B + kDhExamples - 1) / kDhExamples));
   return launch_k(k_fc_bwd_dh<T, 100>, grid, kBwdPairs * kBwdChunks, 0, s, dlogits, w, w_rs, dh,
                   B, fin, rt);
 }

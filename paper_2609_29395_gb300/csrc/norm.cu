@@ -10,10 +10,13 @@
 // H x W; BatchNorm one channel over B x H x W.
 //
 // Both directions go through per-(example, channel) partial sums over the
-// pixels (fp32, pixels in a fixed order), combined per set in fp64 by a
-// small finalize kernel (which also folds the normalisation into a
-// per-channel affine form), then an elementwise apply.  Every sum has a fixed
-// order, so results do not depend on C or on launch geometry.
+// pixels (fp32, pixels in a fixed order), combined per set by a small
+// finalize kernel (which also folds the normalisation into a per-channel
+// affine form), then an elementwise apply.  Every sum has a fixed order, so
+// results do not depend on C or on launch geometry.  All of it is fp32: the
+// sets combine at most B = 1024 partials, and GB300 executes fp64 at 1/64 of
+// the fp32 rate, which made fp64 finalize kernels latency-bound on the fp64
+// pipe.
 #include "common.cuh"
 #include "sm100.cuh"
 
@@ -22,7 +25,7 @@ namespace gcpsl {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr double kEps = 1e-5;
+constexpr float kEps = 1e-5f;
 
 __device__ __forceinline__ void unpack8(const uint4& u, float* f) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
@@ -75,27 +78,48 @@ k_chan_sums(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* 
     }
   }
   if (threadIdx.x < L * V) {
-    for (int p = l; p < HW; p += L) {
-      const int64_t o = base + (int64_t)p * ch + v * 8;
-      float a[8];
-      unpack8(*reinterpret_cast<const uint4*>(BWD ? d + o : y + o), a);
-      if (!BWD) {
+    // four pixels per step: their loads are issued together, the sums
+    // still taken in pixel order
+    constexpr int U = 4;
+    for (int p0 = l; p0 < HW; p0 += U * L) {
+      uint4 ua[U], uy[U], um[U];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) { s1[i] += a[i]; s2[i] = fmaf(a[i], a[i], s2[i]); }
-      } else {
-        if (mask) {
-          float m[8];
-          unpack8(*reinterpret_cast<const uint4*>(mask + o), m);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) a[i] = m[i] > 0.f ? a[i] : 0.f;
-          if (dz_out) *reinterpret_cast<uint4*>(dz_out + o) = pack8(a);
+      for (int j = 0; j < U; ++j) {
+        const int p = p0 + j * L;
+        if (p < HW) {
+          const int64_t o = base + (int64_t)p * ch + v * 8;
+          ua[j] = *reinterpret_cast<const uint4*>(BWD ? d + o : y + o);
+          if (BWD) {
+            uy[j] = *reinterpret_cast<const uint4*>(y + o);
+            if (mask) um[j] = *reinterpret_cast<const uint4*>(mask + o);
+          }
         }
-        float yy[8];
-        unpack8(*reinterpret_cast<const uint4*>(y + o), yy);
+      }
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          s1[i] += a[i];
-          s2[i] = fmaf(a[i], (yy[i] - mu[i]) * rs[i], s2[i]);
+      for (int j = 0; j < U; ++j) {
+        const int p = p0 + j * L;
+        if (p >= HW) break;
+        float a[8];
+        unpack8(ua[j], a);
+        if (!BWD) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) { s1[i] += a[i]; s2[i] = fmaf(a[i], a[i], s2[i]); }
+        } else {
+          if (mask) {
+            float m[8];
+            unpack8(um[j], m);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) a[i] = m[i] > 0.f ? a[i] : 0.f;
+            if (dz_out)
+              *reinterpret_cast<uint4*>(dz_out + base + (int64_t)p * ch + v * 8) = pack8(a);
+          }
+          float yy[8];
+          unpack8(uy[j], yy);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            s1[i] += a[i];
+            s2[i] = fmaf(a[i], (yy[i] - mu[i]) * rs[i], s2[i]);
+          }
         }
       }
     }
@@ -117,13 +141,13 @@ k_chan_sums(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* 
 
 // Per-channel sums over the batch: a block of 8 warps per (replica, chunk of
 // 32 channels); lane = channel (coalesced loads of the [b][ch][2] sums), warp
-// w takes the examples b = w, w + 8, ... in fp64, and the eight warp partials
-// are added in warp order.  Fixed order, independent of C.
+// w takes the examples b = w, w + 8, ... , and the eight warp partials are
+// added in warp order.  Fixed order, independent of C.
 constexpr int kChanWarps = 8;
 __device__ __forceinline__ void batch_sums(const float* __restrict__ sums, int c, int chn, int B,
-                                           int ch, double* red, double& s1, double& s2) {
+                                           int ch, float* red, float& s1, float& s2) {
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  double a = 0.0, q = 0.0;
+  float a = 0.f, q = 0.f;
   for (int b = w; b < B; b += kChanWarps) {
     const float2 v = *reinterpret_cast<const float2*>(sums + (((int64_t)c * B + b) * ch + chn) * 2);
     a += v.x;
@@ -132,8 +156,8 @@ __device__ __forceinline__ void batch_sums(const float* __restrict__ sums, int c
   red[(w * 32 + lane) * 2] = a;
   red[(w * 32 + lane) * 2 + 1] = q;
   __syncthreads();
-  s1 = 0.0;
-  s2 = 0.0;
+  s1 = 0.f;
+  s2 = 0.f;
   if (w == 0) {
     for (int k = 0; k < kChanWarps; ++k) {
       s1 += red[(k * 32 + lane) * 2];
@@ -154,7 +178,7 @@ k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ ga
                     float* __restrict__ rstd, float2* __restrict__ ss, float* __restrict__ run,
                     int64_t run_rs, int C, int B, int HW, int ch, int gn,
                     const int32_t* __restrict__ upd) {
-  __shared__ double red[kChanWarps * 32 * 2];
+  __shared__ float red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
   const int cpg = ch / 32;
@@ -163,47 +187,47 @@ k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ ga
     if (i >= (int64_t)C * B * 32) return;
     const int64_t cbv = i / 32;                     // c * B + b
     const int g = (int)(i % 32), c = (int)(cbv / B);
-    double s1 = 0.0, s2 = 0.0;
+    float s1 = 0.f, s2 = 0.f;
     for (int k = 0; k < cpg; ++k) {
       const int64_t o = (cbv * ch + g * cpg + k) * 2;
       s1 += sums[o]; s2 += sums[o + 1];
     }
-    const double n = (double)cpg * HW, mu = s1 / n;
-    double var = s2 / n - mu * mu;
-    var = var > 0.0 ? var : 0.0;
-    const double r = 1.0 / sqrt(var + kEps);
-    mean[i] = (float)mu;
-    rstd[i] = (float)r;
+    const float n = (float)cpg * (float)HW, mu = s1 / n;
+    float var = s2 / n - mu * mu;
+    var = var > 0.f ? var : 0.f;
+    const float r = 1.f / sqrtf(var + kEps);
+    mean[i] = mu;
+    rstd[i] = r;
     const float* gm = gamma + (int64_t)c * g_rs;
     const float* bt = beta + (int64_t)c * g_rs;
     for (int k = 0; k < cpg; ++k) {
       const int chn = g * cpg + k;
-      const float sc = (float)((double)gm[chn] * r);
-      ss[cbv * ch + chn] = make_float2(sc, (float)((double)bt[chn] - mu * sc));
+      const float sc = gm[chn] * r;
+      ss[cbv * ch + chn] = make_float2(sc, bt[chn] - mu * sc);
     }
     return;
   }
   const int chunks = ch / 32;
   const int c = blockIdx.x / chunks, s = (blockIdx.x % chunks) * 32 + (threadIdx.x & 31);
-  double s1, s2;
+  float s1, s2;
   batch_sums(sums, c, s, B, ch, red, s1, s2);
   if (threadIdx.x >= 32) return;
-  const double n = (double)B * HW, mu = s1 / n;
-  double var = s2 / n - mu * mu;
-  var = var > 0.0 ? var : 0.0;
-  const double r = 1.0 / sqrt(var + kEps);
+  const float n = (float)B * (float)HW, mu = s1 / n;
+  float var = s2 / n - mu * mu;
+  var = var > 0.f ? var : 0.f;
+  const float r = 1.f / sqrtf(var + kEps);
   const int64_t w = (int64_t)c * ch + s;
-  mean[w] = (float)mu;
-  rstd[w] = (float)r;
+  mean[w] = mu;
+  rstd[w] = r;
   if (run && (!upd || upd[c])) {          // replicas at the fusion barrier keep theirs
     float* rm = run + (int64_t)c * run_rs;
     float* rv = rm + ch;
-    rm[s] = (float)(0.9 * (double)rm[s] + 0.1 * mu);
-    rv[s] = (float)(0.9 * (double)rv[s] + 0.1 * var * n / (n - 1.0));
+    rm[s] = 0.9f * rm[s] + 0.1f * mu;
+    rv[s] = 0.9f * rv[s] + 0.1f * (var * (n / (n - 1.f)));
   }
   const float gsv = gamma[(int64_t)c * g_rs + s], bsv = beta[(int64_t)c * g_rs + s];
-  const float sc = (float)((double)gsv * r);
-  ss[w] = make_float2(sc, (float)((double)bsv - mu * sc));
+  const float sc = gsv * r;
+  ss[w] = make_float2(sc, bsv - mu * sc);
 }
 
 // Backward: per set m1 = mean(dz gamma), m2 = mean(dz gamma x_hat), and the
@@ -220,7 +244,7 @@ k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ ga
                     float4* __restrict__ kk, float* __restrict__ dgamma,
                     float* __restrict__ dbeta, int64_t d_rs, int C, int B, int HW, int ch,
                     int gn) {
-  __shared__ double red[kChanWarps * 32 * 2];
+  __shared__ float red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
   const int cpg = ch / 32;
@@ -228,19 +252,18 @@ k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ ga
   const int nb = C * chunks;
   if ((int)blockIdx.x < nb) {
     const int c = blockIdx.x / chunks, chn = (blockIdx.x % chunks) * 32 + (threadIdx.x & 31);
-    double a, b2;
+    float a, b2;
     batch_sums(sums, c, chn, B, ch, red, a, b2);
     if (threadIdx.x >= 32) return;
-    dgamma[(int64_t)c * d_rs + chn] = (float)b2;
-    dbeta[(int64_t)c * d_rs + chn] = (float)a;
+    dgamma[(int64_t)c * d_rs + chn] = b2;
+    dbeta[(int64_t)c * d_rs + chn] = a;
     if (!gn) {
       const int64_t w = (int64_t)c * ch + chn;
-      const double g = gamma[(int64_t)c * g_rs + chn];
-      const double n = (double)B * HW;
-      const double m1 = g * a / n, m2 = g * b2 / n;
-      const double mu = mean[w], r = rstd[w];
-      kk[w] = make_float4((float)(g * r), (float)(-r * r * m2), (float)(r * r * m2 * mu - r * m1),
-                          0.f);
+      const float g = gamma[(int64_t)c * g_rs + chn];
+      const float n = (float)B * (float)HW;
+      const float m1 = g * a / n, m2 = g * b2 / n;
+      const float mu = mean[w], r = rstd[w];
+      kk[w] = make_float4(g * r, -r * r * m2, r * r * m2 * mu - r * m1, 0.f);
     }
     return;
   }
@@ -250,20 +273,19 @@ k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ ga
   const int64_t cbv = i / 32;
   const int g = (int)(i % 32), c = (int)(cbv / B);
   const float* gm = gamma + (int64_t)c * g_rs;
-  double a = 0.0, b2 = 0.0;
+  float a = 0.f, b2 = 0.f;
   for (int k = 0; k < cpg; ++k) {
     const int chn = g * cpg + k;
     const int64_t o = (cbv * ch + chn) * 2;
-    a += (double)gm[chn] * sums[o];
-    b2 += (double)gm[chn] * sums[o + 1];
+    a = fmaf(gm[chn], sums[o], a);
+    b2 = fmaf(gm[chn], sums[o + 1], b2);
   }
-  const double n = (double)cpg * HW;
-  const double m1 = a / n, m2 = b2 / n;
-  const double mu = mean[i], r = rstd[i];
+  const float n = (float)cpg * (float)HW;
+  const float m1 = a / n, m2 = b2 / n;
+  const float mu = mean[i], r = rstd[i];
   for (int k = 0; k < cpg; ++k) {
     const int chn = g * cpg + k;
-    kk[cbv * ch + chn] = make_float4((float)(gm[chn] * r), (float)(-r * r * m2),
-                                     (float)(r * r * m2 * mu - r * m1), 0.f);
+    kk[cbv * ch + chn] = make_float4(gm[chn] * r, -r * r * m2, r * r * m2 * mu - r * m1, 0.f);
   }
 }
 
@@ -311,6 +333,7 @@ k_norm_apply(const bf16* __restrict__ y, const void* __restrict__ aff, int aff_g
         sc2[2 * k] = q.x; sh2[2 * k] = q.y; sc2[2 * k + 1] = q.z; sh2[2 * k + 1] = q.w;
       }
     }
+#pragma unroll 4
     for (int p = p0 + l; p < p1; p += L) {
       const int64_t o = (cb * HW + p) * ch + v * 8;
       float yy[8], r[8] = {0, 0, 0, 0, 0, 0, 0, 0}, o8[8];
@@ -338,6 +361,7 @@ k_norm_apply(const bf16* __restrict__ y, const void* __restrict__ aff, int aff_g
       const float4 q = k4[k];
       k1[k] = q.x; k2[k] = q.y; k3[k] = q.z;
     }
+#pragma unroll 4
     for (int p = p0 + l; p < p1; p += L) {
       const int64_t o = (cb * HW + p) * ch + v * 8;
       float yy[8], dz[8], o8[8];
@@ -473,35 +497,34 @@ k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* _
   __syncthreads();
   if (threadIdx.x < 32) {
     const int g = threadIdx.x;
-    const double n = (double)cpg * HW;
+    const float n = (float)cpg * (float)HW;
     if (!BWD) {
-      double a = 0.0, q2 = 0.0;
+      float a = 0.f, q2 = 0.f;
       for (int k = 0; k < cpg; ++k) { a += csum[(g * cpg + k) * 2]; q2 += csum[(g * cpg + k) * 2 + 1]; }
-      const double m = a / n;
-      double var = q2 / n - m * m;
-      var = var > 0.0 ? var : 0.0;
-      const double r = 1.0 / sqrt(var + kEps);
-      mean[cb * 32 + g] = (float)m;
-      rstd[cb * 32 + g] = (float)r;
+      const float m = a / n;
+      float var = q2 / n - m * m;
+      var = var > 0.f ? var : 0.f;
+      const float r = 1.f / sqrtf(var + kEps);
+      mean[cb * 32 + g] = m;
+      rstd[cb * 32 + g] = r;
       const float* bt = beta + (int64_t)c * g_rs;
       for (int k = 0; k < cpg; ++k) {
         const int chn = g * cpg + k;
-        const float sc = (float)((double)gm[chn] * r);
-        aff[chn] = make_float4(sc, (float)((double)bt[chn] - m * sc), 0.f, 0.f);
+        const float sc = gm[chn] * r;
+        aff[chn] = make_float4(sc, bt[chn] - m * sc, 0.f, 0.f);
       }
     } else {
-      double a = 0.0, b2 = 0.0;
+      float a = 0.f, b2 = 0.f;
       for (int k = 0; k < cpg; ++k) {
         const int chn = g * cpg + k;
-        a += (double)gm[chn] * csum[chn * 2];
-        b2 += (double)gm[chn] * csum[chn * 2 + 1];
+        a = fmaf(gm[chn], csum[chn * 2], a);
+        b2 = fmaf(gm[chn], csum[chn * 2 + 1], b2);
       }
-      const double m1 = a / n, m2 = b2 / n;
-      const double m = mean[cb * 32 + g], r = rstd[cb * 32 + g];
+      const float m1 = a / n, m2 = b2 / n;
+      const float m = mean[cb * 32 + g], r = rstd[cb * 32 + g];
       for (int k = 0; k < cpg; ++k) {
         const int chn = g * cpg + k;
-        aff[chn] = make_float4((float)(gm[chn] * r), (float)(-r * r * m2),
-                               (float)(r * r * m2 * m - r * m1), 0.f);
+        aff[chn] = make_float4(gm[chn] * r, -r * r * m2, r * r * m2 * m - r * m1, 0.f);
       }
     }
   }
