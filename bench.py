@@ -62,9 +62,9 @@ NCU_TRAFFIC = {
     "conv_wgrad_tc.L2": {"bytes": 2.523e+07, "src_hash": "9edb62919210128c"},
     "conv_wgrad_tc.L3": {"bytes": 8.43e+06, "src_hash": "9edb62919210128c"},
     "sgd": {"bytes": 6.11e+07, "src_hash": "483ce6954d2d1468", "per": "C", "C": 4},
-    "rn_norm_gn_bwd": {"bytes": 9.8362e+07, "src_hash": "d7895818885460a1", "family": "resnet",
+    "rn_norm_gn_bwd": {"bytes": 9.828e+07, "src_hash": "caff47aac58097a3", "family": "resnet",
                        "examples": 256},
-    "rn_norm_gn": {"bytes": 4.7124e+07, "src_hash": "d7895818885460a1", "family": "resnet",
+    "rn_norm_gn": {"bytes": 4.714e+07, "src_hash": "caff47aac58097a3", "family": "resnet",
                    "examples": 256},
 }
 for _k, _v in NCU_TRAFFIC.items():
