@@ -102,6 +102,8 @@ def _declare(L):
     L.orn_set_relu_tol.restype = None
     L.orc_set_relu_masks.argtypes = [ct.c_void_p, _p(ct.c_uint8)]
     L.orc_get_relu_masks.argtypes = [ct.c_void_p, _p(ct.c_uint8)]
+    L.orn_set_norm.argtypes = [ct.c_int, ct.c_double, ct.c_double]
+    L.orc_set_norm.argtypes = [ct.c_void_p, ct.c_int, ct.c_double, ct.c_double]
     L.orn_init_bn_state.argtypes = [f64p]
     L.orn_init_bn_state.restype = None
     L.orc_set_threads.argtypes = [ct.c_int]
@@ -186,11 +188,15 @@ def resnet_mask_elems() -> int:
 
 def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False,
                             label_smoothing: float = 0.0, want_grad: bool = True,
-                            masks_in=None, want_masks: bool = False, classes: int = 10):
-    """ResNet-18 split with a `classes`-way head (10 or 100): (loss, grad[P] or None, cut_act, cut_grad, logits, bn_state
-    after this batch's update of the running statistics[, masks]).  masks:
-    [B][resnet_mask_elems()] uint8 ReLU decisions (stem, then per block those
-    of a1 and of the output, NCHW); masks_in replays given decisions."""
+                            masks_in=None, want_masks: bool = False, classes: int = 10,
+                            gn_groups: int = 32, norm_eps: float = 1e-5,
+                            bn_momentum: float = 0.1):
+    """ResNet-18 split with a `classes`-way head (10 or 100): (loss, grad[P]
+    or None, cut_act, cut_grad, logits, bn_state after this batch's update of
+    the running statistics[, masks]).  masks: [B][resnet_mask_elems()] uint8
+    ReLU decisions (stem, then per block those of a1 and of the output, NCHW);
+    masks_in replays given decisions.  gn_groups / norm_eps / bn_momentum:
+    the norms' hyper-parameters (PyTorch's defaults with 32 groups)."""
     params = np.ascontiguousarray(params, dtype=np.float64)
     x = np.ascontiguousarray(x, dtype=np.float64)
     labels = np.ascontiguousarray(labels, dtype=np.int32)
@@ -201,7 +207,7 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
                               dtype=np.float64).copy()
     loss = np.zeros(1)
     grad = np.zeros(P) if want_grad else None
-    ncut = _cut_elems(RESNET18, B)
+    ncut = _cut_elems(arch, B)
     ca, cg = np.zeros(ncut), np.zeros(ncut)
     logits = np.zeros(B * classes)
     mo = np.zeros((B, resnet_mask_elems()), dtype=np.uint8) if want_masks else None
@@ -209,17 +215,28 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
     if masks_in is not None:
         mi = np.ascontiguousarray(masks_in, dtype=np.uint8)
         assert mi.size == B * resnet_mask_elems()
-    rc = lib().orn_forward_backward_masks(
+    if lib().orn_set_norm(gn_groups, norm_eps, bn_momentum):
+        raise ValueError("bad norm hyper-parameters")
+    try:
+        rc = _resnet_pass(classes, bf16, label_smoothing, params, bn, B, x, labels, loss, grad,
+                          want_grad, ca, cg, logits, mi, mo)
+    finally:
+        lib().orn_set_norm(32, 1e-5, 0.1)
+    if rc:
+        raise RuntimeError(f"oracle resnet forward_backward failed: {rc}")
+    out = (float(loss[0]), grad, ca, cg, logits.reshape(B, classes), bn)
+    return out + (mo,) if want_masks else out
+
+
+def _resnet_pass(classes, bf16, label_smoothing, params, bn, B, x, labels, loss, grad, want_grad,
+                 ca, cg, logits, mi, mo):
+    return lib().orn_forward_backward_masks(
         classes, int(bf16), label_smoothing, _ptr(params, ct.c_double), _ptr(bn, ct.c_double), B,
         _ptr(x, ct.c_double), _ptr(labels, ct.c_int32), _ptr(loss, ct.c_double),
         _ptr(grad, ct.c_double) if want_grad else None, _ptr(ca, ct.c_double),
         _ptr(cg, ct.c_double), _ptr(logits, ct.c_double),
         _ptr(mi, ct.c_uint8) if mi is not None else None,
         _ptr(mo, ct.c_uint8) if mo is not None else None)
-    if rc:
-        raise RuntimeError(f"oracle resnet forward_backward failed: {rc}")
-    out = (float(loss[0]), grad, ca, cg, logits.reshape(B, classes), bn)
-    return out + (mo,) if want_masks else out
 
 
 def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smoothing: float = 0.0,
@@ -276,7 +293,8 @@ class Oracle:
 
     def __init__(self, arch, K, C, assignment, B, F, seed, images, labels, owner, init_params,
                  lr=0.05, momentum=0.0, weight_decay=0.0, nesterov=False, label_smoothing=0.0,
-                 bf16=False, cluster_base=0, augment=False):
+                 bf16=False, cluster_base=0, augment=False, gn_groups=32, norm_eps=1e-5,
+                 bn_momentum=0.1):
         self.arch, self.K, self.C, self.B = arch, K, C, B
         # the context reads the images in place: keep them alive here
         self._images = np.ascontiguousarray(images, dtype=np.float32)
@@ -294,6 +312,9 @@ class Oracle:
             raise ValueError(f"oracle init failed: {rc}")
         self._h = h
         lib().orc_set_augment(h, int(augment))
+        if lib().orc_set_norm(h, gn_groups, norm_eps, bn_momentum):
+            self.__del__()
+            raise ValueError("bad norm hyper-parameters")
         self.P_client = num_params(arch, 0)
         self.P_server = num_params(arch, 1)
 

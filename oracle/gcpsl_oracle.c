@@ -50,6 +50,7 @@ int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const do
                                const uint8_t* masks_in, uint8_t* masks_out);
 int64_t orn_mask_elems(void);
 void orn_init_bn_state(double* state);
+int orn_set_norm(int groups, double eps, double momentum);
 #define ORC_RESNET18 2
 #define ORC_RESNET18_C100 3
 
@@ -558,6 +559,8 @@ typedef struct {
   uint8_t* cand[4];                           /* [C][B][cout][Ho][Wo] of the last round */
   int32_t* ties;                              /* [C][B] ambiguous windows per example */
   int augment;                                /* crop + flip of the sampled images */
+  int gn_groups;                              /* ResNet norms: GroupNorm groups, */
+  double norm_eps, bn_momentum;               /* eps, BatchNorm momentum */
   int64_t R;                                  /* F = -1: rounds per system epoch, else 0 */
   int32_t* upd;                               /* [C] the cluster updated in the last round */
 } orc_ctx;
@@ -587,6 +590,7 @@ int orc_init(int arch, int bf16, double lr, double momentum, double wd, int nest
   c->lr = lr; c->momentum = momentum; c->wd = wd; c->ls = label_smoothing; c->seed = seed;
   c->a = a;
   c->resnet = resnet;
+  c->gn_groups = 32; c->norm_eps = 1e-5; c->bn_momentum = 0.1;
   c->J = J;
   if (resnet) {
     memset(&c->o, 0, sizeof(c->o));
@@ -743,6 +747,14 @@ void orc_augment_image(const float* src, int dy, int dx, int flip, double* dst) 
 
 void orc_set_augment(orc_ctx* c, int on) { c->augment = on != 0; }
 
+/* the ResNet split's norm hyper-parameters (defaults 32, 1e-5, 0.1) */
+int orc_set_norm(orc_ctx* c, int groups, double eps, double momentum) {
+  if (groups < 1 || 64 % groups || !(eps > 0.0) || !(momentum > 0.0 && momentum <= 1.0))
+    return ORC_EINVAL;
+  c->gn_groups = groups; c->norm_eps = eps; c->bn_momentum = momentum;
+  return ORC_OK;
+}
+
 /* the batch's images of cluster k in round t (augmented when set) */
 static void batch_images(const orc_ctx* c, int k, const int32_t* idx, double* dst) {
   for (int b = 0; b < c->B; ++b) {
@@ -784,6 +796,7 @@ int orc_step(orc_ctx* c) {
     c->active[k] = orc_sample_round(c->perm[k], s, B, c->owner, c->K, idx,
                                     c->counts + (int64_t)k * c->K);
     if (c->resnet) {
+      orn_set_norm(c->gn_groups, c->norm_eps, c->bn_momentum);
       batch_images(c, k, idx, c->xbuf);
       for (int b = 0; b < B; ++b) c->ybuf[b] = c->labels[idx[b]];
       int64_t P = c->o.p_total;

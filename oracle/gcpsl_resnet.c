@@ -5,8 +5,9 @@
  * for architectures 2 and 3).  Plain fp64 loops in PyTorch's NCHW / OIHW layouts.
  *
  * Model (the workload's split of the CIFAR ResNet-18):
- *   client: stem conv3x3 3->64 (stride 1, pad 1, no bias), GroupNorm(32), ReLU;
- *           stage 1 = two basic blocks of 64 channels (GroupNorm(32)).
+ *   client: stem conv3x3 3->64 (stride 1, pad 1, no bias), GroupNorm, ReLU;
+ *           stage 1 = two basic blocks of 64 channels (GroupNorm); 32 groups
+ *           unless orn_set_norm chooses another divisor of 64.
  *   server: stages 2-4 (128 / 256 / 512 channels, two basic blocks each, the
  *           first with stride 2 and a 1x1 stride-2 convolution + norm on the
  *           shortcut), train-mode BatchNorm; global average pool over 4x4;
@@ -14,11 +15,13 @@
  *           100 for architecture 3, the CIFAR-100 shape of Section V-A).
  *   basic block: out = relu(N2(conv2(relu(N1(conv1(x))))) + s),
  *                s = x, or Ns(conv_s(x)) when the shape changes.
- *   norms: x_hat = (y - mean) / sqrt(var + 1e-5), var biased, then
+ *   norms: x_hat = (y - mean) / sqrt(var + eps), var biased (eps 1e-5 unless
+ *          orn_set_norm sets it), then
  *          gamma * x_hat + beta; GroupNorm over (channels of the group, H, W)
  *          per example, BatchNorm over (B, H, W) per channel.  BatchNorm's
- *          running statistics follow PyTorch: momentum 0.1, the running
- *          variance takes the unbiased batch variance.
+ *          running statistics follow PyTorch: momentum 0.1 (or the one given
+ *          to orn_set_norm), the running variance takes the unbiased batch
+ *          variance.
  *
  * Canonical parameter blob: PyTorch's named_parameters() order (conv1.weight,
  * bn1.weight, bn1.bias, layer1.0.conv1.weight, ..., shortcut.0.weight,
@@ -37,9 +40,22 @@
 #include <stdlib.h>
 #include <string.h>
 
-#define RN_EPS 1e-5
-#define RN_BN_MOMENTUM 0.1
-#define RN_GROUPS 32
+/* norm hyper-parameters: GroupNorm groups, eps of both norms, BatchNorm
+ * running-statistics momentum (PyTorch's defaults; orn_set_norm) */
+static int RN_GROUPS = 32;
+static double RN_EPS = 1e-5;
+static double RN_BN_MOMENTUM = 0.1;
+
+/* returns nonzero when the group count does not divide every GroupNorm
+ * layer's 64 channels */
+int orn_set_norm(int groups, double eps, double momentum) {
+  if (groups < 1 || 64 % groups || !(eps > 0.0) || !(momentum > 0.0 && momentum <= 1.0))
+    return 1;
+  RN_GROUPS = groups;
+  RN_EPS = eps;
+  RN_BN_MOMENTUM = momentum;
+  return 0;
+}
 
 typedef struct { int cin, cout, k, stride, hin, win; int64_t w; } rn_conv;
 typedef struct { int ch, gn; int64_t g, b; int64_t s; } rn_norm;   /* s: BN state offset */

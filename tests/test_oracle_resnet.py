@@ -15,7 +15,8 @@ RES = synth.ARCH_RESNET18
 RES100 = synth.ARCH_RESNET18_C100
 
 
-def torch_model(blob, x, y, bn_state, label_smoothing=0.0, arch=RES):
+def torch_model(blob, x, y, bn_state, label_smoothing=0.0, arch=RES, groups=32, eps=1e-5,
+                momentum=0.1):
     """Loss, parameter tensors (requires_grad), cut activation (retained
     grad), logits and the BatchNorm state after the batch, with the blob in
     PyTorch's named_parameters() order."""
@@ -36,10 +37,10 @@ def torch_model(blob, x, y, bn_state, label_smoothing=0.0, arch=RES):
         rv = state[soff[0] + c:soff[0] + 2 * c]
         soff[0] += 2 * c
         return F.batch_norm(t, rm, rv, prm[pre + ".weight"], prm[pre + ".bias"], training=True,
-                            momentum=0.1, eps=1e-5)
+                            momentum=momentum, eps=eps)
 
     def gn(t, pre):
-        return F.group_norm(t, 32, prm[pre + ".weight"], prm[pre + ".bias"], eps=1e-5)
+        return F.group_norm(t, groups, prm[pre + ".weight"], prm[pre + ".bias"], eps=eps)
 
     h = F.relu(gn(F.conv2d(x, prm["conv1.weight"], padding=1), "bn1"))
     cut = None
@@ -122,6 +123,30 @@ def test_resnet_matches_torch_fp64_autograd(case, ls):
     scale = np.abs(tgrad).max()
     np.testing.assert_allclose(grad, tgrad, rtol=0, atol=1e-10 * scale)
     np.testing.assert_allclose(bn1, tstate, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("groups,eps,momentum", [(8, 1e-3, 0.2), (1, 1e-4, 1.0)])
+def test_resnet_norm_hyperparameters_match_torch(case, groups, eps, momentum):
+    """Other GroupNorm group counts, norm eps and BatchNorm momentum (the
+    model description's gn_groups / norm_eps / bn_momentum) against PyTorch's
+    group_norm / batch_norm with the same values."""
+    blob, x, y, bn0 = case
+    loss, grad, ca, cg, logits, bn1 = oracle.resnet_forward_backward(
+        blob, x, y, bn_state=bn0, gn_groups=groups, norm_eps=eps, bn_momentum=momentum)
+    tl, tparams, tcut, tlogits, tstate = torch_model(blob, torch.tensor(x), y, bn0,
+                                                     groups=groups, eps=eps, momentum=momentum)
+    tl.backward()
+    tgrad = np.concatenate([p.grad.numpy().ravel() for p in tparams])
+    assert abs(loss - tl.item()) < 1e-12 * max(1.0, abs(loss))
+    np.testing.assert_allclose(ca, tcut.detach().numpy().ravel(), rtol=0, atol=1e-11)
+    np.testing.assert_allclose(grad, tgrad, rtol=0, atol=1e-10 * np.abs(tgrad).max())
+    np.testing.assert_allclose(bn1, tstate, rtol=0, atol=1e-12)
+    # the defaults come back after the call
+    l_def = oracle.resnet_forward_backward(blob, x, y, bn_state=bn0, want_grad=False)[0]
+    t_def = torch_model(blob, torch.tensor(x), y, bn0)[0].item()
+    assert abs(l_def - t_def) < 1e-12 * max(1.0, abs(t_def))
+    with pytest.raises(ValueError):
+        oracle.resnet_forward_backward(blob, x, y, bn_state=bn0, gn_groups=3)
 
 
 def test_resnet100_param_count():
