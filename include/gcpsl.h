@@ -78,7 +78,12 @@ enum { GCPSL_CUT_ACT = 0, GCPSL_CUT_GRAD = 1 };
  *    `seed`: dy = (o0 * 9) >> 32, dx = (o1 * 9) >> 32, flip = o2 & 1, and
  *    out[ch][y][x] = img[ch][y + dy - 4][x' + dx - 4], x' = flip ? 31 - x : x,
  *    0 outside the image.  (The synthetic images are N(0,1) already, so the
- *    dataset normalisation of Section V-A is the identity.)              */
+ *    dataset normalisation of Section V-A is the identity.)
+ *  gn_groups, bn_momentum, norm_eps (ResNet-18 split; Section IV-B keeps
+ *    BatchNorm in the server and puts GroupNorm in the client without fixing
+ *    these): GroupNorm's group count, one of 1, 2, 4, 8, 16, 32 (0 selects
+ *    32); the BatchNorm running-statistics momentum in (0, 1] (0 selects
+ *    PyTorch's 0.1); the eps of both norms, > 0 (0 selects 1e-5).        */
 typedef struct {
   int arch;
   int operand_dtype;
@@ -88,6 +93,8 @@ typedef struct {
   int cluster_id_base;
   int data_on_host;
   int augment;
+  int gn_groups;
+  float bn_momentum, norm_eps;
 } gcpsl_model_desc;
 
 /* Training data of all K clients (Section III-A: client k owns D_k).
@@ -132,7 +139,8 @@ typedef struct gcpsl_ctx gcpsl_ctx;
  *    weights OIHW, linear weight [out][in]); NULL draws them from a fixed
  *    Philox stream as U(-1/sqrt(fan_in), 1/sqrt(fan_in));
  *  out: receives the context.
- * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < -1, assignment
+ * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < -1, norm
+ * hyper-parameters outside the ranges above, assignment
  * outside [-1, C), owner outside [0, K), num_classes other than the
  * architecture's, labels outside [0, num_classes), a cluster with fewer
  * than B examples.  Fusion weights are

@@ -286,8 +286,10 @@ cudaError_t launch_wgrad0_tc(cudaStream_t s, const CUtensorMap& g, const CUtenso
 cudaError_t launch_wgrad_reduce(cudaStream_t s, const float* partial, float* dw, int64_t dw_rs,
                                 int splits, int64_t per, int C, int64_t count = -1);
 
-// norm.cu (GroupNorm with 32 groups / train-mode BatchNorm on [C][B][HW][ch]
-// bf16 tensors; statistics per set: GroupNorm (c, b, group), BatchNorm (c, ch))
+// norm.cu (GroupNorm / train-mode BatchNorm on [C][B][HW][ch] bf16 tensors;
+// statistics per set: GroupNorm (c, b, group), BatchNorm (c, ch)).  gn is the
+// GroupNorm group count (a divisor of ch, at most 32; the per-example mean /
+// rstd arrays keep a stride of 32), 0 for BatchNorm.
 // per-(c, b, ch) pixel sums: forward (sum y, sum y^2); backward (sum dz,
 // sum dz x_hat) with dz = d (times [mask > 0], written to dz_out if set)
 cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16* d,
@@ -300,7 +302,8 @@ cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16
 cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const float* gamma,
                                      const float* beta, int64_t g_rs, float* mean, float* rstd,
                                      float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
-                                     int ch, int gn, const int32_t* upd = nullptr);
+                                     int ch, int gn, float eps, float momentum,
+                                     const int32_t* upd = nullptr);
 // backward affine form kk = (k1, k2, k3, 0): dy = k1 dz + k2 y + k3 per
 // (c, [b,] ch); per channel dgamma, dbeta
 cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,
@@ -315,7 +318,7 @@ cudaError_t launch_norm_apply_fwd(cudaStream_t s, const bf16* y, const float2* s
 cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* kk, int gn,
                                   const bf16* d, const bf16* mask, bf16* out, int C, int B, int HW,
                                   int ch);
-// GroupNorm (32 groups) of one example per block, statistics and apply in
+// GroupNorm (`groups` groups) of one example per block, statistics and apply in
 // one launch: forward out = relu?(norm(y) + res) (res nullable), writing the
 // per-set mean / rstd; backward dy from d (times [mask > 0], kept in dz_out
 // when set) with the per-(example, channel) sums for dgamma / dbeta, which
@@ -323,11 +326,11 @@ cudaError_t launch_norm_apply_bwd(cudaStream_t s, const bf16* y, const float4* k
 cudaError_t launch_gn_fused_fwd(cudaStream_t s, const bf16* y, const bf16* res,
                                 const float* gamma, const float* beta, int64_t g_rs, float* mean,
                                 float* rstd, bf16* out, int C, int B, int HW, int ch, int relu,
-                                int* err);
+                                int groups, float eps, int* err);
 cudaError_t launch_gn_fused_bwd(cudaStream_t s, const bf16* y, const bf16* d, const bf16* mask,
                                 bf16* dz_out, const float* gamma, int64_t g_rs, const float* mean,
                                 const float* rstd, float* sums, bf16* out, int C, int B, int HW,
-                                int ch, int* err);
+                                int ch, int groups, int* err);
 cudaError_t launch_norm_finalize_bwd_channels(cudaStream_t s, const float* sums, float* dgamma,
                                               float* dbeta, int64_t d_rs, int C, int B, int ch);
 cudaError_t launch_avgpool(cudaStream_t s, const bf16* x, bf16* h, int CB, int HW, int ch);

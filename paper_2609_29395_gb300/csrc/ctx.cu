@@ -660,6 +660,9 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
                        const gcpsl_dataset* data, const float* init_params) {
   c->desc = *desc;
   c->K = K; c->C = C; c->B = B; c->F = F; c->seed = seed;
+  c->gn_groups = desc->gn_groups ? desc->gn_groups : 32;
+  c->bn_momentum = desc->bn_momentum > 0.f ? desc->bn_momentum : 0.1f;
+  c->norm_eps = desc->norm_eps > 0.f ? desc->norm_eps : 1e-5f;
   c->bf = desc->operand_dtype == GCPSL_BF16;
   c->esz = c->bf ? 2 : 4;
   c->x0c = c->bf ? 32 : 3;
@@ -882,6 +885,11 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
     return fail(nullptr, GCPSL_E_INVAL, "unknown operand_dtype %d", desc->operand_dtype);
   if (desc->augment != 0 && desc->augment != 1)
     return fail(nullptr, GCPSL_E_INVAL, "augment must be 0 or 1");
+  if (desc->gn_groups < 0 || desc->gn_groups > 32 || (desc->gn_groups && 64 % desc->gn_groups) ||
+      !(desc->bn_momentum >= 0.f && desc->bn_momentum <= 1.f) ||
+      !(desc->norm_eps >= 0.f && desc->norm_eps < 1.f))
+    return fail(nullptr, GCPSL_E_INVAL, "bad norm hyper-parameters (groups %d, momentum %g, eps %g)",
+                desc->gn_groups, (double)desc->bn_momentum, (double)desc->norm_eps);
   if (!(desc->lr >= 0.f) || !(desc->label_smoothing >= 0.f && desc->label_smoothing < 1.f))
     return fail(nullptr, GCPSL_E_INVAL, "bad lr or label_smoothing");
   ArchSpec a;

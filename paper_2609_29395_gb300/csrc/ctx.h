@@ -102,6 +102,9 @@ struct gcpsl_ctx {
   ArchSpec a{};
   int K = 0, C = 0, B = 0, F = 0;
   int J = 10;                       // classes (outputs of the linear head)
+  // ResNet norms: GroupNorm groups, eps of both norms, BatchNorm momentum
+  int gn_groups = 32;
+  float norm_eps = 1e-5f, bn_momentum = 0.1f;
   uint64_t seed = 0;
   bool bf = false;
   size_t esz = 4;

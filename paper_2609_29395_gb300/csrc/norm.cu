@@ -25,7 +25,8 @@ namespace gcpsl {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr float kEps = 1e-5f;
+// per-example stride of the GroupNorm mean / rstd arrays: at most 32 groups
+constexpr int kMaxGroups = 32;
 
 __device__ __forceinline__ void unpack8(const uint4& u, float* f) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
@@ -63,7 +64,7 @@ k_chan_sums(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* 
   const int V = ch / 8;
   const int L = kThreads / V > 0 ? kThreads / V : 1;
   const int v = threadIdx.x % V, l = threadIdx.x / V;
-  const int cpg = ch / 32;
+  const int cpg = gn ? ch / gn : 1;
   const int64_t base = (int64_t)cb * HW * ch;
   float s1[8] = {0, 0, 0, 0, 0, 0, 0, 0}, s2[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   float mu[8], rs[8];
@@ -72,7 +73,8 @@ k_chan_sums(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* 
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int chn = v * 8 + i;
-      const int64_t set = gn ? ((int64_t)c * B + b) * 32 + chn / cpg : (int64_t)c * ch + chn;
+      const int64_t set =
+          gn ? ((int64_t)c * B + b) * kMaxGroups + chn / cpg : (int64_t)c * ch + chn;
       mu[i] = mean[set];
       rs[i] = rstd[set];
     }
@@ -176,17 +178,18 @@ __global__ void __launch_bounds__(kChanWarps * 32)
 k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ gamma,
                     const float* __restrict__ beta, int64_t g_rs, float* __restrict__ mean,
                     float* __restrict__ rstd, float2* __restrict__ ss, float* __restrict__ run,
-                    int64_t run_rs, int C, int B, int HW, int ch, int gn,
-                    const int32_t* __restrict__ upd) {
+                    int64_t run_rs, int C, int B, int HW, int ch, int gn, float eps,
+                    float momentum, const int32_t* __restrict__ upd) {
   __shared__ float red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
-  const int cpg = ch / 32;
   if (gn) {
+    const int cpg = ch / gn;
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= (int64_t)C * B * 32) return;
-    const int64_t cbv = i / 32;                     // c * B + b
-    const int g = (int)(i % 32), c = (int)(cbv / B);
+    if (i >= (int64_t)C * B * gn) return;
+    const int64_t cbv = i / gn;                     // c * B + b
+    const int g = (int)(i % gn), c = (int)(cbv / B);
+    const int64_t set = cbv * kMaxGroups + g;
     float s1 = 0.f, s2 = 0.f;
     for (int k = 0; k < cpg; ++k) {
       const int64_t o = (cbv * ch + g * cpg + k) * 2;
@@ -195,9 +198,9 @@ k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ ga
     const float n = (float)cpg * (float)HW, mu = s1 / n;
     float var = s2 / n - mu * mu;
     var = var > 0.f ? var : 0.f;
-    const float r = 1.f / sqrtf(var + kEps);
-    mean[i] = mu;
-    rstd[i] = r;
+    const float r = 1.f / sqrtf(var + eps);
+    mean[set] = mu;
+    rstd[set] = r;
     const float* gm = gamma + (int64_t)c * g_rs;
     const float* bt = beta + (int64_t)c * g_rs;
     for (int k = 0; k < cpg; ++k) {
@@ -215,15 +218,15 @@ k_norm_finalize_fwd(const float* __restrict__ sums, const float* __restrict__ ga
   const float n = (float)B * (float)HW, mu = s1 / n;
   float var = s2 / n - mu * mu;
   var = var > 0.f ? var : 0.f;
-  const float r = 1.f / sqrtf(var + kEps);
+  const float r = 1.f / sqrtf(var + eps);
   const int64_t w = (int64_t)c * ch + s;
   mean[w] = mu;
   rstd[w] = r;
   if (run && (!upd || upd[c])) {          // replicas at the fusion barrier keep theirs
     float* rm = run + (int64_t)c * run_rs;
     float* rv = rm + ch;
-    rm[s] = 0.9f * rm[s] + 0.1f * mu;
-    rv[s] = 0.9f * rv[s] + 0.1f * (var * (n / (n - 1.f)));
+    rm[s] = (1.f - momentum) * rm[s] + momentum * mu;
+    rv[s] = (1.f - momentum) * rv[s] + momentum * (var * (n / (n - 1.f)));
   }
   const float gsv = gamma[(int64_t)c * g_rs + s], bsv = beta[(int64_t)c * g_rs + s];
   const float sc = gsv * r;
@@ -247,7 +250,6 @@ k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ ga
   __shared__ float red[kChanWarps * 32 * 2];
   pdl_wait();
   pdl_trigger();
-  const int cpg = ch / 32;
   const int chunks = ch / 32;
   const int nb = C * chunks;
   if ((int)blockIdx.x < nb) {
@@ -268,10 +270,12 @@ k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ ga
     return;
   }
   if (!gn) return;
+  const int cpg = ch / gn;
   const int64_t i = (int64_t)(blockIdx.x - nb) * blockDim.x + threadIdx.x;  // set (c, b, g)
-  if (i >= (int64_t)C * B * 32) return;
-  const int64_t cbv = i / 32;
-  const int g = (int)(i % 32), c = (int)(cbv / B);
+  if (i >= (int64_t)C * B * gn) return;
+  const int64_t cbv = i / gn;
+  const int g = (int)(i % gn), c = (int)(cbv / B);
+  const int64_t set = cbv * kMaxGroups + g;
   const float* gm = gamma + (int64_t)c * g_rs;
   float a = 0.f, b2 = 0.f;
   for (int k = 0; k < cpg; ++k) {
@@ -282,7 +286,7 @@ k_norm_finalize_bwd(const float* __restrict__ sums, const float* __restrict__ ga
   }
   const float n = (float)cpg * (float)HW;
   const float m1 = a / n, m2 = b2 / n;
-  const float mu = mean[i], r = rstd[i];
+  const float mu = mean[set], r = rstd[set];
   for (int k = 0; k < cpg; ++k) {
     const int chn = g * cpg + k;
     kk[cbv * ch + chn] = make_float4(gm[chn] * r, -r * r * m2, r * r * m2 * mu - r * m1, 0.f);
@@ -401,7 +405,7 @@ k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* _
            const bf16* __restrict__ res, const float* __restrict__ gamma,
            const float* __restrict__ beta, int64_t g_rs, float* __restrict__ mean,
            float* __restrict__ rstd, float* __restrict__ sums, bf16* __restrict__ dz_out,
-           bf16* __restrict__ out, int B, int HW, int ch, int relu, int* err) {
+           bf16* __restrict__ out, int B, int HW, int ch, int relu, int G, float eps, int* err) {
   extern __shared__ uint4 gsm4[];
   __shared__ uint64_t bar;
   uint8_t* stage = reinterpret_cast<uint8_t*>(gsm4);             // HW x ch bf16
@@ -426,14 +430,14 @@ k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* _
   const int c = (int)(cb / B);
   const int v = threadIdx.x % V, l = threadIdx.x / V;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int cpg = ch / 32;
+  const int cpg = ch / G;
   const int64_t base = cb * HW * ch + v * 8;
   const float* gm = gamma + (int64_t)c * g_rs;
   float mu[8], rs[8];
   if (BWD) {
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const int64_t set = cb * 32 + (v * 8 + i) / cpg;
+      const int64_t set = cb * kMaxGroups + (v * 8 + i) / cpg;
       mu[i] = mean[set];
       rs[i] = rstd[set];
     }
@@ -495,7 +499,7 @@ k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* _
     if (BWD) sums[(cb * ch + chn) * 2 + (k >> 3)] = t;
   }
   __syncthreads();
-  if (threadIdx.x < 32) {
+  if (threadIdx.x < G) {
     const int g = threadIdx.x;
     const float n = (float)cpg * (float)HW;
     if (!BWD) {
@@ -504,9 +508,9 @@ k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* _
       const float m = a / n;
       float var = q2 / n - m * m;
       var = var > 0.f ? var : 0.f;
-      const float r = 1.f / sqrtf(var + kEps);
-      mean[cb * 32 + g] = m;
-      rstd[cb * 32 + g] = r;
+      const float r = 1.f / sqrtf(var + eps);
+      mean[cb * kMaxGroups + g] = m;
+      rstd[cb * kMaxGroups + g] = r;
       const float* bt = beta + (int64_t)c * g_rs;
       for (int k = 0; k < cpg; ++k) {
         const int chn = g * cpg + k;
@@ -521,7 +525,7 @@ k_gn_fused(const bf16* __restrict__ y, const bf16* __restrict__ d, const bf16* _
         b2 = fmaf(gm[chn], csum[chn * 2 + 1], b2);
       }
       const float m1 = a / n, m2 = b2 / n;
-      const float m = mean[cb * 32 + g], r = rstd[cb * 32 + g];
+      const float m = mean[cb * kMaxGroups + g], r = rstd[cb * kMaxGroups + g];
       for (int k = 0; k < cpg; ++k) {
         const int chn = g * cpg + k;
         aff[chn] = make_float4(gm[chn] * r, -r * r * m2, r * r * m2 * m - r * m1, 0.f);
@@ -579,10 +583,13 @@ inline unsigned nblk(int64_t n, int t) { return (unsigned)((n + t - 1) / t); }
 
 }  // namespace
 
+// gn: GroupNorm's group count (it divides ch, at most kMaxGroups), 0 for BatchNorm
+static bool groups_ok(int gn, int ch) { return gn == 0 || (gn > 0 && gn <= kMaxGroups && ch % gn == 0); }
+
 cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16* d,
                              const bf16* mask, const float* mean, const float* rstd, bf16* dz_out,
                              float* sums, int C, int B, int HW, int ch, int gn) {
-  if (ch % 32 || ch / 8 > kThreads) return cudaErrorInvalidValue;
+  if (ch % 32 || ch / 8 > kThreads || !groups_ok(gn, ch)) return cudaErrorInvalidValue;
   const int V = ch / 8, L = kThreads / V;
   const size_t smem = sizeof(float) * (size_t)L * V * 16;
   if (bwd)
@@ -595,19 +602,20 @@ cudaError_t launch_norm_sums(cudaStream_t s, bool bwd, const bf16* y, const bf16
 cudaError_t launch_norm_finalize_fwd(cudaStream_t s, const float* sums, const float* gamma,
                                      const float* beta, int64_t g_rs, float* mean, float* rstd,
                                      float2* ss, float* run, int64_t run_rs, int C, int B, int HW,
-                                     int ch, int gn, const int32_t* upd) {
-  if (ch % 32) return cudaErrorInvalidValue;
-  const unsigned blocks = gn ? nblk((int64_t)C * B * 32, 256) : (unsigned)(C * (ch / 32));
+                                     int ch, int gn, float eps, float momentum,
+                                     const int32_t* upd) {
+  if (ch % 32 || !groups_ok(gn, ch)) return cudaErrorInvalidValue;
+  const unsigned blocks = gn ? nblk((int64_t)C * B * gn, 256) : (unsigned)(C * (ch / 32));
   return launch_k(k_norm_finalize_fwd, blocks, 256, 0, s, sums, gamma, beta, g_rs,
-                  mean, rstd, ss, run, run_rs, C, B, HW, ch, gn, upd);
+                  mean, rstd, ss, run, run_rs, C, B, HW, ch, gn, eps, momentum, upd);
 }
 
 cudaError_t launch_norm_finalize_bwd(cudaStream_t s, const float* sums, const float* gamma,
                                      int64_t g_rs, const float* mean, const float* rstd,
                                      float4* kk, float* dgamma, float* dbeta, int64_t d_rs, int C,
                                      int B, int HW, int ch, int gn) {
-  if (ch % 32) return cudaErrorInvalidValue;
-  const unsigned blocks = (unsigned)(C * (ch / 32)) + (gn ? nblk((int64_t)C * B * 32, 256) : 0u);
+  if (ch % 32 || !groups_ok(gn, ch)) return cudaErrorInvalidValue;
+  const unsigned blocks = (unsigned)(C * (ch / 32)) + (gn ? nblk((int64_t)C * B * gn, 256) : 0u);
   return launch_k(k_norm_finalize_bwd, blocks, 256, 0, s, sums, gamma, g_rs, mean,
                   rstd, kk, dgamma, dbeta, d_rs, C, B, HW, ch, gn);
 }
@@ -655,22 +663,25 @@ static bool gn_shape_ok(int HW, int ch) {
 cudaError_t launch_gn_fused_fwd(cudaStream_t s, const bf16* y, const bf16* res,
                                 const float* gamma, const float* beta, int64_t g_rs, float* mean,
                                 float* rstd, bf16* out, int C, int B, int HW, int ch, int relu,
-                                int* err) {
-  if (!gn_shape_ok(HW, ch) || !gn_attr<false>()) return cudaErrorInvalidValue;
+                                int groups, float eps, int* err) {
+  if (!gn_shape_ok(HW, ch) || groups < 1 || !groups_ok(groups, ch) || !gn_attr<false>())
+    return cudaErrorInvalidValue;
   return launch_k(k_gn_fused<false>, (unsigned)(C * B), kGnThreads, gn_smem(ch), s, y,
                   (const bf16*)nullptr, (const bf16*)nullptr, res, gamma, beta, g_rs, mean, rstd,
-                  (float*)nullptr, (bf16*)nullptr, out, B, HW, ch, relu, err);
+                  (float*)nullptr, (bf16*)nullptr, out, B, HW, ch, relu, groups, eps, err);
 }
 
 cudaError_t launch_gn_fused_bwd(cudaStream_t s, const bf16* y, const bf16* d, const bf16* mask,
                                 bf16* dz_out, const float* gamma, int64_t g_rs, const float* mean,
                                 const float* rstd, float* sums, bf16* out, int C, int B, int HW,
-                                int ch, int* err) {
-  if (!gn_shape_ok(HW, ch) || (dz_out && !mask) || !gn_attr<true>()) return cudaErrorInvalidValue;
+                                int ch, int groups, int* err) {
+  if (!gn_shape_ok(HW, ch) || groups < 1 || !groups_ok(groups, ch) || (dz_out && !mask) ||
+      !gn_attr<true>())
+    return cudaErrorInvalidValue;
   return launch_k(k_gn_fused<true>, (unsigned)(C * B), kGnThreads, gn_smem(ch), s, y, d, mask,
                   (const bf16*)nullptr, gamma, (const float*)nullptr, g_rs,
                   const_cast<float*>(mean), const_cast<float*>(rstd), sums, dz_out, out, B, HW,
-                  ch, 0, err);
+                  ch, 0, groups, 0.f, err);
 }
 
 cudaError_t launch_norm_finalize_bwd_channels(cudaStream_t s, const float* sums, float* dgamma,

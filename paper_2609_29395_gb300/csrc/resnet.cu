@@ -149,6 +149,7 @@ const char* const kDgradName[5] = {"rn_conv_dgrad.stem", "rn_conv_dgrad.s1", "rn
 const char* const kWgradName[5] = {"rn_conv_wgrad.stem", "rn_conv_wgrad.s1", "rn_conv_wgrad.s2",
                                    "rn_conv_wgrad.s3", "rn_conv_wgrad.s4"};
 
+// GroupNorm statistics keep a stride of 32 sets per example (the most groups)
 int64_t sets_of(const RnNorm& n, int B) { return n.gn ? (int64_t)B * 32 : n.ch; }
 
 }  // namespace
@@ -230,6 +231,11 @@ gcpsl_status rn_setup(gcpsl_ctx* c) {
   if (!c->rn) return fail(c, GCPSL_E_NOMEM, "host allocation failed");
   RnState& r = *c->rn;
   rn_layout(r, c->J);
+  // the GroupNorm layers take the context's group count
+  r.stem_n.gn = c->gn_groups;
+  for (auto& b : r.blk)
+    for (RnNorm* n : {&b.n1, &b.n2, &b.ns})
+      if (n->gn) n->gn = c->gn_groups;
   const int C = c->C, B = c->B;
   const int64_t P = c->P_pad;
   auto act = [&](bf16*& p, int64_t elems) -> gcpsl_status {
@@ -459,7 +465,8 @@ gcpsl_status norm_stats(gcpsl_ctx* c, const RnNorm& n, const bf16* y) {
   LAUNCH("rn_norm_finalize",
          launch_norm_finalize_fwd(c->stream, r.sums, th + n.off_g, th + n.off_b, c->P_pad, n.mean,
                                   n.rstd, n.ss, n.gn ? nullptr : r.bn + n.s_off, r.S_pad, c->C,
-                                  c->B, n.hw, n.ch, n.gn, c->d_upd));
+                                  c->B, n.hw, n.ch, n.gn, c->norm_eps, c->bn_momentum,
+                                  c->d_upd));
   return GCPSL_OK;
 }
 
@@ -468,7 +475,7 @@ gcpsl_status gn_fwd(gcpsl_ctx* c, const RnNorm& n, const bf16* y, const bf16* re
   const float* th = c->d_theta;
   LAUNCH("rn_norm_gn", launch_gn_fused_fwd(c->stream, y, res, th + n.off_g, th + n.off_b,
                                            c->P_pad, n.mean, n.rstd, out, c->C, c->B, n.hw, n.ch,
-                                           1, c->d_err));
+                                           1, n.gn, c->norm_eps, c->d_err));
   return GCPSL_OK;
 }
 
@@ -483,7 +490,7 @@ gcpsl_status norm_bwd(gcpsl_ctx* c, const RnNorm& n, const bf16* y, const bf16* 
     // then dgamma / dbeta over the batch
     LAUNCH("rn_norm_gn_bwd",
            launch_gn_fused_bwd(c->stream, y, d, mask, dz_out, th + n.off_g, c->P_pad, n.mean,
-                               n.rstd, r.sums, dy, c->C, c->B, n.hw, n.ch, c->d_err));
+                               n.rstd, r.sums, dy, c->C, c->B, n.hw, n.ch, n.gn, c->d_err));
     LAUNCH("rn_norm_bwd_finalize",
            launch_norm_finalize_bwd_channels(c->stream, r.sums, c->d_grad + n.off_g,
                                              c->d_grad + n.off_b, c->P_pad, c->C, c->B, n.ch));

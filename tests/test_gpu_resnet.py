@@ -135,6 +135,25 @@ def test_resnet18_rounds_against_oracle():
     assert (gpu.bn_state(0) == gpu.bn_state(1)).all()
 
 
+def test_resnet18_norm_hyperparameters_against_oracle():
+    """GroupNorm with 8 groups, eps 1e-3 and BatchNorm momentum 0.2 (the
+    model description's gn_groups / norm_eps / bn_momentum) on both sides."""
+    ds, assign, params = _small(seed=13)
+    kw = dict(lr=0.05, momentum=0.9, gn_groups=8, norm_eps=1e-3, bn_momentum=0.2)
+    gpu = pkg.Context(RES, 8, 2, assign, 8, 0, 4, ds.images, ds.labels, ds.owner, params,
+                      bf16=True, **kw)
+    orc = oracle.Oracle(RES, 8, 2, assign, 8, 0, 4, ds.images, ds.labels, ds.owner, params,
+                        bf16=True, **kw)
+    bn0 = orc.bn_state(0).copy()
+    for _ in range(2):
+        print("cut grad, update:", _round(gpu, orc))
+    # the running statistics moved by the chosen momentum, not PyTorch's 0.1
+    plain = oracle.Oracle(RES, 8, 2, assign, 8, 0, 4, ds.images, ds.labels, ds.owner, params,
+                          bf16=True, lr=0.05, momentum=0.9)
+    plain.step()
+    assert rel_l2(plain.bn_state(0) - bn0, orc.bn_state(0) - bn0) > 0.1
+
+
 def test_resnet18_epoch_schedule_keeps_waiting_batchnorm_state():
     """F = -1 with unequal clusters: a cluster waiting at the fusion barrier
     keeps its parameters, momentum and BatchNorm running statistics (its

@@ -51,8 +51,28 @@ def _ds(n=256, K=8):
     return synth.make_dataset(n, 10, K, 0.5, balanced=False)
 
 
+def test_binding_structs_follow_the_header():
+    """The ctypes mirrors list the header's struct members in order."""
+    hdr = open(os.path.join(ROOT, "include", "gcpsl.h")).read()
+    for struct, cls in (("gcpsl_model_desc", binding.gcpsl_model_desc),
+                        ("gcpsl_dataset", binding.gcpsl_dataset)):
+        body = re.search(r"typedef struct \{([^{}]*)\}\s*" + struct + ";", hdr).group(1)
+        body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+        names = []
+        for decl in body.split(";"):
+            decl = decl.strip()
+            if not decl:
+                continue
+            # "float lr, momentum, weight_decay" / "const float* images"
+            parts = [p.strip() for p in decl.split(",")]
+            names.append(re.findall(r"(\w+)\s*$", parts[0])[0])
+            names += [p.strip("* ") for p in parts[1:]]
+        assert names == [f[0] for f in cls._fields_], (struct, names)
+
+
 @pytest.mark.parametrize("case", ["small_cluster", "assign_range", "owner_range", "label_range",
-                                  "bad_B", "bad_arch", "bad_dtype", "class_count"])
+                                  "bad_B", "bad_arch", "bad_dtype", "class_count", "gn_groups",
+                                  "bn_momentum"])
 def test_init_rejects_bad_arguments(lib, case):
     ds = _ds()
     K, C, B = 8, 2, 16
@@ -71,6 +91,10 @@ def test_init_rejects_bad_arguments(lib, case):
         kw["B"] = 0
     elif case == "bad_arch":
         kw["arch"] = 9
+    elif case == "gn_groups":
+        kw["gn_groups"] = 3             # does not divide the 64 GroupNorm channels
+    elif case == "bn_momentum":
+        kw["bn_momentum"] = 1.5
     with pytest.raises(binding.GcpslError) as e:
         if case == "class_count":
             # a 10-class dataset declared to a 100-class architecture
