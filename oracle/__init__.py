@@ -96,7 +96,7 @@ def _declare(L):
                                        f64p, f64p, f64p, f64p, f64p]
     L.orn_forward_backward_masks.argtypes = [ct.c_int, ct.c_int, ct.c_double, f64p, f64p, ct.c_int, f64p,
                                              i32p, f64p, f64p, f64p, f64p, f64p,
-                                             _p(ct.c_uint8), _p(ct.c_uint8)]
+                                             _p(ct.c_uint8), _p(ct.c_uint8), f64p]
     L.orn_mask_elems.restype = ct.c_int64
     L.orn_set_relu_tol.argtypes = [ct.c_double]
     L.orn_set_relu_tol.restype = None
@@ -104,6 +104,7 @@ def _declare(L):
     L.orc_get_relu_masks.argtypes = [ct.c_void_p, _p(ct.c_uint8)]
     L.orn_set_norm.argtypes = [ct.c_int, ct.c_double, ct.c_double]
     L.orc_set_norm.argtypes = [ct.c_void_p, ct.c_int, ct.c_double, ct.c_double]
+    L.orc_set_client_average.argtypes = [ct.c_void_p, ct.c_int]
     L.orn_init_bn_state.argtypes = [f64p]
     L.orn_init_bn_state.restype = None
     L.orc_set_threads.argtypes = [ct.c_int]
@@ -190,13 +191,15 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
                             label_smoothing: float = 0.0, want_grad: bool = True,
                             masks_in=None, want_masks: bool = False, classes: int = 10,
                             gn_groups: int = 32, norm_eps: float = 1e-5,
-                            bn_momentum: float = 0.1):
+                            bn_momentum: float = 0.1, cut_scale=None):
     """ResNet-18 split with a `classes`-way head (10 or 100): (loss, grad[P]
     or None, cut_act, cut_grad, logits, bn_state after this batch's update of
     the running statistics[, masks]).  masks: [B][resnet_mask_elems()] uint8
     ReLU decisions (stem, then per block those of a1 and of the output, NCHW);
     masks_in replays given decisions.  gn_groups / norm_eps / bn_momentum:
-    the norms' hyper-parameters (PyTorch's defaults with 32 groups)."""
+    the norms' hyper-parameters (PyTorch's defaults with 32 groups).
+    cut_scale ([B], optional) multiplies each example's gradient at the cut
+    before the client backward."""
     params = np.ascontiguousarray(params, dtype=np.float64)
     x = np.ascontiguousarray(x, dtype=np.float64)
     labels = np.ascontiguousarray(labels, dtype=np.int32)
@@ -218,8 +221,10 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
     if lib().orn_set_norm(gn_groups, norm_eps, bn_momentum):
         raise ValueError("bad norm hyper-parameters")
     try:
+        cs = None if cut_scale is None else np.ascontiguousarray(cut_scale, dtype=np.float64)
+        assert cs is None or cs.size == B
         rc = _resnet_pass(classes, bf16, label_smoothing, params, bn, B, x, labels, loss, grad,
-                          want_grad, ca, cg, logits, mi, mo)
+                          want_grad, ca, cg, logits, mi, mo, cs)
     finally:
         lib().orn_set_norm(32, 1e-5, 0.1)
     if rc:
@@ -229,14 +234,15 @@ def resnet_forward_backward(params, x, labels, bn_state=None, bf16: bool = False
 
 
 def _resnet_pass(classes, bf16, label_smoothing, params, bn, B, x, labels, loss, grad, want_grad,
-                 ca, cg, logits, mi, mo):
+                 ca, cg, logits, mi, mo, cs):
     return lib().orn_forward_backward_masks(
         classes, int(bf16), label_smoothing, _ptr(params, ct.c_double), _ptr(bn, ct.c_double), B,
         _ptr(x, ct.c_double), _ptr(labels, ct.c_int32), _ptr(loss, ct.c_double),
         _ptr(grad, ct.c_double) if want_grad else None, _ptr(ca, ct.c_double),
         _ptr(cg, ct.c_double), _ptr(logits, ct.c_double),
         _ptr(mi, ct.c_uint8) if mi is not None else None,
-        _ptr(mo, ct.c_uint8) if mo is not None else None)
+        _ptr(mo, ct.c_uint8) if mo is not None else None,
+        _ptr(cs, ct.c_double) if cs is not None else None)
 
 
 def forward_backward(arch: int, params, x, labels, bf16: bool = False, label_smoothing: float = 0.0,
@@ -294,7 +300,7 @@ class Oracle:
     def __init__(self, arch, K, C, assignment, B, F, seed, images, labels, owner, init_params,
                  lr=0.05, momentum=0.0, weight_decay=0.0, nesterov=False, label_smoothing=0.0,
                  bf16=False, cluster_base=0, augment=False, gn_groups=32, norm_eps=1e-5,
-                 bn_momentum=0.1):
+                 bn_momentum=0.1, client_average=False):
         self.arch, self.K, self.C, self.B = arch, K, C, B
         # the context reads the images in place: keep them alive here
         self._images = np.ascontiguousarray(images, dtype=np.float32)
@@ -315,6 +321,9 @@ class Oracle:
         if lib().orc_set_norm(h, gn_groups, norm_eps, bn_momentum):
             self.__del__()
             raise ValueError("bad norm hyper-parameters")
+        if lib().orc_set_client_average(h, int(client_average)):
+            self.__del__()
+            raise MemoryError("oracle allocation failed")
         self.P_client = num_params(arch, 0)
         self.P_server = num_params(arch, 1)
 

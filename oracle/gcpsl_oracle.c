@@ -47,7 +47,8 @@ int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const do
                                double* bn_state, int B, const double* x,
                                const int32_t* labels, double* loss_out, double* grad,
                                double* cut_act, double* cut_grad, double* logits_out,
-                               const uint8_t* masks_in, uint8_t* masks_out);
+                               const uint8_t* masks_in, uint8_t* masks_out,
+                               const double* cut_scale);
 int64_t orn_mask_elems(void);
 void orn_init_bn_state(double* state);
 int orn_set_norm(int groups, double eps, double momentum);
@@ -411,9 +412,11 @@ static int work_alloc(work_t* w, const arch_t* a, const offs_t* o, int B) {
   return ORC_OK;
 }
 
+/* cut_scale (nullable, [B]): per-example factor on the gradient at the cut
+ * before the client segment's backward (see orc_set_client_average) */
 static int fwd_bwd(const arch_t* a, const offs_t* o, int bf16, double label_smoothing,
                    const double* params, int B, const int32_t* labels, work_t* w,
-                   double* loss_out, double* grad, double tie_tol) {
+                   double* loss_out, double* grad, double tie_tol, const double* cut_scale) {
   int L = a->ncl + a->nsv;
   /* operand copy: bf16(theta) for weights in bf16 mode; biases stay exact */
   memcpy(w->wr, params, sizeof(double) * (size_t)o->p_total);
@@ -481,6 +484,11 @@ static int fwd_bwd(const arch_t* a, const offs_t* o, int bf16, double label_smoo
   /* conv layers backward, last to first; layer 0 needs no data gradient */
   for (int i = L - 1; i >= 0; --i) {
     const conv_l* c = &a->conv[i];
+    if (i == a->ncl - 1 && cut_scale) {
+      const int64_t per = conv_out_elems(c, 1), n = per * B;
+      for (int64_t k = 0; k < n; ++k) w->dact[i + 1][k] *= cut_scale[k / per];
+      round_buf(w->dact[i + 1], n, bf16);
+    }
     int64_t np = (int64_t)B * c->cout * c->h * c->w;
     relu_pool_bwd(B, c->cout, c->h, c->w, c->pool, w->pre[i], w->arg[i], w->dact[i + 1], w->dpre);
     round_buf(w->dpre, np, bf16);
@@ -506,7 +514,7 @@ int orc_forward_backward(int arch, int bf16, double label_smoothing, const doubl
   if (work_alloc(&w, &a, &o, B)) return ORC_ENOMEM;
   memcpy(w.act[0], x, sizeof(double) * (size_t)B * 3072);
   double* g = grad ? grad : NULL;
-  int rc = fwd_bwd(&a, &o, bf16, label_smoothing, params, B, labels, &w, loss, g, 0.0);
+  int rc = fwd_bwd(&a, &o, bf16, label_smoothing, params, B, labels, &w, loss, g, 0.0, NULL);
   int64_t ncut = conv_out_elems(&a.conv[a.ncl - 1], B);
   if (cut_act) memcpy(cut_act, w.act[a.ncl], sizeof(double) * (size_t)ncut);
   if (cut_grad && g) memcpy(cut_grad, w.dact[a.ncl], sizeof(double) * (size_t)ncut);
@@ -559,6 +567,8 @@ typedef struct {
   uint8_t* cand[4];                           /* [C][B][cout][Ho][Wo] of the last round */
   int32_t* ties;                              /* [C][B] ambiguous windows per example */
   int augment;                                /* crop + flip of the sampled images */
+  int client_average;                         /* see orc_set_client_average */
+  double* cut_scale;                          /* [B] factors of the current cluster */
   int gn_groups;                              /* ResNet norms: GroupNorm groups, */
   double norm_eps, bn_momentum;               /* eps, BatchNorm momentum */
   int64_t R;                                  /* F = -1: rounds per system epoch, else 0 */
@@ -674,7 +684,7 @@ void orc_destroy(orc_ctx* c) {
   free(c->ids); free(c->perm); free(c->nc); free(c->cur_epoch); free(c->q); free(c->upd);
   free(c->labels); free(c->owner); free(c->theta); free(c->mom); free(c->grad);
   free(c->idx); free(c->counts); free(c->loss); free(c->active);
-  free(c->cut_act); free(c->cut_grad); free(c->ybuf); free(c->ties); free(c->xbuf); free(c->bn); free(c->relu_rec); free(c->relu_in);
+  free(c->cut_act); free(c->cut_grad); free(c->cut_scale); free(c->ybuf); free(c->ties); free(c->xbuf); free(c->bn); free(c->relu_rec); free(c->relu_in);
   for (int i = 0; i < 4; ++i) free(c->cand[i]);
   work_free(&c->w);
   free(c);
@@ -747,6 +757,21 @@ void orc_augment_image(const float* src, int dy, int dx, int flip, double* dst) 
 
 void orc_set_augment(orc_ctx* c, int on) { c->augment = on != 0; }
 
+/* Sec. IV-B's "average active client gradients", read as the unweighted
+ * mean over the round's active clients of each client's mean-loss
+ * gradient: the client segment's gradient then weights example i of client
+ * k by 1 / (|A| b_k) instead of 1 / B, i.e. the gradient at the cut is
+ * scaled by B / (|A| b_k) before the client backward (0: off, the
+ * example-weighted default, the gradient of the batch-mean loss). */
+int orc_set_client_average(orc_ctx* c, int on) {
+  c->client_average = on != 0;
+  if (on && !c->cut_scale) {
+    c->cut_scale = (double*)malloc(sizeof(double) * (size_t)c->B);
+    if (!c->cut_scale) return ORC_ENOMEM;
+  }
+  return ORC_OK;
+}
+
 /* the ResNet split's norm hyper-parameters (defaults 32, 1e-5, 0.1) */
 int orc_set_norm(orc_ctx* c, int groups, double eps, double momentum) {
   if (groups < 1 || 64 % groups || !(eps > 0.0) || !(momentum > 0.0 && momentum <= 1.0))
@@ -795,6 +820,14 @@ int orc_step(orc_ctx* c) {
     int32_t* idx = c->idx + (int64_t)k * B;
     c->active[k] = orc_sample_round(c->perm[k], s, B, c->owner, c->K, idx,
                                     c->counts + (int64_t)k * c->K);
+    const double* cut_scale = NULL;
+    if (c->client_average) {
+      /* example b of client k: B / (|A| b_k) */
+      const int32_t* cnt = c->counts + (int64_t)k * c->K;
+      for (int b = 0; b < B; ++b)
+        c->cut_scale[b] = (double)B / ((double)c->active[k] * (double)cnt[c->owner[idx[b]]]);
+      cut_scale = c->cut_scale;
+    }
     if (c->resnet) {
       orn_set_norm(c->gn_groups, c->norm_eps, c->bn_momentum);
       batch_images(c, k, idx, c->xbuf);
@@ -811,7 +844,8 @@ int orc_step(orc_ctx* c) {
       int rc = orn_forward_backward_masks(
           c->J, c->bf16, c->ls, c->theta + k * P, c->bn + k * c->S, B, c->xbuf, c->ybuf, &c->loss[k],
           c->grad + k * P, c->cut_act + k * c->ncut, c->cut_grad + k * c->ncut, NULL,
-          c->replay ? c->relu_in + (int64_t)k * B * E : NULL, c->relu_rec + (int64_t)k * B * E);
+          c->replay ? c->relu_in + (int64_t)k * B * E : NULL, c->relu_rec + (int64_t)k * B * E,
+          cut_scale);
       if (bn_keep) {
         memcpy(c->bn + k * c->S, bn_keep, sizeof(double) * (size_t)c->S);
         free(bn_keep);
@@ -823,7 +857,7 @@ int orc_step(orc_ctx* c) {
     for (int b = 0; b < B; ++b) c->ybuf[b] = c->labels[idx[b]];
     int64_t P = c->o.p_total;
     int rc = fwd_bwd(&c->a, &c->o, c->bf16, c->ls, c->theta + k * P, B, c->ybuf, &c->w,
-                     &c->loss[k], c->grad + k * P, c->tie_tol);
+                     &c->loss[k], c->grad + k * P, c->tie_tol, cut_scale);
     if (rc) return rc;
     for (int b = 0; b < B; ++b) c->ties[(int64_t)k * B + b] = 0;
     for (int i = 0; i < c->a.ncl + c->a.nsv; ++i) {

@@ -363,14 +363,16 @@ int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const do
                                double* bn_state, int B, const double* x,
                                const int32_t* labels, double* loss_out, double* grad,
                                double* cut_act, double* cut_grad, double* logits_out,
-                               const uint8_t* masks_in, uint8_t* masks_out);
+                               const uint8_t* masks_in, uint8_t* masks_out,
+                               const double* cut_scale);
 
 int orn_forward_backward(int J, int bf16, double label_smoothing, const double* params,
                          double* bn_state, int B, const double* x, const int32_t* labels,
                          double* loss_out, double* grad, double* cut_act, double* cut_grad,
                          double* logits_out) {
   return orn_forward_backward_masks(J, bf16, label_smoothing, params, bn_state, B, x, labels,
-                                    loss_out, grad, cut_act, cut_grad, logits_out, NULL, NULL);
+                                    loss_out, grad, cut_act, cut_grad, logits_out, NULL, NULL,
+                                    NULL);
 }
 
 /* ReLU decisions per example: the stem's then, per block, those of a1 and of
@@ -390,12 +392,16 @@ int64_t orn_mask_elems(void) {
  * decision record ([B][orn_mask_elems()] in the order stem, block 0 a1,
  * block 0 out, ...; bits as in norm_fwd), and masks_in (nullable) replaces
  * the sign tests by the given decisions (bit 0), so that a run can follow
- * another run's (e.g. the GPU's) branches exactly. */
+ * another run's (e.g. the GPU's) branches exactly.  cut_scale (nullable,
+ * [B]) multiplies each example's gradient at the cut before the client
+ * segment's backward (the per-client average of Sec. IV-B's other reading;
+ * cut_grad receives the scaled gradient). */
 int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const double* params,
                                double* bn_state, int B, const double* x,
                                const int32_t* labels, double* loss_out, double* grad,
                                double* cut_act, double* cut_grad, double* logits_out,
-                               const uint8_t* masks_in, uint8_t* masks_out) {
+                               const uint8_t* masks_in, uint8_t* masks_out,
+                               const double* cut_scale) {
   rn_net n;
   if (B <= 0 || J < 2) return 1;
   rn_build(&n, J);
@@ -606,6 +612,11 @@ int orn_forward_backward_masks(int J, int bf16, double label_smoothing, const do
         for (int64_t k = 0; k < in_e; ++k) dx[k] += dz[k];
       }
       rn_round(dx, in_e, bf16);
+      if (i == 2 && cut_scale) {
+        const int64_t per = in_e / B;
+        for (int64_t k = 0; k < in_e; ++k) dx[k] *= cut_scale[k / per];
+        rn_round(dx, in_e, bf16);
+      }
       if (i == 2 && cut_grad) memcpy(cut_grad, dx, sizeof(double) * (size_t)in_e);
       free(dz); free(dy2); free(da1); free(dy1);
       free(dout);

@@ -460,3 +460,38 @@ def test_epoch_schedule_barrier_and_fusion():
     np.testing.assert_allclose(fused, expect, rtol=0, atol=1e-12 * np.abs(expect).max())
     s, e = clustering.ideal_schedule_speedup(sizes, B)
     assert abs(s - r.sum() / R) < 1e-12 and abs(e - s / 3) < 1e-12
+
+
+@pytest.mark.parametrize("arch", [synth.ARCH_TINY_CNN, synth.ARCH_SPLIT_CNN])
+def test_client_average_is_the_mean_of_per_client_gradients(arch):
+    """client_average (Sec. IV-B's other reading): the client segment's
+    gradient is the unweighted mean over the round's active clients of each
+    client's mean-loss gradient, each computed by an independent forward /
+    backward of that client's examples alone; the server segment keeps the
+    gradient of the batch-mean loss.  fp64, lr 1, no momentum: the update
+    is minus the gradient."""
+    B, K = 16, 8
+    ds = _tiny_world(K=K, seed=4)
+    blob = synth.init_params(arch, seed=5).astype(np.float64)
+    orc = oracle.Oracle(arch, K, 1, np.zeros(K, np.int32), B, 0, 4, ds.images, ds.labels,
+                        ds.owner, blob, lr=1.0, client_average=True)
+    orc.step()
+    idx, counts = orc.sample()
+    idx = idx[0]
+    owners = ds.owner[idx]
+    active = np.flatnonzero(counts[0])
+    assert len(active) > 1 and len(set(counts[0][active])) > 1   # unequal b_k
+    g = blob - orc.all_params(0)
+    pc = oracle.num_params(arch, 0)
+    want_c = np.zeros(pc)
+    for k in active:
+        sel = idx[owners == k]
+        gk = oracle.forward_backward(arch, blob, ds.images[sel].astype(np.float64),
+                                     ds.labels[sel])[1]
+        want_c += gk[:pc] / len(active)
+    full = oracle.forward_backward(arch, blob, ds.images[idx].astype(np.float64),
+                                   ds.labels[idx])[1]
+    np.testing.assert_allclose(g[:pc], want_c, rtol=0, atol=1e-10 * np.abs(want_c).max())
+    np.testing.assert_allclose(g[pc:], full[pc:], rtol=0, atol=1e-10 * np.abs(full[pc:]).max())
+    # and it differs from the example-weighted default when the b_k differ
+    assert np.abs(g[:pc] - full[:pc]).max() > 1e-3 * np.abs(full[:pc]).max()

@@ -149,6 +149,30 @@ def test_resnet_norm_hyperparameters_match_torch(case, groups, eps, momentum):
         oracle.resnet_forward_backward(blob, x, y, bn_state=bn0, gn_groups=3)
 
 
+def test_resnet_cut_scale_matches_torch(case):
+    """The per-client average's cut scaling on the ResNet split: the client
+    segment's gradient is the backward of (cut gradient x s_b) through the
+    client (PyTorch: autograd.grad with those grad_outputs); the server's
+    gradient and the loss are unchanged."""
+    blob, x, y, bn0 = case
+    s = np.array([0.5, 2.0, 1.25])
+    loss, grad, ca, cg, logits, bn1 = oracle.resnet_forward_backward(
+        blob, x, y, bn_state=bn0, cut_scale=s)
+    plain = oracle.resnet_forward_backward(blob, x, y, bn_state=bn0)
+    tl, tparams, tcut, tlogits, tstate = torch_model(blob, torch.tensor(x), y, bn0)
+    tl.backward(retain_graph=True)
+    pc = oracle.num_params(RES, 0)
+    ncl = len(synth.param_shapes(RES, "client"))
+    client = tparams[:ncl]
+    go = tcut.grad.clone() * torch.tensor(s).view(-1, 1, 1, 1)
+    tc = torch.autograd.grad(tcut, client, grad_outputs=go)
+    want_c = np.concatenate([t.numpy().ravel() for t in tc])
+    assert abs(loss - plain[0]) == 0.0
+    np.testing.assert_allclose(grad[:pc], want_c, rtol=0, atol=1e-10 * np.abs(want_c).max())
+    np.testing.assert_array_equal(grad[pc:], plain[1][pc:])
+    np.testing.assert_allclose(cg, go.numpy().ravel(), rtol=0, atol=1e-12 * np.abs(cg).max())
+
+
 def test_resnet100_param_count():
     assert oracle.num_params(RES100, 0) == oracle.num_params(RES, 0) == 149824
     assert oracle.num_params(RES100, 1) == synth.num_params(RES100, "server") == \
