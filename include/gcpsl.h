@@ -83,7 +83,15 @@ enum { GCPSL_CUT_ACT = 0, GCPSL_CUT_GRAD = 1 };
  *    BatchNorm in the server and puts GroupNorm in the client without fixing
  *    these): GroupNorm's group count, one of 1, 2, 4, 8, 16, 32 (0 selects
  *    32); the BatchNorm running-statistics momentum in (0, 1] (0 selects
- *    PyTorch's 0.1); the eps of both norms, > 0 (0 selects 1e-5).        */
+ *    PyTorch's 0.1); the eps of both norms, > 0 (0 selects 1e-5).
+ *  client_average: how a cluster's client gradient averages the round's
+ *    active clients (Sec. IV-B).  0 (default): the gradient of the
+ *    batch-mean loss, i.e. each client weighted by its b_{k,t} examples.
+ *    1: the unweighted mean over the active clients A of each client's
+ *    mean-loss gradient: the gradient at the cut is multiplied, example by
+ *    example, by B / (|A| b_{k,t}) before the client segment's backward
+ *    (the server segment keeps the batch mean; gcpsl_get_cut's gradient is
+ *    the scaled one).                                                     */
 typedef struct {
   int arch;
   int operand_dtype;
@@ -95,6 +103,7 @@ typedef struct {
   int augment;
   int gn_groups;
   float bn_momentum, norm_eps;
+  int client_average;
 } gcpsl_model_desc;
 
 /* Training data of all K clients (Section III-A: client k owns D_k).
@@ -140,7 +149,8 @@ typedef struct gcpsl_ctx gcpsl_ctx;
  *    Philox stream as U(-1/sqrt(fan_in), 1/sqrt(fan_in));
  *  out: receives the context.
  * Rejects (GCPSL_E_INVAL): NULL pointers, K/C/B <= 0, F < -1, norm
- * hyper-parameters outside the ranges above, assignment
+ * hyper-parameters outside the ranges above, augment or client_average
+ * other than 0 / 1, assignment
  * outside [-1, C), owner outside [0, K), num_classes other than the
  * architecture's, labels outside [0, num_classes), a cluster with fewer
  * than B examples.  Fusion weights are

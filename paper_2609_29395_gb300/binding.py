@@ -41,7 +41,8 @@ class gcpsl_model_desc(ct.Structure):
                 ("momentum", ct.c_float), ("weight_decay", ct.c_float), ("nesterov", ct.c_int),
                 ("label_smoothing", ct.c_float), ("cluster_id_base", ct.c_int),
                 ("data_on_host", ct.c_int), ("augment", ct.c_int), ("gn_groups", ct.c_int),
-                ("bn_momentum", ct.c_float), ("norm_eps", ct.c_float)]
+                ("bn_momentum", ct.c_float), ("norm_eps", ct.c_float),
+                ("client_average", ct.c_int)]
 
 
 class gcpsl_dataset(ct.Structure):
@@ -163,13 +164,14 @@ class Context:
     def __init__(self, arch, K, C, assignment, B, F, seed, images, labels, owner,
                  init_params=None, lr=0.05, momentum=0.0, weight_decay=0.0, nesterov=False,
                  label_smoothing=0.0, bf16=True, cluster_id_base=0, data_on_host=False,
-                 augment=False, gn_groups=32, norm_eps=1e-5, bn_momentum=0.1):
+                 augment=False, gn_groups=32, norm_eps=1e-5, bn_momentum=0.1,
+                 client_average=False):
         L = load()
         self.K, self.C, self.B, self.arch = K, C, B, arch
         desc = gcpsl_model_desc(arch, GCPSL_BF16 if bf16 else GCPSL_F32, lr, momentum,
                                 weight_decay, int(nesterov), label_smoothing, cluster_id_base,
                                 int(data_on_host), int(augment), gn_groups, bn_momentum,
-                                norm_eps)
+                                norm_eps, int(client_average))
         images = np.ascontiguousarray(images, dtype=np.float32)
         labels = np.ascontiguousarray(labels, dtype=np.int32)
         owner = np.ascontiguousarray(owner, dtype=np.int32)

@@ -140,6 +140,14 @@ cudaError_t launch_gather<float>(cudaStream_t s, const float* images, const int3
 template <>
 cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
                                 bf16* x0, const AugArgs& aug);
+// per-client average (Sec. IV-B, the unweighted reading): a ([C B][per_a])
+// and b ([C B][per_b], nullable) scaled in place, example cb by
+// B / (active[c] counts[c][owner[idx[cb]]]); per_* multiples of 8
+template <typename T>
+cudaError_t launch_client_avg_scale(cudaStream_t s, T* a, int64_t per_a, T* b, int64_t per_b,
+                                    const int32_t* idx, const int32_t* owner,
+                                    const int32_t* counts, const int32_t* active, int C, int B,
+                                    int K);
 
 // conv_simt.cu
 template <typename T>

@@ -371,6 +371,13 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
     if (!g_ready[i])
       LAUNCH("relu_pool_bwd", launch_relu_pool_bwd<T>(s, dact[i + 1], c->d_code[i], act[i + 1],
                                                       g, C, B, cs));
+    if (i == a.ncl - 1 && c->desc.client_average)
+      // the per-client average: g of the client's last layer and the stored
+      // cut gradient, per example by B / (|A| b_k)
+      LAUNCH("client_avg", launch_client_avg_scale<T>(
+                               s, g, (int64_t)cs.h * cs.w * cs.cout, dact[a.ncl],
+                               act_elems(c, a.ncl) / ((int64_t)C * B), c->d_idx, c->d_owner,
+                               c->d_counts, c->d_active, C, B, c->K));
     const auto& R = c->red[i];
     if (L.on) {
       // weights and bias together (the bias follows the weight in the store);
@@ -885,6 +892,8 @@ gcpsl_status gcpsl_init(const gcpsl_model_desc* desc, int K, int C, const int32_
     return fail(nullptr, GCPSL_E_INVAL, "unknown operand_dtype %d", desc->operand_dtype);
   if (desc->augment != 0 && desc->augment != 1)
     return fail(nullptr, GCPSL_E_INVAL, "augment must be 0 or 1");
+  if (desc->client_average != 0 && desc->client_average != 1)
+    return fail(nullptr, GCPSL_E_INVAL, "client_average must be 0 or 1");
   if (desc->gn_groups < 0 || desc->gn_groups > 32 || (desc->gn_groups && 64 % desc->gn_groups) ||
       !(desc->bn_momentum >= 0.f && desc->bn_momentum <= 1.f) ||
       !(desc->norm_eps >= 0.f && desc->norm_eps < 1.f))

@@ -192,6 +192,35 @@ k_gather_im2col(const float* __restrict__ images, const int32_t* __restrict__ id
   }
 }
 
+// The per-client average of Sec. IV-B's other reading: example b of cluster
+// c, owned by client k, has its gradient at the cut multiplied by
+// B / (|A_c| b_k) before the client segment's backward.  Grid (chunks of
+// kScaleThreads x 8 elements, C B examples); a and b (nullable) are
+// [C B][per] tensors scaled in place, 8 elements per thread.
+constexpr int kScaleThreads = 256;
+template <typename T>
+__global__ void __launch_bounds__(kScaleThreads)
+k_client_avg_scale(T* __restrict__ a, T* __restrict__ b2, int64_t per_a, int64_t per_b,
+                   const int32_t* __restrict__ idx, const int32_t* __restrict__ owner,
+                   const int32_t* __restrict__ counts, const int32_t* __restrict__ active, int B,
+                   int K) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t cb = blockIdx.y;
+  const int c = (int)(cb / B);
+  const int cnt = counts[(int64_t)c * K + owner[idx[cb]]];
+  const float sc = (float)B / ((float)active[c] * (float)cnt);
+  const int64_t e = ((int64_t)blockIdx.x * kScaleThreads + threadIdx.x) * 8;
+  for (int t = 0; t < 2; ++t) {
+    T* p = t == 0 ? a : b2;
+    const int64_t per = t == 0 ? per_a : per_b;
+    if (!p || e >= per) continue;
+    T* q = p + cb * per + e;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) q[i] = from_f<T>(to_f(q[i]) * sc);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_epoch_keys(cudaStream_t s, const int32_t* ids, const int64_t* off,
@@ -230,5 +259,24 @@ cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32
                                 bf16* x0, const AugArgs& aug) {
   return launch_k(k_gather_im2col, (unsigned)CB, kIm2colThreads, 0, s, images, idx, x0, aug);
 }
+
+template <typename T>
+cudaError_t launch_client_avg_scale(cudaStream_t s, T* a, int64_t per_a, T* b, int64_t per_b,
+                                    const int32_t* idx, const int32_t* owner,
+                                    const int32_t* counts, const int32_t* active, int C, int B,
+                                    int K) {
+  if (per_a % 8 || per_b % 8 || (uintptr_t)a % 16 || (uintptr_t)b % 16)
+    return cudaErrorInvalidValue;
+  const int64_t per = per_a > per_b ? per_a : per_b;
+  const dim3 grid((unsigned)((per / 8 + kScaleThreads - 1) / kScaleThreads), (unsigned)(C * B));
+  return launch_k(k_client_avg_scale<T>, grid, kScaleThreads, 0, s, a, b, per_a, per_b, idx,
+                  owner, counts, active, B, K);
+}
+template cudaError_t launch_client_avg_scale<float>(cudaStream_t, float*, int64_t, float*, int64_t,
+                                                    const int32_t*, const int32_t*,
+                                                    const int32_t*, const int32_t*, int, int, int);
+template cudaError_t launch_client_avg_scale<bf16>(cudaStream_t, bf16*, int64_t, bf16*, int64_t,
+                                                   const int32_t*, const int32_t*, const int32_t*,
+                                                   const int32_t*, int, int, int);
 
 }  // namespace gcpsl

@@ -170,6 +170,36 @@ def test_splitcnn_bf16_rounds_with_fusion():
         check_round(gpu, orc, synth.ARCH_SPLIT_CNN)
 
 
+def test_client_average_rounds_bf16_and_fp32():
+    """The per-client average (client_average = 1): the cut gradient scaled by
+    B / (|A| b_k) per example before the client backward, on the bf16
+    tensor-core path (SplitCNN) and the fp32 path (the 512-image workload);
+    the usual bars against the oracle with the same flag, and the client
+    update differs from the example-weighted one."""
+    ds, assign, params = _splitcnn_small(C=4, n=4096)
+    kw = dict(lr=0.05, momentum=0.9, client_average=True)
+    gpu, orc = pair(synth.ARCH_SPLIT_CNN, 32, 4, assign, 32, 2, ds, params, True, **kw)
+    for _ in range(3):
+        check_round(gpu, orc, synth.ARCH_SPLIT_CNN)
+    plain = pkg.Context(synth.ARCH_SPLIT_CNN, 32, 4, assign, 32, 2, 4, ds.images, ds.labels,
+                        ds.owner, params, lr=0.05, momentum=0.9)
+    avg = pkg.Context(synth.ARCH_SPLIT_CNN, 32, 4, assign, 32, 2, 4, ds.images, ds.labels,
+                      ds.owner, params, **kw)
+    plain.step()
+    avg.step()
+    pc = plain.P_client
+    assert not np.array_equal(plain.all_params(0)[:pc], avg.all_params(0)[:pc])
+    np.testing.assert_array_equal(plain.all_params(0)[pc:], avg.all_params(0)[pc:])
+    plain.close()
+    avg.close()
+    w = configs.WORKLOADS["tiny"]
+    ds, assign, params = configs.build_inputs(w)
+    gpu, orc = pair(w.arch, w.num_clients, w.num_clusters, assign, w.B, w.F, ds, params, False,
+                    lr=w.lr, momentum=w.momentum, client_average=True)
+    for _ in range(3):
+        check_round(gpu, orc, w.arch, tol=1e-3, loss_tol=1e-4, fwd_tol=1e-5)
+
+
 def test_augmented_rounds_bf16_and_fp32():
     """The crop + flip augmentation of Section V-A fused into the gather (the
     bf16 path's im2col gather and the fp32 path's gather): every round's

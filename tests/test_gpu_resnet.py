@@ -154,6 +154,19 @@ def test_resnet18_norm_hyperparameters_against_oracle():
     assert rel_l2(plain.bn_state(0) - bn0, orc.bn_state(0) - bn0) > 0.1
 
 
+def test_resnet18_client_average_against_oracle():
+    """The per-client average on the ResNet split: the cut gradient scaled
+    per example by B / (|A| b_k) before the client's blocks."""
+    ds, assign, params = _small(seed=17)
+    kw = dict(lr=0.05, momentum=0.9, client_average=True)
+    gpu = pkg.Context(RES, 8, 2, assign, 8, 0, 4, ds.images, ds.labels, ds.owner, params,
+                      bf16=True, **kw)
+    orc = oracle.Oracle(RES, 8, 2, assign, 8, 0, 4, ds.images, ds.labels, ds.owner, params,
+                        bf16=True, **kw)
+    for _ in range(2):
+        print("cut grad, update:", _round(gpu, orc))
+
+
 def test_resnet18_epoch_schedule_keeps_waiting_batchnorm_state():
     """F = -1 with unequal clusters: a cluster waiting at the fusion barrier
     keeps its parameters, momentum and BatchNorm running statistics (its
