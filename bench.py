@@ -311,24 +311,35 @@ def _oracle_pass(oracle, w, blob, x, y):
                                 label_smoothing=w.label_smoothing)
 
 
-def cpu_baseline(w, ds, assign, params, budget_s=15.0):
+def cpu_baseline(w, ds, assign, params, budget_s=15.0, single_s=6.0):
     """The oracle as it stands, on this host's cores: repeated forward/
     backward of a small batch of cluster-0 examples (bf16-operand mode when
-    the workload is bf16).  Returns (examples/s, threads, description)."""
+    the workload is bf16), on all cores and then on one.  Returns
+    (examples/s, threads, description, one-thread examples/s)."""
     import oracle
     ids = np.flatnonzero(assign[ds.owner] == 0)[:8]
     x = ds.images[ids].astype(np.float64)
     y = ds.labels[ids]
-    done, t0 = 0, time.perf_counter()
-    while True:
-        _oracle_pass(oracle, w, params.astype(np.float64), x, y)
-        done += len(ids)
-        if time.perf_counter() - t0 > budget_s:
-            break
-    dt = time.perf_counter() - t0
-    return done / dt, oracle.get_threads(), (
+    blob = params.astype(np.float64)
+
+    def run(budget):
+        done, t0 = 0, time.perf_counter()
+        while True:
+            _oracle_pass(oracle, w, blob, x, y)
+            done += len(ids)
+            if time.perf_counter() - t0 > budget:
+                return done, time.perf_counter() - t0
+    done, dt = run(budget_s)
+    threads = oracle.get_threads()
+    oracle.set_threads(1)
+    try:
+        done1, dt1 = run(single_s)
+    finally:
+        oracle.set_threads(threads)
+    return done / dt, threads, (
         f"{done} examples of cluster 0 in batches of {len(ids)} (forward+backward, fp64, "
-        f"{'bf16-operand' if w.bf16 else 'fp32'} rounding), {dt:.1f} s")
+        f"{'bf16-operand' if w.bf16 else 'fp32'} rounding), {dt:.1f} s on {threads} threads; "
+        f"{done1} examples in {dt1:.1f} s on one thread"), done1 / dt1
 
 
 def run_reference(args, w):
@@ -515,9 +526,10 @@ def main():
                                             max(5, K // 6), value)
         line["fusion"] = fusion_leg(ctx, w, torch, flush, peaks)
     if rank == 0 and not args.no_cpu_baseline:
-        v, cores, desc = cpu_baseline(w, ds, assign, params)
+        v, cores, desc, v1 = cpu_baseline(w, ds, assign, params)
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
-                                "sample": desc}
+                                "sample": desc, "single_thread": v1,
+                                "host_cpus": os.cpu_count()}
     ctx.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
