@@ -62,9 +62,9 @@ NCU_TRAFFIC = {
     "conv_wgrad_tc.L2": {"bytes": 2.523e+07, "src_hash": "9edb62919210128c"},
     "conv_wgrad_tc.L3": {"bytes": 8.43e+06, "src_hash": "9edb62919210128c"},
     "sgd": {"bytes": 6.11e+07, "src_hash": "483ce6954d2d1468", "per": "C", "C": 4},
-    "rn_norm_gn_bwd": {"bytes": 9.828e+07, "src_hash": "caff47aac58097a3", "family": "resnet",
+    "rn_norm_gn_bwd": {"bytes": 9.828e+07, "src_hash": "f5d44459e8a8b047", "family": "resnet",
                        "examples": 256},
-    "rn_norm_gn": {"bytes": 4.714e+07, "src_hash": "caff47aac58097a3", "family": "resnet",
+    "rn_norm_gn": {"bytes": 4.715e+07, "src_hash": "f5d44459e8a8b047", "family": "resnet",
                    "examples": 256},
 }
 for _k, _v in NCU_TRAFFIC.items():
@@ -122,6 +122,14 @@ def load_peaks():
 # for the elementwise/bandwidth kernels)
 # ---------------------------------------------------------------------------
 ARCH_NAMES = {1: "SplitCNN", 2: "ResNet-18 split", 3: "ResNet-18 split, 100 classes"}
+
+
+def bench_config(w, world):
+    """The `config` object of both arms' JSON lines."""
+    return {"workload": f"{w.name}: n={w.n} K={w.num_clients} C={w.num_clusters} B={w.B} "
+                        f"F={w.F} {ARCH_NAMES.get(w.arch, '')}",
+            "global_batch": w.num_clusters * w.B * world, "parallelism": f"replicas{world}",
+            "l2": "flushed between timed steps (256 MiB write)"}
 
 
 def work_per_round_resnet(w):
@@ -369,8 +377,7 @@ def run_reference(args, w):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "B": w.B, "C": w.num_clusters, "K": w.num_clients,
-                   "n": w.n, "sample": f"{len(ids)} examples of cluster 0 per step"},
+        "config": {**bench_config(w, world), "sample": f"{len(ids)} examples of cluster 0 per step"},
         "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.get_threads(),
                          "kind": "oracle",
                          "sample": f"forward+backward of {len(ids)} cluster-0 examples per step"},
@@ -503,11 +510,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": step_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.bf16 else "f32",
         "data": "synthetic",
-        "config": {"workload": f"{w.name}: n={w.n} K={w.num_clients} C={w.num_clusters} "
-                               f"B={w.B} F={w.F} "
-                               f"{ARCH_NAMES.get(w.arch, '')}",
-                   "global_batch": w.num_clusters * w.B * world, "parallelism": f"replicas{world}",
-                   "l2": "flushed between timed steps (256 MiB write)"},
+        "config": bench_config(w, world),
         "roofline": roof, "gpu_launches": launches, "wall_s": wall,
         # per-kernel device time from the breakdown pass (each kind timed alone)
         "kernels": breakdown,
