@@ -108,6 +108,19 @@ def dist_env():
     return rank, world, local
 
 
+def job_rate(local_ms, local_units, world, device):
+    """Whole-job rate of N independent replicas: every rank's units over the
+    slowest rank's time (MAX all-reduce when world > 1).  Returns (the max
+    time in ms, units per second)."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        local_ms = float(t.item())
+    return local_ms, local_units * world / (local_ms / 1e3)
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -469,13 +482,8 @@ def main():
     ktimes = ctx.kernel_times()
     ctx.set_timing(False)
     ctx.set_timing_filter(None)
-    step_ms = sum(a.elapsed_time(b) for a, b in ev)
-    if world > 1:
-        t = torch.tensor([step_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        step_ms = float(t.item())
-    examples = w.num_clusters * w.B * K * world
-    value = examples / (step_ms / 1e3)
+    step_ms, value = job_rate(sum(a.elapsed_time(b) for a, b in ev),
+                              w.num_clusters * w.B * K, world, "cuda")
 
     # dominant kernel and its roofline
     peaks = load_peaks()
