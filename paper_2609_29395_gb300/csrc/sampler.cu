@@ -151,39 +151,44 @@ __global__ void k_gather_f32(const float* __restrict__ images, const int32_t* __
 // bf16 storage: the input layer's im2col, x0[c][b][y][x][32] with column
 // k = tap * 3 + ch (tap = 3 ky + kx) = image[ch][y + ky - 1][x + kx - 1]
 // (0 outside the image), k = 27 = 1 (its weight-gradient column is the
-// bias gradient) and k = 28..31 = 0.  One block per sampled image: the
-// image is staged with a zero border in shared memory, then every thread
+// bias gradient) and k = 28..31 = 0.  A block per (sampled image, band of
+// kIm2colRows output rows): the band's rows of the image and their one-row
+// halo are staged with a zero border in shared memory, then every thread
 // writes 16-byte groups of 8 columns (a warp writes 512 contiguous bytes).
-constexpr int kIm2colThreads = 256;
+constexpr int kIm2colThreads = 256, kIm2colRows = 8;
 __global__ void __launch_bounds__(kIm2colThreads)
 k_gather_im2col(const float* __restrict__ images, const int32_t* __restrict__ idx,
                 bf16* __restrict__ x0, const AugArgs aug) {
-  __shared__ float tile[3][34][34];
+  constexpr int TR = kIm2colRows + 2;              // staged rows (padded rows r0 .. r0 + TR - 1)
+  __shared__ float tile[3][TR][34];
   pdl_wait();
   pdl_trigger();
-  const int64_t cb = blockIdx.x;
+  constexpr int bands = 32 / kIm2colRows;
+  const int64_t cb = blockIdx.x / bands;
+  const int r0 = (int)(blockIdx.x % bands) * kIm2colRows;   // first output row of the band
   const float* src = images + (int64_t)idx[cb] * 3072;
   int dy, dx, flip;
   aug_params(aug, cb, dy, dx, flip);
-  for (int i = threadIdx.x; i < 3 * 34 * 34; i += kIm2colThreads) {
-    const int ch = i / (34 * 34), yy = (i / 34) % 34, xx = i % 34;
-    // (yy - 1, xx - 1): the augmented image's pixel, zero around it
-    const int y = yy - 1, x = xx - 1;
+  for (int i = threadIdx.x; i < 3 * TR * 34; i += kIm2colThreads) {
+    const int ch = i / (TR * 34), t = (i / 34) % TR, xx = i % 34;
+    // padded pixel (r0 + t, xx) = the augmented image's (r0 + t - 1, xx - 1),
+    // zero around it
+    const int y = r0 + t - 1, x = xx - 1;
     const int sy = y + dy - 4, sx = (flip ? 31 - x : x) + dx - 4;
     const bool in = y >= 0 && y < 32 && x >= 0 && x < 32 && sy >= 0 && sy < 32 && sx >= 0 &&
                     sx < 32;
-    tile[ch][yy][xx] = in ? src[ch * 1024 + sy * 32 + sx] : 0.f;
+    tile[ch][t][xx] = in ? src[ch * 1024 + sy * 32 + sx] : 0.f;
   }
   __syncthreads();
-  uint4* dst = reinterpret_cast<uint4*>(x0 + cb * 1024 * 32);
-  for (int q = threadIdx.x; q < 1024 * 4; q += kIm2colThreads) {
-    const int pix = q >> 2, g = q & 3, y = pix >> 5, x = pix & 31;
+  uint4* dst = reinterpret_cast<uint4*>(x0 + (cb * 1024 + r0 * 32) * 32);
+  for (int q = threadIdx.x; q < kIm2colRows * 32 * 4; q += kIm2colThreads) {
+    const int pix = q >> 2, g = q & 3, yl = pix >> 5, x = pix & 31;
     float v[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
       const int k = 8 * g + e;
       const int tap = k / 3, ch = k - 3 * tap;
-      v[e] = k < 27 ? tile[ch][y + tap / 3][x + tap % 3] : (k == 27 ? 1.f : 0.f);
+      v[e] = k < 27 ? tile[ch][yl + tap / 3][x + tap % 3] : (k == 27 ? 1.f : 0.f);
     }
     __align__(16) bf16 h[8];
 #pragma unroll
@@ -257,7 +262,8 @@ cudaError_t launch_gather<float>(cudaStream_t s, const float* images, const int3
 template <>
 cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
                                 bf16* x0, const AugArgs& aug) {
-  return launch_k(k_gather_im2col, (unsigned)CB, kIm2colThreads, 0, s, images, idx, x0, aug);
+  return launch_k(k_gather_im2col, (unsigned)(CB * (32 / kIm2colRows)), kIm2colThreads, 0, s,
+                  images, idx, x0, aug);
 }
 
 template <typename T>
