@@ -23,7 +23,6 @@ namespace gcpsl {
 
 namespace {
 
-constexpr int kFwdEx = 4;          // examples per forward block
 constexpr int kFwdSlices = 8;      // warps (feature slices) per forward block
 constexpr int kBwdPairs = 32;      // feature pairs per backward block (one per lane)
 constexpr int kBwdChunks = 8;      // example chunks per backward block (one per warp)
@@ -64,7 +63,7 @@ template <typename T> struct VecLoad<T, 1> {
   __device__ static void run(const T* p, float* o) { o[0] = to_f(p[0]); }
 };
 
-// Block = (replica c, kFwdEx consecutive examples); warp w takes the k
+// Block = (replica c, EX consecutive examples); warp w takes the k
 // slices w, w + kFwdSlices, ... of VEC * 32 features (one slice each when
 // fin = kFwdSlices * 32 * VEC), so every load of the block is issued at
 // once.  The classes are taken JC at a time (JC weight rows in registers);
@@ -72,33 +71,33 @@ template <typename T> struct VecLoad<T, 1> {
 // warp order; then one warp per example takes the softmax: with J <= 32
 // every lane reads all J logits, otherwise lane l holds the logits
 // l, l + 32, ... and max, sum and loss are xor-tree warp reductions.
-template <typename T, int VEC, int J, int JC>
+template <typename T, int VEC, int J, int JC, int EX>
 __global__ void __launch_bounds__(kFwdSlices * 32)
 k_fc_fwd_ce(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
             const float* __restrict__ bias, int64_t b_rs, const int32_t* __restrict__ y,
             float* __restrict__ loss_ex, float* __restrict__ dlogits, int C, int B, int fin,
             float eps) {
   static_assert(J % JC == 0, "class chunks must tile J");
-  __shared__ float part[kFwdSlices][kFwdEx * J];
-  __shared__ float logit[kFwdEx][J];
+  __shared__ float part[kFwdSlices][EX * J];
+  __shared__ float logit[EX][J];
   pdl_wait();
   pdl_trigger();
-  const int per_c = (B + kFwdEx - 1) / kFwdEx;
-  const int c = blockIdx.x / per_c, e0 = (blockIdx.x % per_c) * kFwdEx;
-  const int ne = B - e0 < kFwdEx ? B - e0 : kFwdEx;
+  const int per_c = (B + EX - 1) / EX;
+  const int c = blockIdx.x / per_c, e0 = (blockIdx.x % per_c) * EX;
+  const int ne = B - e0 < EX ? B - e0 : EX;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const T* hp = h + ((int64_t)c * B + e0) * fin;
   const T* wp = w + (int64_t)c * w_rs;
   for (int j0 = 0; j0 < J; j0 += JC) {
-    float acc[kFwdEx][JC];
+    float acc[EX][JC];
 #pragma unroll
-    for (int e = 0; e < kFwdEx; ++e)
+    for (int e = 0; e < EX; ++e)
 #pragma unroll
       for (int j = 0; j < JC; ++j) acc[e][j] = 0.f;
     for (int k = (warp * 32 + lane) * VEC; k < fin; k += kFwdSlices * 32 * VEC) {
-      float hv[kFwdEx][VEC], wv[JC][VEC];
+      float hv[EX][VEC], wv[JC][VEC];
 #pragma unroll
-      for (int e = 0; e < kFwdEx; ++e) {
+      for (int e = 0; e < EX; ++e) {
         if (e < ne) VecLoad<T, VEC>::run(hp + (int64_t)e * fin + k, hv[e]);
         else
 #pragma unroll
@@ -107,14 +106,14 @@ k_fc_fwd_ce(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
 #pragma unroll
       for (int j = 0; j < JC; ++j) VecLoad<T, VEC>::run(wp + (int64_t)(j0 + j) * fin + k, wv[j]);
 #pragma unroll
-      for (int e = 0; e < kFwdEx; ++e)
+      for (int e = 0; e < EX; ++e)
 #pragma unroll
         for (int j = 0; j < JC; ++j)
 #pragma unroll
           for (int v = 0; v < VEC; ++v) acc[e][j] = fmaf(hv[e][v], wv[j][v], acc[e][j]);
     }
 #pragma unroll
-    for (int e = 0; e < kFwdEx; ++e)
+    for (int e = 0; e < EX; ++e)
 #pragma unroll
       for (int j = 0; j < JC; ++j) {
 #pragma unroll
@@ -123,7 +122,7 @@ k_fc_fwd_ce(const T* __restrict__ h, const T* __restrict__ w, int64_t w_rs,
       }
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < kFwdEx * J; i += kFwdSlices * 32) {
+  for (int i = threadIdx.x; i < EX * J; i += kFwdSlices * 32) {
     const int e = i / J, j = i % J;
     float z = 0.f;
 #pragma unroll
@@ -403,19 +402,24 @@ cudaError_t launch_fc_fwd_ce(cudaStream_t s, const T* h, const T* w, int64_t w_r
                              float label_smoothing) {
   if (fout != 10 && fout != 100) return cudaErrorInvalidValue;
   constexpr int VEC = 16 / (int)sizeof(T);
-  const unsigned grid = (unsigned)((int64_t)C * ((B + kFwdEx - 1) / kFwdEx));
+  // two examples per block for the 10-way head (more blocks), four for the
+  // 100-way head (each block reads its W chunks once for more examples)
+  const int ex = fout == 10 ? 2 : 4;
+  const unsigned grid = (unsigned)((int64_t)C * ((B + ex - 1) / ex));
   // 16-byte loads need every row of h and of each replica's W on a 16-byte boundary
   const bool vec = fin % VEC == 0 && (w_rs * (int64_t)sizeof(T)) % 16 == 0 && aligned16(h) &&
                    aligned16(w);
 #define FWD_ARGS s, h, w, w_rs, b, b_rs, y, loss_ex, dlogits, C, B, fin, label_smoothing
   if (fout == 10)
-    return vec ? launch_k(k_fc_fwd_ce<T, VEC, 10, 10>, grid, kFwdSlices * 32, 0, FWD_ARGS)
-               : launch_k(k_fc_fwd_ce<T, 1, 10, 10>, grid, kFwdSlices * 32, 0, FWD_ARGS);
+    return vec ? launch_k(k_fc_fwd_ce<T, VEC, 10, 10, 2>, grid, kFwdSlices * 32, 0, FWD_ARGS)
+               : launch_k(k_fc_fwd_ce<T, 1, 10, 10, 2>, grid, kFwdSlices * 32, 0, FWD_ARGS);
   // the 100-way head loads pairs, so that all eight warps share fin = 512
   const bool vec2 = fin % 2 == 0 && w_rs % 2 == 0 && (uintptr_t)h % (2 * sizeof(T)) == 0 &&
                     (uintptr_t)w % (2 * sizeof(T)) == 0;
-  return vec2 ? launch_k(k_fc_fwd_ce<T, 2, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS)
-              : launch_k(k_fc_fwd_ce<T, 1, 100, kClassChunk>, grid, kFwdSlices * 32, 0, FWD_ARGS);
+  return vec2 ? launch_k(k_fc_fwd_ce<T, 2, 100, kClassChunk, 4>, grid, kFwdSlices * 32, 0,
+                         FWD_ARGS)
+              : launch_k(k_fc_fwd_ce<T, 1, 100, kClassChunk, 4>, grid, kFwdSlices * 32, 0,
+                         FWD_ARGS);
 #undef FWD_ARGS
 }
 

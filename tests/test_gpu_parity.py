@@ -271,6 +271,22 @@ def test_batch_of_one():
     assert (counts.sum(1) == 1).all()
 
 
+def test_largest_batch():
+    """B = 1024, the largest batch gcpsl_init accepts (one sampler block of
+    1024 threads per cluster), two clusters: one round against the oracle,
+    and B = 1025 rejected."""
+    ds, assign, params = _splitcnn_small(C=2, n=4096, K=16, seed=9)
+    gpu, orc = pair(synth.ARCH_SPLIT_CNN, 16, 2, assign, 1024, 0, ds, params, True,
+                    momentum=0.9)
+    check_round(gpu, orc, synth.ARCH_SPLIT_CNN)
+    _, counts = gpu.sample()
+    assert (counts.sum(1) == 1024).all()
+    gpu.close()
+    with pytest.raises(pkg.binding.GcpslError):
+        pkg.Context(synth.ARCH_SPLIT_CNN, 16, 1, np.zeros(16, np.int32), 1025, 0, 4, ds.images,
+                    ds.labels, ds.owner, params)
+
+
 def test_grouped_equals_serialized_bit_exact():
     """C clusters in one context == C one-cluster contexts (cluster_id_base=n):
     bit-identical parameters, momentum, cuts and samples."""
