@@ -108,12 +108,14 @@ cudaError_t launch_epoch_rank(cudaStream_t s, const int32_t* ids, const int64_t*
 // The round's batch of every cluster: local round s = t % period[n] of its
 // epoch when s < rounds[n]; a cluster past its r_n rounds (epoch schedule)
 // waits at the fusion barrier: upd[n] = 0 (nullable), its batch is its last
-// one (s = r_n - 1) and active[n] = 0.
+// one (s = r_n - 1) and active[n] = 0.  cut_scale (nullable, [C][B]):
+// B / (|A| b_k) of every batch position (|A| of the batch itself, also for a
+// waiting cluster), the per-client average's factor.
 cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* off,
                           const int32_t* rounds, const int32_t* period, const int64_t* d_t,
                           const int32_t* owner, const int32_t* labels, int K, int B, int C,
                           int32_t* idx, int32_t* counts, int32_t* active, int32_t* y,
-                          int32_t* upd);
+                          int32_t* upd, float* cut_scale = nullptr);
 // Training augmentation of the gathered images (Sec. V-A: random crops and
 // horizontal flips): sampled image b of cluster n in round t is cropped
 // from its 4-pixel zero-padded version at offset (dy, dx) in [0, 8]^2 and
@@ -141,13 +143,11 @@ template <>
 cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32_t* idx, int CB,
                                 bf16* x0, const AugArgs& aug);
 // per-client average (Sec. IV-B, the unweighted reading): a ([C B][per_a])
-// and b ([C B][per_b], nullable) scaled in place, example cb by
-// B / (active[c] counts[c][owner[idx[cb]]]); per_* multiples of 8
+// and b ([C B][per_b], nullable) scaled in place, example cb by scale[cb]
+// (the sampler's cut_scale); per_* multiples of 8
 template <typename T>
 cudaError_t launch_client_avg_scale(cudaStream_t s, T* a, int64_t per_a, T* b, int64_t per_b,
-                                    const int32_t* idx, const int32_t* owner,
-                                    const int32_t* counts, const int32_t* active, int C, int B,
-                                    int K);
+                                    const float* scale, int CB);
 
 // conv_simt.cu
 template <typename T>

@@ -273,7 +273,7 @@ gcpsl_status enqueue_sample(gcpsl_ctx* c, bool boundary) {
   }
   LAUNCH("sample", launch_sample(s, c->d_perm, c->d_off, c->d_rounds, c->d_period, c->d_t,
                                  c->d_owner, c->d_labels, c->K, B, C, c->d_idx, c->d_counts,
-                                 c->d_active, c->d_y, c->d_upd));
+                                 c->d_active, c->d_y, c->d_upd, c->d_cut_scale));
   const AugArgs aug{c->desc.augment, (uint32_t)c->seed, (uint32_t)(c->seed >> 32), c->d_t,
                     c->desc.cluster_id_base, B};
   LAUNCH("gather", launch_gather<T>(s, c->d_images, c->d_idx, C * B, (T*)c->d_act[0], aug));
@@ -376,8 +376,7 @@ gcpsl_status enqueue_round(gcpsl_ctx* c, bool boundary) {
       // cut gradient, per example by B / (|A| b_k)
       LAUNCH("client_avg", launch_client_avg_scale<T>(
                                s, g, (int64_t)cs.h * cs.w * cs.cout, dact[a.ncl],
-                               act_elems(c, a.ncl) / ((int64_t)C * B), c->d_idx, c->d_owner,
-                               c->d_counts, c->d_active, C, B, c->K));
+                               act_elems(c, a.ncl) / ((int64_t)C * B), c->d_cut_scale, C * B));
     const auto& R = c->red[i];
     if (L.on) {
       // weights and bias together (the bias follows the weight in the store);
@@ -789,6 +788,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     DALLOC(c->d_idx, sizeof(int32_t) * C * B);
     DALLOC(c->d_counts, sizeof(int32_t) * (size_t)C * K);
     DALLOC(c->d_active, sizeof(int32_t) * C);
+    if (desc->client_average) DALLOC(c->d_cut_scale, sizeof(float) * C * B);
     DALLOC(c->d_loss, sizeof(float) * C);
     DALLOC(c->d_t, sizeof(int64_t));
     CK(cudaMemset(c->d_t, 0, sizeof(int64_t)));
@@ -826,6 +826,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   DALLOC(c->d_idx, sizeof(int32_t) * C * B);
   DALLOC(c->d_counts, sizeof(int32_t) * (size_t)C * K);
   DALLOC(c->d_active, sizeof(int32_t) * C);
+  if (desc->client_average) DALLOC(c->d_cut_scale, sizeof(float) * C * B);
   DALLOC(c->d_loss, sizeof(float) * C);
   DALLOC(c->d_t, sizeof(int64_t));
   CK(cudaMemset(c->d_t, 0, sizeof(int64_t)));

@@ -206,6 +206,7 @@ struct gcpsl_ctx {
   int32_t* d_idx = nullptr;
   int32_t* d_counts = nullptr;
   int32_t* d_active = nullptr;
+  float* d_cut_scale = nullptr;    // [C][B] B / (|A| b_k), with client_average only
   float* d_loss = nullptr;
   int64_t* d_t = nullptr;
   float* h_loss = nullptr;         // pinned staging

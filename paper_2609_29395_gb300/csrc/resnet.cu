@@ -613,8 +613,8 @@ gcpsl_status rn_enqueue_round(gcpsl_ctx* c) {
     if (i == 2 && c->desc.client_average)
       // the per-client average: the cut gradient, per example by B / (|A| b_k)
       LAUNCH("client_avg", launch_client_avg_scale<bf16>(s, r.cutg, (int64_t)64 * 32 * 32,
-                                                         (bf16*)nullptr, 0, c->d_idx, c->d_owner,
-                                                         c->d_counts, c->d_active, C, B, c->K));
+                                                         (bf16*)nullptr, 0, c->d_cut_scale,
+                                                         C * B));
   }
   // stem: its ReLU and GroupNorm, then the weight gradient over the im2col
   RN(norm_bwd(c, r.stem_n, r.ystem, d, r.astem, nullptr, r.dy));

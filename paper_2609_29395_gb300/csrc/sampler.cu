@@ -80,7 +80,7 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
                          const int32_t* __restrict__ labels, int K, int B,
                          int32_t* __restrict__ idx, int32_t* __restrict__ counts,
                          int32_t* __restrict__ active, int32_t* __restrict__ y,
-                         int32_t* __restrict__ upd) {
+                         int32_t* __restrict__ upd, float* __restrict__ cut_scale) {
   extern __shared__ int32_t sm[];
   int32_t* sid = sm;          // [B] ids of the round
   int32_t* sown = sm + B;     // [B] their owners
@@ -112,6 +112,8 @@ __global__ void k_sample(const int32_t* __restrict__ perm, const int64_t* __rest
     active[c] = updates ? first : 0;
     if (upd) upd[c] = updates;
   }
+  if (cut_scale)   // B / (|A| b_k): the counts are complete after the barrier above
+    cut_scale[(int64_t)c * B + rank] = (float)B / ((float)first * (float)cnt[own]);
 }
 
 // crop offsets and flip of sampled image cb = c * B + b (see AugArgs)
@@ -197,24 +199,20 @@ k_gather_im2col(const float* __restrict__ images, const int32_t* __restrict__ id
   }
 }
 
-// The per-client average of Sec. IV-B's other reading: example b of cluster
-// c, owned by client k, has its gradient at the cut multiplied by
-// B / (|A_c| b_k) before the client segment's backward.  Grid (chunks of
+// The per-client average of Sec. IV-B's other reading: example cb's gradient
+// at the cut is multiplied by scale[cb] = B / (|A| b_k) (written by the
+// sampler) before the client segment's backward.  Grid (chunks of
 // kScaleThreads x 8 elements, C B examples); a and b (nullable) are
 // [C B][per] tensors scaled in place, 8 elements per thread.
 constexpr int kScaleThreads = 256;
 template <typename T>
 __global__ void __launch_bounds__(kScaleThreads)
 k_client_avg_scale(T* __restrict__ a, T* __restrict__ b2, int64_t per_a, int64_t per_b,
-                   const int32_t* __restrict__ idx, const int32_t* __restrict__ owner,
-                   const int32_t* __restrict__ counts, const int32_t* __restrict__ active, int B,
-                   int K) {
+                   const float* __restrict__ scale) {
   pdl_wait();
   pdl_trigger();
   const int64_t cb = blockIdx.y;
-  const int c = (int)(cb / B);
-  const int cnt = counts[(int64_t)c * K + owner[idx[cb]]];
-  const float sc = (float)B / ((float)active[c] * (float)cnt);
+  const float sc = scale[cb];
   const int64_t e = ((int64_t)blockIdx.x * kScaleThreads + threadIdx.x) * 8;
   for (int t = 0; t < 2; ++t) {
     T* p = t == 0 ? a : b2;
@@ -247,9 +245,9 @@ cudaError_t launch_sample(cudaStream_t s, const int32_t* perm, const int64_t* of
                           const int32_t* rounds, const int32_t* period, const int64_t* d_t,
                           const int32_t* owner, const int32_t* labels, int K, int B, int C,
                           int32_t* idx, int32_t* counts, int32_t* active, int32_t* y,
-                          int32_t* upd) {
+                          int32_t* upd, float* cut_scale) {
   return launch_k(k_sample, C, B, 3 * B * sizeof(int32_t), s, perm, off, rounds, period, d_t,
-                  owner, labels, K, B, idx, counts, active, y, upd);
+                  owner, labels, K, B, idx, counts, active, y, upd, cut_scale);
 }
 
 template <>
@@ -268,21 +266,16 @@ cudaError_t launch_gather<bf16>(cudaStream_t s, const float* images, const int32
 
 template <typename T>
 cudaError_t launch_client_avg_scale(cudaStream_t s, T* a, int64_t per_a, T* b, int64_t per_b,
-                                    const int32_t* idx, const int32_t* owner,
-                                    const int32_t* counts, const int32_t* active, int C, int B,
-                                    int K) {
-  if (per_a % 8 || per_b % 8 || (uintptr_t)a % 16 || (uintptr_t)b % 16)
+                                    const float* scale, int CB) {
+  if (per_a % 8 || per_b % 8 || (uintptr_t)a % 16 || (uintptr_t)b % 16 || CB > 65535)
     return cudaErrorInvalidValue;
   const int64_t per = per_a > per_b ? per_a : per_b;
-  const dim3 grid((unsigned)((per / 8 + kScaleThreads - 1) / kScaleThreads), (unsigned)(C * B));
-  return launch_k(k_client_avg_scale<T>, grid, kScaleThreads, 0, s, a, b, per_a, per_b, idx,
-                  owner, counts, active, B, K);
+  const dim3 grid((unsigned)((per / 8 + kScaleThreads - 1) / kScaleThreads), (unsigned)CB);
+  return launch_k(k_client_avg_scale<T>, grid, kScaleThreads, 0, s, a, b, per_a, per_b, scale);
 }
 template cudaError_t launch_client_avg_scale<float>(cudaStream_t, float*, int64_t, float*, int64_t,
-                                                    const int32_t*, const int32_t*,
-                                                    const int32_t*, const int32_t*, int, int, int);
+                                                    const float*, int);
 template cudaError_t launch_client_avg_scale<bf16>(cudaStream_t, bf16*, int64_t, bf16*, int64_t,
-                                                   const int32_t*, const int32_t*, const int32_t*,
-                                                   const int32_t*, int, int, int);
+                                                   const float*, int);
 
 }  // namespace gcpsl

@@ -251,6 +251,35 @@ def test_epoch_schedule_with_fusion_barrier():
             assert all((gpu.all_params(n) == gpu.all_params(0)).all() for n in range(3))
 
 
+def test_client_average_with_waiting_clusters():
+    """The per-client average under the epoch schedule: a cluster waiting at
+    the fusion barrier still computes its round (not applied), with the
+    factor B / (|A| b_k) of its own batch, as the oracle does."""
+    ds = synth.make_dataset(768, 10, 12, 0.3, balanced=False, seed_data=4, seed_split=5)
+    assign = (np.arange(12) % 3 == 0).astype(np.int32)
+    params = synth.init_params(synth.ARCH_SPLIT_CNN)
+    B = 64
+    r = np.bincount(assign[ds.owner], minlength=2) // B
+    assert r.min() < r.max() <= 12, r
+    gpu, orc = pair(synth.ARCH_SPLIT_CNN, 12, 2, assign, B, -1, ds, params, True, lr=0.05,
+                    momentum=0.9, client_average=True)
+    for t in range(int(r.max())):
+        # the scaled cut gradient is compared below with the factor divided
+        # out: a factor up to B / |A| on a client with one example would let
+        # one valid tie routing (check_decisions) outweigh the aggregate bar
+        check_round(gpu, orc, synth.ARCH_SPLIT_CNN, grad=False)
+        idx, counts = orc.sample()
+        g = gpu.cut(pkg.binding.GCPSL_CUT_GRAD).reshape(2, B, -1).astype(np.float64)
+        o = orc.cut(1).reshape(2, B, -1)
+        for n in range(2):
+            own = ds.owner[idx[n]]
+            act = np.count_nonzero(counts[n])
+            scale = B / (act * counts[n][own])
+            assert rel_l2(g[n] / scale[:, None], o[n] / scale[:, None]) < REL_L2, (t, n)
+            assert rel_l2(g[n], o[n]) < 0.1, (t, n)   # the factors themselves agree
+    assert (orc.stats()[1] == 0).any()          # a cluster waited in the last round
+
+
 def test_ragged_batch_nesterov_wd_label_smoothing():
     """B = 24 (not a power of two), C = 6, Nesterov, weight decay, label
     smoothing."""
