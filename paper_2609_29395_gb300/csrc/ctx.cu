@@ -658,6 +658,7 @@ void free_all(gcpsl_ctx* c) {
   if (c->h_images) cudaFreeHost(c->h_images);
   if (c->h_loss) cudaFreeHost(c->h_loss);
   if (c->h_active) cudaFreeHost(c->h_active);
+  if (c->h_err) cudaFreeHost(c->h_err);
   if (c->own_stream) cudaStreamDestroy(c->own_stream);
 }
 
@@ -796,6 +797,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
     CK(cudaMemset(c->d_counts, 0, sizeof(int32_t) * (size_t)C * K));
     CK(cudaHostAlloc((void**)&c->h_loss, sizeof(float) * C, cudaHostAllocDefault));
     CK(cudaHostAlloc((void**)&c->h_active, sizeof(int32_t) * C, cudaHostAllocDefault));
+    CK(cudaHostAlloc((void**)&c->h_err, sizeof(int), cudaHostAllocDefault));
     c->w0_off = 0;                                // the stem convolution
     c->w0_cout = 64;
     gcpsl_status st = rn_setup(c);
@@ -834,6 +836,7 @@ gcpsl_status init_impl(gcpsl_ctx* c, const gcpsl_model_desc* desc, int K, int C,
   CK(cudaMemset(c->d_counts, 0, sizeof(int32_t) * (size_t)C * K));
   CK(cudaHostAlloc((void**)&c->h_loss, sizeof(float) * C, cudaHostAllocDefault));
   CK(cudaHostAlloc((void**)&c->h_active, sizeof(int32_t) * C, cudaHostAllocDefault));
+  CK(cudaHostAlloc((void**)&c->h_err, sizeof(int), cudaHostAllocDefault));
   // reduction shapes (per replica only, so that the summation order does not
   // depend on C) and the partial-sum scratch
   int64_t bpart = 0;
@@ -961,7 +964,11 @@ gcpsl_status gcpsl_step(gcpsl_ctx* c, gcpsl_step_stats* stats) {
                        c->stream));
     CK(cudaMemcpyAsync(c->h_active, c->d_active, sizeof(int32_t) * c->C, cudaMemcpyDeviceToHost,
                        c->stream));
-    SYNC_CHECK(c);
+    // the device error word comes back with the statistics: one synchronisation
+    CK(cudaMemcpyAsync(c->h_err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+    CK(cudaStreamSynchronize(c->stream));
+    if (*c->h_err)
+      return fail(c, GCPSL_E_TIMEOUT, "device-side wait gave up (error word 0x%x)", *c->h_err);
     // a cluster waiting at the fusion barrier took no update: loss 0
     for (int n = 0; n < c->C; ++n)
       if ((c->t - 1) % c->h_period[n] >= c->h_rounds[n]) c->h_loss[n] = 0.f;

@@ -207,6 +207,7 @@ struct gcpsl_ctx {
   int32_t* d_counts = nullptr;
   int32_t* d_active = nullptr;
   float* d_cut_scale = nullptr;    // [C][B] B / (|A| b_k), with client_average only
+  int* h_err = nullptr;            // pinned copy of d_err (read back with the step statistics)
   float* d_loss = nullptr;
   int64_t* d_t = nullptr;
   float* h_loss = nullptr;         // pinned staging
