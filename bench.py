@@ -569,7 +569,7 @@ def e2e_leg(pkg, w, ds, assign, params, torch, flush, K):
     ctx.close()
     return {"value": w.num_clusters * w.B * K / tot, "unit": UNIT,
             "h2d_bytes_per_step": w.num_clusters * w.B * 3072 * 4,
-            "d2h_bytes_per_step": w.num_clusters * 8,
+            "d2h_bytes_per_step": w.num_clusters * 8 + 4,   # loss, |A|, the error word
             "how": "gcpsl_step(stats) wall time; images gathered from pinned host memory"}
 
 
