@@ -303,6 +303,18 @@ gcpsl_status gcpsl_sample_round_noalloc(const int32_t* ids, const int64_t* clust
                                         int32_t* idx, int32_t* counts, int32_t* active,
                                         int32_t* batch_labels, void* stream);
 
+/* gcpsl_check_wait_timeout -- exercises the failure path of the library's
+ * bounded device-side waits: one block waits on a shared-memory mbarrier
+ * that nothing arrives on, gives up after limit_ns nanoseconds of device
+ * time (1 <= limit_ns <= 1e9), sets the context's device error word and
+ * exits, as every kernel of the library does when a TMA, MMA or bulk-copy
+ * completion never comes.  Returns GCPSL_E_TIMEOUT (after which the context
+ * is in the error state: later calls return GCPSL_E_STATE); GCPSL_E_INVAL
+ * for a bad limit; GCPSL_E_STATE on a context already in the error state.
+ * No fault, trap or unbounded wait is involved: the GPU stays usable for
+ * other contexts.                                                         */
+gcpsl_status gcpsl_check_wait_timeout(gcpsl_ctx* ctx, uint64_t limit_ns);
+
 /* gcpsl_last_error -- static description of the context's last failure
  * (or of the last failed gcpsl_init when ctx is NULL).                   */
 const char* gcpsl_last_error(const gcpsl_ctx* ctx);

@@ -32,8 +32,8 @@ EXPORTS = ("gcpsl_init", "gcpsl_step", "gcpsl_fuse", "gcpsl_get_params", "gcpsl_
            "gcpsl_rounds", "gcpsl_set_stream", "gcpsl_set_graph", "gcpsl_set_timing",
            "gcpsl_set_timing_filter", "gcpsl_kernels_launched",
            "gcpsl_kernel_times",
-           "gcpsl_reset_kernel_times", "gcpsl_sample_round_noalloc", "gcpsl_last_error",
-           "gcpsl_destroy")
+           "gcpsl_reset_kernel_times", "gcpsl_sample_round_noalloc",
+           "gcpsl_check_wait_timeout", "gcpsl_last_error", "gcpsl_destroy")
 
 
 class gcpsl_model_desc(ct.Structure):
@@ -94,6 +94,7 @@ def load() -> ct.CDLL:
     L.gcpsl_set_stream.argtypes = [vp, vp]
     L.gcpsl_set_timing.argtypes = [vp, ct.c_int]
     L.gcpsl_set_graph.argtypes = [vp, ct.c_int]
+    L.gcpsl_check_wait_timeout.argtypes = [vp, ct.c_uint64]
     L.gcpsl_set_bn_state.argtypes = [vp, ct.c_int, f32p, ct.c_size_t]
     L.gcpsl_get_relu_masks.argtypes = [vp, ct.POINTER(ct.c_uint8), ct.c_size_t,
                                        ct.POINTER(ct.c_size_t)]
@@ -299,6 +300,11 @@ class Context:
         """Time only kernels whose name starts with prefix (None: all)."""
         _check(load().gcpsl_set_timing_filter(self._h, prefix.encode() if prefix else None),
                self._h)
+
+    def check_wait_timeout(self, limit_ns: int):
+        """Runs the bounded-wait failure path (see gcpsl.h); raises the
+        resulting GcpslError (GCPSL_E_TIMEOUT)."""
+        _check(load().gcpsl_check_wait_timeout(self._h, int(limit_ns)), self._h)
 
     def set_graph(self, on: bool):
         """Replay rounds from CUDA graphs (default) or launch them eagerly."""

@@ -380,4 +380,8 @@ cudaError_t launch_sgd(cudaStream_t s, float* theta, float* mom, const float* gr
 cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,
                         int64_t P);
 
+// one block waiting, bounded by limit_ns, on an mbarrier nothing arrives on:
+// sets bit 256 of err (the library's bounded-wait failure path)
+cudaError_t launch_wait_probe(cudaStream_t s, int* err, uint64_t limit_ns);
+
 }  // namespace gcpsl

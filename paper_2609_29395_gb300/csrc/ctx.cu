@@ -1190,6 +1190,17 @@ gcpsl_status gcpsl_set_timing_filter(gcpsl_ctx* c, const char* prefix) {
   return GCPSL_OK;
 }
 
+gcpsl_status gcpsl_check_wait_timeout(gcpsl_ctx* c, uint64_t limit_ns) {
+  gcpsl_status st = check_usable(c);
+  if (st != GCPSL_OK) return st;
+  if (limit_ns < 1 || limit_ns > 1000000000ull)
+    return fail(c, GCPSL_E_INVAL, "limit_ns %llu outside [1, 1e9]", (unsigned long long)limit_ns);
+  SYNC_CHECK(c);
+  CK(launch_wait_probe(c->stream, c->d_err, limit_ns));
+  SYNC_CHECK(c);      // the probe's error word: GCPSL_E_TIMEOUT
+  return fail(c, GCPSL_E_CUDA, "the bounded wait did not report its timeout");
+}
+
 gcpsl_status gcpsl_set_graph(gcpsl_ctx* c, int enable) {
   gcpsl_status st = check_usable(c);
   if (st != GCPSL_OK) return st;

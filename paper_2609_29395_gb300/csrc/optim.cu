@@ -9,6 +9,7 @@
 //   is evaluated as theta_0 + sum_{n>=1} q_n (theta_n - theta_0) in fp32,
 //   which returns theta exactly when all replicas are equal.
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace gcpsl {
 
@@ -178,6 +179,23 @@ cudaError_t launch_sgd_seg(cudaStream_t s, float* theta, float* mom, bf16* shado
 cudaError_t launch_fuse(cudaStream_t s, float* theta, bf16* shadow, const float* q, int C,
                         int64_t P) {
   return launch_k(k_fuse, grid_for(P, 256), 256, 0, s, theta, shadow, q, C, P);
+}
+
+// The failure path of the bounded waits: one thread waits on an mbarrier
+// that expects one arrival which never comes, gives up after limit_ns and
+// records bit 256 in the error word.
+namespace {
+__global__ void k_wait_probe(int* err, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  sm100::mbar_init(&bar, 1);
+  sm100::fence_mbar_init();
+  if (!sm100::mbar_wait(&bar, 0, limit_ns)) atomicOr(err, 256);
+}
+}  // namespace
+
+cudaError_t launch_wait_probe(cudaStream_t s, int* err, uint64_t limit_ns) {
+  k_wait_probe<<<1, 1, 0, s>>>(err, limit_ns);
+  return cudaGetLastError();
 }
 
 }  // namespace gcpsl
